@@ -1,0 +1,361 @@
+"""Model-level pins of the oracle (no GPU): the invariants the paper's
+definitions fix, and special weight settings whose result has a closed form."""
+import math
+
+import numpy as np
+import pytest
+import scipy.special
+
+import oracle
+import synth
+from helpers import bf16_round, identity_bits, micro, one_hot_matrix, to_bf16_bits, zeros_like_bits
+
+TINY = synth.CONFIGS["tiny"]
+
+
+def _run(shape, model, taus, n=None, readouts=True, force=None):
+    o = oracle.Oracle(shape, model, readouts=readouts)
+    first, steps = o.generate(synth.prompt(shape), n or shape.new_tokens, taus, force_schedule=force)
+    return o, first, steps
+
+
+# ------------------------------------------------------------- I-1
+def test_tau_above_one_reproduces_the_plain_model():
+    """Section 2 / Section 4 step five: a gate that never passes leaves the
+    full model's greedy output untouched."""
+    model = synth.make_model(TINY)
+    og, first_g, gated = _run(TINY, model, [1.01])
+    op, first_p, plain = _run(TINY, model, [], readouts=False)
+    assert first_g == first_p
+    assert [s["token"] for s in gated] == [s["token"] for s in plain]
+    assert all(not s["exited"] for s in gated) and og.stats()["exits"] == [0]
+    for j in range(TINY.n_layers):
+        for t in (0, TINY.prompt_len, TINY.max_ctx - 1):
+            kg, vg, sg = og.kv(j, t)
+            kp, vp, sp = op.kv(j, t)
+            assert np.array_equal(kg, kp) and np.array_equal(vg, vp) and sg == sp == 1
+
+
+# ------------------------------------------------------------- I-2
+def test_tau_zero_always_exits_and_never_reads_upper_layer_q_o_ffn():
+    """tau = 0 exits every step at layer k (p >= 1/V > 0); the upper layers'
+    query, output and FFN weights are then never read, so editing them after
+    prefill changes nothing."""
+    shape = TINY
+    k = shape.readout_layers[0]
+    ref_model = synth.make_model(shape)
+    o_ref, f_ref, s_ref = _run(shape, ref_model, [0.0])
+    edit = synth.make_model(shape)
+    o = oracle.Oracle(shape, edit)
+    first = o.prefill(synth.prompt(shape))
+    rng = np.random.default_rng(5)
+    for j in range(k, shape.n_layers):
+        for key in ("wq", "wo", "wg", "wu", "wd"):
+            edit["layers"][j][key][...] = rng.integers(0, 65535, edit["layers"][j][key].shape, dtype=np.uint16)
+    tok, steps = first, []
+    for _ in range(shape.new_tokens):
+        s = o.decode_step(tok, [0.0])
+        steps.append(s)
+        tok = s["token"]
+    assert first == f_ref
+    assert all(s["exited"] and s["exit_layer"] == k for s in steps)
+    assert [s["token"] for s in steps] == [s["token"] for s in s_ref]
+    assert [s["confidence"] for s in steps] == [s["confidence"] for s in s_ref]
+    assert o.stats()["exits"] == [shape.new_tokens]
+    assert all(s["token"] == s["readout_token"][0] for s in steps)
+    for j in range(shape.n_layers):
+        for t in range(shape.prompt_len, shape.max_ctx):
+            assert o.kv(j, t)[2] == (2 if j >= k else 1)
+
+
+# ------------------------------------------------------------- I-3
+def _with_identity_readout_at_L(shape, model):
+    d = shape.d_model
+    model = dict(model)
+    model["readouts"] = [(shape.n_layers, identity_bits(d), zeros_like_bits(np.zeros(d)))]
+    return shape.replace(readout_layers=(shape.n_layers,)), model
+
+
+def test_identity_readout_at_last_layer_reproduces_final_logits():
+    """Section 2: the readout's output passes through the model's own final
+    normalisation and unembedding unchanged, so an identity readout at layer L
+    gives the final logits (bit for bit without activation rounding)."""
+    shape, model = _with_identity_readout_at_L(micro(), synth.make_model(micro()))
+    o = oracle.Oracle(shape, model, pure_fp32=True)
+    tok = o.prefill(synth.prompt(shape))
+    for _ in range(6):
+        s = o.decode_step(tok, [1.01], capture=True)
+        cap = s["capture"]
+        assert np.array_equal(cap["readout_logits"][0], cap["final_logits"])
+        assert s["readout_token"][0] == s["full_token"]
+        tok = s["token"]
+    # with activation rounding the readout input is bf16(h): logits agree to 1e-2
+    o2 = oracle.Oracle(shape, model)
+    tok = o2.prefill(synth.prompt(shape))
+    for _ in range(6):
+        s = o2.decode_step(tok, [1.01], capture=True)
+        r, f = s["capture"]["readout_logits"][0], s["capture"]["final_logits"]
+        assert np.max(np.abs(r - f)) <= 1e-2 * np.max(np.abs(f))
+        tok = s["token"]
+
+
+def test_identity_readout_tau_zero_equals_tau_above_one():
+    shape, model = _with_identity_readout_at_L(micro(), synth.make_model(micro()))
+    _, f1, a = _run(shape, model, [0.0])
+    _, f2, b = _run(shape, model, [1.01])
+    assert f1 == f2 and [s["token"] for s in a] == [s["token"] for s in b]
+    assert all(s["exited"] for s in a) and not any(s["exited"] for s in b)
+
+
+# ------------------------------------------------------------- I-4
+def test_kv_fill_equals_full_path_when_upper_layers_leave_the_residual_unchanged():
+    """Section 4 step five: the fill projects the exit-layer state through the
+    skipped layers' key/value matrices.  If those layers add nothing to the
+    residual (zero output and down projections) the full path computes exactly
+    the same keys and values."""
+    shape = micro()
+    k = shape.readout_layers[0]
+    model = synth.make_model(shape)
+    for j in range(k, shape.n_layers):
+        model["layers"][j]["wo"] = zeros_like_bits(model["layers"][j]["wo"])
+        model["layers"][j]["wd"] = zeros_like_bits(model["layers"][j]["wd"])
+    full = oracle.Oracle(shape, model)
+    ex = oracle.Oracle(shape, model)
+    tok = full.prefill(synth.prompt(shape))
+    assert ex.prefill(synth.prompt(shape)) == tok
+    for _ in range(shape.new_tokens):
+        a = full.decode_step(tok, [0.5], oracle.FORCE_FULL)
+        b = ex.decode_step(tok, [0.5], oracle.FORCE_EXIT_AT(0))
+        t = full.pos - 1
+        for j in range(shape.n_layers):
+            ka, va, sa = full.kv(j, t)
+            kb, vb, sb = ex.kv(j, t)
+            assert np.array_equal(ka, kb) and np.array_equal(va, vb)
+            assert sa == 1 and sb == (2 if j >= k else 1)
+        assert a["confidence"] == b["confidence"]
+        tok = a["token"]
+
+
+# ------------------------------------------------------------- multi-exit
+def test_multiple_readouts_shallowest_passing_exits():
+    """Section 4 step three: several exit points; the first passing one is taken
+    and every layer above it is filled."""
+    shape = micro(readout_layers=(1, 2, 3))
+    model = synth.make_model(shape)
+    cases = [([1.01, 0.0, 0.0], 1), ([0.0, 0.0, 0.0], 0), ([1.01, 1.01, 0.0], 2), ([1.01] * 3, None)]
+    for taus, expect in cases:
+        o, _, steps = _run(shape, model, taus, n=4)
+        for s in steps:
+            if expect is None:
+                assert not s["exited"] and s["n_evaluated"] == 3 and s["exit_layer"] == shape.n_layers
+            else:
+                assert s["exited"] and s["exit_readout"] == expect and s["n_evaluated"] == expect + 1
+                assert s["exit_layer"] == shape.readout_layers[expect]
+        e_layer = shape.n_layers if expect is None else shape.readout_layers[expect]
+        for j in range(shape.n_layers):
+            assert o.kv(j, shape.prompt_len + 1)[2] == (1 if j < e_layer else 2)
+    # forced exit at the last readout still reports the earlier gates' verdicts
+    o = oracle.Oracle(shape, model)
+    tok = o.prefill(synth.prompt(shape))
+    s = o.decode_step(tok, [0.0, 0.0, 0.0], oracle.FORCE_EXIT_AT(2))
+    assert s["exit_readout"] == 2 and s["gate_pass"] == [1, 1, 1] and s["n_evaluated"] == 3
+
+
+# ------------------------------------------------------------- I-6
+def test_exit_count_non_increasing_in_tau():
+    model = synth.make_model(TINY)
+    _, _, steps = _run(TINY, model, [0.5], force=[oracle.FORCE_FULL] * TINY.new_tokens)
+    p = np.array([s["confidence"][0] for s in steps], np.float32)
+    taus = np.linspace(0, 1.01, 50).astype(np.float32)
+    counts = [int(np.sum(p > t)) for t in taus]
+    assert counts[0] == len(p) and counts[-1] == 0
+    assert all(a >= b for a, b in zip(counts, counts[1:]))
+    # the free gate agrees with its recorded confidence
+    for t in (0.3, 0.6):
+        _, _, free = _run(TINY, model, [t])
+        assert all(s["exited"] == (s["confidence"][0] > np.float32(t)) for s in free)
+
+
+def test_gate_is_strict():
+    """Section 2: the early answer is accepted when its probability exceeds the
+    threshold; a threshold equal to the probability does not pass."""
+    model = synth.make_model(TINY)
+    o = oracle.Oracle(TINY, model)
+    tok = o.prefill(synth.prompt(TINY))
+    s0 = o.decode_step(tok, [0.5], oracle.FORCE_FULL)
+    p = np.float32(s0["confidence"][0])
+    for tau, expect in ((p, 0), (np.nextafter(p, np.float32(-1)), 1), (np.float32(1.0), 0)):
+        o2 = oracle.Oracle(TINY, model)
+        o2.prefill(synth.prompt(TINY))
+        s = o2.decode_step(tok, [tau], oracle.FORCE_FULL)
+        assert s["confidence"][0] == p and s["gate_pass"][0] == expect
+
+
+# ------------------------------------------------------------- structure
+def _trace_step(shape, model, force=oracle.FORCE_FULL, taus=(0.5,)):
+    o = oracle.Oracle(shape, model)
+    tok = o.prefill(synth.prompt(shape))
+    s = o.decode_step(tok, list(taus), force, trace=True)
+    return o, tok, s
+
+
+def test_residual_stream_passes_through_zeroed_layers():
+    """With every projection zero, each layer adds nothing: the residual at the
+    top is the input token's embedding row, and the logits are the
+    unembedding of its RMSNorm."""
+    shape = micro()
+    model = synth.make_model(shape)
+    for lw in model["layers"]:
+        for key in ("wq", "wk", "wv", "wo", "wg", "wu", "wd"):
+            lw[key] = zeros_like_bits(lw[key])
+    o, tok, s = _trace_step(shape, model)
+    E = synth.bf16_to_f32(model["embed"])
+    h = s["capture"]["h_final"]
+    assert np.array_equal(h, E[tok])
+    g = synth.bf16_to_f32(model["final_norm"]).astype(np.float64)
+    z = bf16_round(E[tok] / np.sqrt(np.mean(E[tok].astype(np.float64) ** 2) + shape.rms_eps) * g)
+    U = synth.bf16_to_f32(model["lm_head"]).astype(np.float64)
+    np.testing.assert_allclose(s["capture"]["final_logits"], U @ z, rtol=1e-5, atol=1e-5)
+
+
+def test_projection_orientations_and_wiring():
+    shape = micro()
+    d, A, KH, D, F = shape.d_model, shape.n_heads, shape.n_kv_heads, shape.head_dim, shape.ffn_dim
+    model = synth.make_model(shape)
+    lw = model["layers"][0]
+    lw["wo"] = one_hot_matrix(d, A * D, 5, 17)       # h_mid - h_in = o[17] at row 5
+    lw["wd"] = one_hot_matrix(d, F, 9, 40)           # h_out - h_mid = a[40] at row 9
+    o, tok, s = _trace_step(shape, model)
+    tr = s["capture"]["layer_trace"]
+    f = lambda name: o.trace_field(tr, 0, name).astype(np.float64)
+    E = synth.bf16_to_f32(model["embed"])
+    assert np.array_equal(f("h_in"), E[tok])
+    d_attn = f("h_mid") - f("h_in")
+    assert d_attn[5] == pytest.approx(f("o")[17], abs=1e-6) and np.count_nonzero(np.delete(d_attn, 5)) == 0
+    d_ffn = f("h_out") - f("h_mid")
+    assert d_ffn[9] == pytest.approx(f("a")[40], abs=1e-6) and np.count_nonzero(np.delete(d_ffn, 9)) == 0
+    # gate and up use W_g and W_u respectively; a = bf16(SiLU(gate) * up)
+    u = o.trace_field(tr, 0, "u_mlp")
+    np.testing.assert_array_equal(o.trace_field(tr, 0, "gate"), oracle.matvec(lw["wg"], u))
+    np.testing.assert_array_equal(o.trace_field(tr, 0, "up"), oracle.matvec(lw["wu"], u))
+    g, up = f("gate"), f("up")
+    np.testing.assert_array_equal(f("a"), bf16_round(oracle.silu(g) * up))
+    # q is W_q u rotated at the step's position; k and v are stored as bf16
+    t = o.pos - 1
+    ua = o.trace_field(tr, 0, "u_attn")
+    q_raw = oracle.matvec(lw["wq"], ua)
+    q_rot = np.concatenate([oracle.rope(q_raw[h * D:(h + 1) * D], t, shape.rope_base) for h in range(A)])
+    np.testing.assert_array_equal(o.trace_field(tr, 0, "q"), q_rot)
+    k_raw = oracle.matvec(lw["wk"], ua)
+    k_rot = np.concatenate([oracle.rope(k_raw[g_ * D:(g_ + 1) * D], t, shape.rope_base) for g_ in range(KH)])
+    kc, vc, src = o.kv(0, t)
+    np.testing.assert_array_equal(kc, bf16_round(k_rot))
+    np.testing.assert_array_equal(vc, bf16_round(oracle.matvec(lw["wv"], ua)))
+
+
+def test_grouped_query_attention_uses_head_div_group():
+    """Query head h reads key-value head h div (A/K)."""
+    shape = micro()
+    A, KH, D = shape.n_heads, shape.n_kv_heads, shape.head_dim
+    group = A // KH
+    for dead in range(KH):
+        model = synth.make_model(shape)
+        wv = synth.bf16_to_f32(model["layers"][1]["wv"]).copy()
+        wv[dead * D:(dead + 1) * D] = 0
+        model["layers"][1]["wv"] = to_bf16_bits(wv)
+        o, tok, s = _trace_step(shape, model)
+        ov = o.trace_field(s["capture"]["layer_trace"], 1, "o").reshape(A, D)
+        for h in range(A):
+            assert (np.count_nonzero(ov[h]) == 0) == (h // group == dead)
+
+
+def test_attention_output_is_softmax_over_cached_positions():
+    shape = micro()
+    A, KH, D = shape.n_heads, shape.n_kv_heads, shape.head_dim
+    model = synth.make_model(shape)
+    o, tok, s = _trace_step(shape, model)
+    tr = s["capture"]["layer_trace"]
+    t = o.pos - 1
+    for j in range(shape.n_layers):
+        q = o.trace_field(tr, j, "q").reshape(A, D).astype(np.float64)
+        Ks = np.stack([o.kv(j, p)[0] for p in range(t + 1)]).reshape(t + 1, KH, D).astype(np.float64)
+        Vs = np.stack([o.kv(j, p)[1] for p in range(t + 1)]).reshape(t + 1, KH, D).astype(np.float64)
+        got = o.trace_field(tr, j, "o").reshape(A, D)
+        for h in range(A):
+            g = h // (A // KH)
+            p = scipy.special.softmax(Ks[:, g] @ q[h] / math.sqrt(D))
+            np.testing.assert_allclose(got[h], bf16_round(p @ Vs[:, g]), rtol=1e-2, atol=1e-6)
+
+
+def test_readout_is_affine_then_final_norm_then_unembedding():
+    """Section 2 / Appendix B: y = W_r h + b_r, then the model's own final norm
+    and unembedding.  W_r = I + e_i e_j^T checks its orientation."""
+    shape = micro()
+    d = shape.d_model
+    model = synth.make_model(shape)
+    W = np.eye(d, dtype=np.float32)
+    W[3, 20] = 1.0
+    b = np.random.default_rng(3).standard_normal(d).astype(np.float32) * 0.1
+    model["readouts"] = [(2, to_bf16_bits(W), to_bf16_bits(b))]
+    o = oracle.Oracle(shape, model)
+    tok = o.prefill(synth.prompt(shape))
+    s = o.decode_step(tok, [1.01], capture=True)
+    h = s["capture"]["h_readout"][0].astype(np.float64)
+    hb = bf16_round(h).astype(np.float64)
+    expect = hb + bf16_round(b)
+    expect[3] += hb[20]
+    np.testing.assert_allclose(s["capture"]["y_readout"][0], expect, rtol=1e-6, atol=1e-7)
+    y = s["capture"]["y_readout"][0]
+    z = bf16_round(oracle.rmsnorm(y, model["final_norm"], shape.rms_eps))
+    np.testing.assert_array_equal(s["capture"]["readout_logits"][0], oracle.matvec(model["lm_head"], z))
+
+
+def test_prefill_equals_forced_full_decode():
+    shape = micro()
+    model = synth.make_model(shape)
+    ids = synth.prompt(shape, shape.prompt_len + 1)
+    a = oracle.Oracle(shape, model)
+    a.prefill(ids[:-1])
+    sa = a.decode_step(int(ids[-1]), [0.5], oracle.FORCE_FULL)
+    b = oracle.Oracle(shape, model)
+    fb = b.prefill(ids)
+    assert sa["token"] == fb
+    for j in range(shape.n_layers):
+        for t in range(len(ids)):
+            ka, va, _ = a.kv(j, t)
+            kb, vb, _ = b.kv(j, t)
+            assert np.array_equal(ka, kb) and np.array_equal(va, vb)
+
+
+def test_qkv_bias_and_tied_head_options():
+    shape = micro(qkv_bias=True, tied_embedding=True)
+    model = synth.make_model(shape)
+    assert model["lm_head"] is None and "bq" in model["layers"][0]
+    o, tok, s = _trace_step(shape, model)
+    tr = s["capture"]["layer_trace"]
+    lw = model["layers"][0]
+    ua = o.trace_field(tr, 0, "u_attn")
+    t = o.pos - 1
+    v_expect = bf16_round(oracle.matvec(lw["wv"], ua) + synth.bf16_to_f32(lw["bv"]))
+    np.testing.assert_allclose(o.kv(0, t)[1], v_expect, rtol=1e-2, atol=1e-6)
+    # tied: logits use the embedding matrix
+    z = bf16_round(oracle.rmsnorm(s["capture"]["h_final"], model["final_norm"], shape.rms_eps))
+    np.testing.assert_array_equal(s["capture"]["final_logits"], oracle.matvec(model["embed"], z))
+
+
+def test_errors_and_determinism():
+    shape = micro()
+    model = synth.make_model(shape)
+    o = oracle.Oracle(shape, model)
+    tok = o.prefill(synth.prompt(shape))
+    with pytest.raises(ValueError):
+        o.decode_step(-1, [0.5])
+    with pytest.raises(ValueError):
+        o.decode_step(shape.vocab, [0.5])
+    for _ in range(shape.new_tokens):
+        tok = o.decode_step(tok, [0.5])["token"]
+    with pytest.raises(ValueError):
+        o.decode_step(tok, [0.5])  # past max_ctx
+    _, f1, a = _run(shape, model, [0.4])
+    _, f2, b = _run(shape, model, [0.4])
+    assert [x["confidence"] for x in a] == [x["confidence"] for x in b]
