@@ -46,7 +46,7 @@ class Config(ctypes.Structure):
     _fields_ = [("n_layers", ctypes.c_int32), ("d_model", ctypes.c_int32), ("n_heads", ctypes.c_int32),
                 ("n_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32), ("ffn_dim", ctypes.c_int32),
                 ("vocab", ctypes.c_int32), ("max_ctx", ctypes.c_int32), ("rms_eps", ctypes.c_double),
-                ("rope_base", ctypes.c_double), ("qkv_bias", ctypes.c_int32), ("pure_fp32", ctypes.c_int32)]
+                ("rope_base", ctypes.c_double), ("qkv_bias", ctypes.c_int32), ("bf16_activations", ctypes.c_int32)]
 
 
 _P = ctypes.c_void_p
@@ -186,13 +186,14 @@ class Oracle:
     """A model instance: weights (numpy bf16 arrays, referenced, not copied),
     readouts, KV cache and position."""
 
-    def __init__(self, shape, model: dict, *, readouts=True, pure_fp32: bool = False, max_ctx: int | None = None):
+    def __init__(self, shape, model: dict, *, readouts=True, bf16_activations: bool = False,
+                 max_ctx: int | None = None):
         self.lib = _load()
         self.shape = shape
         L = shape.n_layers
         self.cfg = Config(L, shape.d_model, shape.n_heads, shape.n_kv_heads, shape.head_dim, shape.ffn_dim,
                           shape.vocab, int(max_ctx or shape.max_ctx), shape.rms_eps, shape.rope_base,
-                          int(shape.qkv_bias), int(pure_fp32))
+                          int(shape.qkv_bias), int(bf16_activations))
         self._keep = []
 
         def arr(a):

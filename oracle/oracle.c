@@ -34,11 +34,12 @@
  *   the lowest token id; prefill runs at full depth with no gate; with
  *   several readouts the shallowest passing one exits.
  *
- * Numerics contract: weights are bf16 values held exactly; every matmul
- * input activation (RMSNorm outputs, attention output, FFN product, readout
- * input) is rounded to bf16 (round to nearest even) unless pure_fp32 is set;
- * products accumulate in double; the residual stream, q, scores, softmax and
- * logits are float; the KV cache holds bf16 values.
+ * Numerics contract: weights are bf16 values held exactly; activations (the
+ * residual stream, RMSNorm outputs, q, scores, softmax, attention output, FFN
+ * product, readout output, logits) are float; products accumulate in double;
+ * the KV cache holds bf16 values (round to nearest even).  The option
+ * bf16_activations additionally rounds every matmul input activation to
+ * bf16, the half-precision activations the paper's own runs used.
  *
  * Parity pins (tests/test_oracle_pins.py, tests/test_oracle_model.py): every
  * exported op is checked against closed forms, library routines or brute
@@ -62,7 +63,7 @@
 typedef struct {
     int32_t n_layers, d_model, n_heads, n_kv_heads, head_dim, ffn_dim, vocab, max_ctx;
     double rms_eps, rope_base;
-    int32_t qkv_bias, pure_fp32;
+    int32_t qkv_bias, bf16_activations;
 } orc_config;
 
 /* Per-layer tensors are arrays of n_layers pointers to bf16 [out, in]. */
@@ -154,7 +155,7 @@ static inline float round_bf16(float f) {
 }
 
 static inline float act_round(const orc_model* m, float f) {
-    return m->c.pure_fp32 ? f : round_bf16(f);
+    return m->c.bf16_activations ? round_bf16(f) : f;
 }
 
 /* ------------------------------------------------------------------ */

@@ -1,0 +1,1082 @@
+// Host engine of libee: workspace layout, weight repack and upload, CUDA graph
+// construction, and the extern "C" entry points declared in include/ee.h.
+//
+// One decode step is one CUDA graph launch.  The graph holds layers 1..k, the
+// readout's affine map and vocabulary pass, and an IF/ELSE conditional node
+// whose condition the vocabulary pass sets on the device from p > tau: the
+// THEN body fills the skipped layers' KV entries, the ELSE body runs the next
+// segment of layers (and, with several readouts, the next readout and its own
+// conditional node, nested) down to the LM head.  ee_decode_n wraps the step
+// in a WHILE conditional node, so n steps run from one launch with the token
+// fed back in device memory and no host round trip.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "ee.h"
+#include "ee_internal.h"
+
+using namespace ee;
+
+namespace {
+
+thread_local std::string g_err = "";
+
+int fail(int code, const std::string& msg) {
+    g_err = msg;
+    return code;
+}
+
+#define EE_CK(call)                                                                                 \
+    do {                                                                                            \
+        cudaError_t e_ = (call);                                                                    \
+        if (e_ != cudaSuccess) return fail(EE_ECUDA, std::string(#call) + ": " + cudaGetErrorString(e_)); \
+    } while (0)
+
+#define EE_TRY(call)             \
+    do {                         \
+        int rc_ = (call);        \
+        if (rc_ != EE_OK) return rc_; \
+    } while (0)
+
+constexpr size_t kAlign = 256;
+constexpr int kMaxGemvCtas = 1024;
+constexpr int kMaxGemvWarps = kMaxGemvCtas * (kGemvThreads / 32);
+constexpr int kMaxVocabCtas = 1024;
+constexpr int kCaptureDepth = kMaxReadouts + 3;
+
+size_t align_up(size_t x, size_t a = kAlign) { return (x + a - 1) / a * a; }
+int64_t align_elems(int64_t x) { return (x + 127) / 128 * 128; }  // 256 bytes of bf16
+
+// Byte offsets of every region of the workspace.
+struct Layout {
+    size_t ctl, rope, layers, embed, lm_head, g_final, ro_w[kMaxReadouts], ro_b[kMaxReadouts];
+    size_t kpool, vpool, page_table, kv_src, h, q, o, a, y, hk, logits_ro, logits_final;
+    size_t gemv_part, gemv_ticket, attn_part, attn_ticket, vocab_part, vocab_ticket;
+    size_t prompt, sched, out_tok, out_exit, out_conf, total;
+    int64_t layer_stride, off_wqkv, off_bqkv, off_gattn, off_wo, off_gmlp, off_wgu, off_wd;
+    int64_t n_units_qkv, kv_layer_stride, gemv_part_stride, gemv_ticket_stride;
+    int n_pages;
+};
+
+int check_config(const ee_model_config* c) {
+    if (!c) return fail(EE_EINVAL, "config is NULL");
+    if (c->n_layers <= 0 || c->d_model <= 0 || c->n_heads <= 0 || c->n_kv_heads <= 0 || c->ffn_dim <= 0 ||
+        c->vocab <= 1 || c->max_ctx <= 0)
+        return fail(EE_EINVAL, "config: sizes must be positive");
+    if (c->head_dim != 64 && c->head_dim != 128) return fail(EE_EINVAL, "config: head_dim must be 64 or 128");
+    if (c->n_heads % c->n_kv_heads || c->n_heads / c->n_kv_heads > 8)
+        return fail(EE_EINVAL, "config: n_heads must be a multiple of n_kv_heads, group <= 8");
+    if (c->d_model % 8 || c->ffn_dim % 8 || (c->n_heads * c->head_dim) % 8)
+        return fail(EE_EINVAL, "config: d_model, ffn_dim and n_heads*head_dim must be multiples of 8");
+    if (c->d_model < 256 || c->ffn_dim < 256 || c->n_heads * c->head_dim < 256)
+        return fail(EE_EINVAL, "config: rows shorter than 256 elements are not supported");
+    if (c->page_size < 16 || c->page_size > 256 || (c->page_size & (c->page_size - 1)))
+        return fail(EE_EINVAL, "config: page_size must be a power of two in [16, 256]");
+    if (c->max_readouts < 0 || c->max_readouts > kMaxReadouts) return fail(EE_EINVAL, "config: max_readouts");
+    if (!(c->rms_eps >= 0.f) || !(c->rope_base > 0.f)) return fail(EE_EINVAL, "config: rms_eps / rope_base");
+    return EE_OK;
+}
+
+Layout make_layout(const ee_model_config& c) {
+    Layout l{};
+    const int64_t d = c.d_model, A = c.n_heads, KH = c.n_kv_heads, D = c.head_dim, F = c.ffn_dim, V = c.vocab;
+    const int64_t L = c.n_layers, R = std::max(1, c.max_readouts);
+    l.n_units_qkv = (A + 2 * KH) * D / 2;
+    int64_t o = 0;
+    l.off_wqkv = o;
+    o += align_elems(l.n_units_qkv * 2 * d);
+    l.off_bqkv = o;
+    o += align_elems(l.n_units_qkv * 2);
+    l.off_gattn = o;
+    o += align_elems(d);
+    l.off_wo = o;
+    o += align_elems(d * A * D);
+    l.off_gmlp = o;
+    o += align_elems(d);
+    l.off_wgu = o;
+    o += align_elems(F * 2 * d);
+    l.off_wd = o;
+    o += align_elems(d * F);
+    l.layer_stride = o;
+    l.n_pages = (c.max_ctx + c.page_size - 1) / c.page_size;
+    l.kv_layer_stride = (int64_t)l.n_pages * KH * c.page_size * D;
+    l.gemv_part_stride = (int64_t)kMaxGemvWarps * 2 * 2;
+    l.gemv_ticket_stride = align_elems(std::max<int64_t>({l.n_units_qkv, d, F}));
+
+    size_t b = 0;
+    auto take = [&](size_t bytes) {
+        const size_t at = b;
+        b = align_up(b + bytes);
+        return at;
+    };
+    l.ctl = take(sizeof(Ctl));
+    l.rope = take(sizeof(float2) * (size_t)c.max_ctx * (D / 2));
+    l.layers = take(2 * (size_t)l.layer_stride * L);
+    l.embed = take(2 * (size_t)V * d);
+    l.lm_head = c.tied_embedding ? l.embed : take(2 * (size_t)V * d);
+    l.g_final = take(2 * (size_t)d);
+    for (int r = 0; r < kMaxReadouts; ++r) {
+        if (r < c.max_readouts) {
+            l.ro_w[r] = take(2 * (size_t)d * d);
+            l.ro_b[r] = take(2 * (size_t)d);
+        } else {
+            l.ro_w[r] = l.ro_b[r] = 0;
+        }
+    }
+    l.kpool = take(2 * (size_t)l.kv_layer_stride * L);
+    l.vpool = take(2 * (size_t)l.kv_layer_stride * L);
+    l.page_table = take(4 * (size_t)l.n_pages);
+    l.kv_src = take((size_t)L * c.max_ctx);
+    l.h = take(4 * (size_t)d);
+    l.q = take(4 * (size_t)A * D);
+    l.o = take(4 * (size_t)A * D);
+    l.a = take(4 * (size_t)F);
+    l.y = take(4 * (size_t)R * d);
+    l.hk = take(4 * (size_t)R * d);
+    l.logits_ro = take(4 * (size_t)R * V);
+    l.logits_final = take(4 * (size_t)V);
+    l.gemv_part = take(4 * (size_t)l.gemv_part_stride * L);
+    l.gemv_ticket = take(4 * (size_t)l.gemv_ticket_stride * L);
+    l.attn_part = take(4 * (size_t)A * kAttnMaxSplits * (D + 2));
+    l.attn_ticket = take(4 * (size_t)KH);
+    l.vocab_part = take(4 * (size_t)kMaxVocabCtas * 4);
+    l.vocab_ticket = take(4);
+    l.prompt = take(4 * (size_t)c.max_ctx);
+    l.sched = take((size_t)c.max_ctx);
+    l.out_tok = take(4 * (size_t)c.max_ctx);
+    l.out_exit = take(4 * (size_t)c.max_ctx);
+    l.out_conf = take(4 * (size_t)c.max_ctx);
+    l.total = b;
+    return l;
+}
+
+}  // namespace
+
+struct ee_ctx {
+    ee_model_config cfg{};
+    Layout lay{};
+    cudaStream_t stream = nullptr;
+    cudaStream_t cap[kCaptureDepth] = {};
+    char* ws = nullptr;
+    bool own_ws = false;
+    int device = 0, n_sm = 0;
+    DevModel dm{};
+    Ctl* d_ctl = nullptr;
+    Ctl* h_ctl = nullptr;  // pinned mirror
+    int n_readouts = 0;
+    int ro_layer[kMaxReadouts] = {};
+    bool weights = false, started = false, prefilled = false;
+    int pos = 0;
+    bool use_graphs = true, use_pdl = true;
+    int dbg = 0;
+    cudaGraphExec_t g_step = nullptr, g_n = nullptr, g_prefill = nullptr;
+    int grid_gemv = 0, grid_vocab = 0;
+};
+
+namespace {
+
+void drop_graphs(ee_ctx* c) {
+    for (cudaGraphExec_t* g : {&c->g_step, &c->g_n, &c->g_prefill})
+        if (*g) {
+            cudaGraphExecDestroy(*g);
+            *g = nullptr;
+        }
+}
+
+// Grid of a flat GEMV launch: one CTA per SM, fewer when the matrix is small
+// (every warp keeps at least 32 chunks = 512 bytes).
+int gemv_grid(const ee_ctx* c, int64_t chunks) {
+    const int64_t per_cta = 32LL * (kGemvThreads / 32);
+    const int64_t g = std::max<int64_t>(1, chunks / per_cta);
+    return (int)std::min<int64_t>(g, c->grid_gemv);
+}
+
+AttnArgs attn_args(const ee_ctx* c, int j) {
+    const DevModel& m = c->dm;
+    AttnArgs a{};
+    a.q = m.q;
+    a.kp = m.kpool + (int64_t)j * m.kv_layer_stride;
+    a.vp = m.vpool + (int64_t)j * m.kv_layer_stride;
+    a.page_table = m.page_table;
+    a.ctl = m.ctl;
+    a.T = 0;
+    a.A = m.A;
+    a.KH = m.KH;
+    a.page_size = m.page_size;
+    a.out = m.o;
+    a.part = m.attn_part;
+    a.ticket = m.attn_ticket;
+    return a;
+}
+
+VocabArgs vocab_args(const ee_ctx* c, int mode, int r, int has_cond, cudaGraphConditionalHandle cond) {
+    const DevModel& m = c->dm;
+    VocabArgs v{};
+    v.x = mode == 1 ? m.y + (int64_t)r * m.d : m.h;
+    v.gain = m.g_final;
+    v.U = m.lm_head;
+    v.V = m.V;
+    v.d = m.d;
+    v.eps = m.eps;
+    v.logits = mode == 1 ? m.logits_ro + (int64_t)r * m.V : m.logits_final;
+    v.logits_if_dbg = 1;
+    v.part = m.vocab_part;
+    v.ticket = m.vocab_ticket;
+    v.mode = mode;
+    v.r = r;
+    v.ctl = m.ctl;
+    v.has_cond = has_cond;
+    v.cond = cond;
+    return v;
+}
+
+// Layers [j0, j1) of one step on stream s.  `pdl` is the attribute for the
+// first launch (false at the start of a graph body).
+int enqueue_layers(ee_ctx* c, cudaStream_t s, int j0, int j1, bool& pdl) {
+    const DevModel& m = c->dm;
+    const int64_t d = m.d, F = m.F, AD = (int64_t)m.A * m.D;
+    const int gq = gemv_grid(c, c->lay.n_units_qkv * 2 * d / 8);
+    const int go = gemv_grid(c, d * AD / 8);
+    const int gu = gemv_grid(c, F * 2 * d / 8);
+    const int gd = gemv_grid(c, d * F / 8);
+    for (int j = j0; j < j1; ++j) {
+        EE_CK(launch_qkv(m, j, j == 0 ? 1 : 0, gq, pdl, s));
+        pdl = c->use_pdl;
+        EE_CK(launch_attention(attn_args(c, j), m.D, pdl, s));
+        EE_CK(launch_oproj(m, j, go, pdl, s));
+        EE_CK(launch_gateup(m, j, gu, pdl, s));
+        EE_CK(launch_down(m, j, gd, pdl, s));
+    }
+    return EE_OK;
+}
+
+int enqueue_readout(ee_ctx* c, cudaStream_t s, int r, int has_cond, cudaGraphConditionalHandle cond, bool& pdl) {
+    const DevModel& m = c->dm;
+    EE_CK(launch_readout(m, r, gemv_grid(c, (int64_t)m.d * m.d / 8), pdl, s));
+    pdl = c->use_pdl;
+    EE_CK(launch_vocab(vocab_args(c, 1, r, has_cond, cond), c->grid_vocab, pdl, s));
+    return EE_OK;
+}
+
+int enqueue_head(ee_ctx* c, cudaStream_t s, bool& pdl) {
+    EE_CK(launch_vocab(vocab_args(c, 2, 0, 0, 0), c->grid_vocab, pdl, s));
+    pdl = c->use_pdl;
+    return EE_OK;
+}
+
+int enqueue_fill(ee_ctx* c, cudaStream_t s, int exit_layer, bool pdl) {
+    const DevModel& m = c->dm;
+    if (exit_layer >= m.L) return EE_OK;
+    const int nl = m.L - exit_layer;
+    const int64_t chunks = (int64_t)m.KH * m.D * 2 * m.d / 8;
+    const int gx = std::max(1, std::min(gemv_grid(c, chunks), (c->grid_gemv + nl - 1) / nl));
+    EE_CK(launch_kvfill(m, exit_layer, gx, pdl, s));
+    return EE_OK;
+}
+
+// Add a conditional node at the current capture point of stream s.
+int add_conditional(cudaStream_t s, cudaGraphConditionalHandle h, cudaGraphConditionalNodeType type,
+                    unsigned size, cudaGraph_t* bodies) {
+    cudaStreamCaptureStatus st;
+    cudaGraph_t g;
+    const cudaGraphNode_t* deps = nullptr;
+    size_t nd = 0;
+    EE_CK(cudaStreamGetCaptureInfo(s, &st, nullptr, &g, &deps, nullptr, &nd));
+    if (st != cudaStreamCaptureStatusActive) return fail(EE_ECUDA, "stream is not capturing");
+    cudaGraphNodeParams p{};
+    p.type = cudaGraphNodeTypeConditional;
+    p.conditional.handle = h;
+    p.conditional.type = type;
+    p.conditional.size = size;
+    cudaGraphNode_t node;
+    EE_CK(cudaGraphAddNode(&node, g, deps, nullptr, nd, &p));
+    for (unsigned i = 0; i < size; ++i) bodies[i] = p.conditional.phGraph_out[i];
+    EE_CK(cudaStreamUpdateCaptureDependencies(s, &node, nullptr, 1, cudaStreamSetCaptureDependencies));
+    return EE_OK;
+}
+
+int current_capture_graph(cudaStream_t s, cudaGraph_t* g) {
+    cudaStreamCaptureStatus st;
+    EE_CK(cudaStreamGetCaptureInfo(s, &st, nullptr, g, nullptr, nullptr, nullptr));
+    if (st != cudaStreamCaptureStatusActive) return fail(EE_ECUDA, "stream is not capturing");
+    return EE_OK;
+}
+
+// Capture layers j0.. of a step with readout r next, into the graph being
+// captured on c->cap[depth].
+int capture_segment(ee_ctx* c, int depth, int j0, int r) {
+    if (depth + 1 >= kCaptureDepth) return fail(EE_EINVAL, "too many nested readouts");
+    cudaStream_t s = c->cap[depth];
+    const int L = c->cfg.n_layers;
+    const int j1 = r < c->n_readouts ? c->ro_layer[r] : L;
+    bool pdl = false;
+    EE_TRY(enqueue_layers(c, s, j0, j1, pdl));
+    if (r >= c->n_readouts) return enqueue_head(c, s, pdl);
+    cudaGraph_t g;
+    EE_TRY(current_capture_graph(s, &g));
+    cudaGraphConditionalHandle h;
+    EE_CK(cudaGraphConditionalHandleCreate(&h, g, 0, 0));
+    EE_TRY(enqueue_readout(c, s, r, 1, h, pdl));
+    cudaGraph_t bodies[2];
+    EE_TRY(add_conditional(s, h, cudaGraphCondTypeIf, 2, bodies));
+    cudaStream_t s2 = c->cap[depth + 1];
+    // THEN: exit at layer j1, fill the layers above it
+    EE_CK(cudaStreamBeginCaptureToGraph(s2, bodies[0], nullptr, nullptr, 0, cudaStreamCaptureModeRelaxed));
+    int rc = EE_OK;
+    if (j1 < L) {
+        rc = enqueue_fill(c, s2, j1, false);
+    }
+    cudaGraph_t tmp;
+    cudaError_t e = cudaStreamEndCapture(s2, &tmp);
+    if (rc != EE_OK) return rc;
+    EE_CK(e);
+    if (j1 >= L) {
+        cudaGraphNode_t empty;
+        EE_CK(cudaGraphAddEmptyNode(&empty, bodies[0], nullptr, 0));
+    }
+    // ELSE: continue to the next readout or the LM head
+    EE_CK(cudaStreamBeginCaptureToGraph(s2, bodies[1], nullptr, nullptr, 0, cudaStreamCaptureModeRelaxed));
+    rc = capture_segment(c, depth + 1, j1, r + 1);
+    e = cudaStreamEndCapture(s2, &tmp);
+    if (rc != EE_OK) return rc;
+    EE_CK(e);
+    return EE_OK;
+}
+
+int instantiate(cudaGraph_t g, cudaGraphExec_t* out) {
+    cudaError_t e = cudaGraphInstantiate(out, g, 0);
+    cudaGraphDestroy(g);
+    EE_CK(e);
+    return EE_OK;
+}
+
+int build_step_graph(ee_ctx* c) {
+    cudaStream_t s = c->cap[0];
+    EE_CK(cudaStreamBeginCapture(s, cudaStreamCaptureModeRelaxed));
+    int rc = capture_segment(c, 0, 0, 0);
+    if (rc == EE_OK) {
+        cudaError_t e = launch_step_end(c->dm, 0, 0, false, s);
+        if (e != cudaSuccess) rc = fail(EE_ECUDA, std::string("step_end: ") + cudaGetErrorString(e));
+    }
+    cudaGraph_t g = nullptr;
+    cudaError_t e = cudaStreamEndCapture(s, &g);
+    if (rc != EE_OK) {
+        if (g) cudaGraphDestroy(g);
+        return rc;
+    }
+    EE_CK(e);
+    return instantiate(g, &c->g_step);
+}
+
+// A graph holding one WHILE conditional node whose body is captured by
+// `fill_body` on c->cap[1]; the body's last kernel sets the condition.
+// Optional `tail` work is captured after the loop on c->cap[0].
+template <class Body, class Tail>
+int build_while_graph(ee_ctx* c, cudaGraphExec_t* out, Body fill_body, Tail tail) {
+    cudaGraph_t g = nullptr;
+    EE_CK(cudaGraphCreate(&g, 0));
+    int rc = EE_OK;
+    do {
+        cudaGraphConditionalHandle h;
+        cudaError_t e = cudaGraphConditionalHandleCreate(&h, g, 1, cudaGraphCondAssignDefault);
+        if (e != cudaSuccess) {
+            rc = fail(EE_ECUDA, std::string("while handle: ") + cudaGetErrorString(e));
+            break;
+        }
+        cudaGraphNodeParams p{};
+        p.type = cudaGraphNodeTypeConditional;
+        p.conditional.handle = h;
+        p.conditional.type = cudaGraphCondTypeWhile;
+        p.conditional.size = 1;
+        cudaGraphNode_t loop;
+        e = cudaGraphAddNode(&loop, g, nullptr, nullptr, 0, &p);
+        if (e != cudaSuccess) {
+            rc = fail(EE_ECUDA, std::string("while node: ") + cudaGetErrorString(e));
+            break;
+        }
+        cudaGraph_t body = p.conditional.phGraph_out[0];
+        cudaStream_t s1 = c->cap[1];
+        e = cudaStreamBeginCaptureToGraph(s1, body, nullptr, nullptr, 0, cudaStreamCaptureModeRelaxed);
+        if (e != cudaSuccess) {
+            rc = fail(EE_ECUDA, std::string("body capture: ") + cudaGetErrorString(e));
+            break;
+        }
+        rc = fill_body(s1, h);
+        cudaGraph_t tmp = nullptr;
+        e = cudaStreamEndCapture(s1, &tmp);
+        if (rc == EE_OK && e != cudaSuccess) rc = fail(EE_ECUDA, std::string("body end: ") + cudaGetErrorString(e));
+        if (rc != EE_OK) break;
+        cudaStream_t s0 = c->cap[0];
+        e = cudaStreamBeginCaptureToGraph(s0, g, &loop, nullptr, 1, cudaStreamCaptureModeRelaxed);
+        if (e != cudaSuccess) {
+            rc = fail(EE_ECUDA, std::string("tail capture: ") + cudaGetErrorString(e));
+            break;
+        }
+        rc = tail(s0);
+        e = cudaStreamEndCapture(s0, &tmp);
+        if (rc == EE_OK && e != cudaSuccess) rc = fail(EE_ECUDA, std::string("tail end: ") + cudaGetErrorString(e));
+    } while (0);
+    if (rc != EE_OK) {
+        cudaGraphDestroy(g);
+        return rc;
+    }
+    return instantiate(g, out);
+}
+
+// n gated steps: WHILE { step body; step_end sets (step < n_steps) }.
+int build_loop_graph(ee_ctx* c) {
+    return build_while_graph(
+        c, &c->g_n,
+        [c](cudaStream_t s1, cudaGraphConditionalHandle h) -> int {
+            EE_TRY(capture_segment(c, 1, 0, 0));
+            EE_CK(launch_step_end(c->dm, 1, h, false, s1));
+            return EE_OK;
+        },
+        [](cudaStream_t) -> int { return EE_OK; });
+}
+
+// Prefill: WHILE { all layers at the prompt position; advance }, then the LM
+// head on the last position and the hand-over of its token.
+int build_prefill_graph(ee_ctx* c) {
+    return build_while_graph(
+        c, &c->g_prefill,
+        [c](cudaStream_t s1, cudaGraphConditionalHandle h) -> int {
+            bool pdl = false;
+            EE_TRY(enqueue_layers(c, s1, 0, c->cfg.n_layers, pdl));
+            EE_CK(launch_prefill_advance(c->dm, 1, h, c->use_pdl, s1));
+            return EE_OK;
+        },
+        [c](cudaStream_t s0) -> int {
+            bool pdl = false;
+            EE_TRY(enqueue_head(c, s0, pdl));
+            EE_CK(launch_prefill_end(c->dm, c->use_pdl, s0));
+            return EE_OK;
+        });
+}
+
+int ensure_graphs(ee_ctx* c) {
+    if (!c->g_step) EE_TRY(build_step_graph(c));
+    if (!c->g_n) EE_TRY(build_loop_graph(c));
+    if (!c->g_prefill) EE_TRY(build_prefill_graph(c));
+    return EE_OK;
+}
+
+int fetch_ctl(ee_ctx* c) {
+    EE_CK(cudaMemcpyAsync(c->h_ctl, c->d_ctl, sizeof(Ctl), cudaMemcpyDeviceToHost, c->stream));
+    EE_CK(cudaStreamSynchronize(c->stream));
+    return EE_OK;
+}
+
+int device_error(const ee_ctx* c) {
+    const int e = c->h_ctl->err;
+    if (!e) return EE_OK;
+    std::string m = "device error:";
+    if (e & kErrNanConfidence) m += " non-finite confidence;";
+    if (e & kErrTokenRange) m += " token out of range;";
+    if (e & kErrPosition) m += " position beyond max_ctx;";
+    return fail(EE_EDEVICE, m);
+}
+
+CtlInputs base_inputs(const ee_ctx* c, const float* taus) {
+    CtlInputs in{};
+    in.set_token = 0;
+    in.n_steps = 1;
+    in.dbg = c->dbg;
+    for (int r = 0; r < kMaxReadouts; ++r) in.tau[r] = (taus && r < c->n_readouts) ? taus[r] : 2.0f;
+    return in;
+}
+
+// Direct launches with the branch taken on the host (EE_OPT_GRAPHS = 0).
+int eager_step(ee_ctx* c) {
+    cudaStream_t s = c->stream;
+    const DevModel& m = c->dm;
+    bool pdl = false;
+    int j0 = 0;
+    for (int r = 0; r <= c->n_readouts; ++r) {
+        const int j1 = r < c->n_readouts ? c->ro_layer[r] : m.L;
+        EE_TRY(enqueue_layers(c, s, j0, j1, pdl));
+        if (r == c->n_readouts) {
+            EE_TRY(enqueue_head(c, s, pdl));
+            break;
+        }
+        EE_TRY(enqueue_readout(c, s, r, 0, 0, pdl));
+        EE_TRY(fetch_ctl(c));
+        pdl = false;
+        if (c->h_ctl->exit_readout == r) {
+            EE_TRY(enqueue_fill(c, s, j1, false));
+            break;
+        }
+        j0 = j1;
+    }
+    EE_CK(launch_step_end(m, 0, 0, false, s));
+    return EE_OK;
+}
+
+}  // namespace
+
+// ======================================================================
+// extern "C" entry points
+// ======================================================================
+
+extern "C" {
+
+const char* ee_last_error(void) { return g_err.c_str(); }
+
+int ee_workspace_bytes(const ee_model_config* cfg, size_t* bytes) {
+    EE_TRY(check_config(cfg));
+    if (!bytes) return fail(EE_EINVAL, "bytes is NULL");
+    *bytes = make_layout(*cfg).total;
+    return EE_OK;
+}
+
+int ee_create(const ee_model_config* cfg, void* d_workspace, size_t workspace_bytes, void* stream, ee_ctx** out) {
+    EE_TRY(check_config(cfg));
+    if (!out) return fail(EE_EINVAL, "out is NULL");
+    *out = nullptr;
+    if (d_workspace && ((uintptr_t)d_workspace % kAlign)) return fail(EE_EINVAL, "workspace not 256-byte aligned");
+    ee_ctx* c = new ee_ctx();
+    c->cfg = *cfg;
+    c->lay = make_layout(*cfg);
+    c->stream = (cudaStream_t)stream;
+    auto bail = [&](int rc) {
+        ee_destroy(c);
+        return rc;
+    };
+    if (cudaGetDevice(&c->device) != cudaSuccess) return bail(fail(EE_ECUDA, "no CUDA device"));
+    cudaDeviceGetAttribute(&c->n_sm, cudaDevAttrMultiProcessorCount, c->device);
+    c->grid_gemv = std::min(c->n_sm, kMaxGemvCtas);
+    c->grid_vocab = std::min(c->n_sm, kMaxVocabCtas);
+    if (d_workspace) {
+        if (workspace_bytes < c->lay.total) return bail(fail(EE_ENOMEM, "workspace too small"));
+        c->ws = (char*)d_workspace;
+    } else {
+        if (cudaMalloc(&c->ws, c->lay.total) != cudaSuccess) {
+            c->ws = nullptr;
+            return bail(fail(EE_ENOMEM, "cudaMalloc of the workspace failed"));
+        }
+        c->own_ws = true;
+    }
+    for (int i = 0; i < kCaptureDepth; ++i)
+        if (cudaStreamCreateWithFlags(&c->cap[i], cudaStreamNonBlocking) != cudaSuccess)
+            return bail(fail(EE_ECUDA, "stream creation failed"));
+    if (cudaMallocHost(&c->h_ctl, sizeof(Ctl)) != cudaSuccess) return bail(fail(EE_ENOMEM, "pinned alloc failed"));
+    const Layout& l = c->lay;
+    char* w = c->ws;
+    DevModel& m = c->dm;
+    m.L = cfg->n_layers;
+    m.d = cfg->d_model;
+    m.A = cfg->n_heads;
+    m.KH = cfg->n_kv_heads;
+    m.D = cfg->head_dim;
+    m.F = cfg->ffn_dim;
+    m.V = cfg->vocab;
+    m.max_ctx = cfg->max_ctx;
+    m.page_size = cfg->page_size;
+    m.n_pages = l.n_pages;
+    m.qkv_bias = cfg->qkv_bias;
+    m.n_readouts = 0;
+    m.eps = cfg->rms_eps;
+    m.layers = (const uint16_t*)(w + l.layers);
+    m.layer_stride = l.layer_stride;
+    m.off_wqkv = l.off_wqkv;
+    m.off_bqkv = l.off_bqkv;
+    m.off_gattn = l.off_gattn;
+    m.off_wo = l.off_wo;
+    m.off_gmlp = l.off_gmlp;
+    m.off_wgu = l.off_wgu;
+    m.off_wd = l.off_wd;
+    m.embed = (const uint16_t*)(w + l.embed);
+    m.lm_head = (const uint16_t*)(w + l.lm_head);
+    m.g_final = (const uint16_t*)(w + l.g_final);
+    for (int r = 0; r < cfg->max_readouts; ++r) {
+        m.ro_w[r] = (const uint16_t*)(w + l.ro_w[r]);
+        m.ro_b[r] = (const uint16_t*)(w + l.ro_b[r]);
+    }
+    m.rope = (const float2*)(w + l.rope);
+    m.kpool = (uint16_t*)(w + l.kpool);
+    m.vpool = (uint16_t*)(w + l.vpool);
+    m.kv_layer_stride = l.kv_layer_stride;
+    m.page_table = (const int32_t*)(w + l.page_table);
+    m.kv_src = (int8_t*)(w + l.kv_src);
+    m.h = (float*)(w + l.h);
+    m.q = (float*)(w + l.q);
+    m.o = (float*)(w + l.o);
+    m.a = (float*)(w + l.a);
+    m.y = (float*)(w + l.y);
+    m.hk = (float*)(w + l.hk);
+    m.logits_ro = (float*)(w + l.logits_ro);
+    m.logits_final = (float*)(w + l.logits_final);
+    m.gemv_part = (float*)(w + l.gemv_part);
+    m.gemv_ticket = (int*)(w + l.gemv_ticket);
+    m.gemv_part_stride = l.gemv_part_stride;
+    m.gemv_ticket_stride = l.gemv_ticket_stride;
+    m.attn_part = (float*)(w + l.attn_part);
+    m.attn_ticket = (int*)(w + l.attn_ticket);
+    m.vocab_part = (float*)(w + l.vocab_part);
+    m.vocab_ticket = (int*)(w + l.vocab_ticket);
+    m.ctl = (Ctl*)(w + l.ctl);
+    c->d_ctl = m.ctl;
+
+    const int kmax = std::max({2 * m.d, m.A * m.D, m.F});
+    if (configure_kernels(kmax) != cudaSuccess) return bail(fail(EE_ECUDA, "kernel configuration failed"));
+
+    // RoPE table: angle t * base^(-2i/D) in double, cos/sin rounded to fp32.
+    std::vector<float2> rope((size_t)m.max_ctx * (m.D / 2));
+    for (int t = 0; t < m.max_ctx; ++t)
+        for (int i = 0; i < m.D / 2; ++i) {
+            const double ang = (double)t * std::pow((double)cfg->rope_base, -2.0 * i / (double)m.D);
+            rope[(size_t)t * (m.D / 2) + i] = make_float2((float)std::cos(ang), (float)std::sin(ang));
+        }
+    if (cudaMemcpy(w + l.rope, rope.data(), rope.size() * sizeof(float2), cudaMemcpyHostToDevice) != cudaSuccess)
+        return bail(fail(EE_ECUDA, "rope upload failed"));
+    std::vector<int32_t> pt(l.n_pages);
+    for (int i = 0; i < l.n_pages; ++i) pt[i] = i;
+    if (cudaMemcpy(w + l.page_table, pt.data(), pt.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess)
+        return bail(fail(EE_ECUDA, "page table upload failed"));
+    // zero the arrival counters (kernels return them to zero after use)
+    if (cudaMemset(w + l.gemv_ticket, 0, 4 * (size_t)l.gemv_ticket_stride * m.L) != cudaSuccess ||
+        cudaMemset(w + l.attn_ticket, 0, 4 * (size_t)m.KH) != cudaSuccess ||
+        cudaMemset(w + l.vocab_ticket, 0, 4) != cudaSuccess)
+        return bail(fail(EE_ECUDA, "memset failed"));
+    *out = c;
+    int rc = ee_reset(c);
+    if (rc != EE_OK) {
+        *out = nullptr;
+        return bail(rc);
+    }
+    return EE_OK;
+}
+
+int ee_destroy(ee_ctx* c) {
+    if (!c) return EE_OK;
+    if (c->stream || c->ws) cudaStreamSynchronize(c->stream);
+    drop_graphs(c);
+    for (int i = 0; i < kCaptureDepth; ++i)
+        if (c->cap[i]) cudaStreamDestroy(c->cap[i]);
+    if (c->h_ctl) cudaFreeHost(c->h_ctl);
+    if (c->own_ws && c->ws) cudaFree(c->ws);
+    delete c;
+    return EE_OK;
+}
+
+int ee_load_weights(ee_ctx* c, const ee_host_weights* w) {
+    if (!c || !w) return fail(EE_EINVAL, "NULL argument");
+    const ee_model_config& cf = c->cfg;
+    const int L = cf.n_layers;
+    const int64_t d = cf.d_model, A = cf.n_heads, KH = cf.n_kv_heads, D = cf.head_dim, F = cf.ffn_dim,
+                  V = cf.vocab;
+    if (!w->embed || !w->final_norm || (!cf.tied_embedding && !w->lm_head) || !w->attn_norm || !w->wq || !w->wk ||
+        !w->wv || !w->wo || !w->mlp_norm || !w->wg || !w->wu || !w->wd)
+        return fail(EE_EINVAL, "missing weight array");
+    if (cf.qkv_bias && (!w->bq || !w->bk || !w->bv)) return fail(EE_EINVAL, "missing bias array");
+    for (int j = 0; j < L; ++j)
+        if (!w->attn_norm[j] || !w->wq[j] || !w->wk[j] || !w->wv[j] || !w->wo[j] || !w->mlp_norm[j] || !w->wg[j] ||
+            !w->wu[j] || !w->wd[j] || (cf.qkv_bias && (!w->bq[j] || !w->bk[j] || !w->bv[j])))
+            return fail(EE_EINVAL, "missing per-layer weight");
+    const Layout& l = c->lay;
+    uint16_t* stage = nullptr;
+    EE_CK(cudaMallocHost(&stage, 2 * (size_t)l.layer_stride));
+    std::memset(stage, 0, 2 * (size_t)l.layer_stride);
+    int rc = EE_OK;
+    const int64_t half = D / 2;
+    auto copy_row = [&](uint16_t* dst, const uint16_t* src) { std::memcpy(dst, src, 2 * (size_t)d); };
+    for (int j = 0; j < L && rc == EE_OK; ++j) {
+        // Q/K/V: units are row pairs (i, i + D/2) of one head, Q heads then K then V
+        uint16_t* wqkv = stage + l.off_wqkv;
+        uint16_t* bqkv = stage + l.off_bqkv;
+        int64_t u = 0;
+        const uint16_t* mats[3] = {w->wq[j], w->wk[j], w->wv[j]};
+        const uint16_t* bias[3] = {cf.qkv_bias ? w->bq[j] : nullptr, cf.qkv_bias ? w->bk[j] : nullptr,
+                                   cf.qkv_bias ? w->bv[j] : nullptr};
+        const int64_t heads[3] = {A, KH, KH};
+        for (int t = 0; t < 3; ++t)
+            for (int64_t h = 0; h < heads[t]; ++h)
+                for (int64_t i = 0; i < half; ++i, ++u) {
+                    const int64_t r0 = h * D + i, r1 = h * D + i + half;
+                    copy_row(wqkv + (u * 2 + 0) * d, mats[t] + r0 * d);
+                    copy_row(wqkv + (u * 2 + 1) * d, mats[t] + r1 * d);
+                    if (bias[t]) {
+                        bqkv[u * 2 + 0] = bias[t][r0];
+                        bqkv[u * 2 + 1] = bias[t][r1];
+                    }
+                }
+        std::memcpy(stage + l.off_gattn, w->attn_norm[j], 2 * (size_t)d);
+        std::memcpy(stage + l.off_wo, w->wo[j], 2 * (size_t)d * A * D);
+        std::memcpy(stage + l.off_gmlp, w->mlp_norm[j], 2 * (size_t)d);
+        // gate/up: unit i is (W_g row i, W_u row i)
+        uint16_t* wgu = stage + l.off_wgu;
+        for (int64_t i = 0; i < F; ++i) {
+            copy_row(wgu + (i * 2 + 0) * d, w->wg[j] + i * d);
+            copy_row(wgu + (i * 2 + 1) * d, w->wu[j] + i * d);
+        }
+        std::memcpy(stage + l.off_wd, w->wd[j], 2 * (size_t)d * F);
+        cudaError_t e = cudaMemcpy(c->ws + l.layers + 2 * (size_t)l.layer_stride * j, stage,
+                                   2 * (size_t)l.layer_stride, cudaMemcpyHostToDevice);
+        if (e != cudaSuccess) rc = fail(EE_ECUDA, std::string("layer upload: ") + cudaGetErrorString(e));
+    }
+    cudaFreeHost(stage);
+    if (rc != EE_OK) return rc;
+    EE_CK(cudaMemcpy(c->ws + l.embed, w->embed, 2 * (size_t)V * d, cudaMemcpyHostToDevice));
+    if (!cf.tied_embedding) EE_CK(cudaMemcpy(c->ws + l.lm_head, w->lm_head, 2 * (size_t)V * d, cudaMemcpyHostToDevice));
+    EE_CK(cudaMemcpy(c->ws + l.g_final, w->final_norm, 2 * (size_t)d, cudaMemcpyHostToDevice));
+    c->weights = true;
+    drop_graphs(c);
+    return EE_OK;
+}
+
+int ee_add_readout(ee_ctx* c, int layer, const uint16_t* wr, const uint16_t* br, int* readout_id) {
+    if (!c || !wr || !br) return fail(EE_EINVAL, "NULL argument");
+    if (c->started) return fail(EE_ESTATE, "readouts must be added before the first prefill");
+    if (c->n_readouts >= c->cfg.max_readouts) return fail(EE_EINVAL, "max_readouts reached");
+    if (layer < 1 || layer > c->cfg.n_layers) return fail(EE_EINVAL, "readout layer outside [1, n_layers]");
+    if (c->n_readouts > 0 && layer <= c->ro_layer[c->n_readouts - 1])
+        return fail(EE_EINVAL, "readouts must be added in increasing layer order");
+    const int r = c->n_readouts;
+    const size_t d = c->cfg.d_model;
+    EE_CK(cudaMemcpy(c->ws + c->lay.ro_w[r], wr, 2 * d * d, cudaMemcpyHostToDevice));
+    EE_CK(cudaMemcpy(c->ws + c->lay.ro_b[r], br, 2 * d, cudaMemcpyHostToDevice));
+    c->ro_layer[r] = layer;
+    c->dm.ro_layer[r] = layer;
+    c->n_readouts = r + 1;
+    c->dm.n_readouts = r + 1;
+    drop_graphs(c);
+    if (readout_id) *readout_id = r;
+    return EE_OK;
+}
+
+int ee_set_page_table(ee_ctx* c, const int32_t* pages, int n_pages) {
+    if (!c || !pages) return fail(EE_EINVAL, "NULL argument");
+    if (n_pages != c->lay.n_pages) return fail(EE_EINVAL, "page table must cover every logical page");
+    if (c->prefilled) return fail(EE_ESTATE, "page table can only change between reset and prefill");
+    std::vector<char> seen(n_pages, 0);
+    for (int i = 0; i < n_pages; ++i) {
+        if (pages[i] < 0 || pages[i] >= n_pages || seen[pages[i]]) return fail(EE_EINVAL, "not a permutation");
+        seen[pages[i]] = 1;
+    }
+    EE_CK(cudaMemcpyAsync(c->ws + c->lay.page_table, pages, 4 * (size_t)n_pages, cudaMemcpyHostToDevice, c->stream));
+    EE_CK(cudaStreamSynchronize(c->stream));
+    return EE_OK;
+}
+
+int ee_reset(ee_ctx* c) {
+    if (!c) return fail(EE_EINVAL, "NULL context");
+    EE_CK(cudaStreamSynchronize(c->stream));
+    std::memset(c->h_ctl, 0, sizeof(Ctl));
+    c->h_ctl->exit_readout = -1;
+    c->h_ctl->full_token = -1;
+    c->h_ctl->max_ctx = c->cfg.max_ctx;
+    EE_CK(cudaMemcpyAsync(c->d_ctl, c->h_ctl, sizeof(Ctl), cudaMemcpyHostToDevice, c->stream));
+    EE_CK(cudaMemsetAsync(c->ws + c->lay.kv_src, 0, (size_t)c->cfg.n_layers * c->cfg.max_ctx, c->stream));
+    EE_CK(cudaStreamSynchronize(c->stream));
+    c->pos = 0;
+    c->prefilled = false;
+    return EE_OK;
+}
+
+int ee_set_option(ee_ctx* c, int option, int value) {
+    if (!c) return fail(EE_EINVAL, "NULL context");
+    switch (option) {
+        case EE_OPT_GRAPHS:
+            c->use_graphs = value != 0;
+            return EE_OK;
+        case EE_OPT_PDL:
+            if (c->use_pdl != (value != 0)) drop_graphs(c);
+            c->use_pdl = value != 0;
+            return EE_OK;
+        case EE_OPT_DEBUG_LOGITS:
+            c->dbg = value != 0;
+            return EE_OK;
+        default:
+            return fail(EE_EINVAL, "unknown option");
+    }
+}
+
+int ee_prefill(ee_ctx* c, const int32_t* ids, int n, int32_t* first_token) {
+    if (!c || !ids) return fail(EE_EINVAL, "NULL argument");
+    if (!c->weights) return fail(EE_ESTATE, "weights not loaded");
+    if (c->prefilled || c->pos != 0) return fail(EE_ESTATE, "prefill needs a fresh or reset context");
+    if (n <= 0) return fail(EE_EINVAL, "empty prompt");
+    if (n > c->cfg.max_ctx) return fail(EE_ERANGE, "prompt longer than max_ctx");
+    for (int i = 0; i < n; ++i)
+        if (ids[i] < 0 || ids[i] >= c->cfg.vocab) return fail(EE_EINVAL, "prompt token out of range");
+    c->started = true;
+    cudaStream_t s = c->stream;
+    int32_t* d_prompt = (int32_t*)(c->ws + c->lay.prompt);
+    EE_CK(cudaMemcpyAsync(d_prompt, ids, 4 * (size_t)n, cudaMemcpyHostToDevice, s));
+    CtlInputs in = base_inputs(c, nullptr);
+    in.set_token = 1;
+    in.in_tok = ids[0];
+    in.prefill_n = n;
+    in.prompt = d_prompt;
+    EE_CK(launch_set_inputs(c->d_ctl, in, s));
+    if (c->use_graphs) {
+        EE_TRY(ensure_graphs(c));
+        EE_CK(cudaGraphLaunch(c->g_prefill, s));
+    } else {
+        for (int i = 0; i < n; ++i) {
+            bool pdl = false;
+            EE_TRY(enqueue_layers(c, s, 0, c->cfg.n_layers, pdl));
+            EE_CK(launch_prefill_advance(c->dm, 0, 0, false, s));
+        }
+        bool pdl = false;
+        EE_TRY(enqueue_head(c, s, pdl));
+        EE_CK(launch_prefill_end(c->dm, false, s));
+    }
+    EE_TRY(fetch_ctl(c));
+    EE_TRY(device_error(c));
+    c->pos = c->h_ctl->pos;
+    if (c->pos != n) return fail(EE_EDEVICE, "prefill ended at an unexpected position");
+    c->prefilled = true;
+    if (first_token) *first_token = c->h_ctl->token;
+    return EE_OK;
+}
+
+int ee_decode_step(ee_ctx* c, int32_t input_token, const float* taus, int force, ee_step_result* out) {
+    if (!c || !out) return fail(EE_EINVAL, "NULL argument");
+    if (!c->prefilled) return fail(EE_ESTATE, "decode before prefill");
+    if (input_token < -1 || input_token >= c->cfg.vocab) return fail(EE_EINVAL, "input token out of range");
+    if (c->n_readouts > 0 && !taus) return fail(EE_EINVAL, "taus is NULL");
+    if (force < 0 || force > 1 + c->n_readouts) return fail(EE_EINVAL, "bad force value");
+    if (c->pos + 1 > c->cfg.max_ctx) return fail(EE_ERANGE, "position would pass max_ctx");
+    cudaStream_t s = c->stream;
+    CtlInputs in = base_inputs(c, taus);
+    in.set_token = input_token >= 0;
+    in.in_tok = input_token;
+    in.force = force;
+    EE_CK(launch_set_inputs(c->d_ctl, in, s));
+    if (c->use_graphs) {
+        EE_TRY(ensure_graphs(c));
+        EE_CK(cudaGraphLaunch(c->g_step, s));
+    } else {
+        EE_TRY(eager_step(c));
+    }
+    EE_TRY(fetch_ctl(c));
+    EE_TRY(device_error(c));
+    const Ctl* h = c->h_ctl;
+    std::memset(out, 0, sizeof(*out));
+    out->token = h->token;
+    out->exit_readout = h->exit_readout;
+    out->exited = h->exit_readout >= 0;
+    out->exit_layer = h->exit_readout >= 0 ? c->ro_layer[h->exit_readout] : c->cfg.n_layers;
+    out->n_evaluated = h->n_evaluated;
+    out->full_token = h->exit_readout >= 0 ? -1 : h->full_token;
+    for (int r = 0; r < h->n_evaluated && r < kMaxReadouts; ++r) {
+        out->gate_pass[r] = h->gate_pass[r];
+        out->readout_token[r] = h->readout_token[r];
+        out->confidence[r] = h->conf[r];
+    }
+    out->full_confidence = h->exit_readout >= 0 ? 0.f : h->full_conf;
+    c->pos = h->pos;
+    return EE_OK;
+}
+
+int ee_decode_n(ee_ctx* c, int n, int32_t input_token, const float* taus, const int8_t* force_schedule,
+                int32_t* tokens, int32_t* exit_readout, float* confidence, int where) {
+    if (!c) return fail(EE_EINVAL, "NULL context");
+    if (!c->prefilled) return fail(EE_ESTATE, "decode before prefill");
+    if (n <= 0) return fail(EE_EINVAL, "n must be positive");
+    if (input_token < -1 || input_token >= c->cfg.vocab) return fail(EE_EINVAL, "input token out of range");
+    if (c->n_readouts > 0 && !taus) return fail(EE_EINVAL, "taus is NULL");
+    if (where != EE_HOST && where != EE_DEVICE) return fail(EE_EINVAL, "where must be EE_HOST or EE_DEVICE");
+    if (c->pos + n > c->cfg.max_ctx) return fail(EE_ERANGE, "steps would pass max_ctx");
+    if (force_schedule)
+        for (int i = 0; i < n; ++i)
+            if (force_schedule[i] < 0 || force_schedule[i] > 1 + c->n_readouts)
+                return fail(EE_EINVAL, "bad force schedule entry");
+    cudaStream_t s = c->stream;
+    CtlInputs in = base_inputs(c, taus);
+    in.set_token = input_token >= 0;
+    in.in_tok = input_token;
+    in.force = EE_FREE;
+    in.n_steps = n;
+    if (force_schedule) {
+        int8_t* d_sched = (int8_t*)(c->ws + c->lay.sched);
+        EE_CK(cudaMemcpyAsync(d_sched, force_schedule, (size_t)n, cudaMemcpyHostToDevice, s));
+        in.sched = d_sched;
+    }
+    int32_t* d_tok = (int32_t*)(c->ws + c->lay.out_tok);
+    int32_t* d_exit = (int32_t*)(c->ws + c->lay.out_exit);
+    float* d_conf = (float*)(c->ws + c->lay.out_conf);
+    if (where == EE_DEVICE) {
+        in.out_tokens = tokens;
+        in.out_exit = exit_readout;
+        in.out_conf = confidence;
+    } else {
+        in.out_tokens = tokens ? d_tok : nullptr;
+        in.out_exit = exit_readout ? d_exit : nullptr;
+        in.out_conf = confidence ? d_conf : nullptr;
+    }
+    EE_CK(launch_set_inputs(c->d_ctl, in, s));
+    if (c->use_graphs) {
+        EE_TRY(ensure_graphs(c));
+        EE_CK(cudaGraphLaunch(c->g_n, s));
+    } else {
+        for (int i = 0; i < n; ++i) EE_TRY(eager_step(c));
+    }
+    c->pos += n;
+    if (where == EE_HOST) {
+        if (tokens) EE_CK(cudaMemcpyAsync(tokens, d_tok, 4 * (size_t)n, cudaMemcpyDeviceToHost, s));
+        if (exit_readout) EE_CK(cudaMemcpyAsync(exit_readout, d_exit, 4 * (size_t)n, cudaMemcpyDeviceToHost, s));
+        if (confidence) EE_CK(cudaMemcpyAsync(confidence, d_conf, 4 * (size_t)n, cudaMemcpyDeviceToHost, s));
+        EE_TRY(fetch_ctl(c));
+        EE_TRY(device_error(c));
+        if (c->h_ctl->pos != c->pos) return fail(EE_EDEVICE, "device position out of step with the host");
+    }
+    return EE_OK;
+}
+
+int ee_sync(ee_ctx* c) {
+    if (!c) return fail(EE_EINVAL, "NULL context");
+    EE_TRY(fetch_ctl(c));
+    return device_error(c);
+}
+
+int ee_get_stats(ee_ctx* c, ee_stats* out) {
+    if (!c || !out) return fail(EE_EINVAL, "NULL argument");
+    EE_TRY(fetch_ctl(c));
+    std::memset(out, 0, sizeof(*out));
+    out->steps = c->h_ctl->steps;
+    out->full_steps = c->h_ctl->full_steps;
+    for (int r = 0; r < kMaxReadouts; ++r) out->exits[r] = c->h_ctl->exits[r];
+    return EE_OK;
+}
+
+int ee_position(ee_ctx* c, int32_t* pos) {
+    if (!c || !pos) return fail(EE_EINVAL, "NULL argument");
+    *pos = c->pos;
+    return EE_OK;
+}
+
+int ee_debug_read(ee_ctx* c, int what, int layer, int pos, void* host_dst, size_t bytes) {
+    if (!c || !host_dst) return fail(EE_EINVAL, "NULL argument");
+    const ee_model_config& cf = c->cfg;
+    const size_t d = cf.d_model, V = cf.vocab, kd = (size_t)cf.n_kv_heads * cf.head_dim;
+    const Layout& l = c->lay;
+    EE_CK(cudaStreamSynchronize(c->stream));
+    auto rd = [&](size_t off, size_t n) -> int {
+        if (bytes != n) return fail(EE_EINVAL, "byte count does not match the requested item");
+        EE_CK(cudaMemcpy(host_dst, c->ws + off, n, cudaMemcpyDeviceToHost));
+        return EE_OK;
+    };
+    switch (what) {
+        case EE_DBG_HIDDEN_READOUT:
+            if (layer < 0 || layer >= c->n_readouts) return fail(EE_EINVAL, "bad readout index");
+            return rd(l.hk + 4 * d * layer, 4 * d);
+        case EE_DBG_READOUT_Y:
+            if (layer < 0 || layer >= c->n_readouts) return fail(EE_EINVAL, "bad readout index");
+            return rd(l.y + 4 * d * layer, 4 * d);
+        case EE_DBG_HIDDEN_FINAL:
+            return rd(l.h, 4 * d);
+        case EE_DBG_READOUT_LOGITS:
+            if (layer < 0 || layer >= c->n_readouts) return fail(EE_EINVAL, "bad readout index");
+            return rd(l.logits_ro + 4 * V * layer, 4 * V);
+        case EE_DBG_FINAL_LOGITS:
+            return rd(l.logits_final, 4 * V);
+        case EE_DBG_KV:
+        case EE_DBG_KV_SRC: {
+            if (layer < 0 || layer >= cf.n_layers || pos < 0 || pos >= cf.max_ctx)
+                return fail(EE_EINVAL, "bad layer or position");
+            if (what == EE_DBG_KV_SRC) return rd(l.kv_src + (size_t)layer * cf.max_ctx + pos, 1);
+            if (bytes != 2 * 2 * kd) return fail(EE_EINVAL, "byte count does not match the requested item");
+            int32_t page;
+            EE_CK(cudaMemcpy(&page, c->ws + l.page_table + 4 * (size_t)(pos / cf.page_size), 4, cudaMemcpyDeviceToHost));
+            const int slot = pos % cf.page_size;
+            uint16_t* dst = (uint16_t*)host_dst;
+            for (int g = 0; g < cf.n_kv_heads; ++g) {
+                const size_t off = 2 * ((size_t)layer * l.kv_layer_stride +
+                                        (((size_t)page * cf.n_kv_heads + g) * cf.page_size + slot) * cf.head_dim);
+                EE_CK(cudaMemcpy(dst + g * cf.head_dim, c->ws + l.kpool + off, 2 * (size_t)cf.head_dim,
+                                 cudaMemcpyDeviceToHost));
+                EE_CK(cudaMemcpy(dst + kd + g * cf.head_dim, c->ws + l.vpool + off, 2 * (size_t)cf.head_dim,
+                                 cudaMemcpyDeviceToHost));
+            }
+            return EE_OK;
+        }
+        default:
+            return fail(EE_EINVAL, "unknown debug item");
+    }
+}
+
+// ---------------------------------------------------------------- standalone ops
+
+int ee_attention_scratch_bytes(int n_heads, int n_kv_heads, int head_dim, size_t* bytes) {
+    if (!bytes || n_heads <= 0 || n_kv_heads <= 0 || (head_dim != 64 && head_dim != 128)) return fail(EE_EINVAL, "bad shape");
+    *bytes = align_up(4 * (size_t)n_heads * kAttnMaxSplits * (head_dim + 2)) + align_up(4 * (size_t)n_kv_heads);
+    return EE_OK;
+}
+
+int ee_attention_decode(const float* q, const uint16_t* k_pages, const uint16_t* v_pages, const int32_t* page_table,
+                        int T, int n_heads, int n_kv_heads, int head_dim, int page_size, void* scratch,
+                        size_t scratch_bytes, float* out, void* stream) {
+    size_t need = 0;
+    EE_TRY(ee_attention_scratch_bytes(n_heads, n_kv_heads, head_dim, &need));
+    if (!q || !k_pages || !v_pages || !page_table || !scratch || !out) return fail(EE_EINVAL, "NULL argument");
+    if (T <= 0) return fail(EE_EINVAL, "T must be positive");
+    if (n_heads % n_kv_heads || n_heads / n_kv_heads > 8) return fail(EE_EINVAL, "bad head grouping");
+    if (page_size <= 0) return fail(EE_EINVAL, "bad page size");
+    if (scratch_bytes < need) return fail(EE_ENOMEM, "scratch too small");
+    cudaStream_t s = (cudaStream_t)stream;
+    char* sc = (char*)scratch;
+    AttnArgs a{};
+    a.q = q;
+    a.kp = k_pages;
+    a.vp = v_pages;
+    a.page_table = page_table;
+    a.ctl = nullptr;
+    a.T = T;
+    a.A = n_heads;
+    a.KH = n_kv_heads;
+    a.page_size = page_size;
+    a.out = out;
+    a.part = (float*)sc;
+    a.ticket = (int*)(sc + align_up(4 * (size_t)n_heads * kAttnMaxSplits * (head_dim + 2)));
+    EE_CK(cudaMemsetAsync(a.ticket, 0, 4 * (size_t)n_kv_heads, s));
+    EE_CK(launch_attention(a, head_dim, false, s));
+    return EE_OK;
+}
+
+int ee_vocab_scratch_bytes(int vocab, int d_model, size_t* bytes) {
+    if (!bytes || vocab <= 1 || d_model < 256 || d_model % 8) return fail(EE_EINVAL, "bad shape");
+    *bytes = align_up(4 * (size_t)kMaxVocabCtas * 4) + align_up(4);
+    return EE_OK;
+}
+
+int ee_vocab_confidence(const float* x, const uint16_t* gain, const uint16_t* U, int vocab, int d_model, float eps,
+                        void* scratch, size_t scratch_bytes, int32_t* out_token, float* out_p, float* logits,
+                        void* stream) {
+    size_t need = 0;
+    EE_TRY(ee_vocab_scratch_bytes(vocab, d_model, &need));
+    if (!x || !gain || !U || !scratch || !out_token || !out_p) return fail(EE_EINVAL, "NULL argument");
+    if (scratch_bytes < need) return fail(EE_ENOMEM, "scratch too small");
+    int dev = 0, nsm = 0;
+    EE_CK(cudaGetDevice(&dev));
+    EE_CK(cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev));
+    if (configure_kernels(d_model) != cudaSuccess) return fail(EE_ECUDA, "kernel configuration failed");
+    cudaStream_t s = (cudaStream_t)stream;
+    char* sc = (char*)scratch;
+    VocabArgs v{};
+    v.x = x;
+    v.gain = gain;
+    v.U = U;
+    v.V = vocab;
+    v.d = d_model;
+    v.eps = eps;
+    v.logits = logits;
+    v.logits_if_dbg = 0;
+    v.part = (float*)sc;
+    v.ticket = (int*)(sc + align_up(4 * (size_t)kMaxVocabCtas * 4));
+    v.mode = 0;
+    v.out_token = out_token;
+    v.out_p = out_p;
+    EE_CK(cudaMemsetAsync(v.ticket, 0, 4, s));
+    EE_CK(launch_vocab(v, std::min(nsm, kMaxVocabCtas), false, s));
+    return EE_OK;
+}
+
+}  // extern "C"

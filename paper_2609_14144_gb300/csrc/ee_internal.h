@@ -1,0 +1,160 @@
+// Internal structures shared by the sm_103a kernels (ee_kernels.cu) and the
+// host engine (ee_engine.cu).  Not part of the public ABI.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "ee.h"
+
+namespace ee {
+
+constexpr int kMaxReadouts = EE_MAX_READOUTS;
+constexpr int kGemvThreads = 512;   // 16 warps per CTA in the streaming GEMVs
+constexpr int kAttnThreads = 256;   // 8 warps per CTA in split-K attention
+constexpr int kAttnMinRows = 32;    // positions per attention split (at least)
+constexpr int kAttnMaxSplits = 128; // splits per key-value head (at most)
+
+// Bits of the device error word.
+constexpr int kErrNanConfidence = 1;
+constexpr int kErrTokenRange = 2;
+constexpr int kErrPosition = 4;
+
+// Device-resident control block: everything a step reads or writes that is
+// not a tensor, so one captured graph serves every step, tau and force.
+struct Ctl {
+    int32_t pos;          // position of the step's input token
+    int32_t in_tok;       // input token of the next step
+    int32_t force;        // EE_FREE / EE_FORCE_FULL / EE_FORCE_EXIT_AT(r)
+    int32_t step;         // step index inside one ee_decode_n call
+    int32_t n_steps;      // steps requested by ee_decode_n
+    int32_t err;          // device error word (kErr* bits)
+    int32_t dbg;          // 1: keep readout / final logits
+    int32_t exit_readout; // readout that emitted this step, -1 = full depth
+    int32_t token;        // emitted token of the last step
+    int32_t full_token;   // LM head token of the last full step, else -1
+    int32_t n_evaluated;  // readouts evaluated this step
+    int32_t prefill_n;    // prompt length of the running prefill
+    int32_t prefill_i;    // prompt index of the running prefill
+    int32_t max_ctx;
+    int32_t pad0, pad1;
+    int32_t gate_pass[kMaxReadouts];
+    int32_t readout_token[kMaxReadouts];
+    float conf[kMaxReadouts];
+    float tau[kMaxReadouts];
+    float full_conf;
+    float pad2[3];
+    long long steps, full_steps, exits[kMaxReadouts];
+    int32_t* out_tokens;   // per-step outputs of ee_decode_n (may be null)
+    int32_t* out_exit;
+    float* out_conf;
+    const int8_t* sched;   // per-step force values (may be null)
+    const int32_t* prompt; // prompt ids of the running prefill
+};
+
+// Device pointers and shape, passed by value to every kernel.
+struct DevModel {
+    int L, d, A, KH, D, F, V, max_ctx, page_size, n_pages, qkv_bias, n_readouts;
+    float eps;
+    // Packed per-layer weights: layer j starts at layers + j * layer_stride.
+    const uint16_t* layers;
+    int64_t layer_stride;
+    int64_t off_wqkv, off_bqkv, off_gattn, off_wo, off_gmlp, off_wgu, off_wd;
+    const uint16_t* embed;
+    const uint16_t* lm_head;
+    const uint16_t* g_final;
+    const uint16_t* ro_w[kMaxReadouts];
+    const uint16_t* ro_b[kMaxReadouts];
+    int ro_layer[kMaxReadouts];
+    const float2* rope;           // [max_ctx][D/2] (cos, sin)
+    uint16_t* kpool;              // [L][n_pages][KH][page_size][D]
+    uint16_t* vpool;
+    int64_t kv_layer_stride;      // elements per layer in a pool
+    const int32_t* page_table;    // [n_pages]
+    int8_t* kv_src;               // [L][max_ctx]
+    float* h;                     // residual stream [d]
+    float* q;                     // rotated queries [A*D]
+    float* o;                     // attention output [A*D]
+    float* a;                     // SwiGLU product [F]
+    float* y;                     // readout outputs [R][d]
+    float* hk;                    // residual seen by each readout [R][d]
+    float* logits_ro;             // [R][V] (debug)
+    float* logits_final;          // [V] (debug)
+    float* gemv_part;             // cross-warp partial sums
+    int* gemv_ticket;             // per-unit arrival counters
+    int64_t gemv_part_stride;     // floats per fill layer in gemv_part
+    int64_t gemv_ticket_stride;   // ints per fill layer in gemv_ticket
+    float* attn_part;             // [A][kAttnMaxSplits][D + 2]
+    int* attn_ticket;             // [KH]
+    float* vocab_part;            // [grid][4]
+    int* vocab_ticket;            // [1]
+    Ctl* ctl;
+};
+
+// Arguments of the split-K attention kernel (engine and standalone op).
+struct AttnArgs {
+    const float* q;
+    const uint16_t* kp;       // pool of this layer: [n_pages][KH][page_size][D]
+    const uint16_t* vp;
+    const int32_t* page_table;
+    const Ctl* ctl;           // if set, T = ctl->pos + 1
+    int T;
+    int A, KH, page_size;
+    float* out;
+    float* part;
+    int* ticket;
+};
+
+// Arguments of the vocabulary pass (readout / LM head / standalone).
+struct VocabArgs {
+    const float* x;           // residual-space input [d]
+    const uint16_t* gain;     // final RMSNorm gain [d]
+    const uint16_t* U;        // [V, d]
+    int V, d;
+    float eps;
+    float* logits;            // optional [V]
+    int logits_if_dbg;        // write logits only when ctl->dbg is set
+    float* part;
+    int* ticket;
+    int mode;                 // 0 standalone, 1 readout r, 2 LM head
+    int r;
+    Ctl* ctl;
+    int32_t* out_token;
+    float* out_p;
+    int has_cond;
+    cudaGraphConditionalHandle cond;
+};
+
+// Per-call inputs of a graph launch.
+struct CtlInputs {
+    int set_token, in_tok, force, n_steps, dbg, prefill_n;
+    float tau[kMaxReadouts];
+    const int8_t* sched;
+    int32_t* out_tokens;
+    int32_t* out_exit;
+    float* out_conf;
+    const int32_t* prompt;
+};
+
+// Launch helpers (ee_kernels.cu).  Each enqueues one kernel on `s`;
+// `pdl` adds the programmatic-stream-serialisation attribute.
+cudaError_t launch_qkv(const DevModel& m, int layer, int first, int grid, bool pdl, cudaStream_t s);
+cudaError_t launch_attention(const AttnArgs& a, int head_dim, bool pdl, cudaStream_t s);
+cudaError_t launch_oproj(const DevModel& m, int layer, int grid, bool pdl, cudaStream_t s);
+cudaError_t launch_gateup(const DevModel& m, int layer, int grid, bool pdl, cudaStream_t s);
+cudaError_t launch_down(const DevModel& m, int layer, int grid, bool pdl, cudaStream_t s);
+cudaError_t launch_readout(const DevModel& m, int r, int grid, bool pdl, cudaStream_t s);
+cudaError_t launch_vocab(const VocabArgs& v, int grid, bool pdl, cudaStream_t s);
+cudaError_t launch_kvfill(const DevModel& m, int exit_layer, int grid_x, bool pdl, cudaStream_t s);
+cudaError_t launch_step_end(const DevModel& m, int has_cond, cudaGraphConditionalHandle cond, bool pdl,
+                            cudaStream_t s);
+cudaError_t launch_prefill_advance(const DevModel& m, int has_cond, cudaGraphConditionalHandle cond, bool pdl,
+                                   cudaStream_t s);
+cudaError_t launch_prefill_end(const DevModel& m, bool pdl, cudaStream_t s);
+cudaError_t launch_set_inputs(Ctl* c, const CtlInputs& in, cudaStream_t s);
+
+// Dynamic shared memory each GEMV kernel asks for, given the largest K.
+size_t gemv_smem_bytes(int kmax);
+cudaError_t configure_kernels(int kmax);
+
+}  // namespace ee

@@ -1,0 +1,911 @@
+// sm_103a kernels of the confidence-gated early-exit decode step.
+//
+// Batch-1 decode is a chain of M = 1 matrix-vector products: about one flop
+// per weight byte, so every kernel here is bound by HBM bandwidth, not by the
+// tensor cores.  The design goals are therefore (1) every weight byte read
+// once, with 16-byte coalesced loads and enough of them in flight,
+// (2) perfect balance across the 152 SMs, and (3) no launch-gap bubbles
+// (programmatic dependent launch: each kernel prefetches its weights into L2
+// before it waits for its predecessor's activations).
+//
+// The streaming GEMV core ("flat GEMV"): a weight matrix of n_units units,
+// each NR rows of K bf16 values stored contiguously, is viewed as one array
+// of 16-byte chunks.  Every warp owns an equal contiguous slice of that array
+// (or, in the row-aligned variant, an equal run of whole units).  Lanes read
+// consecutive chunks (512 bytes per warp instruction), multiply by the
+// activation vector held in shared memory as fp32, and keep one running sum
+// per lane; a warp reduction closes each row.  Units cut by a slice boundary
+// are finished by whichever contributing warp arrives last, summing the
+// contributions in warp order, so results do not depend on timing.
+#include <cuda_bf16.h>
+#include <math_constants.h>
+
+#include "ee_internal.h"
+
+namespace ee {
+
+// ------------------------------------------------------------------ helpers
+
+__device__ __forceinline__ float bf_lo(uint32_t u) { return __uint_as_float(u << 16); }
+__device__ __forceinline__ float bf_hi(uint32_t u) { return __uint_as_float(u & 0xffff0000u); }
+__device__ __forceinline__ float bf2f(uint16_t b) { return __uint_as_float((uint32_t)b << 16); }
+__device__ __forceinline__ uint16_t f2bf(float f) { return __bfloat16_as_ushort(__float2bfloat16_rn(f)); }
+
+// Streaming 16-byte load of read-only weights: no L1 allocation, 256-byte
+// L2 sector promotion.
+__device__ __forceinline__ uint4 ldg_stream(const uint4* p) {
+    uint4 r;
+    asm("ld.global.nc.L1::no_allocate.L2::256B.v4.u32 {%0,%1,%2,%3}, [%4];"
+        : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+        : "l"(p));
+    return r;
+}
+
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+__device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+// Sum over the block; every thread gets the same value (fixed order).
+__device__ __forceinline__ float block_sum(float v, float* red) {
+    v = warp_sum(v);
+    const int w = threadIdx.x >> 5, l = threadIdx.x & 31, nw = blockDim.x >> 5;
+    __syncthreads();
+    if (l == 0) red[w] = v;
+    __syncthreads();
+    float t = (l < nw) ? red[l] : 0.f;
+    return warp_sum(t);
+}
+
+// x = src / sqrt(mean(src^2) + eps) * g, fp32 statistics, into smem.
+__device__ __forceinline__ void rmsnorm_to_smem(const float* src, const uint16_t* g, int d, float eps, float* x,
+                                                float* red) {
+    float ss = 0.f;
+    for (int i = threadIdx.x; i < d; i += blockDim.x) {
+        const float v = src[i];
+        ss = fmaf(v, v, ss);
+    }
+    ss = block_sum(ss, red);
+    const float inv = 1.0f / sqrtf(ss / (float)d + eps);
+    for (int i = threadIdx.x; i < d; i += blockDim.x) x[i] = src[i] * inv * bf2f(g[i]);
+    __syncthreads();
+}
+
+// Dot product of 8 packed bf16 weights with 8 fp32 activations.
+__device__ __forceinline__ float dot8(const uint4 w, const float* x) {
+    const float4 a = *reinterpret_cast<const float4*>(x);
+    const float4 b = *reinterpret_cast<const float4*>(x + 4);
+    float s = bf_lo(w.x) * a.x;
+    s = fmaf(bf_hi(w.x), a.y, s);
+    s = fmaf(bf_lo(w.y), a.z, s);
+    s = fmaf(bf_hi(w.y), a.w, s);
+    s = fmaf(bf_lo(w.z), b.x, s);
+    s = fmaf(bf_hi(w.z), b.y, s);
+    s = fmaf(bf_lo(w.w), b.z, s);
+    s = fmaf(bf_hi(w.w), b.w, s);
+    return s;
+}
+
+// Chunk range [c0, c1) of `warp` out of `nwarps` over n_units units of Cu chunks.
+template <bool ALIGNED>
+__device__ __forceinline__ void warp_range(int64_t n_units, int64_t Cu, int warp, int nwarps, int64_t& c0,
+                                           int64_t& c1) {
+    if (ALIGNED) {
+        c0 = (n_units * warp / nwarps) * Cu;
+        c1 = (n_units * (warp + 1) / nwarps) * Cu;
+    } else {
+        const int64_t Ct = n_units * Cu;
+        c0 = Ct * warp / nwarps;
+        c1 = Ct * (warp + 1) / nwarps;
+    }
+}
+
+// Before waiting on the predecessor kernel: pull the head of this warp's
+// weight slice into L2 so the stream starts at full rate.
+constexpr uint32_t kPrefetchCap = 16384;
+
+template <int NR, bool ALIGNED>
+__device__ __forceinline__ void prefetch_slice(const uint16_t* W, int K, int64_t n_units, int warp, int nwarps) {
+    if ((threadIdx.x & 31) != 0) return;
+    int64_t c0, c1;
+    warp_range<ALIGNED>(n_units, (int64_t)NR * (K >> 3), warp, nwarps, c0, c1);
+    if (c1 <= c0) return;
+    const int64_t bytes = (c1 - c0) * 16;
+    prefetch_l2(W + c0 * 8, (uint32_t)(bytes < kPrefetchCap ? bytes : kPrefetchCap));
+}
+
+// The flat GEMV core (see the file comment).  Epi is called by lane 0 with
+// the unit index and its NR row sums.  Requires K % 8 == 0 and K >= 256.
+template <int NR, bool ALIGNED, int U, class Epi>
+__device__ __forceinline__ void flat_gemv(const uint16_t* __restrict__ W, int K, int64_t n_units,
+                                          const float* __restrict__ xs, int warp, int nwarps,
+                                          float* __restrict__ part, int* __restrict__ ticket, Epi& epi) {
+    const int lane = threadIdx.x & 31;
+    const int Rc = K >> 3;
+    const int64_t Cu = (int64_t)NR * Rc;
+    const int64_t Ct = n_units * Cu;
+    int64_t c0, c1;
+    warp_range<ALIGNED>(n_units, Cu, warp, nwarps, c0, c1);
+    if (c0 >= c1) return;
+    const uint4* Wc = reinterpret_cast<const uint4*>(W);
+
+    int64_t row = c0 / Rc;
+    int o0 = (int)(c0 - row * Rc);  // offset of lane 0's chunk inside `row`, in [0, Rc)
+    int col = o0 + lane;            // offset of this lane's chunk inside its row
+    if (col >= Rc) col -= Rc;
+    float acc = 0.f;
+    float rs[NR];
+#pragma unroll
+    for (int r = 0; r < NR; ++r) rs[r] = 0.f;
+
+    auto owner = [&](int64_t c) -> int64_t { return ((c + 1) * (int64_t)nwarps - 1) / Ct; };
+
+    auto finish_row = [&](int64_t rw, float s) {
+        const int64_t unit = rw / NR;
+        const int ri = (int)(rw - unit * NR);
+#pragma unroll
+        for (int r = 0; r < NR; ++r)
+            if (r == ri) rs[r] = s;
+        if (ri == NR - 1 || (rw + 1) * Rc >= c1) {
+            const bool whole = ALIGNED || (unit * Cu >= c0 && (unit + 1) * Cu <= c1);
+            if (lane == 0) {
+                if (whole) {
+                    epi(unit, rs);
+                } else {
+                    const bool first = unit * Cu < c0;
+                    const int64_t slot = (int64_t)warp * 2 + (first ? 0 : 1);
+#pragma unroll
+                    for (int r = 0; r < NR; ++r) part[slot * NR + r] = rs[r];
+                    __threadfence();
+                    const int64_t wa = owner(unit * Cu), wb = owner((unit + 1) * Cu - 1);
+                    const int n = (int)(wb - wa + 1);
+                    const int old = atomicAdd(&ticket[unit], 1);
+                    if (old == n - 1) {
+                        __threadfence();
+                        float sum[NR];
+#pragma unroll
+                        for (int r = 0; r < NR; ++r) sum[r] = __ldcg(&part[(wa * 2 + 1) * NR + r]);
+                        for (int64_t w = wa + 1; w <= wb; ++w)
+#pragma unroll
+                            for (int r = 0; r < NR; ++r) sum[r] += __ldcg(&part[(w * 2) * NR + r]);
+                        epi(unit, sum);
+                        ticket[unit] = 0;
+                    }
+                }
+            }
+#pragma unroll
+            for (int r = 0; r < NR; ++r) rs[r] = 0.f;
+        }
+    };
+
+    for (int64_t g = c0; g < c1; g += 32 * U) {
+        uint4 w[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int64_t c = g + 32 * u + lane;
+            w[u] = (c < c1) ? ldg_stream(Wc + c) : make_uint4(0u, 0u, 0u, 0u);
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            if (g + 32 * u >= c1) break;
+            const float v = dot8(w[u], xs + col * 8);
+            const int b = Rc - o0;  // first lane that belongs to the next row
+            if (b < 32) {
+                acc += (lane < b) ? v : 0.f;
+                finish_row(row, warp_sum(acc));
+                acc = (lane >= b) ? v : 0.f;
+                ++row;
+                o0 += 32 - Rc;
+            } else {
+                acc += v;
+                o0 += 32;
+                if (o0 == Rc) {
+                    finish_row(row, warp_sum(acc));
+                    acc = 0.f;
+                    ++row;
+                    o0 = 0;
+                }
+            }
+            col += 32;
+            if (col >= Rc) col -= Rc;
+        }
+    }
+    if (row * Rc < c1) finish_row(row, warp_sum(acc));
+}
+
+// ------------------------------------------------------------------ epilogues
+
+// Q/K/V unit: the row pair (i, i + D/2) of one head.  Q is rotated and kept
+// in fp32; K is rotated and V copied into the paged cache as bf16.
+struct EpiQKV {
+    float* q;
+    uint16_t* kdst;  // this layer's K page slot base for kv head 0 (stride per head below)
+    uint16_t* vdst;
+    int64_t head_stride;  // elements between kv heads inside a page
+    const uint16_t* bias; // packed [unit][2] or null
+    const float2* cs;     // rope row of this position
+    int64_t unit_offset;
+    int D, nq_units, nk_units;
+    __device__ __forceinline__ void operator()(int64_t unit_local, const float* s) const {
+        const int64_t u = unit_local + unit_offset;
+        float r0 = s[0], r1 = s[1];
+        if (bias) {
+            r0 += bf2f(bias[2 * u]);
+            r1 += bf2f(bias[2 * u + 1]);
+        }
+        const int half = D >> 1;
+        if (u < nq_units) {
+            const int h = (int)(u / half), i = (int)(u - (int64_t)h * half);
+            const float2 c = cs[i];
+            q[h * D + i] = r0 * c.x - r1 * c.y;
+            q[h * D + i + half] = r0 * c.y + r1 * c.x;
+        } else if (u < nq_units + nk_units) {
+            const int64_t uu = u - nq_units;
+            const int g = (int)(uu / half), i = (int)(uu - (int64_t)g * half);
+            const float2 c = cs[i];
+            uint16_t* k = kdst + g * head_stride;
+            k[i] = f2bf(r0 * c.x - r1 * c.y);
+            k[i + half] = f2bf(r0 * c.y + r1 * c.x);
+        } else {
+            const int64_t uu = u - nq_units - nk_units;
+            const int g = (int)(uu / half), i = (int)(uu - (int64_t)g * half);
+            uint16_t* v = vdst + g * head_stride;
+            v[i] = f2bf(r0);
+            v[i + half] = f2bf(r1);
+        }
+    }
+};
+
+struct EpiAddH {
+    float* h;
+    __device__ __forceinline__ void operator()(int64_t u, const float* s) const { h[u] += s[0]; }
+};
+
+struct EpiBias {
+    float* y;
+    const uint16_t* b;
+    __device__ __forceinline__ void operator()(int64_t u, const float* s) const { y[u] = s[0] + bf2f(b[u]); }
+};
+
+struct EpiSwiGLU {
+    float* a;
+    __device__ __forceinline__ void operator()(int64_t u, const float* s) const {
+        const float g = s[0];
+        const float silu = g / (1.0f + expf(-g));
+        a[u] = silu * s[1];
+    }
+};
+
+// Running (max, sum of exp, lowest argmax) over logits, plus optional logits.
+struct EpiVocab {
+    float* logits;
+    float m, s;
+    int a;
+    __device__ __forceinline__ void operator()(int64_t u, const float* r) {
+        const float l = r[0];
+        if (logits) logits[u] = l;
+        if (l > m) {
+            s = s * expf(m - l) + 1.0f;
+            m = l;
+            a = (int)u;
+        } else {
+            s += expf(l - m);
+        }
+    }
+};
+
+// Merge (m2, s2, a2) into (m, s, a): max, rescaled sum, lowest index at the max.
+__device__ __forceinline__ void merge_stats(float& m, float& s, int& a, float m2, float s2, int a2) {
+    if (s2 == 0.f && m2 == -CUDART_INF_F) return;
+    if (s == 0.f && m == -CUDART_INF_F) {
+        m = m2;
+        s = s2;
+        a = a2;
+        return;
+    }
+    if (m2 > m) {
+        s = s * expf(m - m2) + s2;
+        m = m2;
+        a = a2;
+    } else if (m2 == m) {
+        s = s + s2;
+        a = a2 < a ? a2 : a;
+    } else {
+        s = s + s2 * expf(m2 - m);
+    }
+}
+
+// Warp-wide merge; lane 0 ends with the merge of all lanes in lane order.
+__device__ __forceinline__ void warp_merge_stats(float& m, float& s, int& a) {
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const float m2 = __shfl_down_sync(0xffffffffu, m, o);
+        const float s2 = __shfl_down_sync(0xffffffffu, s, o);
+        const int a2 = __shfl_down_sync(0xffffffffu, a, o);
+        if (((threadIdx.x & 31) & ((o << 1) - 1)) == 0) merge_stats(m, s, a, m2, s2, a2);
+    }
+}
+
+__device__ __forceinline__ const uint16_t* layer_base(const DevModel& m, int j) {
+    return m.layers + (int64_t)j * m.layer_stride;
+}
+
+__device__ __forceinline__ int64_t kv_slot_offset(const DevModel& m, int j, int pos) {
+    const int page = m.page_table[pos / m.page_size];
+    const int slot = pos - (pos / m.page_size) * m.page_size;
+    return (int64_t)j * m.kv_layer_stride + ((int64_t)page * m.KH * m.page_size + slot) * m.D;
+}
+
+__device__ __forceinline__ void global_warp(int& warp, int& nwarps) {
+    const int wpb = blockDim.x >> 5;
+    warp = blockIdx.x * wpb + (threadIdx.x >> 5);
+    nwarps = gridDim.x * wpb;
+}
+
+constexpr int kUnroll = 8;
+
+// ------------------------------------------------------------------ kernels
+
+// Attention input of layer j: [embedding gather,] RMSNorm, Q/K/V GEMV, RoPE,
+// KV append at the step's position.
+__global__ void __launch_bounds__(kGemvThreads) k_qkv(DevModel m, int layer, int first) {
+    extern __shared__ float4 smem_f4[];
+    float* xs = reinterpret_cast<float*>(smem_f4);
+    __shared__ float red[32];
+    const uint16_t* lw = layer_base(m, layer);
+    const uint16_t* W = lw + m.off_wqkv;
+    const int64_t nq = (int64_t)m.A * m.D / 2, nk = (int64_t)m.KH * m.D / 2;
+    const int64_t n_units = nq + 2 * nk;
+    int warp, nwarps;
+    global_warp(warp, nwarps);
+    prefetch_slice<2, false>(W, m.d, n_units, warp, nwarps);
+    pdl_wait();
+    pdl_launch_dependents();
+    Ctl* c = m.ctl;
+    int pos = c->pos;
+    const bool pos_ok = pos >= 0 && pos < m.max_ctx;
+    if (!pos_ok) pos = 0;
+    const float* src = m.h;
+    if (first) {
+        int tok = c->in_tok;
+        const bool tok_ok = tok >= 0 && tok < m.V;
+        if (!tok_ok) tok = 0;
+        float* hl = xs + m.d;
+        const uint16_t* e = m.embed + (int64_t)tok * m.d;
+        for (int i = threadIdx.x; i < m.d; i += blockDim.x) {
+            const float v = bf2f(e[i]);
+            hl[i] = v;
+            if (blockIdx.x == 0) m.h[i] = v;
+        }
+        if (blockIdx.x == 0 && threadIdx.x == 0) {
+            c->exit_readout = -1;
+            c->n_evaluated = 0;
+            c->full_token = -1;
+            if (!tok_ok) atomicOr(&c->err, kErrTokenRange);
+        }
+        __syncthreads();
+        src = hl;
+    }
+    if (!pos_ok) {
+        if (blockIdx.x == 0 && threadIdx.x == 0) atomicOr(&c->err, kErrPosition);
+        return;
+    }
+    rmsnorm_to_smem(src, lw + m.off_gattn, m.d, m.eps, xs, red);
+    const int64_t kvo = kv_slot_offset(m, layer, pos);
+    EpiQKV epi{m.q,
+               m.kpool + kvo,
+               m.vpool + kvo,
+               (int64_t)m.page_size * m.D,
+               m.qkv_bias ? lw + m.off_bqkv : nullptr,
+               m.rope + (int64_t)pos * (m.D / 2),
+               0,
+               m.D,
+               (int)nq,
+               (int)nk};
+    flat_gemv<2, false, kUnroll>(W, m.d, n_units, xs, warp, nwarps, m.gemv_part, m.gemv_ticket, epi);
+    if (blockIdx.x == 0 && threadIdx.x == 0) m.kv_src[(int64_t)layer * m.max_ctx + pos] = 1;
+}
+
+// KV repair for the skipped layers exit_layer .. L-1 (0-based) at the step's
+// position: K = RoPE(W_K RMSNorm_j(h_k)), V = W_V RMSNorm_j(h_k), stored bf16.
+__global__ void __launch_bounds__(kGemvThreads) k_kvfill(DevModel m, int exit_layer) {
+    extern __shared__ float4 smem_f4[];
+    float* xs = reinterpret_cast<float*>(smem_f4);
+    __shared__ float red[32];
+    const int j = exit_layer + blockIdx.y;
+    const uint16_t* lw = layer_base(m, j);
+    const int64_t nq = (int64_t)m.A * m.D / 2, nk = (int64_t)m.KH * m.D / 2;
+    const uint16_t* W = lw + m.off_wqkv + nq * 2 * m.d;
+    const int64_t n_units = 2 * nk;
+    int warp, nwarps;
+    global_warp(warp, nwarps);
+    prefetch_slice<2, false>(W, m.d, n_units, warp, nwarps);
+    pdl_wait();
+    pdl_launch_dependents();
+    const int pos = m.ctl->pos;
+    if (pos < 0 || pos >= m.max_ctx) return;
+    rmsnorm_to_smem(m.h, lw + m.off_gattn, m.d, m.eps, xs, red);
+    const int64_t kvo = kv_slot_offset(m, j, pos);
+    EpiQKV epi{m.q,
+               m.kpool + kvo,
+               m.vpool + kvo,
+               (int64_t)m.page_size * m.D,
+               m.qkv_bias ? lw + m.off_bqkv : nullptr,
+               m.rope + (int64_t)pos * (m.D / 2),
+               nq,
+               m.D,
+               (int)nq,
+               (int)nk};
+    flat_gemv<2, false, kUnroll>(W, m.d, n_units, xs, warp, nwarps, m.gemv_part + blockIdx.y * m.gemv_part_stride,
+                                 m.gemv_ticket + blockIdx.y * m.gemv_ticket_stride, epi);
+    if (blockIdx.x == 0 && threadIdx.x == 0) m.kv_src[(int64_t)j * m.max_ctx + pos] = 2;
+}
+
+// Output projection with the residual add: h += W_o o.
+__global__ void __launch_bounds__(kGemvThreads) k_oproj(DevModel m, int layer) {
+    extern __shared__ float4 smem_f4[];
+    float* xs = reinterpret_cast<float*>(smem_f4);
+    const uint16_t* W = layer_base(m, layer) + m.off_wo;
+    const int K = m.A * m.D;
+    int warp, nwarps;
+    global_warp(warp, nwarps);
+    prefetch_slice<1, false>(W, K, m.d, warp, nwarps);
+    pdl_wait();
+    pdl_launch_dependents();
+    for (int i = threadIdx.x; i < K; i += blockDim.x) xs[i] = m.o[i];
+    __syncthreads();
+    EpiAddH epi{m.h};
+    flat_gemv<1, false, kUnroll>(W, K, m.d, xs, warp, nwarps, m.gemv_part, m.gemv_ticket, epi);
+}
+
+// Gated feed-forward up: a = SiLU(W_g x) * (W_u x), x = RMSNorm(h) * g_mlp.
+__global__ void __launch_bounds__(kGemvThreads) k_gateup(DevModel m, int layer) {
+    extern __shared__ float4 smem_f4[];
+    float* xs = reinterpret_cast<float*>(smem_f4);
+    __shared__ float red[32];
+    const uint16_t* lw = layer_base(m, layer);
+    const uint16_t* W = lw + m.off_wgu;
+    int warp, nwarps;
+    global_warp(warp, nwarps);
+    prefetch_slice<2, false>(W, m.d, m.F, warp, nwarps);
+    pdl_wait();
+    pdl_launch_dependents();
+    rmsnorm_to_smem(m.h, lw + m.off_gmlp, m.d, m.eps, xs, red);
+    EpiSwiGLU epi{m.a};
+    flat_gemv<2, false, kUnroll>(W, m.d, m.F, xs, warp, nwarps, m.gemv_part, m.gemv_ticket, epi);
+}
+
+// Gated feed-forward down with the residual add: h += W_d a.
+__global__ void __launch_bounds__(kGemvThreads) k_down(DevModel m, int layer) {
+    extern __shared__ float4 smem_f4[];
+    float* xs = reinterpret_cast<float*>(smem_f4);
+    const uint16_t* W = layer_base(m, layer) + m.off_wd;
+    int warp, nwarps;
+    global_warp(warp, nwarps);
+    prefetch_slice<1, false>(W, m.F, m.d, warp, nwarps);
+    pdl_wait();
+    pdl_launch_dependents();
+    for (int i = threadIdx.x; i < m.F; i += blockDim.x) xs[i] = m.a[i];
+    __syncthreads();
+    EpiAddH epi{m.h};
+    flat_gemv<1, false, kUnroll>(W, m.F, m.d, xs, warp, nwarps, m.gemv_part, m.gemv_ticket, epi);
+}
+
+// Readout affine map r: y_r = W_r h + b_r; also keeps h_k for debug.
+__global__ void __launch_bounds__(kGemvThreads) k_readout(DevModel m, int r) {
+    extern __shared__ float4 smem_f4[];
+    float* xs = reinterpret_cast<float*>(smem_f4);
+    const uint16_t* W = m.ro_w[r];
+    int warp, nwarps;
+    global_warp(warp, nwarps);
+    prefetch_slice<1, false>(W, m.d, m.d, warp, nwarps);
+    pdl_wait();
+    pdl_launch_dependents();
+    for (int i = threadIdx.x; i < m.d; i += blockDim.x) {
+        const float v = m.h[i];
+        xs[i] = v;
+        if (blockIdx.x == 0) m.hk[(int64_t)r * m.d + i] = v;
+    }
+    __syncthreads();
+    EpiBias epi{m.y + (int64_t)r * m.d, m.ro_b[r]};
+    flat_gemv<1, false, kUnroll>(W, m.d, m.d, xs, warp, nwarps, m.gemv_part, m.gemv_ticket, epi);
+}
+
+// One pass over the unembedding: z = RMSNorm(x) * gain, l = U z, then
+// max, sum of exp and lowest argmax; the last CTA to finish turns them into
+// the top-1 probability p = 1 / sum exp(l - max) and, for a readout, the gate
+// decision p > tau (which also selects the graph's branch).
+__global__ void __launch_bounds__(kGemvThreads) k_vocab(VocabArgs v) {
+    extern __shared__ float4 smem_f4[];
+    float* xs = reinterpret_cast<float*>(smem_f4);
+    __shared__ float red[32];
+    __shared__ float sm_m[32], sm_s[32];
+    __shared__ int sm_a[32];
+    __shared__ int is_last;
+    int warp, nwarps;
+    global_warp(warp, nwarps);
+    prefetch_slice<1, true>(v.U, v.d, v.V, warp, nwarps);
+    pdl_wait();
+    pdl_launch_dependents();
+    rmsnorm_to_smem(v.x, v.gain, v.d, v.eps, xs, red);
+    const bool keep = v.logits && (!v.logits_if_dbg || (v.ctl && v.ctl->dbg));
+    EpiVocab epi{keep ? v.logits : nullptr, -CUDART_INF_F, 0.f, 0x7fffffff};
+    flat_gemv<1, true, kUnroll>(v.U, v.d, v.V, xs, warp, nwarps, nullptr, nullptr, epi);
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+    if (lane == 0) {
+        sm_m[w] = epi.m;
+        sm_s[w] = epi.s;
+        sm_a[w] = epi.a;
+    }
+    __syncthreads();
+    if (w == 0) {
+        const int nw = blockDim.x >> 5;
+        float m = lane < nw ? sm_m[lane] : -CUDART_INF_F;
+        float s = lane < nw ? sm_s[lane] : 0.f;
+        int a = lane < nw ? sm_a[lane] : 0x7fffffff;
+        warp_merge_stats(m, s, a);
+        if (lane == 0) {
+            v.part[blockIdx.x * 4 + 0] = m;
+            v.part[blockIdx.x * 4 + 1] = s;
+            reinterpret_cast<int*>(v.part)[blockIdx.x * 4 + 2] = a;
+            __threadfence();
+            is_last = atomicAdd(v.ticket, 1) == (int)gridDim.x - 1;
+        }
+    }
+    __syncthreads();
+    if (!is_last || w != 0) return;
+    __threadfence();
+    float m = -CUDART_INF_F, s = 0.f;
+    int a = 0x7fffffff;
+    for (int b = lane; b < (int)gridDim.x; b += 32)
+        merge_stats(m, s, a, __ldcg(&v.part[b * 4 + 0]), __ldcg(&v.part[b * 4 + 1]),
+                    __ldcg(reinterpret_cast<const int*>(v.part) + b * 4 + 2));
+    warp_merge_stats(m, s, a);
+    if (lane != 0) return;
+    *v.ticket = 0;
+    const float p = 1.0f / s;
+    if (v.mode == 0) {
+        *v.out_token = a;
+        *v.out_p = p;
+        return;
+    }
+    Ctl* c = v.ctl;
+    if (!(p == p) || a < 0 || a >= v.V) atomicOr(&c->err, kErrNanConfidence);
+    if (v.mode == 1) {
+        const int r = v.r;
+        const int f = c->sched ? (int)c->sched[c->step] : c->force;
+        const int pass = p > c->tau[r] ? 1 : 0;
+        c->conf[r] = p;
+        c->readout_token[r] = a;
+        c->gate_pass[r] = pass;
+        c->n_evaluated = r + 1;
+        const int take = (f == EE_FREE) ? pass : (f == EE_FORCE_EXIT_AT(r) ? 1 : 0);
+        if (take) {
+            c->exit_readout = r;
+            c->token = a;
+        }
+        if (v.has_cond) cudaGraphSetConditional(v.cond, take);
+    } else {
+        c->token = a;
+        c->full_token = a;
+        c->full_conf = p;
+        c->exit_readout = -1;
+    }
+}
+
+// Split-K decode attention over the paged cache.  Grid (splits, KH): CTA
+// (s, g) covers a contiguous run of positions for the A/K query heads of
+// key-value head g with a per-lane online softmax; the last CTA of head g
+// merges the splits and writes o = softmax(q K^T / sqrt(D)) V (fp32).
+template <int D>
+__global__ void __launch_bounds__(kAttnThreads) k_attention(AttnArgs a) {
+    constexpr int LPR = D / 8;  // lanes per position (8 dims each)
+    constexpr int RPW = 32 / LPR;
+    constexpr int NW = kAttnThreads / 32;
+    constexpr int GMAX = 8;
+    __shared__ __align__(16) float qs[GMAX * D];
+    __shared__ float wm[NW][GMAX], wl[NW][GMAX];
+    __shared__ __align__(16) float wacc[NW][GMAX][D];
+    __shared__ int is_last;
+    pdl_wait();
+    pdl_launch_dependents();
+    const int T = a.ctl ? a.ctl->pos + 1 : a.T;
+    const int G = a.A / a.KH;
+    int S = (T + kAttnMinRows - 1) / kAttnMinRows;
+    if (S > (int)gridDim.x) S = gridDim.x;
+    const int chunk = (T + S - 1) / S;
+    const int s = blockIdx.x, g = blockIdx.y;
+    if (s >= S) return;
+    const int t0 = s * chunk, t1 = min(T, t0 + chunk);
+    const float scale = 1.0f / sqrtf((float)D);
+    for (int i = threadIdx.x; i < G * D; i += blockDim.x) qs[i] = a.q[(int64_t)g * G * D + i] * scale;
+    __syncthreads();
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int grp = lane / LPR, e0 = (lane % LPR) * 8;
+    float mx[GMAX], ls[GMAX], acc[GMAX][8];
+#pragma unroll
+    for (int h = 0; h < GMAX; ++h) {
+        mx[h] = -CUDART_INF_F;
+        ls[h] = 0.f;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) acc[h][e] = 0.f;
+    }
+    const int P = a.page_size;
+    for (int tt = t0 + warp * RPW; tt < t1; tt += NW * RPW) {
+        const int t = tt + grp;
+        const bool valid = t < t1;
+        float kf[8], vf[8];
+        if (valid) {
+            const int page = a.page_table[t / P];
+            const int64_t off = (((int64_t)page * a.KH + g) * P + (t % P)) * D + e0;
+            const uint4 kw = *reinterpret_cast<const uint4*>(a.kp + off);
+            const uint4 vw = *reinterpret_cast<const uint4*>(a.vp + off);
+            kf[0] = bf_lo(kw.x); kf[1] = bf_hi(kw.x); kf[2] = bf_lo(kw.y); kf[3] = bf_hi(kw.y);
+            kf[4] = bf_lo(kw.z); kf[5] = bf_hi(kw.z); kf[6] = bf_lo(kw.w); kf[7] = bf_hi(kw.w);
+            vf[0] = bf_lo(vw.x); vf[1] = bf_hi(vw.x); vf[2] = bf_lo(vw.y); vf[3] = bf_hi(vw.y);
+            vf[4] = bf_lo(vw.z); vf[5] = bf_hi(vw.z); vf[6] = bf_lo(vw.w); vf[7] = bf_hi(vw.w);
+        } else {
+#pragma unroll
+            for (int e = 0; e < 8; ++e) kf[e] = vf[e] = 0.f;
+        }
+#pragma unroll
+        for (int h = 0; h < GMAX; ++h) {
+            if (h >= G) break;
+            float d = 0.f;
+#pragma unroll
+            for (int e = 0; e < 8; ++e) d = fmaf(kf[e], qs[h * D + e0 + e], d);
+#pragma unroll
+            for (int o = LPR / 2; o; o >>= 1) d += __shfl_xor_sync(0xffffffffu, d, o);
+            if (valid) {
+                const float mn = fmaxf(mx[h], d);
+                const float corr = expf(mx[h] - mn);
+                const float p = expf(d - mn);
+                ls[h] = ls[h] * corr + p;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) acc[h][e] = fmaf(p, vf[e], acc[h][e] * corr);
+                mx[h] = mn;
+            }
+        }
+    }
+    // merge the position groups of this warp (lanes with equal e0)
+#pragma unroll
+    for (int o = LPR; o < 32; o <<= 1) {
+#pragma unroll
+        for (int h = 0; h < GMAX; ++h) {
+            if (h >= G) break;
+            const float m2 = __shfl_xor_sync(0xffffffffu, mx[h], o);
+            const float l2 = __shfl_xor_sync(0xffffffffu, ls[h], o);
+            float a2[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) a2[e] = __shfl_xor_sync(0xffffffffu, acc[h][e], o);
+            const float M = fmaxf(mx[h], m2);
+            if (M != -CUDART_INF_F) {
+                const float c1 = expf(mx[h] - M), c2 = expf(m2 - M);
+                ls[h] = ls[h] * c1 + l2 * c2;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) acc[h][e] = acc[h][e] * c1 + a2[e] * c2;
+                mx[h] = M;
+            }
+        }
+    }
+    if (grp == 0) {
+#pragma unroll
+        for (int h = 0; h < GMAX; ++h) {
+            if (h >= G) break;
+            if (lane == 0) {
+                wm[warp][h] = mx[h];
+                wl[warp][h] = ls[h];
+            }
+#pragma unroll
+            for (int e = 0; e < 8; ++e) wacc[warp][h][e0 + e] = acc[h][e];
+        }
+    }
+    __syncthreads();
+    // merge warps; write this split's partial (acc[D], m, l) per query head
+    const int S_stride = kAttnMaxSplits;
+    for (int i = threadIdx.x; i < G * D; i += blockDim.x) {
+        const int h = i / D, e = i - h * D;
+        float M = -CUDART_INF_F, L = 0.f, O = 0.f;
+        for (int w = 0; w < NW; ++w) {
+            const float m2 = wm[w][h];
+            const float Mn = fmaxf(M, m2);
+            if (Mn == -CUDART_INF_F) continue;
+            const float c1 = expf(M - Mn), c2 = expf(m2 - Mn);
+            L = L * c1 + wl[w][h] * c2;
+            O = O * c1 + wacc[w][h][e] * c2;
+            M = Mn;
+        }
+        float* pp = a.part + ((int64_t)(g * G + h) * S_stride + s) * (D + 2);
+        pp[e] = O;
+        if (e == 0) {
+            pp[D] = M;
+            pp[D + 1] = L;
+        }
+    }
+    __threadfence();
+    __syncthreads();
+    if (threadIdx.x == 0) is_last = atomicAdd(&a.ticket[g], 1) == S - 1;
+    __syncthreads();
+    if (!is_last) return;
+    __threadfence();
+    for (int i = threadIdx.x; i < G * D; i += blockDim.x) {
+        const int h = i / D, e = i - h * D;
+        const float* base = a.part + (int64_t)(g * G + h) * S_stride * (D + 2);
+        float M = -CUDART_INF_F;
+        for (int sp = 0; sp < S; ++sp) M = fmaxf(M, __ldcg(&base[sp * (D + 2) + D]));
+        float L = 0.f, O = 0.f;
+        for (int sp = 0; sp < S; ++sp) {
+            const float ms = __ldcg(&base[sp * (D + 2) + D]);
+            if (ms == -CUDART_INF_F) continue;
+            const float c = expf(ms - M);
+            L = fmaf(__ldcg(&base[sp * (D + 2) + D + 1]), c, L);
+            O = fmaf(__ldcg(&base[sp * (D + 2) + e]), c, O);
+        }
+        a.out[(int64_t)(g * G + h) * D + e] = O / L;
+    }
+    if (threadIdx.x == 0) a.ticket[g] = 0;
+}
+
+// End of a decode step: emit, record, count, advance, feed the token back.
+__global__ void k_step_end(DevModel m, int has_cond, cudaGraphConditionalHandle cond) {
+    pdl_wait();
+    pdl_launch_dependents();
+    if (threadIdx.x != 0) return;
+    Ctl* c = m.ctl;
+    const int tok = c->token;
+    const int r = c->exit_readout;
+    const int st = c->step;
+    float conf = 0.f;
+    if (r >= 0)
+        conf = c->conf[r];
+    else if (c->n_evaluated > 0)
+        conf = c->conf[c->n_evaluated - 1];
+    if (c->out_tokens) c->out_tokens[st] = tok;
+    if (c->out_exit) c->out_exit[st] = r;
+    if (c->out_conf) c->out_conf[st] = conf;
+    c->steps += 1;
+    if (r >= 0)
+        c->exits[r] += 1;
+    else
+        c->full_steps += 1;
+    c->pos += 1;
+    c->in_tok = tok;
+    c->step = st + 1;
+    if (has_cond) cudaGraphSetConditional(cond, (c->step < c->n_steps && c->err == 0) ? 1u : 0u);
+}
+
+// Prefill bookkeeping between prompt positions.
+__global__ void k_prefill_advance(DevModel m, int has_cond, cudaGraphConditionalHandle cond) {
+    pdl_wait();
+    pdl_launch_dependents();
+    if (threadIdx.x != 0) return;
+    Ctl* c = m.ctl;
+    c->pos += 1;
+    c->prefill_i += 1;
+    const int more = c->prefill_i < c->prefill_n;
+    if (more) c->in_tok = c->prompt[c->prefill_i];
+    if (has_cond) cudaGraphSetConditional(cond, (more && c->err == 0) ? 1u : 0u);
+}
+
+// After the prefill's LM head: the full model's token becomes the next input.
+__global__ void k_prefill_end(DevModel m) {
+    pdl_wait();
+    pdl_launch_dependents();
+    if (threadIdx.x != 0) return;
+    Ctl* c = m.ctl;
+    c->in_tok = c->token;
+    c->exit_readout = -1;
+    c->n_evaluated = 0;
+}
+
+// Per-call inputs written into the control block ahead of a graph launch.
+__global__ void k_set_inputs(Ctl* c, CtlInputs in) {
+    if (threadIdx.x != 0) return;
+    if (in.set_token) c->in_tok = in.in_tok;
+    c->force = in.force;
+    c->step = 0;
+    c->n_steps = in.n_steps;
+    c->dbg = in.dbg;
+    for (int r = 0; r < kMaxReadouts; ++r) c->tau[r] = in.tau[r];
+    c->sched = in.sched;
+    c->out_tokens = in.out_tokens;
+    c->out_exit = in.out_exit;
+    c->out_conf = in.out_conf;
+    if (in.prefill_n > 0) {
+        c->prefill_n = in.prefill_n;
+        c->prefill_i = 0;
+        c->prompt = in.prompt;
+    }
+}
+
+// ------------------------------------------------------------------ launchers
+
+template <typename... KArgs, typename... Args>
+static cudaError_t launch_k(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, bool pdl, cudaStream_t s,
+                            Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, kern, args...);
+}
+
+static size_t g_smem = 0;
+
+size_t gemv_smem_bytes(int kmax) { return (size_t)kmax * sizeof(float); }
+
+cudaError_t configure_kernels(int kmax) {
+    if (gemv_smem_bytes(kmax) > g_smem) g_smem = gemv_smem_bytes(kmax);
+    const int bytes = (int)g_smem;
+    cudaError_t e;
+    if ((e = cudaFuncSetAttribute(k_qkv, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes))) return e;
+    if ((e = cudaFuncSetAttribute(k_kvfill, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes))) return e;
+    if ((e = cudaFuncSetAttribute(k_oproj, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes))) return e;
+    if ((e = cudaFuncSetAttribute(k_gateup, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes))) return e;
+    if ((e = cudaFuncSetAttribute(k_down, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes))) return e;
+    if ((e = cudaFuncSetAttribute(k_readout, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes))) return e;
+    if ((e = cudaFuncSetAttribute(k_vocab, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes))) return e;
+    return cudaSuccess;
+}
+
+static size_t smem_for(int k) { return (size_t)k * sizeof(float); }
+
+cudaError_t launch_qkv(const DevModel& m, int layer, int first, int grid, bool pdl, cudaStream_t s) {
+    return launch_k(k_qkv, dim3(grid), dim3(kGemvThreads), smem_for(2 * m.d), pdl, s, m, layer, first);
+}
+cudaError_t launch_kvfill(const DevModel& m, int exit_layer, int grid_x, bool pdl, cudaStream_t s) {
+    return launch_k(k_kvfill, dim3(grid_x, m.L - exit_layer), dim3(kGemvThreads), smem_for(m.d), pdl, s, m,
+                    exit_layer);
+}
+cudaError_t launch_oproj(const DevModel& m, int layer, int grid, bool pdl, cudaStream_t s) {
+    return launch_k(k_oproj, dim3(grid), dim3(kGemvThreads), smem_for(m.A * m.D), pdl, s, m, layer);
+}
+cudaError_t launch_gateup(const DevModel& m, int layer, int grid, bool pdl, cudaStream_t s) {
+    return launch_k(k_gateup, dim3(grid), dim3(kGemvThreads), smem_for(m.d), pdl, s, m, layer);
+}
+cudaError_t launch_down(const DevModel& m, int layer, int grid, bool pdl, cudaStream_t s) {
+    return launch_k(k_down, dim3(grid), dim3(kGemvThreads), smem_for(m.F), pdl, s, m, layer);
+}
+cudaError_t launch_readout(const DevModel& m, int r, int grid, bool pdl, cudaStream_t s) {
+    return launch_k(k_readout, dim3(grid), dim3(kGemvThreads), smem_for(m.d), pdl, s, m, r);
+}
+cudaError_t launch_vocab(const VocabArgs& v, int grid, bool pdl, cudaStream_t s) {
+    return launch_k(k_vocab, dim3(grid), dim3(kGemvThreads), smem_for(v.d), pdl, s, v);
+}
+cudaError_t launch_attention(const AttnArgs& a, int head_dim, bool pdl, cudaStream_t s) {
+    const dim3 grid(kAttnMaxSplits, a.KH);
+    if (head_dim == 64) return launch_k(k_attention<64>, grid, dim3(kAttnThreads), 0, pdl, s, a);
+    if (head_dim == 128) return launch_k(k_attention<128>, grid, dim3(kAttnThreads), 0, pdl, s, a);
+    return cudaErrorInvalidValue;
+}
+cudaError_t launch_step_end(const DevModel& m, int has_cond, cudaGraphConditionalHandle cond, bool pdl,
+                            cudaStream_t s) {
+    return launch_k(k_step_end, dim3(1), dim3(32), 0, pdl, s, m, has_cond, cond);
+}
+cudaError_t launch_prefill_advance(const DevModel& m, int has_cond, cudaGraphConditionalHandle cond, bool pdl,
+                                   cudaStream_t s) {
+    return launch_k(k_prefill_advance, dim3(1), dim3(32), 0, pdl, s, m, has_cond, cond);
+}
+cudaError_t launch_prefill_end(const DevModel& m, bool pdl, cudaStream_t s) {
+    return launch_k(k_prefill_end, dim3(1), dim3(32), 0, pdl, s, m);
+}
+cudaError_t launch_set_inputs(Ctl* c, const CtlInputs& in, cudaStream_t s) {
+    return launch_k(k_set_inputs, dim3(1), dim3(32), 0, false, s, c, in);
+}
+
+}  // namespace ee

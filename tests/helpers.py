@@ -36,3 +36,106 @@ def one_hot_matrix(rows: int, cols: int, i: int, j: int, value: float = 1.0) -> 
 
 def identity_bits(n: int) -> np.ndarray:
     return to_bf16_bits(np.eye(n, dtype=np.float32))
+
+
+# ---------------------------------------------------------------- GPU parity harness
+EXCLUDE_EPS = 1e-3    # exclusion band on |p - tau| and on the top-2 probability gap
+P_TOL = 1e-3          # |p_gpu - p_oracle| on every evaluated readout (the exclusion band)
+REL_TOL = 1e-2        # max|diff| / max|ref| on hidden states, logits and KV vectors
+
+
+def rel_err(a, b) -> float:
+    a = np.asarray(a, np.float64)
+    b = np.asarray(b, np.float64)
+    den = np.max(np.abs(b))
+    return float(np.max(np.abs(a - b)) / den) if den > 0 else float(np.max(np.abs(a)))
+
+
+def is_excluded(o: dict, taus) -> bool:
+    """A step whose decision or token sits within the band where rounding
+    order may flip it: |p - tau| or a top-2 gap below EXCLUDE_EPS."""
+    for r in range(o["n_evaluated"]):
+        if abs(o["confidence"][r] - taus[r]) < EXCLUDE_EPS or o["gap"][r] < EXCLUDE_EPS:
+            return True
+    return (not o["exited"]) and o["full_gap"] < EXCLUDE_EPS
+
+
+def forced(o: dict) -> int:
+    from paper_2609_14144_gb300 import FORCE_EXIT_AT, FORCE_FULL
+    return FORCE_EXIT_AT(o["exit_readout"]) if o["exited"] else FORCE_FULL
+
+
+def teacher_forced(shape, model, n: int, taus, *, prompt=None, capture: bool = True, graphs: bool = True,
+                   pdl: bool = True, page_perm=None, page_size: int = 64):
+    """Run the oracle free and the GPU engine teacher-forced on the oracle's
+    input tokens and exit decisions.  Returns (first_o, first_g, records,
+    oracle, engine)."""
+    import oracle
+    from paper_2609_14144_gb300 import OPT_DEBUG_LOGITS, OPT_GRAPHS, OPT_PDL, Engine
+
+    prompt = synth.prompt(shape) if prompt is None else np.asarray(prompt, np.int32)
+    max_ctx = len(prompt) + n
+    orc = oracle.Oracle(shape, model, max_ctx=max_ctx)
+    eng = Engine(shape, model, max_ctx=max_ctx, page_size=page_size)
+    eng.set_option(OPT_GRAPHS, graphs)
+    eng.set_option(OPT_PDL, pdl)
+    eng.set_option(OPT_DEBUG_LOGITS, capture)
+    if page_perm is not None:
+        eng.set_page_table(page_perm)
+    first_o = orc.prefill(prompt)
+    first_g = eng.prefill(prompt)
+    recs, tok = [], first_o
+    for _ in range(n):
+        o = orc.decode_step(tok, taus, capture=capture)
+        g = eng.decode_step(tok, taus, forced(o))
+        rec = {"o": o, "g": g, "input": tok}
+        if capture:
+            rec["g_h"] = [eng.hidden_at_readout(r) for r in range(o["n_evaluated"])]
+            rec["g_y"] = [eng.readout_output(r) for r in range(o["n_evaluated"])]
+            rec["g_rl"] = [eng.readout_logits(r) for r in range(o["n_evaluated"])]
+            if not o["exited"]:
+                rec["g_hL"] = eng.hidden_final()
+                rec["g_fl"] = eng.final_logits()
+        recs.append(rec)
+        tok = o["token"]
+    return first_o, first_g, recs, orc, eng
+
+
+def check_records(recs, taus, capture: bool = True) -> int:
+    """Assert the parity rules; returns the number of excluded steps."""
+    excluded = 0
+    for i, rec in enumerate(recs):
+        o, g = rec["o"], rec["g"]
+        assert g["exited"] == o["exited"] and g["exit_readout"] == o["exit_readout"], i
+        assert g["n_evaluated"] == o["n_evaluated"], i
+        for r in range(o["n_evaluated"]):
+            assert abs(g["confidence"][r] - o["confidence"][r]) <= P_TOL, (i, r, g["confidence"], o["confidence"])
+        if capture:
+            cap = o["capture"]
+            for r in range(o["n_evaluated"]):
+                assert rel_err(rec["g_h"][r], cap["h_readout"][r]) <= REL_TOL, (i, r)
+                assert rel_err(rec["g_y"][r], cap["y_readout"][r]) <= REL_TOL, (i, r)
+                assert rel_err(rec["g_rl"][r], cap["readout_logits"][r]) <= REL_TOL, (i, r)
+            if not o["exited"]:
+                assert rel_err(rec["g_hL"], cap["h_final"]) <= REL_TOL, i
+                assert rel_err(rec["g_fl"], cap["final_logits"]) <= REL_TOL, i
+        if is_excluded(o, taus):
+            excluded += 1
+            continue
+        assert g["token"] == o["token"], (i, g["token"], o["token"])
+        assert g["gate_pass"] == o["gate_pass"], (i, g["gate_pass"], o["gate_pass"])
+        assert g["readout_token"] == o["readout_token"], (i, g["readout_token"], o["readout_token"])
+        if not o["exited"]:
+            assert g["full_token"] == o["full_token"], i
+    return excluded
+
+
+def check_kv(orc, eng, shape, n_pos: int):
+    """KV positions: which (layer, pos) were written and how, bit for bit;
+    values within REL_TOL per vector."""
+    for j in range(shape.n_layers):
+        for t in range(n_pos):
+            ko, vo, so = orc.kv(j, t)
+            assert eng.kv_src(j, t) == so, (j, t)
+            kg, vg = eng.kv(j, t)
+            assert rel_err(kg, ko) <= REL_TOL and rel_err(vg, vo) <= REL_TOL, (j, t)
