@@ -212,6 +212,26 @@ int ee_set_option(ee_ctx* ctx, int option, int value);
  * Synchronous. */
 int ee_debug_read(ee_ctx* ctx, int what, int layer, int pos, void* host_dst, size_t bytes);
 
+/* ---- measurement ------------------------------------------------------- */
+
+#define EE_KERNEL_QKV 0      /* RMSNorm + Q/K/V GEMV + RoPE + KV append (one layer) */
+#define EE_KERNEL_ATTN 1     /* split-K paged attention (one layer)                 */
+#define EE_KERNEL_OPROJ 2    /* output projection + residual (one layer)            */
+#define EE_KERNEL_GATEUP 3   /* RMSNorm + gate/up GEMV + SiLU product (one layer)   */
+#define EE_KERNEL_DOWN 4     /* down projection + residual (one layer)              */
+#define EE_KERNEL_READOUT 5  /* readout affine map                                  */
+#define EE_KERNEL_VOCAB 6    /* unembedding pass with the confidence statistics     */
+#define EE_KERNEL_KVFILL 7   /* KV fill of the layers above the first readout       */
+#define EE_NUM_KERNELS 8
+/* Average device time (ms) of each decode kernel, from CUDA events around
+ * `iters` back-to-back direct launches on the context's stream, cycling
+ * through the layers so consecutive launches read different weights.  No
+ * counterpart in the paper (measurement only).  Needs a prefilled context
+ * with at least one readout; leaves the KV entries of the next position and
+ * the residual scratch overwritten, which the next step rewrites anyway.
+ * ms_out: host float[EE_NUM_KERNELS]. */
+int ee_profile_kernels(ee_ctx* ctx, int iters, float* ms_out);
+
 /* ---- standalone kernels on caller buffers ----------------------------- */
 
 /* Split-K decode attention of one query position over a paged bf16 KV cache

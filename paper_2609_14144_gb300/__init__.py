@@ -177,6 +177,12 @@ class Engine:
         check(self.lib.ee_position(self.ctx, ctypes.byref(p)))
         return p.value
 
+    def profile_kernels(self, iters: int = 56) -> dict:
+        """Average device ms of each decode kernel (direct launches, CUDA events)."""
+        out = np.zeros(len(_lib.KERNELS), np.float32)
+        check(self.lib.ee_profile_kernels(self.ctx, int(iters), out.ctypes.data))
+        return {k: float(v) for k, v in zip(_lib.KERNELS, out)}
+
     # ------------------------------------------------------------ debug
     def _read(self, what: int, layer: int, pos: int, out: np.ndarray) -> np.ndarray:
         check(self.lib.ee_debug_read(self.ctx, what, layer, pos, out.ctypes.data, out.nbytes))

@@ -1003,6 +1003,62 @@ int ee_debug_read(ee_ctx* c, int what, int layer, int pos, void* host_dst, size_
     }
 }
 
+int ee_profile_kernels(ee_ctx* c, int iters, float* ms_out) {
+    if (!c || !ms_out || iters <= 0) return fail(EE_EINVAL, "bad argument");
+    if (!c->prefilled || c->n_readouts == 0) return fail(EE_ESTATE, "needs a prefilled context with a readout");
+    if (c->pos >= c->cfg.max_ctx) return fail(EE_ERANGE, "no free position to profile at");
+    const DevModel& m = c->dm;
+    cudaStream_t s = c->stream;
+    const int L = m.L;
+    const int64_t d = m.d, F = m.F, AD = (int64_t)m.A * m.D;
+    const int gq = gemv_grid(c, c->lay.n_units_qkv * 2 * d / 8), go = gemv_grid(c, d * AD / 8);
+    const int gu = gemv_grid(c, F * 2 * d / 8), gd = gemv_grid(c, d * F / 8), gr = gemv_grid(c, d * d / 8);
+    char* scratch = c->ws + c->lay.out_tok;  // int32 token + float p of the standalone vocab mode
+    VocabArgs va = vocab_args(c, 2, 0, 0, 0);
+    va.mode = 0;
+    va.logits = nullptr;
+    va.out_token = (int32_t*)scratch;
+    va.out_p = (float*)(scratch + 4);
+    cudaEvent_t e0, e1;
+    EE_CK(cudaEventCreate(&e0));
+    EE_CK(cudaEventCreate(&e1));
+    int rc = EE_OK;
+    for (int k = 0; k < EE_NUM_KERNELS && rc == EE_OK; ++k) {
+        auto one = [&](int i) -> cudaError_t {
+            const int j = i % L;
+            switch (k) {
+                case EE_KERNEL_QKV: return launch_qkv(m, j, 0, gq, false, s);
+                case EE_KERNEL_ATTN: return launch_attention(attn_args(c, j), m.D, false, s);
+                case EE_KERNEL_OPROJ: return launch_oproj(m, j, go, false, s);
+                case EE_KERNEL_GATEUP: return launch_gateup(m, j, gu, false, s);
+                case EE_KERNEL_DOWN: return launch_down(m, j, gd, false, s);
+                case EE_KERNEL_READOUT: return launch_readout(m, i % c->n_readouts, gr, false, s);
+                case EE_KERNEL_VOCAB: return launch_vocab(va, c->grid_vocab, false, s);
+                default: {
+                    const int e = c->ro_layer[0];
+                    if (e >= L) return cudaSuccess;
+                    const int nl = L - e;
+                    const int64_t ch = (int64_t)m.KH * m.D * 2 * m.d / 8;
+                    const int gx = std::max(1, std::min(gemv_grid(c, ch), (c->grid_gemv + nl - 1) / nl));
+                    return launch_kvfill(m, e, gx, false, s);
+                }
+            }
+        };
+        cudaError_t e = one(0);  // warm the launch path
+        if (e == cudaSuccess) e = cudaEventRecord(e0, s);
+        for (int i = 0; i < iters && e == cudaSuccess; ++i) e = one(i + 1);
+        if (e == cudaSuccess) e = cudaEventRecord(e1, s);
+        if (e == cudaSuccess) e = cudaEventSynchronize(e1);
+        float ms = 0.f;
+        if (e == cudaSuccess) e = cudaEventElapsedTime(&ms, e0, e1);
+        if (e != cudaSuccess) rc = fail(EE_ECUDA, std::string("profile: ") + cudaGetErrorString(e));
+        ms_out[k] = ms / iters;
+    }
+    cudaEventDestroy(e0);
+    cudaEventDestroy(e1);
+    return rc;
+}
+
 // ---------------------------------------------------------------- standalone ops
 
 int ee_attention_scratch_bytes(int n_heads, int n_kv_heads, int head_dim, size_t* bytes) {

@@ -52,6 +52,8 @@ struct Ctl {
     const int32_t* prompt; // prompt ids of the running prefill
 };
 
+static_assert(sizeof(Ctl) == 328, "control block size is part of the host read-back accounting");
+
 // Device pointers and shape, passed by value to every kernel.
 struct DevModel {
     int L, d, A, KH, D, F, V, max_ctx, page_size, n_pages, qkv_bias, n_readouts;
