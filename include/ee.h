@@ -248,6 +248,28 @@ int ee_attention_decode(const float* q, const uint16_t* k_pages, const uint16_t*
                         const int32_t* page_table, int T, int n_heads, int n_kv_heads, int head_dim,
                         int page_size, void* scratch, size_t scratch_bytes, float* out, void* stream);
 
+/* Split-K decode attention for callers that cannot allocate device memory:
+ * the same computation, arguments and result as ee_attention_decode, minus
+ * the scratch buffer.  The paper has no counterpart; this exists for callers
+ * whose device memory belongs entirely to another allocator, whose hot path
+ * must not call cudaMalloc/cudaFree (which may synchronise the device), or
+ * that have no allocator at all.
+ *   Scratch lives in one fixed device area of EE_STATIC_ATTN_SCRATCH_BYTES
+ *   inside this library, held by every GPU that loads the library until the
+ *   process exits.  Shapes needing more (n_heads * (head_dim + 2) above about
+ *   4096) are rejected with EE_EINVAL and a message.
+ *   The area is shared by every call and keeps the previous call's contents;
+ *   each call clears the part that must start at zero.  Calls whose work
+ *   overlaps on the GPU (other streams, other threads) race on the area:
+ *   order them on one stream.
+ *   The first call on each device looks up the area's device address (with
+ *   that device current); make that first call before any stream capture.
+ *   No cudaMalloc, cudaFree or other allocating call is made. */
+#define EE_STATIC_ATTN_SCRATCH_BYTES (2u << 20)
+int ee_attention_decode_static(const float* q, const uint16_t* k_pages, const uint16_t* v_pages,
+                               const int32_t* page_table, int T, int n_heads, int n_kv_heads, int head_dim,
+                               int page_size, float* out, void* stream);
+
 /* One pass over an unembedding matrix with the readout's confidence test
  * (Section 2 readout + confidence gate; Section 4 step five):
  *   x        device fp32 [d] residual-space vector (a readout output or h_L)

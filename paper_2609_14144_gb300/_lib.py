@@ -18,7 +18,8 @@ DBG_HIDDEN_READOUT, DBG_READOUT_Y, DBG_HIDDEN_FINAL, DBG_READOUT_LOGITS, DBG_FIN
 SYMBOLS = ("ee_workspace_bytes", "ee_create", "ee_destroy", "ee_last_error", "ee_load_weights", "ee_add_readout",
            "ee_set_page_table", "ee_reset", "ee_prefill", "ee_decode_step", "ee_decode_n", "ee_sync",
            "ee_get_stats", "ee_position", "ee_set_option", "ee_debug_read", "ee_attention_scratch_bytes",
-           "ee_attention_decode", "ee_vocab_scratch_bytes", "ee_vocab_confidence", "ee_profile_kernels")
+           "ee_attention_decode", "ee_vocab_scratch_bytes", "ee_vocab_confidence", "ee_profile_kernels",
+           "ee_attention_decode_static")
 KERNELS = ("qkv", "attention", "oproj", "gateup", "down", "readout", "vocab", "kvfill")
 
 
@@ -108,6 +109,8 @@ def load(allow_build: bool = False):
     lib.ee_vocab_confidence.argtypes = [_P, _P, _P, ctypes.c_int, ctypes.c_int, ctypes.c_float, _P, sz, _P, _P, _P,
                                         _P]
     lib.ee_profile_kernels.argtypes = [_P, ctypes.c_int, _P]
+    lib.ee_attention_decode_static.argtypes = [_P, _P, _P, _P, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                                               ctypes.c_int, _P, _P]
     for name in SYMBOLS:
         f = getattr(lib, name)
         if name != "ee_last_error":

@@ -158,6 +158,8 @@ Layout make_layout(const ee_model_config& c) {
 
 }  // namespace
 
+int ee::set_last_error(int code, const char* msg) { return fail(code, msg); }
+
 struct ee_ctx {
     ee_model_config cfg{};
     Layout lay{};

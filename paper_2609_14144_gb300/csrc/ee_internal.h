@@ -155,6 +155,9 @@ cudaError_t launch_prefill_advance(const DevModel& m, int has_cond, cudaGraphCon
 cudaError_t launch_prefill_end(const DevModel& m, bool pdl, cudaStream_t s);
 cudaError_t launch_set_inputs(Ctl* c, const CtlInputs& in, cudaStream_t s);
 
+// Record `msg` as the calling thread's last error and return `code`.
+int set_last_error(int code, const char* msg);
+
 // Dynamic shared memory each GEMV kernel asks for, given the largest K.
 size_t gemv_smem_bytes(int kmax);
 cudaError_t configure_kernels(int kmax);
