@@ -16,6 +16,7 @@
 #include <cstdio>
 #include <cstring>
 #include <string>
+#include <thread>
 #include <vector>
 
 #include "ee.h"
@@ -46,7 +47,6 @@ int fail(int code, const std::string& msg) {
 
 constexpr size_t kAlign = 256;
 constexpr int kMaxGemvCtas = 1024;
-constexpr int kMaxGemvWarps = kMaxGemvCtas * (kGemvThreads / 32);
 constexpr int kMaxVocabCtas = 1024;
 constexpr int kCaptureDepth = kMaxReadouts + 3;
 
@@ -60,7 +60,7 @@ struct Layout {
     size_t gemv_part, gemv_ticket, attn_part, attn_ticket, vocab_part, vocab_ticket;
     size_t prompt, sched, out_tok, out_exit, out_conf, total;
     int64_t layer_stride, off_wqkv, off_bqkv, off_gattn, off_wo, off_gmlp, off_wgu, off_wd;
-    int64_t n_units_qkv, kv_layer_stride, gemv_part_stride, gemv_ticket_stride;
+    int64_t n_units_qkv, kv_layer_stride, gemv_ticket_stride;
     int n_pages;
 };
 
@@ -90,24 +90,24 @@ Layout make_layout(const ee_model_config& c) {
     l.n_units_qkv = (A + 2 * KH) * D / 2;
     int64_t o = 0;
     l.off_wqkv = o;
-    o += align_elems(l.n_units_qkv * 2 * d);
+    o += align_elems(tiled_elems(l.n_units_qkv * 2, d));
     l.off_bqkv = o;
     o += align_elems(l.n_units_qkv * 2);
     l.off_gattn = o;
     o += align_elems(d);
     l.off_wo = o;
-    o += align_elems(d * A * D);
+    o += align_elems(tiled_elems(d, A * D));
     l.off_gmlp = o;
     o += align_elems(d);
     l.off_wgu = o;
-    o += align_elems(F * 2 * d);
+    o += align_elems(tiled_elems(2 * F, d));
     l.off_wd = o;
-    o += align_elems(d * F);
+    o += align_elems(tiled_elems(d, F));
     l.layer_stride = o;
     l.n_pages = (c.max_ctx + c.page_size - 1) / c.page_size;
     l.kv_layer_stride = (int64_t)l.n_pages * KH * c.page_size * D;
-    l.gemv_part_stride = (int64_t)kMaxGemvWarps * 2 * 2;
-    l.gemv_ticket_stride = align_elems(std::max<int64_t>({l.n_units_qkv, d, F}));
+    l.gemv_ticket_stride = align_elems(std::max<int64_t>({tile_count(2 * l.n_units_qkv), tile_count(d),
+                                                         tile_count(2 * F)}));
 
     size_t b = 0;
     auto take = [&](size_t bytes) {
@@ -119,11 +119,11 @@ Layout make_layout(const ee_model_config& c) {
     l.rope = take(sizeof(float2) * (size_t)c.max_ctx * (D / 2));
     l.layers = take(2 * (size_t)l.layer_stride * L);
     l.embed = take(2 * (size_t)V * d);
-    l.lm_head = c.tied_embedding ? l.embed : take(2 * (size_t)V * d);
+    l.lm_head = take(2 * (size_t)tiled_elems(V, d));
     l.g_final = take(2 * (size_t)d);
     for (int r = 0; r < kMaxReadouts; ++r) {
         if (r < c.max_readouts) {
-            l.ro_w[r] = take(2 * (size_t)d * d);
+            l.ro_w[r] = take(2 * (size_t)tiled_elems(d, d));
             l.ro_b[r] = take(2 * (size_t)d);
         } else {
             l.ro_w[r] = l.ro_b[r] = 0;
@@ -141,7 +141,7 @@ Layout make_layout(const ee_model_config& c) {
     l.hk = take(4 * (size_t)R * d);
     l.logits_ro = take(4 * (size_t)R * V);
     l.logits_final = take(4 * (size_t)V);
-    l.gemv_part = take(4 * (size_t)l.gemv_part_stride * L);
+    l.gemv_part = take(4 * (size_t)(kMaxGemvCtas + L) * 2 * kTileRows);
     l.gemv_ticket = take(4 * (size_t)l.gemv_ticket_stride * L);
     l.attn_part = take(4 * (size_t)A * kAttnMaxSplits * (D + 2));
     l.attn_ticket = take(4 * (size_t)KH);
@@ -154,6 +154,36 @@ Layout make_layout(const ee_model_config& c) {
     l.out_conf = take(4 * (size_t)c.max_ctx);
     l.total = b;
     return l;
+}
+
+// Copy rows (nullptr = zero padding) of K bf16 values into the tiled layout:
+// element (row, k) goes to ((row / 32 * K / 8 + k / 8) * 32 + row % 32) * 8 + k % 8.
+void pack_tiles(uint16_t* dst, const std::vector<const uint16_t*>& rows, int64_t K) {
+    const int64_t n_tiles = tile_count((int64_t)rows.size()), Rc = K / 8;
+    auto work = [&](int64_t t0, int64_t t1) {
+        for (int64_t t = t0; t < t1; ++t)
+            for (int r = 0; r < kTileRows; ++r) {
+                const int64_t row = t * kTileRows + r;
+                const uint16_t* src = row < (int64_t)rows.size() ? rows[row] : nullptr;
+                for (int64_t cc = 0; cc < Rc; ++cc) {
+                    uint16_t* o = dst + ((t * Rc + cc) * kTileRows + r) * 8;
+                    if (src)
+                        std::memcpy(o, src + cc * 8, 16);
+                    else
+                        std::memset(o, 0, 16);
+                }
+            }
+    };
+    const int nt = (int)std::max(1u, std::min(16u, std::thread::hardware_concurrency()));
+    std::vector<std::thread> pool;
+    for (int i = 0; i < nt; ++i) pool.emplace_back(work, n_tiles * i / nt, n_tiles * (i + 1) / nt);
+    for (auto& th : pool) th.join();
+}
+
+std::vector<const uint16_t*> row_ptrs(const uint16_t* base, int64_t n_rows, int64_t K) {
+    std::vector<const uint16_t*> v(n_rows);
+    for (int64_t i = 0; i < n_rows; ++i) v[i] = base + i * K;
+    return v;
 }
 
 }  // namespace
@@ -191,12 +221,14 @@ void drop_graphs(ee_ctx* c) {
         }
 }
 
-// Grid of a flat GEMV launch: one CTA per SM, fewer when the matrix is small
-// (every warp keeps at least 32 chunks = 512 bytes).
-int gemv_grid(const ee_ctx* c, int64_t chunks) {
-    const int64_t per_cta = 32LL * (kGemvThreads / 32);
-    const int64_t g = std::max<int64_t>(1, chunks / per_cta);
-    return (int)std::min<int64_t>(g, c->grid_gemv);
+// Grid of a tiled GEMV launch over `rows` rows of length K: one CTA per SM,
+// fewer when each warp would get less than one 512-byte item, but enough that
+// no CTA touches more than kGemvSlotTiles tiles.
+int gemv_grid(const ee_ctx* c, int64_t rows, int64_t K) {
+    const int64_t tiles = tile_count(rows), items = tiles * (K / 8);
+    int64_t g = std::min<int64_t>(c->grid_gemv, std::max<int64_t>(1, items / (kGemvThreads / 32)));
+    const int64_t need = (tiles + kGemvSlotTiles - 3) / (kGemvSlotTiles - 2);
+    return (int)std::max<int64_t>(g, need);
 }
 
 AttnArgs attn_args(const ee_ctx* c, int j) {
@@ -223,6 +255,7 @@ VocabArgs vocab_args(const ee_ctx* c, int mode, int r, int has_cond, cudaGraphCo
     v.x = mode == 1 ? m.y + (int64_t)r * m.d : m.h;
     v.gain = m.g_final;
     v.U = m.lm_head;
+    v.tiled = 1;
     v.V = m.V;
     v.d = m.d;
     v.eps = m.eps;
@@ -243,10 +276,10 @@ VocabArgs vocab_args(const ee_ctx* c, int mode, int r, int has_cond, cudaGraphCo
 int enqueue_layers(ee_ctx* c, cudaStream_t s, int j0, int j1, bool& pdl) {
     const DevModel& m = c->dm;
     const int64_t d = m.d, F = m.F, AD = (int64_t)m.A * m.D;
-    const int gq = gemv_grid(c, c->lay.n_units_qkv * 2 * d / 8);
-    const int go = gemv_grid(c, d * AD / 8);
-    const int gu = gemv_grid(c, F * 2 * d / 8);
-    const int gd = gemv_grid(c, d * F / 8);
+    const int gq = gemv_grid(c, c->lay.n_units_qkv * 2, d);
+    const int go = gemv_grid(c, d, AD);
+    const int gu = gemv_grid(c, 2 * F, d);
+    const int gd = gemv_grid(c, d, F);
     for (int j = j0; j < j1; ++j) {
         EE_CK(launch_qkv(m, j, j == 0 ? 1 : 0, gq, pdl, s));
         pdl = c->use_pdl;
@@ -260,7 +293,7 @@ int enqueue_layers(ee_ctx* c, cudaStream_t s, int j0, int j1, bool& pdl) {
 
 int enqueue_readout(ee_ctx* c, cudaStream_t s, int r, int has_cond, cudaGraphConditionalHandle cond, bool& pdl) {
     const DevModel& m = c->dm;
-    EE_CK(launch_readout(m, r, gemv_grid(c, (int64_t)m.d * m.d / 8), pdl, s));
+    EE_CK(launch_readout(m, r, gemv_grid(c, m.d, m.d), pdl, s));
     pdl = c->use_pdl;
     EE_CK(launch_vocab(vocab_args(c, 1, r, has_cond, cond), c->grid_vocab, pdl, s));
     return EE_OK;
@@ -272,13 +305,19 @@ int enqueue_head(ee_ctx* c, cudaStream_t s, bool& pdl) {
     return EE_OK;
 }
 
+// CTAs per layer of the KV fill: the SMs shared between the filled layers.
+int fill_grid_x(const ee_ctx* c, int n_layers) {
+    const int64_t rows = 2LL * c->dm.KH * c->dm.D;
+    const int g = gemv_grid(c, rows, c->dm.d);
+    const int need = (int)((tile_count(rows) + kGemvSlotTiles - 3) / (kGemvSlotTiles - 2));
+    return std::max(need, std::min(g, (c->grid_gemv + n_layers - 1) / n_layers));
+}
+
 int enqueue_fill(ee_ctx* c, cudaStream_t s, int exit_layer, bool pdl) {
     const DevModel& m = c->dm;
     if (exit_layer >= m.L) return EE_OK;
     const int nl = m.L - exit_layer;
-    const int64_t chunks = (int64_t)m.KH * m.D * 2 * m.d / 8;
-    const int gx = std::max(1, std::min(gemv_grid(c, chunks), (c->grid_gemv + nl - 1) / nl));
-    EE_CK(launch_kvfill(m, exit_layer, gx, pdl, s));
+    EE_CK(launch_kvfill(m, exit_layer, fill_grid_x(c, nl), pdl, s));
     return EE_OK;
 }
 
@@ -552,8 +591,8 @@ int ee_create(const ee_model_config* cfg, void* d_workspace, size_t workspace_by
     };
     if (cudaGetDevice(&c->device) != cudaSuccess) return bail(fail(EE_ECUDA, "no CUDA device"));
     cudaDeviceGetAttribute(&c->n_sm, cudaDevAttrMultiProcessorCount, c->device);
-    c->grid_gemv = std::min(c->n_sm, kMaxGemvCtas);
-    c->grid_vocab = std::min(c->n_sm, kMaxVocabCtas);
+    c->grid_gemv = std::min(2 * c->n_sm, kMaxGemvCtas);  // two 512-thread CTAs per SM
+    c->grid_vocab = std::min(2 * c->n_sm, kMaxVocabCtas);
     if (d_workspace) {
         if (workspace_bytes < c->lay.total) return bail(fail(EE_ENOMEM, "workspace too small"));
         c->ws = (char*)d_workspace;
@@ -615,8 +654,7 @@ int ee_create(const ee_model_config* cfg, void* d_workspace, size_t workspace_by
     m.logits_ro = (float*)(w + l.logits_ro);
     m.logits_final = (float*)(w + l.logits_final);
     m.gemv_part = (float*)(w + l.gemv_part);
-    m.gemv_ticket = (int*)(w + l.gemv_ticket);
-    m.gemv_part_stride = l.gemv_part_stride;
+    m.gemv_ticket = (unsigned*)(w + l.gemv_ticket);
     m.gemv_ticket_stride = l.gemv_ticket_stride;
     m.attn_part = (float*)(w + l.attn_part);
     m.attn_ticket = (int*)(w + l.attn_ticket);
@@ -687,10 +725,10 @@ int ee_load_weights(ee_ctx* c, const ee_host_weights* w) {
     std::memset(stage, 0, 2 * (size_t)l.layer_stride);
     int rc = EE_OK;
     const int64_t half = D / 2;
-    auto copy_row = [&](uint16_t* dst, const uint16_t* src) { std::memcpy(dst, src, 2 * (size_t)d); };
     for (int j = 0; j < L && rc == EE_OK; ++j) {
-        // Q/K/V: units are row pairs (i, i + D/2) of one head, Q heads then K then V
-        uint16_t* wqkv = stage + l.off_wqkv;
+        // Q/K/V: 16 units per tile, a unit being the row pair (i, i + D/2) of
+        // one head (first row on the even lane); Q heads, then K, then V.
+        std::vector<const uint16_t*> rows;
         uint16_t* bqkv = stage + l.off_bqkv;
         int64_t u = 0;
         const uint16_t* mats[3] = {w->wq[j], w->wk[j], w->wv[j]};
@@ -701,23 +739,25 @@ int ee_load_weights(ee_ctx* c, const ee_host_weights* w) {
             for (int64_t h = 0; h < heads[t]; ++h)
                 for (int64_t i = 0; i < half; ++i, ++u) {
                     const int64_t r0 = h * D + i, r1 = h * D + i + half;
-                    copy_row(wqkv + (u * 2 + 0) * d, mats[t] + r0 * d);
-                    copy_row(wqkv + (u * 2 + 1) * d, mats[t] + r1 * d);
+                    rows.push_back(mats[t] + r0 * d);
+                    rows.push_back(mats[t] + r1 * d);
                     if (bias[t]) {
                         bqkv[u * 2 + 0] = bias[t][r0];
                         bqkv[u * 2 + 1] = bias[t][r1];
                     }
                 }
+        pack_tiles(stage + l.off_wqkv, rows, d);
         std::memcpy(stage + l.off_gattn, w->attn_norm[j], 2 * (size_t)d);
-        std::memcpy(stage + l.off_wo, w->wo[j], 2 * (size_t)d * A * D);
+        pack_tiles(stage + l.off_wo, row_ptrs(w->wo[j], d, A * D), A * D);
         std::memcpy(stage + l.off_gmlp, w->mlp_norm[j], 2 * (size_t)d);
-        // gate/up: unit i is (W_g row i, W_u row i)
-        uint16_t* wgu = stage + l.off_wgu;
+        // gate/up: 16 units per tile, unit i = (W_g row i, W_u row i)
+        rows.clear();
         for (int64_t i = 0; i < F; ++i) {
-            copy_row(wgu + (i * 2 + 0) * d, w->wg[j] + i * d);
-            copy_row(wgu + (i * 2 + 1) * d, w->wu[j] + i * d);
+            rows.push_back(w->wg[j] + i * d);
+            rows.push_back(w->wu[j] + i * d);
         }
-        std::memcpy(stage + l.off_wd, w->wd[j], 2 * (size_t)d * F);
+        pack_tiles(stage + l.off_wgu, rows, d);
+        pack_tiles(stage + l.off_wd, row_ptrs(w->wd[j], d, F), F);
         cudaError_t e = cudaMemcpy(c->ws + l.layers + 2 * (size_t)l.layer_stride * j, stage,
                                    2 * (size_t)l.layer_stride, cudaMemcpyHostToDevice);
         if (e != cudaSuccess) rc = fail(EE_ECUDA, std::string("layer upload: ") + cudaGetErrorString(e));
@@ -725,7 +765,11 @@ int ee_load_weights(ee_ctx* c, const ee_host_weights* w) {
     cudaFreeHost(stage);
     if (rc != EE_OK) return rc;
     EE_CK(cudaMemcpy(c->ws + l.embed, w->embed, 2 * (size_t)V * d, cudaMemcpyHostToDevice));
-    if (!cf.tied_embedding) EE_CK(cudaMemcpy(c->ws + l.lm_head, w->lm_head, 2 * (size_t)V * d, cudaMemcpyHostToDevice));
+    {
+        std::vector<uint16_t> tiled((size_t)tiled_elems(V, d));
+        pack_tiles(tiled.data(), row_ptrs(cf.tied_embedding ? w->embed : w->lm_head, V, d), d);
+        EE_CK(cudaMemcpy(c->ws + l.lm_head, tiled.data(), 2 * tiled.size(), cudaMemcpyHostToDevice));
+    }
     EE_CK(cudaMemcpy(c->ws + l.g_final, w->final_norm, 2 * (size_t)d, cudaMemcpyHostToDevice));
     c->weights = true;
     drop_graphs(c);
@@ -741,7 +785,9 @@ int ee_add_readout(ee_ctx* c, int layer, const uint16_t* wr, const uint16_t* br,
         return fail(EE_EINVAL, "readouts must be added in increasing layer order");
     const int r = c->n_readouts;
     const size_t d = c->cfg.d_model;
-    EE_CK(cudaMemcpy(c->ws + c->lay.ro_w[r], wr, 2 * d * d, cudaMemcpyHostToDevice));
+    std::vector<uint16_t> tiled((size_t)tiled_elems(d, d));
+    pack_tiles(tiled.data(), row_ptrs(wr, d, d), d);
+    EE_CK(cudaMemcpy(c->ws + c->lay.ro_w[r], tiled.data(), 2 * tiled.size(), cudaMemcpyHostToDevice));
     EE_CK(cudaMemcpy(c->ws + c->lay.ro_b[r], br, 2 * d, cudaMemcpyHostToDevice));
     c->ro_layer[r] = layer;
     c->dm.ro_layer[r] = layer;
@@ -1013,8 +1059,8 @@ int ee_profile_kernels(ee_ctx* c, int iters, float* ms_out) {
     cudaStream_t s = c->stream;
     const int L = m.L;
     const int64_t d = m.d, F = m.F, AD = (int64_t)m.A * m.D;
-    const int gq = gemv_grid(c, c->lay.n_units_qkv * 2 * d / 8), go = gemv_grid(c, d * AD / 8);
-    const int gu = gemv_grid(c, F * 2 * d / 8), gd = gemv_grid(c, d * F / 8), gr = gemv_grid(c, d * d / 8);
+    const int gq = gemv_grid(c, c->lay.n_units_qkv * 2, d), go = gemv_grid(c, d, AD);
+    const int gu = gemv_grid(c, 2 * F, d), gd = gemv_grid(c, d, F), gr = gemv_grid(c, d, d);
     char* scratch = c->ws + c->lay.out_tok;  // int32 token + float p of the standalone vocab mode
     VocabArgs va = vocab_args(c, 2, 0, 0, 0);
     va.mode = 0;
@@ -1039,10 +1085,7 @@ int ee_profile_kernels(ee_ctx* c, int iters, float* ms_out) {
                 default: {
                     const int e = c->ro_layer[0];
                     if (e >= L) return cudaSuccess;
-                    const int nl = L - e;
-                    const int64_t ch = (int64_t)m.KH * m.D * 2 * m.d / 8;
-                    const int gx = std::max(1, std::min(gemv_grid(c, ch), (c->grid_gemv + nl - 1) / nl));
-                    return launch_kvfill(m, e, gx, false, s);
+                    return launch_kvfill(m, e, fill_grid_x(c, L - e), false, s);
                 }
             }
         };
@@ -1122,6 +1165,7 @@ int ee_vocab_confidence(const float* x, const uint16_t* gain, const uint16_t* U,
     v.x = x;
     v.gain = gain;
     v.U = U;
+    v.tiled = 0;
     v.V = vocab;
     v.d = d_model;
     v.eps = eps;

@@ -19,6 +19,7 @@ constexpr int kAttnMaxSplits = 128; // splits per key-value head (at most)
 constexpr int kErrNanConfidence = 1;
 constexpr int kErrTokenRange = 2;
 constexpr int kErrPosition = 4;
+constexpr int kErrShape = 8;  // a GEMV CTA would touch more tiles than it can hold
 
 // Device-resident control block: everything a step reads or writes that is
 // not a tensor, so one captured graph serves every step, tau and force.
@@ -82,10 +83,9 @@ struct DevModel {
     float* hk;                    // residual seen by each readout [R][d]
     float* logits_ro;             // [R][V] (debug)
     float* logits_final;          // [V] (debug)
-    float* gemv_part;             // cross-warp partial sums
-    int* gemv_ticket;             // per-unit arrival counters
-    int64_t gemv_part_stride;     // floats per fill layer in gemv_part
-    int64_t gemv_ticket_stride;   // ints per fill layer in gemv_ticket
+    float* gemv_part;             // cross-CTA tile partials: [CTA slot][2][32]
+    unsigned* gemv_ticket;        // per-tile arrival counters
+    int64_t gemv_ticket_stride;   // counters per fill layer in gemv_ticket
     float* attn_part;             // [A][kAttnMaxSplits][D + 2]
     int* attn_ticket;             // [KH]
     float* vocab_part;            // [grid][4]
@@ -111,7 +111,8 @@ struct AttnArgs {
 struct VocabArgs {
     const float* x;           // residual-space input [d]
     const uint16_t* gain;     // final RMSNorm gain [d]
-    const uint16_t* U;        // [V, d]
+    const uint16_t* U;        // [V, d], tiled (engine) or row-major (standalone)
+    int tiled;
     int V, d;
     float eps;
     float* logits;            // optional [V]
@@ -161,5 +162,11 @@ int set_last_error(int code, const char* msg);
 // Dynamic shared memory each GEMV kernel asks for, given the largest K.
 size_t gemv_smem_bytes(int kmax);
 cudaError_t configure_kernels(int kmax);
+
+// Geometry of the tiled weight layout (rows grouped by 32, see ee_kernels.cu).
+constexpr int kTileRows = 32;
+constexpr int kGemvSlotTiles = 8;   // tiles one GEMV CTA may touch
+inline int64_t tile_count(int64_t rows) { return (rows + kTileRows - 1) / kTileRows; }
+inline int64_t tiled_elems(int64_t rows, int64_t K) { return tile_count(rows) * kTileRows * K; }
 
 }  // namespace ee

@@ -18,6 +18,7 @@
 // are finished by whichever contributing warp arrives last, summing the
 // contributions in warp order, so results do not depend on timing.
 #include <cuda_bf16.h>
+#include <math.h>
 #include <math_constants.h>
 
 #include "ee_internal.h"
@@ -35,7 +36,7 @@ __device__ __forceinline__ uint16_t f2bf(float f) { return __bfloat16_as_ushort(
 // L2 sector promotion.
 __device__ __forceinline__ uint4 ldg_stream(const uint4* p) {
     uint4 r;
-    asm("ld.global.nc.L1::no_allocate.L2::256B.v4.u32 {%0,%1,%2,%3}, [%4];"
+    asm volatile("ld.global.nc.L1::no_allocate.L2::256B.v4.u32 {%0,%1,%2,%3}, [%4];"
         : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
         : "l"(p));
     return r;
@@ -106,20 +107,6 @@ __device__ __forceinline__ void warp_range(int64_t n_units, int64_t Cu, int warp
         c0 = Ct * warp / nwarps;
         c1 = Ct * (warp + 1) / nwarps;
     }
-}
-
-// Before waiting on the predecessor kernel: pull the head of this warp's
-// weight slice into L2 so the stream starts at full rate.
-constexpr uint32_t kPrefetchCap = 16384;
-
-template <int NR, bool ALIGNED>
-__device__ __forceinline__ void prefetch_slice(const uint16_t* W, int K, int64_t n_units, int warp, int nwarps) {
-    if ((threadIdx.x & 31) != 0) return;
-    int64_t c0, c1;
-    warp_range<ALIGNED>(n_units, (int64_t)NR * (K >> 3), warp, nwarps, c0, c1);
-    if (c1 <= c0) return;
-    const int64_t bytes = (c1 - c0) * 16;
-    prefetch_l2(W + c0 * 8, (uint32_t)(bytes < kPrefetchCap ? bytes : kPrefetchCap));
 }
 
 // The flat GEMV core (see the file comment).  Epi is called by lane 0 with
@@ -221,84 +208,227 @@ __device__ __forceinline__ void flat_gemv(const uint16_t* __restrict__ W, int K,
     if (row * Rc < c1) finish_row(row, warp_sum(acc));
 }
 
-// ------------------------------------------------------------------ epilogues
+// ------------------------------------------------------------------ tiled GEMV
+//
+// Engine weights are repacked into tiles of 32 rows: for each 16-byte column
+// chunk c, the 32 rows' chunks are stored back to back (512 bytes), so one
+// warp instruction streams 512 contiguous bytes and lane r owns row r of the
+// tile: it accumulates that row's dot product on its own, and the activation
+// chunk it multiplies is the same for every lane (a shared-memory broadcast).
+// Element (row, k) of an n_rows x K matrix lives at
+//     ((tile * Rc + c) * 32 + r) * 8 + e,   tile = row / 32, r = row % 32,
+//     c = k / 8, e = k % 8, Rc = K / 8;   rows past n_rows are zero padding.
+// An "item" is one (tile, c) pair; a matrix is n_tiles * Rc items.
 
-// Q/K/V unit: the row pair (i, i + D/2) of one head.  Q is rotated and kept
-// in fp32; K is rotated and V copied into the paged cache as bf16.
+constexpr int kWarps = kGemvThreads / 32;  // warps per GEMV CTA
+constexpr int kSlotTiles = kGemvSlotTiles;  // tiles one CTA may touch
+constexpr int kWindow = 8;                 // loads each lane issues per batch
+
+// The items of one CTA: [C0, C1) of Ct, an equal share of the matrix
+// (item counts fit in 32 bits: the engine checks).
+struct CoopRange {
+    int C0, C1, Ct;
+    int Rc, cta, n_cta;
+};
+
+__device__ __forceinline__ CoopRange coop_range(int64_t n_tiles, int K, int cta, int n_cta) {
+    CoopRange r;
+    r.Rc = K >> 3;
+    r.Ct = (int)(n_tiles * r.Rc);
+    r.C0 = (int)((int64_t)r.Ct * cta / n_cta);
+    r.C1 = (int)((int64_t)r.Ct * (cta + 1) / n_cta);
+    r.cta = cta;
+    r.n_cta = n_cta;
+    return r;
+}
+
+// Warp w of the CTA consumes items C0 + w, C0 + w + 16, ...; the first
+// kWindow of them are loaded here (before the kernel waits on its
+// predecessor: weights never depend on it).
+__device__ __forceinline__ void coop_prefetch(const uint4* W, const CoopRange& r, uint4 (&buf)[kWindow]) {
+    const int lane = threadIdx.x & 31, wl = threadIdx.x >> 5;
+#pragma unroll
+    for (int u = 0; u < kWindow; ++u) {
+        const int it = r.C0 + wl + kWarps * u;
+        buf[u] = it < r.C1 ? ldg_stream(W + (int64_t)it * 32 + lane) : make_uint4(0u, 0u, 0u, 0u);
+    }
+}
+
+// Stream the CTA's items against x (fp32 in shared memory), leaving each
+// warp's share of every tile it touched in sm_part[tile][warp][lane], then
+// synchronise the CTA.  Loads go in batches of kWindow issued back to back
+// before any is used (the first batch was issued by coop_prefetch).  Returns
+// false (before touching anything) if the CTA would touch more than
+// kSlotTiles tiles.
+__device__ __forceinline__ bool coop_stream(const uint4* __restrict__ W, const CoopRange& r,
+                                            uint4 (&buf)[kWindow], const float* __restrict__ xs,
+                                            float* __restrict__ sm_part) {
+    const int lane = threadIdx.x & 31, wl = threadIdx.x >> 5;
+    const int t_first = r.C0 / r.Rc, t_last = (r.C1 - 1) / r.Rc;
+    if (t_last - t_first + 1 > kSlotTiles) return false;
+    const int it = r.C0 + wl;
+    int slot = it / r.Rc - t_first;
+    int c = it - (slot + t_first) * r.Rc;
+    float acc = 0.f;
+    bool pending = false;
+    for (int base = it; base < r.C1; base += kWarps * kWindow) {
+        if (base != it) {
+#pragma unroll
+            for (int u = 0; u < kWindow; ++u) {
+                const int cur = base + kWarps * u;
+                buf[u] = cur < r.C1 ? ldg_stream(W + (int64_t)cur * 32 + lane) : make_uint4(0u, 0u, 0u, 0u);
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < kWindow; ++u) {
+            if (base + kWarps * u >= r.C1) break;
+            acc += dot8(buf[u], xs + c * 8);
+            pending = true;
+            c += kWarps;
+            if (c >= r.Rc) {
+                sm_part[(slot * kWarps + wl) * 32 + lane] = acc;
+                acc = 0.f;
+                pending = false;
+                c -= r.Rc;
+                ++slot;
+            }
+        }
+    }
+    if (pending) sm_part[(slot * kWarps + wl) * 32 + lane] = acc;
+    __syncthreads();
+    return true;
+}
+
+// Combine a tile shared by several CTAs: each contributor leaves its
+// 32 row sums in its slot; the last to arrive sums them in CTA order and
+// runs the epilogue.  kind 0: the tile began before this CTA's range;
+// kind 1: it began inside and runs past the end.
+template <class Epi>
+__device__ __forceinline__ void cross_cta_combine(const CoopRange& r, int tile, float s, int kind, float* g_part,
+                                                  int slot_base, unsigned* ticket, const Epi& epi) {
+    const int lane = threadIdx.x & 31;
+    g_part[((int64_t)(slot_base + r.cta) * 2 + kind) * 32 + lane] = s;
+    __threadfence();
+    __syncwarp();
+    unsigned old = 0;
+    if (lane == 0) old = atomicAdd(&ticket[tile], 1u);
+    old = __shfl_sync(0xffffffffu, old, 0);
+    auto owner = [&](int64_t it) -> int { return (int)(((it + 1) * (int64_t)r.n_cta - 1) / r.Ct); };
+    const int ca = owner((int64_t)tile * r.Rc), cb = owner((int64_t)(tile + 1) * r.Rc - 1);
+    if ((int)old != cb - ca) return;
+    __threadfence();
+    float v = __ldcg(&g_part[((int64_t)(slot_base + ca) * 2 + 1) * 32 + lane]);
+    for (int c = ca + 1; c <= cb; ++c) v += __ldcg(&g_part[((int64_t)(slot_base + c) * 2 + 0) * 32 + lane]);
+    epi(tile, v);
+    if (lane == 0) ticket[tile] = 0;
+}
+
+// Finish every tile the CTA touched (after coop_stream): sum the warps'
+// shares in warp order; whole tiles run the epilogue here, tiles shared with
+// a neighbouring CTA go through cross_cta_combine.
+template <class Epi>
+__device__ __forceinline__ void coop_finish(const CoopRange& r, const float* __restrict__ sm_part, float* g_part,
+                                            int slot_base, unsigned* ticket, const Epi& epi) {
+    const int lane = threadIdx.x & 31, wl = threadIdx.x >> 5;
+    const int t_first = r.C0 / r.Rc, t_last = (r.C1 - 1) / r.Rc;
+    for (int tt = t_first + wl; tt <= t_last; tt += kWarps) {
+        float s = 0.f;
+#pragma unroll
+        for (int w = 0; w < kWarps; ++w) s += sm_part[((tt - t_first) * kWarps + w) * 32 + lane];
+        const bool head = tt * r.Rc < r.C0, tail = (tt + 1) * r.Rc > r.C1;
+        if (!head && !tail)
+            epi(tt, s);
+        else
+            cross_cta_combine(r, tt, s, head ? 0 : 1, g_part, slot_base, ticket, epi);
+    }
+}
+
+// Zero the per-warp tile partials (they must start at zero: a warp may not
+// touch every tile of its CTA).
+__device__ __forceinline__ void zero_sm_part(float* sm_part) {
+    for (int i = threadIdx.x; i < kSlotTiles * kWarps * 32; i += blockDim.x) sm_part[i] = 0.f;
+}
+
+// ------------------------------------------------------------------ epilogues
+// Called by all 32 lanes of a warp with the tile index and lane's row sum.
+
+// Q/K/V tile: 16 units of a row pair (i, i + D/2) of one head, first row on
+// the even lane.  Q is rotated and kept in fp32; K is rotated and V copied
+// into the paged cache as bf16.
 struct EpiQKV {
     float* q;
-    uint16_t* kdst;  // this layer's K page slot base for kv head 0 (stride per head below)
+    uint16_t* kdst;       // this layer's page slot, kv head 0
     uint16_t* vdst;
     int64_t head_stride;  // elements between kv heads inside a page
     const uint16_t* bias; // packed [unit][2] or null
     const float2* cs;     // rope row of this position
-    int64_t unit_offset;
+    int64_t unit_offset;  // unit index of the tile-0 unit
     int D, nq_units, nk_units;
-    __device__ __forceinline__ void operator()(int64_t unit_local, const float* s) const {
-        const int64_t u = unit_local + unit_offset;
-        float r0 = s[0], r1 = s[1];
-        if (bias) {
-            r0 += bf2f(bias[2 * u]);
-            r1 += bf2f(bias[2 * u + 1]);
-        }
+    __device__ __forceinline__ void operator()(int64_t tile, float s) const {
+        const int lane = threadIdx.x & 31, odd = lane & 1;
+        const int64_t u = tile * 16 + (lane >> 1) + unit_offset;
+        if (bias) s += bf2f(bias[2 * u + odd]);
+        const float other = __shfl_xor_sync(0xffffffffu, s, 1);
+        const float r0 = odd ? other : s, r1 = odd ? s : other;
         const int half = D >> 1;
         if (u < nq_units) {
             const int h = (int)(u / half), i = (int)(u - (int64_t)h * half);
             const float2 c = cs[i];
-            q[h * D + i] = r0 * c.x - r1 * c.y;
-            q[h * D + i + half] = r0 * c.y + r1 * c.x;
+            if (!odd)
+                q[h * D + i] = r0 * c.x - r1 * c.y;
+            else
+                q[h * D + i + half] = r0 * c.y + r1 * c.x;
         } else if (u < nq_units + nk_units) {
             const int64_t uu = u - nq_units;
             const int g = (int)(uu / half), i = (int)(uu - (int64_t)g * half);
             const float2 c = cs[i];
             uint16_t* k = kdst + g * head_stride;
-            k[i] = f2bf(r0 * c.x - r1 * c.y);
-            k[i + half] = f2bf(r0 * c.y + r1 * c.x);
+            if (!odd)
+                k[i] = f2bf(r0 * c.x - r1 * c.y);
+            else
+                k[i + half] = f2bf(r0 * c.y + r1 * c.x);
         } else {
             const int64_t uu = u - nq_units - nk_units;
             const int g = (int)(uu / half), i = (int)(uu - (int64_t)g * half);
             uint16_t* v = vdst + g * head_stride;
-            v[i] = f2bf(r0);
-            v[i + half] = f2bf(r1);
+            if (!odd)
+                v[i] = f2bf(r0);
+            else
+                v[i + half] = f2bf(r1);
         }
     }
 };
 
+// Residual add: h[row] += s.
 struct EpiAddH {
     float* h;
-    __device__ __forceinline__ void operator()(int64_t u, const float* s) const { h[u] += s[0]; }
+    int n_rows;
+    __device__ __forceinline__ void operator()(int64_t tile, float s) const {
+        const int64_t row = tile * 32 + (threadIdx.x & 31);
+        if (row < n_rows) h[row] += s;
+    }
 };
 
+// Readout affine map: y[row] = s + b[row].
 struct EpiBias {
     float* y;
     const uint16_t* b;
-    __device__ __forceinline__ void operator()(int64_t u, const float* s) const { y[u] = s[0] + bf2f(b[u]); }
-};
-
-struct EpiSwiGLU {
-    float* a;
-    __device__ __forceinline__ void operator()(int64_t u, const float* s) const {
-        const float g = s[0];
-        const float silu = g / (1.0f + expf(-g));
-        a[u] = silu * s[1];
+    int n_rows;
+    __device__ __forceinline__ void operator()(int64_t tile, float s) const {
+        const int64_t row = tile * 32 + (threadIdx.x & 31);
+        if (row < n_rows) y[row] = s + bf2f(b[row]);
     }
 };
 
-// Running (max, sum of exp, lowest argmax) over logits, plus optional logits.
-struct EpiVocab {
-    float* logits;
-    float m, s;
-    int a;
-    __device__ __forceinline__ void operator()(int64_t u, const float* r) {
-        const float l = r[0];
-        if (logits) logits[u] = l;
-        if (l > m) {
-            s = s * expf(m - l) + 1.0f;
-            m = l;
-            a = (int)u;
-        } else {
-            s += expf(l - m);
-        }
+// Gated FFN tile: 16 units (gate row on the even lane, up row on the odd).
+struct EpiSwiGLU {
+    float* a;
+    int F;
+    __device__ __forceinline__ void operator()(int64_t tile, float s) const {
+        const int lane = threadIdx.x & 31;
+        const float up = __shfl_xor_sync(0xffffffffu, s, 1);
+        const int64_t u = tile * 16 + (lane >> 1);
+        if (!(lane & 1) && u < F) a[u] = s / (1.0f + expf(-s)) * up;
     }
 };
 
@@ -334,6 +464,23 @@ __device__ __forceinline__ void warp_merge_stats(float& m, float& s, int& a) {
     }
 }
 
+// Running (max, sum of exp, lowest argmax) of one lane's rows, plus the
+// logits themselves when requested.
+struct LaneStats {
+    float m, s;
+    int a;
+    __device__ __forceinline__ LaneStats() : m(-INFINITY), s(0.f), a(0x7fffffff) {}
+    __device__ __forceinline__ void add(float l, int row) {
+        if (l > m) {
+            s = s * expf(m - l) + 1.0f;
+            m = l;
+            a = row;
+        } else {
+            s += expf(l - m);
+        }
+    }
+};
+
 __device__ __forceinline__ const uint16_t* layer_base(const DevModel& m, int j) {
     return m.layers + (int64_t)j * m.layer_stride;
 }
@@ -350,23 +497,33 @@ __device__ __forceinline__ void global_warp(int& warp, int& nwarps) {
     nwarps = gridDim.x * wpb;
 }
 
-constexpr int kUnroll = 8;
+__device__ __forceinline__ int64_t tiles_of(int64_t rows) { return (rows + 31) / 32; }
+
+__device__ __forceinline__ void flag_error(Ctl* c, int bit) {
+    if (c && threadIdx.x == 0) atomicOr(&c->err, bit);
+}
+
+// Shared-memory layout of every GEMV kernel: x (K floats), then the tile
+// partials (kSlotTiles * kWarps * 32 floats), then a second K-float area
+// for the first layer's embedding row.
+__device__ __forceinline__ float* sm_partials(float* xs, int K) { return xs + ((K + 3) & ~3); }
 
 // ------------------------------------------------------------------ kernels
 
 // Attention input of layer j: [embedding gather,] RMSNorm, Q/K/V GEMV, RoPE,
 // KV append at the step's position.
-__global__ void __launch_bounds__(kGemvThreads) k_qkv(DevModel m, int layer, int first) {
+__global__ void __launch_bounds__(kGemvThreads, 2) k_qkv(DevModel m, int layer, int first) {
     extern __shared__ float4 smem_f4[];
     float* xs = reinterpret_cast<float*>(smem_f4);
+    float* sm_part = sm_partials(xs, m.d);
     __shared__ float red[32];
     const uint16_t* lw = layer_base(m, layer);
-    const uint16_t* W = lw + m.off_wqkv;
+    const uint4* W = reinterpret_cast<const uint4*>(lw + m.off_wqkv);
     const int64_t nq = (int64_t)m.A * m.D / 2, nk = (int64_t)m.KH * m.D / 2;
-    const int64_t n_units = nq + 2 * nk;
-    int warp, nwarps;
-    global_warp(warp, nwarps);
-    prefetch_slice<2, false>(W, m.d, n_units, warp, nwarps);
+    const CoopRange r = coop_range((nq + 2 * nk) / 16, m.d, blockIdx.x, gridDim.x);
+    uint4 buf[kWindow];
+    coop_prefetch(W, r, buf);
+    zero_sm_part(sm_part);
     pdl_wait();
     pdl_launch_dependents();
     Ctl* c = m.ctl;
@@ -378,7 +535,7 @@ __global__ void __launch_bounds__(kGemvThreads) k_qkv(DevModel m, int layer, int
         int tok = c->in_tok;
         const bool tok_ok = tok >= 0 && tok < m.V;
         if (!tok_ok) tok = 0;
-        float* hl = xs + m.d;
+        float* hl = sm_part + kSlotTiles * kWarps * 32;
         const uint16_t* e = m.embed + (int64_t)tok * m.d;
         for (int i = threadIdx.x; i < m.d; i += blockDim.x) {
             const float v = bf2f(e[i]);
@@ -395,118 +552,133 @@ __global__ void __launch_bounds__(kGemvThreads) k_qkv(DevModel m, int layer, int
         src = hl;
     }
     if (!pos_ok) {
-        if (blockIdx.x == 0 && threadIdx.x == 0) atomicOr(&c->err, kErrPosition);
+        if (blockIdx.x == 0) flag_error(c, kErrPosition);
         return;
     }
     rmsnorm_to_smem(src, lw + m.off_gattn, m.d, m.eps, xs, red);
+    if (!coop_stream(W, r, buf, xs, sm_part)) {
+        flag_error(c, kErrShape);
+        return;
+    }
     const int64_t kvo = kv_slot_offset(m, layer, pos);
-    EpiQKV epi{m.q,
-               m.kpool + kvo,
-               m.vpool + kvo,
-               (int64_t)m.page_size * m.D,
-               m.qkv_bias ? lw + m.off_bqkv : nullptr,
-               m.rope + (int64_t)pos * (m.D / 2),
-               0,
-               m.D,
-               (int)nq,
-               (int)nk};
-    flat_gemv<2, false, kUnroll>(W, m.d, n_units, xs, warp, nwarps, m.gemv_part, m.gemv_ticket, epi);
+    const EpiQKV epi{m.q, m.kpool + kvo, m.vpool + kvo, (int64_t)m.page_size * m.D,
+                     m.qkv_bias ? lw + m.off_bqkv : nullptr, m.rope + (int64_t)pos * (m.D / 2), 0, m.D, (int)nq, (int)nk};
+    coop_finish(r, sm_part, m.gemv_part, 0, m.gemv_ticket, epi);
     if (blockIdx.x == 0 && threadIdx.x == 0) m.kv_src[(int64_t)layer * m.max_ctx + pos] = 1;
 }
 
 // KV repair for the skipped layers exit_layer .. L-1 (0-based) at the step's
 // position: K = RoPE(W_K RMSNorm_j(h_k)), V = W_V RMSNorm_j(h_k), stored bf16.
-__global__ void __launch_bounds__(kGemvThreads) k_kvfill(DevModel m, int exit_layer) {
+// blockIdx.y selects the layer; each layer's K/V tiles are split over
+// gridDim.x CTAs.
+__global__ void __launch_bounds__(kGemvThreads, 2) k_kvfill(DevModel m, int exit_layer) {
     extern __shared__ float4 smem_f4[];
     float* xs = reinterpret_cast<float*>(smem_f4);
+    float* sm_part = sm_partials(xs, m.d);
     __shared__ float red[32];
     const int j = exit_layer + blockIdx.y;
     const uint16_t* lw = layer_base(m, j);
     const int64_t nq = (int64_t)m.A * m.D / 2, nk = (int64_t)m.KH * m.D / 2;
-    const uint16_t* W = lw + m.off_wqkv + nq * 2 * m.d;
-    const int64_t n_units = 2 * nk;
-    int warp, nwarps;
-    global_warp(warp, nwarps);
-    prefetch_slice<2, false>(W, m.d, n_units, warp, nwarps);
+    const uint4* W = reinterpret_cast<const uint4*>(lw + m.off_wqkv + nq * 2 * m.d);
+    const CoopRange r = coop_range(2 * nk / 16, m.d, blockIdx.x, gridDim.x);
+    uint4 buf[kWindow];
+    coop_prefetch(W, r, buf);
+    zero_sm_part(sm_part);
     pdl_wait();
     pdl_launch_dependents();
     const int pos = m.ctl->pos;
     if (pos < 0 || pos >= m.max_ctx) return;
     rmsnorm_to_smem(m.h, lw + m.off_gattn, m.d, m.eps, xs, red);
+    if (!coop_stream(W, r, buf, xs, sm_part)) {
+        flag_error(m.ctl, kErrShape);
+        return;
+    }
     const int64_t kvo = kv_slot_offset(m, j, pos);
-    EpiQKV epi{m.q,
-               m.kpool + kvo,
-               m.vpool + kvo,
-               (int64_t)m.page_size * m.D,
-               m.qkv_bias ? lw + m.off_bqkv : nullptr,
-               m.rope + (int64_t)pos * (m.D / 2),
-               nq,
-               m.D,
-               (int)nq,
-               (int)nk};
-    flat_gemv<2, false, kUnroll>(W, m.d, n_units, xs, warp, nwarps, m.gemv_part + blockIdx.y * m.gemv_part_stride,
-                                 m.gemv_ticket + blockIdx.y * m.gemv_ticket_stride, epi);
+    const EpiQKV epi{m.q, m.kpool + kvo, m.vpool + kvo, (int64_t)m.page_size * m.D,
+                     m.qkv_bias ? lw + m.off_bqkv : nullptr, m.rope + (int64_t)pos * (m.D / 2), nq, m.D, (int)nq, (int)nk};
+    coop_finish(r, sm_part, m.gemv_part, blockIdx.y * gridDim.x, m.gemv_ticket + blockIdx.y * m.gemv_ticket_stride,
+                epi);
     if (blockIdx.x == 0 && threadIdx.x == 0) m.kv_src[(int64_t)j * m.max_ctx + pos] = 2;
 }
 
 // Output projection with the residual add: h += W_o o.
-__global__ void __launch_bounds__(kGemvThreads) k_oproj(DevModel m, int layer) {
+__global__ void __launch_bounds__(kGemvThreads, 2) k_oproj(DevModel m, int layer) {
     extern __shared__ float4 smem_f4[];
     float* xs = reinterpret_cast<float*>(smem_f4);
-    const uint16_t* W = layer_base(m, layer) + m.off_wo;
     const int K = m.A * m.D;
-    int warp, nwarps;
-    global_warp(warp, nwarps);
-    prefetch_slice<1, false>(W, K, m.d, warp, nwarps);
+    float* sm_part = sm_partials(xs, K);
+    const uint4* W = reinterpret_cast<const uint4*>(layer_base(m, layer) + m.off_wo);
+    const CoopRange r = coop_range(tiles_of(m.d), K, blockIdx.x, gridDim.x);
+    uint4 buf[kWindow];
+    coop_prefetch(W, r, buf);
+    zero_sm_part(sm_part);
     pdl_wait();
     pdl_launch_dependents();
     for (int i = threadIdx.x; i < K; i += blockDim.x) xs[i] = m.o[i];
     __syncthreads();
-    EpiAddH epi{m.h};
-    flat_gemv<1, false, kUnroll>(W, K, m.d, xs, warp, nwarps, m.gemv_part, m.gemv_ticket, epi);
+    if (!coop_stream(W, r, buf, xs, sm_part)) {
+        flag_error(m.ctl, kErrShape);
+        return;
+    }
+    const EpiAddH epi{m.h, m.d};
+    coop_finish(r, sm_part, m.gemv_part, 0, m.gemv_ticket, epi);
 }
 
 // Gated feed-forward up: a = SiLU(W_g x) * (W_u x), x = RMSNorm(h) * g_mlp.
-__global__ void __launch_bounds__(kGemvThreads) k_gateup(DevModel m, int layer) {
+__global__ void __launch_bounds__(kGemvThreads, 2) k_gateup(DevModel m, int layer) {
     extern __shared__ float4 smem_f4[];
     float* xs = reinterpret_cast<float*>(smem_f4);
+    float* sm_part = sm_partials(xs, m.d);
     __shared__ float red[32];
     const uint16_t* lw = layer_base(m, layer);
-    const uint16_t* W = lw + m.off_wgu;
-    int warp, nwarps;
-    global_warp(warp, nwarps);
-    prefetch_slice<2, false>(W, m.d, m.F, warp, nwarps);
+    const uint4* W = reinterpret_cast<const uint4*>(lw + m.off_wgu);
+    const CoopRange r = coop_range(tiles_of(2 * (int64_t)m.F), m.d, blockIdx.x, gridDim.x);
+    uint4 buf[kWindow];
+    coop_prefetch(W, r, buf);
+    zero_sm_part(sm_part);
     pdl_wait();
     pdl_launch_dependents();
     rmsnorm_to_smem(m.h, lw + m.off_gmlp, m.d, m.eps, xs, red);
-    EpiSwiGLU epi{m.a};
-    flat_gemv<2, false, kUnroll>(W, m.d, m.F, xs, warp, nwarps, m.gemv_part, m.gemv_ticket, epi);
+    if (!coop_stream(W, r, buf, xs, sm_part)) {
+        flag_error(m.ctl, kErrShape);
+        return;
+    }
+    const EpiSwiGLU epi{m.a, m.F};
+    coop_finish(r, sm_part, m.gemv_part, 0, m.gemv_ticket, epi);
 }
 
 // Gated feed-forward down with the residual add: h += W_d a.
-__global__ void __launch_bounds__(kGemvThreads) k_down(DevModel m, int layer) {
+__global__ void __launch_bounds__(kGemvThreads, 2) k_down(DevModel m, int layer) {
     extern __shared__ float4 smem_f4[];
     float* xs = reinterpret_cast<float*>(smem_f4);
-    const uint16_t* W = layer_base(m, layer) + m.off_wd;
-    int warp, nwarps;
-    global_warp(warp, nwarps);
-    prefetch_slice<1, false>(W, m.F, m.d, warp, nwarps);
+    float* sm_part = sm_partials(xs, m.F);
+    const uint4* W = reinterpret_cast<const uint4*>(layer_base(m, layer) + m.off_wd);
+    const CoopRange r = coop_range(tiles_of(m.d), m.F, blockIdx.x, gridDim.x);
+    uint4 buf[kWindow];
+    coop_prefetch(W, r, buf);
+    zero_sm_part(sm_part);
     pdl_wait();
     pdl_launch_dependents();
     for (int i = threadIdx.x; i < m.F; i += blockDim.x) xs[i] = m.a[i];
     __syncthreads();
-    EpiAddH epi{m.h};
-    flat_gemv<1, false, kUnroll>(W, m.F, m.d, xs, warp, nwarps, m.gemv_part, m.gemv_ticket, epi);
+    if (!coop_stream(W, r, buf, xs, sm_part)) {
+        flag_error(m.ctl, kErrShape);
+        return;
+    }
+    const EpiAddH epi{m.h, m.d};
+    coop_finish(r, sm_part, m.gemv_part, 0, m.gemv_ticket, epi);
 }
 
 // Readout affine map r: y_r = W_r h + b_r; also keeps h_k for debug.
-__global__ void __launch_bounds__(kGemvThreads) k_readout(DevModel m, int r) {
+__global__ void __launch_bounds__(kGemvThreads, 2) k_readout(DevModel m, int r) {
     extern __shared__ float4 smem_f4[];
     float* xs = reinterpret_cast<float*>(smem_f4);
-    const uint16_t* W = m.ro_w[r];
-    int warp, nwarps;
-    global_warp(warp, nwarps);
-    prefetch_slice<1, false>(W, m.d, m.d, warp, nwarps);
+    float* sm_part = sm_partials(xs, m.d);
+    const uint4* W = reinterpret_cast<const uint4*>(m.ro_w[r]);
+    const CoopRange rg = coop_range(tiles_of(m.d), m.d, blockIdx.x, gridDim.x);
+    uint4 buf[kWindow];
+    coop_prefetch(W, rg, buf);
+    zero_sm_part(sm_part);
     pdl_wait();
     pdl_launch_dependents();
     for (int i = threadIdx.x; i < m.d; i += blockDim.x) {
@@ -515,35 +687,27 @@ __global__ void __launch_bounds__(kGemvThreads) k_readout(DevModel m, int r) {
         if (blockIdx.x == 0) m.hk[(int64_t)r * m.d + i] = v;
     }
     __syncthreads();
-    EpiBias epi{m.y + (int64_t)r * m.d, m.ro_b[r]};
-    flat_gemv<1, false, kUnroll>(W, m.d, m.d, xs, warp, nwarps, m.gemv_part, m.gemv_ticket, epi);
+    if (!coop_stream(W, rg, buf, xs, sm_part)) {
+        flag_error(m.ctl, kErrShape);
+        return;
+    }
+    const EpiBias epi{m.y + (int64_t)r * m.d, m.ro_b[r], m.d};
+    coop_finish(rg, sm_part, m.gemv_part, 0, m.gemv_ticket, epi);
 }
 
-// One pass over the unembedding: z = RMSNorm(x) * gain, l = U z, then
-// max, sum of exp and lowest argmax; the last CTA to finish turns them into
-// the top-1 probability p = 1 / sum exp(l - max) and, for a readout, the gate
-// decision p > tau (which also selects the graph's branch).
-__global__ void __launch_bounds__(kGemvThreads) k_vocab(VocabArgs v) {
-    extern __shared__ float4 smem_f4[];
-    float* xs = reinterpret_cast<float*>(smem_f4);
-    __shared__ float red[32];
+// After the vocabulary pass: merge the per-lane statistics of the CTA, then
+// (last CTA) of the grid, turn them into p = 1 / sum exp(l - max) and, for a
+// readout, the gate decision p > tau, which also selects the graph's branch.
+__device__ __forceinline__ void vocab_finish(const VocabArgs& v, LaneStats st) {
     __shared__ float sm_m[32], sm_s[32];
     __shared__ int sm_a[32];
     __shared__ int is_last;
-    int warp, nwarps;
-    global_warp(warp, nwarps);
-    prefetch_slice<1, true>(v.U, v.d, v.V, warp, nwarps);
-    pdl_wait();
-    pdl_launch_dependents();
-    rmsnorm_to_smem(v.x, v.gain, v.d, v.eps, xs, red);
-    const bool keep = v.logits && (!v.logits_if_dbg || (v.ctl && v.ctl->dbg));
-    EpiVocab epi{keep ? v.logits : nullptr, -CUDART_INF_F, 0.f, 0x7fffffff};
-    flat_gemv<1, true, kUnroll>(v.U, v.d, v.V, xs, warp, nwarps, nullptr, nullptr, epi);
     const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+    warp_merge_stats(st.m, st.s, st.a);
     if (lane == 0) {
-        sm_m[w] = epi.m;
-        sm_s[w] = epi.s;
-        sm_a[w] = epi.a;
+        sm_m[w] = st.m;
+        sm_s[w] = st.s;
+        sm_a[w] = st.a;
     }
     __syncthreads();
     if (w == 0) {
@@ -599,6 +763,85 @@ __global__ void __launch_bounds__(kGemvThreads) k_vocab(VocabArgs v) {
         c->full_conf = p;
         c->exit_readout = -1;
     }
+}
+
+// One pass over the (tiled) unembedding: z = RMSNorm(x) * gain, l = U z,
+// with max, sum of exp and lowest argmax.  Each warp owns a run of whole
+// tiles (no cross-warp combine), lane r the rows r, r + 32, ...
+__global__ void __launch_bounds__(kGemvThreads, 2) k_vocab(VocabArgs v) {
+    extern __shared__ float4 smem_f4[];
+    float* xs = reinterpret_cast<float*>(smem_f4);
+    __shared__ float red[32];
+    const int lane = threadIdx.x & 31;
+    int warp, nwarps;
+    global_warp(warp, nwarps);
+    const int Rc = v.d >> 3;
+    const int64_t n_tiles = (v.V + 31) / 32;
+    const int64_t t0 = n_tiles * warp / nwarps, t1 = n_tiles * (warp + 1) / nwarps;
+    const int64_t i0 = t0 * Rc, i1 = t1 * Rc;
+    const uint4* W = reinterpret_cast<const uint4*>(v.U);
+    uint4 buf[kWindow];
+#pragma unroll
+    for (int u = 0; u < kWindow; ++u)
+        buf[u] = i0 + u < i1 ? ldg_stream(W + (i0 + u) * 32 + lane) : make_uint4(0u, 0u, 0u, 0u);
+    pdl_wait();
+    pdl_launch_dependents();
+    rmsnorm_to_smem(v.x, v.gain, v.d, v.eps, xs, red);
+    const bool keep = v.logits && (!v.logits_if_dbg || (v.ctl && v.ctl->dbg));
+    LaneStats st;
+    int64_t t = t0;
+    int c = 0;
+    float acc = 0.f;
+    for (int64_t base = i0; base < i1; base += kWindow) {
+        if (base != i0) {
+#pragma unroll
+            for (int u = 0; u < kWindow; ++u)
+                buf[u] = base + u < i1 ? ldg_stream(W + (base + u) * 32 + lane) : make_uint4(0u, 0u, 0u, 0u);
+        }
+#pragma unroll
+        for (int u = 0; u < kWindow; ++u) {
+            if (base + u >= i1) break;
+            acc += dot8(buf[u], xs + c * 8);
+            if (++c == Rc) {
+                const int64_t row = t * 32 + lane;
+                if (row < v.V) {
+                    if (keep) v.logits[row] = acc;
+                    st.add(acc, (int)row);
+                }
+                acc = 0.f;
+                c = 0;
+                ++t;
+            }
+        }
+    }
+    vocab_finish(v, st);
+}
+
+// The same pass over a row-major [V, d] matrix (standalone op): the flat
+// streaming core, one warp per run of whole rows.
+struct EpiVocabRowMajor {
+    float* logits;
+    LaneStats st;
+    __device__ __forceinline__ void operator()(int64_t u, const float* r) {
+        if (logits) logits[u] = r[0];
+        st.add(r[0], (int)u);
+    }
+};
+
+__global__ void __launch_bounds__(kGemvThreads, 2) k_vocab_rowmajor(VocabArgs v) {
+    extern __shared__ float4 smem_f4[];
+    float* xs = reinterpret_cast<float*>(smem_f4);
+    __shared__ float red[32];
+    int warp, nwarps;
+    global_warp(warp, nwarps);
+    pdl_wait();
+    pdl_launch_dependents();
+    rmsnorm_to_smem(v.x, v.gain, v.d, v.eps, xs, red);
+    EpiVocabRowMajor epi{v.logits, LaneStats()};
+    flat_gemv<1, true, 8>(v.U, v.d, v.V, xs, warp, nwarps, nullptr, nullptr, epi);
+    // lane 0 holds this warp's statistics; the others hold none
+    LaneStats st = (threadIdx.x & 31) == 0 ? epi.st : LaneStats();
+    vocab_finish(v, st);
 }
 
 // Split-K decode attention over the paged cache.  Grid (splits, KH): CTA
@@ -847,7 +1090,9 @@ static cudaError_t launch_k(void (*kern)(KArgs...), dim3 grid, dim3 block, size_
 
 static size_t g_smem = 0;
 
-size_t gemv_smem_bytes(int kmax) { return (size_t)kmax * sizeof(float); }
+size_t gemv_smem_bytes(int kmax) {
+    return ((size_t)((kmax + 3) & ~3) * 2 + (size_t)kSlotTiles * kWarps * 32) * sizeof(float);
+}
 
 cudaError_t configure_kernels(int kmax) {
     if (gemv_smem_bytes(kmax) > g_smem) g_smem = gemv_smem_bytes(kmax);
@@ -860,13 +1105,17 @@ cudaError_t configure_kernels(int kmax) {
     if ((e = cudaFuncSetAttribute(k_down, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes))) return e;
     if ((e = cudaFuncSetAttribute(k_readout, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes))) return e;
     if ((e = cudaFuncSetAttribute(k_vocab, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes))) return e;
+    if ((e = cudaFuncSetAttribute(k_vocab_rowmajor, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes))) return e;
     return cudaSuccess;
 }
 
-static size_t smem_for(int k) { return (size_t)k * sizeof(float); }
+// x (K floats, padded to 16 bytes) + tile partials [+ the first layer's embedding row].
+static size_t smem_for(int k, int extra = 0) {
+    return ((size_t)((k + 3) & ~3) + (size_t)kSlotTiles * kWarps * 32 + (size_t)extra) * sizeof(float);
+}
 
 cudaError_t launch_qkv(const DevModel& m, int layer, int first, int grid, bool pdl, cudaStream_t s) {
-    return launch_k(k_qkv, dim3(grid), dim3(kGemvThreads), smem_for(2 * m.d), pdl, s, m, layer, first);
+    return launch_k(k_qkv, dim3(grid), dim3(kGemvThreads), smem_for(m.d, m.d), pdl, s, m, layer, first);
 }
 cudaError_t launch_kvfill(const DevModel& m, int exit_layer, int grid_x, bool pdl, cudaStream_t s) {
     return launch_k(k_kvfill, dim3(grid_x, m.L - exit_layer), dim3(kGemvThreads), smem_for(m.d), pdl, s, m,
@@ -885,7 +1134,9 @@ cudaError_t launch_readout(const DevModel& m, int r, int grid, bool pdl, cudaStr
     return launch_k(k_readout, dim3(grid), dim3(kGemvThreads), smem_for(m.d), pdl, s, m, r);
 }
 cudaError_t launch_vocab(const VocabArgs& v, int grid, bool pdl, cudaStream_t s) {
-    return launch_k(k_vocab, dim3(grid), dim3(kGemvThreads), smem_for(v.d), pdl, s, v);
+    const size_t smem = (size_t)((v.d + 3) & ~3) * sizeof(float);
+    if (v.tiled) return launch_k(k_vocab, dim3(grid), dim3(kGemvThreads), smem, pdl, s, v);
+    return launch_k(k_vocab_rowmajor, dim3(grid), dim3(kGemvThreads), smem, pdl, s, v);
 }
 cudaError_t launch_attention(const AttnArgs& a, int head_dim, bool pdl, cudaStream_t s) {
     const dim3 grid(kAttnMaxSplits, a.KH);
