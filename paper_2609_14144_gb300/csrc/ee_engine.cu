@@ -209,6 +209,7 @@ struct ee_ctx {
     int dbg = 0;
     cudaGraphExec_t g_step = nullptr, g_n = nullptr, g_prefill = nullptr;
     int grid_gemv = 0, grid_vocab = 0;
+    int attn_cluster = 8;  // CTAs per key-value head in the attention kernel
 };
 
 namespace {
@@ -221,11 +222,17 @@ void drop_graphs(ee_ctx* c) {
         }
 }
 
-// Grid of a tiled GEMV launch over `rows` rows of length K: one CTA per SM,
-// fewer when each warp would get less than one 512-byte item, but enough that
-// no CTA touches more than kGemvSlotTiles tiles.
+// Matrices whose tiles are at most this many bytes, and that have no more
+// tiles than the GEMV grid, run one CTA per tile: no cross-CTA combine.
+constexpr int64_t kWholeTileBytes = 192 * 1024;
+
+// Grid of a tiled GEMV launch over `rows` rows of length K: two CTAs per SM,
+// or one per tile for small matrices, fewer when each warp would get less
+// than one 512-byte item, but enough that no CTA touches more than
+// kGemvSlotTiles tiles.
 int gemv_grid(const ee_ctx* c, int64_t rows, int64_t K) {
     const int64_t tiles = tile_count(rows), items = tiles * (K / 8);
+    if (tiles <= c->grid_gemv && 2 * kTileRows * K <= kWholeTileBytes) return (int)tiles;
     int64_t g = std::min<int64_t>(c->grid_gemv, std::max<int64_t>(1, items / (kGemvThreads / 32)));
     const int64_t need = (tiles + kGemvSlotTiles - 3) / (kGemvSlotTiles - 2);
     return (int)std::max<int64_t>(g, need);
@@ -283,7 +290,7 @@ int enqueue_layers(ee_ctx* c, cudaStream_t s, int j0, int j1, bool& pdl) {
     for (int j = j0; j < j1; ++j) {
         EE_CK(launch_qkv(m, j, j == 0 ? 1 : 0, gq, pdl, s));
         pdl = c->use_pdl;
-        EE_CK(launch_attention(attn_args(c, j), m.D, pdl, s));
+        EE_CK(launch_attention_cluster(attn_args(c, j), m.D, c->attn_cluster, pdl, s));
         EE_CK(launch_oproj(m, j, go, pdl, s));
         EE_CK(launch_gateup(m, j, gu, pdl, s));
         EE_CK(launch_down(m, j, gd, pdl, s));
@@ -593,6 +600,7 @@ int ee_create(const ee_model_config* cfg, void* d_workspace, size_t workspace_by
     cudaDeviceGetAttribute(&c->n_sm, cudaDevAttrMultiProcessorCount, c->device);
     c->grid_gemv = std::min(2 * c->n_sm, kMaxGemvCtas);  // two 512-thread CTAs per SM
     c->grid_vocab = std::min(2 * c->n_sm, kMaxVocabCtas);
+    c->attn_cluster = cfg->max_ctx > 4096 ? 16 : 8;
     if (d_workspace) {
         if (workspace_bytes < c->lay.total) return bail(fail(EE_ENOMEM, "workspace too small"));
         c->ws = (char*)d_workspace;
@@ -1076,7 +1084,7 @@ int ee_profile_kernels(ee_ctx* c, int iters, float* ms_out) {
             const int j = i % L;
             switch (k) {
                 case EE_KERNEL_QKV: return launch_qkv(m, j, 0, gq, false, s);
-                case EE_KERNEL_ATTN: return launch_attention(attn_args(c, j), m.D, false, s);
+                case EE_KERNEL_ATTN: return launch_attention_cluster(attn_args(c, j), m.D, c->attn_cluster, false, s);
                 case EE_KERNEL_OPROJ: return launch_oproj(m, j, go, false, s);
                 case EE_KERNEL_GATEUP: return launch_gateup(m, j, gu, false, s);
                 case EE_KERNEL_DOWN: return launch_down(m, j, gd, false, s);

@@ -143,6 +143,8 @@ struct CtlInputs {
 // `pdl` adds the programmatic-stream-serialisation attribute.
 cudaError_t launch_qkv(const DevModel& m, int layer, int first, int grid, bool pdl, cudaStream_t s);
 cudaError_t launch_attention(const AttnArgs& a, int head_dim, bool pdl, cudaStream_t s);
+// The engine's attention: one thread-block cluster of `cluster` CTAs per kv head.
+cudaError_t launch_attention_cluster(const AttnArgs& a, int head_dim, int cluster, bool pdl, cudaStream_t s);
 cudaError_t launch_oproj(const DevModel& m, int layer, int grid, bool pdl, cudaStream_t s);
 cudaError_t launch_gateup(const DevModel& m, int layer, int grid, bool pdl, cudaStream_t s);
 cudaError_t launch_down(const DevModel& m, int layer, int grid, bool pdl, cudaStream_t s);

@@ -17,6 +17,7 @@
 // per lane; a warp reduction closes each row.  Units cut by a slice boundary
 // are finished by whichever contributing warp arrives last, summing the
 // contributions in warp order, so results do not depend on timing.
+#include <cooperative_groups.h>
 #include <cuda_bf16.h>
 #include <math.h>
 #include <math_constants.h>
@@ -998,6 +999,164 @@ __global__ void __launch_bounds__(kAttnThreads) k_attention(AttnArgs a) {
     if (threadIdx.x == 0) a.ticket[g] = 0;
 }
 
+// Decode attention of one layer on a thread-block cluster per key-value head
+// (grid (CL, KH), cluster (CL, 1, 1)).  Rank r covers a contiguous run of
+// positions for all A/K query heads of head g with a per-lane online softmax;
+// the 8 warps merge in shared memory, and the CL ranks merge through
+// distributed shared memory, each rank finishing a share of the outputs:
+// o = softmax(q K^T / sqrt(D)) V (fp32).  Before waiting on the QKV kernel,
+// each CTA pulls its past K/V rows into L2 (only position T-1 is new).
+namespace cg = cooperative_groups;
+
+template <int D>
+__global__ void __launch_bounds__(kAttnThreads) k_attn_cluster(AttnArgs a) {
+    constexpr int LPR = D / 8;
+    constexpr int RPW = 32 / LPR;
+    constexpr int NW = kAttnThreads / 32;
+    constexpr int GMAX = 8;
+    __shared__ __align__(16) float qs[GMAX * D];
+    __shared__ float wm[NW][GMAX], wl[NW][GMAX];
+    __shared__ __align__(16) float wacc[NW][GMAX][D];
+    __shared__ float cm[GMAX], cl[GMAX];
+    cg::cluster_group cluster = cg::this_cluster();
+    const int rank = (int)cluster.block_rank(), CL = (int)cluster.num_blocks();
+    const int g = blockIdx.y, G = a.A / a.KH, P = a.page_size;
+    const int T = a.ctl->pos + 1;
+    const int chunk = (T + CL - 1) / CL;
+    const int t0 = min(T, rank * chunk), t1 = min(T, t0 + chunk);
+    if (threadIdx.x == 0) {
+        const int te = min(t1, T - 1);
+        for (int t = t0; t < te;) {
+            const int page = a.page_table[t / P], slot = t % P, n = min(te - t, P - slot);
+            const int64_t off = (((int64_t)page * a.KH + g) * P + slot) * D;
+            prefetch_l2(a.kp + off, (uint32_t)(n * D * 2));
+            prefetch_l2(a.vp + off, (uint32_t)(n * D * 2));
+            t += n;
+        }
+    }
+    pdl_wait();
+    pdl_launch_dependents();
+    const float scale = 1.0f / sqrtf((float)D);
+    for (int i = threadIdx.x; i < G * D; i += blockDim.x) qs[i] = a.q[(int64_t)g * G * D + i] * scale;
+    __syncthreads();
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int grp = lane / LPR, e0 = (lane % LPR) * 8;
+    float mx[GMAX], ls[GMAX], acc[GMAX][8];
+#pragma unroll
+    for (int h = 0; h < GMAX; ++h) {
+        mx[h] = -CUDART_INF_F;
+        ls[h] = 0.f;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) acc[h][e] = 0.f;
+    }
+    for (int tt = t0 + warp * RPW; tt < t1; tt += NW * RPW) {
+        const int t = tt + grp;
+        const bool valid = t < t1;
+        float kf[8], vf[8];
+        if (valid) {
+            const int page = a.page_table[t / P];
+            const int64_t off = (((int64_t)page * a.KH + g) * P + (t % P)) * D + e0;
+            const uint4 kw = *reinterpret_cast<const uint4*>(a.kp + off);
+            const uint4 vw = *reinterpret_cast<const uint4*>(a.vp + off);
+            kf[0] = bf_lo(kw.x); kf[1] = bf_hi(kw.x); kf[2] = bf_lo(kw.y); kf[3] = bf_hi(kw.y);
+            kf[4] = bf_lo(kw.z); kf[5] = bf_hi(kw.z); kf[6] = bf_lo(kw.w); kf[7] = bf_hi(kw.w);
+            vf[0] = bf_lo(vw.x); vf[1] = bf_hi(vw.x); vf[2] = bf_lo(vw.y); vf[3] = bf_hi(vw.y);
+            vf[4] = bf_lo(vw.z); vf[5] = bf_hi(vw.z); vf[6] = bf_lo(vw.w); vf[7] = bf_hi(vw.w);
+        } else {
+#pragma unroll
+            for (int e = 0; e < 8; ++e) kf[e] = vf[e] = 0.f;
+        }
+#pragma unroll
+        for (int h = 0; h < GMAX; ++h) {
+            if (h >= G) break;
+            float d = 0.f;
+#pragma unroll
+            for (int e = 0; e < 8; ++e) d = fmaf(kf[e], qs[h * D + e0 + e], d);
+#pragma unroll
+            for (int o = LPR / 2; o; o >>= 1) d += __shfl_xor_sync(0xffffffffu, d, o);
+            if (valid) {
+                const float mn = fmaxf(mx[h], d);
+                const float corr = expf(mx[h] - mn);
+                const float p = expf(d - mn);
+                ls[h] = ls[h] * corr + p;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) acc[h][e] = fmaf(p, vf[e], acc[h][e] * corr);
+                mx[h] = mn;
+            }
+        }
+    }
+#pragma unroll
+    for (int o = LPR; o < 32; o <<= 1) {
+#pragma unroll
+        for (int h = 0; h < GMAX; ++h) {
+            if (h >= G) break;
+            const float m2 = __shfl_xor_sync(0xffffffffu, mx[h], o);
+            const float l2 = __shfl_xor_sync(0xffffffffu, ls[h], o);
+            float a2[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) a2[e] = __shfl_xor_sync(0xffffffffu, acc[h][e], o);
+            const float M = fmaxf(mx[h], m2);
+            if (M != -CUDART_INF_F) {
+                const float c1 = expf(mx[h] - M), c2 = expf(m2 - M);
+                ls[h] = ls[h] * c1 + l2 * c2;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) acc[h][e] = acc[h][e] * c1 + a2[e] * c2;
+                mx[h] = M;
+            }
+        }
+    }
+    if (grp == 0) {
+#pragma unroll
+        for (int h = 0; h < GMAX; ++h) {
+            if (h >= G) break;
+            if (lane == 0) {
+                wm[warp][h] = mx[h];
+                wl[warp][h] = ls[h];
+            }
+#pragma unroll
+            for (int e = 0; e < 8; ++e) wacc[warp][h][e0 + e] = acc[h][e];
+        }
+    }
+    __syncthreads();
+    // this CTA's partial: (cm, cl) per head, accumulator in wacc[0]
+    for (int i = threadIdx.x; i < G * D; i += blockDim.x) {
+        const int h = i / D, e = i - h * D;
+        float M = -CUDART_INF_F, L = 0.f, O = 0.f;
+        for (int w = 0; w < NW; ++w) {
+            const float m2 = wm[w][h];
+            const float Mn = fmaxf(M, m2);
+            if (Mn == -CUDART_INF_F) continue;
+            const float c1 = expf(M - Mn), c2 = expf(m2 - Mn);
+            L = L * c1 + wl[w][h] * c2;
+            O = O * c1 + wacc[w][h][e] * c2;
+            M = Mn;
+        }
+        wacc[0][h][e] = O;
+        if (e == 0) {
+            cm[h] = M;
+            cl[h] = L;
+        }
+    }
+    cluster.sync();
+    // merge the ranks' partials; rank r finishes outputs r*blockDim.x + tid, ...
+    for (int i = rank * blockDim.x + threadIdx.x; i < G * D; i += CL * blockDim.x) {
+        const int h = i / D, e = i - h * D;
+        float M = -CUDART_INF_F;
+        for (int r = 0; r < CL; ++r) M = fmaxf(M, cluster.map_shared_rank(cm, r)[h]);
+        float L = 0.f, O = 0.f;
+        for (int r = 0; r < CL; ++r) {
+            const float mr = cluster.map_shared_rank(cm, r)[h];
+            if (mr == -CUDART_INF_F) continue;
+            const float c = expf(mr - M);
+            L = fmaf(cluster.map_shared_rank(cl, r)[h], c, L);
+            O = fmaf(cluster.map_shared_rank(&wacc[0][0][0], r)[h * D + e], c, O);
+        }
+        a.out[(int64_t)(g * G + h) * D + e] = O / L;
+    }
+    cluster.sync();  // keep every rank's shared memory alive until all have read it
+}
+
 // End of a decode step: emit, record, count, advance, feed the token back.
 __global__ void k_step_end(DevModel m, int has_cond, cudaGraphConditionalHandle cond) {
     pdl_wait();
@@ -1106,6 +1265,8 @@ cudaError_t configure_kernels(int kmax) {
     if ((e = cudaFuncSetAttribute(k_readout, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes))) return e;
     if ((e = cudaFuncSetAttribute(k_vocab, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes))) return e;
     if ((e = cudaFuncSetAttribute(k_vocab_rowmajor, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes))) return e;
+    if ((e = cudaFuncSetAttribute(k_attn_cluster<64>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1))) return e;
+    if ((e = cudaFuncSetAttribute(k_attn_cluster<128>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1))) return e;
     return cudaSuccess;
 }
 
@@ -1142,6 +1303,25 @@ cudaError_t launch_attention(const AttnArgs& a, int head_dim, bool pdl, cudaStre
     const dim3 grid(kAttnMaxSplits, a.KH);
     if (head_dim == 64) return launch_k(k_attention<64>, grid, dim3(kAttnThreads), 0, pdl, s, a);
     if (head_dim == 128) return launch_k(k_attention<128>, grid, dim3(kAttnThreads), 0, pdl, s, a);
+    return cudaErrorInvalidValue;
+}
+cudaError_t launch_attention_cluster(const AttnArgs& a, int head_dim, int cluster, bool pdl, cudaStream_t s) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(cluster, a.KH);
+    cfg.blockDim = dim3(kAttnThreads);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = cluster;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl ? 2 : 1;
+    if (head_dim == 64) return cudaLaunchKernelEx(&cfg, k_attn_cluster<64>, a);
+    if (head_dim == 128) return cudaLaunchKernelEx(&cfg, k_attn_cluster<128>, a);
     return cudaErrorInvalidValue;
 }
 cudaError_t launch_step_end(const DevModel& m, int has_cond, cudaGraphConditionalHandle cond, bool pdl,
