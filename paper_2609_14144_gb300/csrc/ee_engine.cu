@@ -223,8 +223,13 @@ void drop_graphs(ee_ctx* c) {
 }
 
 // Matrices whose tiles are at most this many bytes, and that have no more
-// tiles than the GEMV grid, run one CTA per tile: no cross-CTA combine.
-constexpr int64_t kWholeTileBytes = 192 * 1024;
+// tiles than the GEMV grid, run one CTA per tile with the tile staged in
+// shared memory before the kernel waits on its predecessor.
+constexpr int64_t kWholeTileBytes = 144 * 1024;
+
+bool gemv_whole(const ee_ctx* c, int64_t rows, int64_t K) {
+    return tile_count(rows) <= c->grid_gemv && 2 * kTileRows * K <= kWholeTileBytes;
+}
 
 // Grid of a tiled GEMV launch over `rows` rows of length K: two CTAs per SM,
 // or one per tile for small matrices, fewer when each warp would get less
@@ -232,7 +237,7 @@ constexpr int64_t kWholeTileBytes = 192 * 1024;
 // kGemvSlotTiles tiles.
 int gemv_grid(const ee_ctx* c, int64_t rows, int64_t K) {
     const int64_t tiles = tile_count(rows), items = tiles * (K / 8);
-    if (tiles <= c->grid_gemv && 2 * kTileRows * K <= kWholeTileBytes) return (int)tiles;
+    if (gemv_whole(c, rows, K)) return (int)tiles;
     int64_t g = std::min<int64_t>(c->grid_gemv, std::max<int64_t>(1, items / (kGemvThreads / 32)));
     const int64_t need = (tiles + kGemvSlotTiles - 3) / (kGemvSlotTiles - 2);
     return (int)std::max<int64_t>(g, need);
@@ -283,24 +288,25 @@ VocabArgs vocab_args(const ee_ctx* c, int mode, int r, int has_cond, cudaGraphCo
 int enqueue_layers(ee_ctx* c, cudaStream_t s, int j0, int j1, bool& pdl) {
     const DevModel& m = c->dm;
     const int64_t d = m.d, F = m.F, AD = (int64_t)m.A * m.D;
-    const int gq = gemv_grid(c, c->lay.n_units_qkv * 2, d);
-    const int go = gemv_grid(c, d, AD);
-    const int gu = gemv_grid(c, 2 * F, d);
-    const int gd = gemv_grid(c, d, F);
+    const int64_t nqkv = c->lay.n_units_qkv * 2;
+    const int gq = gemv_grid(c, nqkv, d), go = gemv_grid(c, d, AD), gu = gemv_grid(c, 2 * F, d),
+              gd = gemv_grid(c, d, F);
+    const bool wq = gemv_whole(c, nqkv, d), wo = gemv_whole(c, d, AD), wu = gemv_whole(c, 2 * F, d),
+               wd = gemv_whole(c, d, F);
     for (int j = j0; j < j1; ++j) {
-        EE_CK(launch_qkv(m, j, j == 0 ? 1 : 0, gq, pdl, s));
+        EE_CK(launch_qkv(m, j, j == 0 ? 1 : 0, gq, wq, pdl, s));
         pdl = c->use_pdl;
         EE_CK(launch_attention_cluster(attn_args(c, j), m.D, c->attn_cluster, pdl, s));
-        EE_CK(launch_oproj(m, j, go, pdl, s));
-        EE_CK(launch_gateup(m, j, gu, pdl, s));
-        EE_CK(launch_down(m, j, gd, pdl, s));
+        EE_CK(launch_oproj(m, j, go, wo, pdl, s));
+        EE_CK(launch_gateup(m, j, gu, wu, pdl, s));
+        EE_CK(launch_down(m, j, gd, wd, pdl, s));
     }
     return EE_OK;
 }
 
 int enqueue_readout(ee_ctx* c, cudaStream_t s, int r, int has_cond, cudaGraphConditionalHandle cond, bool& pdl) {
     const DevModel& m = c->dm;
-    EE_CK(launch_readout(m, r, gemv_grid(c, m.d, m.d), pdl, s));
+    EE_CK(launch_readout(m, r, gemv_grid(c, m.d, m.d), gemv_whole(c, m.d, m.d), pdl, s));
     pdl = c->use_pdl;
     EE_CK(launch_vocab(vocab_args(c, 1, r, has_cond, cond), c->grid_vocab, pdl, s));
     return EE_OK;
@@ -324,7 +330,9 @@ int enqueue_fill(ee_ctx* c, cudaStream_t s, int exit_layer, bool pdl) {
     const DevModel& m = c->dm;
     if (exit_layer >= m.L) return EE_OK;
     const int nl = m.L - exit_layer;
-    EE_CK(launch_kvfill(m, exit_layer, fill_grid_x(c, nl), pdl, s));
+    const int64_t rows = 2LL * m.KH * m.D;
+    const int gx = fill_grid_x(c, nl);
+    EE_CK(launch_kvfill(m, exit_layer, gx, gx == tile_count(rows) && gemv_whole(c, rows, m.d), pdl, s));
     return EE_OK;
 }
 
@@ -600,7 +608,7 @@ int ee_create(const ee_model_config* cfg, void* d_workspace, size_t workspace_by
     cudaDeviceGetAttribute(&c->n_sm, cudaDevAttrMultiProcessorCount, c->device);
     c->grid_gemv = std::min(2 * c->n_sm, kMaxGemvCtas);  // two 512-thread CTAs per SM
     c->grid_vocab = std::min(2 * c->n_sm, kMaxVocabCtas);
-    c->attn_cluster = cfg->max_ctx > 4096 ? 16 : 8;
+    c->attn_cluster = 0;  // chosen after the kernels are configured
     if (d_workspace) {
         if (workspace_bytes < c->lay.total) return bail(fail(EE_ENOMEM, "workspace too small"));
         c->ws = (char*)d_workspace;
@@ -673,6 +681,7 @@ int ee_create(const ee_model_config* cfg, void* d_workspace, size_t workspace_by
 
     const int kmax = std::max({2 * m.d, m.A * m.D, m.F});
     if (configure_kernels(kmax) != cudaSuccess) return bail(fail(EE_ECUDA, "kernel configuration failed"));
+    c->attn_cluster = attention_cluster_size(m.D, m.KH);
 
     // RoPE table: angle t * base^(-2i/D) in double, cos/sin rounded to fp32.
     std::vector<float2> rope((size_t)m.max_ctx * (m.D / 2));
@@ -1083,17 +1092,20 @@ int ee_profile_kernels(ee_ctx* c, int iters, float* ms_out) {
         auto one = [&](int i) -> cudaError_t {
             const int j = i % L;
             switch (k) {
-                case EE_KERNEL_QKV: return launch_qkv(m, j, 0, gq, false, s);
+                case EE_KERNEL_QKV: return launch_qkv(m, j, 0, gq, gemv_whole(c, c->lay.n_units_qkv * 2, d), false, s);
                 case EE_KERNEL_ATTN: return launch_attention_cluster(attn_args(c, j), m.D, c->attn_cluster, false, s);
-                case EE_KERNEL_OPROJ: return launch_oproj(m, j, go, false, s);
-                case EE_KERNEL_GATEUP: return launch_gateup(m, j, gu, false, s);
-                case EE_KERNEL_DOWN: return launch_down(m, j, gd, false, s);
-                case EE_KERNEL_READOUT: return launch_readout(m, i % c->n_readouts, gr, false, s);
+                case EE_KERNEL_OPROJ: return launch_oproj(m, j, go, gemv_whole(c, d, AD), false, s);
+                case EE_KERNEL_GATEUP: return launch_gateup(m, j, gu, gemv_whole(c, 2 * F, d), false, s);
+                case EE_KERNEL_DOWN: return launch_down(m, j, gd, gemv_whole(c, d, F), false, s);
+                case EE_KERNEL_READOUT:
+                    return launch_readout(m, i % c->n_readouts, gr, gemv_whole(c, d, d), false, s);
                 case EE_KERNEL_VOCAB: return launch_vocab(va, c->grid_vocab, false, s);
                 default: {
                     const int e = c->ro_layer[0];
                     if (e >= L) return cudaSuccess;
-                    return launch_kvfill(m, e, fill_grid_x(c, L - e), false, s);
+                    const int64_t rows = 2LL * m.KH * m.D;
+                    const int gx = fill_grid_x(c, L - e);
+                    return launch_kvfill(m, e, gx, gx == tile_count(rows) && gemv_whole(c, rows, m.d), false, s);
                 }
             }
         };

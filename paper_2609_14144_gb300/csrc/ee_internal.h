@@ -141,16 +141,19 @@ struct CtlInputs {
 
 // Launch helpers (ee_kernels.cu).  Each enqueues one kernel on `s`;
 // `pdl` adds the programmatic-stream-serialisation attribute.
-cudaError_t launch_qkv(const DevModel& m, int layer, int first, int grid, bool pdl, cudaStream_t s);
+// `whole`: one CTA per tile, the tile staged in shared memory before the wait.
+cudaError_t launch_qkv(const DevModel& m, int layer, int first, int grid, bool whole, bool pdl, cudaStream_t s);
 cudaError_t launch_attention(const AttnArgs& a, int head_dim, bool pdl, cudaStream_t s);
 // The engine's attention: one thread-block cluster of `cluster` CTAs per kv head.
 cudaError_t launch_attention_cluster(const AttnArgs& a, int head_dim, int cluster, bool pdl, cudaStream_t s);
-cudaError_t launch_oproj(const DevModel& m, int layer, int grid, bool pdl, cudaStream_t s);
-cudaError_t launch_gateup(const DevModel& m, int layer, int grid, bool pdl, cudaStream_t s);
-cudaError_t launch_down(const DevModel& m, int layer, int grid, bool pdl, cudaStream_t s);
-cudaError_t launch_readout(const DevModel& m, int r, int grid, bool pdl, cudaStream_t s);
+// Largest cluster size (16 or 8) the attention kernel can be resident with.
+int attention_cluster_size(int head_dim, int n_kv_heads);
+cudaError_t launch_oproj(const DevModel& m, int layer, int grid, bool whole, bool pdl, cudaStream_t s);
+cudaError_t launch_gateup(const DevModel& m, int layer, int grid, bool whole, bool pdl, cudaStream_t s);
+cudaError_t launch_down(const DevModel& m, int layer, int grid, bool whole, bool pdl, cudaStream_t s);
+cudaError_t launch_readout(const DevModel& m, int r, int grid, bool whole, bool pdl, cudaStream_t s);
 cudaError_t launch_vocab(const VocabArgs& v, int grid, bool pdl, cudaStream_t s);
-cudaError_t launch_kvfill(const DevModel& m, int exit_layer, int grid_x, bool pdl, cudaStream_t s);
+cudaError_t launch_kvfill(const DevModel& m, int exit_layer, int grid_x, bool whole, bool pdl, cudaStream_t s);
 cudaError_t launch_step_end(const DevModel& m, int has_cond, cudaGraphConditionalHandle cond, bool pdl,
                             cudaStream_t s);
 cudaError_t launch_prefill_advance(const DevModel& m, int has_cond, cudaGraphConditionalHandle cond, bool pdl,
@@ -168,6 +171,7 @@ cudaError_t configure_kernels(int kmax);
 // Geometry of the tiled weight layout (rows grouped by 32, see ee_kernels.cu).
 constexpr int kTileRows = 32;
 constexpr int kGemvSlotTiles = 8;   // tiles one GEMV CTA may touch
+constexpr int kGemvMaxSmem = 227 * 1024;  // dynamic shared memory a GEMV CTA may use
 inline int64_t tile_count(int64_t rows) { return (rows + kTileRows - 1) / kTileRows; }
 inline int64_t tiled_elems(int64_t rows, int64_t K) { return tile_count(rows) * kTileRows * K; }
 

@@ -209,6 +209,30 @@ __device__ __forceinline__ void flat_gemv(const uint16_t* __restrict__ W, int K,
     if (row * Rc < c1) finish_row(row, warp_sum(acc));
 }
 
+__device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"((uint32_t)__cvta_generic_to_shared(smem)),
+                 "l"(gmem)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
+
+// Distributed shared memory: the address of a shared-memory location in the
+// CTA of cluster rank `rank`, and a load from it.
+__device__ __forceinline__ uint32_t dsmem_rank(uint32_t smem_addr, uint32_t rank) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_addr), "r"(rank));
+    return r;
+}
+__device__ __forceinline__ uint32_t dsmem_addr(const void* p, uint32_t rank) {
+    return dsmem_rank((uint32_t)__cvta_generic_to_shared(p), rank);
+}
+__device__ __forceinline__ float ld_dsmem(uint32_t addr) {
+    float v;
+    asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(addr) : "memory");
+    return v;
+}
+
 // ------------------------------------------------------------------ tiled GEMV
 //
 // Engine weights are repacked into tiles of 32 rows: for each 16-byte column
@@ -348,6 +372,67 @@ __device__ __forceinline__ void coop_finish(const CoopRange& r, const float* __r
 // touch every tile of its CTA).
 __device__ __forceinline__ void zero_sm_part(float* sm_part) {
     for (int i = threadIdx.x; i < kSlotTiles * kWarps * 32; i += blockDim.x) sm_part[i] = 0.f;
+}
+
+// Whole-tile mode (one CTA per tile, small matrices): the CTA's tile is
+// copied into shared memory with cp.async before the kernel waits on its
+// predecessor, so after the wait only the activation vector is fetched.
+// The streaming mode (coop_prefetch / coop_stream) serves the rest.
+template <bool WHOLE>
+struct GemvFront {
+    CoopRange r;
+    uint4 buf[kWindow];
+    __device__ __forceinline__ void begin(const uint4* W, int64_t n_tiles, int K, uint4* tile_sm) {
+        if (WHOLE) {
+            r.Rc = K >> 3;
+            r.Ct = (int)(n_tiles * r.Rc);
+            r.C0 = blockIdx.x * r.Rc;
+            r.C1 = r.C0 + r.Rc;
+            r.cta = blockIdx.x;
+            r.n_cta = gridDim.x;
+            const uint4* src = W + (int64_t)r.C0 * 32;
+            for (int i = threadIdx.x; i < r.Rc * 32; i += blockDim.x) cp_async16(tile_sm + i, src + i);
+            cp_async_commit();
+        } else {
+            r = coop_range(n_tiles, K, blockIdx.x, gridDim.x);
+            coop_prefetch(W, r, buf);
+        }
+    }
+    // Leaves each warp's share of the CTA's tiles in sm_part and synchronises.
+    __device__ __forceinline__ bool stream(const uint4* W, const float* xs, float* sm_part, const uint4* tile_sm) {
+        if (!WHOLE) return coop_stream(W, r, buf, xs, sm_part);
+        const int lane = threadIdx.x & 31, wl = threadIdx.x >> 5;
+        cp_async_wait_all();
+        __syncthreads();
+        float acc = 0.f;
+        for (int it = wl; it < r.Rc; it += kWarps) acc += dot8(tile_sm[it * 32 + lane], xs + it * 8);
+        sm_part[wl * 32 + lane] = acc;
+        __syncthreads();
+        return true;
+    }
+    // Columns [lo, hi) of x this CTA multiplies (all of them when the range
+    // wraps or covers a whole row).
+    __device__ __forceinline__ void x_range(int K, int& lo, int& hi) const {
+        if (WHOLE || r.C1 - r.C0 >= r.Rc) {
+            lo = 0;
+            hi = K;
+            return;
+        }
+        const int a = r.C0 % r.Rc, b = (r.C1 - 1) % r.Rc;
+        if (a <= b) {
+            lo = a * 8;
+            hi = b * 8 + 8;
+        } else {
+            lo = 0;
+            hi = K;
+        }
+    }
+};
+
+// Shared-memory pointer of the staged tile: after x, the tile partials and
+// `extra` floats.
+__device__ __forceinline__ uint4* sm_tile(float* xs, int K, int extra) {
+    return reinterpret_cast<uint4*>(xs + ((K + 3) & ~3) + kSlotTiles * kWarps * 32 + extra);
 }
 
 // ------------------------------------------------------------------ epilogues
@@ -513,18 +598,20 @@ __device__ __forceinline__ float* sm_partials(float* xs, int K) { return xs + ((
 
 // Attention input of layer j: [embedding gather,] RMSNorm, Q/K/V GEMV, RoPE,
 // KV append at the step's position.
+template <bool WHOLE>
 __global__ void __launch_bounds__(kGemvThreads, 2) k_qkv(DevModel m, int layer, int first) {
     extern __shared__ float4 smem_f4[];
     float* xs = reinterpret_cast<float*>(smem_f4);
     float* sm_part = sm_partials(xs, m.d);
+    uint4* tile_sm = sm_tile(xs, m.d, m.d);
     __shared__ float red[32];
     const uint16_t* lw = layer_base(m, layer);
     const uint4* W = reinterpret_cast<const uint4*>(lw + m.off_wqkv);
     const int64_t nq = (int64_t)m.A * m.D / 2, nk = (int64_t)m.KH * m.D / 2;
-    const CoopRange r = coop_range((nq + 2 * nk) / 16, m.d, blockIdx.x, gridDim.x);
-    uint4 buf[kWindow];
-    coop_prefetch(W, r, buf);
-    zero_sm_part(sm_part);
+    GemvFront<WHOLE> fr;
+    fr.begin(W, (nq + 2 * nk) / 16, m.d, tile_sm);
+    const CoopRange& r = fr.r;
+    if (!WHOLE) zero_sm_part(sm_part);
     pdl_wait();
     pdl_launch_dependents();
     Ctl* c = m.ctl;
@@ -554,10 +641,11 @@ __global__ void __launch_bounds__(kGemvThreads, 2) k_qkv(DevModel m, int layer, 
     }
     if (!pos_ok) {
         if (blockIdx.x == 0) flag_error(c, kErrPosition);
+        cp_async_wait_all();
         return;
     }
     rmsnorm_to_smem(src, lw + m.off_gattn, m.d, m.eps, xs, red);
-    if (!coop_stream(W, r, buf, xs, sm_part)) {
+    if (!fr.stream(W, xs, sm_part, tile_sm)) {
         flag_error(c, kErrShape);
         return;
     }
@@ -572,25 +660,30 @@ __global__ void __launch_bounds__(kGemvThreads, 2) k_qkv(DevModel m, int layer, 
 // position: K = RoPE(W_K RMSNorm_j(h_k)), V = W_V RMSNorm_j(h_k), stored bf16.
 // blockIdx.y selects the layer; each layer's K/V tiles are split over
 // gridDim.x CTAs.
+template <bool WHOLE>
 __global__ void __launch_bounds__(kGemvThreads, 2) k_kvfill(DevModel m, int exit_layer) {
     extern __shared__ float4 smem_f4[];
     float* xs = reinterpret_cast<float*>(smem_f4);
     float* sm_part = sm_partials(xs, m.d);
+    uint4* tile_sm = sm_tile(xs, m.d, 0);
     __shared__ float red[32];
     const int j = exit_layer + blockIdx.y;
     const uint16_t* lw = layer_base(m, j);
     const int64_t nq = (int64_t)m.A * m.D / 2, nk = (int64_t)m.KH * m.D / 2;
     const uint4* W = reinterpret_cast<const uint4*>(lw + m.off_wqkv + nq * 2 * m.d);
-    const CoopRange r = coop_range(2 * nk / 16, m.d, blockIdx.x, gridDim.x);
-    uint4 buf[kWindow];
-    coop_prefetch(W, r, buf);
-    zero_sm_part(sm_part);
+    GemvFront<WHOLE> fr;
+    fr.begin(W, 2 * nk / 16, m.d, tile_sm);
+    const CoopRange& r = fr.r;
+    if (!WHOLE) zero_sm_part(sm_part);
     pdl_wait();
     pdl_launch_dependents();
     const int pos = m.ctl->pos;
-    if (pos < 0 || pos >= m.max_ctx) return;
+    if (pos < 0 || pos >= m.max_ctx) {
+        cp_async_wait_all();
+        return;
+    }
     rmsnorm_to_smem(m.h, lw + m.off_gattn, m.d, m.eps, xs, red);
-    if (!coop_stream(W, r, buf, xs, sm_part)) {
+    if (!fr.stream(W, xs, sm_part, tile_sm)) {
         flag_error(m.ctl, kErrShape);
         return;
     }
@@ -603,21 +696,25 @@ __global__ void __launch_bounds__(kGemvThreads, 2) k_kvfill(DevModel m, int exit
 }
 
 // Output projection with the residual add: h += W_o o.
+template <bool WHOLE>
 __global__ void __launch_bounds__(kGemvThreads, 2) k_oproj(DevModel m, int layer) {
     extern __shared__ float4 smem_f4[];
     float* xs = reinterpret_cast<float*>(smem_f4);
     const int K = m.A * m.D;
     float* sm_part = sm_partials(xs, K);
+    uint4* tile_sm = sm_tile(xs, K, 0);
     const uint4* W = reinterpret_cast<const uint4*>(layer_base(m, layer) + m.off_wo);
-    const CoopRange r = coop_range(tiles_of(m.d), K, blockIdx.x, gridDim.x);
-    uint4 buf[kWindow];
-    coop_prefetch(W, r, buf);
-    zero_sm_part(sm_part);
+    GemvFront<WHOLE> fr;
+    fr.begin(W, tiles_of(m.d), K, tile_sm);
+    const CoopRange& r = fr.r;
+    if (!WHOLE) zero_sm_part(sm_part);
     pdl_wait();
     pdl_launch_dependents();
-    for (int i = threadIdx.x; i < K; i += blockDim.x) xs[i] = m.o[i];
+    int lo, hi;
+    fr.x_range(K, lo, hi);
+    for (int i = lo + threadIdx.x; i < hi; i += blockDim.x) xs[i] = m.o[i];
     __syncthreads();
-    if (!coop_stream(W, r, buf, xs, sm_part)) {
+    if (!fr.stream(W, xs, sm_part, tile_sm)) {
         flag_error(m.ctl, kErrShape);
         return;
     }
@@ -626,21 +723,23 @@ __global__ void __launch_bounds__(kGemvThreads, 2) k_oproj(DevModel m, int layer
 }
 
 // Gated feed-forward up: a = SiLU(W_g x) * (W_u x), x = RMSNorm(h) * g_mlp.
+template <bool WHOLE>
 __global__ void __launch_bounds__(kGemvThreads, 2) k_gateup(DevModel m, int layer) {
     extern __shared__ float4 smem_f4[];
     float* xs = reinterpret_cast<float*>(smem_f4);
     float* sm_part = sm_partials(xs, m.d);
+    uint4* tile_sm = sm_tile(xs, m.d, 0);
     __shared__ float red[32];
     const uint16_t* lw = layer_base(m, layer);
     const uint4* W = reinterpret_cast<const uint4*>(lw + m.off_wgu);
-    const CoopRange r = coop_range(tiles_of(2 * (int64_t)m.F), m.d, blockIdx.x, gridDim.x);
-    uint4 buf[kWindow];
-    coop_prefetch(W, r, buf);
-    zero_sm_part(sm_part);
+    GemvFront<WHOLE> fr;
+    fr.begin(W, tiles_of(2 * (int64_t)m.F), m.d, tile_sm);
+    const CoopRange& r = fr.r;
+    if (!WHOLE) zero_sm_part(sm_part);
     pdl_wait();
     pdl_launch_dependents();
     rmsnorm_to_smem(m.h, lw + m.off_gmlp, m.d, m.eps, xs, red);
-    if (!coop_stream(W, r, buf, xs, sm_part)) {
+    if (!fr.stream(W, xs, sm_part, tile_sm)) {
         flag_error(m.ctl, kErrShape);
         return;
     }
@@ -649,20 +748,24 @@ __global__ void __launch_bounds__(kGemvThreads, 2) k_gateup(DevModel m, int laye
 }
 
 // Gated feed-forward down with the residual add: h += W_d a.
+template <bool WHOLE>
 __global__ void __launch_bounds__(kGemvThreads, 2) k_down(DevModel m, int layer) {
     extern __shared__ float4 smem_f4[];
     float* xs = reinterpret_cast<float*>(smem_f4);
     float* sm_part = sm_partials(xs, m.F);
+    uint4* tile_sm = sm_tile(xs, m.F, 0);
     const uint4* W = reinterpret_cast<const uint4*>(layer_base(m, layer) + m.off_wd);
-    const CoopRange r = coop_range(tiles_of(m.d), m.F, blockIdx.x, gridDim.x);
-    uint4 buf[kWindow];
-    coop_prefetch(W, r, buf);
-    zero_sm_part(sm_part);
+    GemvFront<WHOLE> fr;
+    fr.begin(W, tiles_of(m.d), m.F, tile_sm);
+    const CoopRange& r = fr.r;
+    if (!WHOLE) zero_sm_part(sm_part);
     pdl_wait();
     pdl_launch_dependents();
-    for (int i = threadIdx.x; i < m.F; i += blockDim.x) xs[i] = m.a[i];
+    int lo, hi;
+    fr.x_range(m.F, lo, hi);
+    for (int i = lo + threadIdx.x; i < hi; i += blockDim.x) xs[i] = m.a[i];
     __syncthreads();
-    if (!coop_stream(W, r, buf, xs, sm_part)) {
+    if (!fr.stream(W, xs, sm_part, tile_sm)) {
         flag_error(m.ctl, kErrShape);
         return;
     }
@@ -671,15 +774,17 @@ __global__ void __launch_bounds__(kGemvThreads, 2) k_down(DevModel m, int layer)
 }
 
 // Readout affine map r: y_r = W_r h + b_r; also keeps h_k for debug.
+template <bool WHOLE>
 __global__ void __launch_bounds__(kGemvThreads, 2) k_readout(DevModel m, int r) {
     extern __shared__ float4 smem_f4[];
     float* xs = reinterpret_cast<float*>(smem_f4);
     float* sm_part = sm_partials(xs, m.d);
+    uint4* tile_sm = sm_tile(xs, m.d, 0);
     const uint4* W = reinterpret_cast<const uint4*>(m.ro_w[r]);
-    const CoopRange rg = coop_range(tiles_of(m.d), m.d, blockIdx.x, gridDim.x);
-    uint4 buf[kWindow];
-    coop_prefetch(W, rg, buf);
-    zero_sm_part(sm_part);
+    GemvFront<WHOLE> fr;
+    fr.begin(W, tiles_of(m.d), m.d, tile_sm);
+    const CoopRange& rg = fr.r;
+    if (!WHOLE) zero_sm_part(sm_part);
     pdl_wait();
     pdl_launch_dependents();
     for (int i = threadIdx.x; i < m.d; i += blockDim.x) {
@@ -688,7 +793,7 @@ __global__ void __launch_bounds__(kGemvThreads, 2) k_readout(DevModel m, int r) 
         if (blockIdx.x == 0) m.hk[(int64_t)r * m.d + i] = v;
     }
     __syncthreads();
-    if (!coop_stream(W, rg, buf, xs, sm_part)) {
+    if (!fr.stream(W, xs, sm_part, tile_sm)) {
         flag_error(m.ctl, kErrShape);
         return;
     }
@@ -1001,158 +1106,202 @@ __global__ void __launch_bounds__(kAttnThreads) k_attention(AttnArgs a) {
 
 // Decode attention of one layer on a thread-block cluster per key-value head
 // (grid (CL, KH), cluster (CL, 1, 1)).  Rank r covers a contiguous run of
-// positions for all A/K query heads of head g with a per-lane online softmax;
-// the 8 warps merge in shared memory, and the CL ranks merge through
-// distributed shared memory, each rank finishing a share of the outputs:
-// o = softmax(q K^T / sqrt(D)) V (fp32).  Before waiting on the QKV kernel,
-// each CTA pulls its past K/V rows into L2 (only position T-1 is new).
+// positions for all A/K query heads of head g, in sub-chunks of NB positions
+// staged in shared memory (K rows XOR-swizzled by 16-byte chunk so that four
+// threads per position read without bank conflicts).  The first sub-chunk's
+// past rows are copied (cp.async) before the kernel waits on the QKV kernel:
+// only position T-1 is new.  Per sub-chunk: scores (4 threads per position),
+// a running softmax per head, and P V with each thread owning output pairs;
+// then the CL ranks merge through distributed shared memory, each finishing
+// a share of o = softmax(q K^T / sqrt(D)) V (fp32).
 namespace cg = cooperative_groups;
+
+
+template <int D>
+struct AttnSmem {
+    static constexpr int NB = 16384 / D;  // positions per sub-chunk (K + V = 64 KB)
+    static constexpr int CH = D / 8;      // 16-byte chunks per row
+    static constexpr int GMAX = 8;
+    static constexpr size_t bytes = (size_t)2 * NB * CH * 16 + (size_t)GMAX * D * 4 + (size_t)GMAX * NB * 4;
+};
+
+// Copy rows [r0, r1) of the CTA's sub-chunk (positions base + r) into smem.
+template <int D>
+__device__ __forceinline__ void attn_stage(const AttnArgs& a, int g, int base, int r0, int r1, uint4* Ks, uint4* Vs,
+                                           bool async) {
+    constexpr int CH = D / 8;
+    const int P = a.page_size;
+    for (int i = r0 * CH + threadIdx.x; i < r1 * CH; i += blockDim.x) {
+        const int r = i / CH, c = i - r * CH;
+        const int t = base + r;
+        const int64_t off = (((int64_t)a.page_table[t / P] * a.KH + g) * P + (t % P)) * D + c * 8;
+        uint4* kd = Ks + r * CH + (c ^ (r & (CH - 1)));
+        uint4* vd = Vs + r * CH + c;
+        if (async) {
+            cp_async16(kd, a.kp + off);
+            cp_async16(vd, a.vp + off);
+        } else {
+            *kd = *reinterpret_cast<const uint4*>(a.kp + off);
+            *vd = *reinterpret_cast<const uint4*>(a.vp + off);
+        }
+    }
+}
 
 template <int D>
 __global__ void __launch_bounds__(kAttnThreads) k_attn_cluster(AttnArgs a) {
-    constexpr int LPR = D / 8;
-    constexpr int RPW = 32 / LPR;
-    constexpr int NW = kAttnThreads / 32;
-    constexpr int GMAX = 8;
-    __shared__ __align__(16) float qs[GMAX * D];
-    __shared__ float wm[NW][GMAX], wl[NW][GMAX];
-    __shared__ __align__(16) float wacc[NW][GMAX][D];
-    __shared__ float cm[GMAX], cl[GMAX];
+    using S = AttnSmem<D>;
+    constexpr int NB = S::NB, CH = S::CH, GMAX = S::GMAX;
+    extern __shared__ __align__(16) unsigned char attn_sm[];
+    uint4* Ks = reinterpret_cast<uint4*>(attn_sm);
+    uint4* Vs = Ks + NB * CH;
+    float* qs = reinterpret_cast<float*>(Vs + NB * CH);
+    float* ps = qs + GMAX * D;
+    __shared__ float hm[GMAX], hl[GMAX], hs[GMAX];
     cg::cluster_group cluster = cg::this_cluster();
     const int rank = (int)cluster.block_rank(), CL = (int)cluster.num_blocks();
-    const int g = blockIdx.y, G = a.A / a.KH, P = a.page_size;
+    const int g = blockIdx.y, G = a.A / a.KH;
     const int T = a.ctl->pos + 1;
     const int chunk = (T + CL - 1) / CL;
     const int t0 = min(T, rank * chunk), t1 = min(T, t0 + chunk);
-    if (threadIdx.x == 0) {
-        const int te = min(t1, T - 1);
-        for (int t = t0; t < te;) {
-            const int page = a.page_table[t / P], slot = t % P, n = min(te - t, P - slot);
-            const int64_t off = (((int64_t)page * a.KH + g) * P + slot) * D;
-            prefetch_l2(a.kp + off, (uint32_t)(n * D * 2));
-            prefetch_l2(a.vp + off, (uint32_t)(n * D * 2));
-            t += n;
-        }
+    // past rows of the first sub-chunk, before waiting on the QKV kernel
+    const int first_end = min(t1, t0 + NB);
+    attn_stage<D>(a, g, t0, 0, max(0, min(first_end, T - 1) - t0), Ks, Vs, true);
+    cp_async_commit();
+    if (threadIdx.x < GMAX) {
+        hm[threadIdx.x] = -CUDART_INF_F;
+        hl[threadIdx.x] = 0.f;
     }
     pdl_wait();
     pdl_launch_dependents();
     const float scale = 1.0f / sqrtf((float)D);
     for (int i = threadIdx.x; i < G * D; i += blockDim.x) qs[i] = a.q[(int64_t)g * G * D + i] * scale;
+    if (T - 1 >= t0 && T - 1 < first_end) attn_stage<D>(a, g, t0, T - 1 - t0, T - t0, Ks, Vs, false);
+    cp_async_wait_all();
     __syncthreads();
 
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int grp = lane / LPR, e0 = (lane % LPR) * 8;
-    float mx[GMAX], ls[GMAX], acc[GMAX][8];
+    // each thread owns output pairs (h, e, e+1) for items tid, tid + blockDim
+    constexpr int ITEMS = (GMAX * D / 2 + kAttnThreads - 1) / kAttnThreads;
+    float acc[ITEMS][2];
 #pragma unroll
-    for (int h = 0; h < GMAX; ++h) {
-        mx[h] = -CUDART_INF_F;
-        ls[h] = 0.f;
-#pragma unroll
-        for (int e = 0; e < 8; ++e) acc[h][e] = 0.f;
-    }
-    for (int tt = t0 + warp * RPW; tt < t1; tt += NW * RPW) {
-        const int t = tt + grp;
-        const bool valid = t < t1;
-        float kf[8], vf[8];
-        if (valid) {
-            const int page = a.page_table[t / P];
-            const int64_t off = (((int64_t)page * a.KH + g) * P + (t % P)) * D + e0;
-            const uint4 kw = *reinterpret_cast<const uint4*>(a.kp + off);
-            const uint4 vw = *reinterpret_cast<const uint4*>(a.vp + off);
-            kf[0] = bf_lo(kw.x); kf[1] = bf_hi(kw.x); kf[2] = bf_lo(kw.y); kf[3] = bf_hi(kw.y);
-            kf[4] = bf_lo(kw.z); kf[5] = bf_hi(kw.z); kf[6] = bf_lo(kw.w); kf[7] = bf_hi(kw.w);
-            vf[0] = bf_lo(vw.x); vf[1] = bf_hi(vw.x); vf[2] = bf_lo(vw.y); vf[3] = bf_hi(vw.y);
-            vf[4] = bf_lo(vw.z); vf[5] = bf_hi(vw.z); vf[6] = bf_lo(vw.w); vf[7] = bf_hi(vw.w);
-        } else {
-#pragma unroll
-            for (int e = 0; e < 8; ++e) kf[e] = vf[e] = 0.f;
+    for (int k = 0; k < ITEMS; ++k) acc[k][0] = acc[k][1] = 0.f;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    (void)lane;
+
+    for (int base = t0; base < t1; base += NB) {
+        const int nb = min(NB, t1 - base);
+        if (base != t0) {
+            __syncthreads();  // everyone is done with the previous sub-chunk
+            attn_stage<D>(a, g, base, 0, nb, Ks, Vs, false);
+            __syncthreads();
         }
+        // scores: one thread per (head, position), the whole dot product
+        for (int w = threadIdx.x; w < G * nb; w += blockDim.x) {
+            const int h = w / nb, p = w - h * nb;
+            const float* qh = qs + h * D;
+            float d0 = 0.f, d1 = 0.f;
 #pragma unroll
-        for (int h = 0; h < GMAX; ++h) {
-            if (h >= G) break;
-            float d = 0.f;
-#pragma unroll
-            for (int e = 0; e < 8; ++e) d = fmaf(kf[e], qs[h * D + e0 + e], d);
-#pragma unroll
-            for (int o = LPR / 2; o; o >>= 1) d += __shfl_xor_sync(0xffffffffu, d, o);
-            if (valid) {
-                const float mn = fmaxf(mx[h], d);
-                const float corr = expf(mx[h] - mn);
-                const float p = expf(d - mn);
-                ls[h] = ls[h] * corr + p;
-#pragma unroll
-                for (int e = 0; e < 8; ++e) acc[h][e] = fmaf(p, vf[e], acc[h][e] * corr);
-                mx[h] = mn;
+            for (int c = 0; c < CH; ++c) {
+                const uint4 kw = Ks[p * CH + (c ^ (p & (CH - 1)))];
+                const float4 q0 = *reinterpret_cast<const float4*>(qh + c * 8);
+                const float4 q1 = *reinterpret_cast<const float4*>(qh + c * 8 + 4);
+                d0 = fmaf(bf_lo(kw.x), q0.x, d0);
+                d1 = fmaf(bf_hi(kw.x), q0.y, d1);
+                d0 = fmaf(bf_lo(kw.y), q0.z, d0);
+                d1 = fmaf(bf_hi(kw.y), q0.w, d1);
+                d0 = fmaf(bf_lo(kw.z), q1.x, d0);
+                d1 = fmaf(bf_hi(kw.z), q1.y, d1);
+                d0 = fmaf(bf_lo(kw.w), q1.z, d0);
+                d1 = fmaf(bf_hi(kw.w), q1.w, d1);
             }
+            ps[h * NB + p] = d0 + d1;
         }
-    }
+        __syncthreads();
+        // softmax statistics of this sub-chunk, one warp per head
+        if (warp < G) {
+            const int h = warp;
+            float m = -CUDART_INF_F;
+            for (int p = lane; p < nb; p += 32) m = fmaxf(m, ps[h * NB + p]);
 #pragma unroll
-    for (int o = LPR; o < 32; o <<= 1) {
-#pragma unroll
-        for (int h = 0; h < GMAX; ++h) {
-            if (h >= G) break;
-            const float m2 = __shfl_xor_sync(0xffffffffu, mx[h], o);
-            const float l2 = __shfl_xor_sync(0xffffffffu, ls[h], o);
-            float a2[8];
-#pragma unroll
-            for (int e = 0; e < 8; ++e) a2[e] = __shfl_xor_sync(0xffffffffu, acc[h][e], o);
-            const float M = fmaxf(mx[h], m2);
-            if (M != -CUDART_INF_F) {
-                const float c1 = expf(mx[h] - M), c2 = expf(m2 - M);
-                ls[h] = ls[h] * c1 + l2 * c2;
-#pragma unroll
-                for (int e = 0; e < 8; ++e) acc[h][e] = acc[h][e] * c1 + a2[e] * c2;
-                mx[h] = M;
+            for (int o = 16; o; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+            const float mo = hm[h];
+            const float mn = fmaxf(mo, m);
+            float l = 0.f;
+            for (int p = lane; p < nb; p += 32) {
+                const float e = expf(ps[h * NB + p] - mn);
+                ps[h * NB + p] = e;
+                l += e;
             }
-        }
-    }
-    if (grp == 0) {
-#pragma unroll
-        for (int h = 0; h < GMAX; ++h) {
-            if (h >= G) break;
+            l = warp_sum(l);
             if (lane == 0) {
-                wm[warp][h] = mx[h];
-                wl[warp][h] = ls[h];
+                const float sc = expf(mo - mn);  // 0 on the first sub-chunk
+                hs[h] = sc;
+                hl[h] = hl[h] * sc + l;
+                hm[h] = mn;
             }
+        }
+        __syncthreads();
+        // P V: acc(h, e..e+1) = acc * rescale + sum_p p(h, p) v(p, e..e+1)
 #pragma unroll
-            for (int e = 0; e < 8; ++e) wacc[warp][h][e0 + e] = acc[h][e];
+        for (int k = 0; k < ITEMS; ++k) {
+            const int it = threadIdx.x + k * kAttnThreads;
+            if (it >= G * D / 2) break;
+            const int h = it / (D / 2), e2 = it - h * (D / 2);
+            const float sc = hs[h];
+            float x0 = acc[k][0] * sc, x1 = acc[k][1] * sc;
+            const uint32_t* vrow = reinterpret_cast<const uint32_t*>(Vs) + e2;
+            const float* pr = ps + h * NB;
+            for (int p = 0; p < nb; ++p) {
+                const uint32_t v2 = vrow[p * (D / 2)];
+                const float w = pr[p];
+                x0 = fmaf(w, bf_lo(v2), x0);
+                x1 = fmaf(w, bf_hi(v2), x1);
+            }
+            acc[k][0] = x0;
+            acc[k][1] = x1;
         }
     }
+    // this CTA's partial: (hm, hl) per head, accumulator pairs in qs (reused)
     __syncthreads();
-    // this CTA's partial: (cm, cl) per head, accumulator in wacc[0]
-    for (int i = threadIdx.x; i < G * D; i += blockDim.x) {
-        const int h = i / D, e = i - h * D;
-        float M = -CUDART_INF_F, L = 0.f, O = 0.f;
-        for (int w = 0; w < NW; ++w) {
-            const float m2 = wm[w][h];
-            const float Mn = fmaxf(M, m2);
-            if (Mn == -CUDART_INF_F) continue;
-            const float c1 = expf(M - Mn), c2 = expf(m2 - Mn);
-            L = L * c1 + wl[w][h] * c2;
-            O = O * c1 + wacc[w][h][e] * c2;
-            M = Mn;
-        }
-        wacc[0][h][e] = O;
-        if (e == 0) {
-            cm[h] = M;
-            cl[h] = L;
-        }
+#pragma unroll
+    for (int k = 0; k < ITEMS; ++k) {
+        const int it = threadIdx.x + k * kAttnThreads;
+        if (it >= G * D / 2) break;
+        qs[2 * it] = acc[k][0];
+        qs[2 * it + 1] = acc[k][1];
     }
     cluster.sync();
-    // merge the ranks' partials; rank r finishes outputs r*blockDim.x + tid, ...
+    // merge the ranks' partials: thread (r, h) weighs rank r for head h
+    // (shuffle reductions over the CL ranks of a head), then each output sums
+    // the CL scaled partials, all remote loads issued before use; outputs are
+    // spread over all ranks
+    __shared__ float rw[16][GMAX];  // exp(m_r - M) / L per rank and head (CL <= 16)
+    if (threadIdx.x < 16 * GMAX) {
+        const int r = threadIdx.x & 15, h = threadIdx.x >> 4;  // 16 lanes per head
+        const bool on = r < CL && h < G;
+        const float mr = on ? ld_dsmem(dsmem_addr(&hm[h], r)) : -CUDART_INF_F;
+        const float lr = on ? ld_dsmem(dsmem_addr(&hl[h], r)) : 0.f;
+        float M = mr;
+#pragma unroll
+        for (int o = 8; o; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+        const float c = mr == -CUDART_INF_F ? 0.f : expf(mr - M);
+        float L = lr * c;
+#pragma unroll
+        for (int o = 8; o; o >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
+        if (on) rw[r][h] = c / L;
+    }
+    __syncthreads();
     for (int i = rank * blockDim.x + threadIdx.x; i < G * D; i += CL * blockDim.x) {
-        const int h = i / D, e = i - h * D;
-        float M = -CUDART_INF_F;
-        for (int r = 0; r < CL; ++r) M = fmaxf(M, cluster.map_shared_rank(cm, r)[h]);
-        float L = 0.f, O = 0.f;
-        for (int r = 0; r < CL; ++r) {
-            const float mr = cluster.map_shared_rank(cm, r)[h];
-            if (mr == -CUDART_INF_F) continue;
-            const float c = expf(mr - M);
-            L = fmaf(cluster.map_shared_rank(cl, r)[h], c, L);
-            O = fmaf(cluster.map_shared_rank(&wacc[0][0][0], r)[h * D + e], c, O);
-        }
-        a.out[(int64_t)(g * G + h) * D + e] = O / L;
+        const int h = i / D;
+        const uint32_t base = (uint32_t)__cvta_generic_to_shared(qs + i);
+        float part[16];
+#pragma unroll
+        for (int r = 0; r < 16; ++r)
+            if (r < CL) part[r] = ld_dsmem(dsmem_rank(base, r));
+        float O = 0.f;
+#pragma unroll
+        for (int r = 0; r < 16; ++r)
+            if (r < CL) O = fmaf(rw[r][h], part[r], O);
+        a.out[(int64_t)g * G * D + i] = O;
     }
     cluster.sync();  // keep every rank's shared memory alive until all have read it
 }
@@ -1255,18 +1404,25 @@ size_t gemv_smem_bytes(int kmax) {
 
 cudaError_t configure_kernels(int kmax) {
     if (gemv_smem_bytes(kmax) > g_smem) g_smem = gemv_smem_bytes(kmax);
-    const int bytes = (int)g_smem;
+    int dev = 0, optin = 0;
     cudaError_t e;
-    if ((e = cudaFuncSetAttribute(k_qkv, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes))) return e;
-    if ((e = cudaFuncSetAttribute(k_kvfill, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes))) return e;
-    if ((e = cudaFuncSetAttribute(k_oproj, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes))) return e;
-    if ((e = cudaFuncSetAttribute(k_gateup, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes))) return e;
-    if ((e = cudaFuncSetAttribute(k_down, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes))) return e;
-    if ((e = cudaFuncSetAttribute(k_readout, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes))) return e;
-    if ((e = cudaFuncSetAttribute(k_vocab, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes))) return e;
-    if ((e = cudaFuncSetAttribute(k_vocab_rowmajor, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes))) return e;
+    if ((e = cudaGetDevice(&dev))) return e;
+    if ((e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev))) return e;
+    cudaFuncAttributes fa;
+    // each kernel may use the opt-in maximum less its own static shared memory
+#define EE_SMEM(k)                                                                                   \
+    if ((e = cudaFuncGetAttributes(&fa, k))) return e;                                                \
+    if ((e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,                     \
+                                  optin - (int)fa.sharedSizeBytes)))                                  \
+        return e;
+    EE_SMEM(k_qkv<true>) EE_SMEM(k_qkv<false>) EE_SMEM(k_kvfill<true>) EE_SMEM(k_kvfill<false>)
+    EE_SMEM(k_oproj<true>) EE_SMEM(k_oproj<false>) EE_SMEM(k_gateup<true>) EE_SMEM(k_gateup<false>)
+    EE_SMEM(k_down<true>) EE_SMEM(k_down<false>) EE_SMEM(k_readout<true>) EE_SMEM(k_readout<false>)
+    EE_SMEM(k_vocab) EE_SMEM(k_vocab_rowmajor)
     if ((e = cudaFuncSetAttribute(k_attn_cluster<64>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1))) return e;
     if ((e = cudaFuncSetAttribute(k_attn_cluster<128>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1))) return e;
+    EE_SMEM(k_attn_cluster<64>) EE_SMEM(k_attn_cluster<128>)
+#undef EE_SMEM
     return cudaSuccess;
 }
 
@@ -1275,24 +1431,42 @@ static size_t smem_for(int k, int extra = 0) {
     return ((size_t)((k + 3) & ~3) + (size_t)kSlotTiles * kWarps * 32 + (size_t)extra) * sizeof(float);
 }
 
-cudaError_t launch_qkv(const DevModel& m, int layer, int first, int grid, bool pdl, cudaStream_t s) {
-    return launch_k(k_qkv, dim3(grid), dim3(kGemvThreads), smem_for(m.d, m.d), pdl, s, m, layer, first);
+// Dynamic shared memory of a GEMV launch: x, tile partials, `extra` floats
+// and, in whole-tile mode, the staged tile (32 rows x K bf16).
+static size_t gemv_smem(int K, int extra, bool whole) {
+    return smem_for(K, extra) + (whole ? (size_t)64 * K : 0);
 }
-cudaError_t launch_kvfill(const DevModel& m, int exit_layer, int grid_x, bool pdl, cudaStream_t s) {
-    return launch_k(k_kvfill, dim3(grid_x, m.L - exit_layer), dim3(kGemvThreads), smem_for(m.d), pdl, s, m,
-                    exit_layer);
+
+cudaError_t launch_qkv(const DevModel& m, int layer, int first, int grid, bool whole, bool pdl, cudaStream_t s) {
+    const size_t sm = gemv_smem(m.d, m.d, whole);
+    if (whole) return launch_k(k_qkv<true>, dim3(grid), dim3(kGemvThreads), sm, pdl, s, m, layer, first);
+    return launch_k(k_qkv<false>, dim3(grid), dim3(kGemvThreads), sm, pdl, s, m, layer, first);
 }
-cudaError_t launch_oproj(const DevModel& m, int layer, int grid, bool pdl, cudaStream_t s) {
-    return launch_k(k_oproj, dim3(grid), dim3(kGemvThreads), smem_for(m.A * m.D), pdl, s, m, layer);
+cudaError_t launch_kvfill(const DevModel& m, int exit_layer, int grid_x, bool whole, bool pdl, cudaStream_t s) {
+    const dim3 grid(grid_x, m.L - exit_layer);
+    const size_t sm = gemv_smem(m.d, 0, whole);
+    if (whole) return launch_k(k_kvfill<true>, grid, dim3(kGemvThreads), sm, pdl, s, m, exit_layer);
+    return launch_k(k_kvfill<false>, grid, dim3(kGemvThreads), sm, pdl, s, m, exit_layer);
 }
-cudaError_t launch_gateup(const DevModel& m, int layer, int grid, bool pdl, cudaStream_t s) {
-    return launch_k(k_gateup, dim3(grid), dim3(kGemvThreads), smem_for(m.d), pdl, s, m, layer);
+cudaError_t launch_oproj(const DevModel& m, int layer, int grid, bool whole, bool pdl, cudaStream_t s) {
+    const size_t sm = gemv_smem(m.A * m.D, 0, whole);
+    if (whole) return launch_k(k_oproj<true>, dim3(grid), dim3(kGemvThreads), sm, pdl, s, m, layer);
+    return launch_k(k_oproj<false>, dim3(grid), dim3(kGemvThreads), sm, pdl, s, m, layer);
 }
-cudaError_t launch_down(const DevModel& m, int layer, int grid, bool pdl, cudaStream_t s) {
-    return launch_k(k_down, dim3(grid), dim3(kGemvThreads), smem_for(m.F), pdl, s, m, layer);
+cudaError_t launch_gateup(const DevModel& m, int layer, int grid, bool whole, bool pdl, cudaStream_t s) {
+    const size_t sm = gemv_smem(m.d, 0, whole);
+    if (whole) return launch_k(k_gateup<true>, dim3(grid), dim3(kGemvThreads), sm, pdl, s, m, layer);
+    return launch_k(k_gateup<false>, dim3(grid), dim3(kGemvThreads), sm, pdl, s, m, layer);
 }
-cudaError_t launch_readout(const DevModel& m, int r, int grid, bool pdl, cudaStream_t s) {
-    return launch_k(k_readout, dim3(grid), dim3(kGemvThreads), smem_for(m.d), pdl, s, m, r);
+cudaError_t launch_down(const DevModel& m, int layer, int grid, bool whole, bool pdl, cudaStream_t s) {
+    const size_t sm = gemv_smem(m.F, 0, whole);
+    if (whole) return launch_k(k_down<true>, dim3(grid), dim3(kGemvThreads), sm, pdl, s, m, layer);
+    return launch_k(k_down<false>, dim3(grid), dim3(kGemvThreads), sm, pdl, s, m, layer);
+}
+cudaError_t launch_readout(const DevModel& m, int r, int grid, bool whole, bool pdl, cudaStream_t s) {
+    const size_t sm = gemv_smem(m.d, 0, whole);
+    if (whole) return launch_k(k_readout<true>, dim3(grid), dim3(kGemvThreads), sm, pdl, s, m, r);
+    return launch_k(k_readout<false>, dim3(grid), dim3(kGemvThreads), sm, pdl, s, m, r);
 }
 cudaError_t launch_vocab(const VocabArgs& v, int grid, bool pdl, cudaStream_t s) {
     const size_t smem = (size_t)((v.d + 3) & ~3) * sizeof(float);
@@ -1309,7 +1483,7 @@ cudaError_t launch_attention_cluster(const AttnArgs& a, int head_dim, int cluste
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(cluster, a.KH);
     cfg.blockDim = dim3(kAttnThreads);
-    cfg.dynamicSmemBytes = 0;
+    cfg.dynamicSmemBytes = head_dim == 64 ? AttnSmem<64>::bytes : AttnSmem<128>::bytes;
     cfg.stream = s;
     cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -1323,6 +1497,27 @@ cudaError_t launch_attention_cluster(const AttnArgs& a, int head_dim, int cluste
     if (head_dim == 64) return cudaLaunchKernelEx(&cfg, k_attn_cluster<64>, a);
     if (head_dim == 128) return cudaLaunchKernelEx(&cfg, k_attn_cluster<128>, a);
     return cudaErrorInvalidValue;
+}
+int attention_cluster_size(int head_dim, int n_kv_heads) {
+    for (int cl : {16, 8}) {
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(cl, n_kv_heads);
+        cfg.blockDim = dim3(kAttnThreads);
+        cfg.dynamicSmemBytes = head_dim == 64 ? AttnSmem<64>::bytes : AttnSmem<128>::bytes;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = cl;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        int n = 0;
+        const cudaError_t e = head_dim == 64 ? cudaOccupancyMaxActiveClusters(&n, k_attn_cluster<64>, &cfg)
+                                             : cudaOccupancyMaxActiveClusters(&n, k_attn_cluster<128>, &cfg);
+        if (e == cudaSuccess && n >= 1) return cl;
+        cudaGetLastError();
+    }
+    return 8;
 }
 cudaError_t launch_step_end(const DevModel& m, int has_cond, cudaGraphConditionalHandle cond, bool pdl,
                             cudaStream_t s) {
