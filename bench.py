@@ -498,16 +498,20 @@ def run_ours(args, rank: int, world: int, local: int):
 
 def profile_run(args, local: int):
     """A short decode for ncu captures: 64-token prompt, two 8-token chunks
-    with exits imposed at 50%, no calibration.  Prints the launch counts."""
+    with exits imposed at 50%, no calibration.  Prints the launch counts.
+    --eager launches every kernel directly (ncu cannot profile single kernel
+    nodes of graphs that hold conditional nodes)."""
     import torch
 
-    from paper_2609_14144_gb300 import DEVICE, FORCE_EXIT_AT, FORCE_FULL, Engine
+    from paper_2609_14144_gb300 import DEVICE, FORCE_EXIT_AT, FORCE_FULL, OPT_GRAPHS, Engine
 
     torch.cuda.set_device(local)
     shape = synth.CONFIGS[WORKLOAD]
     model = synth.make_model(shape)
     P, C = 64, 8
     eng = Engine(shape, model, max_ctx=P + 2 * C, device=local)
+    if args.eager:
+        eng.set_option(OPT_GRAPHS, 0)
     eng.prefill(synth.prompt(shape, P))
     sched = np.where(synth.exit_schedule(shape, 2 * C, 0.5, index=1) == 1, FORCE_EXIT_AT(0), FORCE_FULL)
     sched = sched.astype(np.int8)
@@ -531,6 +535,7 @@ def main():
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--profile-run", action="store_true", help="short decode for ncu captures")
+    ap.add_argument("--eager", action="store_true", help="with --profile-run: direct launches, no graphs")
     ap.add_argument("--workload", default=WORKLOAD, choices=sorted(synth.CONFIGS),
                     help="synthetic shape (the benchmark workload is 1.5b)")
     args = ap.parse_args()
