@@ -202,7 +202,7 @@ int ee_position(ee_ctx* ctx, int32_t* pos);
 int ee_set_option(ee_ctx* ctx, int option, int value);
 
 #define EE_DBG_HIDDEN_READOUT 1 /* layer = readout r: residual h_k it read, d floats   */
-#define EE_DBG_READOUT_Y 2      /* layer = readout r: W_r bf16(h_k) + b_r, d floats    */
+#define EE_DBG_READOUT_Y 2      /* layer = readout r: W_r h_k + b_r, d floats          */
 #define EE_DBG_HIDDEN_FINAL 3   /* residual after layer L of the last full step        */
 #define EE_DBG_READOUT_LOGITS 4 /* layer = readout r: V floats (EE_OPT_DEBUG_LOGITS)   */
 #define EE_DBG_FINAL_LOGITS 5   /* V floats (EE_OPT_DEBUG_LOGITS)                      */

@@ -33,13 +33,21 @@ __device__ __forceinline__ float bf_hi(uint32_t u) { return __uint_as_float(u & 
 __device__ __forceinline__ float bf2f(uint16_t b) { return __uint_as_float((uint32_t)b << 16); }
 __device__ __forceinline__ uint16_t f2bf(float f) { return __bfloat16_as_ushort(__float2bfloat16_rn(f)); }
 
+// L2 policy for data read once per step (weights): its lines are the first
+// evicted, so the streamed matrices do not push out the KV cache and the
+// activations.  (Not volatile: a pure value the compiler may hoist.)
+__device__ __forceinline__ uint64_t l2_evict_first_policy() {
+    uint64_t pol;
+    asm("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+    return pol;
+}
 // Streaming 16-byte load of read-only weights: no L1 allocation, 256-byte
-// L2 sector promotion.
+// L2 sector promotion, evict-first in L2.
 __device__ __forceinline__ uint4 ldg_stream(const uint4* p) {
     uint4 r;
-    asm volatile("ld.global.nc.L1::no_allocate.L2::256B.v4.u32 {%0,%1,%2,%3}, [%4];"
+    asm volatile("ld.global.nc.L1::no_allocate.L2::cache_hint.L2::256B.v4.u32 {%0,%1,%2,%3}, [%4], %5;"
         : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
-        : "l"(p));
+        : "l"(p), "l"(l2_evict_first_policy()));
     return r;
 }
 
@@ -212,6 +220,12 @@ __device__ __forceinline__ void flat_gemv(const uint16_t* __restrict__ W, int K,
 __device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"((uint32_t)__cvta_generic_to_shared(smem)),
                  "l"(gmem)
+                 : "memory");
+}
+// Weight copy that marks its L2 line first to be evicted (read once per step).
+__device__ __forceinline__ void cp_async16_stream(void* smem, const void* gmem, uint64_t pol) {
+    asm volatile("cp.async.cg.shared.global.L2::cache_hint [%0], [%1], 16, %2;"
+                 ::"r"((uint32_t)__cvta_generic_to_shared(smem)), "l"(gmem), "l"(pol)
                  : "memory");
 }
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
@@ -391,7 +405,8 @@ struct GemvFront {
             r.cta = blockIdx.x;
             r.n_cta = gridDim.x;
             const uint4* src = W + (int64_t)r.C0 * 32;
-            for (int i = threadIdx.x; i < r.Rc * 32; i += blockDim.x) cp_async16(tile_sm + i, src + i);
+            const uint64_t pol = l2_evict_first_policy();
+            for (int i = threadIdx.x; i < r.Rc * 32; i += blockDim.x) cp_async16_stream(tile_sm + i, src + i, pol);
             cp_async_commit();
         } else {
             r = coop_range(n_tiles, K, blockIdx.x, gridDim.x);
