@@ -162,12 +162,21 @@ def tau_for_rate(p: np.ndarray, rate: float) -> float:
     return float(s[max(0, min(len(s) - 1, k - 1))])
 
 
-def step_launches(L: int, readout_layers, exit_readout: int) -> int:
+def layer_launches(L: int, bounds, persistent: bool) -> int:
+    """Launches that run layers [b_i, b_{i+1}) for consecutive bounds: five per
+    layer, or one persistent launch per non-empty run."""
+    runs = [b - a for a, b in zip(bounds[:-1], bounds[1:])]
+    return sum(1 for r in runs if r > 0) if persistent else 5 * sum(runs)
+
+
+def step_launches(L: int, readout_layers, exit_readout: int, persistent: bool = False) -> int:
     """Kernels one gated decode step launches (graph nodes of libee)."""
+    ro = list(readout_layers)
     if exit_readout < 0:
-        return 5 * L + 2 * len(readout_layers) + 1 + 1
-    e = readout_layers[exit_readout]
-    return 5 * e + 2 * (exit_readout + 1) + (1 if e < L else 0) + 1
+        return layer_launches(L, [0] + ro + [L], persistent) + 2 * len(ro) + 1 + 1
+    e = ro[exit_readout]
+    return layer_launches(L, [0] + ro[:exit_readout + 1], persistent) + 2 * (exit_readout + 1) + \
+        (1 if e < L else 0) + 1
 
 
 def kernel_bytes(dims: bm.Dims, T: int, k_layer: int) -> dict:
@@ -182,14 +191,26 @@ def kernel_bytes(dims: bm.Dims, T: int, k_layer: int) -> dict:
         "readout": 2 * (d * d + d),
         "vocab": 2 * (V * d + d),
         "kvfill": (L - k_layer) * (2 * (2 * K * D * d + d) + 4 * K * D),
+        # the persistent kernel over layers 1..k: their weights and KV traffic
+        "layers": k_layer * (2 * ((A + 2 * K) * D * d + d) + 4 * K * D + 4 * K * D * T + 2 * d * A * D
+                             + 2 * (2 * F * d + d) + 2 * d * F),
     }
 
 
-def kernel_launches_per_token(L: int, k: int, exit_rate: float) -> dict:
+def kernel_launches_per_token(L: int, k: int, exit_rate: float, persistent: bool = False) -> dict:
+    """Launches of each kernel per token.  With the persistent kernel, the
+    upper run of layers counts as (L - k) / k launches of the measured
+    layers-1..k launch (same per-layer work)."""
     full = 1.0 - exit_rate
     layers = k + full * (L - k)
-    return {"qkv": layers, "attention": layers, "oproj": layers, "gateup": layers, "down": layers,
-            "readout": 1.0, "vocab": 1.0 + full, "kvfill": exit_rate}
+    out = {"readout": 1.0, "vocab": 1.0 + full, "kvfill": exit_rate}
+    if persistent:
+        out.update({"qkv": 0.0, "attention": 0.0, "oproj": 0.0, "gateup": 0.0, "down": 0.0,
+                    "layers": 1.0 + full * (L - k) / k})
+    else:
+        out.update({"qkv": layers, "attention": layers, "oproj": layers, "gateup": layers, "down": layers,
+                    "layers": 0.0})
+    return out
 
 
 def ncu_traffic(kernel: str, shape_name: str) -> float | None:
@@ -337,7 +358,7 @@ class Runner:
         ro = list(self.shape.readout_layers)
         bytes_total = sum(bm.step_bytes(self.dims, T0 + i + 1, ro, None if e < 0 else int(e))
                           for i, e in enumerate(timed))
-        launches = sum(step_launches(self.shape.n_layers, ro, int(e)) for e in timed) + steps
+        launches = sum(step_launches(self.shape.n_layers, ro, int(e), self.eng.persistent) for e in timed) + steps
         n_tok = steps * C
         return {"ms": ms_max, "tokens": n_tok * self.world, "tok_s": n_tok * self.world / (ms_max / 1e3),
                 "exit_rate": float(np.mean(timed >= 0)) if len(ro) else 0.0,
@@ -453,7 +474,7 @@ def run_ours(args, rank: int, world: int, local: int):
     kms = eng.profile_kernels(iters=2 * shape.n_layers)
     T_prof = eng.position + 1
     kb = kernel_bytes(run.dims, T_prof, shape.readout_layers[0])
-    per_tok = kernel_launches_per_token(shape.n_layers, shape.readout_layers[0], head["exit_rate"])
+    per_tok = kernel_launches_per_token(shape.n_layers, shape.readout_layers[0], head["exit_rate"], eng.persistent)
     share = {k: kms[k] * per_tok[k] for k in kms}
     dom = max(share, key=share.get)
     peak = _peaks()
@@ -519,8 +540,8 @@ def profile_run(args, local: int):
         eng.decode_n(C, [0.5], schedule=sched[i * C:(i + 1) * C], where=DEVICE)
     eng.sync()
     L = shape.n_layers
-    prefill_launches = 1 + P * (5 * L + 1) + 2
-    decode = sum(step_launches(L, shape.readout_layers, 0 if e else -1) for e in (sched >= 2)) + 2
+    prefill_launches = 1 + P * (layer_launches(L, [0, L], eng.persistent) + 1) + 2
+    decode = sum(step_launches(L, shape.readout_layers, 0 if e else -1, eng.persistent) for e in (sched >= 2)) + 2
     print(json.dumps({"prefill_launches": prefill_launches, "decode_launches": decode, "tokens": 2 * C}))
 
 

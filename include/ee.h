@@ -199,6 +199,11 @@ int ee_position(ee_ctx* ctx, int32_t* pos);
                                  0: direct launches, branch decided on the host */
 #define EE_OPT_PDL 2          /* 1 (default): programmatic dependent launch    */
 #define EE_OPT_DEBUG_LOGITS 3 /* 1: keep each step's readout and final logits  */
+#define EE_OPT_PERSISTENT 4   /* 1 (default where supported): each run of layers
+                                 between readouts is one persistent launch, one
+                                 CTA per SM streaming weights through a shared-
+                                 memory ring; 0: five launches per layer.
+                                 EE_EINVAL if the shape is not supported      */
 int ee_set_option(ee_ctx* ctx, int option, int value);
 
 #define EE_DBG_HIDDEN_READOUT 1 /* layer = readout r: residual h_k it read, d floats   */
@@ -222,7 +227,9 @@ int ee_debug_read(ee_ctx* ctx, int what, int layer, int pos, void* host_dst, siz
 #define EE_KERNEL_READOUT 5  /* readout affine map                                  */
 #define EE_KERNEL_VOCAB 6    /* unembedding pass with the confidence statistics     */
 #define EE_KERNEL_KVFILL 7   /* KV fill of the layers above the first readout       */
-#define EE_NUM_KERNELS 8
+#define EE_KERNEL_LAYERS 8   /* persistent kernel over layers 1..k (first readout);
+                                0 when the shape does not support it               */
+#define EE_NUM_KERNELS 9
 /* Average device time (ms) of each decode kernel, from CUDA events around
  * `iters` back-to-back direct launches on the context's stream, cycling
  * through the layers so consecutive launches read different weights.  No

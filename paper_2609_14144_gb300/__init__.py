@@ -11,8 +11,8 @@ import ctypes
 import numpy as np
 
 from . import _lib
-from ._lib import (DEVICE, FORCE_FULL, FREE, HOST, MAX_READOUTS, OPT_DEBUG_LOGITS, OPT_GRAPHS, OPT_PDL, EEError,
-                   FORCE_EXIT_AT, check)
+from ._lib import (DEVICE, FORCE_FULL, FREE, HOST, MAX_READOUTS, OPT_DEBUG_LOGITS, OPT_GRAPHS, OPT_PDL,
+                   OPT_PERSISTENT, EEError, FORCE_EXIT_AT, check)
 
 __all__ = ["Engine", "EEError", "FREE", "FORCE_FULL", "FORCE_EXIT_AT", "HOST", "DEVICE", "attention_decode",
            "vocab_confidence", "library_path"]
@@ -53,6 +53,8 @@ class Engine:
                                      self.workspace_bytes, ctypes.c_void_p(self.stream.cuda_stream),
                                      ctypes.byref(ctx)))
         self.ctx = ctx
+        # the persistent layer kernel is on by default where the shape allows it
+        self.persistent = self.lib.ee_set_option(self.ctx, OPT_PERSISTENT, 1) == 0
         self.n_readouts = 0
         self.readout_layers = []
         self.load_weights(model)
@@ -97,6 +99,8 @@ class Engine:
 
     def set_option(self, option: int, value: int):
         check(self.lib.ee_set_option(self.ctx, option, int(value)))
+        if option == OPT_PERSISTENT:
+            self.persistent = bool(value)
 
     def set_page_table(self, pages):
         p = np.ascontiguousarray(pages, dtype=np.int32)

@@ -10,7 +10,7 @@ MAX_READOUTS = 8
 EE_OK, EE_EINVAL, EE_ENOMEM, EE_ECUDA, EE_ERANGE, EE_EDEVICE, EE_ESTATE = 0, -1, -2, -3, -4, -5, -6
 FREE, FORCE_FULL = 0, 1
 HOST, DEVICE = 0, 1
-OPT_GRAPHS, OPT_PDL, OPT_DEBUG_LOGITS = 1, 2, 3
+OPT_GRAPHS, OPT_PDL, OPT_DEBUG_LOGITS, OPT_PERSISTENT = 1, 2, 3, 4
 DBG_HIDDEN_READOUT, DBG_READOUT_Y, DBG_HIDDEN_FINAL, DBG_READOUT_LOGITS, DBG_FINAL_LOGITS, DBG_KV, DBG_KV_SRC = \
     1, 2, 3, 4, 5, 6, 7
 
@@ -20,7 +20,7 @@ SYMBOLS = ("ee_workspace_bytes", "ee_create", "ee_destroy", "ee_last_error", "ee
            "ee_get_stats", "ee_position", "ee_set_option", "ee_debug_read", "ee_attention_scratch_bytes",
            "ee_attention_decode", "ee_vocab_scratch_bytes", "ee_vocab_confidence", "ee_profile_kernels",
            "ee_attention_decode_static")
-KERNELS = ("qkv", "attention", "oproj", "gateup", "down", "readout", "vocab", "kvfill")
+KERNELS = ("qkv", "attention", "oproj", "gateup", "down", "readout", "vocab", "kvfill", "layers")
 
 
 def FORCE_EXIT_AT(r: int) -> int:

@@ -58,6 +58,7 @@ struct Layout {
     size_t ctl, rope, layers, embed, lm_head, g_final, ro_w[kMaxReadouts], ro_b[kMaxReadouts];
     size_t kpool, vpool, page_table, kv_src, h, q, o, a, y, hk, logits_ro, logits_final;
     size_t gemv_part, gemv_ticket, attn_part, attn_ticket, vocab_part, vocab_ticket;
+    size_t seg_part[4], seg_hbuf, seg_sync;
     size_t prompt, sched, out_tok, out_exit, out_conf, total;
     int64_t layer_stride, off_wqkv, off_bqkv, off_gattn, off_wo, off_gmlp, off_wgu, off_wd;
     int64_t n_units_qkv, kv_layer_stride, gemv_ticket_stride;
@@ -147,6 +148,13 @@ Layout make_layout(const ee_model_config& c) {
     l.attn_ticket = take(4 * (size_t)KH);
     l.vocab_part = take(4 * (size_t)kMaxVocabCtas * 4);
     l.vocab_ticket = take(4);
+    {   // persistent layer kernel: tile partials of Q/K/V, O, gate/up, down
+        const int64_t rows[4] = {(A + 2 * KH) * D, d, 2 * F, d}, Ks[4] = {d, A * D, d, F};
+        for (int i = 0; i < 4; ++i)
+            l.seg_part[i] = take(4 * (size_t)tile_count(rows[i]) * ((Ks[i] + 255) / 256) * kTileRows);
+        l.seg_hbuf = take(4 * 2 * (size_t)d);
+        l.seg_sync = take(4 * (size_t)(5 * L + 8));
+    }
     l.prompt = take(4 * (size_t)c.max_ctx);
     l.sched = take((size_t)c.max_ctx);
     l.out_tok = take(4 * (size_t)c.max_ctx);
@@ -206,6 +214,8 @@ struct ee_ctx {
     bool weights = false, started = false, prefilled = false;
     int pos = 0;
     bool use_graphs = true, use_pdl = true;
+    bool seg_ok = false, use_persistent = true;  // persistent layer kernel supported / chosen
+    SegPlan seg{};
     int dbg = 0;
     cudaGraphExec_t g_step = nullptr, g_n = nullptr, g_prefill = nullptr;
     int grid_gemv = 0, grid_vocab = 0;
@@ -293,6 +303,11 @@ int enqueue_layers(ee_ctx* c, cudaStream_t s, int j0, int j1, bool& pdl) {
               gd = gemv_grid(c, d, F);
     const bool wq = gemv_whole(c, nqkv, d), wo = gemv_whole(c, d, AD), wu = gemv_whole(c, 2 * F, d),
                wd = gemv_whole(c, d, F);
+    if (c->seg_ok && c->use_persistent && j1 > j0) {
+        EE_CK(launch_layers(m, c->seg, j0, j1, j0 == 0 ? 1 : 0, s));
+        pdl = c->use_pdl;
+        return EE_OK;
+    }
     for (int j = j0; j < j1; ++j) {
         EE_CK(launch_qkv(m, j, j == 0 ? 1 : 0, gq, wq, pdl, s));
         pdl = c->use_pdl;
@@ -536,6 +551,7 @@ int device_error(const ee_ctx* c) {
     if (e & kErrNanConfidence) m += " non-finite confidence;";
     if (e & kErrTokenRange) m += " token out of range;";
     if (e & kErrPosition) m += " position beyond max_ctx;";
+    if (e & kErrStall) m += " a wait of the persistent layer kernel timed out (call ee_reset);";
     return fail(EE_EDEVICE, m);
 }
 
@@ -682,6 +698,15 @@ int ee_create(const ee_model_config* cfg, void* d_workspace, size_t workspace_by
     const int kmax = std::max({2 * m.d, m.A * m.D, m.F});
     if (configure_kernels(kmax) != cudaSuccess) return bail(fail(EE_ECUDA, "kernel configuration failed"));
     c->attn_cluster = attention_cluster_size(m.D, m.KH);
+    if (seg_plan(m, c->n_sm, c->seg) && configure_layers(c->seg.smem) == cudaSuccess &&
+        layers_blocks_per_sm(c->seg.smem) >= 1) {
+        for (int i = 0; i < 4; ++i) c->seg.part[i] = (float*)(w + l.seg_part[i]);
+        c->seg.attn_part = m.attn_part;
+        c->seg.hbuf = (float*)(w + l.seg_hbuf);
+        c->seg.sync = (unsigned*)(w + l.seg_sync);
+        c->seg_ok = true;
+    }
+    cudaGetLastError();
 
     // RoPE table: angle t * base^(-2i/D) in double, cos/sin rounded to fp32.
     std::vector<float2> rope((size_t)m.max_ctx * (m.D / 2));
@@ -838,6 +863,8 @@ int ee_reset(ee_ctx* c) {
     c->h_ctl->max_ctx = c->cfg.max_ctx;
     EE_CK(cudaMemcpyAsync(c->d_ctl, c->h_ctl, sizeof(Ctl), cudaMemcpyHostToDevice, c->stream));
     EE_CK(cudaMemsetAsync(c->ws + c->lay.kv_src, 0, (size_t)c->cfg.n_layers * c->cfg.max_ctx, c->stream));
+    // phase counters of the persistent layer kernel (left set by a timed-out wait)
+    EE_CK(cudaMemsetAsync(c->ws + c->lay.seg_sync, 0, 4 * (size_t)(5 * c->cfg.n_layers + 8), c->stream));
     EE_CK(cudaStreamSynchronize(c->stream));
     c->pos = 0;
     c->prefilled = false;
@@ -856,6 +883,11 @@ int ee_set_option(ee_ctx* c, int option, int value) {
             return EE_OK;
         case EE_OPT_DEBUG_LOGITS:
             c->dbg = value != 0;
+            return EE_OK;
+        case EE_OPT_PERSISTENT:
+            if (value && !c->seg_ok) return fail(EE_EINVAL, "the persistent layer kernel does not support this shape");
+            if (c->use_persistent != (value != 0)) drop_graphs(c);
+            c->use_persistent = value != 0;
             return EE_OK;
         default:
             return fail(EE_EINVAL, "unknown option");
@@ -1100,6 +1132,9 @@ int ee_profile_kernels(ee_ctx* c, int iters, float* ms_out) {
                 case EE_KERNEL_READOUT:
                     return launch_readout(m, i % c->n_readouts, gr, gemv_whole(c, d, d), false, s);
                 case EE_KERNEL_VOCAB: return launch_vocab(va, c->grid_vocab, false, s);
+                case EE_KERNEL_LAYERS:
+                    if (!c->seg_ok) return cudaSuccess;
+                    return launch_layers(m, c->seg, 0, c->ro_layer[0], 0, s);
                 default: {
                     const int e = c->ro_layer[0];
                     if (e >= L) return cudaSuccess;

@@ -20,6 +20,7 @@ constexpr int kErrNanConfidence = 1;
 constexpr int kErrTokenRange = 2;
 constexpr int kErrPosition = 4;
 constexpr int kErrShape = 8;  // a GEMV CTA would touch more tiles than it can hold
+constexpr int kErrStall = 16; // a wait of the persistent layer kernel ran out of time
 
 // Device-resident control block: everything a step reads or writes that is
 // not a tensor, so one captured graph serves every step, tau and force.
@@ -160,6 +161,34 @@ cudaError_t launch_prefill_advance(const DevModel& m, int has_cond, cudaGraphCon
                                    cudaStream_t s);
 cudaError_t launch_prefill_end(const DevModel& m, bool pdl, cudaStream_t s);
 cudaError_t launch_set_inputs(Ctl* c, const CtlInputs& in, cudaStream_t s);
+
+// Persistent layer-segment kernel (ee_persist.cu): one CTA per SM, warps
+// 0..7 consume a shared-memory ring that warp 8 fills with cp.async.bulk.
+constexpr int kSegConsumerWarps = 8;
+constexpr int kSegThreads = 32 * (kSegConsumerWarps + 1);
+constexpr int kSegChunk = 16384;   // bytes per ring stage: 32 rows x 256 bf16 columns
+constexpr int kSegMaxSplits = 32;  // attention splits per kv head (at most)
+constexpr int kSegMaxGroup = 8;    // query heads per kv head (at most)
+struct SegPlan {
+    int G;                  // CTAs (one per SM)
+    int stages;             // ring stages
+    int max_pps;            // attention pages per split (at most)
+    int rows_per_kv_chunk;  // cache positions per ring chunk
+    int n_tiles[4], n_chunks[4], K[4];  // Q/K/V, O, gate/up, down
+    float* part[4];         // per-matrix tile partials [tile][n_chunks][32]
+    float* attn_part;       // [A][kAttnMaxSplits][D + 2]
+    float* hbuf;            // [2][d] residual at each layer's input
+    unsigned* sync;         // [5 L + 1] phase counters and the exit ticket, zero between launches
+    size_t smem;            // dynamic shared memory per CTA
+};
+// Geometry and shared-memory plan for `m` on n_sm SMs (pointers left
+// unset); false if the shape is outside what the kernel supports.
+bool seg_plan(const DevModel& m, int n_sm, SegPlan& p);
+cudaError_t configure_layers(size_t smem);
+int layers_blocks_per_sm(size_t smem);
+// Layers [j0, j1) of the step at ctl->pos; `first`: layer j0 takes the
+// embedding of ctl->in_tok.  A cooperative launch of p.G CTAs.
+cudaError_t launch_layers(const DevModel& m, const SegPlan& p, int j0, int j1, int first, cudaStream_t s);
 
 // Record `msg` as the calling thread's last error and return `code`.
 int set_last_error(int code, const char* msg);

@@ -65,3 +65,12 @@ def test_launch_and_byte_accounting_agree_with_the_cost_model():
     assert per_token_full == pytest.approx(model_full, rel=2e-3)
     lt = bench.kernel_launches_per_token(L, k, 0.5)
     assert lt["gateup"] == k + 0.5 * (L - k) and lt["vocab"] == 1.5 and lt["kvfill"] == 0.5
+    # persistent layer kernel: one launch per run of layers between readouts
+    assert bench.step_launches(L, [k], -1, True) == 2 + 2 + 1 + 1
+    assert bench.step_launches(L, [k], 0, True) == 1 + 2 + 1 + 1
+    assert bench.step_launches(L, [7, 14, 21], 1, True) == 2 + 4 + 1 + 1
+    assert bench.step_launches(L, [L], -1, True) == 1 + 2 + 1 + 1
+    lp = bench.kernel_launches_per_token(L, k, 0.5, True)
+    assert lp["qkv"] == 0 and lp["layers"] == 1 + 0.5 * (L - k) / k
+    per_token_pers = kb["layers"] * L / k + kb["readout"] + 2 * kb["vocab"]
+    assert per_token_pers == pytest.approx(model_full, rel=2e-3)
