@@ -58,7 +58,7 @@ struct Layout {
     size_t ctl, rope, layers, embed, lm_head, g_final, ro_w[kMaxReadouts], ro_b[kMaxReadouts];
     size_t kpool, vpool, page_table, kv_src, h, q, o, a, y, hk, logits_ro, logits_final;
     size_t gemv_part, gemv_ticket, attn_part, attn_ticket, vocab_part, vocab_ticket;
-    size_t seg_part[4], seg_hbuf, seg_sync;
+    size_t seg_dpart, seg_hmid, seg_sync;
     size_t prompt, sched, out_tok, out_exit, out_conf, total;
     int64_t layer_stride, off_wqkv, off_bqkv, off_gattn, off_wo, off_gmlp, off_wgu, off_wd;
     int64_t n_units_qkv, kv_layer_stride, gemv_ticket_stride;
@@ -148,13 +148,10 @@ Layout make_layout(const ee_model_config& c) {
     l.attn_ticket = take(4 * (size_t)KH);
     l.vocab_part = take(4 * (size_t)kMaxVocabCtas * 4);
     l.vocab_ticket = take(4);
-    {   // persistent layer kernel: tile partials of Q/K/V, O, gate/up, down
-        const int64_t rows[4] = {(A + 2 * KH) * D, d, 2 * F, d}, Ks[4] = {d, A * D, d, F};
-        for (int i = 0; i < 4; ++i)
-            l.seg_part[i] = take(4 * (size_t)tile_count(rows[i]) * ((Ks[i] + 255) / 256) * kTileRows);
-        l.seg_hbuf = take(4 * 2 * (size_t)d);
-        l.seg_sync = take(4 * (size_t)(5 * L + 8));
-    }
+    // persistent layer kernel: down-projection partials, mid residual, counters
+    l.seg_dpart = take(4 * (size_t)tile_count(d) * ((F + 255) / 256) * kTileRows);
+    l.seg_hmid = take(4 * (size_t)d);
+    l.seg_sync = take(4 * (size_t)(5 * L + 8));
     l.prompt = take(4 * (size_t)c.max_ctx);
     l.sched = take((size_t)c.max_ctx);
     l.out_tok = take(4 * (size_t)c.max_ctx);
@@ -214,7 +211,7 @@ struct ee_ctx {
     bool weights = false, started = false, prefilled = false;
     int pos = 0;
     bool use_graphs = true, use_pdl = true;
-    bool seg_ok = false, use_persistent = true;  // persistent layer kernel supported / chosen
+    bool seg_ok = false, use_persistent = false;  // persistent layer kernel supported / chosen
     SegPlan seg{};
     int dbg = 0;
     cudaGraphExec_t g_step = nullptr, g_n = nullptr, g_prefill = nullptr;
@@ -700,9 +697,9 @@ int ee_create(const ee_model_config* cfg, void* d_workspace, size_t workspace_by
     c->attn_cluster = attention_cluster_size(m.D, m.KH);
     if (seg_plan(m, c->n_sm, c->seg) && configure_layers(c->seg.smem) == cudaSuccess &&
         layers_blocks_per_sm(c->seg.smem) >= 1) {
-        for (int i = 0; i < 4; ++i) c->seg.part[i] = (float*)(w + l.seg_part[i]);
+        c->seg.dpart = (float*)(w + l.seg_dpart);
         c->seg.attn_part = m.attn_part;
-        c->seg.hbuf = (float*)(w + l.seg_hbuf);
+        c->seg.hmid = (float*)(w + l.seg_hmid);
         c->seg.sync = (unsigned*)(w + l.seg_sync);
         c->seg_ok = true;
     }

@@ -17,17 +17,20 @@
 // the producer runs ahead of the data dependencies and HBM stays busy while
 // the consumers wait for one.  Warps 0..7 consume the ring in the same order.
 //
-// Phases hand results to each other through global memory: a phase writes
-// per-tile partial sums ([tile][slot][32], one slot per CTA that covered part
-// of the tile), bumps a completion counter with a release, and the next
-// phase's CTAs acquire the counter once every CTA has bumped it and rebuild
-// exactly the inputs they need by summing the slots in slot order (the
-// result does not depend on timing).  The residual stream is never updated
-// in place inside the segment: h_in of layer j lives in hbuf[j & 1] and
-// h_out = h_in + (O-projection slots) + (down slots), rebuilt by whoever
-// reads it; the last phase writes h_out of the last layer to the model's h.
+// Phases hand results to each other through global memory and completion
+// counters: a CTA bumps a phase's counter with a release once its share is
+// written, and a consumer of the phase acquires the counter once every CTA
+// has bumped it.  Q/K/V, O and gate/up are split by whole 32-row tiles, so
+// each tile's epilogue (bias, RoPE and the KV append; the residual add;
+// SiLU(gate) * up) runs in the CTA that owns it.  The down projection has
+// few, long rows: it is split into (tile, chunk) items over all CTAs, each
+// writing the partial sums of the tiles it touched into its slot
+// [tile][slot][32]; the next layer's Q/K/V tiles and the O-projection
+// epilogue add the slots in slot order (no dependence on timing).  The
+// attention of kv head g over the step's positions is split over CTAs by
+// pages; the O tiles merge the splits (flash-decoding combine).
 //
-// Every wait is bounded: after kStallNs the waiting thread sets kErrStall in
+// Every wait is bounded: after kStallCycles the waiting thread sets kErrStall in
 // the control block and the CTA winds down (the producer first waits, again
 // with a bound, for the copies it still has in flight).  Co-residency of all
 // CTAs, which the cross-CTA waits rely on, comes from a cooperative launch.
@@ -44,7 +47,11 @@ namespace {
 constexpr int kCW = kSegConsumerWarps;
 constexpr int kCT = 32 * kCW;              // consumer threads
 constexpr int kColsPerChunk = kSegChunk / (2 * kTileRows);  // 256
-constexpr unsigned long long kStallNs = 2000000000ull;     // 2 s
+// Wait bounds in SM clock cycles (clock64 is cheap to read; the global
+// timer and the error word in global memory are not, so a waiting thread
+// looks at them only about once per millisecond).
+constexpr long long kStallCycles = 4000000000ll;  // about 2 s
+constexpr long long kCheckCycles = 2000000ll;     // about 1 ms
 
 enum { kPhQKV = 0, kPhAttn = 1, kPhO = 2, kPhGU = 3, kPhDn = 4, kPhases = 5 };
 
@@ -54,11 +61,19 @@ __device__ __forceinline__ float bfhi(uint32_t v) { return __uint_as_float(v & 0
 __device__ __forceinline__ uint16_t tobf(float f) { return __bfloat16_as_ushort(__float2bfloat16_rn(f)); }
 __device__ __forceinline__ float round_bf(float f) { return bf(tobf(f)); }
 
-__device__ __forceinline__ unsigned long long now_ns() {
-    unsigned long long t;
-    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-    return t;
-}
+__device__ __forceinline__ long long cycles() { return clock64(); }
+// Bookkeeping of a bounded wait: true once the wait has run out of time or
+// another thread has flagged a stall.
+struct Bound {
+    long long t0, tc;
+    __device__ __forceinline__ Bound() : t0(cycles()), tc(t0) {}
+    __device__ __forceinline__ bool expired(const volatile int* err) {
+        const long long t = cycles();
+        if (t - tc < kCheckCycles) return false;
+        tc = t;
+        return (*err & kErrStall) || t - t0 > kStallCycles;
+    }
+};
 __device__ __forceinline__ uint32_t saddr(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
 
 // ---------------------------------------------------------------- mbarriers
@@ -78,10 +93,31 @@ __device__ __forceinline__ bool mb_test(uint64_t* b, int parity) {
 // limit or once another thread has flagged a stall.
 __device__ __forceinline__ bool mb_wait(uint64_t* b, int parity, const volatile int* err) {
     if (mb_test(b, parity)) return true;
-    const unsigned long long t0 = now_ns();
+    Bound bd;
     for (unsigned it = 1;; ++it) {
         if (mb_test(b, parity)) return true;
-        if ((it & 63) == 0 && ((*err & kErrStall) || now_ns() - t0 > kStallNs)) return false;
+        if ((it & 15) == 0 && bd.expired(err)) return false;
+    }
+}
+// Non-blocking test with a sleeping back-off, for the producer: it waits
+// for ring space while the consumers work, and must not compete with them
+// for issue slots or the shared-memory pipe.
+__device__ __forceinline__ bool mb_probe(uint64_t* b, int parity) {
+    uint32_t ok;
+    asm volatile(
+        "{ .reg .pred p; mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p; }"
+        : "=r"(ok)
+        : "r"(saddr(b)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+__device__ __forceinline__ bool mb_wait_sleep(uint64_t* b, int parity, const volatile int* err) {
+    if (mb_probe(b, parity)) return true;
+    Bound bd;
+    for (unsigned it = 1;; ++it) {
+        __nanosleep(32);
+        if (mb_probe(b, parity)) return true;
+        if ((it & 15) == 0 && bd.expired(err)) return false;
     }
 }
 __device__ __forceinline__ void mb_arrive(uint64_t* b) {
@@ -110,6 +146,29 @@ __device__ __forceinline__ uint64_t evict_normal() {
     return pol;
 }
 
+// Explicit shared-memory loads (32-bit shared-window addresses).
+__device__ __forceinline__ uint4 lds128(uint32_t a) {
+    uint4 v;
+    asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(a));
+    return v;
+}
+__device__ __forceinline__ float4 lds128f(uint32_t a) {
+    float4 v;
+    asm volatile("ld.shared.v4.f32 {%0,%1,%2,%3}, [%4];" : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(a));
+    return v;
+}
+__device__ __forceinline__ uint2 lds64(uint32_t a) {
+    uint2 v;
+    asm volatile("ld.shared.v2.u32 {%0,%1}, [%2];" : "=r"(v.x), "=r"(v.y) : "r"(a));
+    return v;
+}
+__device__ __forceinline__ uint32_t lds32(uint32_t a) {
+    uint32_t v;
+    asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(a));
+    return v;
+}
+__device__ __forceinline__ float ldsf(uint32_t a) { return __uint_as_float(lds32(a)); }
+
 // Barrier of the consumer warps only (the producer never joins it).
 __device__ __forceinline__ void csync() { asm volatile("bar.sync 1, %0;" ::"r"(kCT) : "memory"); }
 
@@ -122,6 +181,19 @@ __device__ __forceinline__ float warp_max(float v) {
 #pragma unroll
     for (int o = 16; o; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
     return v;
+}
+__device__ __forceinline__ float dot8s(const uint4 w, uint32_t xa) {
+    const float4 a = lds128f(xa);
+    const float4 b = lds128f(xa + 16);
+    float s = bflo(w.x) * a.x;
+    s = fmaf(bfhi(w.x), a.y, s);
+    s = fmaf(bflo(w.y), a.z, s);
+    s = fmaf(bfhi(w.y), a.w, s);
+    s = fmaf(bflo(w.z), b.x, s);
+    s = fmaf(bfhi(w.z), b.y, s);
+    s = fmaf(bflo(w.w), b.z, s);
+    s = fmaf(bfhi(w.w), b.w, s);
+    return s;
 }
 __device__ __forceinline__ float dot8(const uint4 w, const float* x) {
     const float4 a = *reinterpret_cast<const float4*>(x);
@@ -138,17 +210,30 @@ __device__ __forceinline__ float dot8(const uint4 w, const float* x) {
 }
 
 // ------------------------------------------------------------ work geometry
-// Matrix mt of layer j as ring items: item i = (tile i / nc, chunk i % nc).
-// Items are split into contiguous ranges over Ge = min(G, N) CTAs.
+// Q/K/V, O and gate/up are split by whole 32-row tiles: rank r < Ge =
+// min(G, n_tiles) owns tiles [r n / Ge, (r + 1) n / Ge) and runs on CTA
+// r G / Ge, so each of those phases finishes its rows in one CTA and applies
+// its epilogue there.  The down projection (few rows, long rows) is split
+// into (tile, 256-column chunk) items over all CTAs; each CTA writes the
+// partial sums of the tiles it touched into its slot [tile][slot][32].
+__device__ __forceinline__ void whole_tiles(int n_t, int G, int cta, int& t0, int& t1) {
+    const int Ge = min(G, n_t);
+    const int r = (int)(((int64_t)cta * Ge + G - 1) / G);
+    if (r < Ge && (int)((int64_t)r * G / Ge) == cta) {
+        t0 = (int)((int64_t)r * n_t / Ge);
+        t1 = (int)((int64_t)(r + 1) * n_t / Ge);
+    } else {
+        t0 = t1 = 0;
+    }
+}
 struct Items {
-    int N, Ge, lo, hi, nc, K, n_tiles;
+    int N, Ge, lo, hi, nc, K;
 };
-__device__ __forceinline__ Items items_of(const SegPlan& p, int mt, int cta) {
+__device__ __forceinline__ Items down_items(const SegPlan& p, int cta) {
     Items it;
-    it.nc = p.n_chunks[mt];
-    it.K = p.K[mt];
-    it.n_tiles = p.n_tiles[mt];
-    it.N = it.n_tiles * it.nc;
+    it.nc = p.n_chunks[3];
+    it.K = p.K[3];
+    it.N = p.n_tiles[3] * it.nc;
     it.Ge = min(p.G, it.N);
     if (cta < it.Ge) {
         it.lo = (int)((int64_t)cta * it.N / it.Ge);
@@ -162,27 +247,12 @@ __device__ __forceinline__ Items items_of(const SegPlan& p, int mt, int cta) {
 __device__ __forceinline__ int item_owner(const Items& it, int i) {
     return (int)(((int64_t)(i + 1) * it.Ge - 1) / it.N);
 }
-__device__ __forceinline__ int tile_slots(const Items& it, int t) {
-    return item_owner(it, t * it.nc + it.nc - 1) - item_owner(it, t * it.nc) + 1;
-}
-// Sum of the slots of row `lane` of tile t (slot order, so deterministic).
-__device__ __forceinline__ float slot_sum(const float* part, const Items& it, int t, int lane) {
-    const int ns = tile_slots(it, t);
-    const float* q = part + (int64_t)t * it.nc * 32 + lane;
-    float s = 0.f;
-    for (int k = 0; k < ns; ++k) s += q[k * 32];
-    return s;
-}
-__device__ __forceinline__ uint32_t chunk_bytes(const Items& it, int c) {
-    return (uint32_t)min(kColsPerChunk, it.K - c * kColsPerChunk) * (2 * kTileRows);
-}
-
-__device__ __forceinline__ const uint8_t* layer_bytes(const DevModel& m, int j, int64_t off) {
-    return reinterpret_cast<const uint8_t*>(m.layers + (int64_t)j * m.layer_stride + off);
+__device__ __forceinline__ uint32_t chunk_bytes(int K, int c) {
+    return (uint32_t)min(kColsPerChunk, K - c * kColsPerChunk) * (2 * kTileRows);
 }
 __device__ __forceinline__ const uint8_t* mat_base(const DevModel& m, int j, int mt) {
     const int64_t off = mt == 0 ? m.off_wqkv : mt == 1 ? m.off_wo : mt == 2 ? m.off_wgu : m.off_wd;
-    return layer_bytes(m, j, off);
+    return reinterpret_cast<const uint8_t*>(m.layers + (int64_t)j * m.layer_stride + off);
 }
 
 // Attention work of one step: kv head g, split s covers logical pages
@@ -201,9 +271,7 @@ __device__ __forceinline__ AttnGeo attn_geo(const DevModel& m, const SegPlan& p,
     a.U = m.KH * a.splits;
     return a;
 }
-// Attention unit of this CTA, or -1.
 __device__ __forceinline__ int attn_unit(const AttnGeo& a, int G, int cta) {
-    // u * G / U == cta  <=>  u = ceil(cta * U / G) when that u maps back to cta
     const int u = (int)(((int64_t)cta * a.U + G - 1) / G);
     if (u < a.U && (int)((int64_t)u * G / a.U) == cta) return u;
     return -1;
@@ -214,14 +282,16 @@ struct Smem {
     uint8_t* ring;      // stages x kSegChunk
     uint64_t* full;     // [stages]
     uint64_t* empty;    // [stages]
-    float* xs;          // [d] normalised input of Q/K/V and gate/up
+    float* xs;          // [max(d, A D)] input vector of a whole-tile phase
     float* hs;          // [d] residual
-    float* xc;          // [256] input columns of an O-projection or down chunk
+    float* xa;          // [max down items][256] staged input columns of the down items
     float* red;         // [2][kCW][32]
-    float* qa;          // [group][D] rotated queries of the attention unit
-    float* kv;          // [2][D] k, v of the step's position (bf16 values)
+    float* qa;          // [group][D] scaled queries of the attention unit
+    float* kv;          // [2][D] k, v of the step's position
     float* sc;          // [group][pps * page_size] scores, then probabilities
     float* ml;          // [group][2] max, sum
+    float* wts;         // [A][kSegMaxSplits] split weights of the attention merge, then [A] denominators
+    uint8_t* nsd;       // [down tiles] slots per down tile
 };
 __device__ __forceinline__ Smem carve(uint8_t* base, const DevModel& m, const SegPlan& p) {
     Smem s;
@@ -234,11 +304,11 @@ __device__ __forceinline__ Smem carve(uint8_t* base, const DevModel& m, const Se
     q += 8 * p.stages;
     float* f = reinterpret_cast<float*>(q);
     s.xs = f;
-    f += (m.d + 3) & ~3;
+    f += (max(m.d, m.A * m.D) + 3) & ~3;
     s.hs = f;
     f += (m.d + 3) & ~3;
-    s.xc = f;
-    f += kColsPerChunk;
+    s.xa = f;
+    f += p.max_dn_items * kColsPerChunk;
     s.red = f;
     f += 2 * kCW * 32;
     const int grp = m.A / m.KH;
@@ -249,36 +319,76 @@ __device__ __forceinline__ Smem carve(uint8_t* base, const DevModel& m, const Se
     s.sc = f;
     f += grp * p.max_pps * m.page_size;
     s.ml = f;
+    f += 2 * grp;
+    s.wts = f;
+    f += m.A * (kSegMaxSplits + 1);
+    s.nsd = reinterpret_cast<uint8_t*>(f);
     return s;
 }
 
 // ------------------------------------------------------------ the producer
+// Ring positions advance by one stage per chunk; (stage, parity) pairs are
+// kept incrementally (no division in the per-chunk path).
+struct RingPos {
+    int st = 0, ph = 0;
+    __device__ __forceinline__ void next(int stages) {
+        if (++st == stages) {
+            st = 0;
+            ph ^= 1;
+        }
+    }
+};
 struct Producer {
     const Smem& s;
-    int stages;
-    long long n;  // chunks issued
+    int stages, inflight;
+    long long n;   // chunks issued
+    RingPos head;  // stage of the next chunk
+    RingPos tail;  // stage of chunk n - inflight (once n >= inflight)
     uint64_t pol_w, pol_kv;
-    const volatile int* err;
+    volatile int* err;
     bool ok = true;
-    __device__ Producer(const Smem& sm, int st, const volatile int* e)
-        : s(sm), stages(st), n(0), pol_w(evict_first()), pol_kv(evict_normal()), err(e) {}
+    __device__ Producer(const Smem& sm, int st, int infl, volatile int* e)
+        : s(sm), stages(st), inflight(infl), n(0), pol_w(evict_first()), pol_kv(evict_normal()), err(e) {}
     __device__ __forceinline__ void push(const void* src, uint32_t bytes, uint64_t pol) {
         if (!ok) return;
-        const int st = (int)(n % stages);
-        if (n >= stages && !mb_wait(&s.empty[st], (int)(((n / stages) - 1) & 1), err)) {
+        // at most `inflight` copies outstanding: the ring still runs up to
+        // `stages` chunks ahead, but the copies queued in HBM stay few
+        if (n >= inflight) {
+            if (!mb_wait_sleep(&s.full[tail.st], tail.ph, err)) {
+                atomicOr((int*)err, kErrStall);
+                ok = false;
+                return;
+            }
+            tail.next(stages);
+        }
+        // the stage is free once the consumers released its previous chunk
+        if (n >= stages && !mb_wait_sleep(&s.empty[head.st], head.ph ^ 1, err)) {
             atomicOr((int*)err, kErrStall);
             ok = false;
             return;
         }
-        mb_expect_tx(&s.full[st], bytes);
-        bulk_load(s.ring + (size_t)st * kSegChunk, src, bytes, &s.full[st], pol);
+        mb_expect_tx(&s.full[head.st], bytes);
+        bulk_load(s.ring + (size_t)head.st * kSegChunk, src, bytes, &s.full[head.st], pol);
+        head.next(stages);
         ++n;
     }
+    __device__ __forceinline__ void tiles(const uint8_t* W, int K, int nc, int t0, int t1) {
+        for (int t = t0; t < t1; ++t)
+            for (int c = 0; c < nc; ++c)
+                push(W + (int64_t)t * kTileRows * K * 2 + (int64_t)c * kSegChunk, chunk_bytes(K, c), pol_w);
+    }
     // Before leaving: every issued copy has landed (the consumers normally
-    // see to that; after a stall they may not have).
+    // see to that; after a stall they may not have).  Walks back over the
+    // last min(n, stages) chunks.
     __device__ void drain() {
-        for (long long i = max(0ll, n - stages); i < n; ++i)
-            mb_wait(&s.full[i % stages], (int)((i / stages) & 1), err);
+        RingPos q = head;
+        for (long long i = 0; i < min(n, (long long)stages); ++i) {
+            if (--q.st < 0) {
+                q.st = stages - 1;
+                q.ph ^= 1;
+            }
+            mb_wait(&s.full[q.st], q.ph, err);
+        }
     }
 };
 
@@ -286,22 +396,21 @@ struct Producer {
 struct Consumer {
     const Smem& s;
     int stages;
-    long long n;
+    RingPos pos;
     volatile int* err;
     bool ok = true;
-    __device__ Consumer(const Smem& sm, int st, volatile int* e) : s(sm), stages(st), n(0), err(e) {}
-    __device__ __forceinline__ const uint8_t* acquire() {
-        const int st = (int)(n % stages);
-        if (ok && !mb_wait(&s.full[st], (int)((n / stages) & 1), err)) {
+    __device__ Consumer(const Smem& sm, int st, volatile int* e) : s(sm), stages(st), err(e) {}
+    __device__ __forceinline__ const uint4* acquire() {
+        if (ok && !mb_wait(&s.full[pos.st], pos.ph, err)) {
             atomicOr((int*)err, kErrStall);
             ok = false;
         }
-        return s.ring + (size_t)st * kSegChunk;
+        return reinterpret_cast<const uint4*>(s.ring + (size_t)pos.st * kSegChunk);
     }
     __device__ __forceinline__ void release() {
         __syncwarp();
-        if ((threadIdx.x & 31) == 0) mb_arrive(&s.empty[n % stages]);
-        ++n;
+        if ((threadIdx.x & 31) == 0) mb_arrive(&s.empty[pos.st]);
+        pos.next(stages);
     }
 };
 
@@ -314,11 +423,11 @@ __device__ __forceinline__ bool wait_count(const unsigned* cnt, unsigned target,
         unsigned v;
         asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(cnt) : "memory");
         if (v < target) {
-            const unsigned long long t0 = now_ns();
-            for (unsigned it = 1;; ++it) {
+            Bound bd;
+            for (;;) {
                 asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(cnt) : "memory");
                 if (v >= target) break;
-                if ((it & 15) == 0 && ((*err & kErrStall) || now_ns() - t0 > kStallNs)) {
+                if (bd.expired(err)) {
                     atomicOr((int*)err, kErrStall);
                     ok = 0;
                     break;
@@ -337,6 +446,20 @@ __device__ __forceinline__ void signal_count(unsigned* cnt) {
     if (threadIdx.x == 0) asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(cnt) : "memory");
 }
 
+// dst[i] = f(i) for i < n, four elements per thread per round with all their
+// loads issued before any store (f reads global memory).
+template <class F>
+__device__ __forceinline__ void gather(float* dst, int n, F f) {
+    for (int b = threadIdx.x; b < n; b += 4 * kCT) {
+        float v[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) v[e] = (b + e * kCT < n) ? f(b + e * kCT) : 0.f;
+#pragma unroll
+        for (int e = 0; e < 4; ++e)
+            if (b + e * kCT < n) dst[b + e * kCT] = v[e];
+    }
+}
+
 // RMSNorm of hs (d values) times gain g into xs (consumer threads).
 __device__ __forceinline__ void rmsnorm_sm(const float* hs, const uint16_t* g, int d, float eps, float* xs,
                                            float* red) {
@@ -353,53 +476,66 @@ __device__ __forceinline__ void rmsnorm_sm(const float* hs, const uint16_t* g, i
     csync();
 }
 
-// Stream this CTA's items of one matrix against x, writing tile partial
-// slots.  xfn(c) returns the 256 input columns of chunk c (it may rebuild
-// them into shared memory; every consumer thread calls it).
-template <class XFn>
-__device__ __forceinline__ void gemv_items(Consumer& cs, const Items& it, int cta, float* part, float* red, XFn xfn) {
+// Whole tiles [t0, t1) of a matrix with rows of length K against x (all K
+// columns in shared memory).  epi(t, s) runs in warp 0 with lane = row of
+// the tile and s its complete dot product.
+template <class Epi>
+__device__ __forceinline__ void tile_gemv(Consumer& cs, int t0, int t1, int K, int nc, const float* x, float* red,
+                                          int& rb, Epi epi) {
     const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    float acc = 0.f;
-    int rb = 0;
-    for (int i = it.lo; i < it.hi; ++i) {
-        const int t = i / it.nc, c = i - t * it.nc;
-        const float* x = xfn(c);
-        const uint4* buf = reinterpret_cast<const uint4*>(cs.acquire());
-        const int ccn = (int)(chunk_bytes(it, c) / 512);
-        if (cs.ok)
-            for (int cc = w; cc < ccn; cc += kCW) acc += dot8(buf[cc * 32 + lane], x + cc * 8);
-        cs.release();
-        if (i + 1 == it.hi || c + 1 == it.nc) {
-            float* r = red + rb * kCW * 32;
-            r[w * 32 + lane] = acc;
-            acc = 0.f;
-            csync();
-            if (w == 0) {
-                float sum = 0.f;
+    for (int t = t0; t < t1; ++t) {
+        float acc = 0.f;
+        for (int c = 0; c < nc; ++c) {
+            const uint32_t buf = saddr(cs.acquire()) + lane * 16;
+            const int ccn = (int)(chunk_bytes(K, c) / 512);
+            const uint32_t xc = saddr(x + c * kColsPerChunk);
+            if (cs.ok) {
+                uint4 wv[4];
 #pragma unroll
-                for (int k = 0; k < kCW; ++k) sum += r[k * 32 + lane];
-                const int slot = cta - item_owner(it, t * it.nc);
-                part[((int64_t)t * it.nc + slot) * 32 + lane] = sum;
+                for (int u = 0; u < 4; ++u)
+                    if (w + u * kCW < ccn) wv[u] = lds128(buf + (w + u * kCW) * 512);
+#pragma unroll
+                for (int u = 0; u < 4; ++u)
+                    if (w + u * kCW < ccn) acc += dot8s(wv[u], xc + (w + u * kCW) * 32);
             }
-            rb ^= 1;
+            cs.release();
         }
+        float* r = red + rb * kCW * 32;
+        r[w * 32 + lane] = acc;
+        csync();
+        if (w == 0) {
+            float sum = 0.f;
+#pragma unroll
+            for (int k = 0; k < kCW; ++k) sum += r[k * 32 + lane];
+            epi(t, sum);
+        }
+        rb ^= 1;
     }
 }
 
-// Residual rebuild: hs = hbuf_prev + O slots + down slots of layer jp (or a
-// plain copy of `src`).
-__device__ __forceinline__ void rebuild_h(const DevModel& m, const SegPlan& p, const float* hin, bool add_parts,
-                                          float* hs) {
-    const Items io = items_of(p, 1, 0), idn = items_of(p, 3, 0);
-    for (int i = threadIdx.x; i < m.d; i += kCT) {
-        float v = hin[i];
-        if (add_parts) {
-            v += slot_sum(p.part[1], io, i >> 5, i & 31);
-            v += slot_sum(p.part[3], idn, i >> 5, i & 31);
+// Residual entering layer j at row i: the embedding (first layer of a step),
+// the model's h (first layer of a later segment), or the previous layer's
+// mid residual plus its down-projection slots.
+struct ResidIn {
+    const DevModel* m;
+    const SegPlan* p;
+    const uint16_t* emb;  // embedding row, or null
+    const float* src;     // m.h or the mid residual
+    bool add_down;
+    const uint8_t* nsd;
+    __device__ __forceinline__ float operator()(int i) const {
+        if (emb) return bf(emb[i]);
+        float v = src[i];
+        if (add_down) {
+            const int t = i >> 5, ns = nsd[t];
+            const float* q = p->dpart + (int64_t)t * p->n_chunks[3] * 32 + (i & 31);
+#pragma unroll
+            for (int k = 0; k < kSegMaxSlots; ++k)
+                if (k < ns) v += q[k * 32];
         }
-        hs[i] = v;
+        return v;
     }
-}
+};
 
 }  // namespace
 
@@ -409,7 +545,7 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
     const int cta = blockIdx.x, G = p.G;
     volatile int* err = &m.ctl->err;
     const int half = m.D >> 1, grp = m.A / m.KH;
-    const int nq = m.A * half, nk = m.KH * half;
+    const int AD = m.A * m.D;
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < p.stages; ++i) {
@@ -426,33 +562,38 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
     const AttnGeo ag = attn_geo(m, p, pos_ok ? pos : 0);
     const int unit = attn_unit(ag, G, cta);
     const int rpc = p.rows_per_kv_chunk, cpp = m.page_size / rpc;
+    int tq0, tq1, to0, to1, tg0, tg1;
+    whole_tiles(p.n_tiles[0], G, cta, tq0, tq1);
+    whole_tiles(p.n_tiles[1], G, cta, to0, to1);
+    whole_tiles(p.n_tiles[2], G, cta, tg0, tg1);
+    const Items idn = down_items(p, cta);
 
     // ---------------------------------------------------------- producer
     if (threadIdx.x >= kCT) {
         if (threadIdx.x != kCT || !pos_ok) return;
-        Producer pr(s, p.stages, err);
+        Producer pr(s, p.stages, min(p.stages, p.inflight), err);
         for (int j = j0; j < j1 && pr.ok; ++j) {
-            for (int mt = 0; mt < 4; ++mt) {
-                const Items it = items_of(p, mt, cta);
-                const uint8_t* W = mat_base(m, j, mt);
-                for (int i = it.lo; i < it.hi; ++i) {
-                    const int t = i / it.nc, ch = i - t * it.nc;
-                    pr.push(W + (int64_t)t * kTileRows * it.K * 2 + (int64_t)ch * kSegChunk, chunk_bytes(it, ch),
-                            pr.pol_w);
-                }
-                if (mt == 0 && unit >= 0) {
-                    const int g = unit / ag.splits, sp = unit - g * ag.splits;
-                    const int pg0 = sp * ag.pps, pg1 = min(ag.n_pages, pg0 + ag.pps);
-                    const uint16_t* pools[2] = {m.kpool + (int64_t)j * m.kv_layer_stride,
-                                                m.vpool + (int64_t)j * m.kv_layer_stride};
-                    for (int kvi = 0; kvi < 2; ++kvi)
-                        for (int pg = pg0; pg < pg1; ++pg) {
-                            const int phys = m.page_table[pg];
-                            for (int q = 0; q < cpp; ++q)
-                                pr.push(pools[kvi] + (((int64_t)phys * m.KH + g) * m.page_size + q * rpc) * m.D,
-                                        (uint32_t)(rpc * m.D * 2), pr.pol_kv);
-                        }
-                }
+            pr.tiles(mat_base(m, j, 0), p.K[0], p.n_chunks[0], tq0, tq1);
+            if (unit >= 0) {
+                const int g = unit / ag.splits, sp = unit - g * ag.splits;
+                const int pg0 = sp * ag.pps, pg1 = min(ag.n_pages, pg0 + ag.pps);
+                const uint16_t* pools[2] = {m.kpool + (int64_t)j * m.kv_layer_stride,
+                                            m.vpool + (int64_t)j * m.kv_layer_stride};
+                for (int kvi = 0; kvi < 2; ++kvi)
+                    for (int pg = pg0; pg < pg1; ++pg) {
+                        const int phys = m.page_table[pg];
+                        for (int q = 0; q < cpp; ++q)
+                            pr.push(pools[kvi] + (((int64_t)phys * m.KH + g) * m.page_size + q * rpc) * m.D,
+                                    (uint32_t)(rpc * m.D * 2), pr.pol_kv);
+                    }
+            }
+            pr.tiles(mat_base(m, j, 1), p.K[1], p.n_chunks[1], to0, to1);
+            pr.tiles(mat_base(m, j, 2), p.K[2], p.n_chunks[2], tg0, tg1);
+            const uint8_t* Wd = mat_base(m, j, 3);
+            for (int i = idn.lo; i < idn.hi; ++i) {
+                const int t = i / idn.nc, ch = i - t * idn.nc;
+                pr.push(Wd + (int64_t)t * kTileRows * idn.K * 2 + (int64_t)ch * kSegChunk, chunk_bytes(idn.K, ch),
+                        pr.pol_w);
             }
         }
         pr.drain();
@@ -470,41 +611,76 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
     const float2* cs_row = m.rope + (int64_t)pos * half;
     const float scale = 1.0f / sqrtf((float)m.D);
     const int slice0 = (int)((int64_t)cta * m.d / G), slice1 = (int)((int64_t)(cta + 1) * m.d / G);
-
-    if (first && cta == 0 && threadIdx.x == 0) {
-        c->exit_readout = -1;
-        c->n_evaluated = 0;
-        c->full_token = -1;
+    const int nq = m.A * half, nk = m.KH * half;
+    const int64_t kvo_pos = ((int64_t)m.page_table[pos / m.page_size] * m.KH * m.page_size + pos % m.page_size) * m.D;
+    {   // slots of each down tile
+        Items all = down_items(p, 0);
+        for (int t = threadIdx.x; t < p.n_tiles[3]; t += kCT)
+            s.nsd[t] = (uint8_t)(item_owner(all, t * all.nc + all.nc - 1) - item_owner(all, t * all.nc) + 1);
     }
+    int tok = c->in_tok;
+    if (first) {
+        if (tok < 0 || tok >= m.V) {
+            if (cta == 0 && threadIdx.x == 0) atomicOr(&c->err, kErrTokenRange);
+            tok = 0;
+        }
+        if (cta == 0 && threadIdx.x == 0) {
+            c->exit_readout = -1;
+            c->n_evaluated = 0;
+            c->full_token = -1;
+        }
+    }
+    csync();
+    int rb = 0;
 
     for (int j = j0; j < j1; ++j) {
         const int li = j - j0;
         unsigned* cnt = sync + li * kPhases;
         const uint16_t* lw = m.layers + (int64_t)j * m.layer_stride;
+        const ResidIn rin{&m, &p, (j == j0 && first) ? m.embed + (int64_t)tok * m.d : nullptr,
+                          j == j0 ? m.h : p.hmid, j > j0, s.nsd};
 
-        // ---------------- Q/K/V: residual in, RMSNorm, projection slots
-        if (j > j0 && !wait_count(cnt - kPhases + kPhDn, G, err)) return;
-        float* hin = p.hbuf + (j & 1) * m.d;
-        if (j == j0 && first) {
-            int tok = c->in_tok;
-            if (tok < 0 || tok >= m.V) {
-                if (cta == 0 && threadIdx.x == 0) atomicOr(&c->err, kErrTokenRange);
-                tok = 0;
-            }
-            const uint16_t* e = m.embed + (int64_t)tok * m.d;
-            for (int i = threadIdx.x; i < m.d; i += kCT) s.hs[i] = bf(e[i]);
-        } else if (j == j0) {
-            rebuild_h(m, p, m.h, false, s.hs);
-        } else {
-            rebuild_h(m, p, p.hbuf + ((j - 1) & 1) * m.d, true, s.hs);
+        // ---------------- Q/K/V tiles: RMSNorm, projection, bias, RoPE, KV append
+        if (tq1 > tq0) {
+            if (j > j0 && !wait_count(cnt - kPhases + kPhDn, G, err)) return;
+            gather(s.hs, m.d, rin);
+            csync();
+            rmsnorm_sm(s.hs, lw + m.off_gattn, m.d, m.eps, s.xs, s.red);
+            const uint16_t* bias = m.qkv_bias ? lw + m.off_bqkv : nullptr;
+            uint16_t* kdst = m.kpool + (int64_t)j * m.kv_layer_stride + kvo_pos;
+            uint16_t* vdst = m.vpool + (int64_t)j * m.kv_layer_stride + kvo_pos;
+            tile_gemv(cs, tq0, tq1, p.K[0], p.n_chunks[0], s.xs, s.red, rb, [&](int t, float v) {
+                const int odd = lane & 1;
+                const int u = t * 16 + (lane >> 1);
+                if (bias) v += bf(bias[2 * u + odd]);
+                const float other = __shfl_xor_sync(0xffffffffu, v, 1);
+                const float r0 = odd ? other : v, r1 = odd ? v : other;
+                if (u < nq) {
+                    const int h = u / half, i = u - h * half;
+                    const float2 cz = cs_row[i];
+                    if (!odd)
+                        m.q[h * m.D + i] = r0 * cz.x - r1 * cz.y;
+                    else
+                        m.q[h * m.D + i + half] = r0 * cz.y + r1 * cz.x;
+                } else if (u < nq + nk) {
+                    const int g = (u - nq) / half, i = (u - nq) - g * half;
+                    const float2 cz = cs_row[i];
+                    uint16_t* k = kdst + (int64_t)g * m.page_size * m.D;
+                    if (!odd)
+                        k[i] = tobf(r0 * cz.x - r1 * cz.y);
+                    else
+                        k[i + half] = tobf(r0 * cz.y + r1 * cz.x);
+                } else if (u < nq + 2 * nk) {
+                    const int g = (u - nq - nk) / half, i = (u - nq - nk) - g * half;
+                    uint16_t* v2 = vdst + (int64_t)g * m.page_size * m.D;
+                    if (!odd)
+                        v2[i] = tobf(r0);
+                    else
+                        v2[i + half] = tobf(r1);
+                }
+            });
         }
-        csync();
-        for (int i = slice0 + threadIdx.x; i < slice1; i += kCT) hin[i] = s.hs[i];
-        rmsnorm_sm(s.hs, lw + m.off_gattn, m.d, m.eps, s.xs, s.red);
-        {
-            const Items it = items_of(p, 0, cta);
-            gemv_items(cs, it, cta, p.part[0], s.red, [&](int ch) { return s.xs + ch * kColsPerChunk; });
-        }
+        if (cta == 0 && threadIdx.x == 0) m.kv_src[(int64_t)j * m.max_ctx + pos] = 1;
         signal_count(cnt + kPhQKV);
 
         // ---------------- attention unit (if this CTA has one)
@@ -514,51 +690,12 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
             const int p0 = pg0 * m.page_size, p1 = min(ag.T, pg1 * m.page_size);
             const int npos = p1 - p0;
             if (!wait_count(cnt + kPhQKV, G, err)) return;
-            // rebuild q (rotated), k and v of the step's position for group g
-            const Items iq = items_of(p, 0, 0);
-            const uint16_t* bias = m.qkv_bias ? lw + m.off_bqkv : nullptr;
-            for (int e = threadIdx.x; e < (grp + 2) * half; e += kCT) {
-                const int hh = e / half, i = e - hh * half;
-                int u;
-                if (hh < grp)
-                    u = (g * grp + hh) * half + i;
-                else if (hh == grp)
-                    u = nq + g * half + i;
-                else
-                    u = nq + nk + g * half + i;
-                const int t = u >> 4, l0 = (u & 15) * 2;
-                float r0 = slot_sum(p.part[0], iq, t, l0), r1 = slot_sum(p.part[0], iq, t, l0 + 1);
-                if (bias) {
-                    r0 += bf(bias[2 * u]);
-                    r1 += bf(bias[2 * u + 1]);
-                }
-                if (hh <= grp) {
-                    const float2 cz = cs_row[i];
-                    const float a0 = r0 * cz.x - r1 * cz.y, a1 = r0 * cz.y + r1 * cz.x;
-                    if (hh < grp) {
-                        s.qa[hh * m.D + i] = a0 * scale;
-                        s.qa[hh * m.D + i + half] = a1 * scale;
-                    } else {
-                        s.kv[i] = round_bf(a0);
-                        s.kv[i + half] = round_bf(a1);
-                    }
-                } else {
-                    s.kv[m.D + i] = round_bf(r0);
-                    s.kv[m.D + i + half] = round_bf(r1);
-                }
-            }
+            const float* qsrc = m.q + (int64_t)g * grp * m.D;
+            const uint16_t* kt = m.kpool + (int64_t)j * m.kv_layer_stride + kvo_pos + (int64_t)g * m.page_size * m.D;
+            const uint16_t* vt = m.vpool + (int64_t)j * m.kv_layer_stride + kvo_pos + (int64_t)g * m.page_size * m.D;
+            gather(s.qa, grp * m.D, [&](int i) { return qsrc[i] * scale; });
+            gather(s.kv, 2 * m.D, [&](int i) { return i < m.D ? bf(kt[i]) : bf(vt[i - m.D]); });
             csync();
-            if (sp == 0) {  // the cache entry of this position, for later steps
-                const int64_t off = (int64_t)j * m.kv_layer_stride +
-                                    (((int64_t)m.page_table[pos / m.page_size] * m.KH + g) * m.page_size +
-                                     pos % m.page_size) *
-                                        m.D;
-                for (int i = threadIdx.x; i < m.D; i += kCT) {
-                    m.kpool[off + i] = tobf(s.kv[i]);
-                    m.vpool[off + i] = tobf(s.kv[m.D + i]);
-                }
-                if (g == 0 && threadIdx.x == 0) m.kv_src[(int64_t)j * m.max_ctx + pos] = 1;
-            }
             // scores: warp per position, lane per D/32 dimensions
             const int dpl = m.D >> 5;  // 2 or 4
             float qr[kSegMaxGroup][4];
@@ -569,24 +706,51 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
             const int spc = p.max_pps * m.page_size;  // score row stride
             for (int pg = pg0; pg < pg1; ++pg)
                 for (int q = 0; q < cpp; ++q) {
-                    const uint16_t* kb = reinterpret_cast<const uint16_t*>(cs.acquire());
+                    const uint32_t kb = saddr(cs.acquire()) + lane * dpl * 2;
                     const int base = pg * m.page_size + q * rpc;
                     for (int r = w; r < rpc; r += kCW) {
                         const int ps = base + r;
                         if (ps >= p1) break;
                         float kd[4];
+                        if (ps == pos) {
 #pragma unroll
-                        for (int k = 0; k < 4; ++k)
-                            kd[k] = k < dpl ? (ps == pos ? s.kv[lane * dpl + k] : bf(kb[r * m.D + lane * dpl + k])) : 0.f;
+                            for (int k = 0; k < 4; ++k) kd[k] = k < dpl ? s.kv[lane * dpl + k] : 0.f;
+                        } else if (dpl == 4) {
+                            const uint2 v = lds64(kb + r * m.D * 2);
+                            kd[0] = bflo(v.x);
+                            kd[1] = bfhi(v.x);
+                            kd[2] = bflo(v.y);
+                            kd[3] = bfhi(v.y);
+                        } else {
+                            const uint32_t v = lds32(kb + r * m.D * 2);
+                            kd[0] = bflo(v);
+                            kd[1] = bfhi(v);
+                            kd[2] = kd[3] = 0.f;
+                        }
+                        float dd[kSegMaxGroup];
 #pragma unroll
                         for (int hh = 0; hh < kSegMaxGroup; ++hh) {
-                            if (hh >= grp) break;
                             float d = 0.f;
 #pragma unroll
                             for (int k = 0; k < 4; ++k) d = fmaf(qr[hh][k], kd[k], d);
-                            d = warp_sum(d);
-                            if (lane == 0) s.sc[hh * spc + (ps - p0)] = d;
+                            dd[hh] = d;
                         }
+                        // reduce-scatter over the warp: lane bits 4, 3, 2 pick the head
+                        const bool b16 = lane & 16, b8 = lane & 8, b4 = lane & 4;
+                        float a4[4], a2[2];
+#pragma unroll
+                        for (int k = 0; k < 4; ++k)
+                            a4[k] = (b16 ? dd[k + 4] : dd[k]) +
+                                    __shfl_xor_sync(0xffffffffu, b16 ? dd[k] : dd[k + 4], 16);
+#pragma unroll
+                        for (int k = 0; k < 2; ++k)
+                            a2[k] = (b8 ? a4[k + 2] : a4[k]) +
+                                    __shfl_xor_sync(0xffffffffu, b8 ? a4[k] : a4[k + 2], 8);
+                        float a1 = (b4 ? a2[1] : a2[0]) + __shfl_xor_sync(0xffffffffu, b4 ? a2[0] : a2[1], 4);
+                        a1 += __shfl_xor_sync(0xffffffffu, a1, 2);
+                        a1 += __shfl_xor_sync(0xffffffffu, a1, 1);
+                        const int hd = (b16 ? 4 : 0) + (b8 ? 2 : 0) + (b4 ? 1 : 0);
+                        if ((lane & 3) == 0 && hd < grp) s.sc[hd * spc + (ps - p0)] = a1;
                     }
                     cs.release();
                 }
@@ -614,18 +778,34 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
                 for (int q = 0; q < cpp; ++q) {
                     const uint16_t* vb = reinterpret_cast<const uint16_t*>(cs.acquire());
                     const int base = pg * m.page_size + q * rpc;
-                    if (w < grp && cs.ok)
-                        for (int r = 0; r < rpc; ++r) {
-                            const int ps = base + r;
-                            if (ps >= p1) break;
-                            const float pr = s.sc[w * spc + (ps - p0)];
+                    const int nr = min(rpc, p1 - base);
+                    if (w < grp && cs.ok) {
+                        const uint32_t pw = saddr(s.sc + w * spc + (base - p0));
+                        const uint32_t vrow = saddr(vb) + lane * dpl * 2;
+                        const int rt = (pos >= base && pos < base + nr) ? pos - base : -1;
+                        const int rs = rt >= 0 ? rt : nr;  // rows before the step's own position
+#pragma unroll 4
+                        for (int r = 0; r < rs; ++r) {
+                            const float pr = ldsf(pw + 4 * r);
+                            if (dpl == 4) {
+                                const uint2 v = lds64(vrow + r * m.D * 2);
+                                oacc[0] = fmaf(pr, bflo(v.x), oacc[0]);
+                                oacc[1] = fmaf(pr, bfhi(v.x), oacc[1]);
+                                oacc[2] = fmaf(pr, bflo(v.y), oacc[2]);
+                                oacc[3] = fmaf(pr, bfhi(v.y), oacc[3]);
+                            } else {
+                                const uint32_t v = lds32(vrow + r * m.D * 2);
+                                oacc[0] = fmaf(pr, bflo(v), oacc[0]);
+                                oacc[1] = fmaf(pr, bfhi(v), oacc[1]);
+                            }
+                        }
+                        if (rt >= 0) {  // the step's own position: v from the Q/K/V phase
+                            const float pr = ldsf(pw + 4 * rt);
 #pragma unroll
                             for (int k = 0; k < 4; ++k)
-                                if (k < dpl)
-                                    oacc[k] = fmaf(pr, ps == pos ? s.kv[m.D + lane * dpl + k]
-                                                                 : bf(vb[r * m.D + lane * dpl + k]),
-                                                   oacc[k]);
+                                if (k < dpl) oacc[k] = fmaf(pr, s.kv[m.D + lane * dpl + k], oacc[k]);
                         }
+                    }
                     cs.release();
                 }
             if (w < grp) {
@@ -641,62 +821,92 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
         }
         signal_count(cnt + kPhAttn);
 
-        // ---------------- O-projection slots (input: merged attention output)
-        if (!wait_count(cnt + kPhAttn, G, err)) return;
-        {
-            const Items it = items_of(p, 1, cta);
-            gemv_items(cs, it, cta, p.part[1], s.red, [&](int ch) {
-                // columns [256 ch, 256 ch + 256) of o: merge the splits of each head
-                csync();  // the previous chunk's readers of xc are done
-                const int c0 = ch * kColsPerChunk, nc = min(kColsPerChunk, m.A * m.D - c0);
-                for (int e = threadIdx.x; e < nc; e += kCT) {
-                    const int col = c0 + e, h = col / m.D, dd = col - h * m.D;
-                    const float* src = p.attn_part + (int64_t)h * kAttnMaxSplits * (m.D + 2);
-                    float mx = -INFINITY;
-                    for (int k = 0; k < ag.splits; ++k) mx = fmaxf(mx, src[k * (m.D + 2) + m.D]);
-                    float num = 0.f, den = 0.f;
-                    for (int k = 0; k < ag.splits; ++k) {
-                        const float* q = src + k * (m.D + 2);
-                        const float wgt = expf(q[m.D] - mx);
-                        num = fmaf(wgt, q[dd], num);
-                        den = fmaf(wgt, q[m.D + 1], den);
-                    }
-                    s.xc[e] = num / den;
-                }
-                csync();
-                return (const float*)s.xc;
+        // ---------------- O tiles: merge the attention splits, project, add the residual
+        if (to1 > to0) {
+            if (!wait_count(cnt + kPhAttn, G, err)) return;
+            const int ns = ag.splits;
+            float* den = s.wts + m.A * kSegMaxSplits;
+            for (int h = w; h < m.A; h += kCW) {  // split weights exp(m_s - M) of each head
+                const float* src = p.attn_part + (int64_t)h * kAttnMaxSplits * (m.D + 2) + m.D;
+                const float ms = lane < ns ? src[lane * (m.D + 2)] : -INFINITY;
+                const float ls = lane < ns ? src[lane * (m.D + 2) + 1] : 0.f;
+                const float mx = warp_max(ms);
+                const float wt = lane < ns ? expf(ms - mx) : 0.f;
+                if (lane < ns) s.wts[h * kSegMaxSplits + lane] = wt;
+                const float dn = warp_sum(wt * ls);
+                if (lane == 0) den[h] = dn;
+            }
+            csync();
+            gather(s.xs, AD, [&](int col) {
+                const int h = col / m.D;
+                const float* src = p.attn_part + (int64_t)h * kAttnMaxSplits * (m.D + 2) + (col - h * m.D);
+                const float* wt = s.wts + h * kSegMaxSplits;
+                float num = 0.f;
+                for (int k = 0; k < ns; ++k) num = fmaf(wt[k], src[k * (m.D + 2)], num);
+                return num / den[h];
+            });
+            csync();
+            tile_gemv(cs, to0, to1, p.K[1], p.n_chunks[1], s.xs, s.red, rb, [&](int t, float v) {
+                const int row = t * 32 + lane;
+                if (row < m.d) p.hmid[row] = rin(row) + v;
             });
         }
         signal_count(cnt + kPhO);
 
-        // ---------------- gate/up slots (input: RMSNorm of the mid residual)
-        if (!wait_count(cnt + kPhO, G, err)) return;
-        {
-            const Items io = items_of(p, 1, 0);
-            for (int i = threadIdx.x; i < m.d; i += kCT) s.hs[i] = hin[i] + slot_sum(p.part[1], io, i >> 5, i & 31);
+        // ---------------- gate/up tiles: RMSNorm of the mid residual, SwiGLU
+        if (tg1 > tg0) {
+            if (!wait_count(cnt + kPhO, G, err)) return;
+            gather(s.hs, m.d, [&](int i) { return p.hmid[i]; });
             csync();
             rmsnorm_sm(s.hs, lw + m.off_gmlp, m.d, m.eps, s.xs, s.red);
-            const Items it = items_of(p, 2, cta);
-            gemv_items(cs, it, cta, p.part[2], s.red, [&](int ch) { return s.xs + ch * kColsPerChunk; });
+            tile_gemv(cs, tg0, tg1, p.K[2], p.n_chunks[2], s.xs, s.red, rb, [&](int t, float v) {
+                const float up = __shfl_xor_sync(0xffffffffu, v, 1);
+                const int f = t * 16 + (lane >> 1);
+                if (!(lane & 1) && f < m.F) m.a[f] = v / (1.0f + expf(-v)) * up;
+            });
         }
         signal_count(cnt + kPhGU);
 
-        // ---------------- down slots (input: SiLU(gate) * up)
-        if (!wait_count(cnt + kPhGU, G, err)) return;
-        {
-            const Items ig = items_of(p, 2, 0);
-            const Items it = items_of(p, 3, cta);
-            gemv_items(cs, it, cta, p.part[3], s.red, [&](int ch) {
-                csync();  // the previous chunk's readers of xc are done
-                const int c0 = ch * kColsPerChunk, nc = min(kColsPerChunk, m.F - c0);
-                for (int e = threadIdx.x; e < nc; e += kCT) {
-                    const int f = c0 + e, t = f >> 4, l0 = (f & 15) * 2;
-                    const float gt = slot_sum(p.part[2], ig, t, l0), up = slot_sum(p.part[2], ig, t, l0 + 1);
-                    s.xc[e] = gt / (1.0f + expf(-gt)) * up;
-                }
-                csync();
-                return (const float*)s.xc;
+        // ---------------- down items: partial slots of h_out - h_mid
+        if (idn.hi > idn.lo) {
+            if (!wait_count(cnt + kPhGU, G, err)) return;
+            gather(s.xa, (idn.hi - idn.lo) * kColsPerChunk, [&](int e) {
+                const int i = idn.lo + e / kColsPerChunk, col = e % kColsPerChunk;
+                const int ch = i % idn.nc, f = ch * kColsPerChunk + col;
+                return f < m.F ? m.a[f] : 0.f;
             });
+            csync();
+            float acc = 0.f;
+            for (int i = idn.lo; i < idn.hi; ++i) {
+                const int t = i / idn.nc, ch = i - t * idn.nc;
+                const uint32_t buf = saddr(cs.acquire()) + lane * 16;
+                const int ccn = (int)(chunk_bytes(idn.K, ch) / 512);
+                const uint32_t x = saddr(s.xa + (i - idn.lo) * kColsPerChunk);
+                if (cs.ok) {
+                    uint4 wv[4];
+#pragma unroll
+                    for (int u = 0; u < 4; ++u)
+                        if (w + u * kCW < ccn) wv[u] = lds128(buf + (w + u * kCW) * 512);
+#pragma unroll
+                    for (int u = 0; u < 4; ++u)
+                        if (w + u * kCW < ccn) acc += dot8s(wv[u], x + (w + u * kCW) * 32);
+                }
+                cs.release();
+                if (i + 1 == idn.hi || ch + 1 == idn.nc) {
+                    float* r = s.red + rb * kCW * 32;
+                    r[w * 32 + lane] = acc;
+                    acc = 0.f;
+                    csync();
+                    if (w == 0) {
+                        float sum = 0.f;
+#pragma unroll
+                        for (int k = 0; k < kCW; ++k) sum += r[k * 32 + lane];
+                        const int slot = cta - item_owner(idn, t * idn.nc);
+                        p.dpart[((int64_t)t * idn.nc + slot) * 32 + lane] = sum;
+                    }
+                    rb ^= 1;
+                }
+            }
         }
         signal_count(cnt + kPhDn);
     }
@@ -704,10 +914,8 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
     // ---------------- the segment's output residual, then the exit ticket
     if (!wait_count(sync + (j1 - 1 - j0) * kPhases + kPhDn, G, err)) return;
     {
-        const Items io = items_of(p, 1, 0), idn = items_of(p, 3, 0);
-        const float* hin = p.hbuf + ((j1 - 1) & 1) * m.d;
-        for (int i = slice0 + threadIdx.x; i < slice1; i += kCT)
-            m.h[i] = hin[i] + slot_sum(p.part[1], io, i >> 5, i & 31) + slot_sum(p.part[3], idn, i >> 5, i & 31);
+        const ResidIn rout{&m, &p, nullptr, p.hmid, true, s.nsd};
+        for (int i = slice0 + threadIdx.x; i < slice1; i += kCT) m.h[i] = rout(i);
     }
     __threadfence();
     csync();
@@ -724,7 +932,7 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
 bool seg_plan(const DevModel& m, int n_sm, SegPlan& p) {
     p.G = n_sm;
     const int grp = m.A / m.KH;
-    if (m.A % m.KH || grp > kSegMaxGroup || (m.D != 64 && m.D != 128)) return false;
+    if (m.A % m.KH || grp > kSegMaxGroup || (m.D != 64 && m.D != 128) || m.A > 32 * kCW) return false;
     const int Ks[4] = {m.d, m.A * m.D, m.d, m.F};
     const int64_t rows[4] = {(int64_t)(m.A + 2 * m.KH) * m.D, m.d, 2LL * m.F, m.d};
     for (int i = 0; i < 4; ++i) {
@@ -733,18 +941,28 @@ bool seg_plan(const DevModel& m, int n_sm, SegPlan& p) {
         p.n_tiles[i] = (int)tile_count(rows[i]);
         p.n_chunks[i] = (Ks[i] + kColsPerChunk - 1) / kColsPerChunk;
     }
+    // down items: slots per tile within kSegMaxSlots, items per CTA sized
+    const int64_t N = (int64_t)p.n_tiles[3] * p.n_chunks[3];
+    const int64_t Ge = std::min<int64_t>(p.G, N);
+    p.max_dn_items = (int)((N + Ge - 1) / Ge);
+    for (int64_t t = 0; t < p.n_tiles[3]; ++t) {
+        const int64_t a = ((t * p.n_chunks[3] + 1) * Ge - 1) / N, b = (((t + 1) * p.n_chunks[3]) * Ge - 1) / N;
+        if (b - a + 1 > kSegMaxSlots) return false;
+    }
     p.rows_per_kv_chunk = std::min(m.page_size, kSegChunk / (2 * m.D));
     if (m.page_size % p.rows_per_kv_chunk) return false;
     const int cap = std::max(1, std::min(kSegMaxSplits, p.G / m.KH));
     const int np_max = (m.max_ctx + m.page_size - 1) / m.page_size;
     p.max_pps = std::max(1, (np_max + cap - 1) / cap);
-    const size_t floats = 2 * (size_t)((m.d + 3) & ~3) + kColsPerChunk + 2 * kCW * 32 + (size_t)grp * m.D +
-                          2 * (size_t)m.D + (size_t)grp * p.max_pps * m.page_size + 2 * (size_t)grp;
-    const size_t fixed = floats * 4 + 256;
+    const size_t floats = (size_t)((std::max(m.d, m.A * m.D) + 3) & ~3) + ((m.d + 3) & ~3) +
+                          (size_t)p.max_dn_items * kColsPerChunk + 2 * kCW * 32 + (size_t)grp * m.D + 2 * (size_t)m.D +
+                          (size_t)grp * p.max_pps * m.page_size + 2 * (size_t)grp + (size_t)m.A * (kSegMaxSplits + 1);
+    const size_t fixed = floats * 4 + (size_t)p.n_tiles[3] + 256;
     const size_t budget = 227 * 1024;
     if (fixed + 4 * (size_t)(kSegChunk + 16) > budget) return false;
     p.stages = (int)std::min<size_t>(16, (budget - fixed) / (kSegChunk + 16));
-    p.smem = (size_t)p.stages * (kSegChunk + 16) + floats * 4;
+    p.smem = (size_t)p.stages * (kSegChunk + 16) + floats * 4 + (size_t)p.n_tiles[3];
+    p.inflight = p.stages;
     return true;
 }
 
