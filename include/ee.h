@@ -199,10 +199,10 @@ int ee_position(ee_ctx* ctx, int32_t* pos);
                                  0: direct launches, branch decided on the host */
 #define EE_OPT_PDL 2          /* 1 (default): programmatic dependent launch    */
 #define EE_OPT_DEBUG_LOGITS 3 /* 1: keep each step's readout and final logits  */
-#define EE_OPT_PERSISTENT 4   /* 1: each run of layers between readouts is one
-                                 persistent launch, one CTA per SM streaming
-                                 weights through a shared-memory ring;
-                                 0 (default): five launches per layer.
+#define EE_OPT_PERSISTENT 4   /* 1 (default where supported): each run of layers
+                                 between readouts is one persistent launch, one
+                                 CTA per SM streaming weights through a shared-
+                                 memory ring; 0: five launches per layer.
                                  EE_EINVAL if the shape is not supported      */
 int ee_set_option(ee_ctx* ctx, int option, int value);
 

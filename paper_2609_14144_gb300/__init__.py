@@ -53,7 +53,8 @@ class Engine:
                                      self.workspace_bytes, ctypes.c_void_p(self.stream.cuda_stream),
                                      ctypes.byref(ctx)))
         self.ctx = ctx
-        self.persistent = False  # EE_OPT_PERSISTENT (off by default)
+        # the persistent layer kernel is on by default where the shape allows it
+        self.persistent = self.lib.ee_set_option(self.ctx, OPT_PERSISTENT, 1) == 0
         self.n_readouts = 0
         self.readout_layers = []
         self.load_weights(model)

@@ -58,7 +58,7 @@ struct Layout {
     size_t ctl, rope, layers, embed, lm_head, g_final, ro_w[kMaxReadouts], ro_b[kMaxReadouts];
     size_t kpool, vpool, page_table, kv_src, h, q, o, a, y, hk, logits_ro, logits_final;
     size_t gemv_part, gemv_ticket, attn_part, attn_ticket, vocab_part, vocab_ticket;
-    size_t seg_dpart, seg_hmid, seg_sync;
+    size_t seg_dpart, seg_opart, seg_sync;
     size_t prompt, sched, out_tok, out_exit, out_conf, total;
     int64_t layer_stride, off_wqkv, off_bqkv, off_gattn, off_wo, off_gmlp, off_wgu, off_wd;
     int64_t n_units_qkv, kv_layer_stride, gemv_ticket_stride;
@@ -149,8 +149,11 @@ Layout make_layout(const ee_model_config& c) {
     l.vocab_part = take(4 * (size_t)kMaxVocabCtas * 4);
     l.vocab_ticket = take(4);
     // persistent layer kernel: down-projection partials, mid residual, counters
-    l.seg_dpart = take(4 * (size_t)tile_count(d) * ((F + 255) / 256) * kTileRows);
-    l.seg_hmid = take(4 * (size_t)d);
+    {
+        const int64_t cols = kSegChunk / (2 * kTileRows);  // columns per ring chunk
+        l.seg_dpart = take(4 * (size_t)tile_count(d) * ((F + cols - 1) / cols) * kTileRows);
+        l.seg_opart = take(2 * 4 * (size_t)tile_count(d) * ((A * D + cols - 1) / cols) * kTileRows);
+    }
     l.seg_sync = take(4 * (size_t)(5 * L + 8));
     l.prompt = take(4 * (size_t)c.max_ctx);
     l.sched = take((size_t)c.max_ctx);
@@ -211,7 +214,7 @@ struct ee_ctx {
     bool weights = false, started = false, prefilled = false;
     int pos = 0;
     bool use_graphs = true, use_pdl = true;
-    bool seg_ok = false, use_persistent = false;  // persistent layer kernel supported / chosen
+    bool seg_ok = false, use_persistent = true;  // persistent layer kernel supported / chosen
     SegPlan seg{};
     int dbg = 0;
     cudaGraphExec_t g_step = nullptr, g_n = nullptr, g_prefill = nullptr;
@@ -699,7 +702,7 @@ int ee_create(const ee_model_config* cfg, void* d_workspace, size_t workspace_by
         layers_blocks_per_sm(c->seg.smem) >= 1) {
         c->seg.dpart = (float*)(w + l.seg_dpart);
         c->seg.attn_part = m.attn_part;
-        c->seg.hmid = (float*)(w + l.seg_hmid);
+        c->seg.opart = (float*)(w + l.seg_opart);
         c->seg.sync = (unsigned*)(w + l.seg_sync);
         c->seg_ok = true;
     }

@@ -166,21 +166,21 @@ cudaError_t launch_set_inputs(Ctl* c, const CtlInputs& in, cudaStream_t s);
 // 0..7 consume a shared-memory ring that warp 8 fills with cp.async.bulk.
 constexpr int kSegConsumerWarps = 8;
 constexpr int kSegThreads = 32 * (kSegConsumerWarps + 1);
-constexpr int kSegChunk = 16384;   // bytes per ring stage: 32 rows x 256 bf16 columns
+constexpr int kSegChunk = 32768;   // bytes per ring stage: 32 rows x 512 bf16 columns
 constexpr int kSegMaxSplits = 32;  // attention splits per kv head (at most)
 constexpr int kSegMaxGroup = 8;    // query heads per kv head (at most)
-constexpr int kSegMaxSlots = 8;    // CTAs sharing one down-projection tile (at most)
+constexpr int kSegMaxSlots = 8;    // CTAs sharing one down tile, chunks of one O tile (at most)
 struct SegPlan {
     int G;                  // CTAs (one per SM)
     int stages;             // ring stages
     int inflight;           // ring chunks a producer keeps in flight (at most)
     int max_pps;            // attention pages per split (at most)
     int rows_per_kv_chunk;  // cache positions per ring chunk
-    int max_dn_items;       // down-projection items per CTA (at most)
+    int max_items;          // O / down-projection items per CTA (at most)
     int n_tiles[4], n_chunks[4], K[4];  // Q/K/V, O, gate/up, down
     float* dpart;           // down-projection partials [tile][n_chunks][32]
-    float* hmid;            // [d] residual after the attention block
-    float* attn_part;       // [A][kAttnMaxSplits][D + 2]
+    float* opart;           // O-projection chunk partials [2][tile][n_chunks][32] (by layer parity)
+    float* attn_part;       // [A][kSegMaxSplits][D + 4]: unnormalised o, max, sum per split
     unsigned* sync;         // [5 L + 1] phase counters and the exit ticket, zero between launches
     size_t smem;            // dynamic shared memory per CTA
 };

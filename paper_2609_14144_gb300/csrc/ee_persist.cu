@@ -10,7 +10,7 @@
 //
 // One CTA per SM.  Warp 8 is the producer: its lane 0 walks the CTA's whole
 // work list for the segment -- its share of every weight matrix, cut into
-// 16 KB chunks of 32 rows x 256 columns of the tile-packed layout, and the
+// 32 KB chunks of 32 rows x 512 columns of the tile-packed layout, and the
 // key/value pages of its attention unit -- and streams each chunk into a
 // shared-memory ring with cp.async.bulk, completing on an mbarrier.  Weights
 // and the cache entries of earlier positions do not depend on the step, so
@@ -46,7 +46,8 @@ namespace {
 
 constexpr int kCW = kSegConsumerWarps;
 constexpr int kCT = 32 * kCW;              // consumer threads
-constexpr int kColsPerChunk = kSegChunk / (2 * kTileRows);  // 256
+constexpr int kColsPerChunk = kSegChunk / (2 * kTileRows);  // 512
+constexpr int kCCPerWarp = (kColsPerChunk / 8 + kCW - 1) / kCW;  // 16-byte column chunks a warp takes per stage
 // Wait bounds in SM clock cycles (clock64 is cheap to read; the global
 // timer and the error word in global memory are not, so a waiting thread
 // looks at them only about once per millisecond).
@@ -195,6 +196,42 @@ __device__ __forceinline__ float dot8s(const uint4 w, uint32_t xa) {
     s = fmaf(bfhi(w.w), b.w, s);
     return s;
 }
+// Dot products of one ring stage for one warp: lane = row of the tile, the
+// warp's 16-byte column chunks are w, w + kCW, ... (stage byte address `wl`
+// already offset by lane * 16 + w * 512, input address `xl` by w * 32).
+// Full stages take the branch-free path with every chunk's product an
+// independent chain; a ragged last stage of a row checks each chunk.
+template <int CC>
+__device__ __forceinline__ float stage_dot(uint32_t wl, uint32_t xl, int cc_first, int ccn) {
+    if (cc_first + (CC - 1) * kSegConsumerWarps < ccn) {
+        uint4 wv[CC];
+#pragma unroll
+        for (int u = 0; u < CC; ++u) wv[u] = lds128(wl + u * kSegConsumerWarps * 512);
+        float a[CC];
+#pragma unroll
+        for (int u = 0; u < CC; ++u) {
+            const float4 x0 = lds128f(xl + u * kSegConsumerWarps * 32);
+            const float4 x1 = lds128f(xl + u * kSegConsumerWarps * 32 + 16);
+            float p0 = bflo(wv[u].x) * x0.x, p1 = bfhi(wv[u].x) * x0.y;
+            p0 = fmaf(bflo(wv[u].y), x0.z, p0);
+            p1 = fmaf(bfhi(wv[u].y), x0.w, p1);
+            p0 = fmaf(bflo(wv[u].z), x1.x, p0);
+            p1 = fmaf(bfhi(wv[u].z), x1.y, p1);
+            p0 = fmaf(bflo(wv[u].w), x1.z, p0);
+            p1 = fmaf(bfhi(wv[u].w), x1.w, p1);
+            a[u] = p0 + p1;
+        }
+        float t = 0.f;
+#pragma unroll
+        for (int u = 0; u < CC; ++u) t += a[u];
+        return t;
+    }
+    float t = 0.f;
+    for (int u = 0; cc_first + u * kSegConsumerWarps < ccn; ++u)
+        t += dot8s(lds128(wl + u * kSegConsumerWarps * 512), xl + u * kSegConsumerWarps * 32);
+    return t;
+}
+
 __device__ __forceinline__ float dot8(const uint4 w, const float* x) {
     const float4 a = *reinterpret_cast<const float4*>(x);
     const float4 b = *reinterpret_cast<const float4*>(x + 4);
@@ -210,12 +247,14 @@ __device__ __forceinline__ float dot8(const uint4 w, const float* x) {
 }
 
 // ------------------------------------------------------------ work geometry
-// Q/K/V, O and gate/up are split by whole 32-row tiles: rank r < Ge =
+// Q/K/V and gate/up are split by whole 32-row tiles: rank r < Ge =
 // min(G, n_tiles) owns tiles [r n / Ge, (r + 1) n / Ge) and runs on CTA
 // r G / Ge, so each of those phases finishes its rows in one CTA and applies
-// its epilogue there.  The down projection (few rows, long rows) is split
-// into (tile, 256-column chunk) items over all CTAs; each CTA writes the
-// partial sums of the tiles it touched into its slot [tile][slot][32].
+// its epilogue there.  The O and down projections (few rows, long rows) are
+// split into (tile, 512-column chunk) items over all CTAs.  An O item writes
+// its chunk's partial sums to slot [tile][chunk][32] (chunk 0 also carries
+// the residual entering the layer), so the mid residual is the sum of a
+// tile's O slots; a down item adds into its CTA's slot [tile][slot][32].
 __device__ __forceinline__ void whole_tiles(int n_t, int G, int cta, int& t0, int& t1) {
     const int Ge = min(G, n_t);
     const int r = (int)(((int64_t)cta * Ge + G - 1) / G);
@@ -229,11 +268,11 @@ __device__ __forceinline__ void whole_tiles(int n_t, int G, int cta, int& t0, in
 struct Items {
     int N, Ge, lo, hi, nc, K;
 };
-__device__ __forceinline__ Items down_items(const SegPlan& p, int cta) {
+__device__ __forceinline__ Items items_for(const SegPlan& p, int mt, int cta) {
     Items it;
-    it.nc = p.n_chunks[3];
-    it.K = p.K[3];
-    it.N = p.n_tiles[3] * it.nc;
+    it.nc = p.n_chunks[mt];
+    it.K = p.K[mt];
+    it.N = p.n_tiles[mt] * it.nc;
     it.Ge = min(p.G, it.N);
     if (cta < it.Ge) {
         it.lo = (int)((int64_t)cta * it.N / it.Ge);
@@ -284,7 +323,11 @@ struct Smem {
     uint64_t* empty;    // [stages]
     float* xs;          // [max(d, A D)] input vector of a whole-tile phase
     float* hs;          // [d] residual
-    float* xa;          // [max down items][256] staged input columns of the down items
+    float* xa;          // [max items][512] staged input columns of the O / down items, then
+                        // [max items][32] residual rows of the O items of chunk 0
+    float2* rope;       // [D/2] (cos, sin) of the step's position
+    uint16_t* ga;       // [d] attention-norm gain of the current layer
+    uint16_t* gm;       // [d] MLP-norm gain of the current layer
     float* red;         // [2][kCW][32]
     float* qa;          // [group][D] scaled queries of the attention unit
     float* kv;          // [2][D] k, v of the step's position
@@ -308,7 +351,13 @@ __device__ __forceinline__ Smem carve(uint8_t* base, const DevModel& m, const Se
     s.hs = f;
     f += (m.d + 3) & ~3;
     s.xa = f;
-    f += p.max_dn_items * kColsPerChunk;
+    f += p.max_items * (kColsPerChunk + 32);
+    s.rope = reinterpret_cast<float2*>(f);
+    f += m.D;
+    s.ga = reinterpret_cast<uint16_t*>(f);
+    f += (m.d + 1) / 2;
+    s.gm = reinterpret_cast<uint16_t*>(f);
+    f += (m.d + 1) / 2;
     s.red = f;
     f += 2 * kCW * 32;
     const int grp = m.A / m.KH;
@@ -439,25 +488,54 @@ __device__ __forceinline__ bool wait_count(const unsigned* cnt, unsigned target,
     csync();
     return ok_s != 0;
 }
-// All consumer threads' global writes, then one release increment.
+// All consumer threads' global writes, then one release increment: the
+// consumer barrier orders the other threads' writes before thread 0's
+// fence and release (the pattern of a cooperative grid barrier).
 __device__ __forceinline__ void signal_count(unsigned* cnt) {
-    __threadfence();
     csync();
-    if (threadIdx.x == 0) asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(cnt) : "memory");
+    if (threadIdx.x == 0) {
+        __threadfence();
+        asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(cnt) : "memory");
+    }
 }
 
-// dst[i] = f(i) for i < n, four elements per thread per round with all their
+// dst[i] = f(i) for i < n, eight elements per thread per round with all their
 // loads issued before any store (f reads global memory).
 template <class F>
 __device__ __forceinline__ void gather(float* dst, int n, F f) {
-    for (int b = threadIdx.x; b < n; b += 4 * kCT) {
-        float v[4];
+    for (int b = threadIdx.x; b < n; b += 8 * kCT) {
+        float v[8];
 #pragma unroll
-        for (int e = 0; e < 4; ++e) v[e] = (b + e * kCT < n) ? f(b + e * kCT) : 0.f;
+        for (int e = 0; e < 8; ++e) v[e] = (b + e * kCT < n) ? f(b + e * kCT) : 0.f;
 #pragma unroll
-        for (int e = 0; e < 4; ++e)
+        for (int e = 0; e < 8; ++e)
             if (b + e * kCT < n) dst[b + e * kCT] = v[e];
     }
+}
+
+// The same with four consecutive elements per call (n and dst 4-aligned):
+// f(i) returns elements i..i+3 as one float4, so a warp's loads are 16 bytes
+// per lane and a thread has fewer of them in flight.
+template <class F>
+__device__ __forceinline__ void gather4(float* dst, int n, F f) {
+    const int n4 = n >> 2;
+    float4* d4 = reinterpret_cast<float4*>(dst);
+    for (int b = threadIdx.x; b < n4; b += 8 * kCT) {
+        float4 v[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) v[e] = (b + e * kCT < n4) ? f(4 * (b + e * kCT)) : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int e = 0; e < 8; ++e)
+            if (b + e * kCT < n4) d4[b + e * kCT] = v[e];
+    }
+}
+__device__ __forceinline__ float4 f4add(float4 a, float4 b) {
+    return make_float4(a.x + b.x, a.y + b.y, a.z + b.z, a.w + b.w);
+}
+__device__ __forceinline__ float4 ldg4(const float* p) { return *reinterpret_cast<const float4*>(p); }
+__device__ __forceinline__ float4 bf4(const uint16_t* p) {
+    const uint2 u = *reinterpret_cast<const uint2*>(p);
+    return make_float4(bflo(u.x), bfhi(u.x), bflo(u.y), bfhi(u.y));
 }
 
 // RMSNorm of hs (d values) times gain g into xs (consumer threads).
@@ -486,18 +564,10 @@ __device__ __forceinline__ void tile_gemv(Consumer& cs, int t0, int t1, int K, i
     for (int t = t0; t < t1; ++t) {
         float acc = 0.f;
         for (int c = 0; c < nc; ++c) {
-            const uint32_t buf = saddr(cs.acquire()) + lane * 16;
+            const uint32_t buf = saddr(cs.acquire()) + lane * 16 + w * 512;
             const int ccn = (int)(chunk_bytes(K, c) / 512);
-            const uint32_t xc = saddr(x + c * kColsPerChunk);
-            if (cs.ok) {
-                uint4 wv[4];
-#pragma unroll
-                for (int u = 0; u < 4; ++u)
-                    if (w + u * kCW < ccn) wv[u] = lds128(buf + (w + u * kCW) * 512);
-#pragma unroll
-                for (int u = 0; u < 4; ++u)
-                    if (w + u * kCW < ccn) acc += dot8s(wv[u], xc + (w + u * kCW) * 32);
-            }
+            const uint32_t xc = saddr(x + c * kColsPerChunk) + w * 32;
+            if (cs.ok) acc += stage_dot<kCCPerWarp>(buf, xc, w, ccn);
             cs.release();
         }
         float* r = red + rb * kCW * 32;
@@ -514,28 +584,63 @@ __device__ __forceinline__ void tile_gemv(Consumer& cs, int t0, int t1, int K, i
 }
 
 // Residual entering layer j at row i: the embedding (first layer of a step),
-// the model's h (first layer of a later segment), or the previous layer's
-// mid residual plus its down-projection slots.
+// the model's h (first layer of a later segment), or the previous layer's O
+// slots (its mid residual) plus its down slots.
 struct ResidIn {
-    const DevModel* m;
     const SegPlan* p;
     const uint16_t* emb;  // embedding row, or null
-    const float* src;     // m.h or the mid residual
-    bool add_down;
+    const float* src;     // m.h, or null for the slot sums
+    const float* opart;   // the previous layer's O slots
     const uint8_t* nsd;
     __device__ __forceinline__ float operator()(int i) const {
         if (emb) return bf(emb[i]);
-        float v = src[i];
-        if (add_down) {
-            const int t = i >> 5, ns = nsd[t];
-            const float* q = p->dpart + (int64_t)t * p->n_chunks[3] * 32 + (i & 31);
+        if (src) return src[i];
+        const int t = i >> 5, l = i & 31, nco = p->n_chunks[1], ns = nsd[t];
+        const float* qo = opart + (int64_t)t * nco * 32 + l;
+        const float* qd = p->dpart + (int64_t)t * p->n_chunks[3] * 32 + l;
+        float v = 0.f;
 #pragma unroll
-            for (int k = 0; k < kSegMaxSlots; ++k)
-                if (k < ns) v += q[k * 32];
-        }
+        for (int k = 0; k < kSegMaxSlots; ++k)
+            if (k < nco) v += qo[k * 32];
+#pragma unroll
+        for (int k = 0; k < kSegMaxSlots; ++k)
+            if (k < ns) v += qd[k * 32];
+        return v;
+    }
+    // rows i..i+3 (i a multiple of 4, same tile)
+    __device__ __forceinline__ float4 four(int i) const {
+        if (emb) return bf4(emb + i);
+        if (src) return ldg4(src + i);
+        const int t = i >> 5, l = i & 31, nco = p->n_chunks[1], ns = nsd[t];
+        const float* qo = opart + (int64_t)t * nco * 32 + l;
+        const float* qd = p->dpart + (int64_t)t * p->n_chunks[3] * 32 + l;
+        float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int k = 0; k < kSegMaxSlots; ++k)
+            if (k < nco) v = f4add(v, ldg4(qo + k * 32));
+#pragma unroll
+        for (int k = 0; k < kSegMaxSlots; ++k)
+            if (k < ns) v = f4add(v, ldg4(qd + k * 32));
         return v;
     }
 };
+// O slots of layer j: two buffers, alternating by layer (a chunk-0 O item
+// reads the previous layer's slots while the other items of its tile write
+// this layer's).
+__device__ __forceinline__ float* opart_of(const SegPlan& p, int j) {
+    return p.opart + (int64_t)(j & 1) * p.n_tiles[1] * p.n_chunks[1] * 32;
+}
+// Mid residual (after the attention block) at rows i..i+3: the sum of the O
+// slots.
+__device__ __forceinline__ float4 resid_mid4(const SegPlan& p, const float* opart, int i) {
+    const int t = i >> 5, nco = p.n_chunks[1];
+    const float* qo = opart + (int64_t)t * nco * 32 + (i & 31);
+    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int k = 0; k < kSegMaxSlots; ++k)
+        if (k < nco) v = f4add(v, ldg4(qo + k * 32));
+    return v;
+}
 
 }  // namespace
 
@@ -562,39 +667,74 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
     const AttnGeo ag = attn_geo(m, p, pos_ok ? pos : 0);
     const int unit = attn_unit(ag, G, cta);
     const int rpc = p.rows_per_kv_chunk, cpp = m.page_size / rpc;
-    int tq0, tq1, to0, to1, tg0, tg1;
+    int tq0, tq1, tg0, tg1;
     whole_tiles(p.n_tiles[0], G, cta, tq0, tq1);
-    whole_tiles(p.n_tiles[1], G, cta, to0, to1);
     whole_tiles(p.n_tiles[2], G, cta, tg0, tg1);
-    const Items idn = down_items(p, cta);
+    const Items io = items_for(p, 1, cta);
+    const Items idn = items_for(p, 3, cta);
 
     // ---------------------------------------------------------- producer
     if (threadIdx.x >= kCT) {
         if (threadIdx.x != kCT || !pos_ok) return;
         Producer pr(s, p.stages, min(p.stages, p.inflight), err);
-        for (int j = j0; j < j1 && pr.ok; ++j) {
-            pr.tiles(mat_base(m, j, 0), p.K[0], p.n_chunks[0], tq0, tq1);
-            if (unit >= 0) {
-                const int g = unit / ag.splits, sp = unit - g * ag.splits;
-                const int pg0 = sp * ag.pps, pg1 = min(ag.n_pages, pg0 + ag.pps);
-                const uint16_t* pools[2] = {m.kpool + (int64_t)j * m.kv_layer_stride,
-                                            m.vpool + (int64_t)j * m.kv_layer_stride};
-                for (int kvi = 0; kvi < 2; ++kvi)
-                    for (int pg = pg0; pg < pg1; ++pg) {
-                        const int phys = m.page_table[pg];
-                        for (int q = 0; q < cpp; ++q)
-                            pr.push(pools[kvi] + (((int64_t)phys * m.KH + g) * m.page_size + q * rpc) * m.D,
-                                    (uint32_t)(rpc * m.D * 2), pr.pol_kv);
-                    }
+        // The CTA's chunk list, layer by layer: its Q/K/V tiles, its
+        // attention unit's K then V pages, its O items, its gate/up tiles,
+        // its down items.
+        const int nc0 = p.n_chunks[0], nc2 = p.n_chunks[2];
+        int pg0 = 0, pg1 = 0, g = 0;
+        if (unit >= 0) {
+            g = unit / ag.splits;
+            const int sp = unit - g * ag.splits;
+            pg0 = sp * ag.pps;
+            pg1 = min(ag.n_pages, pg0 + ag.pps);
+        }
+        const int nq = (tq1 - tq0) * nc0, nkv = 2 * (pg1 - pg0) * cpp, no = io.hi - io.lo;
+        const int ng = (tg1 - tg0) * nc2, nd = idn.hi - idn.lo;
+        const int per = nq + nkv + no + ng + nd;
+        const long long total = (long long)per * (j1 - j0);
+        auto chunk = [&](long long n, const void*& src, uint32_t& bytes) -> bool {  // true: a cache page
+            const int j = j0 + (int)(n / per);
+            int r = (int)(n - (long long)(j - j0) * per);
+            if (r < nq) {
+                const int t = tq0 + r / nc0, ch = r - (r / nc0) * nc0;
+                src = mat_base(m, j, 0) + (int64_t)t * kTileRows * p.K[0] * 2 + (int64_t)ch * kSegChunk;
+                bytes = chunk_bytes(p.K[0], ch);
+                return false;
             }
-            pr.tiles(mat_base(m, j, 1), p.K[1], p.n_chunks[1], to0, to1);
-            pr.tiles(mat_base(m, j, 2), p.K[2], p.n_chunks[2], tg0, tg1);
-            const uint8_t* Wd = mat_base(m, j, 3);
-            for (int i = idn.lo; i < idn.hi; ++i) {
-                const int t = i / idn.nc, ch = i - t * idn.nc;
-                pr.push(Wd + (int64_t)t * kTileRows * idn.K * 2 + (int64_t)ch * kSegChunk, chunk_bytes(idn.K, ch),
-                        pr.pol_w);
+            r -= nq;
+            if (r < nkv) {
+                const int per_kv = (pg1 - pg0) * cpp, kvi = r / per_kv, r2 = r - kvi * per_kv;
+                const int pg = pg0 + r2 / cpp, q = r2 - (r2 / cpp) * cpp;
+                const uint16_t* pool = (kvi ? m.vpool : m.kpool) + (int64_t)j * m.kv_layer_stride;
+                src = pool + (((int64_t)m.page_table[pg] * m.KH + g) * m.page_size + q * rpc) * m.D;
+                bytes = (uint32_t)(rpc * m.D * 2);
+                return true;
             }
+            r -= nkv;
+            if (r < no) {
+                const int i = io.lo + r, t = i / io.nc, ch = i - t * io.nc;
+                src = mat_base(m, j, 1) + (int64_t)t * kTileRows * io.K * 2 + (int64_t)ch * kSegChunk;
+                bytes = chunk_bytes(io.K, ch);
+                return false;
+            }
+            r -= no;
+            if (r < ng) {
+                const int t = tg0 + r / nc2, ch = r - (r / nc2) * nc2;
+                src = mat_base(m, j, 2) + (int64_t)t * kTileRows * p.K[2] * 2 + (int64_t)ch * kSegChunk;
+                bytes = chunk_bytes(p.K[2], ch);
+                return false;
+            }
+            r -= ng;
+            const int i = idn.lo + r, t = i / idn.nc, ch = i - t * idn.nc;
+            src = mat_base(m, j, 3) + (int64_t)t * kTileRows * idn.K * 2 + (int64_t)ch * kSegChunk;
+            bytes = chunk_bytes(idn.K, ch);
+            return false;
+        };
+        for (long long n = 0; n < total && pr.ok; ++n) {
+            const void* src;
+            uint32_t bytes;
+            const bool kv = chunk(n, src, bytes);
+            pr.push(src, bytes, kv ? pr.pol_kv : pr.pol_w);
         }
         pr.drain();
         return;
@@ -608,13 +748,14 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
     }
     Consumer cs(s, p.stages, err);
     unsigned* sync = p.sync;
-    const float2* cs_row = m.rope + (int64_t)pos * half;
+    for (int i = threadIdx.x; i < half; i += kCT) s.rope[i] = m.rope[(int64_t)pos * half + i];
+    const float2* cs_row = s.rope;
     const float scale = 1.0f / sqrtf((float)m.D);
     const int slice0 = (int)((int64_t)cta * m.d / G), slice1 = (int)((int64_t)(cta + 1) * m.d / G);
     const int nq = m.A * half, nk = m.KH * half;
     const int64_t kvo_pos = ((int64_t)m.page_table[pos / m.page_size] * m.KH * m.page_size + pos % m.page_size) * m.D;
     {   // slots of each down tile
-        Items all = down_items(p, 0);
+        Items all = items_for(p, 3, 0);
         for (int t = threadIdx.x; t < p.n_tiles[3]; t += kCT)
             s.nsd[t] = (uint8_t)(item_owner(all, t * all.nc + all.nc - 1) - item_owner(all, t * all.nc) + 1);
     }
@@ -637,15 +778,27 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
         const int li = j - j0;
         unsigned* cnt = sync + li * kPhases;
         const uint16_t* lw = m.layers + (int64_t)j * m.layer_stride;
-        const ResidIn rin{&m, &p, (j == j0 && first) ? m.embed + (int64_t)tok * m.d : nullptr,
-                          j == j0 ? m.h : p.hmid, j > j0, s.nsd};
+        float* op_cur = opart_of(p, j);
+        const ResidIn rin{&p, (j == j0 && first) ? m.embed + (int64_t)tok * m.d : nullptr, j == j0 ? m.h : nullptr,
+                          opart_of(p, j - 1), s.nsd};
+        {   // this layer's norm gains, ahead of the waits
+            const uint32_t* g1 = reinterpret_cast<const uint32_t*>(lw + m.off_gattn);
+            const uint32_t* g2 = reinterpret_cast<const uint32_t*>(lw + m.off_gmlp);
+            uint32_t* d1 = reinterpret_cast<uint32_t*>(s.ga);
+            uint32_t* d2 = reinterpret_cast<uint32_t*>(s.gm);
+            for (int i = threadIdx.x; i < m.d / 2; i += kCT) {
+                const uint32_t a1 = g1[i], a2 = g2[i];
+                d1[i] = a1;
+                d2[i] = a2;
+            }
+        }
 
         // ---------------- Q/K/V tiles: RMSNorm, projection, bias, RoPE, KV append
         if (tq1 > tq0) {
             if (j > j0 && !wait_count(cnt - kPhases + kPhDn, G, err)) return;
-            gather(s.hs, m.d, rin);
+            gather4(s.hs, m.d, [&](int i) { return rin.four(i); });
             csync();
-            rmsnorm_sm(s.hs, lw + m.off_gattn, m.d, m.eps, s.xs, s.red);
+            rmsnorm_sm(s.hs, s.ga, m.d, m.eps, s.xs, s.red);
             const uint16_t* bias = m.qkv_bias ? lw + m.off_bqkv : nullptr;
             uint16_t* kdst = m.kpool + (int64_t)j * m.kv_layer_stride + kvo_pos;
             uint16_t* vdst = m.vpool + (int64_t)j * m.kv_layer_stride + kvo_pos;
@@ -693,29 +846,39 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
             const float* qsrc = m.q + (int64_t)g * grp * m.D;
             const uint16_t* kt = m.kpool + (int64_t)j * m.kv_layer_stride + kvo_pos + (int64_t)g * m.page_size * m.D;
             const uint16_t* vt = m.vpool + (int64_t)j * m.kv_layer_stride + kvo_pos + (int64_t)g * m.page_size * m.D;
-            gather(s.qa, grp * m.D, [&](int i) { return qsrc[i] * scale; });
-            gather(s.kv, 2 * m.D, [&](int i) { return i < m.D ? bf(kt[i]) : bf(vt[i - m.D]); });
+            gather4(s.qa, grp * m.D, [&](int i) {
+                const float4 q = ldg4(qsrc + i);
+                return make_float4(q.x * scale, q.y * scale, q.z * scale, q.w * scale);
+            });
+            gather4(s.kv, 2 * m.D, [&](int i) { return i < m.D ? bf4(kt + i) : bf4(vt + i - m.D); });
             csync();
-            // scores: warp per position, lane per D/32 dimensions
+            // scores: warp per position, lane per D/32 dimensions, q read from
+            // shared memory per head
             const int dpl = m.D >> 5;  // 2 or 4
+            const int spc = p.max_pps * m.page_size;  // score row stride
             float qr[kSegMaxGroup][4];
 #pragma unroll
             for (int hh = 0; hh < kSegMaxGroup; ++hh)
 #pragma unroll
                 for (int k = 0; k < 4; ++k) qr[hh][k] = (hh < grp && k < dpl) ? s.qa[hh * m.D + lane * dpl + k] : 0.f;
-            const int spc = p.max_pps * m.page_size;  // score row stride
+            // k and v of the step's own position (the ring holds the cache's
+            // stale copy of that row): substituted by a select, not a branch
+            float kvt[4], vvt[4];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                kvt[k] = k < dpl ? s.kv[lane * dpl + k] : 0.f;
+                vvt[k] = k < dpl ? s.kv[m.D + lane * dpl + k] : 0.f;
+            }
             for (int pg = pg0; pg < pg1; ++pg)
                 for (int q = 0; q < cpp; ++q) {
                     const uint32_t kb = saddr(cs.acquire()) + lane * dpl * 2;
                     const int base = pg * m.page_size + q * rpc;
-                    for (int r = w; r < rpc; r += kCW) {
+                    const int nr = min(rpc, p1 - base);
+#pragma unroll 2
+                    for (int r = w; r < nr; r += kCW) {
                         const int ps = base + r;
-                        if (ps >= p1) break;
                         float kd[4];
-                        if (ps == pos) {
-#pragma unroll
-                            for (int k = 0; k < 4; ++k) kd[k] = k < dpl ? s.kv[lane * dpl + k] : 0.f;
-                        } else if (dpl == 4) {
+                        if (dpl == 4) {
                             const uint2 v = lds64(kb + r * m.D * 2);
                             kd[0] = bflo(v.x);
                             kd[1] = bfhi(v.x);
@@ -727,12 +890,15 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
                             kd[1] = bfhi(v);
                             kd[2] = kd[3] = 0.f;
                         }
+#pragma unroll
+                        for (int k = 0; k < 4; ++k) kd[k] = ps == pos ? kvt[k] : kd[k];
                         float dd[kSegMaxGroup];
 #pragma unroll
                         for (int hh = 0; hh < kSegMaxGroup; ++hh) {
-                            float d = 0.f;
-#pragma unroll
-                            for (int k = 0; k < 4; ++k) d = fmaf(qr[hh][k], kd[k], d);
+                            float d = qr[hh][0] * kd[0];
+                            d = fmaf(qr[hh][1], kd[1], d);
+                            d = fmaf(qr[hh][2], kd[2], d);
+                            d = fmaf(qr[hh][3], kd[3], d);
                             dd[hh] = d;
                         }
                         // reduce-scatter over the warp: lane bits 4, 3, 2 pick the head
@@ -772,64 +938,88 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
                 }
             }
             csync();
-            // P V: warp per head, lane per D/32 dimensions
-            float oacc[4] = {0.f, 0.f, 0.f, 0.f};
+            // P V: warp w works on head w % grp for the positions r with
+            // r % nsp == w / grp; the nsp partial sums meet in xs (free here)
+            const int nsp = max(1, min(kCW / grp, max(m.d, AD) / (grp * m.D)));
+            const int hw = w % grp, part = w / grp;
+            const bool pv = w < grp * nsp;
+            float oacc[4] = {0.f, 0.f, 0.f, 0.f}, obcc[4] = {0.f, 0.f, 0.f, 0.f};
             for (int pg = pg0; pg < pg1; ++pg)
                 for (int q = 0; q < cpp; ++q) {
-                    const uint16_t* vb = reinterpret_cast<const uint16_t*>(cs.acquire());
+                    const uint32_t vb = saddr(cs.acquire()) + lane * dpl * 2;
                     const int base = pg * m.page_size + q * rpc;
                     const int nr = min(rpc, p1 - base);
-                    if (w < grp && cs.ok) {
-                        const uint32_t pw = saddr(s.sc + w * spc + (base - p0));
-                        const uint32_t vrow = saddr(vb) + lane * dpl * 2;
-                        const int rt = (pos >= base && pos < base + nr) ? pos - base : -1;
-                        const int rs = rt >= 0 ? rt : nr;  // rows before the step's own position
-#pragma unroll 4
-                        for (int r = 0; r < rs; ++r) {
-                            const float pr = ldsf(pw + 4 * r);
+                    if (pv && cs.ok) {
+                        const uint32_t pw = saddr(s.sc + hw * spc + (base - p0));
+                        // two positions per step into two accumulator sets
+                        for (int r = part; r < nr; r += 2 * nsp) {
+                            const int r2 = r + nsp;
+                            const bool two = r2 < nr;
+                            const float pa = ldsf(pw + 4 * r), pb = two ? ldsf(pw + 4 * r2) : 0.f;
+                            float va[4], vb2[4];
                             if (dpl == 4) {
-                                const uint2 v = lds64(vrow + r * m.D * 2);
-                                oacc[0] = fmaf(pr, bflo(v.x), oacc[0]);
-                                oacc[1] = fmaf(pr, bfhi(v.x), oacc[1]);
-                                oacc[2] = fmaf(pr, bflo(v.y), oacc[2]);
-                                oacc[3] = fmaf(pr, bfhi(v.y), oacc[3]);
+                                const uint2 ua = lds64(vb + r * m.D * 2);
+                                const uint2 ub = lds64(vb + (two ? r2 : r) * m.D * 2);
+                                va[0] = bflo(ua.x), va[1] = bfhi(ua.x), va[2] = bflo(ua.y), va[3] = bfhi(ua.y);
+                                vb2[0] = bflo(ub.x), vb2[1] = bfhi(ub.x), vb2[2] = bflo(ub.y), vb2[3] = bfhi(ub.y);
                             } else {
-                                const uint32_t v = lds32(vrow + r * m.D * 2);
-                                oacc[0] = fmaf(pr, bflo(v), oacc[0]);
-                                oacc[1] = fmaf(pr, bfhi(v), oacc[1]);
+                                const uint32_t ua = lds32(vb + r * m.D * 2);
+                                const uint32_t ub = lds32(vb + (two ? r2 : r) * m.D * 2);
+                                va[0] = bflo(ua), va[1] = bfhi(ua), va[2] = va[3] = 0.f;
+                                vb2[0] = bflo(ub), vb2[1] = bfhi(ub), vb2[2] = vb2[3] = 0.f;
                             }
-                        }
-                        if (rt >= 0) {  // the step's own position: v from the Q/K/V phase
-                            const float pr = ldsf(pw + 4 * rt);
+                            // the stale cache row of the step's own position (and the
+                            // stand-in row when there is no second position) is
+                            // selected away, never multiplied by zero: it may hold
+                            // anything, NaN included
 #pragma unroll
-                            for (int k = 0; k < 4; ++k)
-                                if (k < dpl) oacc[k] = fmaf(pr, s.kv[m.D + lane * dpl + k], oacc[k]);
+                            for (int k = 0; k < 4; ++k) {
+                                oacc[k] = fmaf(pa, base + r == pos ? vvt[k] : va[k], oacc[k]);
+                                const float v2 = !two ? 0.f : (base + r2 == pos ? vvt[k] : vb2[k]);
+                                obcc[k] = fmaf(pb, v2, obcc[k]);
+                            }
                         }
                     }
                     cs.release();
                 }
-            if (w < grp) {
-                float* dst = p.attn_part + ((int64_t)(g * grp + w) * kAttnMaxSplits + sp) * (m.D + 2);
+#pragma unroll
+            for (int k = 0; k < 4; ++k) oacc[k] += obcc[k];
+            if (pv && part > 0) {
+                float* dst = s.xs + ((part - 1) * grp + hw) * m.D + lane * dpl;
+#pragma unroll
+                for (int k = 0; k < 4; ++k)
+                    if (k < dpl) dst[k] = oacc[k];
+            }
+            csync();
+            if (pv && part == 0) {
+                for (int pp = 1; pp < nsp; ++pp) {
+                    const float* src = s.xs + ((pp - 1) * grp + hw) * m.D + lane * dpl;
+#pragma unroll
+                    for (int k = 0; k < 4; ++k)
+                        if (k < dpl) oacc[k] += src[k];
+                }
+                float* dst = p.attn_part + ((int64_t)(g * grp + hw) * kSegMaxSplits + sp) * (m.D + 4);
 #pragma unroll
                 for (int k = 0; k < 4; ++k)
                     if (k < dpl) dst[lane * dpl + k] = oacc[k];
                 if (lane == 0) {
-                    dst[m.D] = s.ml[2 * w];
-                    dst[m.D + 1] = s.ml[2 * w + 1];
+                    dst[m.D] = s.ml[2 * hw];
+                    dst[m.D + 1] = s.ml[2 * hw + 1];
                 }
             }
         }
         signal_count(cnt + kPhAttn);
 
-        // ---------------- O tiles: merge the attention splits, project, add the residual
-        if (to1 > to0) {
+        // ---------------- O items: merge the attention splits of the chunk's heads,
+        // project, write the chunk's slot (chunk 0 adds the residual)
+        if (io.hi > io.lo) {
             if (!wait_count(cnt + kPhAttn, G, err)) return;
             const int ns = ag.splits;
             float* den = s.wts + m.A * kSegMaxSplits;
             for (int h = w; h < m.A; h += kCW) {  // split weights exp(m_s - M) of each head
-                const float* src = p.attn_part + (int64_t)h * kAttnMaxSplits * (m.D + 2) + m.D;
-                const float ms = lane < ns ? src[lane * (m.D + 2)] : -INFINITY;
-                const float ls = lane < ns ? src[lane * (m.D + 2) + 1] : 0.f;
+                const float* src = p.attn_part + (int64_t)h * kSegMaxSplits * (m.D + 4) + m.D;
+                const float ms = lane < ns ? src[lane * (m.D + 4)] : -INFINITY;
+                const float ls = lane < ns ? src[lane * (m.D + 4) + 1] : 0.f;
                 const float mx = warp_max(ms);
                 const float wt = lane < ns ? expf(ms - mx) : 0.f;
                 if (lane < ns) s.wts[h * kSegMaxSplits + lane] = wt;
@@ -837,28 +1027,60 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
                 if (lane == 0) den[h] = dn;
             }
             csync();
-            gather(s.xs, AD, [&](int col) {
+            const int nit = io.hi - io.lo, ncol = nit * kColsPerChunk;
+            const float* rows = s.xa + ncol;
+            gather4(s.xa, ncol + nit * 32, [&](int e) {
+                if (e >= ncol) {  // residual rows of the chunk-0 items
+                    const int it = (e - ncol) >> 5, i = io.lo + it, t = i / io.nc;
+                    const int row = t * 32 + ((e - ncol) & 31);
+                    return (i - t * io.nc == 0 && row < m.d) ? rin.four(row) : make_float4(0.f, 0.f, 0.f, 0.f);
+                }
+                const int i = io.lo + e / kColsPerChunk, ch = i % io.nc;
+                const int col = ch * kColsPerChunk + e % kColsPerChunk;
+                if (col >= AD) return make_float4(0.f, 0.f, 0.f, 0.f);
                 const int h = col / m.D;
-                const float* src = p.attn_part + (int64_t)h * kAttnMaxSplits * (m.D + 2) + (col - h * m.D);
+                const float* src = p.attn_part + (int64_t)h * kSegMaxSplits * (m.D + 4) + (col - h * m.D);
                 const float* wt = s.wts + h * kSegMaxSplits;
-                float num = 0.f;
-                for (int k = 0; k < ns; ++k) num = fmaf(wt[k], src[k * (m.D + 2)], num);
-                return num / den[h];
+                float4 num = make_float4(0.f, 0.f, 0.f, 0.f);
+                for (int k = 0; k < ns; ++k) {
+                    const float4 o = ldg4(src + k * (m.D + 4));
+                    const float wk = wt[k];
+                    num.x = fmaf(wk, o.x, num.x);
+                    num.y = fmaf(wk, o.y, num.y);
+                    num.z = fmaf(wk, o.z, num.z);
+                    num.w = fmaf(wk, o.w, num.w);
+                }
+                const float inv = 1.0f / den[h];
+                return make_float4(num.x * inv, num.y * inv, num.z * inv, num.w * inv);
             });
             csync();
-            tile_gemv(cs, to0, to1, p.K[1], p.n_chunks[1], s.xs, s.red, rb, [&](int t, float v) {
-                const int row = t * 32 + lane;
-                if (row < m.d) p.hmid[row] = rin(row) + v;
-            });
+            for (int i = io.lo; i < io.hi; ++i) {
+                const int t = i / io.nc, ch = i - t * io.nc;
+                const uint32_t buf = saddr(cs.acquire()) + lane * 16 + w * 512;
+                const int ccn = (int)(chunk_bytes(io.K, ch) / 512);
+                const uint32_t x = saddr(s.xa + (i - io.lo) * kColsPerChunk) + w * 32;
+                const float acc = cs.ok ? stage_dot<kCCPerWarp>(buf, x, w, ccn) : 0.f;
+                cs.release();
+                float* r = s.red + rb * kCW * 32;
+                r[w * 32 + lane] = acc;
+                csync();
+                if (w == 0) {
+                    float sum = ch == 0 ? rows[(i - io.lo) * 32 + lane] : 0.f;
+#pragma unroll
+                    for (int k = 0; k < kCW; ++k) sum += r[k * 32 + lane];
+                    op_cur[((int64_t)t * io.nc + ch) * 32 + lane] = sum;
+                }
+                rb ^= 1;
+            }
         }
         signal_count(cnt + kPhO);
 
         // ---------------- gate/up tiles: RMSNorm of the mid residual, SwiGLU
         if (tg1 > tg0) {
             if (!wait_count(cnt + kPhO, G, err)) return;
-            gather(s.hs, m.d, [&](int i) { return p.hmid[i]; });
+            gather4(s.hs, m.d, [&](int i) { return resid_mid4(p, op_cur, i); });
             csync();
-            rmsnorm_sm(s.hs, lw + m.off_gmlp, m.d, m.eps, s.xs, s.red);
+            rmsnorm_sm(s.hs, s.gm, m.d, m.eps, s.xs, s.red);
             tile_gemv(cs, tg0, tg1, p.K[2], p.n_chunks[2], s.xs, s.red, rb, [&](int t, float v) {
                 const float up = __shfl_xor_sync(0xffffffffu, v, 1);
                 const int f = t * 16 + (lane >> 1);
@@ -870,27 +1092,19 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
         // ---------------- down items: partial slots of h_out - h_mid
         if (idn.hi > idn.lo) {
             if (!wait_count(cnt + kPhGU, G, err)) return;
-            gather(s.xa, (idn.hi - idn.lo) * kColsPerChunk, [&](int e) {
+            gather4(s.xa, (idn.hi - idn.lo) * kColsPerChunk, [&](int e) {
                 const int i = idn.lo + e / kColsPerChunk, col = e % kColsPerChunk;
                 const int ch = i % idn.nc, f = ch * kColsPerChunk + col;
-                return f < m.F ? m.a[f] : 0.f;
+                return f < m.F ? ldg4(m.a + f) : make_float4(0.f, 0.f, 0.f, 0.f);
             });
             csync();
             float acc = 0.f;
             for (int i = idn.lo; i < idn.hi; ++i) {
                 const int t = i / idn.nc, ch = i - t * idn.nc;
-                const uint32_t buf = saddr(cs.acquire()) + lane * 16;
+                const uint32_t buf = saddr(cs.acquire()) + lane * 16 + w * 512;
                 const int ccn = (int)(chunk_bytes(idn.K, ch) / 512);
-                const uint32_t x = saddr(s.xa + (i - idn.lo) * kColsPerChunk);
-                if (cs.ok) {
-                    uint4 wv[4];
-#pragma unroll
-                    for (int u = 0; u < 4; ++u)
-                        if (w + u * kCW < ccn) wv[u] = lds128(buf + (w + u * kCW) * 512);
-#pragma unroll
-                    for (int u = 0; u < 4; ++u)
-                        if (w + u * kCW < ccn) acc += dot8s(wv[u], x + (w + u * kCW) * 32);
-                }
+                const uint32_t x = saddr(s.xa + (i - idn.lo) * kColsPerChunk) + w * 32;
+                if (cs.ok) acc += stage_dot<kCCPerWarp>(buf, x, w, ccn);
                 cs.release();
                 if (i + 1 == idn.hi || ch + 1 == idn.nc) {
                     float* r = s.red + rb * kCW * 32;
@@ -914,8 +1128,8 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
     // ---------------- the segment's output residual, then the exit ticket
     if (!wait_count(sync + (j1 - 1 - j0) * kPhases + kPhDn, G, err)) return;
     {
-        const ResidIn rout{&m, &p, nullptr, p.hmid, true, s.nsd};
-        for (int i = slice0 + threadIdx.x; i < slice1; i += kCT) m.h[i] = rout(i);
+        const ResidIn rout{&p, nullptr, nullptr, opart_of(p, j1 - 1), s.nsd};
+        for (int i = slice0 + threadIdx.x; i < slice1; i += kCT) m.h[i] = rout(i);  // slice: scalar
     }
     __threadfence();
     csync();
@@ -941,10 +1155,13 @@ bool seg_plan(const DevModel& m, int n_sm, SegPlan& p) {
         p.n_tiles[i] = (int)tile_count(rows[i]);
         p.n_chunks[i] = (Ks[i] + kColsPerChunk - 1) / kColsPerChunk;
     }
-    // down items: slots per tile within kSegMaxSlots, items per CTA sized
+    // O and down items: chunks per O tile and slots per down tile within
+    // kSegMaxSlots; items per CTA size the staging buffer
+    if (p.n_chunks[1] > kSegMaxSlots) return false;
     const int64_t N = (int64_t)p.n_tiles[3] * p.n_chunks[3];
     const int64_t Ge = std::min<int64_t>(p.G, N);
-    p.max_dn_items = (int)((N + Ge - 1) / Ge);
+    const int64_t No = (int64_t)p.n_tiles[1] * p.n_chunks[1], Geo = std::min<int64_t>(p.G, No);
+    p.max_items = (int)std::max((N + Ge - 1) / Ge, (No + Geo - 1) / Geo);
     for (int64_t t = 0; t < p.n_tiles[3]; ++t) {
         const int64_t a = ((t * p.n_chunks[3] + 1) * Ge - 1) / N, b = (((t + 1) * p.n_chunks[3]) * Ge - 1) / N;
         if (b - a + 1 > kSegMaxSlots) return false;
@@ -955,7 +1172,7 @@ bool seg_plan(const DevModel& m, int n_sm, SegPlan& p) {
     const int np_max = (m.max_ctx + m.page_size - 1) / m.page_size;
     p.max_pps = std::max(1, (np_max + cap - 1) / cap);
     const size_t floats = (size_t)((std::max(m.d, m.A * m.D) + 3) & ~3) + ((m.d + 3) & ~3) +
-                          (size_t)p.max_dn_items * kColsPerChunk + 2 * kCW * 32 + (size_t)grp * m.D + 2 * (size_t)m.D +
+                          (size_t)p.max_items * (kColsPerChunk + 32) + (size_t)m.D + (size_t)m.d + 2 * kCW * 32 + (size_t)grp * m.D + 2 * (size_t)m.D +
                           (size_t)grp * p.max_pps * m.page_size + 2 * (size_t)grp + (size_t)m.A * (kSegMaxSplits + 1);
     const size_t fixed = floats * 4 + (size_t)p.n_tiles[3] + 256;
     const size_t budget = 227 * 1024;

@@ -66,7 +66,7 @@ def forced(o: dict) -> int:
 
 
 def teacher_forced(shape, model, n: int, taus, *, prompt=None, capture: bool = True, graphs: bool = True,
-                   pdl: bool = True, persistent: bool = False, page_perm=None, page_size: int = 64):
+                   pdl: bool = True, persistent: bool = True, page_perm=None, page_size: int = 64):
     """Run the oracle free and the GPU engine teacher-forced on the oracle's
     input tokens and exit decisions.  Returns (first_o, first_g, records,
     oracle, engine)."""
@@ -79,8 +79,7 @@ def teacher_forced(shape, model, n: int, taus, *, prompt=None, capture: bool = T
     eng = Engine(shape, model, max_ctx=max_ctx, page_size=page_size)
     eng.set_option(OPT_GRAPHS, graphs)
     eng.set_option(OPT_PDL, pdl)
-    if persistent:
-        eng.set_option(OPT_PERSISTENT, 1)
+    eng.set_option(OPT_PERSISTENT, 1 if persistent else 0)
     eng.set_option(OPT_DEBUG_LOGITS, capture)
     if page_perm is not None:
         eng.set_page_table(page_perm)

@@ -24,9 +24,10 @@ def tiny_model():
 
 
 @pytest.mark.parametrize("tau", [0.5, 0.0, 1.01])
-def test_tiny_teacher_forced(tiny_model, tau):
+@pytest.mark.parametrize("persistent", [True, False])
+def test_tiny_teacher_forced(tiny_model, tau, persistent):
     n = TINY.new_tokens
-    fo, fg, recs, orc, eng = teacher_forced(TINY, tiny_model, n, [tau])
+    fo, fg, recs, orc, eng = teacher_forced(TINY, tiny_model, n, [tau], persistent=persistent)
     assert fo == fg
     excluded = check_records(recs, [tau])
     assert excluded <= n // 8

@@ -1,6 +1,7 @@
-"""The persistent layer-segment kernel (EE_OPT_PERSISTENT) against the CPU
-oracle under teacher forcing, and against the five-launch path (needs a
-GB300).  Same parity rules as test_gpu_parity."""
+"""The persistent layer-segment kernel (EE_OPT_PERSISTENT, the default) against
+the CPU oracle under teacher forcing with small pages and other shapes, and
+against the five-launch path (needs a GB300).  Same parity rules as
+test_gpu_parity."""
 import numpy as np
 import pytest
 
