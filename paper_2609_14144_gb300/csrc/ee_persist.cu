@@ -874,49 +874,69 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
                     const uint32_t kb = saddr(cs.acquire()) + lane * dpl * 2;
                     const int base = pg * m.page_size + q * rpc;
                     const int nr = min(rpc, p1 - base);
-#pragma unroll 2
-                    for (int r = w; r < nr; r += kCW) {
-                        const int ps = base + r;
-                        float kd[4];
-                        if (dpl == 4) {
-                            const uint2 v = lds64(kb + r * m.D * 2);
-                            kd[0] = bflo(v.x);
-                            kd[1] = bfhi(v.x);
-                            kd[2] = bflo(v.y);
-                            kd[3] = bfhi(v.y);
-                        } else {
-                            const uint32_t v = lds32(kb + r * m.D * 2);
-                            kd[0] = bflo(v);
-                            kd[1] = bfhi(v);
-                            kd[2] = kd[3] = 0.f;
-                        }
+                    // two positions per step (r and r + kCW), their reductions interleaved
+                    for (int r = w; r < nr; r += 2 * kCW) {
+                        const int rb2 = r + kCW;
+                        const bool two = rb2 < nr;
+                        float kd[2][4];
 #pragma unroll
-                        for (int k = 0; k < 4; ++k) kd[k] = ps == pos ? kvt[k] : kd[k];
-                        float dd[kSegMaxGroup];
+                        for (int e = 0; e < 2; ++e) {
+                            const int rr = e == 0 ? r : (two ? rb2 : r);
+                            if (dpl == 4) {
+                                const uint2 v = lds64(kb + rr * m.D * 2);
+                                kd[e][0] = bflo(v.x);
+                                kd[e][1] = bfhi(v.x);
+                                kd[e][2] = bflo(v.y);
+                                kd[e][3] = bfhi(v.y);
+                            } else {
+                                const uint32_t v = lds32(kb + rr * m.D * 2);
+                                kd[e][0] = bflo(v);
+                                kd[e][1] = bfhi(v);
+                                kd[e][2] = kd[e][3] = 0.f;
+                            }
+                            const bool own = base + rr == pos;
 #pragma unroll
-                        for (int hh = 0; hh < kSegMaxGroup; ++hh) {
-                            float d = qr[hh][0] * kd[0];
-                            d = fmaf(qr[hh][1], kd[1], d);
-                            d = fmaf(qr[hh][2], kd[2], d);
-                            d = fmaf(qr[hh][3], kd[3], d);
-                            dd[hh] = d;
+                            for (int k = 0; k < 4; ++k) kd[e][k] = own ? kvt[k] : kd[e][k];
                         }
+                        float dd[2][kSegMaxGroup];
+#pragma unroll
+                        for (int e = 0; e < 2; ++e)
+#pragma unroll
+                            for (int hh = 0; hh < kSegMaxGroup; ++hh) {
+                                float d = qr[hh][0] * kd[e][0];
+                                d = fmaf(qr[hh][1], kd[e][1], d);
+                                d = fmaf(qr[hh][2], kd[e][2], d);
+                                d = fmaf(qr[hh][3], kd[e][3], d);
+                                dd[e][hh] = d;
+                            }
                         // reduce-scatter over the warp: lane bits 4, 3, 2 pick the head
                         const bool b16 = lane & 16, b8 = lane & 8, b4 = lane & 4;
-                        float a4[4], a2[2];
+                        float a4[2][4], a2[2][2], a1[2];
 #pragma unroll
-                        for (int k = 0; k < 4; ++k)
-                            a4[k] = (b16 ? dd[k + 4] : dd[k]) +
-                                    __shfl_xor_sync(0xffffffffu, b16 ? dd[k] : dd[k + 4], 16);
+                        for (int e = 0; e < 2; ++e)
 #pragma unroll
-                        for (int k = 0; k < 2; ++k)
-                            a2[k] = (b8 ? a4[k + 2] : a4[k]) +
-                                    __shfl_xor_sync(0xffffffffu, b8 ? a4[k] : a4[k + 2], 8);
-                        float a1 = (b4 ? a2[1] : a2[0]) + __shfl_xor_sync(0xffffffffu, b4 ? a2[0] : a2[1], 4);
-                        a1 += __shfl_xor_sync(0xffffffffu, a1, 2);
-                        a1 += __shfl_xor_sync(0xffffffffu, a1, 1);
+                            for (int k = 0; k < 4; ++k)
+                                a4[e][k] = (b16 ? dd[e][k + 4] : dd[e][k]) +
+                                           __shfl_xor_sync(0xffffffffu, b16 ? dd[e][k] : dd[e][k + 4], 16);
+#pragma unroll
+                        for (int e = 0; e < 2; ++e)
+#pragma unroll
+                            for (int k = 0; k < 2; ++k)
+                                a2[e][k] = (b8 ? a4[e][k + 2] : a4[e][k]) +
+                                           __shfl_xor_sync(0xffffffffu, b8 ? a4[e][k] : a4[e][k + 2], 8);
+#pragma unroll
+                        for (int e = 0; e < 2; ++e)
+                            a1[e] = (b4 ? a2[e][1] : a2[e][0]) +
+                                    __shfl_xor_sync(0xffffffffu, b4 ? a2[e][0] : a2[e][1], 4);
+#pragma unroll
+                        for (int e = 0; e < 2; ++e) a1[e] += __shfl_xor_sync(0xffffffffu, a1[e], 2);
+#pragma unroll
+                        for (int e = 0; e < 2; ++e) a1[e] += __shfl_xor_sync(0xffffffffu, a1[e], 1);
                         const int hd = (b16 ? 4 : 0) + (b8 ? 2 : 0) + (b4 ? 1 : 0);
-                        if ((lane & 3) == 0 && hd < grp) s.sc[hd * spc + (ps - p0)] = a1;
+                        if ((lane & 3) == 0 && hd < grp) {
+                            s.sc[hd * spc + (base + r - p0)] = a1[0];
+                            if (two) s.sc[hd * spc + (base + rb2 - p0)] = a1[1];
+                        }
                     }
                     cs.release();
                 }
@@ -944,6 +964,7 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
             const int hw = w % grp, part = w / grp;
             const bool pv = w < grp * nsp;
             float oacc[4] = {0.f, 0.f, 0.f, 0.f}, obcc[4] = {0.f, 0.f, 0.f, 0.f};
+            float occc[4] = {0.f, 0.f, 0.f, 0.f}, odcc[4] = {0.f, 0.f, 0.f, 0.f};
             for (int pg = pg0; pg < pg1; ++pg)
                 for (int q = 0; q < cpp; ++q) {
                     const uint32_t vb = saddr(cs.acquire()) + lane * dpl * 2;
@@ -951,39 +972,41 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
                     const int nr = min(rpc, p1 - base);
                     if (pv && cs.ok) {
                         const uint32_t pw = saddr(s.sc + hw * spc + (base - p0));
-                        // two positions per step into two accumulator sets
-                        for (int r = part; r < nr; r += 2 * nsp) {
-                            const int r2 = r + nsp;
-                            const bool two = r2 < nr;
-                            const float pa = ldsf(pw + 4 * r), pb = two ? ldsf(pw + 4 * r2) : 0.f;
-                            float va[4], vb2[4];
-                            if (dpl == 4) {
-                                const uint2 ua = lds64(vb + r * m.D * 2);
-                                const uint2 ub = lds64(vb + (two ? r2 : r) * m.D * 2);
-                                va[0] = bflo(ua.x), va[1] = bfhi(ua.x), va[2] = bflo(ua.y), va[3] = bfhi(ua.y);
-                                vb2[0] = bflo(ub.x), vb2[1] = bfhi(ub.x), vb2[2] = bflo(ub.y), vb2[3] = bfhi(ub.y);
-                            } else {
-                                const uint32_t ua = lds32(vb + r * m.D * 2);
-                                const uint32_t ub = lds32(vb + (two ? r2 : r) * m.D * 2);
-                                va[0] = bflo(ua), va[1] = bfhi(ua), va[2] = va[3] = 0.f;
-                                vb2[0] = bflo(ub), vb2[1] = bfhi(ub), vb2[2] = vb2[3] = 0.f;
+                        // four positions per step into four accumulator sets; a
+                        // slot past the chunk gets probability 0 and value 0 (a
+                        // select: the stand-in row may hold anything)
+                        for (int r = part; r < nr; r += 4 * nsp) {
+                            float pq[4], vq[4][4];
+#pragma unroll
+                            for (int e = 0; e < 4; ++e) {
+                                const int re = r + e * nsp;
+                                const bool in = re < nr;
+                                const int rr = in ? re : r;
+                                pq[e] = in ? ldsf(pw + 4 * rr) : 0.f;
+                                if (dpl == 4) {
+                                    const uint2 u = lds64(vb + rr * m.D * 2);
+                                    vq[e][0] = bflo(u.x), vq[e][1] = bfhi(u.x), vq[e][2] = bflo(u.y), vq[e][3] = bfhi(u.y);
+                                } else {
+                                    const uint32_t u = lds32(vb + rr * m.D * 2);
+                                    vq[e][0] = bflo(u), vq[e][1] = bfhi(u), vq[e][2] = vq[e][3] = 0.f;
+                                }
+#pragma unroll
+                                for (int k = 0; k < 4; ++k)
+                                    vq[e][k] = !in ? 0.f : (base + re == pos ? vvt[k] : vq[e][k]);
                             }
-                            // the stale cache row of the step's own position (and the
-                            // stand-in row when there is no second position) is
-                            // selected away, never multiplied by zero: it may hold
-                            // anything, NaN included
 #pragma unroll
                             for (int k = 0; k < 4; ++k) {
-                                oacc[k] = fmaf(pa, base + r == pos ? vvt[k] : va[k], oacc[k]);
-                                const float v2 = !two ? 0.f : (base + r2 == pos ? vvt[k] : vb2[k]);
-                                obcc[k] = fmaf(pb, v2, obcc[k]);
+                                oacc[k] = fmaf(pq[0], vq[0][k], oacc[k]);
+                                obcc[k] = fmaf(pq[1], vq[1][k], obcc[k]);
+                                occc[k] = fmaf(pq[2], vq[2][k], occc[k]);
+                                odcc[k] = fmaf(pq[3], vq[3][k], odcc[k]);
                             }
                         }
                     }
                     cs.release();
                 }
 #pragma unroll
-            for (int k = 0; k < 4; ++k) oacc[k] += obcc[k];
+            for (int k = 0; k < 4; ++k) oacc[k] = (oacc[k] + obcc[k]) + (occc[k] + odcc[k]);
             if (pv && part > 0) {
                 float* dst = s.xs + ((part - 1) * grp + hw) * m.D + lane * dpl;
 #pragma unroll
