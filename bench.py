@@ -213,28 +213,33 @@ def kernel_launches_per_token(L: int, k: int, exit_rate: float, persistent: bool
     return out
 
 
-def ncu_traffic(kernel: str, shape_name: str) -> float | None:
+def ncu_traffic(kernel: str, shape_name: str, attended: int | None = None, dims=None) -> float | None:
     """Per-launch DRAM bytes from a committed ncu summary, if its recorded
-    kernel-source hash still matches the current source."""
+    kernel-source hash still matches the current source.  For the layer
+    kernel, the capture's cache reads are moved to `attended` positions (the
+    weights do not depend on the position)."""
     path = os.path.join(ROOT, "profiles", f"ncu_{kernel}_{shape_name.replace('.', 'p')}.md")
     if not os.path.exists(path):
         return None
-    src = open(os.path.join(ROOT, "paper_2609_14144_gb300", "csrc", "ee_kernels.cu"), "rb").read()
-    sha = hashlib.sha256(src).hexdigest()[:16]
     vals = {}
     for line in open(path):
         if ":" in line and line.strip().startswith("- "):
             k, v = line.strip()[2:].split(":", 1)
             vals[k.strip()] = v.strip()
-    if vals.get("kernel_source_sha256") != sha:
+    src_name = vals.get("kernel_source", "ee_kernels.cu")
+    src = open(os.path.join(ROOT, "paper_2609_14144_gb300", "csrc", src_name), "rb").read()
+    if vals.get("kernel_source_sha256") != hashlib.sha256(src).hexdigest()[:16]:
         return None
     try:
-        return float(vals["dram_bytes_per_launch"])
+        traffic = float(vals["dram_bytes_per_launch"])
+        if attended is not None and dims is not None and "attended_positions" in vals:
+            layers = int(vals.get("layers_per_launch", "1"))
+            traffic += layers * 4 * dims.K * dims.D * (attended - int(vals["attended_positions"]))
+        return traffic
     except Exception:
         return None
 
 
-# --------------------------------------------------------------------- CPU oracle
 def oracle_sample(shape, model, seconds: float, prompt_len: int = 16, rate: float = HEADLINE_RATE,
                   min_steps: int = 4) -> dict:
     """Time the CPU oracle's gated decode on a bounded sample of the workload:
@@ -481,7 +486,8 @@ def run_ours(args, rank: int, world: int, local: int):
     ach = kb[dom] / (kms[dom] / 1e3) / 1e9
     roofline = {"bound": "hbm", "kernel": dom, "achieved": ach, "peak": peak["hbm_gbs"], "unit": "GB/s",
                 "frac": ach / peak["hbm_gbs"], "peak_source": peak["source"],
-                "traffic": ncu_traffic(dom, WORKLOAD), "bytes_per_launch": kb[dom], "ms_per_launch": kms[dom],
+                "traffic": ncu_traffic(dom, WORKLOAD, T_prof, run.dims), "bytes_per_launch": kb[dom],
+                "ms_per_launch": kms[dom],
                 "kernels": {k: {"ms": kms[k], "GBps": kb[k] / (kms[k] / 1e3) / 1e9 if kms[k] > 0 else None,
                                 "share": share[k] / sum(share.values())} for k in kms}}
     step_roof = {"achieved": head["gbs"], "peak": peak["hbm_gbs"], "unit": "GB/s",
