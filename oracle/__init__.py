@@ -24,6 +24,8 @@ _lib = None
 MAX_READOUTS = 8
 FORCE_FREE = 0
 FORCE_FULL = 1
+# Section 10 confidence signals the gate may compare with tau
+CONF_PMAX, CONF_MARGIN, CONF_NEGENT = 0, 1, 2
 
 
 def FORCE_EXIT_AT(r: int) -> int:
@@ -61,7 +63,7 @@ class Weights(ctypes.Structure):
 
 class Conf(ctypes.Structure):
     _fields_ = [("p1", ctypes.c_float), ("p2", ctypes.c_float), ("gap", ctypes.c_float),
-                ("max_logit", ctypes.c_float), ("argmax", ctypes.c_int32)]
+                ("max_logit", ctypes.c_float), ("argmax", ctypes.c_int32), ("neg_entropy", ctypes.c_float)]
 
 
 class StepResult(ctypes.Structure):
@@ -108,6 +110,7 @@ def _load():
             lib.orc_free.argtypes = [_P]
             lib.orc_add_readout.argtypes = [_P, ctypes.c_int, _P, _P]
             lib.orc_reset.argtypes = [_P]
+            lib.orc_set_confidence.argtypes = [_P, ctypes.c_int]
             lib.orc_prefill.argtypes = [_P, _P, ctypes.c_int, ctypes.POINTER(ctypes.c_int32),
                                         ctypes.POINTER(Capture)]
             lib.orc_decode_step.argtypes = [_P, ctypes.c_int32, _P, ctypes.c_int, ctypes.POINTER(StepResult),
@@ -175,7 +178,8 @@ def confidence(logits) -> dict:
     l = _f32(logits)
     c = Conf()
     _load().orc_op_confidence(l.ctypes.data, l.size, ctypes.byref(c))
-    return {"p1": c.p1, "p2": c.p2, "gap": c.gap, "max_logit": c.max_logit, "argmax": c.argmax}
+    return {"p1": c.p1, "p2": c.p2, "gap": c.gap, "max_logit": c.max_logit, "argmax": c.argmax,
+            "neg_entropy": c.neg_entropy}
 
 
 # ---------------------------------------------------------------- model
@@ -247,6 +251,11 @@ class Oracle:
 
     def reset(self):
         self.lib.orc_reset(self.ptr)
+
+    def set_confidence(self, kind: int):
+        """Gate signal: CONF_PMAX (default), CONF_MARGIN or CONF_NEGENT (Section 10)."""
+        if self.lib.orc_set_confidence(self.ptr, int(kind)) != 0:
+            raise ValueError("oracle: bad confidence kind")
 
     @property
     def pos(self) -> int:

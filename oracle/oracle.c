@@ -20,6 +20,10 @@
  *     exit-layer state through those layers' key and value matrices.
  *   - Section 4, step three: more than one exit point is possible.
  *   - Appendix B: greedy decoding (the emitted token is the top-scoring one).
+ *   - Section 10: the probability of the best token, the margin between the
+ *     best and second-best probabilities, and the negative entropy of the
+ *     readout's distribution are interchangeable softmax confidences; the
+ *     gate can use any of them (orc_set_confidence).
  *   - Appendix C: the layer is four attention projections with grouped-query
  *     attention (A query heads, K key-value heads of size D) and a gated
  *     feed-forward block of three matrices of width F.
@@ -56,6 +60,9 @@
 #include <string.h>
 
 #define ORC_MAX_READOUTS 8
+#define ORC_CONF_PMAX 0    /* p1: probability of the best token           */
+#define ORC_CONF_MARGIN 1  /* p1 - p2: margin to the second-best token     */
+#define ORC_CONF_NEGENT 2  /* sum_v p_v log p_v: negative entropy (<= 0)   */
 #define ORC_FORCE_FREE 0
 #define ORC_FORCE_FULL 1
 #define ORC_FORCE_EXIT_AT(r) (2 + (r))
@@ -91,6 +98,7 @@ typedef struct {
     float gap;       /* p1 - p2 */
     float max_logit;
     int32_t argmax;  /* lowest index attaining the maximum */
+    float neg_entropy; /* sum_v p_v log p_v */
 } orc_conf;
 
 typedef struct {
@@ -124,6 +132,7 @@ typedef struct {
     float* vc;
     int8_t* kv_src;  /* [L][max_ctx]: 0 empty, 1 computed by the layer, 2 filled */
     int pos;
+    int conf_kind; /* ORC_CONF_*: the signal the gate compares with tau */
     int64_t steps, full_steps, exits[ORC_MAX_READOUTS];
     float *h, *u, *q, *kk, *vv, *o, *g, *up, *a, *y, *z, *logits, *tmp;
 } orc_model;
@@ -256,6 +265,28 @@ void orc_op_confidence(const float* l, int64_t V, orc_conf* out) {
     out->gap = out->p1 - out->p2;
     out->max_logit = mx;
     out->argmax = (int32_t)arg;
+    /* negative entropy straight from its definition, p log p with 0 log 0 = 0 */
+    double ne = 0.0;
+    for (int64_t v = 0; v < V; ++v) {
+        const double p = exp((double)l[v] - (double)mx) / sum;
+        if (p > 0.0) ne += p * log(p);
+    }
+    out->neg_entropy = (float)ne;
+}
+
+/* The gate's signal under the model's confidence kind (Section 10). */
+static float conf_signal(const orc_model* m, const orc_conf* cf) {
+    switch (m->conf_kind) {
+        case ORC_CONF_MARGIN: return cf->gap;
+        case ORC_CONF_NEGENT: return cf->neg_entropy;
+        default: return cf->p1;
+    }
+}
+
+int orc_set_confidence(orc_model* m, int kind) {
+    if (!m || kind < ORC_CONF_PMAX || kind > ORC_CONF_NEGENT) return -1;
+    m->conf_kind = kind;
+    return 0;
 }
 
 /* ------------------------------------------------------------------ */
@@ -532,10 +563,10 @@ int orc_decode_step(orc_model* m, int32_t in_tok, const float* taus, int force, 
             readout(m, r, m->h, m->y, m->logits);
             orc_conf cf;
             orc_op_confidence(m->logits, V, &cf);
-            res->confidence[r] = cf.p1;
+            res->confidence[r] = conf_signal(m, &cf);
             res->gap[r] = cf.gap;
             res->readout_token[r] = cf.argmax;
-            res->gate_pass[r] = cf.p1 > taus[r];
+            res->gate_pass[r] = res->confidence[r] > taus[r];
             res->n_evaluated = r + 1;
             if (cap && cap->h_readout) memcpy(cap->h_readout + (size_t)r * d, m->h, sizeof(float) * d);
             if (cap && cap->y_readout) memcpy(cap->y_readout + (size_t)r * d, m->y, sizeof(float) * d);
@@ -559,7 +590,7 @@ int orc_decode_step(orc_model* m, int32_t in_tok, const float* taus, int force, 
         orc_op_confidence(m->logits, V, &cf);
         res->token = cf.argmax;
         res->full_token = cf.argmax;
-        res->full_confidence = cf.p1;
+        res->full_confidence = conf_signal(m, &cf);
         res->full_gap = cf.gap;
         if (cap && cap->h_final) memcpy(cap->h_final, m->h, sizeof(float) * d);
         if (cap && cap->final_logits) memcpy(cap->final_logits, m->logits, sizeof(float) * V);

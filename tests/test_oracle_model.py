@@ -191,6 +191,39 @@ def test_gate_is_strict():
         assert s["confidence"][0] == p and s["gate_pass"][0] == expect
 
 
+def test_gate_with_margin_and_negative_entropy():
+    """Section 10: the gate may compare the margin p1 - p2 or the negative
+    entropy with tau instead of p1; the recorded confidence is that signal
+    of the readout's distribution, and the gate is still strict."""
+    model = synth.make_model(TINY)
+    for kind, key in ((oracle.CONF_MARGIN, "gap"), (oracle.CONF_NEGENT, "neg_entropy")):
+        o = oracle.Oracle(TINY, model)
+        o.set_confidence(kind)
+        tok = o.prefill(synth.prompt(TINY))
+        sigs = []
+        for _ in range(12):
+            s = o.decode_step(tok, [0.5], oracle.FORCE_FULL, capture=True)
+            c = oracle.confidence(s["capture"]["readout_logits"][0])
+            assert s["confidence"][0] == np.float32(c[key])
+            assert s["gate_pass"][0] == int(np.float32(c[key]) > np.float32(0.5))
+            sigs.append(s["confidence"][0])
+            tok = s["token"]
+        sigs = np.array(sigs, np.float32)
+        if kind == oracle.CONF_MARGIN:
+            assert np.all((0.0 <= sigs) & (sigs < 1.0))
+        else:
+            assert np.all((-math.log(TINY.vocab) - 1e-4 <= sigs) & (sigs <= 0.0))
+    # always / never exit at thresholds below and above the signal's range
+    for kind, lo, hi in ((oracle.CONF_MARGIN, -0.5, 1.0), (oracle.CONF_NEGENT, -math.log(TINY.vocab) - 1.0, 0.0)):
+        for tau, expect in ((lo, TINY.new_tokens), (hi, 0)):
+            o = oracle.Oracle(TINY, model)
+            o.set_confidence(kind)
+            o.generate(synth.prompt(TINY), TINY.new_tokens, [tau])
+            assert o.stats()["exits"] == [expect]
+    with pytest.raises(ValueError):
+        oracle.Oracle(TINY, model).set_confidence(3)
+
+
 # ------------------------------------------------------------- structure
 def _trace_step(shape, model, force=oracle.FORCE_FULL, taus=(0.5,)):
     o = oracle.Oracle(shape, model)

@@ -6,6 +6,7 @@ import math
 import numpy as np
 import pytest
 import scipy.special
+import scipy.stats
 import torch
 
 import oracle
@@ -187,3 +188,38 @@ def test_confidence_special_cases():
     c = oracle.confidence(np.array([1.5, 0.25], np.float32))
     assert c["p1"] == pytest.approx(1 / (1 + math.exp(-1.25)), rel=1e-7)
     assert c["gap"] == pytest.approx(c["p1"] - (1 - c["p1"]), rel=1e-6)
+
+
+def test_negative_entropy_and_margin_against_scipy():
+    """Section 10's other two signals: margin p1 - p2 and negative entropy
+    sum p log p, against scipy's entropy and a sorted softmax."""
+    for V in (2, 17, 4096, 151936):
+        l = (RNG.standard_normal(V) * 5).astype(np.float32)
+        c = oracle.confidence(l)
+        p = scipy.special.softmax(l.astype(np.float64))
+        assert c["neg_entropy"] == pytest.approx(-scipy.stats.entropy(p), rel=1e-6, abs=1e-7)
+        top = np.sort(p)[-2:]
+        assert c["gap"] == pytest.approx(top[1] - top[0], rel=1e-5, abs=1e-7)
+
+
+def test_negative_entropy_and_margin_closed_forms():
+    V = 1000
+    c = oracle.confidence(np.zeros(V, np.float32))  # uniform: -log V, no margin
+    assert c["neg_entropy"] == pytest.approx(-math.log(V), rel=1e-6) and c["gap"] == 0.0
+    # one logit a above V - 1 equal ones: p1 = e^a / (e^a + V - 1), the rest q
+    a = 4.0
+    l = np.zeros(V, np.float32)
+    l[7] = a
+    c = oracle.confidence(l)
+    z = math.exp(a) + V - 1
+    p1, q = math.exp(a) / z, 1.0 / z
+    assert c["neg_entropy"] == pytest.approx(p1 * math.log(p1) + (V - 1) * q * math.log(q), rel=1e-6)
+    assert c["gap"] == pytest.approx(p1 - q, rel=1e-6)
+    # near one-hot: negative entropy tends to 0 from below
+    l[7] = 60.0
+    c = oracle.confidence(l)
+    assert -1e-20 < -c["neg_entropy"] < 1e-20 + 1e-12 and c["neg_entropy"] <= 0.0
+    # two logits: -H = p log p + (1 - p) log(1 - p)
+    c = oracle.confidence(np.array([0.5, -0.75], np.float32))
+    p = 1 / (1 + math.exp(-1.25))
+    assert c["neg_entropy"] == pytest.approx(p * math.log(p) + (1 - p) * math.log(1 - p), rel=1e-6)
