@@ -199,6 +199,12 @@ int ee_position(ee_ctx* ctx, int32_t* pos);
                                  0: direct launches, branch decided on the host */
 #define EE_OPT_PDL 2          /* 1 (default): programmatic dependent launch    */
 #define EE_OPT_DEBUG_LOGITS 3 /* 1: keep each step's readout and final logits  */
+#define EE_OPT_CONFIDENCE 5   /* the signal each gate compares with its tau: */
+#define EE_CONF_PMAX 0        /*   top-1 probability p1 (Section 2; default)   */
+#define EE_CONF_MARGIN 1      /*   p1 - p2, the margin to the second-best token */
+#define EE_CONF_NEGENT 2      /*   sum_v p_v log p_v, the negative entropy (<= 0)
+                                 (Section 10: the three are interchangeable);
+                                 the step result's confidence reports it    */
 #define EE_OPT_PERSISTENT 4   /* 1 (default where supported): each run of layers
                                  between readouts is one persistent launch, one
                                  CTA per SM streaming weights through a shared-
@@ -290,6 +296,13 @@ int ee_vocab_scratch_bytes(int vocab, int d_model, size_t* bytes);
 int ee_vocab_confidence(const float* x, const uint16_t* gain, const uint16_t* U, int vocab, int d_model,
                         float eps, void* scratch, size_t scratch_bytes, int32_t* out_token, float* out_p,
                         float* logits, void* stream);
+/* The same pass returning all three confidence signals of Section 10:
+ *   out_signals device float[3] = { p1, p1 - p2, sum_v p_v log p_v }
+ * where p2 is the second-best probability (p1 again if the maximum is tied).
+ * Other arguments and errors as for ee_vocab_confidence. */
+int ee_vocab_signals(const float* x, const uint16_t* gain, const uint16_t* U, int vocab, int d_model,
+                     float eps, void* scratch, size_t scratch_bytes, int32_t* out_token, float* out_signals,
+                     float* logits, void* stream);
 
 #ifdef __cplusplus
 }

@@ -11,11 +11,12 @@ import ctypes
 import numpy as np
 
 from . import _lib
-from ._lib import (DEVICE, FORCE_FULL, FREE, HOST, MAX_READOUTS, OPT_DEBUG_LOGITS, OPT_GRAPHS, OPT_PDL,
-                   OPT_PERSISTENT, EEError, FORCE_EXIT_AT, check)
+from ._lib import (CONF_MARGIN, CONF_NEGENT, CONF_PMAX, DEVICE, FORCE_FULL, FREE, HOST, MAX_READOUTS,
+                   OPT_CONFIDENCE, OPT_DEBUG_LOGITS, OPT_GRAPHS, OPT_PDL, OPT_PERSISTENT, EEError, FORCE_EXIT_AT,
+                   check)
 
 __all__ = ["Engine", "EEError", "FREE", "FORCE_FULL", "FORCE_EXIT_AT", "HOST", "DEVICE", "attention_decode",
-           "vocab_confidence", "library_path"]
+           "vocab_confidence", "vocab_signals", "library_path"]
 
 
 def library_path() -> str:
@@ -256,3 +257,23 @@ def vocab_confidence(x, gain, U, eps: float, logits=None, scratch=None, stream=N
                                   scratch.numel(), tok.data_ptr(), p.data_ptr(),
                                   None if logits is None else logits.data_ptr(), s.cuda_stream))
     return tok, p
+
+
+def vocab_signals(x, gain, U, eps: float, logits=None, scratch=None, stream=None):
+    """The same pass returning (token, signals): signals is a float32 tensor
+    [3] = (top-1 probability, margin to the second-best, negative entropy)."""
+    import torch
+
+    lib = _lib.load()
+    V, d = U.shape
+    nb = ctypes.c_size_t(0)
+    check(lib.ee_vocab_scratch_bytes(V, d, ctypes.byref(nb)))
+    if scratch is None:
+        scratch = torch.empty(nb.value, dtype=torch.uint8, device=x.device)
+    tok = torch.empty(1, dtype=torch.int32, device=x.device)
+    sig = torch.empty(3, dtype=torch.float32, device=x.device)
+    s = stream if stream is not None else torch.cuda.current_stream(x.device)
+    check(lib.ee_vocab_signals(x.data_ptr(), gain.data_ptr(), U.data_ptr(), V, d, float(eps), scratch.data_ptr(),
+                               scratch.numel(), tok.data_ptr(), sig.data_ptr(),
+                               None if logits is None else logits.data_ptr(), s.cuda_stream))
+    return tok, sig

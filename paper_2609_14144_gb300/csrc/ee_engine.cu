@@ -146,7 +146,7 @@ Layout make_layout(const ee_model_config& c) {
     l.gemv_ticket = take(4 * (size_t)l.gemv_ticket_stride * L);
     l.attn_part = take(4 * (size_t)A * kAttnMaxSplits * (D + 2));
     l.attn_ticket = take(4 * (size_t)KH);
-    l.vocab_part = take(4 * (size_t)kMaxVocabCtas * 4);
+    l.vocab_part = take(4 * (size_t)kMaxVocabCtas * 8);
     l.vocab_ticket = take(4);
     // persistent layer kernel: down-projection partials, mid residual, counters
     {
@@ -217,6 +217,7 @@ struct ee_ctx {
     bool seg_ok = false, use_persistent = true;  // persistent layer kernel supported / chosen
     SegPlan seg{};
     int dbg = 0;
+    int conf_kind = EE_CONF_PMAX;  // signal the gates compare with tau
     cudaGraphExec_t g_step = nullptr, g_n = nullptr, g_prefill = nullptr;
     int grid_gemv = 0, grid_vocab = 0;
     int attn_cluster = 8;  // CTAs per key-value head in the attention kernel
@@ -560,6 +561,7 @@ CtlInputs base_inputs(const ee_ctx* c, const float* taus) {
     in.set_token = 0;
     in.n_steps = 1;
     in.dbg = c->dbg;
+    in.conf_kind = c->conf_kind;
     for (int r = 0; r < kMaxReadouts; ++r) in.tau[r] = (taus && r < c->n_readouts) ? taus[r] : 2.0f;
     return in;
 }
@@ -884,6 +886,10 @@ int ee_set_option(ee_ctx* c, int option, int value) {
         case EE_OPT_DEBUG_LOGITS:
             c->dbg = value != 0;
             return EE_OK;
+        case EE_OPT_CONFIDENCE:
+            if (value < EE_CONF_PMAX || value > EE_CONF_NEGENT) return fail(EE_EINVAL, "unknown confidence signal");
+            c->conf_kind = value;
+            return EE_OK;
         case EE_OPT_PERSISTENT:
             if (value && !c->seg_ok) return fail(EE_EINVAL, "the persistent layer kernel does not support this shape");
             if (c->use_persistent != (value != 0)) drop_graphs(c);
@@ -1199,16 +1205,17 @@ int ee_attention_decode(const float* q, const uint16_t* k_pages, const uint16_t*
 
 int ee_vocab_scratch_bytes(int vocab, int d_model, size_t* bytes) {
     if (!bytes || vocab <= 1 || d_model < 256 || d_model % 8) return fail(EE_EINVAL, "bad shape");
-    *bytes = align_up(4 * (size_t)kMaxVocabCtas * 4) + align_up(4);
+    *bytes = align_up(4 * (size_t)kMaxVocabCtas * 8) + align_up(4);
     return EE_OK;
 }
 
-int ee_vocab_confidence(const float* x, const uint16_t* gain, const uint16_t* U, int vocab, int d_model, float eps,
-                        void* scratch, size_t scratch_bytes, int32_t* out_token, float* out_p, float* logits,
-                        void* stream) {
+namespace {
+int vocab_standalone(const float* x, const uint16_t* gain, const uint16_t* U, int vocab, int d_model, float eps,
+                     void* scratch, size_t scratch_bytes, int32_t* out_token, float* out_p, float* out_sig,
+                     float* logits, void* stream) {
     size_t need = 0;
     EE_TRY(ee_vocab_scratch_bytes(vocab, d_model, &need));
-    if (!x || !gain || !U || !scratch || !out_token || !out_p) return fail(EE_EINVAL, "NULL argument");
+    if (!x || !gain || !U || !scratch || !out_token || (!out_p && !out_sig)) return fail(EE_EINVAL, "NULL argument");
     if (scratch_bytes < need) return fail(EE_ENOMEM, "scratch too small");
     int dev = 0, nsm = 0;
     EE_CK(cudaGetDevice(&dev));
@@ -1227,13 +1234,31 @@ int ee_vocab_confidence(const float* x, const uint16_t* gain, const uint16_t* U,
     v.logits = logits;
     v.logits_if_dbg = 0;
     v.part = (float*)sc;
-    v.ticket = (int*)(sc + align_up(4 * (size_t)kMaxVocabCtas * 4));
+    v.ticket = (int*)(sc + align_up(4 * (size_t)kMaxVocabCtas * 8));
     v.mode = 0;
     v.out_token = out_token;
     v.out_p = out_p;
+    v.out_sig = out_sig;
     EE_CK(cudaMemsetAsync(v.ticket, 0, 4, s));
     EE_CK(launch_vocab(v, std::min(nsm, kMaxVocabCtas), false, s));
     return EE_OK;
+}
+}  // namespace
+
+int ee_vocab_confidence(const float* x, const uint16_t* gain, const uint16_t* U, int vocab, int d_model, float eps,
+                        void* scratch, size_t scratch_bytes, int32_t* out_token, float* out_p, float* logits,
+                        void* stream) {
+    if (!out_p) return fail(EE_EINVAL, "NULL argument");
+    return vocab_standalone(x, gain, U, vocab, d_model, eps, scratch, scratch_bytes, out_token, out_p, nullptr,
+                            logits, stream);
+}
+
+int ee_vocab_signals(const float* x, const uint16_t* gain, const uint16_t* U, int vocab, int d_model, float eps,
+                     void* scratch, size_t scratch_bytes, int32_t* out_token, float* out_signals, float* logits,
+                     void* stream) {
+    if (!out_signals) return fail(EE_EINVAL, "NULL argument");
+    return vocab_standalone(x, gain, U, vocab, d_model, eps, scratch, scratch_bytes, out_token, nullptr,
+                            out_signals, logits, stream);
 }
 
 }  // extern "C"

@@ -39,7 +39,8 @@ struct Ctl {
     int32_t prefill_n;    // prompt length of the running prefill
     int32_t prefill_i;    // prompt index of the running prefill
     int32_t max_ctx;
-    int32_t pad0, pad1;
+    int32_t conf_kind;    // EE_CONF_*: the signal the gates compare with tau
+    int32_t pad1;
     int32_t gate_pass[kMaxReadouts];
     int32_t readout_token[kMaxReadouts];
     float conf[kMaxReadouts];
@@ -89,7 +90,7 @@ struct DevModel {
     int64_t gemv_ticket_stride;   // counters per fill layer in gemv_ticket
     float* attn_part;             // [A][kAttnMaxSplits][D + 2]
     int* attn_ticket;             // [KH]
-    float* vocab_part;            // [grid][4]
+    float* vocab_part;            // [grid][8]
     int* vocab_ticket;            // [1]
     Ctl* ctl;
 };
@@ -125,13 +126,14 @@ struct VocabArgs {
     Ctl* ctl;
     int32_t* out_token;
     float* out_p;
+    float* out_sig;           // standalone: [3] p_max, margin, negative entropy (may be null)
     int has_cond;
     cudaGraphConditionalHandle cond;
 };
 
 // Per-call inputs of a graph launch.
 struct CtlInputs {
-    int set_token, in_tok, force, n_steps, dbg, prefill_n;
+    int set_token, in_tok, force, n_steps, dbg, prefill_n, conf_kind;
     float tau[kMaxReadouts];
     const int8_t* sched;
     int32_t* out_tokens;

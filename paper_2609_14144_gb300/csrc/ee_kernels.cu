@@ -533,54 +533,75 @@ struct EpiSwiGLU {
     }
 };
 
-// Merge (m2, s2, a2) into (m, s, a): max, rescaled sum, lowest index at the max.
-__device__ __forceinline__ void merge_stats(float& m, float& s, int& a, float m2, float s2, int a2) {
-    if (s2 == 0.f && m2 == -CUDART_INF_F) return;
-    if (s == 0.f && m == -CUDART_INF_F) {
-        m = m2;
-        s = s2;
-        a = a2;
-        return;
-    }
-    if (m2 > m) {
-        s = s * expf(m - m2) + s2;
-        m = m2;
-        a = a2;
-    } else if (m2 == m) {
-        s = s + s2;
-        a = a2 < a ? a2 : a;
-    } else {
-        s = s + s2 * expf(m2 - m);
-    }
-}
-
-// Warp-wide merge; lane 0 ends with the merge of all lanes in lane order.
-__device__ __forceinline__ void warp_merge_stats(float& m, float& s, int& a) {
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-        const float m2 = __shfl_down_sync(0xffffffffu, m, o);
-        const float s2 = __shfl_down_sync(0xffffffffu, s, o);
-        const int a2 = __shfl_down_sync(0xffffffffu, a, o);
-        if (((threadIdx.x & 31) & ((o << 1) - 1)) == 0) merge_stats(m, s, a, m2, s2, a2);
-    }
-}
-
-// Running (max, sum of exp, lowest argmax) of one lane's rows, plus the
-// logits themselves when requested.
-struct LaneStats {
-    float m, s;
+// Online softmax statistics of a set of logits (Section 2 confidence and
+// the Section 10 alternatives), all from one pass:
+//   m  = max l,  s = sum exp(l - m),  t = sum exp(l - m) (l - m),
+//   m2 = the second largest logit (m again if the maximum is tied),
+//   a  = lowest index attaining m.
+// Then p_max = 1/s, margin = (1 - exp(m2 - m))/s, negative entropy =
+// sum p log p = t/s - log s.
+struct SoftStats {
+    float m, s, t, m2;
     int a;
-    __device__ __forceinline__ LaneStats() : m(-INFINITY), s(0.f), a(0x7fffffff) {}
+    __device__ __forceinline__ SoftStats() : m(-INFINITY), s(0.f), t(0.f), m2(-INFINITY), a(0x7fffffff) {}
     __device__ __forceinline__ void add(float l, int row) {
-        if (l > m) {
-            s = s * expf(m - l) + 1.0f;
+        if (s == 0.f) {
+            m = l;
+            s = 1.f;
+            t = 0.f;
+            a = row;
+        } else if (l > m) {
+            const float dl = m - l, e = expf(dl);
+            t = e * (t + dl * s);
+            s = s * e + 1.0f;
+            m2 = m;
             m = l;
             a = row;
         } else {
-            s += expf(l - m);
+            const float dl = l - m, e = expf(dl);
+            s += e;
+            t = fmaf(e, dl, t);
+            if (l > m2) m2 = l;
         }
     }
+    // Merge another set (its indices all differ from this one's).
+    __device__ __forceinline__ void merge(const SoftStats& o) {
+        if (o.s == 0.f) return;
+        if (s == 0.f) {
+            *this = o;
+            return;
+        }
+        const float M = fmaxf(m, o.m);
+        const float ea = expf(m - M), eb = expf(o.m - M);
+        t = ea * (t + (m - M) * s) + eb * (o.t + (o.m - M) * o.s);
+        s = s * ea + o.s * eb;
+        m2 = fmaxf(fminf(m, o.m), fmaxf(m2, o.m2));
+        a = m > o.m ? a : (o.m > m ? o.a : min(a, o.a));
+        m = M;
+    }
 };
+
+__device__ __forceinline__ SoftStats shfl_down_stats(const SoftStats& x, int o) {
+    SoftStats y;
+    y.m = __shfl_down_sync(0xffffffffu, x.m, o);
+    y.s = __shfl_down_sync(0xffffffffu, x.s, o);
+    y.t = __shfl_down_sync(0xffffffffu, x.t, o);
+    y.m2 = __shfl_down_sync(0xffffffffu, x.m2, o);
+    y.a = __shfl_down_sync(0xffffffffu, x.a, o);
+    return y;
+}
+
+// Warp-wide merge; lane 0 ends with the merge of all lanes in lane order.
+__device__ __forceinline__ void warp_merge_stats(SoftStats& st) {
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const SoftStats y = shfl_down_stats(st, o);
+        if (((threadIdx.x & 31) & ((o << 1) - 1)) == 0) st.merge(y);
+    }
+}
+
+// Running statistics of one lane's rows.
+using LaneStats = SoftStats;
 
 __device__ __forceinline__ const uint16_t* layer_base(const DevModel& m, int j) {
     return m.layers + (int64_t)j * m.layer_stride;
@@ -817,30 +838,42 @@ __global__ void __launch_bounds__(kGemvThreads, 2) k_readout(DevModel m, int r) 
 }
 
 // After the vocabulary pass: merge the per-lane statistics of the CTA, then
-// (last CTA) of the grid, turn them into p = 1 / sum exp(l - max) and, for a
-// readout, the gate decision p > tau, which also selects the graph's branch.
+// (last CTA) of the grid; turn them into the confidence signals and, for a
+// readout, the gate decision signal > tau, which also selects the graph's
+// branch.  The signal is the top-1 probability (Section 2) or, by the
+// context's choice, the margin or the negative entropy (Section 10).
 __device__ __forceinline__ void vocab_finish(const VocabArgs& v, LaneStats st) {
-    __shared__ float sm_m[32], sm_s[32];
+    __shared__ float sm_m[32], sm_s[32], sm_t[32], sm_m2[32];
     __shared__ int sm_a[32];
     __shared__ int is_last;
     const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-    warp_merge_stats(st.m, st.s, st.a);
+    warp_merge_stats(st);
     if (lane == 0) {
         sm_m[w] = st.m;
         sm_s[w] = st.s;
+        sm_t[w] = st.t;
+        sm_m2[w] = st.m2;
         sm_a[w] = st.a;
     }
     __syncthreads();
     if (w == 0) {
         const int nw = blockDim.x >> 5;
-        float m = lane < nw ? sm_m[lane] : -CUDART_INF_F;
-        float s = lane < nw ? sm_s[lane] : 0.f;
-        int a = lane < nw ? sm_a[lane] : 0x7fffffff;
-        warp_merge_stats(m, s, a);
+        SoftStats x;
+        if (lane < nw) {
+            x.m = sm_m[lane];
+            x.s = sm_s[lane];
+            x.t = sm_t[lane];
+            x.m2 = sm_m2[lane];
+            x.a = sm_a[lane];
+        }
+        warp_merge_stats(x);
         if (lane == 0) {
-            v.part[blockIdx.x * 4 + 0] = m;
-            v.part[blockIdx.x * 4 + 1] = s;
-            reinterpret_cast<int*>(v.part)[blockIdx.x * 4 + 2] = a;
+            float* q = v.part + blockIdx.x * 8;
+            q[0] = x.m;
+            q[1] = x.s;
+            q[2] = x.t;
+            q[3] = x.m2;
+            reinterpret_cast<int*>(q)[4] = x.a;
             __threadfence();
             is_last = atomicAdd(v.ticket, 1) == (int)gridDim.x - 1;
         }
@@ -848,27 +881,43 @@ __device__ __forceinline__ void vocab_finish(const VocabArgs& v, LaneStats st) {
     __syncthreads();
     if (!is_last || w != 0) return;
     __threadfence();
-    float m = -CUDART_INF_F, s = 0.f;
-    int a = 0x7fffffff;
-    for (int b = lane; b < (int)gridDim.x; b += 32)
-        merge_stats(m, s, a, __ldcg(&v.part[b * 4 + 0]), __ldcg(&v.part[b * 4 + 1]),
-                    __ldcg(reinterpret_cast<const int*>(v.part) + b * 4 + 2));
-    warp_merge_stats(m, s, a);
+    SoftStats x;
+    for (int b = lane; b < (int)gridDim.x; b += 32) {
+        const float* q = v.part + b * 8;
+        SoftStats y;
+        y.m = __ldcg(q + 0);
+        y.s = __ldcg(q + 1);
+        y.t = __ldcg(q + 2);
+        y.m2 = __ldcg(q + 3);
+        y.a = __ldcg(reinterpret_cast<const int*>(q) + 4);
+        x.merge(y);
+    }
+    warp_merge_stats(x);
     if (lane != 0) return;
     *v.ticket = 0;
-    const float p = 1.0f / s;
+    const int a = x.a;
+    const float p = 1.0f / x.s;
+    const float margin = (1.0f - expf(x.m2 - x.m)) / x.s;
+    const float negent = x.t / x.s - logf(x.s);
     if (v.mode == 0) {
         *v.out_token = a;
-        *v.out_p = p;
+        if (v.out_p) *v.out_p = p;
+        if (v.out_sig) {
+            v.out_sig[0] = p;
+            v.out_sig[1] = margin;
+            v.out_sig[2] = negent;
+        }
         return;
     }
     Ctl* c = v.ctl;
-    if (!(p == p) || a < 0 || a >= v.V) atomicOr(&c->err, kErrNanConfidence);
+    const int kind = c->conf_kind;
+    const float sig = kind == EE_CONF_MARGIN ? margin : (kind == EE_CONF_NEGENT ? negent : p);
+    if (!(sig == sig) || !(p == p) || a < 0 || a >= v.V) atomicOr(&c->err, kErrNanConfidence);
     if (v.mode == 1) {
         const int r = v.r;
         const int f = c->sched ? (int)c->sched[c->step] : c->force;
-        const int pass = p > c->tau[r] ? 1 : 0;
-        c->conf[r] = p;
+        const int pass = sig > c->tau[r] ? 1 : 0;
+        c->conf[r] = sig;
         c->readout_token[r] = a;
         c->gate_pass[r] = pass;
         c->n_evaluated = r + 1;
@@ -881,7 +930,7 @@ __device__ __forceinline__ void vocab_finish(const VocabArgs& v, LaneStats st) {
     } else {
         c->token = a;
         c->full_token = a;
-        c->full_conf = p;
+        c->full_conf = sig;
         c->exit_readout = -1;
     }
 }
@@ -1381,6 +1430,7 @@ __global__ void k_set_inputs(Ctl* c, CtlInputs in) {
     c->step = 0;
     c->n_steps = in.n_steps;
     c->dbg = in.dbg;
+    c->conf_kind = in.conf_kind;
     for (int r = 0; r < kMaxReadouts; ++r) c->tau[r] = in.tau[r];
     c->sched = in.sched;
     c->out_tokens = in.out_tokens;

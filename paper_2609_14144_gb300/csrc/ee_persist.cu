@@ -60,7 +60,6 @@ __device__ __forceinline__ float bf(uint16_t b) { return __uint_as_float((uint32
 __device__ __forceinline__ float bflo(uint32_t v) { return __uint_as_float(v << 16); }
 __device__ __forceinline__ float bfhi(uint32_t v) { return __uint_as_float(v & 0xffff0000u); }
 __device__ __forceinline__ uint16_t tobf(float f) { return __bfloat16_as_ushort(__float2bfloat16_rn(f)); }
-__device__ __forceinline__ float round_bf(float f) { return bf(tobf(f)); }
 
 __device__ __forceinline__ long long cycles() { return clock64(); }
 // Bookkeeping of a bounded wait: true once the wait has run out of time or
@@ -232,19 +231,6 @@ __device__ __forceinline__ float stage_dot(uint32_t wl, uint32_t xl, int cc_firs
     return t;
 }
 
-__device__ __forceinline__ float dot8(const uint4 w, const float* x) {
-    const float4 a = *reinterpret_cast<const float4*>(x);
-    const float4 b = *reinterpret_cast<const float4*>(x + 4);
-    float s = bflo(w.x) * a.x;
-    s = fmaf(bfhi(w.x), a.y, s);
-    s = fmaf(bflo(w.y), a.z, s);
-    s = fmaf(bfhi(w.y), a.w, s);
-    s = fmaf(bflo(w.z), b.x, s);
-    s = fmaf(bfhi(w.z), b.y, s);
-    s = fmaf(bflo(w.w), b.z, s);
-    s = fmaf(bfhi(w.w), b.w, s);
-    return s;
-}
 
 // ------------------------------------------------------------ work geometry
 // Q/K/V and gate/up are split by whole 32-row tiles: rank r < Ge =
@@ -420,11 +406,6 @@ struct Producer {
         bulk_load(s.ring + (size_t)head.st * kSegChunk, src, bytes, &s.full[head.st], pol);
         head.next(stages);
         ++n;
-    }
-    __device__ __forceinline__ void tiles(const uint8_t* W, int K, int nc, int t0, int t1) {
-        for (int t = t0; t < t1; ++t)
-            for (int c = 0; c < nc; ++c)
-                push(W + (int64_t)t * kTileRows * K * 2 + (int64_t)c * kSegChunk, chunk_bytes(K, c), pol_w);
     }
     // Before leaving: every issued copy has landed (the consumers normally
     // see to that; after a stall they may not have).  Walks back over the

@@ -66,20 +66,23 @@ def forced(o: dict) -> int:
 
 
 def teacher_forced(shape, model, n: int, taus, *, prompt=None, capture: bool = True, graphs: bool = True,
-                   pdl: bool = True, persistent: bool = True, page_perm=None, page_size: int = 64):
+                   pdl: bool = True, persistent: bool = True, page_perm=None, page_size: int = 64,
+                   conf_kind: int = 0):
     """Run the oracle free and the GPU engine teacher-forced on the oracle's
     input tokens and exit decisions.  Returns (first_o, first_g, records,
     oracle, engine)."""
     import oracle
-    from paper_2609_14144_gb300 import OPT_DEBUG_LOGITS, OPT_GRAPHS, OPT_PDL, OPT_PERSISTENT, Engine
+    from paper_2609_14144_gb300 import OPT_CONFIDENCE, OPT_DEBUG_LOGITS, OPT_GRAPHS, OPT_PDL, OPT_PERSISTENT, Engine
 
     prompt = synth.prompt(shape) if prompt is None else np.asarray(prompt, np.int32)
     max_ctx = len(prompt) + n
     orc = oracle.Oracle(shape, model, max_ctx=max_ctx)
+    orc.set_confidence(conf_kind)
     eng = Engine(shape, model, max_ctx=max_ctx, page_size=page_size)
     eng.set_option(OPT_GRAPHS, graphs)
     eng.set_option(OPT_PDL, pdl)
     eng.set_option(OPT_PERSISTENT, 1 if persistent else 0)
+    eng.set_option(OPT_CONFIDENCE, conf_kind)
     eng.set_option(OPT_DEBUG_LOGITS, capture)
     if page_perm is not None:
         eng.set_page_table(page_perm)

@@ -74,6 +74,54 @@ def test_vocab_confidence(V, d):
         assert int(tok.item()) == c["argmax"]
 
 
+@pytest.mark.parametrize("V,d", [(4096, 256), (151936, 1536), (1000, 2048)])
+def test_vocab_signals(V, d):
+    """Section 10's three signals from one pass, against the oracle's
+    definitions on the same logits."""
+    import torch
+
+    from paper_2609_14144_gb300 import vocab_signals
+
+    rng = np.random.default_rng(V * 3 + d)
+    x = rng.standard_normal(d).astype(np.float32)
+    gain = synth.const_bf16(d, 4.0 / (0.02 * math.sqrt(d)))
+    U = synth.normal_bf16(6, 0x778, (V, d))
+    tok, sig = vocab_signals(_dev(x), _dev(gain), _dev(U), 1e-6)
+    torch.cuda.synchronize()
+    c = oracle.confidence(oracle.matvec(U, oracle.rmsnorm(x, gain, 1e-6)))
+    got = sig.cpu().numpy()
+    assert abs(got[0] - c["p1"]) <= 1e-4
+    assert abs(got[1] - c["gap"]) <= 1e-4
+    assert abs(got[2] - c["neg_entropy"]) <= 1e-4 * max(1.0, abs(c["neg_entropy"]))
+    if c["gap"] >= 1e-3:
+        assert int(tok.item()) == c["argmax"]
+
+
+def test_vocab_signals_tie_and_uniform():
+    import torch
+
+    from paper_2609_14144_gb300 import vocab_signals
+
+    V, d = 50000, 256
+    U = np.zeros((V, d), np.uint16)
+    row = to_bf16_bits(np.linspace(-1, 1, d).astype(np.float32))
+    for v in (40000, 12345, 49999):
+        U[v] = row
+    x = np.linspace(-1, 1, d).astype(np.float32)
+    gain = synth.const_bf16(d, 1.0)
+    tok, sig = vocab_signals(_dev(x), _dev(gain), _dev(U), 1e-6)
+    torch.cuda.synchronize()
+    c = oracle.confidence(oracle.matvec(U, oracle.rmsnorm(x, gain, 1e-6)))
+    assert int(tok.item()) == 12345 and float(sig[1].item()) == 0.0
+    assert abs(float(sig[2].item()) - c["neg_entropy"]) <= 1e-4 * abs(c["neg_entropy"])
+    # all-zero matrix: uniform distribution, p1 = 1/V, margin 0, -log V
+    tok, sig = vocab_signals(_dev(x), _dev(gain), _dev(np.zeros((V, d), np.uint16)), 1e-6)
+    torch.cuda.synchronize()
+    got = sig.cpu().numpy()
+    assert int(tok.item()) == 0 and got[1] == 0.0
+    assert abs(got[0] - 1.0 / V) <= 1e-9 and abs(got[2] + math.log(V)) <= 1e-4
+
+
 def test_vocab_confidence_ties_lowest_index():
     import torch
 

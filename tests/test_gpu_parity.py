@@ -219,3 +219,26 @@ def test_1p5b_long_three_readouts_structure():
     fo, fg, recs, orc, eng = teacher_forced(shape, model, shape.new_tokens, taus, capture=False)
     assert fo == fg
     check_records(recs, taus, capture=False)
+
+
+@pytest.mark.parametrize("kind,tau", [(1, 0.25), (2, -2.0)])
+@pytest.mark.parametrize("persistent", [True, False])
+def test_tiny_margin_and_entropy_gates(tiny_model, kind, tau, persistent):
+    """Section 10: the gate on the margin p1 - p2 or on the negative entropy;
+    tokens, verdicts and recorded signals against the oracle's."""
+    n = TINY.new_tokens
+    fo, fg, recs, orc, eng = teacher_forced(TINY, tiny_model, n, [tau], conf_kind=kind, persistent=persistent)
+    assert fo == fg
+    excluded = check_records(recs, [tau])
+    assert excluded <= n // 8
+    st, so = eng.stats(), orc.stats()
+    assert 0 < so["exits"][0] < n
+    assert st["exits"] == so["exits"]
+
+
+def test_1p5b_entropy_gate():
+    shape = synth.CONFIGS["1.5b"].replace(new_tokens=6)
+    model = synth.make_model(shape)
+    fo, fg, recs, orc, eng = teacher_forced(shape, model, shape.new_tokens, [-3.0], conf_kind=2)
+    assert fo == fg
+    check_records(recs, [-3.0])
