@@ -71,7 +71,8 @@ class StepResult(ctypes.Structure):
                 ("exit_layer", ctypes.c_int32), ("n_evaluated", ctypes.c_int32), ("full_token", ctypes.c_int32),
                 ("gate_pass", ctypes.c_int32 * MAX_READOUTS), ("readout_token", ctypes.c_int32 * MAX_READOUTS),
                 ("confidence", ctypes.c_float * MAX_READOUTS), ("gap", ctypes.c_float * MAX_READOUTS),
-                ("full_confidence", ctypes.c_float), ("full_gap", ctypes.c_float)]
+                ("full_confidence", ctypes.c_float), ("full_gap", ctypes.c_float),
+                ("nucleus_member", ctypes.c_int32), ("nucleus_mass", ctypes.c_float)]
 
     def as_dict(self) -> dict:
         n = self.n_evaluated
@@ -79,7 +80,8 @@ class StepResult(ctypes.Structure):
                 "exit_layer": self.exit_layer, "n_evaluated": n, "full_token": self.full_token,
                 "gate_pass": list(self.gate_pass[:n]), "readout_token": list(self.readout_token[:n]),
                 "confidence": list(self.confidence[:n]), "gap": list(self.gap[:n]),
-                "full_confidence": self.full_confidence, "full_gap": self.full_gap}
+                "full_confidence": self.full_confidence, "full_gap": self.full_gap,
+                "nucleus_member": self.nucleus_member, "nucleus_mass": self.nucleus_mass}
 
 
 class Capture(ctypes.Structure):
@@ -111,6 +113,10 @@ def _load():
             lib.orc_add_readout.argtypes = [_P, ctypes.c_int, _P, _P]
             lib.orc_reset.argtypes = [_P]
             lib.orc_set_confidence.argtypes = [_P, ctypes.c_int]
+            lib.orc_set_nucleus.argtypes = [_P, ctypes.c_double]
+            lib.orc_op_nucleus_member.argtypes = [_P, ctypes.c_int64, ctypes.c_int32, ctypes.c_double,
+                                                  ctypes.POINTER(ctypes.c_double)]
+            lib.orc_select_tau.argtypes = [_P, _P, ctypes.c_int, ctypes.c_double, ctypes.POINTER(ctypes.c_float)]
             lib.orc_prefill.argtypes = [_P, _P, ctypes.c_int, ctypes.POINTER(ctypes.c_int32),
                                         ctypes.POINTER(Capture)]
             lib.orc_decode_step.argtypes = [_P, ctypes.c_int32, _P, ctypes.c_int, ctypes.POINTER(StepResult),
@@ -182,6 +188,26 @@ def confidence(logits) -> dict:
             "neg_entropy": c.neg_entropy}
 
 
+def nucleus_member(logits, token: int, p_nuc: float = 0.9):
+    """Section 2: (member, mass) -- whether `token` lies in the nucleus of
+    share p_nuc, and the probability of the tokens strictly above it."""
+    l = _f32(logits)
+    mass = ctypes.c_double(0.0)
+    r = _load().orc_op_nucleus_member(l.ctypes.data, l.size, int(token), float(p_nuc), ctypes.byref(mass))
+    return bool(r), mass.value
+
+
+def select_tau(conf, member, target: float = 0.9) -> float:
+    """Section 4, step four: the lowest tau at which at least `target` of the
+    early answers (conf > tau) are acceptable; inf if none."""
+    c = _f32(conf)
+    mb = np.ascontiguousarray(member, dtype=np.int32)
+    tau = ctypes.c_float(0.0)
+    if _load().orc_select_tau(c.ctypes.data, mb.ctypes.data, c.size, float(target), ctypes.byref(tau)) != 0:
+        raise ValueError("oracle: select_tau failed")
+    return tau.value
+
+
 # ---------------------------------------------------------------- model
 TRACE_FIELDS = ("h_in", "u_attn", "q", "k", "v", "o", "h_mid", "u_mlp", "gate", "up", "a", "h_out")
 
@@ -251,6 +277,10 @@ class Oracle:
 
     def reset(self):
         self.lib.orc_reset(self.ptr)
+
+    def set_nucleus(self, p_nuc: float):
+        if self.lib.orc_set_nucleus(self.ptr, float(p_nuc)) != 0:
+            raise ValueError("oracle: bad nucleus share")
 
     def set_confidence(self, kind: int):
         """Gate signal: CONF_PMAX (default), CONF_MARGIN or CONF_NEGENT (Section 10)."""

@@ -24,6 +24,11 @@
  *     best and second-best probabilities, and the negative entropy of the
  *     readout's distribution are interchangeable softmax confidences; the
  *     gate can use any of them (orc_set_confidence).
+ *   - Section 2 (nucleus, acceptance) and Section 4, step four: an early
+ *     answer is acceptable when it lies in the full model's nucleus (the
+ *     most probable tokens holding 90 percent of the probability); the
+ *     threshold is the lowest one at which the required share of early
+ *     answers is acceptable (orc_select_tau).
  *   - Appendix C: the layer is four attention projections with grouped-query
  *     attention (A query heads, K key-value heads of size D) and a gated
  *     feed-forward block of three matrices of width F.
@@ -108,6 +113,11 @@ typedef struct {
     float confidence[ORC_MAX_READOUTS];
     float gap[ORC_MAX_READOUTS];
     float full_confidence, full_gap;
+    /* Full steps with a readout: whether readout 0's token lies in the full
+     * model's nucleus (1/0; -1 when not computed) and the full-model
+     * probability of the tokens strictly more probable than it. */
+    int32_t nucleus_member;
+    float nucleus_mass;
 } orc_step_result;
 
 /* Optional captures of one step; any pointer may be NULL. */
@@ -133,6 +143,7 @@ typedef struct {
     int8_t* kv_src;  /* [L][max_ctx]: 0 empty, 1 computed by the layer, 2 filled */
     int pos;
     int conf_kind; /* ORC_CONF_*: the signal the gate compares with tau */
+    double nucleus_p; /* share of probability the nucleus holds */
     int64_t steps, full_steps, exits[ORC_MAX_READOUTS];
     float *h, *u, *q, *kk, *vv, *o, *g, *up, *a, *y, *z, *logits, *tmp;
 } orc_model;
@@ -283,6 +294,54 @@ static float conf_signal(const orc_model* m, const orc_conf* cf) {
     }
 }
 
+/* Nucleus membership (Section 2): token x belongs to the nucleus of share
+ * p_nuc when the tokens strictly more probable than x hold less than p_nuc
+ * of the probability (the smallest top set reaching p_nuc then includes x,
+ * a tied group at the boundary included).  Returns that mass in *mass. */
+int orc_op_nucleus_member(const float* l, int64_t V, int32_t x, double p_nuc, double* mass) {
+    float mx = l[0];
+    for (int64_t v = 1; v < V; ++v)
+        if (l[v] > mx) mx = l[v];
+    double sum = 0.0, above = 0.0;
+    for (int64_t v = 0; v < V; ++v) {
+        const double e = exp((double)l[v] - (double)mx);
+        sum += e;
+        if (l[v] > l[x]) above += e;
+    }
+    const double mabove = above / sum;
+    if (mass) *mass = mabove;
+    return mabove < p_nuc ? 1 : 0;
+}
+
+int orc_set_nucleus(orc_model* m, double p_nuc) {
+    if (!m || !(p_nuc > 0.0 && p_nuc <= 1.0)) return -1;
+    m->nucleus_p = p_nuc;
+    return 0;
+}
+
+/* Section 4, step four: given the readout's confidence conf[i] and whether
+ * its answer was acceptable (member[i]) at n held-out positions, the lowest
+ * threshold tau at which at least `target` of the early answers (the
+ * positions with conf > tau) are acceptable.  Candidates are -inf (every
+ * position exits) and each observed confidence; a candidate with no early
+ * answer does not count.  *tau = +inf when none meets the target. */
+int orc_select_tau(const float* conf, const int32_t* member, int n, double target, float* tau) {
+    if (!conf || !member || !tau || n < 0) return -1;
+    *tau = INFINITY;
+    for (int c = -1; c < n; ++c) {
+        const float cand = c < 0 ? -INFINITY : conf[c];
+        if (c >= 0 && !(cand < *tau)) continue; /* only lower candidates can improve */
+        int early = 0, good = 0;
+        for (int i = 0; i < n; ++i)
+            if (conf[i] > cand) {
+                ++early;
+                good += member[i] != 0;
+            }
+        if (early > 0 && (double)good >= target * (double)early && cand < *tau) *tau = cand;
+    }
+    return 0;
+}
+
 int orc_set_confidence(orc_model* m, int kind) {
     if (!m || kind < ORC_CONF_PMAX || kind > ORC_CONF_NEGENT) return -1;
     m->conf_kind = kind;
@@ -331,6 +390,7 @@ orc_model* orc_create(const orc_config* c, const orc_weights* w) {
     orc_model* m = (orc_model*)calloc(1, sizeof(orc_model));
     if (!m) return NULL;
     m->c = *c;
+    m->nucleus_p = 0.9;
     const int L = c->n_layers;
     m->ptrs = (const uint16_t**)calloc((size_t)L * 13, sizeof(uint16_t*));
     const uint16_t* const* src[13] = {w->attn_norm, w->wq, w->wk, w->wv, w->bq, w->bk, w->bv,
@@ -548,6 +608,7 @@ int orc_decode_step(orc_model* m, int32_t in_tok, const float* taus, int force, 
     const int d = c->d_model, L = c->n_layers, V = c->vocab;
     const int t = m->pos;
     memset(res, 0, sizeof(*res));
+    res->nucleus_member = -1;
     res->exit_readout = -1;
     res->full_token = -1;
     res->exit_layer = L;
@@ -592,6 +653,11 @@ int orc_decode_step(orc_model* m, int32_t in_tok, const float* taus, int force, 
         res->full_token = cf.argmax;
         res->full_confidence = conf_signal(m, &cf);
         res->full_gap = cf.gap;
+        if (m->n_readouts > 0 && res->n_evaluated > 0) {
+            double mass = 0.0;
+            res->nucleus_member = orc_op_nucleus_member(m->logits, V, res->readout_token[0], m->nucleus_p, &mass);
+            res->nucleus_mass = (float)mass;
+        }
         if (cap && cap->h_final) memcpy(cap->h_final, m->h, sizeof(float) * d);
         if (cap && cap->final_logits) memcpy(cap->final_logits, m->logits, sizeof(float) * V);
         m->full_steps++;

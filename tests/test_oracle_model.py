@@ -224,6 +224,31 @@ def test_gate_with_margin_and_negative_entropy():
         oracle.Oracle(TINY, model).set_confidence(3)
 
 
+def test_nucleus_membership_of_the_readout_answer():
+    """Section 2 acceptance: on full steps the oracle reports whether readout
+    0's token lies in the full model's nucleus (from the final logits); on
+    exit steps it is not computed."""
+    model = synth.make_model(TINY)
+    o = oracle.Oracle(TINY, model)
+    tok = o.prefill(synth.prompt(TINY))
+    seen = set()
+    for i in range(24):
+        force = oracle.FORCE_EXIT_AT(0) if i % 4 == 3 else oracle.FORCE_FULL
+        s = o.decode_step(tok, [0.5], force, capture=True)
+        if s["exited"]:
+            assert s["nucleus_member"] == -1
+        else:
+            m, mass = oracle.nucleus_member(s["capture"]["final_logits"], s["readout_token"][0], 0.9)
+            assert s["nucleus_member"] == int(m) and s["nucleus_mass"] == np.float32(mass)
+            seen.add(s["nucleus_member"])
+        tok = s["token"]
+    o.set_nucleus(1.0)
+    s = o.decode_step(tok, [0.5], oracle.FORCE_FULL)
+    assert s["nucleus_member"] == 1
+    with pytest.raises(ValueError):
+        o.set_nucleus(0.0)
+
+
 # ------------------------------------------------------------- structure
 def _trace_step(shape, model, force=oracle.FORCE_FULL, taus=(0.5,)):
     o = oracle.Oracle(shape, model)

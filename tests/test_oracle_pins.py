@@ -223,3 +223,66 @@ def test_negative_entropy_and_margin_closed_forms():
     c = oracle.confidence(np.array([0.5, -0.75], np.float32))
     p = 1 / (1 + math.exp(-1.25))
     assert c["neg_entropy"] == pytest.approx(p * math.log(p) + (1 - p) * math.log(1 - p), rel=1e-6)
+
+
+def _nucleus_by_sorting(l, x, p_nuc):
+    """The nucleus as the smallest set of most probable tokens whose
+    probability reaches p_nuc, by sorting (continuous logits, no ties)."""
+    p = scipy.special.softmax(l.astype(np.float64))
+    order = np.argsort(-p, kind="stable")
+    k = int(np.searchsorted(np.cumsum(p[order]), p_nuc)) + 1
+    return x in set(order[:k].tolist())
+
+
+def test_nucleus_membership_against_sorting():
+    """Section 2: a token is in the nucleus when it belongs to the smallest
+    set of most probable tokens holding 90 percent of the probability."""
+    for V, scale in ((50, 1.0), (4096, 3.0), (151936, 6.0)):
+        l = (RNG.standard_normal(V) * scale).astype(np.float32)
+        order = np.argsort(-l)
+        for x in list(order[:40]) + list(RNG.integers(0, V, 20)):
+            got, mass = oracle.nucleus_member(l, int(x), 0.9)
+            assert got == _nucleus_by_sorting(l, int(x), 0.9), (V, x, mass)
+            p = scipy.special.softmax(l.astype(np.float64))
+            assert mass == pytest.approx(float(p[p > p[x]].sum()), rel=1e-9, abs=1e-12)
+
+
+def test_nucleus_membership_special_cases():
+    V = 1000
+    # uniform: nothing is more probable than any token, all are members
+    assert all(oracle.nucleus_member(np.zeros(V, np.float32), x)[0] for x in (0, 499, 999))
+    # one token holding more than 90 percent: the nucleus is that token alone
+    l = np.zeros(V, np.float32)
+    l[5] = 20.0
+    assert oracle.nucleus_member(l, 5)[0] and not oracle.nucleus_member(l, 6)[0]
+    # share 1.0 keeps every token
+    l = (RNG.standard_normal(V) * 4).astype(np.float32)
+    assert all(oracle.nucleus_member(l, x, 1.0)[0] for x in range(0, V, 97))
+
+
+def _select_tau_brute(conf, member, target):
+    best = math.inf
+    for cand in [-math.inf] + sorted(set(float(c) for c in conf)):
+        early = [m for c, m in zip(conf, member) if c > cand]
+        if early and sum(early) >= target * len(early):
+            best = min(best, cand)
+    return best
+
+
+def test_select_tau_against_brute_force():
+    """Section 4, step four: the lowest threshold at which the required share
+    of early answers is acceptable."""
+    for n, q in ((1, 0.5), (7, 0.5), (200, 0.8), (2000, 0.6)):
+        conf = RNG.random(n).astype(np.float32)
+        member = (RNG.random(n) < q * (0.5 + conf)).astype(np.int32)
+        for target in (0.5, 0.9, 0.99):
+            assert oracle.select_tau(conf, member, target) == np.float32(_select_tau_brute(conf, member, target))
+    # every answer acceptable: everything may exit; none acceptable: nothing may
+    conf = RNG.random(50).astype(np.float32)
+    assert oracle.select_tau(conf, np.ones(50, np.int32), 0.9) == -math.inf
+    assert oracle.select_tau(conf, np.zeros(50, np.int32), 0.9) == math.inf
+    # acceptability rising with confidence: tau sits just below the good run
+    conf = np.arange(10, dtype=np.float32) / 10
+    member = np.array([0, 0, 0, 1, 0, 1, 1, 1, 1, 1], np.int32)
+    assert oracle.select_tau(conf, member, 1.0) == np.float32(0.4)
+    assert oracle.select_tau(conf, member, 0.8) == np.float32(0.2)
