@@ -117,6 +117,11 @@ typedef struct {
     int32_t readout_token[EE_MAX_READOUTS]; /* argmax of each evaluated readout */
     float confidence[EE_MAX_READOUTS];      /* p_r of each evaluated readout   */
     float full_confidence;                  /* LM head top-1 probability      */
+    int32_t nucleus_member; /* EE_OPT_NUCLEUS on a full-depth step: 1 if readout 0's
+                               token lies in the LM head's nucleus (Section 2
+                               acceptance), else 0; -1 when not computed      */
+    float nucleus_mass;     /* LM head probability of the tokens strictly more
+                               probable than readout 0's token (0 if not computed) */
 } ee_step_result;
 
 /* Exit statistics since the last ee_reset (Section 2, "exit rate"). */
@@ -187,6 +192,32 @@ int ee_decode_step(ee_ctx* ctx, int32_t input_token, const float* taus, int forc
 int ee_decode_n(ee_ctx* ctx, int n, int32_t input_token, const float* taus, const int8_t* force_schedule,
                 int32_t* tokens, int32_t* exit_readout, float* confidence, int where);
 
+/* Fidelity calibration pass (Section 2 acceptance; Section 4, step four).
+ * n teacher-forced full-depth steps from the current position: step i takes
+ * ids[i] as its input token, every readout is evaluated (its gate never
+ * taken) and the LM head checks whether readout 0's token lies in the full
+ * model's nucleus of share p_nuc, the smallest set of most probable tokens
+ * whose probability reaches p_nuc: it does when the tokens strictly more
+ * probable than it hold less than p_nuc.  One graph launch, no host round
+ * trip between steps.
+ *   ids    [n] int32 in [0, V)
+ *   p_nuc  in (0, 1]
+ *   conf   [n][n_readouts] float: each readout's confidence signal (the
+ *          EE_OPT_CONFIDENCE kind) at step i, row-major; may be NULL
+ *   member [n] int32: 1/0 nucleus membership of readout 0's token; may be NULL
+ *   mass   [n] float: probability of the tokens above it; may be NULL
+ *   where  EE_HOST: host arrays (ids read, results written before return);
+ *          EE_DEVICE: device arrays, the call returns once enqueued.
+ * The position advances by n; the KV cache holds the full model's entries of
+ * ids and the next input is the full model's token after ids[n - 1].  The
+ * steps count as full-depth steps in ee_get_stats.  Requires at least one
+ * readout (EE_ESTATE otherwise); EE_EINVAL for a bad argument (ids are
+ * range-checked on the host when where = EE_HOST, on the device otherwise:
+ * an out-of-range id sets the device error word); EE_ERANGE if the steps
+ * would pass max_ctx. */
+int ee_calibrate(ee_ctx* ctx, const int32_t* ids, int n, float p_nuc, float* conf, int32_t* member, float* mass,
+                 int where);
+
 /* Wait for the context's stream and report the device error word. */
 int ee_sync(ee_ctx* ctx);
 int ee_get_stats(ee_ctx* ctx, ee_stats* out);
@@ -210,6 +241,10 @@ int ee_position(ee_ctx* ctx, int32_t* pos);
                                  CTA per SM streaming weights through a shared-
                                  memory ring; 0: five launches per layer.
                                  EE_EINVAL if the shape is not supported      */
+#define EE_OPT_NUCLEUS 6      /* 0 (default): off; 1..1000: full-depth steps of
+                                 ee_decode_step report the nucleus membership of
+                                 readout 0's token at share value/1000
+                                 (Section 2 acceptance)                      */
 int ee_set_option(ee_ctx* ctx, int option, int value);
 
 #define EE_DBG_HIDDEN_READOUT 1 /* layer = readout r: residual h_k it read, d floats   */
@@ -303,6 +338,23 @@ int ee_vocab_confidence(const float* x, const uint16_t* gain, const uint16_t* U,
 int ee_vocab_signals(const float* x, const uint16_t* gain, const uint16_t* U, int vocab, int d_model,
                      float eps, void* scratch, size_t scratch_bytes, int32_t* out_token, float* out_signals,
                      float* logits, void* stream);
+
+/* Threshold selection (Section 4, step four): the lowest tau at which at
+ * least a share `target` of the early answers (the positions with
+ * conf > tau) are acceptable.  Candidates are -inf (every position exits)
+ * and each conf[i * conf_stride]; a candidate with no early answer does not
+ * count; *tau = +inf when no candidate reaches the target.  The acceptance
+ * test is good >= target * early in double precision.
+ *   conf    device float, n entries at stride conf_stride (>= 1), e.g. one
+ *           column of ee_calibrate's conf
+ *   member  device int32 [n], nonzero = acceptable
+ *   target  in [0, 1]
+ *   tau     device float [1] (result)
+ *   scratch device workspace of 8 bytes
+ * Enqueued on stream (n >= 1; EE_EINVAL otherwise).  The work is n + 1
+ * candidates times n comparisons, spread over the whole GPU. */
+int ee_select_tau(const float* conf, int conf_stride, const int32_t* member, int n, float target, float* tau,
+                  void* scratch, void* stream);
 
 #ifdef __cplusplus
 }

@@ -12,11 +12,11 @@ import numpy as np
 
 from . import _lib
 from ._lib import (CONF_MARGIN, CONF_NEGENT, CONF_PMAX, DEVICE, FORCE_FULL, FREE, HOST, MAX_READOUTS,
-                   OPT_CONFIDENCE, OPT_DEBUG_LOGITS, OPT_GRAPHS, OPT_PDL, OPT_PERSISTENT, EEError, FORCE_EXIT_AT,
-                   check)
+                   OPT_CONFIDENCE, OPT_DEBUG_LOGITS, OPT_GRAPHS, OPT_NUCLEUS, OPT_PDL, OPT_PERSISTENT, EEError,
+                   FORCE_EXIT_AT, check)
 
 __all__ = ["Engine", "EEError", "FREE", "FORCE_FULL", "FORCE_EXIT_AT", "HOST", "DEVICE", "attention_decode",
-           "vocab_confidence", "vocab_signals", "library_path"]
+           "vocab_confidence", "vocab_signals", "select_tau", "library_path"]
 
 
 def library_path() -> str:
@@ -168,6 +168,36 @@ class Engine:
                                    exit_readout.data_ptr(), confidence.data_ptr(), DEVICE))
         return tokens, exit_readout, confidence
 
+    def calibrate(self, ids, p_nuc: float = 0.9, where: int = HOST, conf=None, member=None, mass=None):
+        """Teacher-forced full-depth pass over ids recording every readout's
+        confidence and whether readout 0's token lies in the full model's
+        nucleus of share p_nuc (Section 2 acceptance, Section 4 step four).
+        where=HOST: ids is a host sequence, returns numpy (conf [n, R], member
+        [n], mass [n]); where=DEVICE: ids is an int32 CUDA tensor, the given
+        (or new) tensors are filled without synchronising."""
+        import torch
+
+        R = self.n_readouts
+        if where == HOST:
+            a = np.ascontiguousarray(ids, dtype=np.int32)
+            n = a.size
+            cf = np.zeros((n, R), np.float32)
+            mb = np.zeros(n, np.int32)
+            ms = np.zeros(n, np.float32)
+            check(self.lib.ee_calibrate(self.ctx, a.ctypes.data, int(n), float(p_nuc), cf.ctypes.data, mb.ctypes.data,
+                                        ms.ctypes.data, HOST))
+            return cf, mb, ms
+        n = ids.numel()
+        if conf is None:
+            conf = torch.empty((n, R), dtype=torch.float32, device=self.device)
+        if member is None:
+            member = torch.empty(n, dtype=torch.int32, device=self.device)
+        if mass is None:
+            mass = torch.empty(n, dtype=torch.float32, device=self.device)
+        check(self.lib.ee_calibrate(self.ctx, ids.data_ptr(), int(n), float(p_nuc), conf.data_ptr(),
+                                    member.data_ptr(), mass.data_ptr(), DEVICE))
+        return conf, member, mass
+
     def sync(self):
         check(self.lib.ee_sync(self.ctx))
 
@@ -277,3 +307,27 @@ def vocab_signals(x, gain, U, eps: float, logits=None, scratch=None, stream=None
                                scratch.numel(), tok.data_ptr(), sig.data_ptr(),
                                None if logits is None else logits.data_ptr(), s.cuda_stream))
     return tok, sig
+
+
+def select_tau(conf, member, target: float, tau=None, scratch=None, stream=None):
+    """Section 4, step four on the device: the lowest tau at which at least
+    `target` of the early answers (conf > tau) are acceptable (member != 0);
+    -inf when every answer may exit, +inf when no threshold reaches the
+    target.  conf: float32 CUDA tensor [n] or a column of [n, R] (any stride);
+    member: int32 CUDA tensor [n].  Returns a float32 tensor [1]."""
+    import torch
+
+    lib = _lib.load()
+    n = member.numel()
+    if conf.dim() != 1 or conf.numel() != n or conf.dtype != torch.float32 or member.dtype != torch.int32:
+        raise ValueError("conf must be float32 [n] and member int32 [n]")
+    if not member.is_contiguous():
+        raise ValueError("member must be contiguous")
+    if tau is None:
+        tau = torch.empty(1, dtype=torch.float32, device=conf.device)
+    if scratch is None:
+        scratch = torch.empty(2, dtype=torch.int32, device=conf.device)
+    s = stream if stream is not None else torch.cuda.current_stream(conf.device)
+    check(lib.ee_select_tau(conf.data_ptr(), int(conf.stride(0)), member.data_ptr(), int(n), float(target),
+                            tau.data_ptr(), scratch.data_ptr(), s.cuda_stream))
+    return tau

@@ -59,7 +59,7 @@ struct Layout {
     size_t kpool, vpool, page_table, kv_src, h, q, o, a, y, hk, logits_ro, logits_final;
     size_t gemv_part, gemv_ticket, attn_part, attn_ticket, vocab_part, vocab_ticket;
     size_t seg_dpart, seg_opart, seg_sync;
-    size_t prompt, sched, out_tok, out_exit, out_conf, total;
+    size_t prompt, sched, out_tok, out_exit, out_conf, out_conf_all, out_member, out_mass, tau_scratch, total;
     int64_t layer_stride, off_wqkv, off_bqkv, off_gattn, off_wo, off_gmlp, off_wgu, off_wd;
     int64_t n_units_qkv, kv_layer_stride, gemv_ticket_stride;
     int n_pages;
@@ -160,6 +160,10 @@ Layout make_layout(const ee_model_config& c) {
     l.out_tok = take(4 * (size_t)c.max_ctx);
     l.out_exit = take(4 * (size_t)c.max_ctx);
     l.out_conf = take(4 * (size_t)c.max_ctx);
+    l.out_conf_all = take(4 * (size_t)c.max_ctx * R);
+    l.out_member = take(4 * (size_t)c.max_ctx);
+    l.out_mass = take(4 * (size_t)c.max_ctx);
+    l.tau_scratch = take(8);
     l.total = b;
     return l;
 }
@@ -218,6 +222,7 @@ struct ee_ctx {
     SegPlan seg{};
     int dbg = 0;
     int conf_kind = EE_CONF_PMAX;  // signal the gates compare with tau
+    int nucleus_permille = 0;      // EE_OPT_NUCLEUS: nucleus share in 1/1000, 0 = off
     cudaGraphExec_t g_step = nullptr, g_n = nullptr, g_prefill = nullptr;
     int grid_gemv = 0, grid_vocab = 0;
     int attn_cluster = 8;  // CTAs per key-value head in the attention kernel
@@ -562,6 +567,8 @@ CtlInputs base_inputs(const ee_ctx* c, const float* taus) {
     in.n_steps = 1;
     in.dbg = c->dbg;
     in.conf_kind = c->conf_kind;
+    in.nucleus_on = c->nucleus_permille > 0 && c->n_readouts > 0;
+    in.nucleus_p = (float)c->nucleus_permille / 1000.0f;
     for (int r = 0; r < kMaxReadouts; ++r) in.tau[r] = (taus && r < c->n_readouts) ? taus[r] : 2.0f;
     return in;
 }
@@ -890,6 +897,10 @@ int ee_set_option(ee_ctx* c, int option, int value) {
             if (value < EE_CONF_PMAX || value > EE_CONF_NEGENT) return fail(EE_EINVAL, "unknown confidence signal");
             c->conf_kind = value;
             return EE_OK;
+        case EE_OPT_NUCLEUS:
+            if (value < 0 || value > 1000) return fail(EE_EINVAL, "nucleus share must be 0..1000 per mille");
+            c->nucleus_permille = value;
+            return EE_OK;
         case EE_OPT_PERSISTENT:
             if (value && !c->seg_ok) return fail(EE_EINVAL, "the persistent layer kernel does not support this shape");
             if (c->use_persistent != (value != 0)) drop_graphs(c);
@@ -975,6 +986,8 @@ int ee_decode_step(ee_ctx* c, int32_t input_token, const float* taus, int force,
         out->confidence[r] = h->conf[r];
     }
     out->full_confidence = h->exit_readout >= 0 ? 0.f : h->full_conf;
+    out->nucleus_member = in.nucleus_on && h->exit_readout < 0 ? h->nucleus_member : -1;
+    out->nucleus_mass = out->nucleus_member >= 0 ? h->nucleus_mass : 0.f;
     c->pos = h->pos;
     return EE_OK;
 }
@@ -1027,6 +1040,67 @@ int ee_decode_n(ee_ctx* c, int n, int32_t input_token, const float* taus, const 
         if (tokens) EE_CK(cudaMemcpyAsync(tokens, d_tok, 4 * (size_t)n, cudaMemcpyDeviceToHost, s));
         if (exit_readout) EE_CK(cudaMemcpyAsync(exit_readout, d_exit, 4 * (size_t)n, cudaMemcpyDeviceToHost, s));
         if (confidence) EE_CK(cudaMemcpyAsync(confidence, d_conf, 4 * (size_t)n, cudaMemcpyDeviceToHost, s));
+        EE_TRY(fetch_ctl(c));
+        EE_TRY(device_error(c));
+        if (c->h_ctl->pos != c->pos) return fail(EE_EDEVICE, "device position out of step with the host");
+    }
+    return EE_OK;
+}
+
+int ee_calibrate(ee_ctx* c, const int32_t* ids, int n, float p_nuc, float* conf, int32_t* member, float* mass,
+                 int where) {
+    if (!c || !ids) return fail(EE_EINVAL, "NULL argument");
+    if (!c->prefilled) return fail(EE_ESTATE, "calibration before prefill");
+    if (c->n_readouts < 1) return fail(EE_ESTATE, "calibration needs a readout");
+    if (n <= 0) return fail(EE_EINVAL, "n must be positive");
+    if (!(p_nuc > 0.0f && p_nuc <= 1.0f)) return fail(EE_EINVAL, "p_nuc must lie in (0, 1]");
+    if (where != EE_HOST && where != EE_DEVICE) return fail(EE_EINVAL, "where must be EE_HOST or EE_DEVICE");
+    if (c->pos + n > c->cfg.max_ctx) return fail(EE_ERANGE, "steps would pass max_ctx");
+    const int R = c->n_readouts;
+    cudaStream_t s = c->stream;
+    int32_t* d_ids = (int32_t*)(c->ws + c->lay.prompt);
+    if (where == EE_HOST) {
+        for (int i = 0; i < n; ++i)
+            if (ids[i] < 0 || ids[i] >= c->cfg.vocab) return fail(EE_EINVAL, "token id out of range");
+        EE_CK(cudaMemcpyAsync(d_ids, ids, 4 * (size_t)n, cudaMemcpyHostToDevice, s));
+    } else {
+        EE_CK(cudaMemcpyAsync(d_ids, ids, 4 * (size_t)n, cudaMemcpyDeviceToDevice, s));
+    }
+    float taus[kMaxReadouts];
+    for (int r = 0; r < kMaxReadouts; ++r) taus[r] = 2.0f;
+    CtlInputs in = base_inputs(c, taus);
+    in.force = EE_FORCE_FULL;
+    in.n_steps = n;
+    in.set_token = 0;
+    in.forced_in = d_ids;
+    in.nucleus_on = 1;
+    in.nucleus_p = p_nuc;
+    float* d_conf = (float*)(c->ws + c->lay.out_conf_all);
+    int32_t* d_member = (int32_t*)(c->ws + c->lay.out_member);
+    float* d_mass = (float*)(c->ws + c->lay.out_mass);
+    if (where == EE_DEVICE) {
+        in.out_conf_all = conf;
+        in.out_member = member;
+        in.out_mass = mass;
+    } else {
+        in.out_conf_all = conf ? d_conf : nullptr;
+        in.out_member = member ? d_member : nullptr;
+        in.out_mass = mass ? d_mass : nullptr;
+    }
+    EE_CK(launch_set_inputs(c->d_ctl, in, s));
+    // step 0's input: ids[0], read on the device
+    EE_CK(cudaMemcpyAsync(&c->d_ctl->in_tok, d_ids, 4, cudaMemcpyDeviceToDevice, s));
+    if (c->use_graphs) {
+        EE_TRY(ensure_graphs(c));
+        EE_CK(cudaGraphLaunch(c->g_n, s));
+    } else {
+        for (int i = 0; i < n; ++i) EE_TRY(eager_step(c));
+    }
+    c->pos += n;
+    if (where == EE_HOST) {
+        if (conf) EE_CK(cudaMemcpyAsync(conf, d_conf, 4 * (size_t)n * R, cudaMemcpyDeviceToHost, s));
+        if (member) EE_CK(cudaMemcpyAsync(member, d_member, 4 * (size_t)n, cudaMemcpyDeviceToHost, s));
+        if (mass) EE_CK(cudaMemcpyAsync(mass, d_mass, 4 * (size_t)n, cudaMemcpyDeviceToHost, s));
         EE_TRY(fetch_ctl(c));
         EE_TRY(device_error(c));
         if (c->h_ctl->pos != c->pos) return fail(EE_EDEVICE, "device position out of step with the host");
@@ -1259,6 +1333,19 @@ int ee_vocab_signals(const float* x, const uint16_t* gain, const uint16_t* U, in
     if (!out_signals) return fail(EE_EINVAL, "NULL argument");
     return vocab_standalone(x, gain, U, vocab, d_model, eps, scratch, scratch_bytes, out_token, nullptr,
                             out_signals, logits, stream);
+}
+
+int ee_select_tau(const float* conf, int conf_stride, const int32_t* member, int n, float target, float* tau,
+                  void* scratch, void* stream) {
+    if (!conf || !member || !tau || !scratch) return fail(EE_EINVAL, "NULL argument");
+    if (n < 1 || conf_stride < 1) return fail(EE_EINVAL, "n and conf_stride must be positive");
+    if (!(target >= 0.0f && target <= 1.0f)) return fail(EE_EINVAL, "target must lie in [0, 1]");
+    int dev = 0, nsm = 0;
+    EE_CK(cudaGetDevice(&dev));
+    EE_CK(cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev));
+    EE_CK(launch_select_tau(conf, conf_stride, member, n, (double)target, tau, (int*)scratch, nsm,
+                            (cudaStream_t)stream));
+    return EE_OK;
 }
 
 }  // extern "C"

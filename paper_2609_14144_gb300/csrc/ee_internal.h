@@ -40,22 +40,28 @@ struct Ctl {
     int32_t prefill_i;    // prompt index of the running prefill
     int32_t max_ctx;
     int32_t conf_kind;    // EE_CONF_*: the signal the gates compare with tau
-    int32_t pad1;
+    int32_t nucleus_on;   // 1: full steps check readout 0's token against the LM head's nucleus
     int32_t gate_pass[kMaxReadouts];
     int32_t readout_token[kMaxReadouts];
     float conf[kMaxReadouts];
     float tau[kMaxReadouts];
     float full_conf;
-    float pad2[3];
+    float nucleus_p;        // share of probability the nucleus holds
+    float nucleus_mass;     // LM head probability of the tokens above readout 0's token
+    int32_t nucleus_member; // readout 0's token in the nucleus (1/0), -1 when not computed
     long long steps, full_steps, exits[kMaxReadouts];
     int32_t* out_tokens;   // per-step outputs of ee_decode_n (may be null)
     int32_t* out_exit;
     float* out_conf;
     const int8_t* sched;   // per-step force values (may be null)
     const int32_t* prompt; // prompt ids of the running prefill
+    float* out_conf_all;   // [n_steps][n_readouts] every readout's signal (may be null)
+    int32_t* out_member;   // [n_steps] nucleus_member per step (may be null)
+    float* out_mass;       // [n_steps] nucleus_mass per step (may be null)
+    const int32_t* forced_in; // [n_steps] teacher-forced inputs (null: the emitted token is fed back)
 };
 
-static_assert(sizeof(Ctl) == 328, "control block size is part of the host read-back accounting");
+static_assert(sizeof(Ctl) == 360, "control block size is part of the host read-back accounting");
 
 // Device pointers and shape, passed by value to every kernel.
 struct DevModel {
@@ -133,13 +139,18 @@ struct VocabArgs {
 
 // Per-call inputs of a graph launch.
 struct CtlInputs {
-    int set_token, in_tok, force, n_steps, dbg, prefill_n, conf_kind;
+    int set_token, in_tok, force, n_steps, dbg, prefill_n, conf_kind, nucleus_on;
+    float nucleus_p;
     float tau[kMaxReadouts];
     const int8_t* sched;
     int32_t* out_tokens;
     int32_t* out_exit;
     float* out_conf;
     const int32_t* prompt;
+    float* out_conf_all;
+    int32_t* out_member;
+    float* out_mass;
+    const int32_t* forced_in;
 };
 
 // Launch helpers (ee_kernels.cu).  Each enqueues one kernel on `s`;
@@ -163,6 +174,10 @@ cudaError_t launch_prefill_advance(const DevModel& m, int has_cond, cudaGraphCon
                                    cudaStream_t s);
 cudaError_t launch_prefill_end(const DevModel& m, bool pdl, cudaStream_t s);
 cudaError_t launch_set_inputs(Ctl* c, const CtlInputs& in, cudaStream_t s);
+// Section 4, step four threshold selection over n (confidence, acceptable)
+// pairs; scratch: 2 device ints.
+cudaError_t launch_select_tau(const float* conf, int stride, const int32_t* member, int n, double target, float* tau,
+                              int* scratch, int n_sm, cudaStream_t s);
 
 // Persistent layer-segment kernel (ee_persist.cu): one CTA per SM, warps
 // 0..7 consume a shared-memory ring that warp 8 fills with cp.async.bulk.

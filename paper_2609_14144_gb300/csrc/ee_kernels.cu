@@ -17,6 +17,7 @@
 // per lane; a warp reduction closes each row.  Units cut by a slice boundary
 // are finished by whichever contributing warp arrives last, summing the
 // contributions in warp order, so results do not depend on timing.
+#include <algorithm>
 #include <cooperative_groups.h>
 #include <cuda_bf16.h>
 #include <math.h>
@@ -537,23 +538,28 @@ struct EpiSwiGLU {
 // the Section 10 alternatives), all from one pass:
 //   m  = max l,  s = sum exp(l - m),  t = sum exp(l - m) (l - m),
 //   m2 = the second largest logit (m again if the maximum is tied),
-//   a  = lowest index attaining m.
+//   a  = lowest index attaining m,
+//   g  = sum exp(l - m) over the rows other than x with l > l_x (the
+//        tokens more probable than a given token x; 0 when x = -1).
 // Then p_max = 1/s, margin = (1 - exp(m2 - m))/s, negative entropy =
-// sum p log p = t/s - log s.
+// sum p log p = t/s - log s, and the probability above x is g/s.
 struct SoftStats {
-    float m, s, t, m2;
+    float m, s, t, m2, g;
     int a;
-    __device__ __forceinline__ SoftStats() : m(-INFINITY), s(0.f), t(0.f), m2(-INFINITY), a(0x7fffffff) {}
-    __device__ __forceinline__ void add(float l, int row) {
+    __device__ __forceinline__ SoftStats() : m(-INFINITY), s(0.f), t(0.f), m2(-INFINITY), g(0.f), a(0x7fffffff) {}
+    __device__ __forceinline__ void add(float l, int row, float lx = INFINITY, int x = -1) {
+        const bool above = l > lx && row != x;
         if (s == 0.f) {
             m = l;
             s = 1.f;
             t = 0.f;
+            g = above ? 1.f : 0.f;
             a = row;
         } else if (l > m) {
             const float dl = m - l, e = expf(dl);
             t = e * (t + dl * s);
             s = s * e + 1.0f;
+            g = above ? fmaf(g, e, 1.0f) : g * e;
             m2 = m;
             m = l;
             a = row;
@@ -561,6 +567,7 @@ struct SoftStats {
             const float dl = l - m, e = expf(dl);
             s += e;
             t = fmaf(e, dl, t);
+            if (above) g += e;
             if (l > m2) m2 = l;
         }
     }
@@ -575,6 +582,7 @@ struct SoftStats {
         const float ea = expf(m - M), eb = expf(o.m - M);
         t = ea * (t + (m - M) * s) + eb * (o.t + (o.m - M) * o.s);
         s = s * ea + o.s * eb;
+        g = g * ea + o.g * eb;
         m2 = fmaxf(fminf(m, o.m), fmaxf(m2, o.m2));
         a = m > o.m ? a : (o.m > m ? o.a : min(a, o.a));
         m = M;
@@ -587,6 +595,7 @@ __device__ __forceinline__ SoftStats shfl_down_stats(const SoftStats& x, int o) 
     y.s = __shfl_down_sync(0xffffffffu, x.s, o);
     y.t = __shfl_down_sync(0xffffffffu, x.t, o);
     y.m2 = __shfl_down_sync(0xffffffffu, x.m2, o);
+    y.g = __shfl_down_sync(0xffffffffu, x.g, o);
     y.a = __shfl_down_sync(0xffffffffu, x.a, o);
     return y;
 }
@@ -670,6 +679,7 @@ __global__ void __launch_bounds__(kGemvThreads, 2) k_qkv(DevModel m, int layer, 
             c->exit_readout = -1;
             c->n_evaluated = 0;
             c->full_token = -1;
+            c->nucleus_member = -1;
             if (!tok_ok) atomicOr(&c->err, kErrTokenRange);
         }
         __syncthreads();
@@ -841,9 +851,12 @@ __global__ void __launch_bounds__(kGemvThreads, 2) k_readout(DevModel m, int r) 
 // (last CTA) of the grid; turn them into the confidence signals and, for a
 // readout, the gate decision signal > tau, which also selects the graph's
 // branch.  The signal is the top-1 probability (Section 2) or, by the
-// context's choice, the margin or the negative entropy (Section 10).
-__device__ __forceinline__ void vocab_finish(const VocabArgs& v, LaneStats st) {
-    __shared__ float sm_m[32], sm_s[32], sm_t[32], sm_m2[32];
+// context's choice, the margin or the negative entropy (Section 10).  With
+// nucleus tracking on, the LM head also reports whether readout 0's token
+// lies in the full model's nucleus (Section 2 acceptance): the probability
+// of the strictly more probable tokens stays below the nucleus share.
+__device__ __forceinline__ void vocab_finish(const VocabArgs& v, LaneStats st, bool nucleus) {
+    __shared__ float sm_m[32], sm_s[32], sm_t[32], sm_m2[32], sm_g[32];
     __shared__ int sm_a[32];
     __shared__ int is_last;
     const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
@@ -853,6 +866,7 @@ __device__ __forceinline__ void vocab_finish(const VocabArgs& v, LaneStats st) {
         sm_s[w] = st.s;
         sm_t[w] = st.t;
         sm_m2[w] = st.m2;
+        sm_g[w] = st.g;
         sm_a[w] = st.a;
     }
     __syncthreads();
@@ -864,6 +878,7 @@ __device__ __forceinline__ void vocab_finish(const VocabArgs& v, LaneStats st) {
             x.s = sm_s[lane];
             x.t = sm_t[lane];
             x.m2 = sm_m2[lane];
+            x.g = sm_g[lane];
             x.a = sm_a[lane];
         }
         warp_merge_stats(x);
@@ -874,6 +889,7 @@ __device__ __forceinline__ void vocab_finish(const VocabArgs& v, LaneStats st) {
             q[2] = x.t;
             q[3] = x.m2;
             reinterpret_cast<int*>(q)[4] = x.a;
+            q[5] = x.g;
             __threadfence();
             is_last = atomicAdd(v.ticket, 1) == (int)gridDim.x - 1;
         }
@@ -890,6 +906,7 @@ __device__ __forceinline__ void vocab_finish(const VocabArgs& v, LaneStats st) {
         y.t = __ldcg(q + 2);
         y.m2 = __ldcg(q + 3);
         y.a = __ldcg(reinterpret_cast<const int*>(q) + 4);
+        y.g = __ldcg(q + 5);
         x.merge(y);
     }
     warp_merge_stats(x);
@@ -932,7 +949,29 @@ __device__ __forceinline__ void vocab_finish(const VocabArgs& v, LaneStats st) {
         c->full_token = a;
         c->full_conf = sig;
         c->exit_readout = -1;
+        if (nucleus) {
+            const float mass = x.g / x.s;
+            c->nucleus_mass = mass;
+            c->nucleus_member = mass < c->nucleus_p ? 1 : 0;
+        }
     }
+}
+
+// The logit of row x of the tiled unembedding, summed in the order the
+// vocabulary pass sums it (chunk by chunk from 0), so the two agree bit for
+// bit.  part: Rc floats of shared memory.  Every thread of the CTA calls it.
+__device__ __forceinline__ float tiled_row_logit(const uint4* W, int64_t x, int Rc, const float* xs, float* part) {
+    __shared__ float lx;
+    const int64_t t = x >> 5, ln = x & 31;
+    for (int c = threadIdx.x; c < Rc; c += blockDim.x) part[c] = dot8(__ldg(W + (t * Rc + c) * 32 + ln), xs + c * 8);
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        float acc = 0.f;
+        for (int c = 0; c < Rc; ++c) acc += part[c];
+        lx = acc;
+    }
+    __syncthreads();
+    return lx;
 }
 
 // One pass over the (tiled) unembedding: z = RMSNorm(x) * gain, l = U z,
@@ -958,6 +997,15 @@ __global__ void __launch_bounds__(kGemvThreads, 2) k_vocab(VocabArgs v) {
     pdl_launch_dependents();
     rmsnorm_to_smem(v.x, v.gain, v.d, v.eps, xs, red);
     const bool keep = v.logits && (!v.logits_if_dbg || (v.ctl && v.ctl->dbg));
+    // nucleus tracking: on full steps, the tokens above readout 0's token
+    const bool nucleus = v.mode == 2 && v.ctl->nucleus_on && v.ctl->n_evaluated > 0;
+    int nx = -1;
+    float lx = INFINITY;
+    if (nucleus) {
+        nx = v.ctl->readout_token[0];
+        if (nx < 0 || nx >= v.V) nx = 0;  // the readout pass flags an out-of-range token
+        lx = tiled_row_logit(W, nx, Rc, xs, xs + ((v.d + 3) & ~3));
+    }
     LaneStats st;
     int64_t t = t0;
     int c = 0;
@@ -976,7 +1024,7 @@ __global__ void __launch_bounds__(kGemvThreads, 2) k_vocab(VocabArgs v) {
                 const int64_t row = t * 32 + lane;
                 if (row < v.V) {
                     if (keep) v.logits[row] = acc;
-                    st.add(acc, (int)row);
+                    st.add(acc, (int)row, lx, nx);
                 }
                 acc = 0.f;
                 c = 0;
@@ -984,7 +1032,7 @@ __global__ void __launch_bounds__(kGemvThreads, 2) k_vocab(VocabArgs v) {
             }
         }
     }
-    vocab_finish(v, st);
+    vocab_finish(v, st, nucleus);
 }
 
 // The same pass over a row-major [V, d] matrix (standalone op): the flat
@@ -1011,7 +1059,7 @@ __global__ void __launch_bounds__(kGemvThreads, 2) k_vocab_rowmajor(VocabArgs v)
     flat_gemv<1, true, 8>(v.U, v.d, v.V, xs, warp, nwarps, nullptr, nullptr, epi);
     // lane 0 holds this warp's statistics; the others hold none
     LaneStats st = (threadIdx.x & 31) == 0 ? epi.st : LaneStats();
-    vocab_finish(v, st);
+    vocab_finish(v, st, false);
 }
 
 // Split-K decode attention over the paged cache.  Grid (splits, KH): CTA
@@ -1387,13 +1435,18 @@ __global__ void k_step_end(DevModel m, int has_cond, cudaGraphConditionalHandle 
     if (c->out_tokens) c->out_tokens[st] = tok;
     if (c->out_exit) c->out_exit[st] = r;
     if (c->out_conf) c->out_conf[st] = conf;
+    if (c->out_conf_all)
+        for (int q = 0; q < m.n_readouts; ++q)
+            c->out_conf_all[(int64_t)st * m.n_readouts + q] = q < c->n_evaluated ? c->conf[q] : NAN;
+    if (c->out_member) c->out_member[st] = c->nucleus_member;
+    if (c->out_mass) c->out_mass[st] = c->nucleus_member >= 0 ? c->nucleus_mass : NAN;
     c->steps += 1;
     if (r >= 0)
         c->exits[r] += 1;
     else
         c->full_steps += 1;
     c->pos += 1;
-    c->in_tok = tok;
+    c->in_tok = (c->forced_in && st + 1 < c->n_steps) ? c->forced_in[st + 1] : tok;
     c->step = st + 1;
     if (has_cond) cudaGraphSetConditional(cond, (c->step < c->n_steps && c->err == 0) ? 1u : 0u);
 }
@@ -1420,6 +1473,7 @@ __global__ void k_prefill_end(DevModel m) {
     c->in_tok = c->token;
     c->exit_readout = -1;
     c->n_evaluated = 0;
+    c->nucleus_member = -1;
 }
 
 // Per-call inputs written into the control block ahead of a graph launch.
@@ -1431,6 +1485,12 @@ __global__ void k_set_inputs(Ctl* c, CtlInputs in) {
     c->n_steps = in.n_steps;
     c->dbg = in.dbg;
     c->conf_kind = in.conf_kind;
+    c->nucleus_on = in.nucleus_on;
+    c->nucleus_p = in.nucleus_p;
+    c->out_conf_all = in.out_conf_all;
+    c->out_member = in.out_member;
+    c->out_mass = in.out_mass;
+    c->forced_in = in.forced_in;
     for (int r = 0; r < kMaxReadouts; ++r) c->tau[r] = in.tau[r];
     c->sched = in.sched;
     c->out_tokens = in.out_tokens;
@@ -1441,6 +1501,77 @@ __global__ void k_set_inputs(Ctl* c, CtlInputs in) {
         c->prefill_i = 0;
         c->prompt = in.prompt;
     }
+}
+
+// Threshold selection (Section 4, step four).  Each thread takes one
+// candidate threshold (-inf, then each observed confidence), counts the
+// early positions (conf > candidate) and the acceptable ones among them over
+// all n positions, staged through shared memory, and offers the candidate to
+// a grid-wide minimum if good >= target * early.  Floats are ordered through
+// their bit patterns (negative values with the magnitude bits flipped), so
+// the minimum is an integer atomicMin.
+constexpr int kTauThreads = 256, kTauTile = 2048;
+
+__device__ __forceinline__ int float_key(float f) {
+    const int b = __float_as_int(f);
+    return b >= 0 ? b : b ^ 0x7fffffff;
+}
+__device__ __forceinline__ float key_float(int k) { return __int_as_float(k >= 0 ? k : k ^ 0x7fffffff); }
+
+__global__ void k_tau_init(int* scratch) {
+    if (threadIdx.x == 0) {
+        scratch[0] = float_key(INFINITY);
+        scratch[1] = 0;
+    }
+}
+
+__global__ void __launch_bounds__(kTauThreads) k_select_tau(const float* conf, int stride, const int32_t* member,
+                                                             int n, double target, float* tau, int* scratch) {
+    __shared__ float sc[kTauTile];
+    __shared__ unsigned char sg[kTauTile];
+    __shared__ int is_last;
+    const int64_t n_cand = (int64_t)n + 1;
+    const int64_t per_pass = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t base = 0; base < n_cand; base += per_pass) {
+        const int64_t ci = base + (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+        const bool have = ci < n_cand;
+        const float cand = !have ? INFINITY : (ci == 0 ? -INFINITY : conf[(ci - 1) * stride]);
+        int early = 0, good = 0;
+        for (int i0 = 0; i0 < n; i0 += kTauTile) {
+            const int len = min(kTauTile, n - i0);
+            __syncthreads();
+            for (int i = threadIdx.x; i < len; i += blockDim.x) {
+                sc[i] = conf[(int64_t)(i0 + i) * stride];
+                sg[i] = member[i0 + i] != 0;
+            }
+            __syncthreads();
+            for (int i = 0; i < len; ++i) {
+                const int e = sc[i] > cand;
+                early += e;
+                good += e & sg[i];
+            }
+        }
+        if (have && early > 0 && (double)good >= target * (double)early) atomicMin(&scratch[0], float_key(cand));
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        __threadfence();
+        is_last = atomicAdd(&scratch[1], 1) == (int)gridDim.x - 1;
+    }
+    __syncthreads();
+    if (is_last && threadIdx.x == 0) {
+        __threadfence();
+        *tau = key_float(atomicAdd(&scratch[0], 0));
+    }
+}
+
+cudaError_t launch_select_tau(const float* conf, int stride, const int32_t* member, int n, double target, float* tau,
+                              int* scratch, int n_sm, cudaStream_t s) {
+    const int64_t want = ((int64_t)n + 1 + kTauThreads - 1) / kTauThreads;
+    const int grid = (int)std::min<int64_t>(want, (int64_t)4 * std::max(n_sm, 1));
+    k_tau_init<<<1, 32, 0, s>>>(scratch);
+    k_select_tau<<<grid, kTauThreads, 0, s>>>(conf, stride, member, n, target, tau, scratch);
+    return cudaGetLastError();
 }
 
 // ------------------------------------------------------------------ launchers
@@ -1534,7 +1665,8 @@ cudaError_t launch_readout(const DevModel& m, int r, int grid, bool whole, bool 
     return launch_k(k_readout<false>, dim3(grid), dim3(kGemvThreads), sm, pdl, s, m, r);
 }
 cudaError_t launch_vocab(const VocabArgs& v, int grid, bool pdl, cudaStream_t s) {
-    const size_t smem = (size_t)((v.d + 3) & ~3) * sizeof(float);
+    // x, then (LM head) the chunk partials of one row's logit
+    const size_t smem = ((size_t)((v.d + 3) & ~3) + (size_t)(v.d / 8)) * sizeof(float);
     if (v.tiled) return launch_k(k_vocab, dim3(grid), dim3(kGemvThreads), smem, pdl, s, v);
     return launch_k(k_vocab_rowmajor, dim3(grid), dim3(kGemvThreads), smem, pdl, s, v);
 }

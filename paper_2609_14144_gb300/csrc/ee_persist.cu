@@ -750,6 +750,7 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
             c->exit_readout = -1;
             c->n_evaluated = 0;
             c->full_token = -1;
+            c->nucleus_member = -1;
         }
     }
     csync();

@@ -24,6 +24,23 @@ def bf16_round(a) -> np.ndarray:
     return torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(torch.bfloat16).float().numpy()
 
 
+def bf16_bits_to_f32(a) -> np.ndarray:
+    return (np.ascontiguousarray(a, dtype=np.uint16).astype(np.uint32) << 16).view(np.float32)
+
+
+def damped_after_readout(shape, model: dict, alpha: float) -> dict:
+    """The model with the output and down projections of every layer from the
+    first readout on scaled by alpha: at alpha = 0 the final residual equals
+    the readout layer's, so the readout's answers mostly fall inside the full
+    model's nucleus and calibration sees both outcomes."""
+    m = dict(model)
+    m["layers"] = [dict(l) for l in model["layers"]]
+    for j in range(min(shape.readout_layers), shape.n_layers):
+        for k in ("wo", "wd"):
+            m["layers"][j][k] = to_bf16_bits(bf16_bits_to_f32(model["layers"][j][k]) * alpha)
+    return m
+
+
 def zeros_like_bits(a) -> np.ndarray:
     return np.zeros_like(np.asarray(a, dtype=np.uint16))
 
@@ -60,6 +77,27 @@ def is_excluded(o: dict, taus) -> bool:
     return (not o["exited"]) and o["full_gap"] < EXCLUDE_EPS
 
 
+NUC_EPS = 1e-3   # exclusion band on |mass - p_nuc|
+MASS_TOL = 2e-3  # |mass_gpu - mass_oracle| outside the ambiguous tokens
+
+
+def nucleus_ambiguity(final_logits, x: int, p_nuc: float, mass: float):
+    """(excluded, bound) for a nucleus check of token x.  Tokens whose logit
+    lies within rounding distance of l_x (1e-3 of the largest logit) may fall
+    on either side of it; bound is their total probability, by which the
+    GPU's mass may differ.  The step is excluded from the bit-exact
+    membership check when the oracle's mass lies within NUC_EPS + bound of
+    the nucleus share."""
+    l = np.asarray(final_logits, np.float64)
+    p = np.exp(l - l.max())
+    p /= p.sum()
+    delta = 1e-3 * max(1.0, float(np.abs(l).max()))
+    near = np.abs(l - l[x]) < delta
+    near[x] = False
+    bound = float(p[near].sum())
+    return abs(mass - p_nuc) < NUC_EPS + bound, bound
+
+
 def forced(o: dict) -> int:
     from paper_2609_14144_gb300 import FORCE_EXIT_AT, FORCE_FULL
     return FORCE_EXIT_AT(o["exit_readout"]) if o["exited"] else FORCE_FULL
@@ -67,12 +105,13 @@ def forced(o: dict) -> int:
 
 def teacher_forced(shape, model, n: int, taus, *, prompt=None, capture: bool = True, graphs: bool = True,
                    pdl: bool = True, persistent: bool = True, page_perm=None, page_size: int = 64,
-                   conf_kind: int = 0):
+                   conf_kind: int = 0, nucleus_permille: int = 0):
     """Run the oracle free and the GPU engine teacher-forced on the oracle's
     input tokens and exit decisions.  Returns (first_o, first_g, records,
     oracle, engine)."""
     import oracle
-    from paper_2609_14144_gb300 import OPT_CONFIDENCE, OPT_DEBUG_LOGITS, OPT_GRAPHS, OPT_PDL, OPT_PERSISTENT, Engine
+    from paper_2609_14144_gb300 import (OPT_CONFIDENCE, OPT_DEBUG_LOGITS, OPT_GRAPHS, OPT_NUCLEUS, OPT_PDL,
+                                        OPT_PERSISTENT, Engine)
 
     prompt = synth.prompt(shape) if prompt is None else np.asarray(prompt, np.int32)
     max_ctx = len(prompt) + n
@@ -84,6 +123,9 @@ def teacher_forced(shape, model, n: int, taus, *, prompt=None, capture: bool = T
     eng.set_option(OPT_PERSISTENT, 1 if persistent else 0)
     eng.set_option(OPT_CONFIDENCE, conf_kind)
     eng.set_option(OPT_DEBUG_LOGITS, capture)
+    if nucleus_permille:
+        orc.set_nucleus(nucleus_permille / 1000.0)
+        eng.set_option(OPT_NUCLEUS, nucleus_permille)
     if page_perm is not None:
         eng.set_page_table(page_perm)
     first_o = orc.prefill(prompt)
