@@ -308,13 +308,12 @@ struct Smem {
     uint64_t* full;     // [stages]
     uint64_t* empty;    // [stages]
     float* xs;          // [max(d, A D)] input vector of a whole-tile phase
-    float* hs;          // [d] residual
     float* xa;          // [max items][512] staged input columns of the O / down items, then
                         // [max items][32] residual rows of the O items of chunk 0
     float2* rope;       // [D/2] (cos, sin) of the step's position
     uint16_t* ga;       // [d] attention-norm gain of the current layer
     uint16_t* gm;       // [d] MLP-norm gain of the current layer
-    float* red;         // [2][kCW][32]
+    float* red;         // [2][kCW][32], then [kCW] sums of squares of the RMSNorm
     float* qa;          // [group][D] scaled queries of the attention unit
     float* kv;          // [2][D] k, v of the step's position
     float* sc;          // [group][pps * page_size] scores, then probabilities
@@ -334,8 +333,6 @@ __device__ __forceinline__ Smem carve(uint8_t* base, const DevModel& m, const Se
     float* f = reinterpret_cast<float*>(q);
     s.xs = f;
     f += (max(m.d, m.A * m.D) + 3) & ~3;
-    s.hs = f;
-    f += (m.d + 3) & ~3;
     s.xa = f;
     f += p.max_items * (kColsPerChunk + 32);
     s.rope = reinterpret_cast<float2*>(f);
@@ -345,7 +342,7 @@ __device__ __forceinline__ Smem carve(uint8_t* base, const DevModel& m, const Se
     s.gm = reinterpret_cast<uint16_t*>(f);
     f += (m.d + 1) / 2;
     s.red = f;
-    f += 2 * kCW * 32;
+    f += 2 * kCW * 32 + kCW;
     const int grp = m.A / m.KH;
     s.qa = f;
     f += grp * m.D;
@@ -469,16 +466,24 @@ __device__ __forceinline__ bool wait_count(const unsigned* cnt, unsigned target,
     csync();
     return ok_s != 0;
 }
-// All consumer threads' global writes, then one release increment: the
+// All consumer threads' global writes, then one release increment.  The
 // consumer barrier orders the other threads' writes before thread 0's
-// fence and release (the pattern of a cooperative grid barrier).
+// release, and a release is cumulative over what its thread has observed,
+// so no separate fence is needed (a reader pairs it with ld.acquire).
 __device__ __forceinline__ void signal_count(unsigned* cnt) {
     csync();
-    if (threadIdx.x == 0) {
-        __threadfence();
-        asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(cnt) : "memory");
-    }
+    if (threadIdx.x == 0) asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(cnt) : "memory");
 }
+
+// Asynchronous copy of n bf16 values (n a multiple of 8, both addresses
+// 16-byte aligned) into shared memory; complete once every consumer thread
+// has passed cp_async_wait() and a consumer barrier.
+__device__ __forceinline__ void copy_async(uint16_t* dst, const uint16_t* src, int n) {
+    for (int i = threadIdx.x; i < (n >> 3); i += kCT)
+        asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(saddr(dst + 8 * i)), "l"(src + 8 * i) : "memory");
+    asm volatile("cp.async.commit_group;" ::: "memory");
+}
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_all;" ::: "memory"); }
 
 // dst[i] = f(i) for i < n, eight elements per thread per round with all their
 // loads issued before any store (f reads global memory).
@@ -519,20 +524,40 @@ __device__ __forceinline__ float4 bf4(const uint16_t* p) {
     return make_float4(bflo(u.x), bfhi(u.x), bflo(u.y), bfhi(u.y));
 }
 
-// RMSNorm of hs (d values) times gain g into xs (consumer threads).
-__device__ __forceinline__ void rmsnorm_sm(const float* hs, const uint16_t* g, int d, float eps, float* xs,
-                                           float* red) {
-    const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+// RMSNorm folded into the gather of its input: xs = h * g (d values, h
+// from f four at a time) and the return value 1 / sqrt(mean(h^2) + eps), the
+// factor the projection's epilogue applies to each row's dot product
+// (W (h * g) / rms = W (RMSNorm(h) * g)).  One consumer barrier; nss: [kCW]
+// floats of shared memory not otherwise in use until the next call.
+template <class F>
+__device__ __forceinline__ float gather_norm(float* xs, const uint16_t* g, int d, float eps, float* nss, F f) {
+    const int n4 = d >> 2;
+    float4* x4 = reinterpret_cast<float4*>(xs);
     float ss = 0.f;
-    for (int i = threadIdx.x; i < d; i += kCT) ss = fmaf(hs[i], hs[i], ss);
+    for (int b = threadIdx.x; b < n4; b += 8 * kCT) {
+        float4 v[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) v[e] = (b + e * kCT < n4) ? f(4 * (b + e * kCT)) : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            const int k = b + e * kCT;
+            if (k < n4) {
+                ss = fmaf(v[e].x, v[e].x, ss);
+                ss = fmaf(v[e].y, v[e].y, ss);
+                ss = fmaf(v[e].z, v[e].z, ss);
+                ss = fmaf(v[e].w, v[e].w, ss);
+                const uint2 gu = *reinterpret_cast<const uint2*>(g + 4 * k);
+                x4[k] = make_float4(v[e].x * bflo(gu.x), v[e].y * bfhi(gu.x), v[e].z * bflo(gu.y), v[e].w * bfhi(gu.y));
+            }
+        }
+    }
     ss = warp_sum(ss);
-    if (l == 0) red[w] = ss;
+    if ((threadIdx.x & 31) == 0) nss[threadIdx.x >> 5] = ss;
     csync();
-    float t = l < kCW ? red[l] : 0.f;
-    t = warp_sum(t);
-    const float inv = 1.0f / sqrtf(t / (float)d + eps);
-    for (int i = threadIdx.x; i < d; i += kCT) xs[i] = hs[i] * inv * bf(g[i]);
-    csync();
+    float t = 0.f;
+#pragma unroll
+    for (int k = 0; k < kCW; ++k) t += nss[k];
+    return 1.0f / sqrtf(t / (float)d + eps);
 }
 
 // Whole tiles [t0, t1) of a matrix with rows of length K against x (all K
@@ -753,6 +778,10 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
             c->nucleus_member = -1;
         }
     }
+    // the first layer's norm gains; later layers' are copied once the
+    // previous layer no longer reads them
+    copy_async(s.ga, m.layers + (int64_t)j0 * m.layer_stride + m.off_gattn, m.d);
+    copy_async(s.gm, m.layers + (int64_t)j0 * m.layer_stride + m.off_gmlp, m.d);
     csync();
     int rb = 0;
 
@@ -763,30 +792,24 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
         float* op_cur = opart_of(p, j);
         const ResidIn rin{&p, (j == j0 && first) ? m.embed + (int64_t)tok * m.d : nullptr, j == j0 ? m.h : nullptr,
                           opart_of(p, j - 1), s.nsd};
-        {   // this layer's norm gains, ahead of the waits
-            const uint32_t* g1 = reinterpret_cast<const uint32_t*>(lw + m.off_gattn);
-            const uint32_t* g2 = reinterpret_cast<const uint32_t*>(lw + m.off_gmlp);
-            uint32_t* d1 = reinterpret_cast<uint32_t*>(s.ga);
-            uint32_t* d2 = reinterpret_cast<uint32_t*>(s.gm);
-            for (int i = threadIdx.x; i < m.d / 2; i += kCT) {
-                const uint32_t a1 = g1[i], a2 = g2[i];
-                d1[i] = a1;
-                d2[i] = a2;
-            }
-        }
+        const uint16_t* lw_next = lw + m.layer_stride;
 
         // ---------------- Q/K/V tiles: RMSNorm, projection, bias, RoPE, KV append
         if (tq1 > tq0) {
-            if (j > j0 && !wait_count(cnt - kPhases + kPhDn, G, err)) return;
-            gather4(s.hs, m.d, [&](int i) { return rin.four(i); });
-            csync();
-            rmsnorm_sm(s.hs, s.ga, m.d, m.eps, s.xs, s.red);
+            cp_async_wait();  // this layer's attention-norm gain
+            if (j > j0) {
+                if (!wait_count(cnt - kPhases + kPhDn, G, err)) return;
+            } else {
+                csync();
+            }
+            const float inv = gather_norm(s.xs, s.ga, m.d, m.eps, s.red + 2 * kCW * 32, [&](int i) { return rin.four(i); });
             const uint16_t* bias = m.qkv_bias ? lw + m.off_bqkv : nullptr;
             uint16_t* kdst = m.kpool + (int64_t)j * m.kv_layer_stride + kvo_pos;
             uint16_t* vdst = m.vpool + (int64_t)j * m.kv_layer_stride + kvo_pos;
             tile_gemv(cs, tq0, tq1, p.K[0], p.n_chunks[0], s.xs, s.red, rb, [&](int t, float v) {
                 const int odd = lane & 1;
                 const int u = t * 16 + (lane >> 1);
+                v *= inv;
                 if (bias) v += bf(bias[2 * u + odd]);
                 const float other = __shfl_xor_sync(0xffffffffu, v, 1);
                 const float r0 = odd ? other : v, r1 = odd ? v : other;
@@ -817,6 +840,10 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
         }
         if (cta == 0 && threadIdx.x == 0) m.kv_src[(int64_t)j * m.max_ctx + pos] = 1;
         signal_count(cnt + kPhQKV);
+        if (j + 1 < j1) {  // the next layer's attention-norm gain (this layer's was read above)
+            cp_async_wait();
+            copy_async(s.ga, lw_next + m.off_gattn, m.d);
+        }
 
         // ---------------- attention unit (if this CTA has one)
         if (unit >= 0) {
@@ -1082,17 +1109,22 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
 
         // ---------------- gate/up tiles: RMSNorm of the mid residual, SwiGLU
         if (tg1 > tg0) {
+            cp_async_wait();  // this layer's MLP-norm gain
             if (!wait_count(cnt + kPhO, G, err)) return;
-            gather4(s.hs, m.d, [&](int i) { return resid_mid4(p, op_cur, i); });
-            csync();
-            rmsnorm_sm(s.hs, s.gm, m.d, m.eps, s.xs, s.red);
+            const float inv = gather_norm(s.xs, s.gm, m.d, m.eps, s.red + 2 * kCW * 32,
+                                          [&](int i) { return resid_mid4(p, op_cur, i); });
             tile_gemv(cs, tg0, tg1, p.K[2], p.n_chunks[2], s.xs, s.red, rb, [&](int t, float v) {
+                v *= inv;
                 const float up = __shfl_xor_sync(0xffffffffu, v, 1);
                 const int f = t * 16 + (lane >> 1);
                 if (!(lane & 1) && f < m.F) m.a[f] = v / (1.0f + expf(-v)) * up;
             });
         }
         signal_count(cnt + kPhGU);
+        if (j + 1 < j1) {  // the next layer's MLP-norm gain
+            cp_async_wait();
+            copy_async(s.gm, lw_next + m.off_gmlp, m.d);
+        }
 
         // ---------------- down items: partial slots of h_out - h_mid
         if (idn.hi > idn.lo) {
@@ -1131,6 +1163,7 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
     }
 
     // ---------------- the segment's output residual, then the exit ticket
+    cp_async_wait();
     if (!wait_count(sync + (j1 - 1 - j0) * kPhases + kPhDn, G, err)) return;
     {
         const ResidIn rout{&p, nullptr, nullptr, opart_of(p, j1 - 1), s.nsd};
@@ -1176,8 +1209,8 @@ bool seg_plan(const DevModel& m, int n_sm, SegPlan& p) {
     const int cap = std::max(1, std::min(kSegMaxSplits, p.G / m.KH));
     const int np_max = (m.max_ctx + m.page_size - 1) / m.page_size;
     p.max_pps = std::max(1, (np_max + cap - 1) / cap);
-    const size_t floats = (size_t)((std::max(m.d, m.A * m.D) + 3) & ~3) + ((m.d + 3) & ~3) +
-                          (size_t)p.max_items * (kColsPerChunk + 32) + (size_t)m.D + (size_t)m.d + 2 * kCW * 32 + (size_t)grp * m.D + 2 * (size_t)m.D +
+    const size_t floats = (size_t)((std::max(m.d, m.A * m.D) + 3) & ~3) +
+                          (size_t)p.max_items * (kColsPerChunk + 32) + (size_t)m.D + (size_t)m.d + 2 * kCW * 32 + kCW + (size_t)grp * m.D + 2 * (size_t)m.D +
                           (size_t)grp * p.max_pps * m.page_size + 2 * (size_t)grp + (size_t)m.A * (kSegMaxSplits + 1);
     const size_t fixed = floats * 4 + (size_t)p.n_tiles[3] + 256;
     const size_t budget = 227 * 1024;
