@@ -58,7 +58,7 @@ struct Layout {
     size_t ctl, rope, layers, embed, lm_head, g_final, ro_w[kMaxReadouts], ro_b[kMaxReadouts];
     size_t kpool, vpool, page_table, kv_src, h, q, o, a, y, hk, logits_ro, logits_final;
     size_t gemv_part, gemv_ticket, attn_part, attn_ticket, vocab_part, vocab_ticket;
-    size_t seg_dpart, seg_opart, seg_sync;
+    size_t seg_dpart, seg_opart, seg_q, seg_kvn, seg_a, seg_attn, seg_sync, seg_end;
     size_t prompt, sched, out_tok, out_exit, out_conf, out_conf_all, out_member, out_mass, tau_scratch, total;
     int64_t layer_stride, off_wqkv, off_bqkv, off_gattn, off_wo, off_gmlp, off_wgu, off_wd;
     int64_t n_units_qkv, kv_layer_stride, gemv_ticket_stride;
@@ -154,7 +154,12 @@ Layout make_layout(const ee_model_config& c) {
         l.seg_dpart = take(4 * (size_t)tile_count(d) * ((F + cols - 1) / cols) * kTileRows);
         l.seg_opart = take(2 * 4 * (size_t)tile_count(d) * ((A * D + cols - 1) / cols) * kTileRows);
     }
-    l.seg_sync = take(4 * (size_t)(5 * L + 8));
+    l.seg_q = take(4 * (size_t)A * D);
+    l.seg_kvn = take(4 * 2 * (size_t)KH * D);
+    l.seg_a = take(4 * (size_t)F);
+    l.seg_attn = take(4 * (size_t)A * kSegMaxSplits * (D + 4));
+    l.seg_sync = take(4 * 8);
+    l.seg_end = b;
     l.prompt = take(4 * (size_t)c.max_ctx);
     l.sched = take((size_t)c.max_ctx);
     l.out_tok = take(4 * (size_t)c.max_ctx);
@@ -710,8 +715,11 @@ int ee_create(const ee_model_config* cfg, void* d_workspace, size_t workspace_by
     if (seg_plan(m, c->n_sm, c->seg) && configure_layers(c->seg.smem) == cudaSuccess &&
         layers_blocks_per_sm(c->seg.smem) >= 1) {
         c->seg.dpart = (float*)(w + l.seg_dpart);
-        c->seg.attn_part = m.attn_part;
         c->seg.opart = (float*)(w + l.seg_opart);
+        c->seg.attn_part = (float*)(w + l.seg_attn);
+        c->seg.q = (float*)(w + l.seg_q);
+        c->seg.kvn = (float*)(w + l.seg_kvn);
+        c->seg.a = (float*)(w + l.seg_a);
         c->seg.sync = (unsigned*)(w + l.seg_sync);
         c->seg_ok = true;
     }
@@ -872,8 +880,9 @@ int ee_reset(ee_ctx* c) {
     c->h_ctl->max_ctx = c->cfg.max_ctx;
     EE_CK(cudaMemcpyAsync(c->d_ctl, c->h_ctl, sizeof(Ctl), cudaMemcpyHostToDevice, c->stream));
     EE_CK(cudaMemsetAsync(c->ws + c->lay.kv_src, 0, (size_t)c->cfg.n_layers * c->cfg.max_ctx, c->stream));
-    // phase counters of the persistent layer kernel (left set by a timed-out wait)
-    EE_CK(cudaMemsetAsync(c->ws + c->lay.seg_sync, 0, 4 * (size_t)(5 * c->cfg.n_layers + 8), c->stream));
+    // the persistent layer kernel's exchange buffers (tags 0: never valid),
+    // exit ticket and launch count
+    EE_CK(cudaMemsetAsync(c->ws + c->lay.seg_dpart, 0, c->lay.seg_end - c->lay.seg_dpart, c->stream));
     EE_CK(cudaStreamSynchronize(c->stream));
     c->pos = 0;
     c->prefilled = false;

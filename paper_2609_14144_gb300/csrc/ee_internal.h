@@ -195,10 +195,15 @@ struct SegPlan {
     int rows_per_kv_chunk;  // cache positions per ring chunk
     int max_items;          // O / down-projection items per CTA (at most)
     int n_tiles[4], n_chunks[4], K[4];  // Q/K/V, O, gate/up, down
+    // Values handed between CTAs, each float carrying its layer's tag in
+    // the low mantissa bits (zero after ee_reset):
     float* dpart;           // down-projection partials [tile][n_chunks][32]
     float* opart;           // O-projection chunk partials [2][tile][n_chunks][32] (by layer parity)
     float* attn_part;       // [A][kSegMaxSplits][D + 4]: unnormalised o, max, sum per split
-    unsigned* sync;         // [5 L + 1] phase counters and the exit ticket, zero between launches
+    float* q;               // [A D] rotated queries
+    float* kvn;             // [2][KH D] the step's k and v (bf16 values)
+    float* a;               // [F] SwiGLU product
+    unsigned* sync;         // [0] exit ticket (zero between launches), [1] launches since ee_reset
     size_t smem;            // dynamic shared memory per CTA
 };
 // Geometry and shared-memory plan for `m` on n_sm SMs (pointers left

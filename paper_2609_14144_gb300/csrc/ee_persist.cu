@@ -54,7 +54,6 @@ constexpr int kCCPerWarp = (kColsPerChunk / 8 + kCW - 1) / kCW;  // 16-byte colu
 constexpr long long kStallCycles = 4000000000ll;  // about 2 s
 constexpr long long kCheckCycles = 2000000ll;     // about 1 ms
 
-enum { kPhQKV = 0, kPhAttn = 1, kPhO = 2, kPhGU = 3, kPhDn = 4, kPhases = 5 };
 
 __device__ __forceinline__ float bf(uint16_t b) { return __uint_as_float((uint32_t)b << 16); }
 __device__ __forceinline__ float bflo(uint32_t v) { return __uint_as_float(v << 16); }
@@ -441,39 +440,89 @@ struct Consumer {
     }
 };
 
-// Wait (one thread) until counter >= target, then sync the consumers.  False
-// on a stall (flagged in the control block).
-__device__ __forceinline__ bool wait_count(const unsigned* cnt, unsigned target, volatile int* err) {
-    __shared__ int ok_s;
-    if (threadIdx.x == 0) {
-        int ok = 1;
-        unsigned v;
-        asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(cnt) : "memory");
-        if (v < target) {
+// ------------------------------------------------------------ tagged values
+// A value one CTA hands to another within a launch carries a tag in its 5
+// lowest mantissa bits: 16 | (seq mod 16), seq counting the layers run
+// since the context was reset (over all launches).  Readers load it with
+// strong loads until the tag is the expected one, so a phase needs no
+// completion counter and its writers no fence: a 32-bit word is observed
+// whole.  The value is first rounded to 19 significant bits (a bf16 value
+// stays exact).  Every word a layer reads is written by every layer (the O
+// slots by every other layer, into the buffer of seq's parity), so before
+// it receives the value of seq it holds the one of seq - 1 or seq - 2, whose
+// tags differ; attention partials of splits a launch does not use are set
+// to 0, which equals no tag, as is every word after a reset.  The readers
+// of a word are done with it before it is written again: every later write
+// depends, through the values it is computed from, on all of them.
+__device__ __forceinline__ uint32_t seq_tag(unsigned seq) { return 16u | (seq & 15u); }
+__device__ __forceinline__ void st_tagged(float* p, float v, uint32_t tag) {
+    const uint32_t b = ((__float_as_uint(v) + 16u) & ~31u) | tag;
+    asm volatile("st.relaxed.gpu.global.b32 [%0], %1;" ::"l"(p), "r"(b) : "memory");
+}
+__device__ __forceinline__ uint32_t ld_strong(const float* p) {
+    uint32_t r;
+    asm volatile("ld.relaxed.gpu.global.b32 %0, [%1];" : "=r"(r) : "l"(p) : "memory");
+    return r;
+}
+__device__ __forceinline__ uint4 ld_strong4(const float* p) {
+    uint4 r;
+    asm volatile("ld.relaxed.gpu.global.v4.b32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+                 : "l"(p)
+                 : "memory");
+    return r;
+}
+__device__ __forceinline__ float untag(uint32_t b) { return __uint_as_float(b & ~31u); }
+__device__ __forceinline__ float4 untag4(uint4 v) { return make_float4(untag(v.x), untag(v.y), untag(v.z), untag(v.w)); }
+// Nonzero if any of the four tags differs from `tag`.
+__device__ __forceinline__ uint32_t mismatch4(uint4 v, uint32_t tag) {
+    return ((v.x ^ tag) | (v.y ^ tag) | (v.z ^ tag) | (v.w ^ tag)) & 31u;
+}
+
+// One thread's bounded waits for tagged values.  After a wait has run out
+// (kErrStall set) the later ones return zeros at once, so the launch still
+// ends; the host reports the stall.
+struct Poll {
+    volatile int* err;
+    bool failed;
+    __device__ explicit Poll(volatile int* e) : err(e), failed(false) {}
+    __device__ __forceinline__ float wait1(const float* p, uint32_t tag) {
+        if (!failed) {
             Bound bd;
             for (;;) {
-                asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(cnt) : "memory");
-                if (v >= target) break;
-                if (bd.expired(err)) {
-                    atomicOr((int*)err, kErrStall);
-                    ok = 0;
-                    break;
-                }
+                __nanosleep(64);
+                const uint32_t b = ld_strong(p);
+                if (((b ^ tag) & 31u) == 0) return untag(b);
+                if (bd.expired(err)) break;
             }
+            atomicOr((int*)err, kErrStall);
+            failed = true;
         }
-        ok_s = ok;
+        return 0.f;
     }
-    csync();
-    return ok_s != 0;
-}
-// All consumer threads' global writes, then one release increment.  The
-// consumer barrier orders the other threads' writes before thread 0's
-// release, and a release is cumulative over what its thread has observed,
-// so no separate fence is needed (a reader pairs it with ld.acquire).
-__device__ __forceinline__ void signal_count(unsigned* cnt) {
-    csync();
-    if (threadIdx.x == 0) asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(cnt) : "memory");
-}
+    // Between two rounds of loads of values not all written yet: false once
+    // the wait has run out (kErrStall set; the caller keeps what it has).
+    __device__ __forceinline__ bool again(Bound& bd) {
+        if (failed) return false;
+        __nanosleep(64);
+        if (!bd.expired(err)) return true;
+        atomicOr((int*)err, kErrStall);
+        failed = true;
+        return false;
+    }
+    // One thread waits until the word at p carries `tag` (loads a little
+    // apart), then the consumer warps sync.  p is one of the phase's inputs:
+    // once it has arrived the others mostly have too, so the gather that
+    // follows finds them written and few threads poll.
+    __device__ __forceinline__ void probe(const float* p, uint32_t tag) {
+        if (threadIdx.x == 0) (void)get(p, tag);
+        csync();
+    }
+    __device__ __forceinline__ float get(const float* p, uint32_t tag) {
+        const uint32_t b = ld_strong(p);
+        return ((b ^ tag) & 31u) == 0 ? untag(b) : wait1(p, tag);
+    }
+};
 
 // Asynchronous copy of n bf16 values (n a multiple of 8, both addresses
 // 16-byte aligned) into shared memory; complete once every consumer thread
@@ -485,31 +534,46 @@ __device__ __forceinline__ void copy_async(uint16_t* dst, const uint16_t* src, i
 }
 __device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_all;" ::: "memory"); }
 
-// dst[i] = f(i) for i < n, eight elements per thread per round with all their
-// loads issued before any store (f reads global memory).
+// Reload the elements of a gather round whose tags were not yet all the
+// expected ones, every such element's loads issued together, until none is
+// left (or the wait has run out).
 template <class F>
-__device__ __forceinline__ void gather(float* dst, int n, F f) {
-    for (int b = threadIdx.x; b < n; b += 8 * kCT) {
-        float v[8];
+__device__ __forceinline__ void retry8(Poll& pl, int b, int n4, float4 (&v)[8], uint32_t (&bad)[8], F f) {
+    uint32_t any = 0;
 #pragma unroll
-        for (int e = 0; e < 8; ++e) v[e] = (b + e * kCT < n) ? f(b + e * kCT) : 0.f;
+    for (int e = 0; e < 8; ++e) any |= bad[e];
+    if (!any) return;
+    Bound bd;
+    while (pl.again(bd)) {
+        any = 0;
 #pragma unroll
         for (int e = 0; e < 8; ++e)
-            if (b + e * kCT < n) dst[b + e * kCT] = v[e];
+            if (bad[e]) {
+                bad[e] = 0;
+                v[e] = f(4 * (b + e * kCT), bad[e]);
+                any |= bad[e];
+            }
+        if (!any) return;
     }
 }
 
-// The same with four consecutive elements per call (n and dst 4-aligned):
-// f(i) returns elements i..i+3 as one float4, so a warp's loads are 16 bytes
-// per lane and a thread has fewer of them in flight.
+// dst[i..i+3] = f(i) for i < n (n and dst 4-aligned), eight float4 per
+// thread per round with all their loads issued before any store.  f(i, bad)
+// loads once and ORs a nonzero value into bad if a tag was not yet the
+// expected one; such elements are loaded again (retry8).
 template <class F>
-__device__ __forceinline__ void gather4(float* dst, int n, F f) {
+__device__ __forceinline__ void gather4(float* dst, int n, Poll& pl, F f) {
     const int n4 = n >> 2;
     float4* d4 = reinterpret_cast<float4*>(dst);
     for (int b = threadIdx.x; b < n4; b += 8 * kCT) {
         float4 v[8];
+        uint32_t bad[8];
 #pragma unroll
-        for (int e = 0; e < 8; ++e) v[e] = (b + e * kCT < n4) ? f(4 * (b + e * kCT)) : make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int e = 0; e < 8; ++e) {
+            bad[e] = 0;
+            v[e] = (b + e * kCT < n4) ? f(4 * (b + e * kCT), bad[e]) : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+        retry8(pl, b, n4, v, bad, f);
 #pragma unroll
         for (int e = 0; e < 8; ++e)
             if (b + e * kCT < n4) d4[b + e * kCT] = v[e];
@@ -519,6 +583,11 @@ __device__ __forceinline__ float4 f4add(float4 a, float4 b) {
     return make_float4(a.x + b.x, a.y + b.y, a.z + b.z, a.w + b.w);
 }
 __device__ __forceinline__ float4 ldg4(const float* p) { return *reinterpret_cast<const float4*>(p); }
+// a + the untagged v, noting a tag mismatch in bad
+__device__ __forceinline__ float4 add_tagged(float4 a, uint4 v, uint32_t tag, uint32_t& bad) {
+    bad |= mismatch4(v, tag);
+    return f4add(a, untag4(v));
+}
 __device__ __forceinline__ float4 bf4(const uint16_t* p) {
     const uint2 u = *reinterpret_cast<const uint2*>(p);
     return make_float4(bflo(u.x), bfhi(u.x), bflo(u.y), bfhi(u.y));
@@ -530,14 +599,19 @@ __device__ __forceinline__ float4 bf4(const uint16_t* p) {
 // (W (h * g) / rms = W (RMSNorm(h) * g)).  One consumer barrier; nss: [kCW]
 // floats of shared memory not otherwise in use until the next call.
 template <class F>
-__device__ __forceinline__ float gather_norm(float* xs, const uint16_t* g, int d, float eps, float* nss, F f) {
+__device__ __forceinline__ float gather_norm(float* xs, const uint16_t* g, int d, float eps, float* nss, Poll& pl, F f) {
     const int n4 = d >> 2;
     float4* x4 = reinterpret_cast<float4*>(xs);
     float ss = 0.f;
     for (int b = threadIdx.x; b < n4; b += 8 * kCT) {
         float4 v[8];
+        uint32_t bad[8];
 #pragma unroll
-        for (int e = 0; e < 8; ++e) v[e] = (b + e * kCT < n4) ? f(4 * (b + e * kCT)) : make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int e = 0; e < 8; ++e) {
+            bad[e] = 0;
+            v[e] = (b + e * kCT < n4) ? f(4 * (b + e * kCT), bad[e]) : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+        retry8(pl, b, n4, v, bad, f);
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
             const int k = b + e * kCT;
@@ -591,30 +665,27 @@ __device__ __forceinline__ void tile_gemv(Consumer& cs, int t0, int t1, int K, i
 
 // Residual entering layer j at row i: the embedding (first layer of a step),
 // the model's h (first layer of a later segment), or the previous layer's O
-// slots (its mid residual) plus its down slots.
+// slots (its mid residual) plus its down slots, tagged with that layer's tag.
 struct ResidIn {
     const SegPlan* p;
     const uint16_t* emb;  // embedding row, or null
     const float* src;     // m.h, or null for the slot sums
     const float* opart;   // the previous layer's O slots
     const uint8_t* nsd;
-    __device__ __forceinline__ float operator()(int i) const {
+    uint32_t tag;         // the previous layer's tag
+    __device__ __forceinline__ float operator()(int i, Poll& pl) const {
         if (emb) return bf(emb[i]);
         if (src) return src[i];
         const int t = i >> 5, l = i & 31, nco = p->n_chunks[1], ns = nsd[t];
         const float* qo = opart + (int64_t)t * nco * 32 + l;
         const float* qd = p->dpart + (int64_t)t * p->n_chunks[3] * 32 + l;
         float v = 0.f;
-#pragma unroll
-        for (int k = 0; k < kSegMaxSlots; ++k)
-            if (k < nco) v += qo[k * 32];
-#pragma unroll
-        for (int k = 0; k < kSegMaxSlots; ++k)
-            if (k < ns) v += qd[k * 32];
+        for (int k = 0; k < nco; ++k) v += pl.get(qo + k * 32, tag);
+        for (int k = 0; k < ns; ++k) v += pl.get(qd + k * 32, tag);
         return v;
     }
-    // rows i..i+3 (i a multiple of 4, same tile)
-    __device__ __forceinline__ float4 four(int i) const {
+    // rows i..i+3 (i a multiple of 4, same tile): one load per slot
+    __device__ __forceinline__ float4 four(int i, uint32_t& bad) const {
         if (emb) return bf4(emb + i);
         if (src) return ldg4(src + i);
         const int t = i >> 5, l = i & 31, nco = p->n_chunks[1], ns = nsd[t];
@@ -623,28 +694,29 @@ struct ResidIn {
         float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
         for (int k = 0; k < kSegMaxSlots; ++k)
-            if (k < nco) v = f4add(v, ldg4(qo + k * 32));
+            if (k < nco) v = add_tagged(v, ld_strong4(qo + k * 32), tag, bad);
 #pragma unroll
         for (int k = 0; k < kSegMaxSlots; ++k)
-            if (k < ns) v = f4add(v, ldg4(qd + k * 32));
+            if (k < ns) v = add_tagged(v, ld_strong4(qd + k * 32), tag, bad);
         return v;
     }
 };
-// O slots of layer j: two buffers, alternating by layer (a chunk-0 O item
+// O slots of layer seq: two buffers, alternating by layer (a chunk-0 O item
 // reads the previous layer's slots while the other items of its tile write
 // this layer's).
-__device__ __forceinline__ float* opart_of(const SegPlan& p, int j) {
-    return p.opart + (int64_t)(j & 1) * p.n_tiles[1] * p.n_chunks[1] * 32;
+__device__ __forceinline__ float* opart_of(const SegPlan& p, unsigned seq) {
+    return p.opart + (int64_t)(seq & 1u) * p.n_tiles[1] * p.n_chunks[1] * 32;
 }
 // Mid residual (after the attention block) at rows i..i+3: the sum of the O
-// slots.
-__device__ __forceinline__ float4 resid_mid4(const SegPlan& p, const float* opart, int i) {
+// slots, tagged with this layer's tag.
+__device__ __forceinline__ float4 resid_mid4(const SegPlan& p, const float* opart, int i, uint32_t tag,
+                                             uint32_t& bad) {
     const int t = i >> 5, nco = p.n_chunks[1];
     const float* qo = opart + (int64_t)t * nco * 32 + (i & 31);
     float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
     for (int k = 0; k < kSegMaxSlots; ++k)
-        if (k < nco) v = f4add(v, ldg4(qo + k * 32));
+        if (k < nco) v = add_tagged(v, ld_strong4(qo + k * 32), tag, bad);
     return v;
 }
 
@@ -753,7 +825,10 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
         return;
     }
     Consumer cs(s, p.stages, err);
+    Poll pl(err);
     unsigned* sync = p.sync;
+    const int64_t last_dn_slot = (int64_t)(p.n_tiles[3] - 1) * p.n_chunks[3];  // first slot of the last down tile
+    const unsigned seq0 = sync[1];  // layers run since the context was reset
     for (int i = threadIdx.x; i < half; i += kCT) s.rope[i] = m.rope[(int64_t)pos * half + i];
     const float2* cs_row = s.rope;
     const float scale = 1.0f / sqrtf((float)m.D);
@@ -778,6 +853,16 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
             c->nucleus_member = -1;
         }
     }
+    {   // attention partials of the splits this launch does not use: 0 (no
+        // tag), so a later launch that uses them again cannot take an old value
+        const int per_head = (kSegMaxSplits - ag.splits) * (m.D + 4);
+        const int64_t n = (int64_t)m.A * per_head;
+        for (int64_t e = (int64_t)cta * kCT + threadIdx.x; e < n; e += (int64_t)G * kCT) {
+            const int h = (int)(e / per_head), r = (int)(e - (int64_t)h * per_head);
+            float* q = p.attn_part + ((int64_t)h * kSegMaxSplits + ag.splits) * (m.D + 4) + r;
+            asm volatile("st.relaxed.gpu.global.b32 [%0], %1;" ::"l"(q), "r"(0u) : "memory");
+        }
+    }
     // the first layer's norm gains; later layers' are copied once the
     // previous layer no longer reads them
     copy_async(s.ga, m.layers + (int64_t)j0 * m.layer_stride + m.off_gattn, m.d);
@@ -786,23 +871,23 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
     int rb = 0;
 
     for (int j = j0; j < j1; ++j) {
-        const int li = j - j0;
-        unsigned* cnt = sync + li * kPhases;
+        const unsigned seq = seq0 + (unsigned)(j - j0);
+        const uint32_t tag = seq_tag(seq);
         const uint16_t* lw = m.layers + (int64_t)j * m.layer_stride;
-        float* op_cur = opart_of(p, j);
-        const ResidIn rin{&p, (j == j0 && first) ? m.embed + (int64_t)tok * m.d : nullptr, j == j0 ? m.h : nullptr,
-                          opart_of(p, j - 1), s.nsd};
+        float* op_cur = opart_of(p, seq);
+        const ResidIn rin{&p,          (j == j0 && first) ? m.embed + (int64_t)tok * m.d : nullptr,
+                          j == j0 ? m.h : nullptr, opart_of(p, seq - 1), s.nsd, seq_tag(seq - 1)};
         const uint16_t* lw_next = lw + m.layer_stride;
 
         // ---------------- Q/K/V tiles: RMSNorm, projection, bias, RoPE, KV append
         if (tq1 > tq0) {
             cp_async_wait();  // this layer's attention-norm gain
-            if (j > j0) {
-                if (!wait_count(cnt - kPhases + kPhDn, G, err)) return;
-            } else {
+            if (j > j0)
+                pl.probe(p.dpart + (last_dn_slot + s.nsd[p.n_tiles[3] - 1] - 1) * 32 + 31, seq_tag(seq - 1));
+            else
                 csync();
-            }
-            const float inv = gather_norm(s.xs, s.ga, m.d, m.eps, s.red + 2 * kCW * 32, [&](int i) { return rin.four(i); });
+            const float inv = gather_norm(s.xs, s.ga, m.d, m.eps, s.red + 2 * kCW * 32, pl,
+                                          [&](int i, uint32_t& bad) { return rin.four(i, bad); });
             const uint16_t* bias = m.qkv_bias ? lw + m.off_bqkv : nullptr;
             uint16_t* kdst = m.kpool + (int64_t)j * m.kv_layer_stride + kvo_pos;
             uint16_t* vdst = m.vpool + (int64_t)j * m.kv_layer_stride + kvo_pos;
@@ -813,33 +898,34 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
                 if (bias) v += bf(bias[2 * u + odd]);
                 const float other = __shfl_xor_sync(0xffffffffu, v, 1);
                 const float r0 = odd ? other : v, r1 = odd ? v : other;
+                // q, and the step's k and v as the cache holds them (bf16), go to
+                // the attention units tagged; k and v also go to the cache
                 if (u < nq) {
                     const int h = u / half, i = u - h * half;
                     const float2 cz = cs_row[i];
                     if (!odd)
-                        m.q[h * m.D + i] = r0 * cz.x - r1 * cz.y;
+                        st_tagged(p.q + h * m.D + i, r0 * cz.x - r1 * cz.y, tag);
                     else
-                        m.q[h * m.D + i + half] = r0 * cz.y + r1 * cz.x;
+                        st_tagged(p.q + h * m.D + i + half, r0 * cz.y + r1 * cz.x, tag);
                 } else if (u < nq + nk) {
                     const int g = (u - nq) / half, i = (u - nq) - g * half;
                     const float2 cz = cs_row[i];
                     uint16_t* k = kdst + (int64_t)g * m.page_size * m.D;
-                    if (!odd)
-                        k[i] = tobf(r0 * cz.x - r1 * cz.y);
-                    else
-                        k[i + half] = tobf(r0 * cz.y + r1 * cz.x);
+                    const int at = odd ? i + half : i;
+                    const uint16_t kb = tobf(odd ? r0 * cz.y + r1 * cz.x : r0 * cz.x - r1 * cz.y);
+                    k[at] = kb;
+                    st_tagged(p.kvn + g * m.D + at, bf(kb), tag);
                 } else if (u < nq + 2 * nk) {
                     const int g = (u - nq - nk) / half, i = (u - nq - nk) - g * half;
                     uint16_t* v2 = vdst + (int64_t)g * m.page_size * m.D;
-                    if (!odd)
-                        v2[i] = tobf(r0);
-                    else
-                        v2[i + half] = tobf(r1);
+                    const int at = odd ? i + half : i;
+                    const uint16_t vb = tobf(odd ? r1 : r0);
+                    v2[at] = vb;
+                    st_tagged(p.kvn + (m.KH + g) * m.D + at, bf(vb), tag);
                 }
             });
         }
         if (cta == 0 && threadIdx.x == 0) m.kv_src[(int64_t)j * m.max_ctx + pos] = 1;
-        signal_count(cnt + kPhQKV);
         if (j + 1 < j1) {  // the next layer's attention-norm gain (this layer's was read above)
             cp_async_wait();
             copy_async(s.ga, lw_next + m.off_gattn, m.d);
@@ -851,15 +937,17 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
             const int pg0 = sp * ag.pps, pg1 = min(ag.n_pages, pg0 + ag.pps);
             const int p0 = pg0 * m.page_size, p1 = min(ag.T, pg1 * m.page_size);
             const int npos = p1 - p0;
-            if (!wait_count(cnt + kPhQKV, G, err)) return;
-            const float* qsrc = m.q + (int64_t)g * grp * m.D;
-            const uint16_t* kt = m.kpool + (int64_t)j * m.kv_layer_stride + kvo_pos + (int64_t)g * m.page_size * m.D;
-            const uint16_t* vt = m.vpool + (int64_t)j * m.kv_layer_stride + kvo_pos + (int64_t)g * m.page_size * m.D;
-            gather4(s.qa, grp * m.D, [&](int i) {
-                const float4 q = ldg4(qsrc + i);
+            pl.probe(p.kvn + 2 * m.KH * m.D - 1, tag);  // the last value row of the Q/K/V phase
+            const float* qsrc = p.q + (int64_t)g * grp * m.D;
+            const float* kt = p.kvn + (int64_t)g * m.D;
+            const float* vt = p.kvn + (int64_t)(m.KH + g) * m.D;
+            gather4(s.qa, grp * m.D, pl, [&](int i, uint32_t& bad) {
+                const float4 q = add_tagged(make_float4(0.f, 0.f, 0.f, 0.f), ld_strong4(qsrc + i), tag, bad);
                 return make_float4(q.x * scale, q.y * scale, q.z * scale, q.w * scale);
             });
-            gather4(s.kv, 2 * m.D, [&](int i) { return i < m.D ? bf4(kt + i) : bf4(vt + i - m.D); });
+            gather4(s.kv, 2 * m.D, pl, [&](int i, uint32_t& bad) {
+                return add_tagged(make_float4(0.f, 0.f, 0.f, 0.f), ld_strong4(i < m.D ? kt + i : vt + i - m.D), tag, bad);
+            });
             csync();
             // scores: warp per position, lane per D/32 dimensions, q read from
             // shared memory per head
@@ -1033,58 +1121,125 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
                 float* dst = p.attn_part + ((int64_t)(g * grp + hw) * kSegMaxSplits + sp) * (m.D + 4);
 #pragma unroll
                 for (int k = 0; k < 4; ++k)
-                    if (k < dpl) dst[lane * dpl + k] = oacc[k];
+                    if (k < dpl) st_tagged(dst + lane * dpl + k, oacc[k], tag);
                 if (lane == 0) {
-                    dst[m.D] = s.ml[2 * hw];
-                    dst[m.D + 1] = s.ml[2 * hw + 1];
+                    st_tagged(dst + m.D, s.ml[2 * hw], tag);
+                    st_tagged(dst + m.D + 1, s.ml[2 * hw + 1], tag);
                 }
             }
         }
-        signal_count(cnt + kPhAttn);
 
         // ---------------- O items: merge the attention splits of the chunk's heads,
         // project, write the chunk's slot (chunk 0 adds the residual)
         if (io.hi > io.lo) {
-            if (!wait_count(cnt + kPhAttn, G, err)) return;
             const int ns = ag.splits;
-            float* den = s.wts + m.A * kSegMaxSplits;
-            for (int h = w; h < m.A; h += kCW) {  // split weights exp(m_s - M) of each head
-                const float* src = p.attn_part + (int64_t)h * kSegMaxSplits * (m.D + 4) + m.D;
-                const float ms = lane < ns ? src[lane * (m.D + 4)] : -INFINITY;
-                const float ls = lane < ns ? src[lane * (m.D + 4) + 1] : 0.f;
-                const float mx = warp_max(ms);
-                const float wt = lane < ns ? expf(ms - mx) : 0.f;
-                if (lane < ns) s.wts[h * kSegMaxSplits + lane] = wt;
-                const float dn = warp_sum(wt * ls);
-                if (lane == 0) den[h] = dn;
+            {   // the last split's maximum of the first item's first head
+                const int h0 = min(m.A - 1, (io.lo % io.nc) * (kColsPerChunk / m.D));
+                pl.probe(p.attn_part + ((int64_t)h0 * kSegMaxSplits + ns - 1) * (m.D + 4) + m.D, tag);
             }
-            csync();
             const int nit = io.hi - io.lo, ncol = nit * kColsPerChunk;
-            const float* rows = s.xa + ncol;
-            gather4(s.xa, ncol + nit * 32, [&](int e) {
-                if (e >= ncol) {  // residual rows of the chunk-0 items
-                    const int it = (e - ncol) >> 5, i = io.lo + it, t = i / io.nc;
-                    const int row = t * 32 + ((e - ncol) & 31);
-                    return (i - t * io.nc == 0 && row < m.d) ? rin.four(row) : make_float4(0.f, 0.f, 0.f, 0.f);
+            const int hpc = kColsPerChunk / m.D;  // heads per chunk
+            float* rows = s.xa + ncol;
+            // One warp per (item, head): the head's split statistics (lane =
+            // split) and this lane's four columns of every split's partial o
+            // in one round of loads, then o = sum_s w_s o_s / sum_s w_s l_s with
+            // w_s = exp(m_s - max m).  One more warp per chunk-0 item gathers
+            // the residual rows its slot carries.
+            for (int wi = w; wi < nit * (hpc + 1); wi += kCW) {
+                if (wi >= nit * hpc) {
+                    const int it = wi - nit * hpc, i = io.lo + it, t = i / io.nc;
+                    if (lane < 8) {
+                        const int row = t * 32 + 4 * lane;
+                        float4 r = make_float4(0.f, 0.f, 0.f, 0.f);
+                        if (i - t * io.nc == 0 && row < m.d) {
+                            uint32_t bad = 0;
+                            r = rin.four(row, bad);
+                            if (bad) {
+                                Bound bd;
+                                while (pl.again(bd)) {
+                                    bad = 0;
+                                    r = rin.four(row, bad);
+                                    if (!bad) break;
+                                }
+                            }
+                        }
+                        reinterpret_cast<float4*>(rows + it * 32)[lane] = r;
+                    }
+                    continue;
                 }
-                const int i = io.lo + e / kColsPerChunk, ch = i % io.nc;
-                const int col = ch * kColsPerChunk + e % kColsPerChunk;
-                if (col >= AD) return make_float4(0.f, 0.f, 0.f, 0.f);
-                const int h = col / m.D;
-                const float* src = p.attn_part + (int64_t)h * kSegMaxSplits * (m.D + 4) + (col - h * m.D);
-                const float* wt = s.wts + h * kSegMaxSplits;
+                const int it = wi / hpc, hc = wi - it * hpc, ch = (io.lo + it) % io.nc;
+                const int h = ch * hpc + hc;
+                const bool cols = lane * 4 < m.D;
+                float4* dst = reinterpret_cast<float4*>(s.xa + it * kColsPerChunk + hc * m.D) + lane;
+                if (h >= m.A) {
+                    if (cols) *dst = make_float4(0.f, 0.f, 0.f, 0.f);
+                    continue;
+                }
+                const float* base = p.attn_part + (int64_t)h * kSegMaxSplits * (m.D + 4);
+                const float* st = base + lane * (m.D + 4) + m.D;
+                const float* oc = base + lane * 4;
+                constexpr int kB = 16;
+                float mk = -INFINITY, lk = 0.f;
+                float4 ob[kB];
+                Bound bd;
+                for (;;) {  // one round of loads, again until every lane has its values
+                    uint32_t bad = 0;
+                    if (lane < ns) {
+                        const uint32_t a = ld_strong(st), b = ld_strong(st + 1);
+                        bad |= ((a ^ tag) | (b ^ tag)) & 31u;
+                        mk = untag(a);
+                        lk = untag(b);
+                    }
+#pragma unroll
+                    for (int u = 0; u < kB; ++u) {
+                        ob[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+                        if (u < ns && cols) {
+                            const uint4 v = ld_strong4(oc + u * (m.D + 4));
+                            bad |= mismatch4(v, tag);
+                            ob[u] = untag4(v);
+                        }
+                    }
+                    if (!__any_sync(0xffffffffu, bad != 0)) break;
+                    const bool more = pl.again(bd);
+                    if (!__all_sync(0xffffffffu, more)) break;
+                }
+                const float mx = warp_max(mk);
+                const float wk = lane < ns ? expf(mk - mx) : 0.f;
+                const float dn = warp_sum(wk * lk);
                 float4 num = make_float4(0.f, 0.f, 0.f, 0.f);
-                for (int k = 0; k < ns; ++k) {
-                    const float4 o = ldg4(src + k * (m.D + 4));
-                    const float wk = wt[k];
-                    num.x = fmaf(wk, o.x, num.x);
-                    num.y = fmaf(wk, o.y, num.y);
-                    num.z = fmaf(wk, o.z, num.z);
-                    num.w = fmaf(wk, o.w, num.w);
+                for (int k0 = 0; k0 < ns; k0 += kB) {
+                    if (k0 > 0) {  // the next splits (their statistics are in hand)
+                        Bound bd2;
+                        for (;;) {
+                            uint32_t bad = 0;
+#pragma unroll
+                            for (int u = 0; u < kB; ++u) {
+                                ob[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+                                if (k0 + u < ns && cols) {
+                                    const uint4 v = ld_strong4(oc + (k0 + u) * (m.D + 4));
+                                    bad |= mismatch4(v, tag);
+                                    ob[u] = untag4(v);
+                                }
+                            }
+                            if (!__any_sync(0xffffffffu, bad != 0)) break;
+                            const bool more = pl.again(bd2);
+                            if (!__all_sync(0xffffffffu, more)) break;
+                        }
+                    }
+#pragma unroll
+                    for (int u = 0; u < kB; ++u) {
+                        const float wu = __shfl_sync(0xffffffffu, wk, (k0 + u) & 31);
+                        if (k0 + u < ns) {
+                            num.x = fmaf(wu, ob[u].x, num.x);
+                            num.y = fmaf(wu, ob[u].y, num.y);
+                            num.z = fmaf(wu, ob[u].z, num.z);
+                            num.w = fmaf(wu, ob[u].w, num.w);
+                        }
+                    }
                 }
-                const float inv = 1.0f / den[h];
-                return make_float4(num.x * inv, num.y * inv, num.z * inv, num.w * inv);
-            });
+                const float inv = 1.0f / dn;
+                if (cols) *dst = make_float4(num.x * inv, num.y * inv, num.z * inv, num.w * inv);
+            }
             csync();
             for (int i = io.lo; i < io.hi; ++i) {
                 const int t = i / io.nc, ch = i - t * io.nc;
@@ -1100,27 +1255,25 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
                     float sum = ch == 0 ? rows[(i - io.lo) * 32 + lane] : 0.f;
 #pragma unroll
                     for (int k = 0; k < kCW; ++k) sum += r[k * 32 + lane];
-                    op_cur[((int64_t)t * io.nc + ch) * 32 + lane] = sum;
+                    st_tagged(op_cur + ((int64_t)t * io.nc + ch) * 32 + lane, sum, tag);
                 }
                 rb ^= 1;
             }
         }
-        signal_count(cnt + kPhO);
 
         // ---------------- gate/up tiles: RMSNorm of the mid residual, SwiGLU
         if (tg1 > tg0) {
             cp_async_wait();  // this layer's MLP-norm gain
-            if (!wait_count(cnt + kPhO, G, err)) return;
-            const float inv = gather_norm(s.xs, s.gm, m.d, m.eps, s.red + 2 * kCW * 32,
-                                          [&](int i) { return resid_mid4(p, op_cur, i); });
+            pl.probe(op_cur + ((int64_t)p.n_tiles[1] * p.n_chunks[1] - 1) * 32 + 31, tag);  // the last O slot
+            const float inv = gather_norm(s.xs, s.gm, m.d, m.eps, s.red + 2 * kCW * 32, pl,
+                                          [&](int i, uint32_t& bad) { return resid_mid4(p, op_cur, i, tag, bad); });
             tile_gemv(cs, tg0, tg1, p.K[2], p.n_chunks[2], s.xs, s.red, rb, [&](int t, float v) {
                 v *= inv;
                 const float up = __shfl_xor_sync(0xffffffffu, v, 1);
                 const int f = t * 16 + (lane >> 1);
-                if (!(lane & 1) && f < m.F) m.a[f] = v / (1.0f + expf(-v)) * up;
+                if (!(lane & 1) && f < m.F) st_tagged(p.a + f, v / (1.0f + expf(-v)) * up, tag);
             });
         }
-        signal_count(cnt + kPhGU);
         if (j + 1 < j1) {  // the next layer's MLP-norm gain
             cp_async_wait();
             copy_async(s.gm, lw_next + m.off_gmlp, m.d);
@@ -1128,11 +1281,12 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
 
         // ---------------- down items: partial slots of h_out - h_mid
         if (idn.hi > idn.lo) {
-            if (!wait_count(cnt + kPhGU, G, err)) return;
-            gather4(s.xa, (idn.hi - idn.lo) * kColsPerChunk, [&](int e) {
+            pl.probe(p.a + m.F - 1, tag);  // the last gate/up tile's product
+            gather4(s.xa, (idn.hi - idn.lo) * kColsPerChunk, pl, [&](int e, uint32_t& bad) {
                 const int i = idn.lo + e / kColsPerChunk, col = e % kColsPerChunk;
                 const int ch = i % idn.nc, f = ch * kColsPerChunk + col;
-                return f < m.F ? ldg4(m.a + f) : make_float4(0.f, 0.f, 0.f, 0.f);
+                return f < m.F ? add_tagged(make_float4(0.f, 0.f, 0.f, 0.f), ld_strong4(p.a + f), tag, bad)
+                               : make_float4(0.f, 0.f, 0.f, 0.f);
             });
             csync();
             float acc = 0.f;
@@ -1153,30 +1307,30 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
 #pragma unroll
                         for (int k = 0; k < kCW; ++k) sum += r[k * 32 + lane];
                         const int slot = cta - item_owner(idn, t * idn.nc);
-                        p.dpart[((int64_t)t * idn.nc + slot) * 32 + lane] = sum;
+                        st_tagged(p.dpart + ((int64_t)t * idn.nc + slot) * 32 + lane, sum, tag);
                     }
                     rb ^= 1;
                 }
             }
         }
-        signal_count(cnt + kPhDn);
     }
 
     // ---------------- the segment's output residual, then the exit ticket
     cp_async_wait();
-    if (!wait_count(sync + (j1 - 1 - j0) * kPhases + kPhDn, G, err)) return;
     {
-        const ResidIn rout{&p, nullptr, nullptr, opart_of(p, j1 - 1), s.nsd};
-        for (int i = slice0 + threadIdx.x; i < slice1; i += kCT) m.h[i] = rout(i);  // slice: scalar
+        const unsigned last = seq0 + (unsigned)(j1 - j0 - 1);
+        pl.probe(p.dpart + (last_dn_slot + s.nsd[p.n_tiles[3] - 1] - 1) * 32 + 31, seq_tag(last));
+        const ResidIn rout{&p, nullptr, nullptr, opart_of(p, last), s.nsd, seq_tag(last)};
+        for (int i = slice0 + threadIdx.x; i < slice1; i += kCT) m.h[i] = rout(i, pl);  // slice: scalar
     }
-    __threadfence();
+    // the exit ticket: once every CTA has taken it, no CTA reads the launch
+    // count any more and the last one advances it for the next launch
     csync();
     if (threadIdx.x == 0) {
-        unsigned* ticket = sync + (j1 - j0) * kPhases;
-        const unsigned prev = atomicAdd(ticket, 1u);
-        if (prev == (unsigned)G - 1) {  // every CTA is past its last wait: reset for the next launch
-            for (int i = 0; i <= (j1 - j0) * kPhases; ++i) sync[i] = 0;
-            __threadfence();
+        const unsigned prev = atomicAdd(&sync[0], 1u);
+        if (prev == (unsigned)G - 1) {
+            sync[0] = 0;
+            sync[1] = seq0 + (unsigned)(j1 - j0);
         }
     }
 }
