@@ -537,17 +537,17 @@ __device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_al
 // Reload the elements of a gather round whose tags were not yet all the
 // expected ones, every such element's loads issued together, until none is
 // left (or the wait has run out).
-template <class F>
-__device__ __forceinline__ void retry8(Poll& pl, int b, int n4, float4 (&v)[8], uint32_t (&bad)[8], F f) {
+template <int U, class F>
+__device__ __forceinline__ void retry(Poll& pl, int b, float4 (&v)[U], uint32_t (&bad)[U], F f) {
     uint32_t any = 0;
 #pragma unroll
-    for (int e = 0; e < 8; ++e) any |= bad[e];
+    for (int e = 0; e < U; ++e) any |= bad[e];
     if (!any) return;
     Bound bd;
     while (pl.again(bd)) {
         any = 0;
 #pragma unroll
-        for (int e = 0; e < 8; ++e)
+        for (int e = 0; e < U; ++e)
             if (bad[e]) {
                 bad[e] = 0;
                 v[e] = f(4 * (b + e * kCT), bad[e]);
@@ -557,25 +557,25 @@ __device__ __forceinline__ void retry8(Poll& pl, int b, int n4, float4 (&v)[8], 
     }
 }
 
-// dst[i..i+3] = f(i) for i < n (n and dst 4-aligned), eight float4 per
-// thread per round with all their loads issued before any store.  f(i, bad)
-// loads once and ORs a nonzero value into bad if a tag was not yet the
-// expected one; such elements are loaded again (retry8).
-template <class F>
+// dst[i..i+3] = f(i) for i < n (n and dst 4-aligned), U float4 per thread
+// per round with all their loads issued before any store.  f(i, bad) loads
+// once and ORs a nonzero value into bad if a tag was not yet the expected
+// one; such elements are loaded again (retry).
+template <int U, class F>
 __device__ __forceinline__ void gather4(float* dst, int n, Poll& pl, F f) {
     const int n4 = n >> 2;
     float4* d4 = reinterpret_cast<float4*>(dst);
-    for (int b = threadIdx.x; b < n4; b += 8 * kCT) {
-        float4 v[8];
-        uint32_t bad[8];
+    for (int b = threadIdx.x; b < n4; b += U * kCT) {
+        float4 v[U];
+        uint32_t bad[U];
 #pragma unroll
-        for (int e = 0; e < 8; ++e) {
+        for (int e = 0; e < U; ++e) {
             bad[e] = 0;
             v[e] = (b + e * kCT < n4) ? f(4 * (b + e * kCT), bad[e]) : make_float4(0.f, 0.f, 0.f, 0.f);
         }
-        retry8(pl, b, n4, v, bad, f);
+        retry<U>(pl, b, v, bad, f);
 #pragma unroll
-        for (int e = 0; e < 8; ++e)
+        for (int e = 0; e < U; ++e)
             if (b + e * kCT < n4) d4[b + e * kCT] = v[e];
     }
 }
@@ -598,22 +598,22 @@ __device__ __forceinline__ float4 bf4(const uint16_t* p) {
 // factor the projection's epilogue applies to each row's dot product
 // (W (h * g) / rms = W (RMSNorm(h) * g)).  One consumer barrier; nss: [kCW]
 // floats of shared memory not otherwise in use until the next call.
-template <class F>
+template <int U, class F>
 __device__ __forceinline__ float gather_norm(float* xs, const uint16_t* g, int d, float eps, float* nss, Poll& pl, F f) {
     const int n4 = d >> 2;
     float4* x4 = reinterpret_cast<float4*>(xs);
     float ss = 0.f;
-    for (int b = threadIdx.x; b < n4; b += 8 * kCT) {
-        float4 v[8];
-        uint32_t bad[8];
+    for (int b = threadIdx.x; b < n4; b += U * kCT) {
+        float4 v[U];
+        uint32_t bad[U];
 #pragma unroll
-        for (int e = 0; e < 8; ++e) {
+        for (int e = 0; e < U; ++e) {
             bad[e] = 0;
             v[e] = (b + e * kCT < n4) ? f(4 * (b + e * kCT), bad[e]) : make_float4(0.f, 0.f, 0.f, 0.f);
         }
-        retry8(pl, b, n4, v, bad, f);
+        retry<U>(pl, b, v, bad, f);
 #pragma unroll
-        for (int e = 0; e < 8; ++e) {
+        for (int e = 0; e < U; ++e) {
             const int k = b + e * kCT;
             if (k < n4) {
                 ss = fmaf(v[e].x, v[e].x, ss);
@@ -886,7 +886,7 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
                 pl.probe(p.dpart + (last_dn_slot + s.nsd[p.n_tiles[3] - 1] - 1) * 32 + 31, seq_tag(seq - 1));
             else
                 csync();
-            const float inv = gather_norm(s.xs, s.ga, m.d, m.eps, s.red + 2 * kCW * 32, pl,
+            const float inv = gather_norm<2>(s.xs, s.ga, m.d, m.eps, s.red + 2 * kCW * 32, pl,
                                           [&](int i, uint32_t& bad) { return rin.four(i, bad); });
             const uint16_t* bias = m.qkv_bias ? lw + m.off_bqkv : nullptr;
             uint16_t* kdst = m.kpool + (int64_t)j * m.kv_layer_stride + kvo_pos;
@@ -941,31 +941,46 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
             const float* qsrc = p.q + (int64_t)g * grp * m.D;
             const float* kt = p.kvn + (int64_t)g * m.D;
             const float* vt = p.kvn + (int64_t)(m.KH + g) * m.D;
-            gather4(s.qa, grp * m.D, pl, [&](int i, uint32_t& bad) {
+            // the group's scaled queries, then k and v, in one round (s.kv follows s.qa)
+            const int nqa = grp * m.D;
+            gather4<1>(s.qa, nqa + 2 * m.D, pl, [&](int i, uint32_t& bad) {
+                if (i >= nqa) {
+                    const int e = i - nqa;
+                    return add_tagged(make_float4(0.f, 0.f, 0.f, 0.f), ld_strong4(e < m.D ? kt + e : vt + e - m.D), tag,
+                                      bad);
+                }
                 const float4 q = add_tagged(make_float4(0.f, 0.f, 0.f, 0.f), ld_strong4(qsrc + i), tag, bad);
                 return make_float4(q.x * scale, q.y * scale, q.z * scale, q.w * scale);
-            });
-            gather4(s.kv, 2 * m.D, pl, [&](int i, uint32_t& bad) {
-                return add_tagged(make_float4(0.f, 0.f, 0.f, 0.f), ld_strong4(i < m.D ? kt + i : vt + i - m.D), tag, bad);
             });
             csync();
             // scores: warp per position, lane per D/32 dimensions, q read from
             // shared memory per head
             const int dpl = m.D >> 5;  // 2 or 4
             const int spc = p.max_pps * m.page_size;  // score row stride
-            float qr[kSegMaxGroup][4];
+            // this lane's dpl dimensions of each query, and of the step's own k
+            // and v (the ring holds the cache's stale copy of that row: they are
+            // substituted by a select, not a branch); vector loads, no conflicts
+            float qr[kSegMaxGroup][4], kvt[4], vvt[4];
+            auto lane_dims = [&](const float* src, float (&dst)[4]) {
+                if (dpl == 4) {
+                    const float4 t = lds128f(saddr(src + lane * 4));
+                    dst[0] = t.x, dst[1] = t.y, dst[2] = t.z, dst[3] = t.w;
+                } else {
+                    const float2 t = *reinterpret_cast<const float2*>(src + lane * 2);
+                    dst[0] = t.x, dst[1] = t.y, dst[2] = dst[3] = 0.f;
+                }
+            };
 #pragma unroll
-            for (int hh = 0; hh < kSegMaxGroup; ++hh)
+            for (int hh = 0; hh < kSegMaxGroup; ++hh) {
+                if (hh < grp) {
+                    lane_dims(s.qa + hh * m.D, qr[hh]);
+                } else {
 #pragma unroll
-                for (int k = 0; k < 4; ++k) qr[hh][k] = (hh < grp && k < dpl) ? s.qa[hh * m.D + lane * dpl + k] : 0.f;
-            // k and v of the step's own position (the ring holds the cache's
-            // stale copy of that row): substituted by a select, not a branch
-            float kvt[4], vvt[4];
-#pragma unroll
-            for (int k = 0; k < 4; ++k) {
-                kvt[k] = k < dpl ? s.kv[lane * dpl + k] : 0.f;
-                vvt[k] = k < dpl ? s.kv[m.D + lane * dpl + k] : 0.f;
+                    for (int k = 0; k < 4; ++k) qr[hh][k] = 0.f;
+                }
             }
+            lane_dims(s.kv, kvt);
+            lane_dims(s.kv + m.D, vvt);
             for (int pg = pg0; pg < pg1; ++pg)
                 for (int q = 0; q < cpp; ++q) {
                     const uint32_t kb = saddr(cs.acquire()) + lane * dpl * 2;
@@ -1178,7 +1193,7 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
                 const float* base = p.attn_part + (int64_t)h * kSegMaxSplits * (m.D + 4);
                 const float* st = base + lane * (m.D + 4) + m.D;
                 const float* oc = base + lane * 4;
-                constexpr int kB = 16;
+                constexpr int kB = 12;
                 float mk = -INFINITY, lk = 0.f;
                 float4 ob[kB];
                 Bound bd;
@@ -1265,7 +1280,7 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
         if (tg1 > tg0) {
             cp_async_wait();  // this layer's MLP-norm gain
             pl.probe(op_cur + ((int64_t)p.n_tiles[1] * p.n_chunks[1] - 1) * 32 + 31, tag);  // the last O slot
-            const float inv = gather_norm(s.xs, s.gm, m.d, m.eps, s.red + 2 * kCW * 32, pl,
+            const float inv = gather_norm<2>(s.xs, s.gm, m.d, m.eps, s.red + 2 * kCW * 32, pl,
                                           [&](int i, uint32_t& bad) { return resid_mid4(p, op_cur, i, tag, bad); });
             tile_gemv(cs, tg0, tg1, p.K[2], p.n_chunks[2], s.xs, s.red, rb, [&](int t, float v) {
                 v *= inv;
@@ -1282,7 +1297,7 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
         // ---------------- down items: partial slots of h_out - h_mid
         if (idn.hi > idn.lo) {
             pl.probe(p.a + m.F - 1, tag);  // the last gate/up tile's product
-            gather4(s.xa, (idn.hi - idn.lo) * kColsPerChunk, pl, [&](int e, uint32_t& bad) {
+            gather4<4>(s.xa, (idn.hi - idn.lo) * kColsPerChunk, pl, [&](int e, uint32_t& bad) {
                 const int i = idn.lo + e / kColsPerChunk, col = e % kColsPerChunk;
                 const int ch = i % idn.nc, f = ch * kColsPerChunk + col;
                 return f < m.F ? add_tagged(make_float4(0.f, 0.f, 0.f, 0.f), ld_strong4(p.a + f), tag, bad)
