@@ -168,6 +168,30 @@ __device__ __forceinline__ uint32_t lds32(uint32_t a) {
 }
 __device__ __forceinline__ float ldsf(uint32_t a) { return __uint_as_float(lds32(a)); }
 
+__device__ __forceinline__ void sts64(uint32_t a, uint32_t x, uint32_t y) {
+    asm volatile("st.shared.v2.b32 [%0], {%1, %2};" ::"r"(a), "r"(x), "r"(y) : "memory");
+}
+// Two floats as bf16 (round to nearest even), the first in the low half.
+__device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
+    return (uint32_t)tobf(a) | ((uint32_t)tobf(b) << 16);
+}
+// x0, x1 as packed bf16 high parts and packed bf16 low parts (x - high).
+__device__ __forceinline__ void split_bf16x2(float x0, float x1, uint32_t& hi, uint32_t& lo) {
+    const uint16_t h0 = tobf(x0), h1 = tobf(x1);
+    hi = (uint32_t)h0 | ((uint32_t)h1 << 16);
+    lo = pack_bf16x2(x0 - bf(h0), x1 - bf(h1));
+}
+// d += A B for one m16n8k16 tile: bf16 A (4 registers, row-major
+// fragment), bf16 B (2 registers, column-major fragment), fp32 accumulators.
+__device__ __forceinline__ void mma_bf16(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3, uint32_t b0,
+                                         uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+        "{%0, %1, %2, %3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
 // Barrier of the consumer warps only (the producer never joins it).
 __device__ __forceinline__ void csync() { asm volatile("bar.sync 1, %0;" ::"r"(kCT) : "memory"); }
 
@@ -953,103 +977,71 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
                 return make_float4(q.x * scale, q.y * scale, q.z * scale, q.w * scale);
             });
             csync();
-            // scores: warp per position, lane per D/32 dimensions, q read from
-            // shared memory per head
-            const int dpl = m.D >> 5;  // 2 or 4
+            // Scores on the tensor cores: S[h][r] = q_h . k_r as mma m16n8k16
+            // (bf16 operands, fp32 accumulation) with A = the group's queries
+            // split into bf16 high parts (rows 0..7) and low parts (rows 8..15,
+            // the bf16 of q - high; high + low keeps q to 16 bits) and B = 8
+            // cached keys.  A lane loads 8 consecutive dimensions of one key row
+            // (16 bytes, no bank conflicts beyond the row stride's); the
+            // product's k index runs over the dimensions in the same permuted
+            // order in A and B.  Row g of the result is head g's high-part dot
+            // product, row g + 8 its low-part one.
             const int spc = p.max_pps * m.page_size;  // score row stride
-            // this lane's dpl dimensions of each query, and of the step's own k
-            // and v (the ring holds the cache's stale copy of that row: they are
-            // substituted by a select, not a branch); vector loads, no conflicts
-            float qr[kSegMaxGroup][4], kvt[4], vvt[4];
-            auto lane_dims = [&](const float* src, float (&dst)[4]) {
-                if (dpl == 4) {
-                    const float4 t = lds128f(saddr(src + lane * 4));
-                    dst[0] = t.x, dst[1] = t.y, dst[2] = t.z, dst[3] = t.w;
-                } else {
-                    const float2 t = *reinterpret_cast<const float2*>(src + lane * 2);
-                    dst[0] = t.x, dst[1] = t.y, dst[2] = dst[3] = 0.f;
-                }
-            };
+            const int npair = m.D >> 5;               // pairs of k16 steps (32 dimensions)
+            const int g8 = lane >> 2, t4 = lane & 3;
+            uint32_t qhi[4][4], qlo[4][4];  // [pair][word]: dimensions pair*32 + 8 t4 .. +7 of query g8
 #pragma unroll
-            for (int hh = 0; hh < kSegMaxGroup; ++hh) {
-                if (hh < grp) {
-                    lane_dims(s.qa + hh * m.D, qr[hh]);
+            for (int pr = 0; pr < 4; ++pr) {
+                float x[8];
+                if (pr < npair && g8 < grp) {
+                    const float* qrow = s.qa + g8 * m.D + pr * 32 + 8 * t4;
+                    const float4 a = lds128f(saddr(qrow)), b = lds128f(saddr(qrow + 4));
+                    x[0] = a.x, x[1] = a.y, x[2] = a.z, x[3] = a.w, x[4] = b.x, x[5] = b.y, x[6] = b.z, x[7] = b.w;
                 } else {
 #pragma unroll
-                    for (int k = 0; k < 4; ++k) qr[hh][k] = 0.f;
+                    for (int k = 0; k < 8; ++k) x[k] = 0.f;
                 }
+#pragma unroll
+                for (int wd = 0; wd < 4; ++wd) split_bf16x2(x[2 * wd], x[2 * wd + 1], qhi[pr][wd], qlo[pr][wd]);
             }
-            lane_dims(s.kv, kvt);
-            lane_dims(s.kv + m.D, vvt);
             for (int pg = pg0; pg < pg1; ++pg)
                 for (int q = 0; q < cpp; ++q) {
-                    const uint32_t kb = saddr(cs.acquire()) + lane * dpl * 2;
+                    const uint32_t kst = saddr(cs.acquire());
                     const int base = pg * m.page_size + q * rpc;
                     const int nr = min(rpc, p1 - base);
-                    // two positions per step (r and r + kCW), their reductions interleaved
-                    for (int r = w; r < nr; r += 2 * kCW) {
-                        const int rb2 = r + kCW;
-                        const bool two = rb2 < nr;
-                        float kd[2][4];
-#pragma unroll
-                        for (int e = 0; e < 2; ++e) {
-                            const int rr = e == 0 ? r : (two ? rb2 : r);
-                            if (dpl == 4) {
-                                const uint2 v = lds64(kb + rr * m.D * 2);
-                                kd[e][0] = bflo(v.x);
-                                kd[e][1] = bfhi(v.x);
-                                kd[e][2] = bflo(v.y);
-                                kd[e][3] = bfhi(v.y);
-                            } else {
-                                const uint32_t v = lds32(kb + rr * m.D * 2);
-                                kd[e][0] = bflo(v);
-                                kd[e][1] = bfhi(v);
-                                kd[e][2] = kd[e][3] = 0.f;
+                    if (cs.ok) {
+                        for (int nt = w; nt * 8 < nr; nt += kCW) {
+                            const int r0 = nt * 8, own = pos - base;
+                            if (own >= r0 && own < r0 + 8) {
+                                // the ring holds the cache's stale copy of the step's
+                                // own row: write the new k over it (bf16, exact)
+                                for (int e = lane; e < (m.D >> 2); e += 32) {
+                                    const float4 kk = lds128f(saddr(s.kv + 4 * e));
+                                    sts64(kst + own * m.D * 2 + 8 * e, pack_bf16x2(kk.x, kk.y), pack_bf16x2(kk.z, kk.w));
+                                }
+                                __syncwarp();
                             }
-                            const bool own = base + rr == pos;
+                            const uint32_t krow = kst + (r0 + g8) * m.D * 2 + 16 * t4;
+                            float acc[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-                            for (int k = 0; k < 4; ++k) kd[e][k] = own ? kvt[k] : kd[e][k];
-                        }
-                        float dd[2][kSegMaxGroup];
-#pragma unroll
-                        for (int e = 0; e < 2; ++e)
-#pragma unroll
-                            for (int hh = 0; hh < kSegMaxGroup; ++hh) {
-                                float d = qr[hh][0] * kd[e][0];
-                                d = fmaf(qr[hh][1], kd[e][1], d);
-                                d = fmaf(qr[hh][2], kd[e][2], d);
-                                d = fmaf(qr[hh][3], kd[e][3], d);
-                                dd[e][hh] = d;
+                            for (int pr = 0; pr < 4; ++pr) {
+                                if (pr < npair) {
+                                    const uint4 kw = lds128(krow + pr * 64);
+                                    mma_bf16(acc, qhi[pr][0], qlo[pr][0], qhi[pr][1], qlo[pr][1], kw.x, kw.y);
+                                    mma_bf16(acc, qhi[pr][2], qlo[pr][2], qhi[pr][3], qlo[pr][3], kw.z, kw.w);
+                                }
                             }
-                        // reduce-scatter over the warp: lane bits 4, 3, 2 pick the head
-                        const bool b16 = lane & 16, b8 = lane & 8, b4 = lane & 4;
-                        float a4[2][4], a2[2][2], a1[2];
-#pragma unroll
-                        for (int e = 0; e < 2; ++e)
-#pragma unroll
-                            for (int k = 0; k < 4; ++k)
-                                a4[e][k] = (b16 ? dd[e][k + 4] : dd[e][k]) +
-                                           __shfl_xor_sync(0xffffffffu, b16 ? dd[e][k] : dd[e][k + 4], 16);
-#pragma unroll
-                        for (int e = 0; e < 2; ++e)
-#pragma unroll
-                            for (int k = 0; k < 2; ++k)
-                                a2[e][k] = (b8 ? a4[e][k + 2] : a4[e][k]) +
-                                           __shfl_xor_sync(0xffffffffu, b8 ? a4[e][k] : a4[e][k + 2], 8);
-#pragma unroll
-                        for (int e = 0; e < 2; ++e)
-                            a1[e] = (b4 ? a2[e][1] : a2[e][0]) +
-                                    __shfl_xor_sync(0xffffffffu, b4 ? a2[e][0] : a2[e][1], 4);
-#pragma unroll
-                        for (int e = 0; e < 2; ++e) a1[e] += __shfl_xor_sync(0xffffffffu, a1[e], 2);
-#pragma unroll
-                        for (int e = 0; e < 2; ++e) a1[e] += __shfl_xor_sync(0xffffffffu, a1[e], 1);
-                        const int hd = (b16 ? 4 : 0) + (b8 ? 2 : 0) + (b4 ? 1 : 0);
-                        if ((lane & 3) == 0 && hd < grp) {
-                            s.sc[hd * spc + (base + r - p0)] = a1[0];
-                            if (two) s.sc[hd * spc + (base + rb2 - p0)] = a1[1];
+                            const int ra = r0 + 2 * t4;
+                            if (g8 < grp) {
+                                float* sr = s.sc + g8 * spc + (base - p0);
+                                if (ra < nr) sr[ra] = acc[0] + acc[2];
+                                if (ra + 1 < nr) sr[ra + 1] = acc[1] + acc[3];
+                            }
                         }
                     }
+                    // generic writes to the stage (the fixed row) before the
+                    // producer's next bulk copy into it
+                    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
                     cs.release();
                 }
             csync();
@@ -1070,76 +1062,93 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
                 }
             }
             csync();
-            // P V: warp w works on head w % grp for the positions r with
-            // r % nsp == w / grp; the nsp partial sums meet in xs (free here)
-            const int nsp = max(1, min(kCW / grp, max(m.d, AD) / (grp * m.D)));
-            const int hw = w % grp, part = w / grp;
-            const bool pv = w < grp * nsp;
-            float oacc[4] = {0.f, 0.f, 0.f, 0.f}, obcc[4] = {0.f, 0.f, 0.f, 0.f};
-            float occc[4] = {0.f, 0.f, 0.f, 0.f}, odcc[4] = {0.f, 0.f, 0.f, 0.f};
+            // P V: warp w takes head group hg = w / npq (hpg heads) and the
+            // positions r = w mod npq (mod npq); lane = dpl dimensions.  Each V
+            // row is read once per head group.  The npq partial sums per head
+            // meet in shared memory (xs and xa, contiguous and free here) and are
+            // added in order.
+            const int dpl = m.D >> 5;  // 2 or 4
+            const int hgn = grp > 4 ? 2 : 1, hpg = (grp + hgn - 1) / hgn;
+            const int avail = ((max(m.d, AD) + 3) & ~3) + p.max_items * (kColsPerChunk + 32);
+            int npq = kCW / hgn;
+            while (npq > 1 && npq * grp * m.D > avail) npq >>= 1;
+            const int hg = w / npq, pq = w - hg * npq;
+            const bool pv = hg < hgn;
+            float vvt[4];  // the step's own v (this lane's dimensions)
+            if (dpl == 4) {
+                const float4 t = lds128f(saddr(s.kv + m.D + lane * 4));
+                vvt[0] = t.x, vvt[1] = t.y, vvt[2] = t.z, vvt[3] = t.w;
+            } else {
+                const float2 t = *reinterpret_cast<const float2*>(s.kv + m.D + lane * 2);
+                vvt[0] = t.x, vvt[1] = t.y, vvt[2] = vvt[3] = 0.f;
+            }
+            float acc[4][4];
+#pragma unroll
+            for (int hh = 0; hh < 4; ++hh)
+#pragma unroll
+                for (int k = 0; k < 4; ++k) acc[hh][k] = 0.f;
             for (int pg = pg0; pg < pg1; ++pg)
                 for (int q = 0; q < cpp; ++q) {
                     const uint32_t vb = saddr(cs.acquire()) + lane * dpl * 2;
                     const int base = pg * m.page_size + q * rpc;
                     const int nr = min(rpc, p1 - base);
                     if (pv && cs.ok) {
-                        const uint32_t pw = saddr(s.sc + hw * spc + (base - p0));
-                        // four positions per step into four accumulator sets; a
-                        // slot past the chunk gets probability 0 and value 0 (a
-                        // select: the stand-in row may hold anything)
-                        for (int r = part; r < nr; r += 4 * nsp) {
-                            float pq[4], vq[4][4];
-#pragma unroll
-                            for (int e = 0; e < 4; ++e) {
-                                const int re = r + e * nsp;
-                                const bool in = re < nr;
-                                const int rr = in ? re : r;
-                                pq[e] = in ? ldsf(pw + 4 * rr) : 0.f;
-                                if (dpl == 4) {
-                                    const uint2 u = lds64(vb + rr * m.D * 2);
-                                    vq[e][0] = bflo(u.x), vq[e][1] = bfhi(u.x), vq[e][2] = bflo(u.y), vq[e][3] = bfhi(u.y);
-                                } else {
-                                    const uint32_t u = lds32(vb + rr * m.D * 2);
-                                    vq[e][0] = bflo(u), vq[e][1] = bfhi(u), vq[e][2] = vq[e][3] = 0.f;
-                                }
-#pragma unroll
-                                for (int k = 0; k < 4; ++k)
-                                    vq[e][k] = !in ? 0.f : (base + re == pos ? vvt[k] : vq[e][k]);
+                        const float* pr0 = s.sc + (hg * hpg) * spc + (base - p0);
+#pragma unroll 2
+                        for (int r = pq; r < nr; r += npq) {
+                            float v[4];
+                            if (dpl == 4) {
+                                const uint2 u = lds64(vb + r * m.D * 2);
+                                v[0] = bflo(u.x), v[1] = bfhi(u.x), v[2] = bflo(u.y), v[3] = bfhi(u.y);
+                            } else {
+                                const uint32_t u = lds32(vb + r * m.D * 2);
+                                v[0] = bflo(u), v[1] = bfhi(u), v[2] = v[3] = 0.f;
                             }
+                            const bool own = base + r == pos;  // the ring's copy of this row is stale
 #pragma unroll
-                            for (int k = 0; k < 4; ++k) {
-                                oacc[k] = fmaf(pq[0], vq[0][k], oacc[k]);
-                                obcc[k] = fmaf(pq[1], vq[1][k], obcc[k]);
-                                occc[k] = fmaf(pq[2], vq[2][k], occc[k]);
-                                odcc[k] = fmaf(pq[3], vq[3][k], odcc[k]);
+                            for (int k = 0; k < 4; ++k) v[k] = own ? vvt[k] : v[k];
+#pragma unroll
+                            for (int hh = 0; hh < 4; ++hh) {
+                                if (hh < hpg && hg * hpg + hh < grp) {
+                                    const float pr = pr0[hh * spc + r];
+#pragma unroll
+                                    for (int k = 0; k < 4; ++k) acc[hh][k] = fmaf(pr, v[k], acc[hh][k]);
+                                }
                             }
                         }
                     }
                     cs.release();
                 }
+            float* part = s.xs;  // [grp][npq][D]
+            if (pv) {
 #pragma unroll
-            for (int k = 0; k < 4; ++k) oacc[k] = (oacc[k] + obcc[k]) + (occc[k] + odcc[k]);
-            if (pv && part > 0) {
-                float* dst = s.xs + ((part - 1) * grp + hw) * m.D + lane * dpl;
+                for (int hh = 0; hh < 4; ++hh) {
+                    const int h = hg * hpg + hh;
+                    if (hh < hpg && h < grp) {
+                        float* dst = part + (h * npq + pq) * m.D + lane * dpl;
 #pragma unroll
-                for (int k = 0; k < 4; ++k)
-                    if (k < dpl) dst[k] = oacc[k];
+                        for (int k = 0; k < 4; ++k)
+                            if (k < dpl) dst[k] = acc[hh][k];
+                    }
+                }
             }
             csync();
-            if (pv && part == 0) {
-                for (int pp = 1; pp < nsp; ++pp) {
-                    const float* src = s.xs + ((pp - 1) * grp + hw) * m.D + lane * dpl;
-#pragma unroll
-                    for (int k = 0; k < 4; ++k)
-                        if (k < dpl) oacc[k] += src[k];
+            {
+                const int d4 = m.D >> 2;
+                for (int e = threadIdx.x; e < grp * d4; e += kCT) {
+                    const int h = e / d4, c = 4 * (e - h * d4);
+                    float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
+                    for (int k = 0; k < npq; ++k) sum = f4add(sum, *reinterpret_cast<const float4*>(part + (h * npq + k) * m.D + c));
+                    float* dst = p.attn_part + ((int64_t)(g * grp + h) * kSegMaxSplits + sp) * (m.D + 4) + c;
+                    st_tagged(dst, sum.x, tag);
+                    st_tagged(dst + 1, sum.y, tag);
+                    st_tagged(dst + 2, sum.z, tag);
+                    st_tagged(dst + 3, sum.w, tag);
                 }
-                float* dst = p.attn_part + ((int64_t)(g * grp + hw) * kSegMaxSplits + sp) * (m.D + 4);
-#pragma unroll
-                for (int k = 0; k < 4; ++k)
-                    if (k < dpl) st_tagged(dst + lane * dpl + k, oacc[k], tag);
-                if (lane == 0) {
-                    st_tagged(dst + m.D, s.ml[2 * hw], tag);
-                    st_tagged(dst + m.D + 1, s.ml[2 * hw + 1], tag);
+                if (threadIdx.x < grp) {
+                    float* dst = p.attn_part + ((int64_t)(g * grp + threadIdx.x) * kSegMaxSplits + sp) * (m.D + 4) + m.D;
+                    st_tagged(dst, s.ml[2 * threadIdx.x], tag);
+                    st_tagged(dst + 1, s.ml[2 * threadIdx.x + 1], tag);
                 }
             }
         }
