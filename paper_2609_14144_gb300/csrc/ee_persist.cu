@@ -334,14 +334,11 @@ struct Smem {
     float* xa;          // [max items][512] staged input columns of the O / down items, then
                         // [max items][32] residual rows of the O items of chunk 0
     float2* rope;       // [D/2] (cos, sin) of the step's position
-    uint16_t* ga;       // [d] attention-norm gain of the current layer
-    uint16_t* gm;       // [d] MLP-norm gain of the current layer
     float* red;         // [2][kCW][32], then [kCW] sums of squares of the RMSNorm
     float* qa;          // [group][D] scaled queries of the attention unit
     float* kv;          // [2][D] k, v of the step's position
     float* sc;          // [group][pps * page_size] scores, then probabilities
     float* ml;          // [group][2] max, sum
-    float* wts;         // [A][kSegMaxSplits] split weights of the attention merge, then [A] denominators
     uint8_t* nsd;       // [down tiles] slots per down tile
 };
 __device__ __forceinline__ Smem carve(uint8_t* base, const DevModel& m, const SegPlan& p) {
@@ -360,10 +357,6 @@ __device__ __forceinline__ Smem carve(uint8_t* base, const DevModel& m, const Se
     f += p.max_items * (kColsPerChunk + 32);
     s.rope = reinterpret_cast<float2*>(f);
     f += m.D;
-    s.ga = reinterpret_cast<uint16_t*>(f);
-    f += (m.d + 1) / 2;
-    s.gm = reinterpret_cast<uint16_t*>(f);
-    f += (m.d + 1) / 2;
     s.red = f;
     f += 2 * kCW * 32 + kCW;
     const int grp = m.A / m.KH;
@@ -375,8 +368,6 @@ __device__ __forceinline__ Smem carve(uint8_t* base, const DevModel& m, const Se
     f += grp * p.max_pps * m.page_size;
     s.ml = f;
     f += 2 * grp;
-    s.wts = f;
-    f += m.A * (kSegMaxSplits + 1);
     s.nsd = reinterpret_cast<uint8_t*>(f);
     return s;
 }
@@ -548,15 +539,6 @@ struct Poll {
     }
 };
 
-// Asynchronous copy of n bf16 values (n a multiple of 8, both addresses
-// 16-byte aligned) into shared memory; complete once every consumer thread
-// has passed cp_async_wait() and a consumer barrier.
-__device__ __forceinline__ void copy_async(uint16_t* dst, const uint16_t* src, int n) {
-    for (int i = threadIdx.x; i < (n >> 3); i += kCT)
-        asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(saddr(dst + 8 * i)), "l"(src + 8 * i) : "memory");
-    asm volatile("cp.async.commit_group;" ::: "memory");
-}
-__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_all;" ::: "memory"); }
 
 // Reload the elements of a gather round whose tags were not yet all the
 // expected ones, every such element's loads issued together, until none is
@@ -618,7 +600,8 @@ __device__ __forceinline__ float4 bf4(const uint16_t* p) {
 }
 
 // RMSNorm folded into the gather of its input: xs = h * g (d values, h
-// from f four at a time) and the return value 1 / sqrt(mean(h^2) + eps), the
+// from f four at a time, g the bf16 gain in global memory) and the return
+// value 1 / sqrt(mean(h^2) + eps), the
 // factor the projection's epilogue applies to each row's dot product
 // (W (h * g) / rms = W (RMSNorm(h) * g)).  One consumer barrier; nss: [kCW]
 // floats of shared memory not otherwise in use until the next call.
@@ -630,10 +613,13 @@ __device__ __forceinline__ float gather_norm(float* xs, const uint16_t* g, int d
     for (int b = threadIdx.x; b < n4; b += U * kCT) {
         float4 v[U];
         uint32_t bad[U];
+        uint2 gg[U];  // the gain (global, read-only), loaded with the values
 #pragma unroll
         for (int e = 0; e < U; ++e) {
             bad[e] = 0;
-            v[e] = (b + e * kCT < n4) ? f(4 * (b + e * kCT), bad[e]) : make_float4(0.f, 0.f, 0.f, 0.f);
+            const bool in = b + e * kCT < n4;
+            gg[e] = in ? __ldg(reinterpret_cast<const uint2*>(g) + (b + e * kCT)) : make_uint2(0u, 0u);
+            v[e] = in ? f(4 * (b + e * kCT), bad[e]) : make_float4(0.f, 0.f, 0.f, 0.f);
         }
         retry<U>(pl, b, v, bad, f);
 #pragma unroll
@@ -644,7 +630,7 @@ __device__ __forceinline__ float gather_norm(float* xs, const uint16_t* g, int d
                 ss = fmaf(v[e].y, v[e].y, ss);
                 ss = fmaf(v[e].z, v[e].z, ss);
                 ss = fmaf(v[e].w, v[e].w, ss);
-                const uint2 gu = *reinterpret_cast<const uint2*>(g + 4 * k);
+                const uint2 gu = gg[e];
                 x4[k] = make_float4(v[e].x * bflo(gu.x), v[e].y * bfhi(gu.x), v[e].z * bflo(gu.y), v[e].w * bfhi(gu.y));
             }
         }
@@ -887,10 +873,6 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
             asm volatile("st.relaxed.gpu.global.b32 [%0], %1;" ::"l"(q), "r"(0u) : "memory");
         }
     }
-    // the first layer's norm gains; later layers' are copied once the
-    // previous layer no longer reads them
-    copy_async(s.ga, m.layers + (int64_t)j0 * m.layer_stride + m.off_gattn, m.d);
-    copy_async(s.gm, m.layers + (int64_t)j0 * m.layer_stride + m.off_gmlp, m.d);
     csync();
     int rb = 0;
 
@@ -901,16 +883,14 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
         float* op_cur = opart_of(p, seq);
         const ResidIn rin{&p,          (j == j0 && first) ? m.embed + (int64_t)tok * m.d : nullptr,
                           j == j0 ? m.h : nullptr, opart_of(p, seq - 1), s.nsd, seq_tag(seq - 1)};
-        const uint16_t* lw_next = lw + m.layer_stride;
 
         // ---------------- Q/K/V tiles: RMSNorm, projection, bias, RoPE, KV append
         if (tq1 > tq0) {
-            cp_async_wait();  // this layer's attention-norm gain
             if (j > j0)
                 pl.probe(p.dpart + (last_dn_slot + s.nsd[p.n_tiles[3] - 1] - 1) * 32 + 31, seq_tag(seq - 1));
             else
                 csync();
-            const float inv = gather_norm<2>(s.xs, s.ga, m.d, m.eps, s.red + 2 * kCW * 32, pl,
+            const float inv = gather_norm<2>(s.xs, lw + m.off_gattn, m.d, m.eps, s.red + 2 * kCW * 32, pl,
                                           [&](int i, uint32_t& bad) { return rin.four(i, bad); });
             const uint16_t* bias = m.qkv_bias ? lw + m.off_bqkv : nullptr;
             uint16_t* kdst = m.kpool + (int64_t)j * m.kv_layer_stride + kvo_pos;
@@ -950,10 +930,6 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
             });
         }
         if (cta == 0 && threadIdx.x == 0) m.kv_src[(int64_t)j * m.max_ctx + pos] = 1;
-        if (j + 1 < j1) {  // the next layer's attention-norm gain (this layer's was read above)
-            cp_async_wait();
-            copy_async(s.ga, lw_next + m.off_gattn, m.d);
-        }
 
         // ---------------- attention unit (if this CTA has one)
         if (unit >= 0) {
@@ -1287,9 +1263,8 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
 
         // ---------------- gate/up tiles: RMSNorm of the mid residual, SwiGLU
         if (tg1 > tg0) {
-            cp_async_wait();  // this layer's MLP-norm gain
             pl.probe(op_cur + ((int64_t)p.n_tiles[1] * p.n_chunks[1] - 1) * 32 + 31, tag);  // the last O slot
-            const float inv = gather_norm<2>(s.xs, s.gm, m.d, m.eps, s.red + 2 * kCW * 32, pl,
+            const float inv = gather_norm<2>(s.xs, lw + m.off_gmlp, m.d, m.eps, s.red + 2 * kCW * 32, pl,
                                           [&](int i, uint32_t& bad) { return resid_mid4(p, op_cur, i, tag, bad); });
             tile_gemv(cs, tg0, tg1, p.K[2], p.n_chunks[2], s.xs, s.red, rb, [&](int t, float v) {
                 v *= inv;
@@ -1297,10 +1272,6 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
                 const int f = t * 16 + (lane >> 1);
                 if (!(lane & 1) && f < m.F) st_tagged(p.a + f, v / (1.0f + expf(-v)) * up, tag);
             });
-        }
-        if (j + 1 < j1) {  // the next layer's MLP-norm gain
-            cp_async_wait();
-            copy_async(s.gm, lw_next + m.off_gmlp, m.d);
         }
 
         // ---------------- down items: partial slots of h_out - h_mid
@@ -1340,7 +1311,6 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
     }
 
     // ---------------- the segment's output residual, then the exit ticket
-    cp_async_wait();
     {
         const unsigned last = seq0 + (unsigned)(j1 - j0 - 1);
         pl.probe(p.dpart + (last_dn_slot + s.nsd[p.n_tiles[3] - 1] - 1) * 32 + 31, seq_tag(last));
@@ -1387,9 +1357,10 @@ bool seg_plan(const DevModel& m, int n_sm, SegPlan& p) {
     const int cap = std::max(1, std::min(kSegMaxSplits, p.G / m.KH));
     const int np_max = (m.max_ctx + m.page_size - 1) / m.page_size;
     p.max_pps = std::max(1, (np_max + cap - 1) / cap);
-    const size_t floats = (size_t)((std::max(m.d, m.A * m.D) + 3) & ~3) +
-                          (size_t)p.max_items * (kColsPerChunk + 32) + (size_t)m.D + (size_t)m.d + 2 * kCW * 32 + kCW + (size_t)grp * m.D + 2 * (size_t)m.D +
-                          (size_t)grp * p.max_pps * m.page_size + 2 * (size_t)grp + (size_t)m.A * (kSegMaxSplits + 1);
+    // xs, xa, rope, red (+ norm partials), qa, kv, sc, ml (the carve above)
+    const size_t floats = (size_t)((std::max(m.d, m.A * m.D) + 3) & ~3) + (size_t)p.max_items * (kColsPerChunk + 32) +
+                          (size_t)m.D + 2 * kCW * 32 + kCW + (size_t)grp * m.D + 2 * (size_t)m.D +
+                          (size_t)grp * p.max_pps * m.page_size + 2 * (size_t)grp;
     const size_t fixed = floats * 4 + (size_t)p.n_tiles[3] + 256;
     const size_t budget = 227 * 1024;
     if (fixed + 4 * (size_t)(kSegChunk + 16) > budget) return false;
