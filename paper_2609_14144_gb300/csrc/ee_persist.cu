@@ -166,7 +166,6 @@ __device__ __forceinline__ uint32_t lds32(uint32_t a) {
     asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(a));
     return v;
 }
-__device__ __forceinline__ float ldsf(uint32_t a) { return __uint_as_float(lds32(a)); }
 
 __device__ __forceinline__ void sts64(uint32_t a, uint32_t x, uint32_t y) {
     asm volatile("st.shared.v2.b32 [%0], {%1, %2};" ::"r"(a), "r"(x), "r"(y) : "memory");
@@ -937,7 +936,7 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
             const int pg0 = sp * ag.pps, pg1 = min(ag.n_pages, pg0 + ag.pps);
             const int p0 = pg0 * m.page_size, p1 = min(ag.T, pg1 * m.page_size);
             const int npos = p1 - p0;
-            pl.probe(p.kvn + 2 * m.KH * m.D - 1, tag);  // the last value row of the Q/K/V phase
+            pl.probe(p.kvn + (m.KH + g + 1) * m.D - 1, tag);  // the last value of this group's v
             const float* qsrc = p.q + (int64_t)g * grp * m.D;
             const float* kt = p.kvn + (int64_t)g * m.D;
             const float* vt = p.kvn + (int64_t)(m.KH + g) * m.D;
@@ -1276,7 +1275,7 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
 
         // ---------------- down items: partial slots of h_out - h_mid
         if (idn.hi > idn.lo) {
-            pl.probe(p.a + m.F - 1, tag);  // the last gate/up tile's product
+            pl.probe(p.a + (idn.lo % idn.nc) * kColsPerChunk, tag);  // the first product this CTA reads
             gather4<4>(s.xa, (idn.hi - idn.lo) * kColsPerChunk, pl, [&](int e, uint32_t& bad) {
                 const int i = idn.lo + e / kColsPerChunk, col = e % kColsPerChunk;
                 const int ch = i % idn.nc, f = ch * kColsPerChunk + col;
