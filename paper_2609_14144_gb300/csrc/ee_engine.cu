@@ -225,6 +225,8 @@ struct ee_ctx {
     bool use_graphs = true, use_pdl = true;
     bool seg_ok = false, use_persistent = true;  // persistent layer kernel supported / chosen
     SegPlan seg{};
+    bool vring_ok = false;  // ring-fed vocabulary pass supported (used with the persistent layers)
+    VocabRing vring{};
     int dbg = 0;
     int conf_kind = EE_CONF_PMAX;  // signal the gates compare with tau
     int nucleus_permille = 0;      // EE_OPT_NUCLEUS: nucleus share in 1/1000, 0 = off
@@ -330,16 +332,23 @@ int enqueue_layers(ee_ctx* c, cudaStream_t s, int j0, int j1, bool& pdl) {
     return EE_OK;
 }
 
+// The vocabulary pass: ring-fed alongside the persistent layer kernel,
+// streaming otherwise.
+cudaError_t enqueue_vocab(const ee_ctx* c, const VocabArgs& v, bool pdl, cudaStream_t s) {
+    if (c->use_persistent && c->seg_ok && c->vring_ok) return launch_vocab_ring(v, c->vring, pdl, s);
+    return launch_vocab(v, c->grid_vocab, pdl, s);
+}
+
 int enqueue_readout(ee_ctx* c, cudaStream_t s, int r, int has_cond, cudaGraphConditionalHandle cond, bool& pdl) {
     const DevModel& m = c->dm;
     EE_CK(launch_readout(m, r, gemv_grid(c, m.d, m.d), gemv_whole(c, m.d, m.d), pdl, s));
     pdl = c->use_pdl;
-    EE_CK(launch_vocab(vocab_args(c, 1, r, has_cond, cond), c->grid_vocab, pdl, s));
+    EE_CK(enqueue_vocab(c, vocab_args(c, 1, r, has_cond, cond), pdl, s));
     return EE_OK;
 }
 
 int enqueue_head(ee_ctx* c, cudaStream_t s, bool& pdl) {
-    EE_CK(launch_vocab(vocab_args(c, 2, 0, 0, 0), c->grid_vocab, pdl, s));
+    EE_CK(enqueue_vocab(c, vocab_args(c, 2, 0, 0, 0), pdl, s));
     pdl = c->use_pdl;
     return EE_OK;
 }
@@ -723,6 +732,8 @@ int ee_create(const ee_model_config* cfg, void* d_workspace, size_t workspace_by
         c->seg.sync = (unsigned*)(w + l.seg_sync);
         c->seg_ok = true;
     }
+    if (vocab_ring_plan(m.d, c->n_sm, c->vring) && configure_vocab_ring(c->vring.smem) == cudaSuccess)
+        c->vring_ok = c->vring.G <= kMaxVocabCtas;
     cudaGetLastError();
 
     // RoPE table: angle t * base^(-2i/D) in double, cos/sin rounded to fp32.
@@ -1220,7 +1231,7 @@ int ee_profile_kernels(ee_ctx* c, int iters, float* ms_out) {
                 case EE_KERNEL_DOWN: return launch_down(m, j, gd, gemv_whole(c, d, F), false, s);
                 case EE_KERNEL_READOUT:
                     return launch_readout(m, i % c->n_readouts, gr, gemv_whole(c, d, d), false, s);
-                case EE_KERNEL_VOCAB: return launch_vocab(va, c->grid_vocab, false, s);
+                case EE_KERNEL_VOCAB: return enqueue_vocab(c, va, false, s);
                 case EE_KERNEL_LAYERS:
                     if (!c->seg_ok) return cudaSuccess;
                     return launch_layers(m, c->seg, 0, c->ro_layer[0], 0, s);

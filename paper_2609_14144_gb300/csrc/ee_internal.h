@@ -215,6 +215,16 @@ int layers_blocks_per_sm(size_t smem);
 // embedding of ctl->in_tok.  A cooperative launch of p.G CTAs.
 cudaError_t launch_layers(const DevModel& m, const SegPlan& p, int j0, int j1, int first, cudaStream_t s);
 
+// The vocabulary pass fed through a shared-memory ring (ee_persist.cu): one
+// CTA per SM, same arguments and results as launch_vocab with a tiled U.
+struct VocabRing {
+    int G = 0, stages = 0;
+    size_t smem = 0;
+};
+bool vocab_ring_plan(int d, int n_sm, VocabRing& vr);
+cudaError_t configure_vocab_ring(size_t smem);
+cudaError_t launch_vocab_ring(const VocabArgs& v, const VocabRing& vr, bool pdl, cudaStream_t s);
+
 // Record `msg` as the calling thread's last error and return `code`.
 int set_last_error(int code, const char* msg);
 

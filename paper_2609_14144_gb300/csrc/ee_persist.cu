@@ -40,6 +40,7 @@
 #include <algorithm>
 
 #include "ee_internal.h"
+#include "ee_vocab.cuh"
 
 namespace ee {
 namespace {
@@ -1326,6 +1327,153 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
             sync[1] = seq0 + (unsigned)(j1 - j0);
         }
     }
+}
+
+namespace {
+
+__device__ __forceinline__ void vr_pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void vr_pdl_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+// The vocabulary pass fed through the shared-memory ring: z = RMSNorm(x) *
+// gain, l = U z over the tile-packed unembedding, with the online softmax
+// statistics of every row (and, for the LM head with nucleus tracking, the
+// mass above readout 0's token), finished like the streaming pass.  One CTA
+// per SM owns whole 32-row tiles; warp 8's lane 0 streams the tiles' 32 KB
+// chunks with cp.async.bulk (it needs nothing from the previous kernel, so it
+// starts before the programmatic wait), warps 0..7 take the dot products.
+__global__ void __launch_bounds__(kSegThreads, 1) k_vocab_ring(VocabArgs v, int stages) {
+    extern __shared__ __align__(128) uint8_t vr_smem[];
+    __shared__ int err_local;  // the stall word when there is no control block
+    __shared__ float lx_s;
+    Smem s{};
+    s.ring = vr_smem;
+    s.full = reinterpret_cast<uint64_t*>(vr_smem + (size_t)stages * kSegChunk);
+    s.empty = s.full + stages;
+    float* xs = reinterpret_cast<float*>(s.empty + stages);
+    float* red = xs + ((v.d + 3) & ~3);      // [2][kCW][32], then [kCW] norm partials
+    float* part = red + 2 * kCW * 32 + kCW;  // [d / 8] partial dot products of one row
+    const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (threadIdx.x == 0) {
+        err_local = 0;
+        for (int i = 0; i < stages; ++i) {
+            mb_init(&s.full[i], 1);
+            mb_init(&s.empty[i], kCW);
+        }
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    __syncthreads();
+    volatile int* err = v.ctl ? &v.ctl->err : &err_local;
+    const int n_tiles = (v.V + kTileRows - 1) / kTileRows, nc = (v.d + kColsPerChunk - 1) / kColsPerChunk;
+    int t0, t1;
+    whole_tiles(n_tiles, gridDim.x, blockIdx.x, t0, t1);
+    const uint8_t* U = reinterpret_cast<const uint8_t*>(v.U);
+
+    if (threadIdx.x >= kCT) {  // producer
+        if (threadIdx.x != kCT) return;
+        Producer pr(s, stages, stages, err);
+        for (int t = t0; t < t1 && pr.ok; ++t)
+            for (int c = 0; c < nc; ++c)
+                pr.push(U + (int64_t)t * kTileRows * v.d * 2 + (int64_t)c * kSegChunk, chunk_bytes(v.d, c), pr.pol_w);
+        pr.drain();
+        return;
+    }
+
+    Consumer cs(s, stages, err);
+    vr_pdl_wait();
+    vr_pdl_launch();
+    // RMSNorm(x) * gain
+    float ss = 0.f;
+    for (int i = threadIdx.x; i < v.d; i += kCT) ss = fmaf(v.x[i], v.x[i], ss);
+    ss = warp_sum(ss);
+    if (lane == 0) red[2 * kCW * 32 + w] = ss;
+    csync();
+    float tot = 0.f;
+#pragma unroll
+    for (int k = 0; k < kCW; ++k) tot += red[2 * kCW * 32 + k];
+    const float inv = 1.0f / sqrtf(tot / (float)v.d + v.eps);
+    for (int i = threadIdx.x; i < v.d; i += kCT) xs[i] = v.x[i] * inv * bf(v.gain[i]);
+    csync();
+    // nucleus tracking: the logit of readout 0's token, then the mass above it
+    const bool nucleus = v.mode == 2 && v.ctl->nucleus_on && v.ctl->n_evaluated > 0;
+    int nx = -1;
+    float lx = INFINITY;
+    if (nucleus) {
+        nx = v.ctl->readout_token[0];
+        if (nx < 0 || nx >= v.V) nx = 0;  // the readout pass flags an out-of-range token
+        const int Rc = v.d >> 3, tx = nx >> 5, lx_lane = nx & 31;
+        const uint4* W = reinterpret_cast<const uint4*>(v.U);
+        for (int c = threadIdx.x; c < Rc; c += kCT) {
+            const uint4 wv = __ldg(W + ((int64_t)tx * Rc + c) * 32 + lx_lane);
+            part[c] = dot8s(wv, saddr(xs + 8 * c));
+        }
+        csync();
+        if (threadIdx.x == 0) {
+            float acc = 0.f;
+            for (int c = 0; c < Rc; ++c) acc += part[c];
+            lx_s = acc;
+        }
+        csync();
+        lx = lx_s;
+    }
+    const bool keep = v.logits && (!v.logits_if_dbg || (v.ctl && v.ctl->dbg));
+    SoftStats st;
+    int rb = 0;
+    for (int t = t0; t < t1; ++t) {
+        float acc = 0.f;
+        for (int c = 0; c < nc; ++c) {
+            const uint32_t buf = saddr(cs.acquire()) + lane * 16 + w * 512;
+            const int ccn = (int)(chunk_bytes(v.d, c) / 512);
+            const uint32_t xc = saddr(xs + c * kColsPerChunk) + w * 32;
+            if (cs.ok) acc += stage_dot<kCCPerWarp>(buf, xc, w, ccn);
+            cs.release();
+        }
+        float* r = red + rb * kCW * 32;
+        r[w * 32 + lane] = acc;
+        csync();
+        if (w == 0) {
+            float sum = 0.f;
+#pragma unroll
+            for (int k = 0; k < kCW; ++k) sum += r[k * 32 + lane];
+            const int row = t * kTileRows + lane;
+            if (row < v.V) {
+                if (keep) v.logits[row] = sum;
+                st.add(sum, row, lx, nx);
+            }
+        }
+        rb ^= 1;
+    }
+    vocab_finish(v, st, nucleus, kCW, [] { csync(); });
+}
+
+}  // namespace
+
+bool vocab_ring_plan(int d, int n_sm, VocabRing& vr) {
+    if (d % 8 || d <= 0 || n_sm <= 0) return false;
+    const size_t fixed = (size_t)(((d + 3) & ~3) + 2 * kCW * 32 + kCW + d / 8) * 4 + 1024;
+    const size_t budget = 227 * 1024;
+    if (fixed + 4 * (size_t)(kSegChunk + 16) > budget) return false;
+    vr.G = n_sm;
+    vr.stages = (int)std::min<size_t>(16, (budget - fixed) / (kSegChunk + 16));
+    vr.smem = (size_t)vr.stages * (kSegChunk + 16) + fixed - 1024;
+    return true;
+}
+
+cudaError_t configure_vocab_ring(size_t smem) {
+    return cudaFuncSetAttribute(k_vocab_ring, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+}
+
+cudaError_t launch_vocab_ring(const VocabArgs& v, const VocabRing& vr, bool pdl, cudaStream_t s) {
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3(vr.G);
+    cfg.blockDim = dim3(kSegThreads);
+    cfg.dynamicSmemBytes = vr.smem;
+    cfg.stream = s;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = pdl ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, k_vocab_ring, v, vr.stages);
 }
 
 bool seg_plan(const DevModel& m, int n_sm, SegPlan& p) {
