@@ -122,6 +122,7 @@ def _load():
             lib.orc_decode_step.argtypes = [_P, ctypes.c_int32, _P, ctypes.c_int, ctypes.POINTER(StepResult),
                                             ctypes.POINTER(Capture)]
             lib.orc_position.argtypes = [_P]
+            lib.orc_repass.argtypes = [_P, ctypes.c_int, ctypes.c_int]
             lib.orc_kv.argtypes = [_P, ctypes.c_int, ctypes.c_int, _P, _P, ctypes.POINTER(ctypes.c_int8)]
             lib.orc_stats.argtypes = [_P, _P]
             del f32p
@@ -290,6 +291,16 @@ class Oracle:
     @property
     def pos(self) -> int:
         return self.lib.orc_position(self.ptr)
+
+    def repass(self, t0: int, t1: int) -> int:
+        """Section 11's full-depth re-pass over positions [t0, t1): every
+        position there that exited runs its skipped layers from the residual it
+        exited with, replacing the filled cache entries.  Returns how many
+        positions were re-passed."""
+        n = self.lib.orc_repass(self.ptr, int(t0), int(t1))
+        if n < 0:
+            raise ValueError("bad re-pass range")
+        return n
 
     def prefill(self, ids, capture: bool = False):
         ids = np.ascontiguousarray(ids, dtype=np.int32)

@@ -29,6 +29,9 @@
  *     most probable tokens holding 90 percent of the probability); the
  *     threshold is the lowest one at which the required share of early
  *     answers is acceptable (orc_select_tau).
+ *   - Section 11: a periodic full-depth pass over the most recent tokens
+ *     recomputes their cache entries exactly (orc_repass): each token that
+ *     exited runs its skipped layers from the residual it exited with.
  *   - Appendix C: the layer is four attention projections with grouped-query
  *     attention (A query heads, K key-value heads of size D) and a gated
  *     feed-forward block of three matrices of width F.
@@ -141,6 +144,8 @@ typedef struct {
     float* kc;       /* [L][K][max_ctx][D], bf16 values */
     float* vc;
     int8_t* kv_src;  /* [L][max_ctx]: 0 empty, 1 computed by the layer, 2 filled */
+    float* h_exit;   /* [max_ctx][d]: the residual a position exited with */
+    int16_t* exit_at; /* [max_ctx]: layer a position exited after (0: ran every layer) */
     int pos;
     int conf_kind; /* ORC_CONF_*: the signal the gate compares with tau */
     double nucleus_p; /* share of probability the nucleus holds */
@@ -377,6 +382,8 @@ void orc_free(orc_model* m) {
     free(m->kc);
     free(m->vc);
     free(m->kv_src);
+    free(m->h_exit);
+    free(m->exit_at);
     free(m->h); free(m->u); free(m->q); free(m->kk); free(m->vv); free(m->o);
     free(m->g); free(m->up); free(m->a); free(m->y); free(m->z); free(m->logits); free(m->tmp);
     free(m);
@@ -415,6 +422,8 @@ orc_model* orc_create(const orc_config* c, const orc_weights* w) {
     m->kc = (float*)calloc(kvn, sizeof(float));
     m->vc = (float*)calloc(kvn, sizeof(float));
     m->kv_src = (int8_t*)calloc((size_t)L * c->max_ctx, 1);
+    m->h_exit = (float*)calloc((size_t)c->max_ctx * c->d_model, 4);
+    m->exit_at = (int16_t*)calloc((size_t)c->max_ctx, 2);
     const size_t d = (size_t)c->d_model, qd = (size_t)c->n_heads * c->head_dim,
                  kd = (size_t)c->n_kv_heads * c->head_dim, F = (size_t)c->ffn_dim;
     const size_t big = d > qd ? d : qd;
@@ -431,7 +440,7 @@ orc_model* orc_create(const orc_config* c, const orc_weights* w) {
     m->z = (float*)calloc(d, 4);
     m->logits = (float*)calloc((size_t)c->vocab, 4);
     m->tmp = (float*)calloc(big > F ? big : F, 4);
-    if (!m->kc || !m->vc || !m->kv_src || !m->logits || !m->tmp) {
+    if (!m->kc || !m->vc || !m->kv_src || !m->h_exit || !m->exit_at || !m->logits || !m->tmp) {
         orc_free(m);
         return NULL;
     }
@@ -455,6 +464,7 @@ void orc_reset(orc_model* m) {
     memset(m->kc, 0, kvn * sizeof(float));
     memset(m->vc, 0, kvn * sizeof(float));
     memset(m->kv_src, 0, (size_t)c->n_layers * c->max_ctx);
+    memset(m->exit_at, 0, (size_t)c->max_ctx * 2);
     m->pos = 0;
     m->steps = m->full_steps = 0;
     memset(m->exits, 0, sizeof(m->exits));
@@ -641,6 +651,8 @@ int orc_decode_step(orc_model* m, int32_t in_tok, const float* taus, int force, 
                 res->exit_layer = j + 1;
                 res->token = cf.argmax;
                 for (int jj = j + 1; jj < L; ++jj) kv_fill(m, jj, t, m->h);
+                memcpy(m->h_exit + (size_t)t * d, m->h, sizeof(float) * d);
+                m->exit_at[t] = (int16_t)(j + 1);
             }
             ++r;
         }
@@ -670,6 +682,28 @@ int orc_decode_step(orc_model* m, int32_t in_tok, const float* taus, int force, 
 }
 
 int orc_position(const orc_model* m) { return m->pos; }
+
+/* Section 11's full-depth re-pass: for each position t in [t0, t1), in
+ * order, whose upper layers still hold filled entries (it exited after layer
+ * k, kv_src[k][t] == 2), run layers k+1..L from the residual it exited with,
+ * storing computed entries in place of the filled ones.  Attention at t sees
+ * the cache as it stands, including positions re-passed just before.  The
+ * decode position is unchanged.  Returns the number of positions re-passed
+ * (-1 on a bad range). */
+int orc_repass(orc_model* m, int t0, int t1) {
+    if (!m || t0 < 0 || t1 < t0 || t1 > m->pos) return -1;
+    const orc_config* c = &m->c;
+    const int d = c->d_model, L = c->n_layers;
+    int n = 0;
+    for (int t = t0; t < t1; ++t) {
+        const int k = m->exit_at[t];
+        if (k <= 0 || k >= L || m->kv_src[(size_t)k * c->max_ctx + t] != 2) continue;
+        memcpy(m->y, m->h_exit + (size_t)t * d, sizeof(float) * d);
+        for (int j = k; j < L; ++j) layer_forward(m, j, t, m->y, NULL);
+        ++n;
+    }
+    return n;
+}
 
 /* Copy the cached K and V (all key-value heads, [K*D] each) of layer j
  * (0-based) at position t, and the entry's origin (0/1/2). */

@@ -249,6 +249,74 @@ def test_nucleus_membership_of_the_readout_answer():
         o.set_nucleus(0.0)
 
 
+def _exit_run(shape, model, n, every=3, extra=0):
+    """Decode n steps with exits imposed at readout 0 on all but every
+    `every`-th step; returns (oracle, input tokens of the steps)."""
+    o = oracle.Oracle(shape, model, max_ctx=shape.prompt_len + n + extra)
+    tok = o.prefill(synth.prompt(shape))
+    ins = []
+    for i in range(n):
+        ins.append(tok)
+        s = o.decode_step(tok, [2.0], oracle.FORCE_FULL if i % every == 0 else oracle.FORCE_EXIT_AT(0))
+        tok = s["token"]
+    return o, ins
+
+
+def _cache(o, shape, t0, t1):
+    return [[o.kv(j, t) for t in range(t0, t1)] for j in range(shape.n_layers)]
+
+
+def test_repass_reproduces_the_full_depth_cache():
+    """Section 11: re-passing every exited position, in order, recomputes
+    the cache the full model would hold for the same tokens, bit for bit."""
+    n = 20
+    model = synth.make_model(TINY)
+    o, ins = _exit_run(TINY, model, n)
+    P = TINY.prompt_len
+    assert o.repass(P, P + n) == n - len(range(0, n, 3))
+    full = oracle.Oracle(TINY, model, max_ctx=P + n)
+    full.prefill(synth.prompt(TINY))
+    for tok in ins:
+        full.decode_step(tok, [2.0], oracle.FORCE_FULL)
+    for j in range(TINY.n_layers):
+        for t in range(P + n):
+            ko, vo, so = o.kv(j, t)
+            kf, vf, sf = full.kv(j, t)
+            assert so == sf == 1, (j, t, so, sf)
+            assert np.array_equal(ko, kf) and np.array_equal(vo, vf), (j, t)
+    assert o.repass(P, P + n) == 0  # nothing left to re-pass
+
+
+def test_repass_of_a_range_changes_only_that_range():
+    n = 24
+    model = synth.make_model(TINY)
+    o, _ = _exit_run(TINY, model, n, every=4, extra=1)
+    P, L = TINY.prompt_len, TINY.n_layers
+    before = _cache(o, TINY, 0, P + n)
+    t0, t1 = P + 8, P + 16
+    assert o.repass(t0, t1) == 6
+    after = _cache(o, TINY, 0, P + n)
+    k0 = TINY.readout_layers[0]
+    for j in range(L):
+        for t in range(P + n):
+            kb, vb, sb = before[j][t]
+            ka, va, sa = after[j][t]
+            inside = t0 <= t < t1 and j >= k0 and sb == 2
+            if inside:
+                assert sa == 1  # now computed by the layer
+                same = np.array_equal(ka, kb) and np.array_equal(va, vb)
+                # the first skipped layer's input is the exit residual itself, so
+                # its fill was already exact; the layers above it change
+                assert same == (j == k0), (j, t)
+            else:
+                assert sa == sb and np.array_equal(ka, kb) and np.array_equal(va, vb), (j, t)
+    # the decode goes on from where it was
+    assert o.pos == P + n
+    o.decode_step(1, [2.0], oracle.FORCE_FULL)
+    with pytest.raises(ValueError):
+        o.repass(P, P + n + 5)
+
+
 # ------------------------------------------------------------- structure
 def _trace_step(shape, model, force=oracle.FORCE_FULL, taus=(0.5,)):
     o = oracle.Oracle(shape, model)
