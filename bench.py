@@ -47,6 +47,7 @@ UNIT = "tokens/s"
 WORKLOAD = "1.5b"
 HEADLINE_RATE = 0.5
 CALIB_TOKENS = 2048
+REPASS_W = 16  # positions in the measured full-depth re-pass
 CTL_BYTES = 360  # device control block read back by a host-buffer ee_decode_n
 
 
@@ -486,6 +487,24 @@ def run_ours(args, rank: int, world: int, local: int):
         eng_plain.close()
         del eng_plain
 
+    # Section 11's full-depth re-pass: decode REPASS_W tokens with every
+    # step exiting, then time one re-pass of them (ee_repass)
+    repass = None
+    if not args.no_sweep:
+        eng.reset()
+        eng.prefill(prompt)
+        sched = np.full(REPASS_W, FORCE_EXIT_AT(0), np.int8)
+        eng.decode_n(REPASS_W, [0.5], schedule=sched)
+        p1 = eng.position
+        torch.cuda.synchronize(local)
+        t0 = time.perf_counter()
+        n_rp = eng.repass(p1 - REPASS_W, p1)
+        dt = time.perf_counter() - t0
+        repass = {"positions": REPASS_W, "repassed": n_rp, "ms": dt * 1e3,
+                  "token_times": dt * head["tok_s"],
+                  "note": "one upper-segment launch per re-passed position (not batched)"}
+        _log(f"[bench] re-pass of {n_rp} exited positions: {dt * 1e3:.2f} ms ({dt * head['tok_s']:.1f} token-times)")
+
     # end to end through the host-buffer API
     e2e = run.run_host([tau_h], W, K)
 
@@ -535,6 +554,7 @@ def run_ours(args, rank: int, world: int, local: int):
         "sweep": sweep,
         "plain_model": plain_line,
         "calibration": cal,
+        "repass": repass,
     }
     eng.close()
     if rank == 0:

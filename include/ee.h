@@ -218,6 +218,19 @@ int ee_decode_n(ee_ctx* ctx, int n, int32_t input_token, const float* taus, cons
 int ee_calibrate(ee_ctx* ctx, const int32_t* ids, int n, float p_nuc, float* conf, int32_t* member, float* mass,
                  int where);
 
+/* Full-depth re-pass over recent tokens (Section 11): every position t in
+ * [t0, t1) whose upper-layer cache entries are still the fills of an early
+ * exit runs those layers again, in position order, from the residual it
+ * exited with (kept by the exit step), so that their entries become the ones
+ * the full model computes given the cache before them (exactly the full
+ * model's when every earlier exited position has been re-passed).  Positions
+ * that ran at full depth are skipped.  The decode position and the next input
+ * token are unchanged; the final hidden state read by EE_DBG_HIDDEN_FINAL is
+ * the last re-passed position's.  *n_repassed (may be NULL) receives the number
+ * of positions re-passed.  Synchronous.  EE_ERANGE unless 0 <= t0 <= t1 <=
+ * position; EE_ESTATE before prefill.  See also EE_OPT_REPASS. */
+int ee_repass(ee_ctx* ctx, int32_t t0, int32_t t1, int32_t* n_repassed);
+
 /* Wait for the context's stream and report the device error word. */
 int ee_sync(ee_ctx* ctx);
 int ee_get_stats(ee_ctx* ctx, ee_stats* out);
@@ -241,6 +254,11 @@ int ee_position(ee_ctx* ctx, int32_t* pos);
                                  CTA per SM streaming weights through a shared-
                                  memory ring; 0: five launches per layer.
                                  EE_EINVAL if the shape is not supported      */
+#define EE_OPT_REPASS 7       /* 0 (default): off; P > 0: ee_decode_n re-passes
+                                 (ee_repass) the P positions decoded since the
+                                 last re-pass every P steps (Section 11's
+                                 periodic full-depth pass); the call then
+                                 synchronises at each re-pass              */
 #define EE_OPT_NUCLEUS 6      /* 0 (default): off; 1..1000: full-depth steps of
                                  ee_decode_step report the nucleus membership of
                                  readout 0's token at share value/1000

@@ -12,8 +12,8 @@ import numpy as np
 
 from . import _lib
 from ._lib import (CONF_MARGIN, CONF_NEGENT, CONF_PMAX, DEVICE, FORCE_FULL, FREE, HOST, MAX_READOUTS,
-                   OPT_CONFIDENCE, OPT_DEBUG_LOGITS, OPT_GRAPHS, OPT_NUCLEUS, OPT_PDL, OPT_PERSISTENT, EEError,
-                   FORCE_EXIT_AT, check)
+                   OPT_CONFIDENCE, OPT_DEBUG_LOGITS, OPT_GRAPHS, OPT_NUCLEUS, OPT_PDL, OPT_PERSISTENT, OPT_REPASS,
+                   EEError, FORCE_EXIT_AT, check)
 
 __all__ = ["Engine", "EEError", "FREE", "FORCE_FULL", "FORCE_EXIT_AT", "HOST", "DEVICE", "attention_decode",
            "vocab_confidence", "vocab_signals", "select_tau", "library_path"]
@@ -197,6 +197,13 @@ class Engine:
         check(self.lib.ee_calibrate(self.ctx, ids.data_ptr(), int(n), float(p_nuc), conf.data_ptr(),
                                     member.data_ptr(), mass.data_ptr(), DEVICE))
         return conf, member, mass
+
+    def repass(self, t0: int, t1: int) -> int:
+        """Section 11's full-depth re-pass over positions [t0, t1): returns the
+        number of exited positions whose skipped layers were run again."""
+        n = ctypes.c_int32(0)
+        check(self.lib.ee_repass(self.ctx, int(t0), int(t1), ctypes.byref(n)))
+        return n.value
 
     def sync(self):
         check(self.lib.ee_sync(self.ctx))

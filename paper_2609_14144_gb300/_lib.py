@@ -10,7 +10,7 @@ MAX_READOUTS = 8
 EE_OK, EE_EINVAL, EE_ENOMEM, EE_ECUDA, EE_ERANGE, EE_EDEVICE, EE_ESTATE = 0, -1, -2, -3, -4, -5, -6
 FREE, FORCE_FULL = 0, 1
 HOST, DEVICE = 0, 1
-OPT_GRAPHS, OPT_PDL, OPT_DEBUG_LOGITS, OPT_PERSISTENT, OPT_CONFIDENCE, OPT_NUCLEUS = 1, 2, 3, 4, 5, 6
+OPT_GRAPHS, OPT_PDL, OPT_DEBUG_LOGITS, OPT_PERSISTENT, OPT_CONFIDENCE, OPT_NUCLEUS, OPT_REPASS = 1, 2, 3, 4, 5, 6, 7
 CONF_PMAX, CONF_MARGIN, CONF_NEGENT = 0, 1, 2
 DBG_HIDDEN_READOUT, DBG_READOUT_Y, DBG_HIDDEN_FINAL, DBG_READOUT_LOGITS, DBG_FINAL_LOGITS, DBG_KV, DBG_KV_SRC = \
     1, 2, 3, 4, 5, 6, 7
@@ -20,7 +20,7 @@ SYMBOLS = ("ee_workspace_bytes", "ee_create", "ee_destroy", "ee_last_error", "ee
            "ee_set_page_table", "ee_reset", "ee_prefill", "ee_decode_step", "ee_decode_n", "ee_sync",
            "ee_get_stats", "ee_position", "ee_set_option", "ee_debug_read", "ee_attention_scratch_bytes",
            "ee_attention_decode", "ee_vocab_scratch_bytes", "ee_vocab_confidence", "ee_vocab_signals", "ee_profile_kernels",
-           "ee_attention_decode_static", "ee_calibrate", "ee_select_tau")
+           "ee_attention_decode_static", "ee_calibrate", "ee_select_tau", "ee_repass")
 KERNELS = ("qkv", "attention", "oproj", "gateup", "down", "readout", "vocab", "kvfill", "layers")
 
 
@@ -115,6 +115,7 @@ def load(allow_build: bool = False):
     lib.ee_profile_kernels.argtypes = [_P, ctypes.c_int, _P]
     lib.ee_attention_decode_static.argtypes = [_P, _P, _P, _P, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
                                                ctypes.c_int, _P, _P]
+    lib.ee_repass.argtypes = [_P, i32, i32, ctypes.POINTER(i32)]
     lib.ee_calibrate.argtypes = [_P, _P, ctypes.c_int, ctypes.c_float, _P, _P, _P, ctypes.c_int]
     lib.ee_select_tau.argtypes = [_P, ctypes.c_int, _P, ctypes.c_int, ctypes.c_float, _P, _P, _P]
     for name in SYMBOLS:

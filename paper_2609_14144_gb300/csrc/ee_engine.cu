@@ -56,7 +56,7 @@ int64_t align_elems(int64_t x) { return (x + 127) / 128 * 128; }  // 256 bytes o
 // Byte offsets of every region of the workspace.
 struct Layout {
     size_t ctl, rope, layers, embed, lm_head, g_final, ro_w[kMaxReadouts], ro_b[kMaxReadouts];
-    size_t kpool, vpool, page_table, kv_src, h, q, o, a, y, hk, logits_ro, logits_final;
+    size_t kpool, vpool, page_table, kv_src, h_exit, exit_at, repass_pos, h, q, o, a, y, hk, logits_ro, logits_final;
     size_t gemv_part, gemv_ticket, attn_part, attn_ticket, vocab_part, vocab_ticket;
     size_t seg_dpart, seg_opart, seg_q, seg_kvn, seg_a, seg_attn, seg_sync, seg_end;
     size_t prompt, sched, out_tok, out_exit, out_conf, out_conf_all, out_member, out_mass, tau_scratch, total;
@@ -134,6 +134,9 @@ Layout make_layout(const ee_model_config& c) {
     l.vpool = take(2 * (size_t)l.kv_layer_stride * L);
     l.page_table = take(4 * (size_t)l.n_pages);
     l.kv_src = take((size_t)L * c.max_ctx);
+    l.h_exit = take(4 * (size_t)c.max_ctx * d);
+    l.exit_at = take(2 * (size_t)c.max_ctx);
+    l.repass_pos = take(4 * ((size_t)c.max_ctx + 1));
     l.h = take(4 * (size_t)d);
     l.q = take(4 * (size_t)A * D);
     l.o = take(4 * (size_t)A * D);
@@ -229,6 +232,8 @@ struct ee_ctx {
     VocabRing vring{};
     int dbg = 0;
     int conf_kind = EE_CONF_PMAX;  // signal the gates compare with tau
+    int repass_period = 0;         // EE_OPT_REPASS: re-pass every this many decode steps (0 = off)
+    int repass_from = 0;           // first position the periodic re-pass has not covered
     int nucleus_permille = 0;      // EE_OPT_NUCLEUS: nucleus share in 1/1000, 0 = off
     cudaGraphExec_t g_step = nullptr, g_n = nullptr, g_prefill = nullptr;
     int grid_gemv = 0, grid_vocab = 0;
@@ -587,6 +592,50 @@ CtlInputs base_inputs(const ee_ctx* c, const float* taus) {
     return in;
 }
 
+// Section 11's full-depth re-pass over positions [t0, t1) (t1 <= pos): each
+// position whose upper layers still hold filled entries runs them again from
+// the residual it exited with (h_exit), in position order, through the same
+// layer kernels as a decode step; the control block's position is pointed at
+// each one in turn and restored at the end.  Synchronous.
+int repass_range(ee_ctx* c, int t0, int t1, int* n_done) {
+    cudaStream_t s = c->stream;
+    const DevModel& m = c->dm;
+    const int L = m.L, W = t1 - t0;
+    if (n_done) *n_done = 0;
+    if (W <= 0) return EE_OK;
+    EE_CK(cudaStreamSynchronize(s));
+    std::vector<int16_t> ex(W);
+    std::vector<int8_t> src((size_t)L * W);
+    EE_CK(cudaMemcpy(ex.data(), m.exit_at + t0, 2 * (size_t)W, cudaMemcpyDeviceToHost));
+    for (int j = 0; j < L; ++j)
+        EE_CK(cudaMemcpy(src.data() + (size_t)j * W, m.kv_src + (int64_t)j * m.max_ctx + t0, (size_t)W,
+                         cudaMemcpyDeviceToHost));
+    std::vector<int32_t> todo, from;
+    for (int i = 0; i < W; ++i) {
+        const int k = ex[i];
+        if (k >= 1 && k < L && src[(size_t)k * W + i] == 2) {
+            todo.push_back(t0 + i);
+            from.push_back(k);
+        }
+    }
+    if (todo.empty()) return EE_OK;
+    int32_t* d_pos = (int32_t*)(c->ws + c->lay.repass_pos);  // the positions, then the decode position
+    std::vector<int32_t> pos_list(todo);
+    pos_list.push_back(c->pos);
+    EE_CK(cudaMemcpy(d_pos, pos_list.data(), 4 * pos_list.size(), cudaMemcpyHostToDevice));
+    for (size_t i = 0; i < todo.size(); ++i) {
+        EE_CK(cudaMemcpyAsync(m.h, m.h_exit + (int64_t)todo[i] * m.d, 4 * (size_t)m.d, cudaMemcpyDeviceToDevice, s));
+        EE_CK(cudaMemcpyAsync(&c->d_ctl->pos, d_pos + i, 4, cudaMemcpyDeviceToDevice, s));
+        bool pdl = false;
+        EE_TRY(enqueue_layers(c, s, from[i], L, pdl));
+    }
+    EE_CK(cudaMemcpyAsync(&c->d_ctl->pos, d_pos + todo.size(), 4, cudaMemcpyDeviceToDevice, s));
+    EE_TRY(fetch_ctl(c));
+    EE_TRY(device_error(c));
+    if (n_done) *n_done = (int)todo.size();
+    return EE_OK;
+}
+
 // Direct launches with the branch taken on the host (EE_OPT_GRAPHS = 0).
 int eager_step(ee_ctx* c) {
     cudaStream_t s = c->stream;
@@ -700,6 +749,8 @@ int ee_create(const ee_model_config* cfg, void* d_workspace, size_t workspace_by
     m.kv_layer_stride = l.kv_layer_stride;
     m.page_table = (const int32_t*)(w + l.page_table);
     m.kv_src = (int8_t*)(w + l.kv_src);
+    m.h_exit = (float*)(w + l.h_exit);
+    m.exit_at = (int16_t*)(w + l.exit_at);
     m.h = (float*)(w + l.h);
     m.q = (float*)(w + l.q);
     m.o = (float*)(w + l.o);
@@ -891,11 +942,13 @@ int ee_reset(ee_ctx* c) {
     c->h_ctl->max_ctx = c->cfg.max_ctx;
     EE_CK(cudaMemcpyAsync(c->d_ctl, c->h_ctl, sizeof(Ctl), cudaMemcpyHostToDevice, c->stream));
     EE_CK(cudaMemsetAsync(c->ws + c->lay.kv_src, 0, (size_t)c->cfg.n_layers * c->cfg.max_ctx, c->stream));
+    EE_CK(cudaMemsetAsync(c->ws + c->lay.exit_at, 0, 2 * (size_t)c->cfg.max_ctx, c->stream));
     // the persistent layer kernel's exchange buffers (tags 0: never valid),
     // exit ticket and launch count
     EE_CK(cudaMemsetAsync(c->ws + c->lay.seg_dpart, 0, c->lay.seg_end - c->lay.seg_dpart, c->stream));
     EE_CK(cudaStreamSynchronize(c->stream));
     c->pos = 0;
+    c->repass_from = 0;
     c->prefilled = false;
     return EE_OK;
 }
@@ -916,6 +969,11 @@ int ee_set_option(ee_ctx* c, int option, int value) {
         case EE_OPT_CONFIDENCE:
             if (value < EE_CONF_PMAX || value > EE_CONF_NEGENT) return fail(EE_EINVAL, "unknown confidence signal");
             c->conf_kind = value;
+            return EE_OK;
+        case EE_OPT_REPASS:
+            if (value < 0) return fail(EE_EINVAL, "re-pass period must be >= 0");
+            c->repass_period = value;
+            c->repass_from = c->pos;
             return EE_OK;
         case EE_OPT_NUCLEUS:
             if (value < 0 || value > 1000) return fail(EE_EINVAL, "nucleus share must be 0..1000 per mille");
@@ -967,6 +1025,7 @@ int ee_prefill(ee_ctx* c, const int32_t* ids, int n, int32_t* first_token) {
     c->pos = c->h_ctl->pos;
     if (c->pos != n) return fail(EE_EDEVICE, "prefill ended at an unexpected position");
     c->prefilled = true;
+    c->repass_from = n;
     if (first_token) *first_token = c->h_ctl->token;
     return EE_OK;
 }
@@ -1026,36 +1085,42 @@ int ee_decode_n(ee_ctx* c, int n, int32_t input_token, const float* taus, const 
             if (force_schedule[i] < 0 || force_schedule[i] > 1 + c->n_readouts)
                 return fail(EE_EINVAL, "bad force schedule entry");
     cudaStream_t s = c->stream;
-    CtlInputs in = base_inputs(c, taus);
-    in.set_token = input_token >= 0;
-    in.in_tok = input_token;
-    in.force = EE_FREE;
-    in.n_steps = n;
-    if (force_schedule) {
-        int8_t* d_sched = (int8_t*)(c->ws + c->lay.sched);
-        EE_CK(cudaMemcpyAsync(d_sched, force_schedule, (size_t)n, cudaMemcpyHostToDevice, s));
-        in.sched = d_sched;
-    }
+    int8_t* d_sched = (int8_t*)(c->ws + c->lay.sched);
+    if (force_schedule) EE_CK(cudaMemcpyAsync(d_sched, force_schedule, (size_t)n, cudaMemcpyHostToDevice, s));
     int32_t* d_tok = (int32_t*)(c->ws + c->lay.out_tok);
     int32_t* d_exit = (int32_t*)(c->ws + c->lay.out_exit);
     float* d_conf = (float*)(c->ws + c->lay.out_conf);
-    if (where == EE_DEVICE) {
-        in.out_tokens = tokens;
-        in.out_exit = exit_readout;
-        in.out_conf = confidence;
-    } else {
-        in.out_tokens = tokens ? d_tok : nullptr;
-        in.out_exit = exit_readout ? d_exit : nullptr;
-        in.out_conf = confidence ? d_conf : nullptr;
+    int32_t* o_tok = where == EE_DEVICE ? tokens : (tokens ? d_tok : nullptr);
+    int32_t* o_exit = where == EE_DEVICE ? exit_readout : (exit_readout ? d_exit : nullptr);
+    float* o_conf = where == EE_DEVICE ? confidence : (confidence ? d_conf : nullptr);
+    // In runs of steps; with a re-pass period, each run ends where the next
+    // periodic re-pass (Section 11) falls due.
+    for (int done = 0; done < n;) {
+        int len = n - done;
+        if (c->repass_period > 0) len = std::min(len, std::max(1, c->repass_from + c->repass_period - c->pos));
+        CtlInputs in = base_inputs(c, taus);
+        in.set_token = done == 0 && input_token >= 0;
+        in.in_tok = input_token;
+        in.force = EE_FREE;
+        in.n_steps = len;
+        in.sched = force_schedule ? d_sched + done : nullptr;
+        in.out_tokens = o_tok ? o_tok + done : nullptr;
+        in.out_exit = o_exit ? o_exit + done : nullptr;
+        in.out_conf = o_conf ? o_conf + done : nullptr;
+        EE_CK(launch_set_inputs(c->d_ctl, in, s));
+        if (c->use_graphs) {
+            EE_TRY(ensure_graphs(c));
+            EE_CK(cudaGraphLaunch(c->g_n, s));
+        } else {
+            for (int i = 0; i < len; ++i) EE_TRY(eager_step(c));
+        }
+        c->pos += len;
+        done += len;
+        if (c->repass_period > 0 && c->pos - c->repass_from >= c->repass_period) {
+            EE_TRY(repass_range(c, c->repass_from, c->pos, nullptr));
+            c->repass_from = c->pos;
+        }
     }
-    EE_CK(launch_set_inputs(c->d_ctl, in, s));
-    if (c->use_graphs) {
-        EE_TRY(ensure_graphs(c));
-        EE_CK(cudaGraphLaunch(c->g_n, s));
-    } else {
-        for (int i = 0; i < n; ++i) EE_TRY(eager_step(c));
-    }
-    c->pos += n;
     if (where == EE_HOST) {
         if (tokens) EE_CK(cudaMemcpyAsync(tokens, d_tok, 4 * (size_t)n, cudaMemcpyDeviceToHost, s));
         if (exit_readout) EE_CK(cudaMemcpyAsync(exit_readout, d_exit, 4 * (size_t)n, cudaMemcpyDeviceToHost, s));
@@ -1125,6 +1190,16 @@ int ee_calibrate(ee_ctx* c, const int32_t* ids, int n, float p_nuc, float* conf,
         EE_TRY(device_error(c));
         if (c->h_ctl->pos != c->pos) return fail(EE_EDEVICE, "device position out of step with the host");
     }
+    return EE_OK;
+}
+
+int ee_repass(ee_ctx* c, int32_t t0, int32_t t1, int32_t* n_repassed) {
+    if (!c) return fail(EE_EINVAL, "NULL context");
+    if (!c->prefilled) return fail(EE_ESTATE, "re-pass before prefill");
+    if (t0 < 0 || t1 < t0 || t1 > c->pos) return fail(EE_ERANGE, "re-pass range outside [0, position]");
+    int n = 0;
+    EE_TRY(repass_range(c, t0, t1, &n));
+    if (n_repassed) *n_repassed = n;
     return EE_OK;
 }
 

@@ -83,6 +83,8 @@ struct DevModel {
     int64_t kv_layer_stride;      // elements per layer in a pool
     const int32_t* page_table;    // [n_pages]
     int8_t* kv_src;               // [L][max_ctx]
+    float* h_exit;                // [max_ctx][d] residual each position exited with
+    int16_t* exit_at;             // [max_ctx] first filled layer of an exited position
     float* h;                     // residual stream [d]
     float* q;                     // rotated queries [A*D]
     float* o;                     // attention output [A*D]

@@ -663,6 +663,10 @@ __global__ void __launch_bounds__(kGemvThreads, 2) k_kvfill(DevModel m, int exit
     coop_finish(r, sm_part, m.gemv_part, blockIdx.y * gridDim.x, m.gemv_ticket + blockIdx.y * m.gemv_ticket_stride,
                 epi);
     if (blockIdx.x == 0 && threadIdx.x == 0) m.kv_src[(int64_t)j * m.max_ctx + pos] = 2;
+    if (blockIdx.x == 0 && blockIdx.y == 0) {  // what a later full-depth re-pass starts from
+        for (int i = threadIdx.x; i < m.d; i += blockDim.x) m.h_exit[(int64_t)pos * m.d + i] = m.h[i];
+        if (threadIdx.x == 0) m.exit_at[pos] = (int16_t)exit_layer;
+    }
 }
 
 // Output projection with the residual add: h += W_o o.
