@@ -965,20 +965,36 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
             const int spc = p.max_pps * m.page_size;  // score row stride
             const int npair = m.D >> 5;               // pairs of k16 steps (32 dimensions)
             const int g8 = lane >> 2, t4 = lane & 3;
+            // The group's queries as bf16 high and low parts, converted once
+            // into rows padded to 16 bytes past D (xs is free here), so that the
+            // fragment loads of 8 heads at one column fall in different banks.
+            {
+                const int qrow = m.D + 8;
+                uint16_t* qhs = reinterpret_cast<uint16_t*>(s.xs);
+                uint16_t* qls = qhs + grp * qrow;
+                for (int e = threadIdx.x; e < nqa / 4; e += kCT) {
+                    const float4 q4 = lds128f(saddr(s.qa + 4 * e));
+                    const int h = (4 * e) / m.D, c = 4 * e - h * m.D;
+                    uint32_t h01, l01, h23, l23;
+                    split_bf16x2(q4.x, q4.y, h01, l01);
+                    split_bf16x2(q4.z, q4.w, h23, l23);
+                    sts64(saddr(qhs + h * qrow + c), h01, h23);
+                    sts64(saddr(qls + h * qrow + c), l01, l23);
+                }
+                csync();
+            }
             uint32_t qhi[4][4], qlo[4][4];  // [pair][word]: dimensions pair*32 + 8 t4 .. +7 of query g8
 #pragma unroll
             for (int pr = 0; pr < 4; ++pr) {
-                float x[8];
                 if (pr < npair && g8 < grp) {
-                    const float* qrow = s.qa + g8 * m.D + pr * 32 + 8 * t4;
-                    const float4 a = lds128f(saddr(qrow)), b = lds128f(saddr(qrow + 4));
-                    x[0] = a.x, x[1] = a.y, x[2] = a.z, x[3] = a.w, x[4] = b.x, x[5] = b.y, x[6] = b.z, x[7] = b.w;
+                    const uint16_t* qhs = reinterpret_cast<const uint16_t*>(s.xs) + g8 * (m.D + 8) + pr * 32 + 8 * t4;
+                    const uint4 a = lds128(saddr(qhs)), b = lds128(saddr(qhs + grp * (m.D + 8)));
+                    qhi[pr][0] = a.x, qhi[pr][1] = a.y, qhi[pr][2] = a.z, qhi[pr][3] = a.w;
+                    qlo[pr][0] = b.x, qlo[pr][1] = b.y, qlo[pr][2] = b.z, qlo[pr][3] = b.w;
                 } else {
 #pragma unroll
-                    for (int k = 0; k < 8; ++k) x[k] = 0.f;
+                    for (int wd = 0; wd < 4; ++wd) qhi[pr][wd] = qlo[pr][wd] = 0u;
                 }
-#pragma unroll
-                for (int wd = 0; wd < 4; ++wd) split_bf16x2(x[2 * wd], x[2 * wd + 1], qhi[pr][wd], qlo[pr][wd]);
             }
             for (int pg = pg0; pg < pg1; ++pg)
                 for (int q = 0; q < cpp; ++q) {

@@ -11,7 +11,7 @@ import pytest
 
 import oracle
 import synth
-from helpers import P_TOL, check_kv, check_records, is_excluded, teacher_forced
+from helpers import P_TOL, check_kv, check_records, is_excluded, rel_err, teacher_forced
 
 pytestmark = pytest.mark.gpu
 
@@ -57,6 +57,26 @@ def test_tiny_permuted_pages(tiny_model):
     assert fo == fg
     check_records(recs, [0.5])
     check_kv(orc, eng, TINY, TINY.max_ctx)
+
+
+@pytest.mark.parametrize("prompt_len,n", [(500, 24), (1000, 40)])
+def test_tiny_attention_split_geometry_changes(tiny_model, prompt_len, n):
+    """16-position pages: past 512 and 1024 positions the pages per attention
+    split grow and the split count drops (32 -> 17, 32 -> 22), so split slots
+    fall out of use and come back later; their partials must never be taken
+    from an earlier layer or launch."""
+    shape = TINY.replace(prompt_len=prompt_len)
+    prompt = synth.prompt(shape)
+    fo, fg, recs, orc, eng = teacher_forced(shape, tiny_model, n, [0.5], prompt=prompt, page_size=16,
+                                            capture=False)
+    assert fo == fg
+    assert check_records(recs, [0.5], capture=False) <= n // 8
+    for j in (0, TINY.n_layers - 1):
+        for t in range(prompt_len - 4, prompt_len + n):
+            ko, vo, so = orc.kv(j, t)
+            kg, vg = eng.kv(j, t)
+            assert eng.kv_src(j, t) == so
+            assert rel_err(kg, ko) <= 1e-2 and rel_err(vg, vo) <= 1e-2, (j, t)
 
 
 def test_tiny_bias_and_tied_head():
