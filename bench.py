@@ -543,7 +543,9 @@ def run_ours(args, rank: int, world: int, local: int):
         "config": {"workload": _workload_desc(shape), "tokens_per_step": C, "exit_rate_target": HEADLINE_RATE,
                    "tau": tau_h, "exit_rate": head["exit_rate"], "parallelism": f"replicas x{world}",
                    "l2": "inputs larger than L2: every token streams 1.8-3.6 GB of weights",
-                   "numerics": "bf16 weights and KV cache, fp32 activations and accumulation"},
+                   "numerics": "bf16 weights and KV cache, fp32 activations and accumulation (values exchanged "
+                               "between CTAs rounded to 19 significant bits; attention scores from bf16 high/low query "
+                               "parts on the tensor cores)"},
         "e2e": {"value": e2e, "unit": UNIT, "h2d_bytes_per_step": 4 * 8,
                 "d2h_bytes_per_step": 12 * C + CTL_BYTES},
         "gpu_launches": head["launches"],
