@@ -200,12 +200,12 @@ struct SegPlan {
     // Values handed between CTAs, each float carrying its layer's tag in
     // the low mantissa bits (zero after ee_reset):
     float* dpart;           // down-projection partials [tile][n_chunks][32]
-    float* opart;           // O-projection chunk partials [2][tile][n_chunks][32] (by layer parity)
+    float* opart;           // O-projection chunk partials [2][tile][n_chunks][32] (by the layer count's parity)
     float* attn_part;       // [A][kSegMaxSplits][D + 4]: unnormalised o, max, sum per split
     float* q;               // [A D] rotated queries
     float* kvn;             // [2][KH D] the step's k and v (bf16 values)
     float* a;               // [F] SwiGLU product
-    unsigned* sync;         // [0] exit ticket (zero between launches), [1] launches since ee_reset
+    unsigned* sync;         // [0] exit ticket (zero between launches), [1] layers run since ee_reset
     size_t smem;            // dynamic shared memory per CTA
 };
 // Geometry and shared-memory plan for `m` on n_sm SMs (pointers left

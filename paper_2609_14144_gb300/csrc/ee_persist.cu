@@ -17,23 +17,27 @@
 // the producer runs ahead of the data dependencies and HBM stays busy while
 // the consumers wait for one.  Warps 0..7 consume the ring in the same order.
 //
-// Phases hand results to each other through global memory and completion
-// counters: a CTA bumps a phase's counter with a release once its share is
-// written, and a consumer of the phase acquires the counter once every CTA
-// has bumped it.  Q/K/V, O and gate/up are split by whole 32-row tiles, so
-// each tile's epilogue (bias, RoPE and the KV append; the residual add;
-// SiLU(gate) * up) runs in the CTA that owns it.  The down projection has
-// few, long rows: it is split into (tile, chunk) items over all CTAs, each
-// writing the partial sums of the tiles it touched into its slot
-// [tile][slot][32]; the next layer's Q/K/V tiles and the O-projection
-// epilogue add the slots in slot order (no dependence on timing).  The
+// Phases hand results to each other through global memory as tagged
+// values (see "tagged values" below): every float one CTA hands to another
+// carries its layer's tag in the low mantissa bits, and the reader loads
+// until the tags are the expected ones, so there are no phase counters and
+// no fences.  Q/K/V and gate/up are split by whole 32-row tiles, so each
+// tile's epilogue (bias, RoPE and the KV append; SiLU(gate) * up) runs in
+// the CTA that owns it.  The O and down projections have few, long rows:
+// they are split into (tile, 512-column chunk) items over all CTAs, each
+// writing the partial sums of its tiles into slots; the residual is rebuilt
+// by its readers from the slots in slot order (no dependence on timing).  The
 // attention of kv head g over the step's positions is split over CTAs by
-// pages; the O tiles merge the splits (flash-decoding combine).
+// pages (scores on the tensor cores); the O items merge the splits
+// (flash-decoding combine).
 //
-// Every wait is bounded: after kStallCycles the waiting thread sets kErrStall in
-// the control block and the CTA winds down (the producer first waits, again
-// with a bound, for the copies it still has in flight).  Co-residency of all
-// CTAs, which the cross-CTA waits rely on, comes from a cooperative launch.
+// Every wait is bounded: after kStallCycles the waiting thread sets kErrStall
+// in the control block, later waits return at once and the launch ends (the
+// producer first waits, again with a bound, for the copies it still has in
+// flight).  Co-residency of all CTAs, which the cross-CTA waits rely on,
+// comes from a cooperative launch.
+//
+// The same ring feeds k_vocab_ring, the vocabulary pass of the default path.
 #include <cuda_bf16.h>
 #include <math.h>
 
