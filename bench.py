@@ -48,6 +48,7 @@ WORKLOAD = "1.5b"
 HEADLINE_RATE = 0.5
 CALIB_TOKENS = 2048
 REPASS_W = 16  # positions in the measured full-depth re-pass
+ROWS_MAX = 64  # positions per batch of the multi-position layer pass (EE_OPT_ROWS)
 CTL_BYTES = 360  # device control block read back by a host-buffer ee_decode_n
 
 
@@ -428,7 +429,7 @@ def calibrate(eng, shape, n: int = CALIB_TOKENS, p_nuc: float = 0.9, fidelity: f
 def run_ours(args, rank: int, world: int, local: int):
     import torch
 
-    from paper_2609_14144_gb300 import FORCE_EXIT_AT, FORCE_FULL, Engine
+    from paper_2609_14144_gb300 import FORCE_EXIT_AT, FORCE_FULL, OPT_ROWS, Engine
 
     torch.cuda.set_device(local)
     shape = synth.CONFIGS[WORKLOAD]
@@ -489,21 +490,49 @@ def run_ours(args, rank: int, world: int, local: int):
 
     # Section 11's full-depth re-pass: decode REPASS_W tokens with every
     # step exiting, then time one re-pass of them (ee_repass)
+    # (timed for the batched pass and for one position at a time)
     repass = None
     if not args.no_sweep:
-        eng.reset()
-        eng.prefill(prompt)
-        sched = np.full(REPASS_W, FORCE_EXIT_AT(0), np.int8)
-        eng.decode_n(REPASS_W, [0.5], schedule=sched)
-        p1 = eng.position
-        torch.cuda.synchronize(local)
-        t0 = time.perf_counter()
-        n_rp = eng.repass(p1 - REPASS_W, p1)
-        dt = time.perf_counter() - t0
-        repass = {"positions": REPASS_W, "repassed": n_rp, "ms": dt * 1e3,
-                  "token_times": dt * head["tok_s"],
-                  "note": "one upper-segment launch per re-passed position (not batched)"}
-        _log(f"[bench] re-pass of {n_rp} exited positions: {dt * 1e3:.2f} ms ({dt * head['tok_s']:.1f} token-times)")
+        repass = {"positions": REPASS_W}
+        for rows in (1, 0, 1):  # the first batched run warms up
+            eng.set_option(OPT_ROWS, rows)
+            eng.reset()
+            eng.prefill(prompt)
+            sched = np.full(REPASS_W, FORCE_EXIT_AT(0), np.int8)
+            eng.decode_n(REPASS_W, [0.5], schedule=sched)
+            p1 = eng.position
+            torch.cuda.synchronize(local)
+            t0 = time.perf_counter()
+            n_rp = eng.repass(p1 - REPASS_W, p1)
+            dt = time.perf_counter() - t0
+            key = "batched" if rows else "one_position_at_a_time"
+            repass[key] = {"repassed": n_rp, "ms": dt * 1e3, "token_times": dt * head["tok_s"]}
+        eng.set_option(OPT_ROWS, 1)
+        b = repass["batched"]
+        _log(f"[bench] re-pass of {b['repassed']} exited positions: {b['ms']:.2f} ms ({b['token_times']:.2f} "
+             f"token-times); one position at a time {repass['one_position_at_a_time']['ms']:.2f} ms")
+
+    # the prompt: batches of up to 64 positions, and one position at a time
+    prefill = None
+    if not args.no_sweep:
+        P = len(prompt)
+        batches = -(-P // ROWS_MAX)
+        prefill = {"positions": P, "batch_rows": ROWS_MAX}
+        for rows in (1, 1, 0):  # the first batched run warms up
+            eng.set_option(OPT_ROWS, rows)
+            eng.reset()
+            torch.cuda.synchronize(local)
+            t0 = time.perf_counter()
+            eng.prefill(prompt)
+            dt = time.perf_counter() - t0
+            key = "batched" if rows else "one_position_at_a_time"
+            passes = batches if rows else P
+            prefill[key] = {"ms": dt * 1e3, "tok_s": P / dt,
+                            "weight_GBps": passes * bm.layer_weight_bytes(run.dims) * shape.n_layers / dt / 1e9}
+        eng.set_option(OPT_ROWS, 1)
+        _log(f"[bench] prompt of {P}: {prefill['batched']['ms']:.2f} ms batched "
+             f"({prefill['batched']['tok_s']:.0f} tok/s), {prefill['one_position_at_a_time']['ms']:.1f} ms "
+             f"one position at a time")
 
     # end to end through the host-buffer API
     e2e = run.run_host([tau_h], W, K)
@@ -557,6 +586,7 @@ def run_ours(args, rank: int, world: int, local: int):
         "plain_model": plain_line,
         "calibration": cal,
         "repass": repass,
+        "prefill": prefill,
     }
     eng.close()
     if rank == 0:
@@ -567,10 +597,12 @@ def profile_run(args, local: int):
     """A short decode for ncu captures: 64-token prompt, two 8-token chunks
     with exits imposed at 50%, no calibration.  Prints the launch counts.
     --eager launches every kernel directly (ncu cannot profile single kernel
-    nodes of graphs that hold conditional nodes)."""
+    nodes of graphs that hold conditional nodes).  The prompt runs one position
+    at a time, so the launches before the decode steps are the fixed count
+    printed here."""
     import torch
 
-    from paper_2609_14144_gb300 import DEVICE, FORCE_EXIT_AT, FORCE_FULL, OPT_GRAPHS, Engine
+    from paper_2609_14144_gb300 import DEVICE, FORCE_EXIT_AT, FORCE_FULL, OPT_GRAPHS, OPT_ROWS, Engine
 
     torch.cuda.set_device(local)
     shape = synth.CONFIGS[WORKLOAD]
@@ -579,6 +611,7 @@ def profile_run(args, local: int):
     eng = Engine(shape, model, max_ctx=P + 2 * C, device=local)
     if args.eager:
         eng.set_option(OPT_GRAPHS, 0)
+    eng.set_option(OPT_ROWS, 0)
     eng.prefill(synth.prompt(shape, P))
     sched = np.where(synth.exit_schedule(shape, 2 * C, 0.5, index=1) == 1, FORCE_EXIT_AT(0), FORCE_FULL)
     sched = sched.astype(np.int8)

@@ -1,6 +1,6 @@
 """Build libee.so (the sm_103a kernels and the C ABI) in-tree with nvcc.
 
-Two translation units compile in parallel, then link into
+The translation units compile in parallel, then link into
 ``paper_2609_14144_gb300/_build/libee.so``.
 """
 from __future__ import annotations
@@ -16,7 +16,7 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libee.so")
-SOURCES = ["ee_kernels.cu", "ee_engine.cu", "ee_persist.cu", "ee_noalloc.cu"]
+SOURCES = ["ee_kernels.cu", "ee_engine.cu", "ee_persist.cu", "ee_noalloc.cu", "ee_rows.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -59,10 +59,11 @@ struct Layout {
     size_t kpool, vpool, page_table, kv_src, h_exit, exit_at, repass_pos, h, q, o, a, y, hk, logits_ro, logits_final;
     size_t gemv_part, gemv_ticket, attn_part, attn_ticket, vocab_part, vocab_ticket;
     size_t seg_dpart, seg_opart, seg_q, seg_kvn, seg_a, seg_attn, seg_sync, seg_end;
+    size_t rows_H, rows_xhi, rows_xlo, rows_Q, rows_part, rows_pos;
     size_t prompt, sched, out_tok, out_exit, out_conf, out_conf_all, out_member, out_mass, tau_scratch, total;
     int64_t layer_stride, off_wqkv, off_bqkv, off_gattn, off_wo, off_gmlp, off_wgu, off_wd;
-    int64_t n_units_qkv, kv_layer_stride, gemv_ticket_stride;
-    int n_pages;
+    int64_t n_units_qkv, kv_layer_stride, gemv_ticket_stride, rows_part_floats;
+    int n_pages, rows_ldx;
 };
 
 int check_config(const ee_model_config* c) {
@@ -163,6 +164,15 @@ Layout make_layout(const ee_model_config& c) {
     l.seg_attn = take(4 * (size_t)A * kSegMaxSplits * (D + 4));
     l.seg_sync = take(4 * 8);
     l.seg_end = b;
+    // multi-position layer pass (prompt and re-pass batches)
+    l.rows_ldx = (int)((std::max({d, F, A * D}) + 7) / 8 * 8);
+    l.rows_part_floats = rows_part_floats((int)d, (int)A, (int)KH, (int)D, (int)F);
+    l.rows_H = take(4 * (size_t)kRowsMax * d);
+    l.rows_xhi = take(2 * (size_t)kRowsMax * l.rows_ldx);
+    l.rows_xlo = take(2 * (size_t)kRowsMax * l.rows_ldx);
+    l.rows_Q = take(4 * (size_t)kRowsMax * A * D);
+    l.rows_part = take(4 * (size_t)l.rows_part_floats);
+    l.rows_pos = take(4 * (size_t)kRowsMax);
     l.prompt = take(4 * (size_t)c.max_ctx);
     l.sched = take((size_t)c.max_ctx);
     l.out_tok = take(4 * (size_t)c.max_ctx);
@@ -230,6 +240,8 @@ struct ee_ctx {
     SegPlan seg{};
     bool vring_ok = false;  // ring-fed vocabulary pass supported (used with the persistent layers)
     VocabRing vring{};
+    bool use_rows = true;   // EE_OPT_ROWS: prompt and re-pass in batches of positions
+    RowsBuf rows{};
     int dbg = 0;
     int conf_kind = EE_CONF_PMAX;  // signal the gates compare with tau
     int repass_period = 0;         // EE_OPT_REPASS: re-pass every this many decode steps (0 = off)
@@ -592,6 +604,61 @@ CtlInputs base_inputs(const ee_ctx* c, const float* taus) {
     return in;
 }
 
+// The re-pass through the multi-position layer pass: batches of kRowsMax
+// positions in position order (a batch's attention reads the entries earlier
+// batches re-passed), the rows of a batch ordered by the layer they start at.
+// The final residual of the last position is left in m.h.
+int rows_repass(ee_ctx* c, const std::vector<int32_t>& todo, const std::vector<int32_t>& from) {
+    cudaStream_t s = c->stream;
+    const DevModel& m = c->dm;
+    const int n = (int)todo.size();
+    std::vector<int32_t> pos(n);
+    std::vector<int> start(n);
+    int last_row = 0;
+    for (int b0 = 0; b0 < n; b0 += kRowsMax) {
+        const int M = std::min(kRowsMax, n - b0);
+        std::vector<int> idx(M);
+        for (int i = 0; i < M; ++i) idx[i] = b0 + i;
+        std::stable_sort(idx.begin(), idx.end(), [&](int a, int b) { return from[a] < from[b]; });
+        for (int i = 0; i < M; ++i) {
+            pos[b0 + i] = todo[idx[i]];
+            start[b0 + i] = from[idx[i]];
+            if (idx[i] == n - 1) last_row = i;
+        }
+    }
+    int32_t* d_pos = (int32_t*)(c->ws + c->lay.repass_pos);
+    EE_CK(cudaMemcpy(d_pos, pos.data(), 4 * (size_t)n, cudaMemcpyHostToDevice));  // the stream is idle
+    for (int b0 = 0; b0 < n; b0 += kRowsMax) {
+        const int M = std::min(kRowsMax, n - b0);
+        const bool last = b0 + M == n;
+        EE_CK(rows_pass(m, c->rows, start.data() + b0, M, d_pos + b0, nullptr, 0, !last, s));
+    }
+    EE_CK(cudaMemcpyAsync(m.h, c->rows.H + (int64_t)last_row * m.d, 4 * (size_t)m.d, cudaMemcpyDeviceToDevice, s));
+    EE_TRY(fetch_ctl(c));
+    return device_error(c);
+}
+
+// The prompt in batches of kRowsMax positions through the multi-position
+// layer pass (only the last batch runs the last layer past its cache
+// entries), then the LM head on the last position's final residual.
+int rows_prefill(ee_ctx* c, const int32_t* d_prompt, int n) {
+    cudaStream_t s = c->stream;
+    const DevModel& m = c->dm;
+    const std::vector<int> start(kRowsMax, 0);
+    int last_row = 0;
+    for (int b0 = 0; b0 < n; b0 += kRowsMax) {
+        const int M = std::min(kRowsMax, n - b0);
+        EE_CK(rows_pass(m, c->rows, start.data(), M, c->rows.pos, d_prompt + b0, b0, b0 + M < n, s));
+        last_row = M - 1;
+    }
+    EE_CK(cudaMemcpyAsync(m.h, c->rows.H + (int64_t)last_row * m.d, 4 * (size_t)m.d, cudaMemcpyDeviceToDevice, s));
+    EE_CK(launch_rows_prefill_done(m, n, s));
+    bool pdl = false;
+    EE_TRY(enqueue_head(c, s, pdl));
+    EE_CK(launch_prefill_end(m, false, s));
+    return EE_OK;
+}
+
 // Section 11's full-depth re-pass over positions [t0, t1) (t1 <= pos): each
 // position whose upper layers still hold filled entries runs them again from
 // the residual it exited with (h_exit), in position order, through the same
@@ -619,6 +686,11 @@ int repass_range(ee_ctx* c, int t0, int t1, int* n_done) {
         }
     }
     if (todo.empty()) return EE_OK;
+    if (c->use_rows) {
+        EE_TRY(rows_repass(c, todo, from));
+        if (n_done) *n_done = (int)todo.size();
+        return EE_OK;
+    }
     int32_t* d_pos = (int32_t*)(c->ws + c->lay.repass_pos);  // the positions, then the decode position
     std::vector<int32_t> pos_list(todo);
     pos_list.push_back(c->pos);
@@ -768,6 +840,14 @@ int ee_create(const ee_model_config* cfg, void* d_workspace, size_t workspace_by
     m.vocab_ticket = (int*)(w + l.vocab_ticket);
     m.ctl = (Ctl*)(w + l.ctl);
     c->d_ctl = m.ctl;
+    c->rows.H = (float*)(w + l.rows_H);
+    c->rows.xhi = (uint16_t*)(w + l.rows_xhi);
+    c->rows.xlo = (uint16_t*)(w + l.rows_xlo);
+    c->rows.Q = (float*)(w + l.rows_Q);
+    c->rows.part = (float*)(w + l.rows_part);
+    c->rows.pos = (int32_t*)(w + l.rows_pos);
+    c->rows.part_floats = l.rows_part_floats;
+    c->rows.ldx = l.rows_ldx;
 
     const int kmax = std::max({2 * m.d, m.A * m.D, m.F});
     if (configure_kernels(kmax) != cudaSuccess) return bail(fail(EE_ECUDA, "kernel configuration failed"));
@@ -979,6 +1059,9 @@ int ee_set_option(ee_ctx* c, int option, int value) {
             if (value < 0 || value > 1000) return fail(EE_EINVAL, "nucleus share must be 0..1000 per mille");
             c->nucleus_permille = value;
             return EE_OK;
+        case EE_OPT_ROWS:
+            c->use_rows = value != 0;
+            return EE_OK;
         case EE_OPT_PERSISTENT:
             if (value && !c->seg_ok) return fail(EE_EINVAL, "the persistent layer kernel does not support this shape");
             if (c->use_persistent != (value != 0)) drop_graphs(c);
@@ -1007,7 +1090,9 @@ int ee_prefill(ee_ctx* c, const int32_t* ids, int n, int32_t* first_token) {
     in.prefill_n = n;
     in.prompt = d_prompt;
     EE_CK(launch_set_inputs(c->d_ctl, in, s));
-    if (c->use_graphs) {
+    if (c->use_rows) {
+        EE_TRY(rows_prefill(c, d_prompt, n));
+    } else if (c->use_graphs) {
         EE_TRY(ensure_graphs(c));
         EE_CK(cudaGraphLaunch(c->g_prefill, s));
     } else {

@@ -227,6 +227,37 @@ bool vocab_ring_plan(int d, int n_sm, VocabRing& vr);
 cudaError_t configure_vocab_ring(size_t smem);
 cudaError_t launch_vocab_ring(const VocabArgs& v, const VocabRing& vr, bool pdl, cudaStream_t s);
 
+// Multi-position layer pass (ee_rows.cu): the prompt and the re-pass run
+// each layer over up to kRowsMax positions at once, every weight byte read
+// once per batch.  Products are tensor-core mma of the bf16 weights with the
+// fp32 activations split into bf16 high and low parts.
+constexpr int kRowsMax = 64;             // positions per batch
+constexpr int kRowsTargetUnits = 2432;   // (tile, K split) units a projection aims for: 152 SMs x 16 warps
+struct RowsBuf {
+    float* H;           // [kRowsMax][d] residual of each row
+    uint16_t* xhi;      // [kRowsMax][ldx] next product's input, bf16 high part
+    uint16_t* xlo;      // [kRowsMax][ldx] low part (x - high, rounded)
+    float* Q;           // [kRowsMax][A D] rotated queries
+    float* part;        // split partials [S][M][n_rows padded to 32]
+    int32_t* pos;       // [kRowsMax] positions of a prompt batch
+    int64_t part_floats;
+    int ldx;
+};
+// Splits along K of an n_tiles x K projection for a batch of M rows.
+int rows_splits(int64_t n_tiles, int K, int M);
+// Floats of the partial buffer every batch size fits in.
+int64_t rows_part_floats(int d, int A, int KH, int D, int F);
+// Run layers over M rows at the device positions d_pos (ascending layer
+// start): row i starts at layer start[i] (host, non-decreasing).  With ids,
+// rows take the embedding of ids[i] and positions pos_base + i (written to
+// d_pos); otherwise each row starts from h_exit at its position.  kv_only:
+// the last layer stops after its cache entries.
+cudaError_t rows_pass(const DevModel& m, const RowsBuf& b, const int* start, int M, int32_t* d_pos,
+                      const int32_t* ids, int pos_base, bool kv_only, cudaStream_t s);
+// After a batched prompt: the control block as the per-position prefill
+// leaves it before its LM head (position n).
+cudaError_t launch_rows_prefill_done(const DevModel& m, int n, cudaStream_t s);
+
 // Record `msg` as the calling thread's last error and return `code`.
 int set_last_error(int code, const char* msg);
 

@@ -4,7 +4,8 @@ Positions that exited keep their exit residual; ee_repass runs their skipped
 layers again in position order.  Checked against the oracle's re-pass
 (entries within 1e-2 relative, kv_src bit for bit), against the GPU's own
 full-depth run of the same tokens (bit for bit once every exited position
-has been re-passed), and through the periodic option of ee_decode_n."""
+has been re-passed, when the re-pass runs one position at a time), and
+through the periodic option of ee_decode_n."""
 import numpy as np
 import pytest
 
@@ -26,14 +27,15 @@ def _force(i, every=3):
     return oracle.FORCE_FULL if i % every == 0 else oracle.FORCE_EXIT_AT(0)
 
 
-def _decode_both(model, n, persistent=True, graphs=True):
-    from paper_2609_14144_gb300 import OPT_GRAPHS, OPT_PERSISTENT, Engine
+def _decode_both(model, n, persistent=True, graphs=True, rows=True):
+    from paper_2609_14144_gb300 import OPT_GRAPHS, OPT_PERSISTENT, OPT_ROWS, Engine
 
     P = TINY.prompt_len
     orc = oracle.Oracle(TINY, model, max_ctx=P + n + 2)
     eng = Engine(TINY, model, max_ctx=P + n + 2)
     eng.set_option(OPT_PERSISTENT, int(persistent))
     eng.set_option(OPT_GRAPHS, int(graphs))
+    eng.set_option(OPT_ROWS, int(rows))
     tok = orc.prefill(synth.prompt(TINY))
     eng.prefill(synth.prompt(TINY))
     ins = []
@@ -54,11 +56,11 @@ def _check_cache(orc, eng, t_end, tol=1e-2):
             assert rel_err(kg, ko) <= tol and rel_err(vg, vo) <= tol, (j, t)
 
 
-@pytest.mark.parametrize("persistent", [True, False])
-def test_tiny_repass_matches_oracle(tiny_model, persistent):
+@pytest.mark.parametrize("persistent,rows", [(True, True), (True, False), (False, False)])
+def test_tiny_repass_matches_oracle(tiny_model, persistent, rows):
     n = 18
     P = TINY.prompt_len
-    orc, eng, _ = _decode_both(tiny_model, n, persistent=persistent)
+    orc, eng, _ = _decode_both(tiny_model, n, persistent=persistent, rows=rows)
     _check_cache(orc, eng, P + n)  # before: filled entries agree
     t0, t1 = P + 4, P + n
     assert eng.repass(t0, t1) == orc.repass(t0, t1) == sum(1 for i in range(4, n) if i % 3)
@@ -72,15 +74,17 @@ def test_tiny_repass_matches_oracle(tiny_model, persistent):
 
 
 def test_repass_gives_the_full_depth_cache_bit_for_bit(tiny_model):
-    """Exits then a re-pass of every exited position equal, bit for bit, the
-    GPU's own full-depth run of the same tokens."""
-    from paper_2609_14144_gb300 import FORCE_FULL, Engine
+    """Exits then a re-pass of every exited position, one position at a time
+    through the decode step's layer kernels, equal bit for bit the GPU's own
+    full-depth run of the same tokens."""
+    from paper_2609_14144_gb300 import FORCE_FULL, OPT_ROWS, Engine
 
     n = 15
     P = TINY.prompt_len
-    _, eng, ins = _decode_both(tiny_model, n)
+    _, eng, ins = _decode_both(tiny_model, n, rows=False)
     assert eng.repass(P, P + n) == sum(1 for i in range(n) if i % 3)
     full = Engine(TINY, tiny_model, max_ctx=P + n + 2)
+    full.set_option(OPT_ROWS, 0)
     full.prefill(synth.prompt(TINY))
     for tok in ins:
         full.decode_step(tok, [2.0], FORCE_FULL)
