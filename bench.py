@@ -607,6 +607,8 @@ def profile_run(args, local: int):
     torch.cuda.set_device(local)
     shape = synth.CONFIGS[WORKLOAD]
     model = synth.make_model(shape)
+    if args.rows:
+        return profile_rows(shape, model, local)
     P, C = 64, 8
     eng = Engine(shape, model, max_ctx=P + 2 * C, device=local)
     if args.eager:
@@ -624,6 +626,35 @@ def profile_run(args, local: int):
     print(json.dumps({"prefill_launches": prefill_launches, "decode_launches": decode, "tokens": 2 * C}))
 
 
+def rows_launches(L: int, M: int, kv_only: bool) -> int:
+    """Kernels of one multi-position batch: the start, nine per layer (the
+    last layer three when only its cache entries are needed), and the final
+    residual add."""
+    return 1 + 9 * (L - 1) + (3 if kv_only else 10)
+
+
+def profile_rows(shape, model, local: int):
+    """--profile-run --rows: the multi-position layer pass for ncu captures.
+    A 128-position prompt in two batches, 16 exit steps (direct launches),
+    then one re-pass of those 16 positions in one batch.  Prints the launch
+    counts of each part."""
+    from paper_2609_14144_gb300 import DEVICE, FORCE_EXIT_AT, OPT_GRAPHS, Engine
+
+    P, n = 128, REPASS_W
+    eng = Engine(shape, model, max_ctx=P + n, device=local)
+    eng.set_option(OPT_GRAPHS, 0)
+    eng.prefill(synth.prompt(shape, P))
+    eng.decode_n(n, [0.5], schedule=np.full(n, FORCE_EXIT_AT(0), np.int8), where=DEVICE)
+    eng.sync()
+    n_rp = eng.repass(P, P + n)
+    L, k = shape.n_layers, shape.readout_layers[0]
+    prefill = rows_launches(L, ROWS_MAX, True) + rows_launches(L, P - ROWS_MAX, False) + 3
+    decode = sum(step_launches(L, shape.readout_layers, 0, eng.persistent) for _ in range(n)) + 1
+    repass = rows_launches(L - k, n, False)
+    print(json.dumps({"prefill_launches": prefill, "decode_launches": decode, "repass_launches": repass,
+                      "repassed": n_rp}))
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -636,6 +667,7 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--profile-run", action="store_true", help="short decode for ncu captures")
     ap.add_argument("--eager", action="store_true", help="with --profile-run: direct launches, no graphs")
+    ap.add_argument("--rows", action="store_true", help="with --profile-run: the multi-position layer pass")
     ap.add_argument("--workload", default=WORKLOAD, choices=sorted(synth.CONFIGS),
                     help="synthetic shape (the benchmark workload is 1.5b)")
     args = ap.parse_args()

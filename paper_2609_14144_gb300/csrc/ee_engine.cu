@@ -674,9 +674,8 @@ int repass_range(ee_ctx* c, int t0, int t1, int* n_done) {
     std::vector<int16_t> ex(W);
     std::vector<int8_t> src((size_t)L * W);
     EE_CK(cudaMemcpy(ex.data(), m.exit_at + t0, 2 * (size_t)W, cudaMemcpyDeviceToHost));
-    for (int j = 0; j < L; ++j)
-        EE_CK(cudaMemcpy(src.data() + (size_t)j * W, m.kv_src + (int64_t)j * m.max_ctx + t0, (size_t)W,
-                         cudaMemcpyDeviceToHost));
+    EE_CK(cudaMemcpy2D(src.data(), (size_t)W, m.kv_src + t0, (size_t)m.max_ctx, (size_t)W, (size_t)L,
+                       cudaMemcpyDeviceToHost));
     std::vector<int32_t> todo, from;
     for (int i = 0; i < W; ++i) {
         const int k = ex[i];

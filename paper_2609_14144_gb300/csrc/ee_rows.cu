@@ -100,21 +100,26 @@ __device__ __forceinline__ int64_t slot_offset(const DevModel& m, int j, int pos
 //
 // part[s][row][n] = sum over the k of split s of W[n][k] x[row][k], for the
 // M rows of x (bf16 high and low parts, row stride ldx) and every output n of
-// the tiled weights.  NB blocks of 8 rows (rows past M read as zero and are
-// not stored).  K splits cover whole 32-column steps; a chunk past K reads as
-// zero on both sides.
-template <int NB>
+// the tiled weights.  A unit is (tile, split, row group): NB blocks of 8 rows
+// starting at row group * 8 NB (rows past M read as zero and are not
+// stored); the row groups of one (tile, split) are neighbouring warps, so a
+// weight chunk read for one is an L2 hit for the others.  K splits cover
+// whole 32-column steps, U steps loaded before any is multiplied; a chunk
+// past K reads as zero on both sides.
+template <int NB, int U>
 __global__ void __launch_bounds__(kRowsThreads) k_rows_mm(const uint4* __restrict__ W, int n_tiles, int K,
                                                           const uint16_t* __restrict__ xhi,
                                                           const uint16_t* __restrict__ xlo, int ldx, int M, int S,
-                                                          float* __restrict__ part, int Np) {
+                                                          int RG, float* __restrict__ part, int Np) {
     const int lane = threadIdx.x & 31, g = lane >> 2, q = lane & 3;
     const int Rc = K >> 3;             // 16-byte chunks per weight row
     const int nsteps = (Rc + 3) >> 2;  // 32-column steps
-    const int units = n_tiles * S;
+    const int units = n_tiles * S * RG;
     const int nw = gridDim.x * kRowsWarps;
     for (int u = blockIdx.x * kRowsWarps + (threadIdx.x >> 5); u < units; u += nw) {
-        const int tile = u / S, s = u - tile * S;
+        const int ts = u / RG, rg = u - ts * RG;
+        const int tile = ts / S, s = ts - tile * S;
+        const int r0 = rg * 8 * NB;
         const int st0 = (int)((int64_t)nsteps * s / S), st1 = (int)((int64_t)nsteps * (s + 1) / S);
         const uint4* wt = W + (int64_t)tile * Rc * 32;
         float acc[2][NB][4];
@@ -124,37 +129,44 @@ __global__ void __launch_bounds__(kRowsThreads) k_rows_mm(const uint4* __restric
             for (int n = 0; n < NB; ++n)
 #pragma unroll
                 for (int e = 0; e < 4; ++e) acc[a][n][e] = 0.f;
-        for (int st = st0; st < st1; ++st) {
-            const int ch = st * 4 + q;  // this lane's chunk of the step
-            const bool ok = ch < Rc;
-            uint4 w[4];
+        for (int st = st0; st < st1; st += U) {
+            uint4 w[U][4], bh[U][NB], bl[U][NB];
 #pragma unroll
-            for (int r = 0; r < 4; ++r)  // rows g, g+8, g+16, g+24 of the tile
-                w[r] = ok ? ld_weights(wt + (int64_t)ch * 32 + g + 8 * r) : make_uint4(0u, 0u, 0u, 0u);
-            uint4 bh[NB], bl[NB];
+            for (int v = 0; v < U; ++v) {
+                const int ch = (st + v) * 4 + q;  // this lane's chunk of the step
+                const bool ok = st + v < st1 && ch < Rc;
 #pragma unroll
-            for (int n = 0; n < NB; ++n) {
-                const int row = n * 8 + g;
-                const bool okx = ok && row < M;
-                const int64_t at = (int64_t)row * ldx + ch * 8;
-                bh[n] = okx ? ld_act(xhi + at) : make_uint4(0u, 0u, 0u, 0u);
-                bl[n] = okx ? ld_act(xlo + at) : make_uint4(0u, 0u, 0u, 0u);
+                for (int r = 0; r < 4; ++r)  // rows g, g+8, g+16, g+24 of the tile
+                    w[v][r] = ok ? ld_weights(wt + (int64_t)ch * 32 + g + 8 * r) : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+                for (int n = 0; n < NB; ++n) {
+                    const int row = r0 + n * 8 + g;
+                    const bool okx = ok && row < M;
+                    const int64_t at = (int64_t)row * ldx + ch * 8;
+                    bh[v][n] = okx ? ld_act(xhi + at) : make_uint4(0u, 0u, 0u, 0u);
+                    bl[v][n] = okx ? ld_act(xlo + at) : make_uint4(0u, 0u, 0u, 0u);
+                }
             }
 #pragma unroll
-            for (int n = 0; n < NB; ++n) {
-                // first mma of the step: chunk elements 0..3; second: 4..7
-                mma_16816(acc[0][n], w[0].x, w[1].x, w[0].y, w[1].y, bh[n].x, bh[n].y);
-                mma_16816(acc[0][n], w[0].x, w[1].x, w[0].y, w[1].y, bl[n].x, bl[n].y);
-                mma_16816(acc[0][n], w[0].z, w[1].z, w[0].w, w[1].w, bh[n].z, bh[n].w);
-                mma_16816(acc[0][n], w[0].z, w[1].z, w[0].w, w[1].w, bl[n].z, bl[n].w);
-                mma_16816(acc[1][n], w[2].x, w[3].x, w[2].y, w[3].y, bh[n].x, bh[n].y);
-                mma_16816(acc[1][n], w[2].x, w[3].x, w[2].y, w[3].y, bl[n].x, bl[n].y);
-                mma_16816(acc[1][n], w[2].z, w[3].z, w[2].w, w[3].w, bh[n].z, bh[n].w);
-                mma_16816(acc[1][n], w[2].z, w[3].z, w[2].w, w[3].w, bl[n].z, bl[n].w);
+            for (int v = 0; v < U; ++v) {
+                const uint4* x = w[v];
+#pragma unroll
+                for (int n = 0; n < NB; ++n) {
+                    const uint4 h = bh[v][n], l = bl[v][n];
+                    // first mma of the step: chunk elements 0..3; second: 4..7
+                    mma_16816(acc[0][n], x[0].x, x[1].x, x[0].y, x[1].y, h.x, h.y);
+                    mma_16816(acc[0][n], x[0].x, x[1].x, x[0].y, x[1].y, l.x, l.y);
+                    mma_16816(acc[0][n], x[0].z, x[1].z, x[0].w, x[1].w, h.z, h.w);
+                    mma_16816(acc[0][n], x[0].z, x[1].z, x[0].w, x[1].w, l.z, l.w);
+                    mma_16816(acc[1][n], x[2].x, x[3].x, x[2].y, x[3].y, h.x, h.y);
+                    mma_16816(acc[1][n], x[2].x, x[3].x, x[2].y, x[3].y, l.x, l.y);
+                    mma_16816(acc[1][n], x[2].z, x[3].z, x[2].w, x[3].w, h.z, h.w);
+                    mma_16816(acc[1][n], x[2].z, x[3].z, x[2].w, x[3].w, l.z, l.w);
+                }
             }
         }
         // accumulator e of block (a, n): output row tile*32 + a*16 + g (+8 for
-        // e >= 2), batch row n*8 + 2q (+1 for odd e)
+        // e >= 2), batch row r0 + n*8 + 2q (+1 for odd e)
         float* ps = part + (int64_t)s * M * Np;
 #pragma unroll
         for (int a = 0; a < 2; ++a)
@@ -162,7 +174,7 @@ __global__ void __launch_bounds__(kRowsThreads) k_rows_mm(const uint4* __restric
             for (int n = 0; n < NB; ++n)
 #pragma unroll
                 for (int e = 0; e < 4; ++e) {
-                    const int row = n * 8 + 2 * q + (e & 1);
+                    const int row = r0 + n * 8 + 2 * q + (e & 1);
                     const int out = tile * 32 + a * 16 + g + (e >> 1) * 8;
                     if (row < M) ps[(int64_t)row * Np + out] = acc[a][n][e];
                 }
@@ -171,44 +183,62 @@ __global__ void __launch_bounds__(kRowsThreads) k_rows_mm(const uint4* __restric
 
 // ------------------------------------------------------------------ per-row epilogues
 
-// Sum over the block; every thread gets the same value (fixed order).
+constexpr int kNormThreads = 768;  // residual add + RMSNorm: one CTA per row
+
+// Sum over the block of NT threads; every thread gets the same value (fixed order).
+template <int NT>
 __device__ __forceinline__ float r_block_sum(float v, float* red) {
     v = r_warp_sum(v);
     const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
     __syncthreads();
     if (l == 0) red[w] = v;
     __syncthreads();
-    float t = l < kRowsWarps ? red[l] : 0.f;
+    float t = l < NT / 32 ? red[l] : 0.f;
     return r_warp_sum(t);
+}
+
+// Sum of the S split partials p[0], p[stride], ..., in a fixed order: four
+// running sums over splits s = 4k + r, added pairwise at the end, so that
+// several loads are in flight.
+__device__ __forceinline__ float split_sum(const float* __restrict__ p, int64_t stride, int S) {
+    float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+    int s = 0;
+#pragma unroll 2
+    for (; s + 4 <= S; s += 4) {
+        a0 += p[(int64_t)s * stride];
+        a1 += p[(int64_t)(s + 1) * stride];
+        a2 += p[(int64_t)(s + 2) * stride];
+        a3 += p[(int64_t)(s + 3) * stride];
+    }
+    for (; s < S; ++s) a0 += p[(int64_t)s * stride];
+    return (a0 + a1) + (a2 + a3);
 }
 
 // One CTA per row i < M_norm.  Rows below M_add first add the split partials
 // of a d-output projection (split stride M_add rows) to their residual.  With
 // a gain, the row's RMSNorm h / sqrt(mean(h^2) + eps) * g goes to x as bf16
 // high and low parts.
-__global__ void __launch_bounds__(kRowsThreads) k_rows_add_norm(float* __restrict__ H, int d,
+__global__ void __launch_bounds__(kNormThreads) k_rows_add_norm(float* __restrict__ H, int d,
                                                                 const float* __restrict__ part, int S, int M_add,
                                                                 int Np, const uint16_t* __restrict__ gain, float eps,
                                                                 uint16_t* __restrict__ xhi, uint16_t* __restrict__ xlo,
                                                                 int ldx) {
-    __shared__ float red[kRowsWarps];
+    __shared__ float red[kNormThreads / 32];
     const int i = blockIdx.x;
     float* h = H + (int64_t)i * d;
     float ss = 0.f;
-    for (int n = threadIdx.x; n < d; n += kRowsThreads) {
+    for (int n = threadIdx.x; n < d; n += kNormThreads) {
         float v = h[n];
         if (i < M_add) {
-            float a = 0.f;
-            for (int s = 0; s < S; ++s) a += part[((int64_t)s * M_add + i) * Np + n];
-            v += a;
+            v += split_sum(part + (int64_t)i * Np + n, (int64_t)M_add * Np, S);
             h[n] = v;
         }
         ss = fmaf(v, v, ss);
     }
     if (!gain) return;  // uniform over the block
-    ss = r_block_sum(ss, red);
+    ss = r_block_sum<kNormThreads>(ss, red);
     const float inv = 1.0f / sqrtf(ss / (float)d + eps);
-    for (int n = threadIdx.x; n < d; n += kRowsThreads) {
+    for (int n = threadIdx.x; n < d; n += kNormThreads) {
         const float x = h[n] * inv * r_bf2f(gain[n]);
         split_store(x, xhi + (int64_t)i * ldx + n, xlo + (int64_t)i * ldx + n);
     }
@@ -225,12 +255,8 @@ __global__ void __launch_bounds__(kRowsThreads) k_rows_qkv(DevModel m, int j, co
     const int half = m.D >> 1;
     const int nq = m.A * half, nk = m.KH * half;
     if (u >= nq + 2 * nk) return;
-    float r0 = 0.f, r1 = 0.f;
-    for (int s = 0; s < S; ++s) {
-        const float* p = part + ((int64_t)s * M + i) * Np + 2 * u;
-        r0 += p[0];
-        r1 += p[1];
-    }
+    const float* p = part + (int64_t)i * Np + 2 * u;
+    float r0 = split_sum(p, (int64_t)M * Np, S), r1 = split_sum(p + 1, (int64_t)M * Np, S);
     if (m.qkv_bias) {
         const uint16_t* b = m.layers + (int64_t)j * m.layer_stride + m.off_bqkv;
         r0 += r_bf2f(b[2 * u]);
@@ -266,12 +292,8 @@ __global__ void __launch_bounds__(kRowsThreads) k_rows_swiglu(const float* __res
     const int i = blockIdx.y;
     const int f = blockIdx.x * kRowsThreads + threadIdx.x;
     if (f >= F) return;
-    float gs = 0.f, us = 0.f;
-    for (int s = 0; s < S; ++s) {
-        const float* p = part + ((int64_t)s * M + i) * Np + 2 * f;
-        gs += p[0];
-        us += p[1];
-    }
+    const float* p = part + (int64_t)i * Np + 2 * f;
+    const float gs = split_sum(p, (int64_t)M * Np, S), us = split_sum(p + 1, (int64_t)M * Np, S);
     const float a = gs / (1.0f + expf(-gs)) * us;
     split_store(a, xhi + (int64_t)i * ldx + f, xlo + (int64_t)i * ldx + f);
 }
@@ -310,22 +332,26 @@ __global__ void k_rows_prefill_done(DevModel m, int n) {
 }
 
 // Causal attention of row blockIdx.y and kv head blockIdx.x over cache
-// positions 0..pos[i] of layer j, for the head group's G query heads: keys
-// in chunks of one per thread, a running maximum and sum per head, the
-// output rescaled with each new maximum (the result is Section 2's softmax
-// attention).  Output o at column h*D + e as bf16 high and low parts.
+// positions 0..pos[i] of layer j, for the head group's G query heads, in
+// chunks of one key per thread: scores q.k / sqrt(D) per thread, a running
+// maximum and sum per head, and the weighted values summed with each warp
+// taking its own 32 keys of the chunk (lane l owning dimensions
+// l*D/32 .. l*D/32 + D/32 - 1 of every head), rescaled whenever the maximum
+// grows; the warps' sums are added in warp order at the end (Section 2's
+// softmax attention).  Output o at column h*D + e as bf16 high and low parts.
+template <int D>
 __global__ void __launch_bounds__(kRowsThreads) k_rows_attn(DevModel m, int j, const float* __restrict__ Q,
                                                             const int32_t* __restrict__ pos,
                                                             uint16_t* __restrict__ xhi, uint16_t* __restrict__ xlo,
                                                             int ldx) {
-    constexpr int kG = kSegMaxGroup;             // query heads per kv head (at most)
-    constexpr int kOut = kG * 128 / kRowsThreads;  // outputs per thread (at most)
-    __shared__ float qs[kG * 128];
+    constexpr int kG = kSegMaxGroup;  // query heads per kv head (at most)
+    constexpr int DL = D / 32;        // dimensions per lane in the value sums
+    __shared__ float qs[kG * D];
     __shared__ float ps[kG * kKeysPerChunk];
     __shared__ int64_t offs[kKeysPerChunk];
     __shared__ float redm[kRowsWarps][kG], reds[kRowsWarps][kG];
     __shared__ float mrun[kG], lrun[kG], resc[kG];
-    const int g = blockIdx.x, i = blockIdx.y, D = m.D, G = m.A / m.KH;
+    const int g = blockIdx.x, i = blockIdx.y, G = m.A / m.KH;
     const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
     const int T = pos[i] + 1;
     const float scale = 1.0f / sqrtf((float)D);
@@ -335,9 +361,11 @@ __global__ void __launch_bounds__(kRowsThreads) k_rows_attn(DevModel m, int j, c
         mrun[tid] = -INFINITY;
         lrun[tid] = 0.f;
     }
-    float o[kOut];
+    float o[kG][DL];
 #pragma unroll
-    for (int k = 0; k < kOut; ++k) o[k] = 0.f;
+    for (int h = 0; h < kG; ++h)
+#pragma unroll
+        for (int x = 0; x < DL; ++x) o[h][x] = 0.f;
     const int64_t head_off = (int64_t)g * m.page_size * D;
     __syncthreads();
     for (int c0 = 0; c0 < T; c0 += kKeysPerChunk) {
@@ -349,15 +377,18 @@ __global__ void __launch_bounds__(kRowsThreads) k_rows_attn(DevModel m, int j, c
 #pragma unroll
         for (int h = 0; h < kG; ++h) sc[h] = 0.f;
         if (valid) {
-            const uint16_t* kr = m.kpool + off;
-            for (int c = 0; c < D; c += 8) {
-                const uint4 kv = *reinterpret_cast<const uint4*>(kr + c);
-                const float kf[8] = {r_lo(kv.x), r_hi(kv.x), r_lo(kv.y), r_hi(kv.y),
-                                     r_lo(kv.z), r_hi(kv.z), r_lo(kv.w), r_hi(kv.w)};
+            const uint4* kr = reinterpret_cast<const uint4*>(m.kpool + off);
+            uint4 kv[D / 8];
+#pragma unroll
+            for (int c = 0; c < D / 8; ++c) kv[c] = kr[c];
+#pragma unroll
+            for (int c = 0; c < D / 8; ++c) {
+                const float kf[8] = {r_lo(kv[c].x), r_hi(kv[c].x), r_lo(kv[c].y), r_hi(kv[c].y),
+                                     r_lo(kv[c].z), r_hi(kv[c].z), r_lo(kv[c].w), r_hi(kv[c].w)};
 #pragma unroll
                 for (int h = 0; h < kG; ++h) {
                     if (h < G) {
-                        const float* qh = qs + h * D + c;
+                        const float* qh = qs + h * D + c * 8;
                         float a = sc[h];
 #pragma unroll
                         for (int e = 0; e < 8; ++e) a = fmaf(qh[e], kf[e], a);
@@ -398,32 +429,73 @@ __global__ void __launch_bounds__(kRowsThreads) k_rows_attn(DevModel m, int j, c
             for (int ww = 0; ww < kRowsWarps; ++ww) sum += reds[ww][tid];
             lrun[tid] = lrun[tid] * resc[tid] + sum;
         }
-        const int nk = min(kKeysPerChunk, T - c0);
 #pragma unroll
-        for (int k = 0; k < kOut; ++k) {
-            const int idx = tid + kRowsThreads * k;
-            if (idx < G * D) {
-                const int h = idx / D, e = idx - h * D;
-                const float* ph = ps + h * kKeysPerChunk;
-                float a = o[k] * resc[h];
-                for (int tt = 0; tt < nk; ++tt) a = fmaf(ph[tt], r_bf2f(m.vpool[offs[tt] + e]), a);
-                o[k] = a;
+        for (int h = 0; h < kG; ++h) {
+            const float r = h < G ? resc[h] : 0.f;
+#pragma unroll
+            for (int x = 0; x < DL; ++x) o[h][x] *= r;
+        }
+        // this warp's keys of the chunk (invalid keys have p = 0 and offset 0)
+        const int k0 = w * 32;
+#pragma unroll 8
+        for (int kk = 0; kk < 32; ++kk) {
+            const int tt = k0 + kk;
+            const uint16_t* vr = m.vpool + offs[tt] + lane * DL;
+            float v[DL];
+            if constexpr (DL == 4) {
+                const uint2 u = *reinterpret_cast<const uint2*>(vr);
+                v[0] = r_lo(u.x);
+                v[1] = r_hi(u.x);
+                v[2] = r_lo(u.y);
+                v[3] = r_hi(u.y);
+            } else {
+                const uint32_t u = *reinterpret_cast<const uint32_t*>(vr);
+                v[0] = r_lo(u);
+                v[1] = r_hi(u);
+            }
+#pragma unroll
+            for (int h = 0; h < kG; ++h) {
+                if (h < G) {
+                    const float p = ps[h * kKeysPerChunk + tt];
+#pragma unroll
+                    for (int x = 0; x < DL; ++x) o[h][x] = fmaf(p, v[x], o[h][x]);
+                }
             }
         }
         __syncthreads();
     }
+    // add the warps' sums in warp order through shared memory (ps is free)
+    float* acc = ps;  // kG * D <= kG * kKeysPerChunk floats
+    for (int ww = 0; ww < kRowsWarps; ++ww) {
+        if (w == ww) {
 #pragma unroll
-    for (int k = 0; k < kOut; ++k) {
-        const int idx = tid + kRowsThreads * k;
-        if (idx < G * D) {
-            const int h = idx / D, e = idx - h * D;
-            const int64_t col = (int64_t)(g * G + h) * D + e;
-            split_store(o[k] / lrun[h], xhi + (int64_t)i * ldx + col, xlo + (int64_t)i * ldx + col);
+            for (int h = 0; h < kG; ++h) {
+                if (h < G) {
+#pragma unroll
+                    for (int x = 0; x < DL; ++x) {
+                        float* a = acc + h * D + lane * DL + x;
+                        *a = ww == 0 ? o[h][x] : *a + o[h][x];
+                    }
+                }
+            }
         }
+        __syncthreads();
+    }
+    for (int idx = tid; idx < G * D; idx += kRowsThreads) {
+        const int h = idx / D, e = idx - h * D;
+        const int64_t col = (int64_t)(g * G + h) * D + e;
+        split_store(acc[idx] / lrun[h], xhi + (int64_t)i * ldx + col, xlo + (int64_t)i * ldx + col);
     }
 }
 
 // ------------------------------------------------------------------ host side
+
+// Row blocks of 8 a warp takes (1, 2 or 4) and the row groups of a batch.
+void row_groups(int M, int& NB, int& RG) {
+    const int blocks = (M + 7) / 8;
+    NB = blocks <= 1 ? 1 : blocks <= 2 ? 2 : 4;
+    RG = (blocks + NB - 1) / NB;
+}
 
 // One projection of the batch: W (n_rows x K, tiled) times the M rows of
 // b.xhi / b.xlo into b.part; returns the split count and padded row count
@@ -431,33 +503,38 @@ __global__ void __launch_bounds__(kRowsThreads) k_rows_attn(DevModel m, int j, c
 cudaError_t launch_mm(const uint16_t* W, int64_t n_rows, int K, const RowsBuf& b, int M, int& S, int& Np,
                       cudaStream_t s) {
     const int64_t nt = tile_count(n_rows);
+    int NB, RG;
+    row_groups(M, NB, RG);
     S = rows_splits(nt, K, M);
     Np = (int)(nt * kTileRows);
-    const int64_t units = nt * S;
+    const int64_t units = nt * S * RG;
     const int grid = (int)std::min<int64_t>((units + kRowsWarps - 1) / kRowsWarps, 65535);
     const uint4* w = reinterpret_cast<const uint4*>(W);
-    const int nb = (M + 7) / 8;
-    if (nb <= 1)
-        k_rows_mm<1><<<grid, kRowsThreads, 0, s>>>(w, (int)nt, K, b.xhi, b.xlo, b.ldx, M, S, b.part, Np);
-    else if (nb <= 2)
-        k_rows_mm<2><<<grid, kRowsThreads, 0, s>>>(w, (int)nt, K, b.xhi, b.xlo, b.ldx, M, S, b.part, Np);
-    else if (nb <= 4)
-        k_rows_mm<4><<<grid, kRowsThreads, 0, s>>>(w, (int)nt, K, b.xhi, b.xlo, b.ldx, M, S, b.part, Np);
+    if (NB == 1)
+        k_rows_mm<1, 2><<<grid, kRowsThreads, 0, s>>>(w, (int)nt, K, b.xhi, b.xlo, b.ldx, M, S, RG, b.part, Np);
+    else if (NB == 2)
+        k_rows_mm<2, 2><<<grid, kRowsThreads, 0, s>>>(w, (int)nt, K, b.xhi, b.xlo, b.ldx, M, S, RG, b.part, Np);
     else
-        k_rows_mm<8><<<grid, kRowsThreads, 0, s>>>(w, (int)nt, K, b.xhi, b.xlo, b.ldx, M, S, b.part, Np);
+        k_rows_mm<4, 1><<<grid, kRowsThreads, 0, s>>>(w, (int)nt, K, b.xhi, b.xlo, b.ldx, M, S, RG, b.part, Np);
     return cudaGetLastError();
 }
 
 }  // namespace
 
-// Enough (tile, split) units to give every warp slot of the GPU one, each at
-// least one 32-column step, and split partials (written and read once) at
-// most half the weight bytes: S * M * 4 B * 2 <= K * 2 B / 2.
+// Enough (tile, split, row group) units to give every resident warp of the
+// GPU one (16 warps per SM; 24 with four row blocks a warp, whose registers
+// leave room for three CTAs), each at least one 32-column step, and split
+// partials (written and read once, in L2) at most the weight bytes,
+// S * M * 4 B * 2 <= K * 2 B, or twice that with four row blocks a warp
+// (whose units are otherwise too few to cover the SMs).
 int rows_splits(int64_t n_tiles, int K, int M) {
     const int nsteps = ((K >> 3) + 3) >> 2;
     const int Mp = std::max(8, (M + 7) & ~7);
-    int S = (int)((kRowsTargetUnits + n_tiles - 1) / n_tiles);
-    S = std::min(S, std::max(1, K / (8 * Mp)));
+    int NB, RG;
+    row_groups(M, NB, RG);
+    const int64_t target = NB == 4 ? kRowsTargetUnits * 3 / 2 : kRowsTargetUnits;
+    int S = (int)((target + n_tiles * RG - 1) / (n_tiles * RG));
+    S = std::min(S, std::max(1, K / ((NB == 4 ? 2 : 4) * Mp)));
     S = std::min(S, nsteps);
     return std::max(S, 1);
 }
@@ -497,7 +574,7 @@ cudaError_t rows_pass(const DevModel& m, const RowsBuf& b, const int* start, int
         const uint16_t* lw = m.layers + (int64_t)j * m.layer_stride;
         int S = 1, Np = 0;
         // the previous layer's down projection into the residual, this layer's input norm
-        k_rows_add_norm<<<Mj, kRowsThreads, 0, s>>>(b.H, d, b.part, S_prev, M_prev, Np_prev, lw + m.off_gattn, m.eps,
+        k_rows_add_norm<<<Mj, kNormThreads, 0, s>>>(b.H, d, b.part, S_prev, M_prev, Np_prev, lw + m.off_gattn, m.eps,
                                                      b.xhi, b.xlo, b.ldx);
         RCK(cudaGetLastError());
         RCK(launch_mm(lw + m.off_wqkv, nqkv, d, b, Mj, S, Np, s));
@@ -506,10 +583,13 @@ cudaError_t rows_pass(const DevModel& m, const RowsBuf& b, const int* start, int
                                                                                              d_pos, b.Q);
         RCK(cudaGetLastError());
         if (kv_only && j == L - 1) return cudaSuccess;
-        k_rows_attn<<<dim3(m.KH, Mj), kRowsThreads, 0, s>>>(m, j, b.Q, d_pos, b.xhi, b.xlo, b.ldx);
+        if (m.D == 128)
+            k_rows_attn<128><<<dim3(m.KH, Mj), kRowsThreads, 0, s>>>(m, j, b.Q, d_pos, b.xhi, b.xlo, b.ldx);
+        else
+            k_rows_attn<64><<<dim3(m.KH, Mj), kRowsThreads, 0, s>>>(m, j, b.Q, d_pos, b.xhi, b.xlo, b.ldx);
         RCK(cudaGetLastError());
         RCK(launch_mm(lw + m.off_wo, d, AD, b, Mj, S, Np, s));
-        k_rows_add_norm<<<Mj, kRowsThreads, 0, s>>>(b.H, d, b.part, S, Mj, Np, lw + m.off_gmlp, m.eps, b.xhi, b.xlo,
+        k_rows_add_norm<<<Mj, kNormThreads, 0, s>>>(b.H, d, b.part, S, Mj, Np, lw + m.off_gmlp, m.eps, b.xhi, b.xlo,
                                                      b.ldx);
         RCK(cudaGetLastError());
         RCK(launch_mm(lw + m.off_wgu, 2LL * m.F, d, b, Mj, S, Np, s));
@@ -522,7 +602,7 @@ cudaError_t rows_pass(const DevModel& m, const RowsBuf& b, const int* start, int
         Np_prev = Np;
     }
     // the last down projection into the residual (no norm)
-    k_rows_add_norm<<<M_prev, kRowsThreads, 0, s>>>(b.H, d, b.part, S_prev, M_prev, Np_prev, nullptr, m.eps, b.xhi,
+    k_rows_add_norm<<<M_prev, kNormThreads, 0, s>>>(b.H, d, b.part, S_prev, M_prev, Np_prev, nullptr, m.eps, b.xhi,
                                                     b.xlo, b.ldx);
     return cudaGetLastError();
 }
