@@ -507,7 +507,7 @@ def run_ours(args, rank: int, world: int, local: int):
             dt = time.perf_counter() - t0
             key = "batched" if rows else "one_position_at_a_time"
             repass[key] = {"repassed": n_rp, "ms": dt * 1e3, "token_times": dt * head["tok_s"]}
-        eng.set_option(OPT_ROWS, 1)
+        eng.set_option(OPT_ROWS, 0)
         b = repass["batched"]
         _log(f"[bench] re-pass of {b['repassed']} exited positions: {b['ms']:.2f} ms ({b['token_times']:.2f} "
              f"token-times); one position at a time {repass['one_position_at_a_time']['ms']:.2f} ms")
@@ -529,7 +529,7 @@ def run_ours(args, rank: int, world: int, local: int):
             passes = batches if rows else P
             prefill[key] = {"ms": dt * 1e3, "tok_s": P / dt,
                             "weight_GBps": passes * bm.layer_weight_bytes(run.dims) * shape.n_layers / dt / 1e9}
-        eng.set_option(OPT_ROWS, 1)
+        eng.set_option(OPT_ROWS, 0)
         _log(f"[bench] prompt of {P}: {prefill['batched']['ms']:.2f} ms batched "
              f"({prefill['batched']['tok_s']:.0f} tok/s), {prefill['one_position_at_a_time']['ms']:.1f} ms "
              f"one position at a time")
@@ -638,11 +638,12 @@ def profile_rows(shape, model, local: int):
     A 128-position prompt in two batches, 16 exit steps (direct launches),
     then one re-pass of those 16 positions in one batch.  Prints the launch
     counts of each part."""
-    from paper_2609_14144_gb300 import DEVICE, FORCE_EXIT_AT, OPT_GRAPHS, Engine
+    from paper_2609_14144_gb300 import DEVICE, FORCE_EXIT_AT, OPT_GRAPHS, OPT_ROWS, Engine
 
     P, n = 128, REPASS_W
     eng = Engine(shape, model, max_ctx=P + n, device=local)
     eng.set_option(OPT_GRAPHS, 0)
+    eng.set_option(OPT_ROWS, 1)
     eng.prefill(synth.prompt(shape, P))
     eng.decode_n(n, [0.5], schedule=np.full(n, FORCE_EXIT_AT(0), np.int8), where=DEVICE)
     eng.sync()

@@ -263,11 +263,13 @@ int ee_position(ee_ctx* ctx, int32_t* pos);
                                  ee_decode_step report the nucleus membership of
                                  readout 0's token at share value/1000
                                  (Section 2 acceptance)                      */
-#define EE_OPT_ROWS 8         /* 1 (default): ee_prefill and ee_repass run each
-                                 layer over batches of up to 64 positions
-                                 (tensor-core products, each weight read once
-                                 per batch); 0: one position at a time through
-                                 the decode step's layer kernels            */
+#define EE_OPT_ROWS 8         /* 1: ee_prefill and ee_repass run each layer
+                                 over batches of up to 64 positions (tensor-
+                                 core products, each weight read once per
+                                 batch, activations carried as bf16 high and
+                                 low parts: 16 significant bits); 0 (default):
+                                 one position at a time through the decode
+                                 step's layer kernels (fp32 activations)    */
 int ee_set_option(ee_ctx* ctx, int option, int value);
 
 #define EE_DBG_HIDDEN_READOUT 1 /* layer = readout r: residual h_k it read, d floats   */

@@ -59,7 +59,7 @@ struct Layout {
     size_t kpool, vpool, page_table, kv_src, h_exit, exit_at, repass_pos, h, q, o, a, y, hk, logits_ro, logits_final;
     size_t gemv_part, gemv_ticket, attn_part, attn_ticket, vocab_part, vocab_ticket;
     size_t seg_dpart, seg_opart, seg_q, seg_kvn, seg_a, seg_attn, seg_sync, seg_end;
-    size_t rows_H, rows_xhi, rows_xlo, rows_Q, rows_part, rows_pos;
+    size_t rows_H, rows_xhi, rows_xmid, rows_xlo, rows_Q, rows_part, rows_pos;
     size_t prompt, sched, out_tok, out_exit, out_conf, out_conf_all, out_member, out_mass, tau_scratch, total;
     int64_t layer_stride, off_wqkv, off_bqkv, off_gattn, off_wo, off_gmlp, off_wgu, off_wd;
     int64_t n_units_qkv, kv_layer_stride, gemv_ticket_stride, rows_part_floats;
@@ -169,6 +169,7 @@ Layout make_layout(const ee_model_config& c) {
     l.rows_part_floats = rows_part_floats((int)d, (int)A, (int)KH, (int)D, (int)F);
     l.rows_H = take(4 * (size_t)kRowsMax * d);
     l.rows_xhi = take(2 * (size_t)kRowsMax * l.rows_ldx);
+    l.rows_xmid = take(2 * (size_t)kRowsMax * l.rows_ldx);
     l.rows_xlo = take(2 * (size_t)kRowsMax * l.rows_ldx);
     l.rows_Q = take(4 * (size_t)kRowsMax * A * D);
     l.rows_part = take(4 * (size_t)l.rows_part_floats);
@@ -240,7 +241,7 @@ struct ee_ctx {
     SegPlan seg{};
     bool vring_ok = false;  // ring-fed vocabulary pass supported (used with the persistent layers)
     VocabRing vring{};
-    bool use_rows = true;   // EE_OPT_ROWS: prompt and re-pass in batches of positions
+    bool use_rows = false;  // EE_OPT_ROWS: prompt and re-pass in batches of positions
     RowsBuf rows{};
     int dbg = 0;
     int conf_kind = EE_CONF_PMAX;  // signal the gates compare with tau
@@ -841,6 +842,7 @@ int ee_create(const ee_model_config* cfg, void* d_workspace, size_t workspace_by
     c->d_ctl = m.ctl;
     c->rows.H = (float*)(w + l.rows_H);
     c->rows.xhi = (uint16_t*)(w + l.rows_xhi);
+    c->rows.xmid = (uint16_t*)(w + l.rows_xmid);
     c->rows.xlo = (uint16_t*)(w + l.rows_xlo);
     c->rows.Q = (float*)(w + l.rows_Q);
     c->rows.part = (float*)(w + l.rows_part);

@@ -230,13 +230,14 @@ cudaError_t launch_vocab_ring(const VocabArgs& v, const VocabRing& vr, bool pdl,
 // Multi-position layer pass (ee_rows.cu): the prompt and the re-pass run
 // each layer over up to kRowsMax positions at once, every weight byte read
 // once per batch.  Products are tensor-core mma of the bf16 weights with the
-// fp32 activations split into bf16 high and low parts.
+// fp32 activations split into three bf16 parts (high, middle, low).
 constexpr int kRowsMax = 64;             // positions per batch
 constexpr int kRowsTargetUnits = 2432;   // (tile, K split) units a projection aims for: 152 SMs x 16 warps
 struct RowsBuf {
     float* H;           // [kRowsMax][d] residual of each row
     uint16_t* xhi;      // [kRowsMax][ldx] next product's input, bf16 high part
-    uint16_t* xlo;      // [kRowsMax][ldx] low part (x - high, rounded)
+    uint16_t* xmid;     // [kRowsMax][ldx] middle part: x - high, rounded
+    uint16_t* xlo;      // [kRowsMax][ldx] low part: x - high - middle, rounded
     float* Q;           // [kRowsMax][A D] rotated queries
     float* part;        // split partials [S][M][n_rows padded to 32]
     int32_t* pos;       // [kRowsMax] positions of a prompt batch

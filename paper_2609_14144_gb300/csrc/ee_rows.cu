@@ -5,8 +5,8 @@
 //
 // A layer is nine launches, each reading what the previous one wrote:
 //   k_rows_add_norm  residual add of the previous projection's split
-//                    partials (in split order), then RMSNorm with the next
-//                    gain, written as bf16 high and low parts
+//                    partials (in a fixed order), then RMSNorm with the next
+//                    gain, written as three bf16 parts
 //   k_rows_mm        a projection: Y[row][n] = sum_k W[n][k] x[row][k]
 //   k_rows_qkv       split sum, bias, RoPE at each row's position; q kept in
 //                    fp32, k and v stored bf16 into the paged cache
@@ -23,9 +23,10 @@
 // operands agree, so a lane's chunk feeds its A fragment as loaded (slots
 // 2q, 2q+1, 2q+8, 2q+9 of the lane's k group q take the chunk's first four
 // elements, the second mma the last four) and the activations are read in the
-// same order.  Activations stay fp32 in meaning: each is split into a bf16
-// high part and the bf16 rounding of the remainder, and both are multiplied
-// (16 significant bits, within ~1e-5 relative of fp32).  Weights are the
+// same order.  Activations keep fp32 precision: each is split into three
+// bf16 parts, x = high + middle + low (each the rounding of what the parts
+// before it leave, 24 significant bits in all), and the weights are
+// multiplied with each; bf16 products are exact in the fp32 accumulator.  Weights are the
 // A operand (16 output rows per mma), positions the B operand (8 per mma).
 //
 // Partial sums of the K splits go to a scratch buffer and the consumer adds
@@ -51,11 +52,21 @@ __device__ __forceinline__ uint16_t r_f2bf(float f) { return __bfloat16_as_ushor
 __device__ __forceinline__ float r_lo(uint32_t u) { return __uint_as_float(u << 16); }
 __device__ __forceinline__ float r_hi(uint32_t u) { return __uint_as_float(u & 0xffff0000u); }
 
-// x as bf16 high part and the bf16 rounding of x - high.
-__device__ __forceinline__ void split_store(float x, uint16_t* hi, uint16_t* lo) {
+// The three bf16 part arrays of a product's input (same layout each).
+struct Parts {
+    uint16_t *hi, *mid, *lo;
+};
+
+// The three bf16 parts of x at element `at` of each part array: high =
+// bf16(x), middle = bf16(x - high), low = bf16(x - high - middle) (each
+// difference exact in fp32).
+__device__ __forceinline__ void split_store(float x, const Parts& p, int64_t at) {
     const uint16_t h = r_f2bf(x);
-    *hi = h;
-    *lo = r_f2bf(x - r_bf2f(h));
+    const float r1 = x - r_bf2f(h);
+    const uint16_t md = r_f2bf(r1);
+    p.hi[at] = h;
+    p.mid[at] = md;
+    p.lo[at] = r_f2bf(r1 - r_bf2f(md));
 }
 
 // Weights are read once per batch: streamed past L1, first out of L2.
@@ -99,7 +110,7 @@ __device__ __forceinline__ int64_t slot_offset(const DevModel& m, int j, int pos
 // ------------------------------------------------------------------ projection
 //
 // part[s][row][n] = sum over the k of split s of W[n][k] x[row][k], for the
-// M rows of x (bf16 high and low parts, row stride ldx) and every output n of
+// M rows of x (three bf16 parts, row stride ldx) and every output n of
 // the tiled weights.  A unit is (tile, split, row group): NB blocks of 8 rows
 // starting at row group * 8 NB (rows past M read as zero and are not
 // stored); the row groups of one (tile, split) are neighbouring warps, so a
@@ -108,8 +119,7 @@ __device__ __forceinline__ int64_t slot_offset(const DevModel& m, int j, int pos
 // past K reads as zero on both sides.
 template <int NB, int U>
 __global__ void __launch_bounds__(kRowsThreads) k_rows_mm(const uint4* __restrict__ W, int n_tiles, int K,
-                                                          const uint16_t* __restrict__ xhi,
-                                                          const uint16_t* __restrict__ xlo, int ldx, int M, int S,
+                                                          const Parts x3, int ldx, int M, int S,
                                                           int RG, float* __restrict__ part, int Np) {
     const int lane = threadIdx.x & 31, g = lane >> 2, q = lane & 3;
     const int Rc = K >> 3;             // 16-byte chunks per weight row
@@ -130,7 +140,7 @@ __global__ void __launch_bounds__(kRowsThreads) k_rows_mm(const uint4* __restric
 #pragma unroll
                 for (int e = 0; e < 4; ++e) acc[a][n][e] = 0.f;
         for (int st = st0; st < st1; st += U) {
-            uint4 w[U][4], bh[U][NB], bl[U][NB];
+            uint4 w[U][4], bh[U][NB], bm[U][NB], bl[U][NB];
 #pragma unroll
             for (int v = 0; v < U; ++v) {
                 const int ch = (st + v) * 4 + q;  // this lane's chunk of the step
@@ -143,8 +153,9 @@ __global__ void __launch_bounds__(kRowsThreads) k_rows_mm(const uint4* __restric
                     const int row = r0 + n * 8 + g;
                     const bool okx = ok && row < M;
                     const int64_t at = (int64_t)row * ldx + ch * 8;
-                    bh[v][n] = okx ? ld_act(xhi + at) : make_uint4(0u, 0u, 0u, 0u);
-                    bl[v][n] = okx ? ld_act(xlo + at) : make_uint4(0u, 0u, 0u, 0u);
+                    bh[v][n] = okx ? ld_act(x3.hi + at) : make_uint4(0u, 0u, 0u, 0u);
+                    bm[v][n] = okx ? ld_act(x3.mid + at) : make_uint4(0u, 0u, 0u, 0u);
+                    bl[v][n] = okx ? ld_act(x3.lo + at) : make_uint4(0u, 0u, 0u, 0u);
                 }
             }
 #pragma unroll
@@ -152,16 +163,16 @@ __global__ void __launch_bounds__(kRowsThreads) k_rows_mm(const uint4* __restric
                 const uint4* x = w[v];
 #pragma unroll
                 for (int n = 0; n < NB; ++n) {
-                    const uint4 h = bh[v][n], l = bl[v][n];
-                    // first mma of the step: chunk elements 0..3; second: 4..7
-                    mma_16816(acc[0][n], x[0].x, x[1].x, x[0].y, x[1].y, h.x, h.y);
-                    mma_16816(acc[0][n], x[0].x, x[1].x, x[0].y, x[1].y, l.x, l.y);
-                    mma_16816(acc[0][n], x[0].z, x[1].z, x[0].w, x[1].w, h.z, h.w);
-                    mma_16816(acc[0][n], x[0].z, x[1].z, x[0].w, x[1].w, l.z, l.w);
-                    mma_16816(acc[1][n], x[2].x, x[3].x, x[2].y, x[3].y, h.x, h.y);
-                    mma_16816(acc[1][n], x[2].x, x[3].x, x[2].y, x[3].y, l.x, l.y);
-                    mma_16816(acc[1][n], x[2].z, x[3].z, x[2].w, x[3].w, h.z, h.w);
-                    mma_16816(acc[1][n], x[2].z, x[3].z, x[2].w, x[3].w, l.z, l.w);
+                    const uint4 parts[3] = {bh[v][n], bm[v][n], bl[v][n]};
+#pragma unroll
+                    for (int pp = 0; pp < 3; ++pp) {
+                        const uint4 b = parts[pp];
+                        // first mma of the step: chunk elements 0..3; second: 4..7
+                        mma_16816(acc[0][n], x[0].x, x[1].x, x[0].y, x[1].y, b.x, b.y);
+                        mma_16816(acc[0][n], x[0].z, x[1].z, x[0].w, x[1].w, b.z, b.w);
+                        mma_16816(acc[1][n], x[2].x, x[3].x, x[2].y, x[3].y, b.x, b.y);
+                        mma_16816(acc[1][n], x[2].z, x[3].z, x[2].w, x[3].w, b.z, b.w);
+                    }
                 }
             }
         }
@@ -216,13 +227,12 @@ __device__ __forceinline__ float split_sum(const float* __restrict__ p, int64_t 
 
 // One CTA per row i < M_norm.  Rows below M_add first add the split partials
 // of a d-output projection (split stride M_add rows) to their residual.  With
-// a gain, the row's RMSNorm h / sqrt(mean(h^2) + eps) * g goes to x as bf16
-// high and low parts.
+// a gain, the row's RMSNorm h / sqrt(mean(h^2) + eps) * g goes to x as three
+// bf16 parts.
 __global__ void __launch_bounds__(kNormThreads) k_rows_add_norm(float* __restrict__ H, int d,
                                                                 const float* __restrict__ part, int S, int M_add,
                                                                 int Np, const uint16_t* __restrict__ gain, float eps,
-                                                                uint16_t* __restrict__ xhi, uint16_t* __restrict__ xlo,
-                                                                int ldx) {
+                                                                const Parts x3, int ldx) {
     __shared__ float red[kNormThreads / 32];
     const int i = blockIdx.x;
     float* h = H + (int64_t)i * d;
@@ -240,7 +250,7 @@ __global__ void __launch_bounds__(kNormThreads) k_rows_add_norm(float* __restric
     const float inv = 1.0f / sqrtf(ss / (float)d + eps);
     for (int n = threadIdx.x; n < d; n += kNormThreads) {
         const float x = h[n] * inv * r_bf2f(gain[n]);
-        split_store(x, xhi + (int64_t)i * ldx + n, xlo + (int64_t)i * ldx + n);
+        split_store(x, x3, (int64_t)i * ldx + n);
     }
 }
 
@@ -285,17 +295,16 @@ __global__ void __launch_bounds__(kRowsThreads) k_rows_qkv(DevModel m, int j, co
 }
 
 // SwiGLU of row blockIdx.y: a = silu(gate) * up from the split sums of the
-// packed (gate, up) row pair, as bf16 high and low parts.
+// packed (gate, up) row pair, as three bf16 parts.
 __global__ void __launch_bounds__(kRowsThreads) k_rows_swiglu(const float* __restrict__ part, int S, int M, int Np,
-                                                              int F, uint16_t* __restrict__ xhi,
-                                                              uint16_t* __restrict__ xlo, int ldx) {
+                                                              int F, const Parts x3, int ldx) {
     const int i = blockIdx.y;
     const int f = blockIdx.x * kRowsThreads + threadIdx.x;
     if (f >= F) return;
     const float* p = part + (int64_t)i * Np + 2 * f;
     const float gs = split_sum(p, (int64_t)M * Np, S), us = split_sum(p + 1, (int64_t)M * Np, S);
     const float a = gs / (1.0f + expf(-gs)) * us;
-    split_store(a, xhi + (int64_t)i * ldx + f, xlo + (int64_t)i * ldx + f);
+    split_store(a, x3, (int64_t)i * ldx + f);
 }
 
 // Starting residual of row blockIdx.x: the embedding of ids[i] (a prompt;
@@ -338,11 +347,10 @@ __global__ void k_rows_prefill_done(DevModel m, int n) {
 // taking its own 32 keys of the chunk (lane l owning dimensions
 // l*D/32 .. l*D/32 + D/32 - 1 of every head), rescaled whenever the maximum
 // grows; the warps' sums are added in warp order at the end (Section 2's
-// softmax attention).  Output o at column h*D + e as bf16 high and low parts.
+// softmax attention).  Output o at column h*D + e as three bf16 parts.
 template <int D>
 __global__ void __launch_bounds__(kRowsThreads) k_rows_attn(DevModel m, int j, const float* __restrict__ Q,
-                                                            const int32_t* __restrict__ pos,
-                                                            uint16_t* __restrict__ xhi, uint16_t* __restrict__ xlo,
+                                                            const int32_t* __restrict__ pos, const Parts x3,
                                                             int ldx) {
     constexpr int kG = kSegMaxGroup;  // query heads per kv head (at most)
     constexpr int DL = D / 32;        // dimensions per lane in the value sums
@@ -484,11 +492,13 @@ __global__ void __launch_bounds__(kRowsThreads) k_rows_attn(DevModel m, int j, c
     for (int idx = tid; idx < G * D; idx += kRowsThreads) {
         const int h = idx / D, e = idx - h * D;
         const int64_t col = (int64_t)(g * G + h) * D + e;
-        split_store(acc[idx] / lrun[h], xhi + (int64_t)i * ldx + col, xlo + (int64_t)i * ldx + col);
+        split_store(acc[idx] / lrun[h], x3, (int64_t)i * ldx + col);
     }
 }
 
 // ------------------------------------------------------------------ host side
+
+Parts parts(const RowsBuf& b) { return Parts{b.xhi, b.xmid, b.xlo}; }
 
 // Row blocks of 8 a warp takes (1, 2 or 4) and the row groups of a batch.
 void row_groups(int M, int& NB, int& RG) {
@@ -498,7 +508,7 @@ void row_groups(int M, int& NB, int& RG) {
 }
 
 // One projection of the batch: W (n_rows x K, tiled) times the M rows of
-// b.xhi / b.xlo into b.part; returns the split count and padded row count
+// b.xhi / b.xmid / b.xlo into b.part; returns the split count and padded row count
 // its consumer needs.
 cudaError_t launch_mm(const uint16_t* W, int64_t n_rows, int K, const RowsBuf& b, int M, int& S, int& Np,
                       cudaStream_t s) {
@@ -511,11 +521,11 @@ cudaError_t launch_mm(const uint16_t* W, int64_t n_rows, int K, const RowsBuf& b
     const int grid = (int)std::min<int64_t>((units + kRowsWarps - 1) / kRowsWarps, 65535);
     const uint4* w = reinterpret_cast<const uint4*>(W);
     if (NB == 1)
-        k_rows_mm<1, 2><<<grid, kRowsThreads, 0, s>>>(w, (int)nt, K, b.xhi, b.xlo, b.ldx, M, S, RG, b.part, Np);
+        k_rows_mm<1, 2><<<grid, kRowsThreads, 0, s>>>(w, (int)nt, K, parts(b), b.ldx, M, S, RG, b.part, Np);
     else if (NB == 2)
-        k_rows_mm<2, 2><<<grid, kRowsThreads, 0, s>>>(w, (int)nt, K, b.xhi, b.xlo, b.ldx, M, S, RG, b.part, Np);
+        k_rows_mm<2, 2><<<grid, kRowsThreads, 0, s>>>(w, (int)nt, K, parts(b), b.ldx, M, S, RG, b.part, Np);
     else
-        k_rows_mm<4, 1><<<grid, kRowsThreads, 0, s>>>(w, (int)nt, K, b.xhi, b.xlo, b.ldx, M, S, RG, b.part, Np);
+        k_rows_mm<4, 1><<<grid, kRowsThreads, 0, s>>>(w, (int)nt, K, parts(b), b.ldx, M, S, RG, b.part, Np);
     return cudaGetLastError();
 }
 
@@ -575,7 +585,7 @@ cudaError_t rows_pass(const DevModel& m, const RowsBuf& b, const int* start, int
         int S = 1, Np = 0;
         // the previous layer's down projection into the residual, this layer's input norm
         k_rows_add_norm<<<Mj, kNormThreads, 0, s>>>(b.H, d, b.part, S_prev, M_prev, Np_prev, lw + m.off_gattn, m.eps,
-                                                     b.xhi, b.xlo, b.ldx);
+                                                     parts(b), b.ldx);
         RCK(cudaGetLastError());
         RCK(launch_mm(lw + m.off_wqkv, nqkv, d, b, Mj, S, Np, s));
         const int nu = (int)(nqkv / 2);
@@ -584,17 +594,17 @@ cudaError_t rows_pass(const DevModel& m, const RowsBuf& b, const int* start, int
         RCK(cudaGetLastError());
         if (kv_only && j == L - 1) return cudaSuccess;
         if (m.D == 128)
-            k_rows_attn<128><<<dim3(m.KH, Mj), kRowsThreads, 0, s>>>(m, j, b.Q, d_pos, b.xhi, b.xlo, b.ldx);
+            k_rows_attn<128><<<dim3(m.KH, Mj), kRowsThreads, 0, s>>>(m, j, b.Q, d_pos, parts(b), b.ldx);
         else
-            k_rows_attn<64><<<dim3(m.KH, Mj), kRowsThreads, 0, s>>>(m, j, b.Q, d_pos, b.xhi, b.xlo, b.ldx);
+            k_rows_attn<64><<<dim3(m.KH, Mj), kRowsThreads, 0, s>>>(m, j, b.Q, d_pos, parts(b), b.ldx);
         RCK(cudaGetLastError());
         RCK(launch_mm(lw + m.off_wo, d, AD, b, Mj, S, Np, s));
-        k_rows_add_norm<<<Mj, kNormThreads, 0, s>>>(b.H, d, b.part, S, Mj, Np, lw + m.off_gmlp, m.eps, b.xhi, b.xlo,
+        k_rows_add_norm<<<Mj, kNormThreads, 0, s>>>(b.H, d, b.part, S, Mj, Np, lw + m.off_gmlp, m.eps, parts(b),
                                                      b.ldx);
         RCK(cudaGetLastError());
         RCK(launch_mm(lw + m.off_wgu, 2LL * m.F, d, b, Mj, S, Np, s));
         k_rows_swiglu<<<dim3((m.F + kRowsThreads - 1) / kRowsThreads, Mj), kRowsThreads, 0, s>>>(b.part, S, Mj, Np, m.F,
-                                                                                                 b.xhi, b.xlo, b.ldx);
+                                                                                                 parts(b), b.ldx);
         RCK(cudaGetLastError());
         RCK(launch_mm(lw + m.off_wd, d, m.F, b, Mj, S, Np, s));
         M_prev = Mj;
@@ -602,8 +612,8 @@ cudaError_t rows_pass(const DevModel& m, const RowsBuf& b, const int* start, int
         Np_prev = Np;
     }
     // the last down projection into the residual (no norm)
-    k_rows_add_norm<<<M_prev, kNormThreads, 0, s>>>(b.H, d, b.part, S_prev, M_prev, Np_prev, nullptr, m.eps, b.xhi,
-                                                    b.xlo, b.ldx);
+    k_rows_add_norm<<<M_prev, kNormThreads, 0, s>>>(b.H, d, b.part, S_prev, M_prev, Np_prev, nullptr, m.eps,
+                                                    parts(b), b.ldx);
     return cudaGetLastError();
 }
 

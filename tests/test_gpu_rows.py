@@ -1,13 +1,13 @@
 """The multi-position layer pass on the GPU (needs a GB300).
 
-With EE_OPT_ROWS = 1 (the default) the prompt and the re-pass run each layer
-over batches of up to 64 positions.  Checked against the oracle (first token
-exact outside the 1e-3 top-2 band, final hidden state and logits and every
-cache entry within 1e-2 relative, which (layer, position) entries were
-computed bit for bit) and against the same engine one position at a time
-(EE_OPT_ROWS = 0): both keep activations at fp32 precision (the batched
-products through bf16 high and low parts), so fp32 results agree within 1e-3
-relative; cache entries are bf16, where one rounding step is 4e-3."""
+With EE_OPT_ROWS = 1 the prompt and the re-pass run each layer over batches
+of up to 64 positions.  Checked against the oracle (first token exact outside
+the 1e-3 top-2 band, final hidden state and logits and every cache entry
+within 1e-2 relative, which (layer, position) entries were computed bit for
+bit) and against the same engine one position at a time (EE_OPT_ROWS = 0,
+the default): both keep activations at fp32 precision (the batched products
+through three bf16 parts of each activation), so fp32 results agree within
+1e-3 relative; cache entries are bf16, where one rounding step is 4e-3."""
 import numpy as np
 import pytest
 
