@@ -649,7 +649,7 @@ def profile_rows(shape, model, local: int):
     eng.sync()
     n_rp = eng.repass(P, P + n)
     L, k = shape.n_layers, shape.readout_layers[0]
-    prefill = rows_launches(L, ROWS_MAX, True) + rows_launches(L, P - ROWS_MAX, False) + 3
+    prefill = rows_launches(L, ROWS_MAX, True) + rows_launches(L, P - ROWS_MAX, False) + 4
     decode = sum(step_launches(L, shape.readout_layers, 0, eng.persistent) for _ in range(n)) + 1
     repass = rows_launches(L - k, n, False)
     print(json.dumps({"prefill_launches": prefill, "decode_launches": decode, "repass_launches": repass,
