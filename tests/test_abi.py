@@ -67,3 +67,12 @@ def test_scratch_sizes_and_null_contexts(lib):
     for f in (lib.ee_reset, lib.ee_sync):
         assert f(None) == _lib.EE_EINVAL
     assert lib.ee_destroy(None) == 0
+
+
+def test_option_constants_match_the_header():
+    """Every EE_OPT_* value include/ee.h defines is the binding's OPT_* value."""
+    src = open(os.path.join(ROOT, "include", "ee.h")).read()
+    defs = dict(re.findall(r"^#define EE_OPT_(\w+)\s+(\d+)", src, flags=re.M))
+    assert len(defs) >= 8
+    for name, value in defs.items():
+        assert getattr(_lib, "OPT_" + name) == int(value), name
