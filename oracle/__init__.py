@@ -123,6 +123,8 @@ def _load():
                                             ctypes.POINTER(Capture)]
             lib.orc_position.argtypes = [_P]
             lib.orc_repass.argtypes = [_P, ctypes.c_int, ctypes.c_int]
+            lib.orc_set_lazy_fill.argtypes = [_P, ctypes.c_int]
+            lib.orc_flush_fills.argtypes = [_P]
             lib.orc_kv.argtypes = [_P, ctypes.c_int, ctypes.c_int, _P, _P, ctypes.POINTER(ctypes.c_int8)]
             lib.orc_stats.argtypes = [_P, _P]
             del f32p
@@ -287,6 +289,18 @@ class Oracle:
         """Gate signal: CONF_PMAX (default), CONF_MARGIN or CONF_NEGENT (Section 10)."""
         if self.lib.orc_set_confidence(self.ptr, int(kind)) != 0:
             raise ValueError("oracle: bad confidence kind")
+
+    def set_lazy_fill(self, on: bool):
+        """Deferred KV fill: exit steps leave their skipped entries empty and
+        the first later step that runs a layer fills that layer's pending
+        entries first (the same projection of the same exit residual).
+        Turning it off fills every pending entry."""
+        if self.lib.orc_set_lazy_fill(self.ptr, int(bool(on))) != 0:
+            raise ValueError("oracle: bad lazy-fill setting")
+
+    def flush_fills(self):
+        """Fill every entry an exit step deferred."""
+        self.lib.orc_flush_fills(self.ptr)
 
     @property
     def pos(self) -> int:

@@ -32,6 +32,10 @@
  *   - Section 11: a periodic full-depth pass over the most recent tokens
  *     recomputes their cache entries exactly (orc_repass): each token that
  *     exited runs its skipped layers from the residual it exited with.
+ *   - Section 4, step five, deferred (orc_set_lazy_fill): a skipped entry is
+ *     only read by a later token that runs its layer, so its fill may wait
+ *     until the first such token; it is the same projection of the same
+ *     exit-layer residual.
  *   - Appendix C: the layer is four attention projections with grouped-query
  *     attention (A query heads, K key-value heads of size D) and a gated
  *     feed-forward block of three matrices of width F.
@@ -143,12 +147,13 @@ typedef struct {
     const uint16_t* readout_b[ORC_MAX_READOUTS];
     float* kc;       /* [L][K][max_ctx][D], bf16 values */
     float* vc;
-    int8_t* kv_src;  /* [L][max_ctx]: 0 empty, 1 computed by the layer, 2 filled */
+    int8_t* kv_src;  /* [L][max_ctx]: 0 empty (or a deferred fill), 1 computed by the layer, 2 filled */
     float* h_exit;   /* [max_ctx][d]: the residual a position exited with */
     int16_t* exit_at; /* [max_ctx]: layer a position exited after (0: ran every layer) */
     int pos;
     int conf_kind; /* ORC_CONF_*: the signal the gate compares with tau */
     double nucleus_p; /* share of probability the nucleus holds */
+    int lazy_fill;    /* 1: exit steps leave their skipped entries empty (flush_layer fills them) */
     int64_t steps, full_steps, exits[ORC_MAX_READOUTS];
     float *h, *u, *q, *kk, *vv, *o, *g, *up, *a, *y, *z, *logits, *tmp;
 } orc_model;
@@ -557,6 +562,40 @@ static void kv_fill(orc_model* m, int j, int t, const float* hk) {
     store_kv(m, j, t, m->kk, m->vv, 2);
 }
 
+/* Deferred fills of layer j (0-based) needed before position t reads it:
+ * every position p < t that exited after layer k <= j and whose entry at
+ * layer j is still empty gets the fill kv_fill would have written in its
+ * exit step, from the residual it exited with.  Nothing to do unless the
+ * lazy fill is on. */
+static void flush_layer(orc_model* m, int j, int t) {
+    if (!m->lazy_fill) return;
+    const orc_config* c = &m->c;
+    for (int p = 0; p < t; ++p) {
+        const int k = m->exit_at[p];
+        if (k > 0 && k <= j && m->kv_src[(size_t)j * c->max_ctx + p] == 0)
+            kv_fill(m, j, p, m->h_exit + (size_t)p * c->d_model);
+    }
+}
+
+/* Every deferred fill at positions before the current one. */
+int orc_flush_fills(orc_model* m) {
+    if (!m) return -1;
+    const int lazy = m->lazy_fill;
+    m->lazy_fill = 1;
+    for (int j = 0; j < m->c.n_layers; ++j) flush_layer(m, j, m->pos);
+    m->lazy_fill = lazy;
+    return 0;
+}
+
+/* on = 1: exit steps defer their fills; on = 0 fills every deferred entry
+ * first, then fills in the exit step again. */
+int orc_set_lazy_fill(orc_model* m, int on) {
+    if (!m || (on != 0 && on != 1)) return -1;
+    if (!on) orc_flush_fills(m);
+    m->lazy_fill = on;
+    return 0;
+}
+
 /* Final normalisation + unembedding of a residual-space vector x:
  * logits = U bf16(RMSNorm(x) * g_final). */
 static void unembed(orc_model* m, const float* x, float* logits) {
@@ -629,6 +668,7 @@ int orc_decode_step(orc_model* m, int32_t in_tok, const float* taus, int force, 
     for (int x = 0; x < d; ++x) m->h[x] = bf16_bits_to_f32(e[x]);
     int r = 0, exited = 0;
     for (int j = 0; j < L && !exited; ++j) {
+        flush_layer(m, j, t);
         layer_forward(m, j, t, m->h, cap && cap->layer_trace ? cap->layer_trace + (size_t)j * tstride : NULL);
         if (r < m->n_readouts && m->readout_layer[r] == j + 1) {
             readout(m, r, m->h, m->y, m->logits);
@@ -650,7 +690,8 @@ int orc_decode_step(orc_model* m, int32_t in_tok, const float* taus, int force, 
                 res->exit_readout = r;
                 res->exit_layer = j + 1;
                 res->token = cf.argmax;
-                for (int jj = j + 1; jj < L; ++jj) kv_fill(m, jj, t, m->h);
+                if (!m->lazy_fill)
+                    for (int jj = j + 1; jj < L; ++jj) kv_fill(m, jj, t, m->h);
                 memcpy(m->h_exit + (size_t)t * d, m->h, sizeof(float) * d);
                 m->exit_at[t] = (int16_t)(j + 1);
             }
@@ -684,12 +725,13 @@ int orc_decode_step(orc_model* m, int32_t in_tok, const float* taus, int force, 
 int orc_position(const orc_model* m) { return m->pos; }
 
 /* Section 11's full-depth re-pass: for each position t in [t0, t1), in
- * order, whose upper layers still hold filled entries (it exited after layer
- * k, kv_src[k][t] == 2), run layers k+1..L from the residual it exited with,
- * storing computed entries in place of the filled ones.  Attention at t sees
- * the cache as it stands, including positions re-passed just before.  The
- * decode position is unchanged.  Returns the number of positions re-passed
- * (-1 on a bad range). */
+ * order, whose upper layers still hold filled (or deferred) entries (it
+ * exited after layer k and kv_src[k][t] is not 1), run layers k+1..L from the
+ * residual it exited with, storing computed entries in place of the filled
+ * ones.  Attention at t sees the cache as it stands (deferred fills of
+ * earlier positions done first), including positions re-passed just before.
+ * The decode position is unchanged.  Returns the number of positions
+ * re-passed (-1 on a bad range). */
 int orc_repass(orc_model* m, int t0, int t1) {
     if (!m || t0 < 0 || t1 < t0 || t1 > m->pos) return -1;
     const orc_config* c = &m->c;
@@ -697,9 +739,12 @@ int orc_repass(orc_model* m, int t0, int t1) {
     int n = 0;
     for (int t = t0; t < t1; ++t) {
         const int k = m->exit_at[t];
-        if (k <= 0 || k >= L || m->kv_src[(size_t)k * c->max_ctx + t] != 2) continue;
+        if (k <= 0 || k >= L || m->kv_src[(size_t)k * c->max_ctx + t] == 1) continue;
         memcpy(m->y, m->h_exit + (size_t)t * d, sizeof(float) * d);
-        for (int j = k; j < L; ++j) layer_forward(m, j, t, m->y, NULL);
+        for (int j = k; j < L; ++j) {
+            flush_layer(m, j, t);
+            layer_forward(m, j, t, m->y, NULL);
+        }
         ++n;
     }
     return n;

@@ -484,3 +484,107 @@ def test_errors_and_determinism():
     _, f1, a = _run(shape, model, [0.4])
     _, f2, b = _run(shape, model, [0.4])
     assert [x["confidence"] for x in a] == [x["confidence"] for x in b]
+
+
+def _forced_run(shape, model, n, force_of, lazy):
+    """Decode n steps with the force values force_of(i); returns (oracle,
+    step results)."""
+    o = oracle.Oracle(shape, model, max_ctx=shape.prompt_len + n + 1)
+    o.set_lazy_fill(lazy)
+    tok = o.prefill(synth.prompt(shape))
+    taus = [2.0] * len(shape.readout_layers)
+    out = []
+    for i in range(n):
+        s = o.decode_step(tok, taus, force_of(i))
+        out.append(s)
+        tok = s["token"]
+    return o, out
+
+
+def _same_cache(a, b, shape, t_end):
+    for j in range(shape.n_layers):
+        for t in range(t_end):
+            ka, va, sa = a.kv(j, t)
+            kb, vb, sb = b.kv(j, t)
+            assert sa == sb and np.array_equal(ka, kb) and np.array_equal(va, vb), (j, t)
+
+
+def _every4_full(i):
+    return oracle.FORCE_FULL if i % 4 == 3 else oracle.FORCE_EXIT_AT(0)
+
+
+def test_lazy_fill_matches_the_eager_fill():
+    """Section 4 step five's fill deferred to the first step that runs the
+    layer: no token or confidence changes (an exit step reads only layers
+    below its exit), and once flushed the cache is the eager one bit for
+    bit (the same projection of the same exit residual)."""
+    model = synth.make_model(TINY)
+    n = 22
+    eager, a = _forced_run(TINY, model, n, _every4_full, False)
+    lazy, b = _forced_run(TINY, model, n, _every4_full, True)
+    for sa, sb in zip(a, b):
+        assert sa["token"] == sb["token"] and sa["exited"] == sb["exited"]
+        assert np.array_equal(sa["confidence"], sb["confidence"])
+    lazy.flush_fills()
+    _same_cache(eager, lazy, TINY, TINY.prompt_len + n)
+
+
+def test_lazy_fill_waits_for_a_step_that_runs_the_layer():
+    model = synth.make_model(TINY)
+    P, L, k = TINY.prompt_len, TINY.n_layers, TINY.readout_layers[0]
+    eager, _ = _forced_run(TINY, model, 6, _every4_full, False)
+    lazy, _ = _forced_run(TINY, model, 6, _every4_full, True)
+    # steps 0-2 exited and step 3 ran at full depth: their fills are done
+    for t in range(P, P + 3):
+        for j in range(k, L):
+            assert lazy.kv(j, t)[2] == 2
+    _same_cache(eager, lazy, TINY, P + 4)
+    # steps 4 and 5 exited after the last full step: still empty above k
+    for t in (P + 4, P + 5):
+        for j in range(L):
+            kl, vl, sl = lazy.kv(j, t)
+            if j < k:
+                assert sl == 1
+            else:
+                assert sl == 0 and not kl.any() and not vl.any()
+                assert eager.kv(j, t)[2] == 2
+
+
+def test_lazy_fill_with_readouts_at_several_depths():
+    """An exit deeper than a pending one fills that one's entries only in
+    the layers it runs; the rest wait for a full step."""
+    shape = TINY.replace(readout_layers=(1, 2, 3))
+    model = synth.make_model(shape)
+    P = shape.prompt_len
+    forces = [oracle.FORCE_EXIT_AT(0), oracle.FORCE_EXIT_AT(2), oracle.FORCE_FULL]
+    lazy, _ = _forced_run(shape, model, 2, lambda i: forces[i], True)
+    assert [lazy.kv(j, P)[2] for j in range(4)] == [1, 2, 2, 0]
+    assert [lazy.kv(j, P + 1)[2] for j in range(4)] == [1, 1, 1, 0]
+    eager, _ = _forced_run(shape, model, 3, lambda i: forces[i], False)
+    lazy, _ = _forced_run(shape, model, 3, lambda i: forces[i], True)
+    _same_cache(eager, lazy, shape, P + 3)
+
+
+def test_lazy_fill_and_the_repass():
+    """A re-pass over positions whose fills are still deferred computes the
+    same cache as a re-pass after eager fills."""
+    model = synth.make_model(TINY)
+    P, n = TINY.prompt_len, 14
+    eager, _ = _forced_run(TINY, model, n, _every4_full, False)
+    lazy, _ = _forced_run(TINY, model, n, _every4_full, True)
+    # the last position first: its attention reads the one before it, whose
+    # fills are still deferred in the lazy run
+    assert eager.repass(P + n - 1, P + n) == lazy.repass(P + n - 1, P + n) == 1
+    _same_cache(eager, lazy, TINY, P + n)
+    exits = sum(1 for i in range(n - 1) if i % 4 != 3)
+    assert eager.repass(P, P + n) == lazy.repass(P, P + n) == exits
+    _same_cache(eager, lazy, TINY, P + n)
+
+
+def test_turning_the_lazy_fill_off_fills_what_is_pending():
+    model = synth.make_model(TINY)
+    P, n = TINY.prompt_len, 6
+    eager, _ = _forced_run(TINY, model, n, _every4_full, False)
+    lazy, _ = _forced_run(TINY, model, n, _every4_full, True)
+    lazy.set_lazy_fill(False)
+    _same_cache(eager, lazy, TINY, P + n)
