@@ -1,0 +1,88 @@
+"""How far two correct implementations of the decode step can drift apart
+under the numerics contract (bf16 weights, fp32 activations, a bf16 KV
+cache), measured on the host with a plain PyTorch forward of the 0.5B shape.
+
+The same forward runs in fp32 and in fp64 over a 16-position prompt and one
+decode position, up to the readout at layer 12.  With the cache kept at
+full precision the two agree to a few 1e-6.  With the cache rounded to bf16,
+a tiny difference before rounding sometimes moves a cached value by one bf16
+step (4e-3 relative), and these moves compound over layers and positions:
+the readout residual and its top-1 probability then differ by about 1e-4.
+The GPU kernels and the oracle differ in summation order in the same way, so
+their agreement cannot be expected to be tighter than this; the effect grows
+with depth.  No GPU and no oracle are involved."""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import synth
+
+SHAPE = synth.CONFIGS["0.5b"].replace(prompt_len=16)
+
+
+@pytest.fixture(scope="module")
+def model():
+    return synth.make_model(SHAPE)
+
+
+def _f(a, dt):
+    return torch.from_numpy((np.asarray(a).astype(np.uint32) << 16).view(np.float32)).to(dt)
+
+
+def _readout(model, ids, dt, bf16_cache):
+    """Residual at the readout layer for the last position, and the readout's
+    top-1 probability (RMSNorm, rotate-half RoPE, grouped-query causal
+    attention, SwiGLU; readout = affine map, final RMSNorm, unembedding)."""
+    s = SHAPE
+    d, A, KH, D = s.d_model, s.n_heads, s.n_kv_heads, s.head_dim
+    T, half = len(ids), D // 2
+    h = torch.stack([_f(model["embed"][i], dt) for i in ids])
+    ang = torch.tensor([[t * math.pow(s.rope_base, -2.0 * i / D) for i in range(half)] for t in range(T)],
+                       dtype=torch.float64)
+    cs = torch.cos(ang).to(torch.float32).to(dt)[:, None]
+    sn = torch.sin(ang).to(torch.float32).to(dt)[:, None]
+
+    def rope(x):
+        a, b = x[..., :half], x[..., half:]
+        return torch.cat([a * cs - b * sn, a * sn + b * cs], -1)
+
+    def rms(x, g):
+        return x / torch.sqrt((x * x).mean(-1, keepdim=True) + s.rms_eps) * _f(g, dt)
+
+    mask = torch.triu(torch.ones(T, T, dtype=torch.bool), 1)
+    for j in range(s.readout_layers[0]):
+        w = model["layers"][j]
+        u = rms(h, w["attn_norm"])
+        q = rope((u @ _f(w["wq"], dt).T).view(T, A, D))
+        k = rope((u @ _f(w["wk"], dt).T).view(T, KH, D))
+        v = (u @ _f(w["wv"], dt).T).view(T, KH, D)
+        if bf16_cache:
+            k, v = k.to(torch.bfloat16).to(dt), v.to(torch.bfloat16).to(dt)
+        k, v = k.repeat_interleave(A // KH, 1), v.repeat_interleave(A // KH, 1)
+        sc = torch.einsum("thd,shd->hts", q, k) / math.sqrt(D)
+        p = torch.softmax(sc.masked_fill(mask, float("-inf")), -1)
+        h = h + torch.einsum("hts,shd->thd", p, v).reshape(T, A * D) @ _f(w["wo"], dt).T
+        u = rms(h, w["mlp_norm"])
+        g, up = u @ _f(w["wg"], dt).T, u @ _f(w["wu"], dt).T
+        h = h + (g / (1 + torch.exp(-g)) * up) @ _f(w["wd"], dt).T
+    _, W, b = model["readouts"][0]
+    y = h[-1] @ _f(W, dt).T + _f(b, dt)
+    logits = _f(model["lm_head"], dt) @ rms(y, model["final_norm"])
+    return h[-1].double(), float(torch.softmax(logits.double(), -1).max())
+
+
+def _gap(model, bf16_cache):
+    ids = list(synth.prompt(SHAPE)) + [7]
+    h64, p64 = _readout(model, ids, torch.float64, bf16_cache)
+    h32, p32 = _readout(model, ids, torch.float32, bf16_cache)
+    return float((h32 - h64).abs().max() / h64.abs().max()), abs(p32 - p64)
+
+
+def test_the_bf16_cache_amplifies_summation_order_differences(model):
+    rel_full, dp_full = _gap(model, bf16_cache=False)
+    rel_bf16, dp_bf16 = _gap(model, bf16_cache=True)
+    assert rel_full < 2e-5 and dp_full < 2e-5
+    assert rel_bf16 > 10 * rel_full
+    assert 1e-5 < rel_bf16 < 1e-2
