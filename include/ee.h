@@ -266,8 +266,8 @@ int ee_position(ee_ctx* ctx, int32_t* pos);
 #define EE_OPT_ROWS 8         /* 1: ee_prefill and ee_repass run each layer
                                  over batches of up to 64 positions (tensor-
                                  core products, each weight read once per
-                                 batch, activations carried as bf16 high and
-                                 low parts: 16 significant bits); 0 (default):
+                                 batch, each activation carried as three bf16
+                                 parts: 24 significant bits); 0 (default):
                                  one position at a time through the decode
                                  step's layer kernels (fp32 activations)    */
 int ee_set_option(ee_ctx* ctx, int option, int value);
