@@ -124,6 +124,7 @@ def _load():
             lib.orc_position.argtypes = [_P]
             lib.orc_repass.argtypes = [_P, ctypes.c_int, ctypes.c_int]
             lib.orc_set_lazy_fill.argtypes = [_P, ctypes.c_int]
+            lib.orc_set_gemm.argtypes = [_P, _P]
             lib.orc_flush_fills.argtypes = [_P]
             lib.orc_kv.argtypes = [_P, ctypes.c_int, ctypes.c_int, _P, _P, ctypes.POINTER(ctypes.c_int8)]
             lib.orc_stats.argtypes = [_P, _P]
@@ -212,6 +213,22 @@ def select_tau(conf, member, target: float = 0.9) -> float:
 
 
 # ---------------------------------------------------------------- model
+def blas_dgemm():
+    """Address of a double-precision BLAS matrix product (scipy's exported
+    Fortran-convention dgemm), or None when scipy is missing."""
+    try:
+        from scipy.linalg import cython_blas
+    except Exception:
+        return None
+    cap = cython_blas.__pyx_capi__["dgemm"]
+    api = ctypes.pythonapi
+    api.PyCapsule_GetName.restype = ctypes.c_char_p
+    api.PyCapsule_GetName.argtypes = [ctypes.py_object]
+    api.PyCapsule_GetPointer.restype = ctypes.c_void_p
+    api.PyCapsule_GetPointer.argtypes = [ctypes.py_object, ctypes.c_char_p]
+    return api.PyCapsule_GetPointer(cap, api.PyCapsule_GetName(cap))
+
+
 TRACE_FIELDS = ("h_in", "u_attn", "q", "k", "v", "o", "h_mid", "u_mlp", "gate", "up", "a", "h_out")
 
 
@@ -220,7 +237,7 @@ class Oracle:
     readouts, KV cache and position."""
 
     def __init__(self, shape, model: dict, *, readouts=True, bf16_activations: bool = False,
-                 max_ctx: int | None = None):
+                 max_ctx: int | None = None, gemm: bool = True):
         self.lib = _load()
         self.shape = shape
         L = shape.n_layers
@@ -252,6 +269,8 @@ class Oracle:
         self.ptr = self.lib.orc_create(ctypes.byref(self.cfg), ctypes.byref(w))
         if not self.ptr:
             raise ValueError("oracle: invalid configuration")
+        # long prompts: the prefill's matrix products as BLAS calls (same steps)
+        self.set_gemm(gemm)
         self.n_readouts = 0
         self.readout_layers = []
         if readouts:
@@ -297,6 +316,12 @@ class Oracle:
         Turning it off fills every pending entry."""
         if self.lib.orc_set_lazy_fill(self.ptr, int(bool(on))) != 0:
             raise ValueError("oracle: bad lazy-fill setting")
+
+    def set_gemm(self, on: bool):
+        """Prompts of 64 positions or more take their matrix products as one
+        BLAS dgemm per projection and block of positions (on, when scipy is
+        present), or run position by position (off)."""
+        self.lib.orc_set_gemm(self.ptr, blas_dgemm() if on else None)
 
     def flush_fills(self):
         """Fill every entry an exit step deferred."""

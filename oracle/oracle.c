@@ -50,6 +50,12 @@
  *   the lowest token id; prefill runs at full depth with no gate; with
  *   several readouts the shallowest passing one exits.
  *
+ * Long prompts (prefill_gemm): when the caller supplies a BLAS dgemm, the
+ * prompt runs layer by layer over blocks of positions and each matrix-vector
+ * product of a block becomes one library matrix product (double sums in the
+ * library's order); every other step is the same code in the same order.
+ * The pins compare it with the position-by-position prefill.
+ *
  * Numerics contract: weights are bf16 values held exactly; activations (the
  * residual stream, RMSNorm outputs, q, scores, softmax, attention output, FFN
  * product, readout output, logits) are float; products accumulate in double;
@@ -127,6 +133,12 @@ typedef struct {
     float nucleus_mass;
 } orc_step_result;
 
+/* A BLAS double-precision matrix product (Fortran dgemm calling convention,
+ * column-major): C = alpha op(A) op(B) + beta C. */
+typedef void (*orc_dgemm_fn)(const char* transa, const char* transb, const int* m, const int* n, const int* k,
+                             const double* alpha, const double* a, const int* lda, const double* b, const int* ldb,
+                             const double* beta, double* c, const int* ldc);
+
 /* Optional captures of one step; any pointer may be NULL. */
 typedef struct {
     float* h_readout;      /* [n_readouts][d]: residual at each evaluated readout */
@@ -154,6 +166,7 @@ typedef struct {
     int conf_kind; /* ORC_CONF_*: the signal the gate compares with tau */
     double nucleus_p; /* share of probability the nucleus holds */
     int lazy_fill;    /* 1: exit steps leave their skipped entries empty (flush_layer fills them) */
+    orc_dgemm_fn gemm; /* if set, long prompts take their products as BLAS calls (prefill_gemm) */
     int64_t steps, full_steps, exits[ORC_MAX_READOUTS];
     float *h, *u, *q, *kk, *vv, *o, *g, *up, *a, *y, *z, *logits, *tmp;
 } orc_model;
@@ -241,6 +254,7 @@ void orc_op_attention(const float* q, const float* K, const float* V, int T, int
     double mx = -INFINITY;
     for (int t = 0; t < T; ++t) {
         double acc = 0.0;
+#pragma omp simd reduction(+ : acc)
         for (int e = 0; e < D; ++e) acc += (double)q[e] * (double)K[(size_t)t * D + e];
         s[t] = acc * scale;
         if (s[t] > mx) mx = s[t];
@@ -250,11 +264,15 @@ void orc_op_attention(const float* q, const float* K, const float* V, int T, int
         s[t] = exp(s[t] - mx);
         sum += s[t];
     }
-    for (int e = 0; e < D; ++e) {
-        double acc = 0.0;
-        for (int t = 0; t < T; ++t) acc += s[t] / sum * (double)V[(size_t)t * D + e];
-        out[e] = (float)acc;
+    /* out_e = sum_t P_t V[t, e], each dimension's sum taken in position order */
+    double* acc = (double*)calloc((size_t)D, sizeof(double));
+    for (int t = 0; t < T; ++t) {
+        const double p = s[t] / sum;
+        const float* vr = V + (size_t)t * D;
+        for (int e = 0; e < D; ++e) acc[e] += p * (double)vr[e];
     }
+    for (int e = 0; e < D; ++e) out[e] = (float)acc[e];
+    free(acc);
     free(s);
 }
 
@@ -517,7 +535,9 @@ static void layer_forward(orc_model* m, int j, int t, float* h, float* tr) {
                 tr[off[4] + g * D + e] = m->vc[kv_index(m, j, g, t) + e];
             }
     }
-    /* attention of each query head over its key-value group, positions 0..t */
+    /* attention of each query head over its key-value group, positions 0..t
+     * (the heads are independent and run on separate host threads) */
+#pragma omp parallel for schedule(static)
     for (int hh = 0; hh < A; ++hh) {
         const int g = hh / group;
         orc_op_attention(m->q + (size_t)hh * D, m->kc + kv_index(m, j, g, 0), m->vc + kv_index(m, j, g, 0),
@@ -620,19 +640,215 @@ static int check_step(const orc_model* m, int32_t tok) {
     return 0;
 }
 
+int orc_set_gemm(orc_model* m, orc_dgemm_fn gemm) {
+    if (!m) return -1;
+    m->gemm = gemm;
+    return 0;
+}
+
+/* Prompts at least this long take the matrix-product form of the prefill
+ * when a BLAS product is set. */
+#define ORC_GEMM_MIN_PROMPT 64
+/* Positions per block of the matrix-product prefill. */
+#define ORC_GEMM_BLOCK 512
+
+/* out[p][i] = (float)(sum_j W[i][j] X[p][j] + b_i) for the n rows of X: the
+ * orc_op_matvec of every row of X, its double sums taken by one BLAS product
+ * (Wd: W as doubles; xb, ob: n * cols and n * rows doubles of scratch). */
+static void project_rows(orc_dgemm_fn gemm, const double* Wd, const uint16_t* b, int rows, int cols,
+                         const float* X, int n, float* out, double* xb, double* ob) {
+    for (int64_t i = 0; i < (int64_t)n * cols; ++i) xb[i] = (double)X[i];
+    /* column-major view: W is cols x rows, X is cols x n, OUT is rows x n */
+    const char tA = 'T', tB = 'N';
+    const double one = 1.0, zero = 0.0;
+    gemm(&tA, &tB, &rows, &n, &cols, &one, Wd, &cols, xb, &cols, &zero, ob, &rows);
+#pragma omp parallel for schedule(static)
+    for (int p = 0; p < n; ++p)
+        for (int i = 0; i < rows; ++i) {
+            double acc = ob[(int64_t)p * rows + i];
+            if (b) acc += (double)bf16_bits_to_f32(b[i]);
+            out[(int64_t)p * rows + i] = (float)acc;
+        }
+}
+
+/* orc_op_attention for the block of positions tb..tb+nb-1 (rotated queries
+ * in Qb, [nb][A*D]) over the cache of layer j: for each query head, the
+ * scores q.k of every position of the block against keys 0..tb+nb-1 are one
+ * BLAS product, each position then takes the softmax of its scores at
+ * positions <= t (the rest weigh 0), and the weighted sums of the values are
+ * a second product.  Scratch: kd, vd (T * D), qb (nb * D), sd (nb * T),
+ * od (nb * D) doubles, T = tb + nb. */
+static void attend_rows(orc_model* m, int j, int tb, int nb, const float* Qb, float* Ob, double* kd, double* vd,
+                        double* qb, double* sd, double* od) {
+    const orc_config* c = &m->c;
+    const int A = c->n_heads, KH = c->n_kv_heads, D = c->head_dim, group = A / KH, qdim = A * D;
+    const int T = tb + nb;
+    const double scale = 1.0 / sqrt((double)D), one = 1.0, zero = 0.0;
+    const char tT = 'T', tN = 'N';
+    for (int g = 0; g < KH; ++g) {
+        const float* Kg = m->kc + kv_index(m, j, g, 0);
+        const float* Vg = m->vc + kv_index(m, j, g, 0);
+#pragma omp parallel for schedule(static)
+        for (int64_t i = 0; i < (int64_t)T * D; ++i) {
+            kd[i] = (double)Kg[i];
+            vd[i] = (double)Vg[i];
+        }
+        for (int hh = g * group; hh < (g + 1) * group; ++hh) {
+            for (int p = 0; p < nb; ++p)
+                for (int e = 0; e < D; ++e) qb[(int64_t)p * D + e] = (double)Qb[(int64_t)p * qdim + (int64_t)hh * D + e];
+            /* column-major: S (T x nb) = K^T-view (T x D) * Q-view (D x nb) */
+            m->gemm(&tT, &tN, &T, &nb, &D, &one, kd, &D, qb, &D, &zero, sd, &T);
+#pragma omp parallel for schedule(static)
+            for (int p = 0; p < nb; ++p) {
+                double* sr = sd + (int64_t)p * T;
+                const int tp = tb + p;
+                double mx = -INFINITY;
+                for (int t = 0; t <= tp; ++t) {
+                    sr[t] *= scale;
+                    if (sr[t] > mx) mx = sr[t];
+                }
+                double sum = 0.0;
+                for (int t = 0; t <= tp; ++t) {
+                    sr[t] = exp(sr[t] - mx);
+                    sum += sr[t];
+                }
+                for (int t = 0; t <= tp; ++t) sr[t] = sr[t] / sum;
+                for (int t = tp + 1; t < T; ++t) sr[t] = 0.0;
+            }
+            /* column-major: O (D x nb) = V-view (D x T) * P-view (T x nb) */
+            m->gemm(&tN, &tN, &D, &nb, &T, &one, vd, &D, sd, &T, &zero, od, &D);
+            for (int p = 0; p < nb; ++p)
+                for (int e = 0; e < D; ++e) Ob[(int64_t)p * qdim + (int64_t)hh * D + e] = (float)od[(int64_t)p * D + e];
+        }
+    }
+}
+
+static void to_double(const uint16_t* W, int64_t n, double* out) {
+#pragma omp parallel for schedule(static)
+    for (int64_t i = 0; i < n; ++i) out[i] = (double)bf16_bits_to_f32(W[i]);
+}
+
+/* The prompt layer by layer, in blocks of positions: each step of the
+ * layer (the same steps as layer_forward, in the same order, rounded to
+ * float at the same points) runs for every position of the block, and each
+ * matrix-vector product of those positions becomes one matrix product.  At
+ * layer j a block's cache entries are stored before its attention, which
+ * reads positions <= t of layer j only: the entries of earlier blocks and of
+ * the block itself.  The products' double sums run in the library's order,
+ * so results may differ from the position-by-position prefill in the last
+ * bit of a float.  Returns 0, or -3 if memory runs out. */
+static int prefill_gemm(orc_model* m, const int32_t* ids, int n) {
+    const orc_config* c = &m->c;
+    const int d = c->d_model, L = c->n_layers, A = c->n_heads, KH = c->n_kv_heads, D = c->head_dim;
+    const int F = c->ffn_dim, t0 = m->pos;
+    const int qd = A * D, kd = KH * D, B = n < ORC_GEMM_BLOCK ? n : ORC_GEMM_BLOCK;
+    const int wide = F > qd ? (F > d ? F : d) : (qd > d ? qd : d);
+    const int64_t wq = (int64_t)qd * d, wk = (int64_t)kd * d, wo = (int64_t)d * qd, wf = (int64_t)F * d;
+    double* Wd = (double*)malloc(sizeof(double) * (size_t)(wq + 2 * wk + wo + 3 * wf));
+    double* xb = (double*)malloc(sizeof(double) * (size_t)B * wide);
+    double* ob = (double*)malloc(sizeof(double) * (size_t)B * wide);
+    float* H = (float*)malloc(sizeof(float) * (size_t)n * d);
+    float* U = (float*)malloc(sizeof(float) * (size_t)B * d);
+    float* Q = (float*)malloc(sizeof(float) * (size_t)B * qd);
+    float* Kb = (float*)malloc(sizeof(float) * (size_t)B * kd);
+    float* Vb = (float*)malloc(sizeof(float) * (size_t)B * kd);
+    float* O = (float*)malloc(sizeof(float) * (size_t)B * qd);
+    float* G = (float*)malloc(sizeof(float) * (size_t)B * F);
+    float* UP = (float*)malloc(sizeof(float) * (size_t)B * F);
+    float* T = (float*)malloc(sizeof(float) * (size_t)B * d);
+    const size_t Tmax = (size_t)t0 + n;
+    double* kdb = (double*)malloc(sizeof(double) * Tmax * D);
+    double* vdb = (double*)malloc(sizeof(double) * Tmax * D);
+    double* qb = (double*)malloc(sizeof(double) * (size_t)B * D);
+    double* sb = (double*)malloc(sizeof(double) * (size_t)B * Tmax);
+    double* odb = (double*)malloc(sizeof(double) * (size_t)B * D);
+    int rc = 0;
+    if (!Wd || !xb || !ob || !H || !U || !Q || !Kb || !Vb || !O || !G || !UP || !T || !kdb || !vdb || !qb || !sb ||
+        !odb) {
+        rc = -3;
+        goto done;
+    }
+    for (int i = 0; i < n; ++i) {
+        const uint16_t* e = m->w.embed + (size_t)ids[i] * d;
+        for (int x = 0; x < d; ++x) H[(size_t)i * d + x] = bf16_bits_to_f32(e[x]);
+    }
+    for (int j = 0; j < L; ++j) {
+        double *Wq = Wd, *Wk = Wq + wq, *Wv = Wk + wk, *Wo = Wv + wk, *Wg = Wo + wo, *Wu = Wg + wf, *Wdn = Wu + wf;
+        to_double(m->w.wq[j], wq, Wq);
+        to_double(m->w.wk[j], wk, Wk);
+        to_double(m->w.wv[j], wk, Wv);
+        to_double(m->w.wo[j], wo, Wo);
+        to_double(m->w.wg[j], wf, Wg);
+        to_double(m->w.wu[j], wf, Wu);
+        to_double(m->w.wd[j], wf, Wdn);
+        for (int p0 = 0; p0 < n; p0 += B) {
+            const int nb = n - p0 < B ? n - p0 : B;
+            float* Hb = H + (size_t)p0 * d;
+            /* attention input, q, k, v; RoPE; the block's cache entries */
+#pragma omp parallel for schedule(static)
+            for (int p = 0; p < nb; ++p) {
+                orc_op_rmsnorm(Hb + (size_t)p * d, m->w.attn_norm[j], d, c->rms_eps, U + (size_t)p * d);
+                for (int i = 0; i < d; ++i) U[(size_t)p * d + i] = act_round(m, U[(size_t)p * d + i]);
+            }
+            project_rows(m->gemm, Wq, c->qkv_bias ? m->w.bq[j] : NULL, qd, d, U, nb, Q, xb, ob);
+            project_rows(m->gemm, Wk, c->qkv_bias ? m->w.bk[j] : NULL, kd, d, U, nb, Kb, xb, ob);
+            project_rows(m->gemm, Wv, c->qkv_bias ? m->w.bv[j] : NULL, kd, d, U, nb, Vb, xb, ob);
+#pragma omp parallel for schedule(static)
+            for (int p = 0; p < nb; ++p) {
+                const int t = t0 + p0 + p;
+                for (int hh = 0; hh < A; ++hh) orc_op_rope(Q + (size_t)p * qd + (size_t)hh * D, D, t, c->rope_base);
+                for (int g = 0; g < KH; ++g) orc_op_rope(Kb + (size_t)p * kd + (size_t)g * D, D, t, c->rope_base);
+                store_kv(m, j, t, Kb + (size_t)p * kd, Vb + (size_t)p * kd, 1);
+            }
+            /* attention of every position and head over positions 0..t */
+            attend_rows(m, j, t0 + p0, nb, Q, O, kdb, vdb, qb, sb, odb);
+            for (int64_t i = 0; i < (int64_t)nb * qd; ++i) O[i] = act_round(m, O[i]);
+            /* output projection and residual add */
+            project_rows(m->gemm, Wo, NULL, d, qd, O, nb, T, xb, ob);
+            for (int64_t i = 0; i < (int64_t)nb * d; ++i) Hb[i] = Hb[i] + T[i];
+            /* gated feed-forward and residual add */
+#pragma omp parallel for schedule(static)
+            for (int p = 0; p < nb; ++p) {
+                orc_op_rmsnorm(Hb + (size_t)p * d, m->w.mlp_norm[j], d, c->rms_eps, U + (size_t)p * d);
+                for (int i = 0; i < d; ++i) U[(size_t)p * d + i] = act_round(m, U[(size_t)p * d + i]);
+            }
+            project_rows(m->gemm, Wg, NULL, F, d, U, nb, G, xb, ob);
+            project_rows(m->gemm, Wu, NULL, F, d, U, nb, UP, xb, ob);
+#pragma omp parallel for schedule(static)
+            for (int64_t i = 0; i < (int64_t)nb * F; ++i)
+                G[i] = act_round(m, (float)(orc_op_silu(G[i]) * (double)UP[i]));
+            project_rows(m->gemm, Wdn, NULL, d, F, G, nb, T, xb, ob);
+            for (int64_t i = 0; i < (int64_t)nb * d; ++i) Hb[i] = Hb[i] + T[i];
+        }
+    }
+    memcpy(m->h, H + (size_t)(n - 1) * d, sizeof(float) * d);
+    m->pos += n;
+done:
+    free(Wd); free(xb); free(ob); free(H); free(U); free(Q); free(Kb); free(Vb); free(O); free(G); free(UP);
+    free(T); free(kdb); free(vdb); free(qb); free(sb); free(odb);
+    return rc;
+}
+
 /* Prefill: every prompt position runs the full depth, no gate; returns the
- * full model's greedy token after the last position. */
+ * full model's greedy token after the last position.  With a BLAS product
+ * set (orc_set_gemm), prompts of ORC_GEMM_MIN_PROMPT positions or more take
+ * the matrix-product form (prefill_gemm). */
 int orc_prefill(orc_model* m, const int32_t* ids, int n, int32_t* first_token, orc_capture* cap) {
     if (!m || n <= 0 || m->pos + n > m->c.max_ctx) return -2;
     for (int i = 0; i < n; ++i)
         if (ids[i] < 0 || ids[i] >= m->c.vocab) return -1;
     const int d = m->c.d_model, L = m->c.n_layers;
-    for (int i = 0; i < n; ++i) {
-        const int t = m->pos;
-        const uint16_t* e = m->w.embed + (size_t)ids[i] * d;
-        for (int x = 0; x < d; ++x) m->h[x] = bf16_bits_to_f32(e[x]);
-        for (int j = 0; j < L; ++j) layer_forward(m, j, t, m->h, NULL);
-        m->pos++;
+    if (m->gemm && n >= ORC_GEMM_MIN_PROMPT) {
+        const int rc = prefill_gemm(m, ids, n);
+        if (rc) return rc;
+    } else {
+        for (int i = 0; i < n; ++i) {
+            const int t = m->pos;
+            const uint16_t* e = m->w.embed + (size_t)ids[i] * d;
+            for (int x = 0; x < d; ++x) m->h[x] = bf16_bits_to_f32(e[x]);
+            for (int j = 0; j < L; ++j) layer_forward(m, j, t, m->h, NULL);
+            m->pos++;
+        }
     }
     unembed(m, m->h, m->logits);
     orc_conf cf;

@@ -452,6 +452,53 @@ def test_prefill_equals_forced_full_decode():
             assert np.array_equal(ka, kb) and np.array_equal(va, vb)
 
 
+def _prefill_both_ways(shape, model, parts):
+    """Prefill the prompt pieces `parts` (consecutive id arrays) with the
+    prefill's matrix products as BLAS calls and position by position."""
+    out = []
+    n = sum(len(p) for p in parts)
+    for gemm in (True, False):
+        o = oracle.Oracle(shape, model, max_ctx=n + 2, gemm=gemm)
+        toks = [o.prefill(p, capture=True) for p in parts]
+        out.append((o, toks))
+    return out
+
+
+@pytest.mark.parametrize("kw,lens", [({}, (100,)), ({"qkv_bias": True}, (7, 600)), ({"n_kv_heads": 1}, (64, 65))])
+def test_prefill_matrix_product_form_matches_position_by_position(kw, lens):
+    """Long prompts run layer by layer with each projection of a block of
+    positions as one BLAS product, and each head's scores and weighted values
+    as two more (the block attending to the cache of its layer).  Same steps,
+    same float roundings: the cache, the final residual and the logits agree
+    with the position-by-position prefill (the products' double sums may
+    round differently in the last bit of a float, so a few cache values may
+    sit one bf16 step apart).  Covers two blocks of 512 positions, a start
+    past position 0 and a prompt that stays position by position (7)."""
+    shape = micro(prompt_len=sum(lens), **kw)
+    model = synth.make_model(shape)
+    ids = synth.prompt(shape, sum(lens))
+    parts, at = [], 0
+    for n in lens:
+        parts.append(ids[at:at + n])
+        at += n
+    (a, ta), (b, tb) = _prefill_both_ways(shape, model, parts)
+    for (xa, ca), (xb, cb) in zip(ta, tb):
+        assert xa == xb
+        np.testing.assert_allclose(ca["h_final"], cb["h_final"], rtol=1e-5, atol=1e-6)
+        np.testing.assert_allclose(ca["final_logits"], cb["final_logits"], rtol=1e-5, atol=1e-5)
+    n_diff = n_all = 0
+    for j in range(shape.n_layers):
+        for t in range(len(ids)):
+            ka, va, sa = a.kv(j, t)
+            kb, vb, sb = b.kv(j, t)
+            assert sa == sb == 1
+            for u, v in ((ka, kb), (va, vb)):
+                n_diff += int(np.sum(u != v))
+                n_all += u.size
+                np.testing.assert_allclose(u, v, rtol=2.0 ** -7, atol=1e-6)
+    assert n_diff <= n_all // 1000
+
+
 def test_qkv_bias_and_tied_head_options():
     shape = micro(qkv_bias=True, tied_embedding=True)
     model = synth.make_model(shape)
