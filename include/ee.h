@@ -270,6 +270,16 @@ int ee_position(ee_ctx* ctx, int32_t* pos);
                                  parts: 24 significant bits); 0 (default):
                                  one position at a time through the decode
                                  step's layer kernels (fp32 activations)    */
+#define EE_OPT_WAIT_LIMIT 9    /* for testing the failure path: the bound, in SM
+                                 clock cycles, on each wait of the persistent
+                                 layer kernel (ring stages, values from other
+                                 CTAs); 0 (default): about 2 s.  A wait that
+                                 runs out sets the device error word, the
+                                 launch ends without waiting further (copies
+                                 in flight still land first) and the call
+                                 returns EE_EDEVICE; ee_reset clears it.  A
+                                 few thousand cycles make ordinary waits run
+                                 out.                                        */
 int ee_set_option(ee_ctx* ctx, int option, int value);
 
 #define EE_DBG_HIDDEN_READOUT 1 /* layer = readout r: residual h_k it read, d floats   */
@@ -335,8 +345,10 @@ int ee_attention_decode(const float* q, const uint16_t* k_pages, const uint16_t*
  *   each call clears the part that must start at zero.  Calls whose work
  *   overlaps on the GPU (other streams, other threads) race on the area:
  *   order them on one stream.
- *   The first call on each device looks up the area's device address (with
- *   that device current); make that first call before any stream capture.
+ *   Every call looks up the area's device address on the current device
+ *   (so an address never outlives a cudaDeviceReset); the first call on a
+ *   device also loads the library's device code there, so make that first
+ *   call before any stream capture.
  *   No cudaMalloc, cudaFree or other allocating call is made. */
 #define EE_STATIC_ATTN_SCRATCH_BYTES (2u << 20)
 int ee_attention_decode_static(const float* q, const uint16_t* k_pages, const uint16_t* v_pages,

@@ -122,6 +122,7 @@ def _load():
             lib.orc_decode_step.argtypes = [_P, ctypes.c_int32, _P, ctypes.c_int, ctypes.POINTER(StepResult),
                                             ctypes.POINTER(Capture)]
             lib.orc_position.argtypes = [_P]
+            lib.orc_truncate.argtypes = [_P, ctypes.c_int]
             lib.orc_repass.argtypes = [_P, ctypes.c_int, ctypes.c_int]
             lib.orc_set_lazy_fill.argtypes = [_P, ctypes.c_int]
             lib.orc_set_gemm.argtypes = [_P, _P]
@@ -330,6 +331,12 @@ class Oracle:
     @property
     def pos(self) -> int:
         return self.lib.orc_position(self.ptr)
+
+    def truncate(self, pos: int):
+        """Forget positions >= pos (cache entries, exit records, step counts):
+        decoding continues from pos as if they had never been decoded."""
+        if self.lib.orc_truncate(self.ptr, int(pos)) != 0:
+            raise ValueError("oracle: bad truncate position")
 
     def repass(self, t0: int, t1: int) -> int:
         """Section 11's full-depth re-pass over positions [t0, t1): every

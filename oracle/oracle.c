@@ -940,6 +940,30 @@ int orc_decode_step(orc_model* m, int32_t in_tok, const float* taus, int force, 
 
 int orc_position(const orc_model* m) { return m->pos; }
 
+/* Forget the positions from pos on, so that decoding continues from there
+ * as if they had never been decoded: their cache entries, exit records and
+ * residuals are cleared, the position moves back to pos and the step counts
+ * restart.  Positions below pos are untouched.  -1 unless 0 <= pos <= the
+ * current position. */
+int orc_truncate(orc_model* m, int pos) {
+    if (!m || pos < 0 || pos > m->pos) return -1;
+    const orc_config* c = &m->c;
+    const int n = c->max_ctx - pos;
+    for (int j = 0; j < c->n_layers; ++j) {
+        memset(m->kv_src + (size_t)j * c->max_ctx + pos, 0, (size_t)n);
+        for (int g = 0; g < c->n_kv_heads; ++g) {
+            memset(m->kc + kv_index(m, j, g, pos), 0, sizeof(float) * (size_t)n * c->head_dim);
+            memset(m->vc + kv_index(m, j, g, pos), 0, sizeof(float) * (size_t)n * c->head_dim);
+        }
+    }
+    memset(m->exit_at + pos, 0, sizeof(int16_t) * (size_t)n);
+    memset(m->h_exit + (size_t)pos * c->d_model, 0, sizeof(float) * (size_t)n * c->d_model);
+    m->pos = pos;
+    m->steps = m->full_steps = 0;
+    memset(m->exits, 0, sizeof(m->exits));
+    return 0;
+}
+
 /* Section 11's full-depth re-pass: for each position t in [t0, t1), in
  * order, whose upper layers still hold filled (or deferred) entries (it
  * exited after layer k and kv_src[k][t] is not 1), run layers k+1..L from the

@@ -13,7 +13,7 @@ import numpy as np
 from . import _lib
 from ._lib import (CONF_MARGIN, CONF_NEGENT, CONF_PMAX, DEVICE, FORCE_FULL, FREE, HOST, MAX_READOUTS,
                    OPT_CONFIDENCE, OPT_DEBUG_LOGITS, OPT_GRAPHS, OPT_NUCLEUS, OPT_PDL, OPT_PERSISTENT, OPT_REPASS,
-                   OPT_ROWS,
+                   OPT_ROWS, OPT_WAIT_LIMIT,
                    EEError, FORCE_EXIT_AT, check)
 
 __all__ = ["Engine", "EEError", "FREE", "FORCE_FULL", "FORCE_EXIT_AT", "HOST", "DEVICE", "attention_decode",

@@ -12,6 +12,7 @@ FREE, FORCE_FULL = 0, 1
 HOST, DEVICE = 0, 1
 OPT_GRAPHS, OPT_PDL, OPT_DEBUG_LOGITS, OPT_PERSISTENT, OPT_CONFIDENCE, OPT_NUCLEUS, OPT_REPASS = 1, 2, 3, 4, 5, 6, 7
 OPT_ROWS = 8
+OPT_WAIT_LIMIT = 9
 CONF_PMAX, CONF_MARGIN, CONF_NEGENT = 0, 1, 2
 DBG_HIDDEN_READOUT, DBG_READOUT_Y, DBG_HIDDEN_FINAL, DBG_READOUT_LOGITS, DBG_FINAL_LOGITS, DBG_KV, DBG_KV_SRC = \
     1, 2, 3, 4, 5, 6, 7

@@ -155,13 +155,13 @@ Layout make_layout(const ee_model_config& c) {
     // persistent layer kernel: down-projection partials, mid residual, counters
     {
         const int64_t cols = kSegChunk / (2 * kTileRows);  // columns per ring chunk
-        l.seg_dpart = take(4 * (size_t)tile_count(d) * ((F + cols - 1) / cols) * kTileRows);
-        l.seg_opart = take(2 * 4 * (size_t)tile_count(d) * ((A * D + cols - 1) / cols) * kTileRows);
+        l.seg_dpart = take(sizeof(Tagged) * (size_t)tile_count(d) * ((F + cols - 1) / cols) * kTileRows);
+        l.seg_opart = take(2 * sizeof(Tagged) * (size_t)tile_count(d) * ((A * D + cols - 1) / cols) * kTileRows);
     }
-    l.seg_q = take(4 * (size_t)A * D);
-    l.seg_kvn = take(4 * 2 * (size_t)KH * D);
-    l.seg_a = take(4 * (size_t)F);
-    l.seg_attn = take(4 * (size_t)A * kSegMaxSplits * (D + 4));
+    l.seg_q = take(sizeof(Tagged) * (size_t)A * D);
+    l.seg_kvn = take(sizeof(Tagged) * 2 * (size_t)KH * D);
+    l.seg_a = take(sizeof(Tagged) * (size_t)F);
+    l.seg_attn = take(sizeof(Tagged) * (size_t)A * kSegMaxSplits * (D + 4));
     l.seg_sync = take(4 * 8);
     l.seg_end = b;
     // multi-position layer pass (prompt and re-pass batches)
@@ -855,13 +855,15 @@ int ee_create(const ee_model_config* cfg, void* d_workspace, size_t workspace_by
     c->attn_cluster = attention_cluster_size(m.D, m.KH);
     if (seg_plan(m, c->n_sm, c->seg) && configure_layers(c->seg.smem) == cudaSuccess &&
         layers_blocks_per_sm(c->seg.smem) >= 1) {
-        c->seg.dpart = (float*)(w + l.seg_dpart);
-        c->seg.opart = (float*)(w + l.seg_opart);
-        c->seg.attn_part = (float*)(w + l.seg_attn);
-        c->seg.q = (float*)(w + l.seg_q);
-        c->seg.kvn = (float*)(w + l.seg_kvn);
-        c->seg.a = (float*)(w + l.seg_a);
+        c->seg.dpart = (Tagged*)(w + l.seg_dpart);
+        c->seg.opart = (Tagged*)(w + l.seg_opart);
+        c->seg.attn_part = (Tagged*)(w + l.seg_attn);
+        c->seg.q = (Tagged*)(w + l.seg_q);
+        c->seg.kvn = (Tagged*)(w + l.seg_kvn);
+        c->seg.a = (Tagged*)(w + l.seg_a);
         c->seg.sync = (unsigned*)(w + l.seg_sync);
+        c->seg.stall_cycles = kSegStallCycles;
+        c->seg.check_cycles = kSegCheckCycles;
         c->seg_ok = true;
     }
     if (vocab_ring_plan(m.d, c->n_sm, c->vring) && configure_vocab_ring(c->vring.smem) == cudaSuccess)
@@ -1062,6 +1064,12 @@ int ee_set_option(ee_ctx* c, int option, int value) {
             return EE_OK;
         case EE_OPT_ROWS:
             c->use_rows = value != 0;
+            return EE_OK;
+        case EE_OPT_WAIT_LIMIT:
+            if (value < 0) return fail(EE_EINVAL, "wait limit must be >= 0");
+            drop_graphs(c);
+            c->seg.stall_cycles = value ? (long long)value : kSegStallCycles;
+            c->seg.check_cycles = value ? std::max(1LL, (long long)value / 4) : kSegCheckCycles;
             return EE_OK;
         case EE_OPT_PERSISTENT:
             if (value && !c->seg_ok) return fail(EE_EINVAL, "the persistent layer kernel does not support this shape");

@@ -189,6 +189,15 @@ constexpr int kSegChunk = 32768;   // bytes per ring stage: 32 rows x 512 bf16 c
 constexpr int kSegMaxSplits = 32;  // attention splits per kv head (at most)
 constexpr int kSegMaxGroup = 8;    // query heads per kv head (at most)
 constexpr int kSegMaxSlots = 8;    // CTAs sharing one down tile, chunks of one O tile (at most)
+// A value handed from one CTA to another inside a launch of the persistent
+// layer kernel: the float's bits in the low word and its layer's tag in the
+// high word, stored and loaded as one 64-bit word (observed whole).
+using Tagged = unsigned long long;
+// Bounds of the persistent kernel's waits, in SM clock cycles: a wait gives
+// up after `stall` cycles; a waiting thread looks at the error word once
+// every `check` cycles.
+constexpr long long kSegStallCycles = 4000000000ll;  // about 2 s
+constexpr long long kSegCheckCycles = 2000000ll;     // about 1 ms
 struct SegPlan {
     int G;                  // CTAs (one per SM)
     int stages;             // ring stages
@@ -197,16 +206,17 @@ struct SegPlan {
     int rows_per_kv_chunk;  // cache positions per ring chunk
     int max_items;          // O / down-projection items per CTA (at most)
     int n_tiles[4], n_chunks[4], K[4];  // Q/K/V, O, gate/up, down
-    // Values handed between CTAs, each float carrying its layer's tag in
-    // the low mantissa bits (zero after ee_reset):
-    float* dpart;           // down-projection partials [tile][n_chunks][32]
-    float* opart;           // O-projection chunk partials [2][tile][n_chunks][32] (by the layer count's parity)
-    float* attn_part;       // [A][kSegMaxSplits][D + 4]: unnormalised o, max, sum per split
-    float* q;               // [A D] rotated queries
-    float* kvn;             // [2][KH D] the step's k and v (bf16 values)
-    float* a;               // [F] SwiGLU product
+    // Values handed between CTAs, each a Tagged word (zero after ee_reset):
+    Tagged* dpart;          // down-projection partials [tile][n_chunks][32]
+    Tagged* opart;          // O-projection chunk partials [2][tile][n_chunks][32] (by the layer count's parity)
+    Tagged* attn_part;      // [A][kSegMaxSplits][D + 4]: unnormalised o, max, sum per split
+    Tagged* q;              // [A D] rotated queries
+    Tagged* kvn;            // [2][KH D] the step's k and v (bf16 values)
+    Tagged* a;              // [F] SwiGLU product
     unsigned* sync;         // [0] exit ticket (zero between launches), [1] layers run since ee_reset
     size_t smem;            // dynamic shared memory per CTA
+    long long stall_cycles; // wait bounds (kSegStallCycles, kSegCheckCycles unless a test lowers them)
+    long long check_cycles;
 };
 // Geometry and shared-memory plan for `m` on n_sm SMs (pointers left
 // unset); false if the shape is outside what the kernel supports.

@@ -12,7 +12,6 @@
 // library holds EE_STATIC_ATTN_SCRATCH_BYTES for it until the process exits.
 #include <cuda_runtime.h>
 
-#include <mutex>
 #include <string>
 
 #include "ee.h"
@@ -27,28 +26,20 @@ constexpr size_t kAlign = 256;
 // symbol: its device address comes from cudaGetSymbolAddress.
 static __device__ __align__(256) unsigned char g_attn_scratch[kStaticBytes];
 
-constexpr int kMaxDevices = 64;
-std::mutex g_mu;
-void* g_addr[kMaxDevices] = {};
-
 size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
-// Device address of the scratch area on the current device, looked up once
-// per device (the first call on a device does this).
+// Device address of the scratch area on the current device.  It is looked
+// up on every call: once the library's device code is loaded on a device the
+// lookup is a host-side table read, and an address kept from an earlier call
+// would go stale if the caller reset the device (cudaDeviceReset), after
+// which the code, and the area with it, may load at another address.  The
+// first call on a device loads the code there.
 int scratch_address(void** out) {
-    int dev = -1;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) return ee::set_last_error(EE_ECUDA, "no current CUDA device");
-    if (dev < 0 || dev >= kMaxDevices) return ee::set_last_error(EE_EINVAL, "device index beyond the supported range");
-    std::lock_guard<std::mutex> lock(g_mu);
-    if (!g_addr[dev]) {
-        void* p = nullptr;
-        e = cudaGetSymbolAddress(&p, g_attn_scratch);
-        if (e != cudaSuccess || !p)
-            return ee::set_last_error(EE_ECUDA, (std::string("cudaGetSymbolAddress: ") + cudaGetErrorString(e)).c_str());
-        g_addr[dev] = p;
-    }
-    *out = g_addr[dev];
+    void* p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_attn_scratch);
+    if (e != cudaSuccess || !p)
+        return ee::set_last_error(EE_ECUDA, (std::string("cudaGetSymbolAddress: ") + cudaGetErrorString(e)).c_str());
+    *out = p;
     return EE_OK;
 }
 

@@ -53,11 +53,9 @@ constexpr int kCW = kSegConsumerWarps;
 constexpr int kCT = 32 * kCW;              // consumer threads
 constexpr int kColsPerChunk = kSegChunk / (2 * kTileRows);  // 512
 constexpr int kCCPerWarp = (kColsPerChunk / 8 + kCW - 1) / kCW;  // 16-byte column chunks a warp takes per stage
-// Wait bounds in SM clock cycles (clock64 is cheap to read; the global
-// timer and the error word in global memory are not, so a waiting thread
-// looks at them only about once per millisecond).
-constexpr long long kStallCycles = 4000000000ll;  // about 2 s
-constexpr long long kCheckCycles = 2000000ll;     // about 1 ms
+// Wait bounds are in SM clock cycles (kSegStallCycles, kSegCheckCycles;
+// clock64 is cheap to read, the error word in global memory is not, so a
+// waiting thread looks at it only once per check interval).
 
 
 __device__ __forceinline__ float bf(uint16_t b) { return __uint_as_float((uint32_t)b << 16); }
@@ -66,16 +64,21 @@ __device__ __forceinline__ float bfhi(uint32_t v) { return __uint_as_float(v & 0
 __device__ __forceinline__ uint16_t tobf(float f) { return __bfloat16_as_ushort(__float2bfloat16_rn(f)); }
 
 __device__ __forceinline__ long long cycles() { return clock64(); }
+// The error word a wait watches and its bounds (cycles).
+struct Waits {
+    volatile int* err;
+    long long stall, check;
+};
 // Bookkeeping of a bounded wait: true once the wait has run out of time or
 // another thread has flagged a stall.
 struct Bound {
     long long t0, tc;
     __device__ __forceinline__ Bound() : t0(cycles()), tc(t0) {}
-    __device__ __forceinline__ bool expired(const volatile int* err) {
+    __device__ __forceinline__ bool expired(const Waits& w) {
         const long long t = cycles();
-        if (t - tc < kCheckCycles) return false;
+        if (t - tc < w.check) return false;
         tc = t;
-        return (*err & kErrStall) || t - t0 > kStallCycles;
+        return (*w.err & kErrStall) || t - t0 > w.stall;
     }
 };
 __device__ __forceinline__ uint32_t saddr(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
@@ -95,12 +98,19 @@ __device__ __forceinline__ bool mb_test(uint64_t* b, int parity) {
 }
 // Wait for the phase of parity `parity` to complete; false after the time
 // limit or once another thread has flagged a stall.
-__device__ __forceinline__ bool mb_wait(uint64_t* b, int parity, const volatile int* err) {
+__device__ __forceinline__ bool mb_wait(uint64_t* b, int parity, const Waits& w) {
     if (mb_test(b, parity)) return true;
     Bound bd;
     for (unsigned it = 1;; ++it) {
         if (mb_test(b, parity)) return true;
-        if ((it & 15) == 0 && bd.expired(err)) return false;
+        if ((it & 15) == 0 && bd.expired(w)) return false;
+    }
+}
+// Wait for a bulk copy issued earlier to land, whatever the error word says
+// (a CTA must not exit with copies into its shared memory in flight; issued
+// copies always land), bounded by `deadline` on the SM clock.
+__device__ __forceinline__ void mb_wait_landed(uint64_t* b, int parity, long long deadline) {
+    while (!mb_test(b, parity) && cycles() < deadline) {
     }
 }
 // Non-blocking test with a sleeping back-off, for the producer: it waits
@@ -115,13 +125,13 @@ __device__ __forceinline__ bool mb_probe(uint64_t* b, int parity) {
         : "memory");
     return ok != 0;
 }
-__device__ __forceinline__ bool mb_wait_sleep(uint64_t* b, int parity, const volatile int* err) {
+__device__ __forceinline__ bool mb_wait_sleep(uint64_t* b, int parity, const Waits& w) {
     if (mb_probe(b, parity)) return true;
     Bound bd;
     for (unsigned it = 1;; ++it) {
         __nanosleep(32);
         if (mb_probe(b, parity)) return true;
-        if ((it & 15) == 0 && bd.expired(err)) return false;
+        if ((it & 15) == 0 && bd.expired(w)) return false;
     }
 }
 __device__ __forceinline__ void mb_arrive(uint64_t* b) {
@@ -179,11 +189,16 @@ __device__ __forceinline__ void sts64(uint32_t a, uint32_t x, uint32_t y) {
 __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
     return (uint32_t)tobf(a) | ((uint32_t)tobf(b) << 16);
 }
-// x0, x1 as packed bf16 high parts and packed bf16 low parts (x - high).
-__device__ __forceinline__ void split_bf16x2(float x0, float x1, uint32_t& hi, uint32_t& lo) {
+// x0, x1 as three packed bf16 parts: high = bf16(x), middle = bf16(x -
+// high), low = bf16(x - high - middle).  Both differences are exact in fp32
+// and the low part holds what is left, so high + middle + low = x.
+__device__ __forceinline__ void split3_bf16x2(float x0, float x1, uint32_t& hi, uint32_t& mid, uint32_t& lo) {
     const uint16_t h0 = tobf(x0), h1 = tobf(x1);
+    const float r0 = x0 - bf(h0), r1 = x1 - bf(h1);
+    const uint16_t m0 = tobf(r0), m1 = tobf(r1);
     hi = (uint32_t)h0 | ((uint32_t)h1 << 16);
-    lo = pack_bf16x2(x0 - bf(h0), x1 - bf(h1));
+    mid = (uint32_t)m0 | ((uint32_t)m1 << 16);
+    lo = pack_bf16x2(r0 - bf(m0), r1 - bf(m1));
 }
 // d += A B for one m16n8k16 tile: bf16 A (4 registers, row-major
 // fragment), bf16 B (2 registers, column-major fragment), fp32 accumulators.
@@ -395,25 +410,25 @@ struct Producer {
     RingPos head;  // stage of the next chunk
     RingPos tail;  // stage of chunk n - inflight (once n >= inflight)
     uint64_t pol_w, pol_kv;
-    volatile int* err;
+    Waits wt;
     bool ok = true;
-    __device__ Producer(const Smem& sm, int st, int infl, volatile int* e)
-        : s(sm), stages(st), inflight(infl), n(0), pol_w(evict_first()), pol_kv(evict_normal()), err(e) {}
+    __device__ Producer(const Smem& sm, int st, int infl, const Waits& w)
+        : s(sm), stages(st), inflight(infl), n(0), pol_w(evict_first()), pol_kv(evict_normal()), wt(w) {}
     __device__ __forceinline__ void push(const void* src, uint32_t bytes, uint64_t pol) {
         if (!ok) return;
         // at most `inflight` copies outstanding: the ring still runs up to
         // `stages` chunks ahead, but the copies queued in HBM stay few
         if (n >= inflight) {
-            if (!mb_wait_sleep(&s.full[tail.st], tail.ph, err)) {
-                atomicOr((int*)err, kErrStall);
+            if (!mb_wait_sleep(&s.full[tail.st], tail.ph, wt)) {
+                atomicOr((int*)wt.err, kErrStall);
                 ok = false;
                 return;
             }
             tail.next(stages);
         }
         // the stage is free once the consumers released its previous chunk
-        if (n >= stages && !mb_wait_sleep(&s.empty[head.st], head.ph ^ 1, err)) {
-            atomicOr((int*)err, kErrStall);
+        if (n >= stages && !mb_wait_sleep(&s.empty[head.st], head.ph ^ 1, wt)) {
+            atomicOr((int*)wt.err, kErrStall);
             ok = false;
             return;
         }
@@ -424,15 +439,17 @@ struct Producer {
     }
     // Before leaving: every issued copy has landed (the consumers normally
     // see to that; after a stall they may not have).  Walks back over the
-    // last min(n, stages) chunks.
+    // last min(n, stages) chunks, whose copies are the only ones that can
+    // still be in flight (chunk n lands before chunk n + stages is issued).
     __device__ void drain() {
         RingPos q = head;
+        const long long deadline = cycles() + kSegStallCycles;
         for (long long i = 0; i < min(n, (long long)stages); ++i) {
             if (--q.st < 0) {
                 q.st = stages - 1;
                 q.ph ^= 1;
             }
-            mb_wait(&s.full[q.st], q.ph, err);
+            mb_wait_landed(&s.full[q.st], q.ph, deadline);
         }
     }
 };
@@ -442,12 +459,12 @@ struct Consumer {
     const Smem& s;
     int stages;
     RingPos pos;
-    volatile int* err;
+    Waits wt;
     bool ok = true;
-    __device__ Consumer(const Smem& sm, int st, volatile int* e) : s(sm), stages(st), err(e) {}
+    __device__ Consumer(const Smem& sm, int st, const Waits& w) : s(sm), stages(st), wt(w) {}
     __device__ __forceinline__ const uint4* acquire() {
-        if (ok && !mb_wait(&s.full[pos.st], pos.ph, err)) {
-            atomicOr((int*)err, kErrStall);
+        if (ok && !mb_wait(&s.full[pos.st], pos.ph, wt)) {
+            atomicOr((int*)wt.err, kErrStall);
             ok = false;
         }
         return reinterpret_cast<const uint4*>(s.ring + (size_t)pos.st * kSegChunk);
@@ -460,61 +477,66 @@ struct Consumer {
 };
 
 // ------------------------------------------------------------ tagged values
-// A value one CTA hands to another within a launch carries a tag in its 5
-// lowest mantissa bits: 16 | (seq mod 16), seq counting the layers run
-// since the context was reset (over all launches).  Readers load it with
-// strong loads until the tag is the expected one, so a phase needs no
-// completion counter and its writers no fence: a 32-bit word is observed
-// whole.  The value is first rounded to 19 significant bits (a bf16 value
-// stays exact).  Every word a layer reads is written by every layer (the O
-// slots by every other layer, into the buffer of seq's parity), so before
-// it receives the value of seq it holds the one of seq - 1 or seq - 2, whose
-// tags differ; attention partials of splits a launch does not use are set
-// to 0, which equals no tag, as is every word after a reset.  The readers
-// of a word are done with it before it is written again: every later write
-// depends, through the values it is computed from, on all of them.
-__device__ __forceinline__ uint32_t seq_tag(unsigned seq) { return 16u | (seq & 15u); }
-__device__ __forceinline__ void st_tagged(float* p, float v, uint32_t tag) {
-    const uint32_t b = ((__float_as_uint(v) + 16u) & ~31u) | tag;
-    asm volatile("st.relaxed.gpu.global.b32 [%0], %1;" ::"l"(p), "r"(b) : "memory");
+// A value one CTA hands to another within a launch is a Tagged word: the
+// float's bits in the low half, its layer's tag in the high half, 0x80000000
+// | (seq mod 2^31), seq counting the layers run since the context was reset
+// (over all launches).  Writers store the word with one 64-bit relaxed store
+// and neither fence nor count; readers load it with 64-bit relaxed loads
+// until the tag is the expected one.  A 64-bit aligned word is observed
+// whole, so value and tag arrive together, and the value keeps all 32 bits
+// (a NaN or an infinity too).  Every word a layer reads is written by every
+// layer (the O slots by every other layer, into the buffer of seq's parity),
+// so before it receives the value of seq it holds the one of seq - 1 or
+// seq - 2, whose tags differ; attention partials of splits a launch does not
+// use are set to 0, which is no tag, as is every word after a reset.  The
+// readers of a word are done with it before it is written again: every later
+// write depends, through the values it is computed from, on all of them.
+__device__ __forceinline__ uint32_t seq_tag(unsigned seq) { return 0x80000000u | (seq & 0x7fffffffu); }
+__device__ __forceinline__ void st_tagged(Tagged* p, float v, uint32_t tag) {
+    const unsigned long long b = (unsigned long long)__float_as_uint(v) | ((unsigned long long)tag << 32);
+    asm volatile("st.relaxed.gpu.global.b64 [%0], %1;" ::"l"(p), "l"(b) : "memory");
 }
-__device__ __forceinline__ uint32_t ld_strong(const float* p) {
-    uint32_t r;
-    asm volatile("ld.relaxed.gpu.global.b32 %0, [%1];" : "=r"(r) : "l"(p) : "memory");
+__device__ __forceinline__ void st_zero(Tagged* p) {
+    asm volatile("st.relaxed.gpu.global.b64 [%0], %1;" ::"l"(p), "l"(0ull) : "memory");
+}
+__device__ __forceinline__ unsigned long long ld_strong(const Tagged* p) {
+    unsigned long long r;
+    asm volatile("ld.relaxed.gpu.global.b64 %0, [%1];" : "=l"(r) : "l"(p) : "memory");
     return r;
 }
-__device__ __forceinline__ uint4 ld_strong4(const float* p) {
-    uint4 r;
-    asm volatile("ld.relaxed.gpu.global.v4.b32 {%0, %1, %2, %3}, [%4];"
-                 : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
-                 : "l"(p)
-                 : "memory");
-    return r;
+// Two consecutive words (p 16-byte aligned): each 64-bit element is observed whole.
+__device__ __forceinline__ void ld_strong2(const Tagged* p, unsigned long long& a, unsigned long long& b) {
+    asm volatile("ld.relaxed.gpu.global.v2.b64 {%0, %1}, [%2];" : "=l"(a), "=l"(b) : "l"(p) : "memory");
 }
-__device__ __forceinline__ float untag(uint32_t b) { return __uint_as_float(b & ~31u); }
-__device__ __forceinline__ float4 untag4(uint4 v) { return make_float4(untag(v.x), untag(v.y), untag(v.z), untag(v.w)); }
-// Nonzero if any of the four tags differs from `tag`.
-__device__ __forceinline__ uint32_t mismatch4(uint4 v, uint32_t tag) {
-    return ((v.x ^ tag) | (v.y ^ tag) | (v.z ^ tag) | (v.w ^ tag)) & 31u;
+__device__ __forceinline__ float untag(unsigned long long b) { return __uint_as_float((uint32_t)b); }
+__device__ __forceinline__ uint32_t tag_of(unsigned long long b) { return (uint32_t)(b >> 32); }
+// Four consecutive words (p 16-byte aligned) as a float4; a tag other than
+// `tag` sets bits in bad.
+__device__ __forceinline__ float4 load4(const Tagged* p, uint32_t tag, uint32_t& bad) {
+    unsigned long long w0, w1, w2, w3;
+    ld_strong2(p, w0, w1);
+    ld_strong2(p + 2, w2, w3);
+    bad |= (tag_of(w0) ^ tag) | (tag_of(w1) ^ tag) | (tag_of(w2) ^ tag) | (tag_of(w3) ^ tag);
+    return make_float4(untag(w0), untag(w1), untag(w2), untag(w3));
 }
 
 // One thread's bounded waits for tagged values.  After a wait has run out
 // (kErrStall set) the later ones return zeros at once, so the launch still
 // ends; the host reports the stall.
 struct Poll {
-    volatile int* err;
+    Waits wt;
     bool failed;
-    __device__ explicit Poll(volatile int* e) : err(e), failed(false) {}
-    __device__ __forceinline__ float wait1(const float* p, uint32_t tag) {
+    __device__ explicit Poll(const Waits& w) : wt(w), failed(false) {}
+    __device__ __forceinline__ float wait1(const Tagged* p, uint32_t tag) {
         if (!failed) {
             Bound bd;
             for (;;) {
                 __nanosleep(64);
-                const uint32_t b = ld_strong(p);
-                if (((b ^ tag) & 31u) == 0) return untag(b);
-                if (bd.expired(err)) break;
+                const unsigned long long b = ld_strong(p);
+                if (tag_of(b) == tag) return untag(b);
+                if (bd.expired(wt)) break;
             }
-            atomicOr((int*)err, kErrStall);
+            atomicOr((int*)wt.err, kErrStall);
             failed = true;
         }
         return 0.f;
@@ -524,8 +546,8 @@ struct Poll {
     __device__ __forceinline__ bool again(Bound& bd) {
         if (failed) return false;
         __nanosleep(64);
-        if (!bd.expired(err)) return true;
-        atomicOr((int*)err, kErrStall);
+        if (!bd.expired(wt)) return true;
+        atomicOr((int*)wt.err, kErrStall);
         failed = true;
         return false;
     }
@@ -533,13 +555,13 @@ struct Poll {
     // apart), then the consumer warps sync.  p is one of the phase's inputs:
     // once it has arrived the others mostly have too, so the gather that
     // follows finds them written and few threads poll.
-    __device__ __forceinline__ void probe(const float* p, uint32_t tag) {
+    __device__ __forceinline__ void probe(const Tagged* p, uint32_t tag) {
         if (threadIdx.x == 0) (void)get(p, tag);
         csync();
     }
-    __device__ __forceinline__ float get(const float* p, uint32_t tag) {
-        const uint32_t b = ld_strong(p);
-        return ((b ^ tag) & 31u) == 0 ? untag(b) : wait1(p, tag);
+    __device__ __forceinline__ float get(const Tagged* p, uint32_t tag) {
+        const unsigned long long b = ld_strong(p);
+        return tag_of(b) == tag ? untag(b) : wait1(p, tag);
     }
 };
 
@@ -593,10 +615,9 @@ __device__ __forceinline__ float4 f4add(float4 a, float4 b) {
     return make_float4(a.x + b.x, a.y + b.y, a.z + b.z, a.w + b.w);
 }
 __device__ __forceinline__ float4 ldg4(const float* p) { return *reinterpret_cast<const float4*>(p); }
-// a + the untagged v, noting a tag mismatch in bad
-__device__ __forceinline__ float4 add_tagged(float4 a, uint4 v, uint32_t tag, uint32_t& bad) {
-    bad |= mismatch4(v, tag);
-    return f4add(a, untag4(v));
+// a + the four tagged values at p, noting a tag mismatch in bad
+__device__ __forceinline__ float4 add_tagged(float4 a, const Tagged* p, uint32_t tag, uint32_t& bad) {
+    return f4add(a, load4(p, tag, bad));
 }
 __device__ __forceinline__ float4 bf4(const uint16_t* p) {
     const uint2 u = *reinterpret_cast<const uint2*>(p);
@@ -684,15 +705,15 @@ struct ResidIn {
     const SegPlan* p;
     const uint16_t* emb;  // embedding row, or null
     const float* src;     // m.h, or null for the slot sums
-    const float* opart;   // the previous layer's O slots
+    const Tagged* opart;  // the previous layer's O slots
     const uint8_t* nsd;
     uint32_t tag;         // the previous layer's tag
     __device__ __forceinline__ float operator()(int i, Poll& pl) const {
         if (emb) return bf(emb[i]);
         if (src) return src[i];
         const int t = i >> 5, l = i & 31, nco = p->n_chunks[1], ns = nsd[t];
-        const float* qo = opart + (int64_t)t * nco * 32 + l;
-        const float* qd = p->dpart + (int64_t)t * p->n_chunks[3] * 32 + l;
+        const Tagged* qo = opart + (int64_t)t * nco * 32 + l;
+        const Tagged* qd = p->dpart + (int64_t)t * p->n_chunks[3] * 32 + l;
         float v = 0.f;
         for (int k = 0; k < nco; ++k) v += pl.get(qo + k * 32, tag);
         for (int k = 0; k < ns; ++k) v += pl.get(qd + k * 32, tag);
@@ -703,34 +724,34 @@ struct ResidIn {
         if (emb) return bf4(emb + i);
         if (src) return ldg4(src + i);
         const int t = i >> 5, l = i & 31, nco = p->n_chunks[1], ns = nsd[t];
-        const float* qo = opart + (int64_t)t * nco * 32 + l;
-        const float* qd = p->dpart + (int64_t)t * p->n_chunks[3] * 32 + l;
+        const Tagged* qo = opart + (int64_t)t * nco * 32 + l;
+        const Tagged* qd = p->dpart + (int64_t)t * p->n_chunks[3] * 32 + l;
         float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
         for (int k = 0; k < kSegMaxSlots; ++k)
-            if (k < nco) v = add_tagged(v, ld_strong4(qo + k * 32), tag, bad);
+            if (k < nco) v = add_tagged(v, qo + k * 32, tag, bad);
 #pragma unroll
         for (int k = 0; k < kSegMaxSlots; ++k)
-            if (k < ns) v = add_tagged(v, ld_strong4(qd + k * 32), tag, bad);
+            if (k < ns) v = add_tagged(v, qd + k * 32, tag, bad);
         return v;
     }
 };
 // O slots of layer seq: two buffers, alternating by layer (a chunk-0 O item
 // reads the previous layer's slots while the other items of its tile write
 // this layer's).
-__device__ __forceinline__ float* opart_of(const SegPlan& p, unsigned seq) {
+__device__ __forceinline__ Tagged* opart_of(const SegPlan& p, unsigned seq) {
     return p.opart + (int64_t)(seq & 1u) * p.n_tiles[1] * p.n_chunks[1] * 32;
 }
 // Mid residual (after the attention block) at rows i..i+3: the sum of the O
 // slots, tagged with this layer's tag.
-__device__ __forceinline__ float4 resid_mid4(const SegPlan& p, const float* opart, int i, uint32_t tag,
+__device__ __forceinline__ float4 resid_mid4(const SegPlan& p, const Tagged* opart, int i, uint32_t tag,
                                              uint32_t& bad) {
     const int t = i >> 5, nco = p.n_chunks[1];
-    const float* qo = opart + (int64_t)t * nco * 32 + (i & 31);
+    const Tagged* qo = opart + (int64_t)t * nco * 32 + (i & 31);
     float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
     for (int k = 0; k < kSegMaxSlots; ++k)
-        if (k < nco) v = add_tagged(v, ld_strong4(qo + k * 32), tag, bad);
+        if (k < nco) v = add_tagged(v, qo + k * 32, tag, bad);
     return v;
 }
 
@@ -740,7 +761,7 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
     extern __shared__ __align__(128) uint8_t seg_smem[];
     const Smem s = carve(seg_smem, m, p);
     const int cta = blockIdx.x, G = p.G;
-    volatile int* err = &m.ctl->err;
+    const Waits wt{&m.ctl->err, p.stall_cycles, p.check_cycles};
     const int half = m.D >> 1, grp = m.A / m.KH;
     const int AD = m.A * m.D;
 
@@ -768,7 +789,7 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
     // ---------------------------------------------------------- producer
     if (threadIdx.x >= kCT) {
         if (threadIdx.x != kCT || !pos_ok) return;
-        Producer pr(s, p.stages, min(p.stages, p.inflight), err);
+        Producer pr(s, p.stages, min(p.stages, p.inflight), wt);
         // The CTA's chunk list, layer by layer: its Q/K/V tiles, its
         // attention unit's K then V pages, its O items, its gate/up tiles,
         // its down items.
@@ -838,8 +859,8 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
         if (cta == 0 && threadIdx.x == 0) atomicOr(&c->err, kErrPosition);
         return;
     }
-    Consumer cs(s, p.stages, err);
-    Poll pl(err);
+    Consumer cs(s, p.stages, wt);
+    Poll pl(wt);
     unsigned* sync = p.sync;
     const int64_t last_dn_slot = (int64_t)(p.n_tiles[3] - 1) * p.n_chunks[3];  // first slot of the last down tile
     const unsigned seq0 = sync[1];  // layers run since the context was reset
@@ -873,8 +894,7 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
         const int64_t n = (int64_t)m.A * per_head;
         for (int64_t e = (int64_t)cta * kCT + threadIdx.x; e < n; e += (int64_t)G * kCT) {
             const int h = (int)(e / per_head), r = (int)(e - (int64_t)h * per_head);
-            float* q = p.attn_part + ((int64_t)h * kSegMaxSplits + ag.splits) * (m.D + 4) + r;
-            asm volatile("st.relaxed.gpu.global.b32 [%0], %1;" ::"l"(q), "r"(0u) : "memory");
+            st_zero(p.attn_part + ((int64_t)h * kSegMaxSplits + ag.splits) * (m.D + 4) + r);
         }
     }
     csync();
@@ -884,7 +904,7 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
         const unsigned seq = seq0 + (unsigned)(j - j0);
         const uint32_t tag = seq_tag(seq);
         const uint16_t* lw = m.layers + (int64_t)j * m.layer_stride;
-        float* op_cur = opart_of(p, seq);
+        Tagged* op_cur = opart_of(p, seq);
         const ResidIn rin{&p,          (j == j0 && first) ? m.embed + (int64_t)tok * m.d : nullptr,
                           j == j0 ? m.h : nullptr, opart_of(p, seq - 1), s.nsd, seq_tag(seq - 1)};
 
@@ -942,62 +962,70 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
             const int p0 = pg0 * m.page_size, p1 = min(ag.T, pg1 * m.page_size);
             const int npos = p1 - p0;
             pl.probe(p.kvn + (m.KH + g + 1) * m.D - 1, tag);  // the last value of this group's v
-            const float* qsrc = p.q + (int64_t)g * grp * m.D;
-            const float* kt = p.kvn + (int64_t)g * m.D;
-            const float* vt = p.kvn + (int64_t)(m.KH + g) * m.D;
+            const Tagged* qsrc = p.q + (int64_t)g * grp * m.D;
+            const Tagged* kt = p.kvn + (int64_t)g * m.D;
+            const Tagged* vt = p.kvn + (int64_t)(m.KH + g) * m.D;
             // the group's scaled queries, then k and v, in one round (s.kv follows s.qa)
             const int nqa = grp * m.D;
             gather4<1>(s.qa, nqa + 2 * m.D, pl, [&](int i, uint32_t& bad) {
                 if (i >= nqa) {
                     const int e = i - nqa;
-                    return add_tagged(make_float4(0.f, 0.f, 0.f, 0.f), ld_strong4(e < m.D ? kt + e : vt + e - m.D), tag,
-                                      bad);
+                    return load4(e < m.D ? kt + e : vt + e - m.D, tag, bad);
                 }
-                const float4 q = add_tagged(make_float4(0.f, 0.f, 0.f, 0.f), ld_strong4(qsrc + i), tag, bad);
+                const float4 q = load4(qsrc + i, tag, bad);
                 return make_float4(q.x * scale, q.y * scale, q.z * scale, q.w * scale);
             });
             csync();
             // Scores on the tensor cores: S[h][r] = q_h . k_r as mma m16n8k16
-            // (bf16 operands, fp32 accumulation) with A = the group's queries
-            // split into bf16 high parts (rows 0..7) and low parts (rows 8..15,
-            // the bf16 of q - high; high + low keeps q to 16 bits) and B = 8
-            // cached keys.  A lane loads 8 consecutive dimensions of one key row
-            // (16 bytes, no bank conflicts beyond the row stride's); the
-            // product's k index runs over the dimensions in the same permuted
-            // order in A and B.  Row g of the result is head g's high-part dot
-            // product, row g + 8 its low-part one.
+            // (bf16 operands, fp32 accumulation) with B = 8 cached keys and A
+            // the group's queries split into three bf16 parts (high + middle +
+            // low = q exactly): one product with the high parts in rows 0..7
+            // and the middle parts in rows 8..15, a second with the low parts
+            // in rows 0..7 (rows 8..15 zero), into the same accumulators.  The
+            // bf16 products are exact in fp32.  A lane loads 8 consecutive
+            // dimensions of one key row (16 bytes, no bank conflicts beyond the
+            // row stride's); the product's k index runs over the dimensions in
+            // the same permuted order in A and B.  Row g of the result holds
+            // head g's high- and low-part dot products, row g + 8 its
+            // middle-part one.
             const int spc = p.max_pps * m.page_size;  // score row stride
             const int npair = m.D >> 5;               // pairs of k16 steps (32 dimensions)
             const int g8 = lane >> 2, t4 = lane & 3;
-            // The group's queries as bf16 high and low parts, converted once
-            // into rows padded to 16 bytes past D (xs is free here), so that the
-            // fragment loads of 8 heads at one column fall in different banks.
+            // The group's queries as three bf16 parts, converted once into
+            // rows padded to 16 bytes past D (xs is free here: seg_plan checks
+            // it holds 3 grp (D + 8) bf16), so that the fragment loads of 8
+            // heads at one column fall in different banks.
             {
                 const int qrow = m.D + 8;
                 uint16_t* qhs = reinterpret_cast<uint16_t*>(s.xs);
-                uint16_t* qls = qhs + grp * qrow;
                 for (int e = threadIdx.x; e < nqa / 4; e += kCT) {
                     const float4 q4 = lds128f(saddr(s.qa + 4 * e));
                     const int h = (4 * e) / m.D, c = 4 * e - h * m.D;
-                    uint32_t h01, l01, h23, l23;
-                    split_bf16x2(q4.x, q4.y, h01, l01);
-                    split_bf16x2(q4.z, q4.w, h23, l23);
+                    uint32_t h01, m01, l01, h23, m23, l23;
+                    split3_bf16x2(q4.x, q4.y, h01, m01, l01);
+                    split3_bf16x2(q4.z, q4.w, h23, m23, l23);
                     sts64(saddr(qhs + h * qrow + c), h01, h23);
-                    sts64(saddr(qls + h * qrow + c), l01, l23);
+                    sts64(saddr(qhs + (grp + h) * qrow + c), m01, m23);
+                    sts64(saddr(qhs + (2 * grp + h) * qrow + c), l01, l23);
                 }
                 csync();
             }
-            uint32_t qhi[4][4], qlo[4][4];  // [pair][word]: dimensions pair*32 + 8 t4 .. +7 of query g8
+            // [pair][word]: dimensions pair*32 + 8 t4 .. +7 of query g8 (the
+            // low parts stay in shared memory: qlo_at, read with each product)
+            uint32_t qhi[4][4], qmid[4][4];
+            const bool qrow_ok = g8 < grp;
+            const uint32_t qlo_at =
+                saddr(reinterpret_cast<const uint16_t*>(s.xs) + (2 * grp + (qrow_ok ? g8 : 0)) * (m.D + 8) + 8 * t4);
 #pragma unroll
             for (int pr = 0; pr < 4; ++pr) {
-                if (pr < npair && g8 < grp) {
+                if (pr < npair && qrow_ok) {
                     const uint16_t* qhs = reinterpret_cast<const uint16_t*>(s.xs) + g8 * (m.D + 8) + pr * 32 + 8 * t4;
                     const uint4 a = lds128(saddr(qhs)), b = lds128(saddr(qhs + grp * (m.D + 8)));
                     qhi[pr][0] = a.x, qhi[pr][1] = a.y, qhi[pr][2] = a.z, qhi[pr][3] = a.w;
-                    qlo[pr][0] = b.x, qlo[pr][1] = b.y, qlo[pr][2] = b.z, qlo[pr][3] = b.w;
+                    qmid[pr][0] = b.x, qmid[pr][1] = b.y, qmid[pr][2] = b.z, qmid[pr][3] = b.w;
                 } else {
 #pragma unroll
-                    for (int wd = 0; wd < 4; ++wd) qhi[pr][wd] = qlo[pr][wd] = 0u;
+                    for (int wd = 0; wd < 4; ++wd) qhi[pr][wd] = qmid[pr][wd] = 0u;
                 }
             }
             for (int pg = pg0; pg < pg1; ++pg)
@@ -1023,8 +1051,12 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
                             for (int pr = 0; pr < 4; ++pr) {
                                 if (pr < npair) {
                                     const uint4 kw = lds128(krow + pr * 64);
-                                    mma_bf16(acc, qhi[pr][0], qlo[pr][0], qhi[pr][1], qlo[pr][1], kw.x, kw.y);
-                                    mma_bf16(acc, qhi[pr][2], qlo[pr][2], qhi[pr][3], qlo[pr][3], kw.z, kw.w);
+                                    mma_bf16(acc, qhi[pr][0], qmid[pr][0], qhi[pr][1], qmid[pr][1], kw.x, kw.y);
+                                    mma_bf16(acc, qhi[pr][2], qmid[pr][2], qhi[pr][3], qmid[pr][3], kw.z, kw.w);
+                                    uint4 lo = lds128(qlo_at + pr * 64);
+                                    if (!qrow_ok) lo = make_uint4(0u, 0u, 0u, 0u);
+                                    mma_bf16(acc, lo.x, 0u, lo.y, 0u, kw.x, kw.y);
+                                    mma_bf16(acc, lo.z, 0u, lo.w, 0u, kw.z, kw.w);
                                 }
                             }
                             const int ra = r0 + 2 * t4;
@@ -1135,14 +1167,14 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
                     const int h = e / d4, c = 4 * (e - h * d4);
                     float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
                     for (int k = 0; k < npq; ++k) sum = f4add(sum, *reinterpret_cast<const float4*>(part + (h * npq + k) * m.D + c));
-                    float* dst = p.attn_part + ((int64_t)(g * grp + h) * kSegMaxSplits + sp) * (m.D + 4) + c;
+                    Tagged* dst = p.attn_part + ((int64_t)(g * grp + h) * kSegMaxSplits + sp) * (m.D + 4) + c;
                     st_tagged(dst, sum.x, tag);
                     st_tagged(dst + 1, sum.y, tag);
                     st_tagged(dst + 2, sum.z, tag);
                     st_tagged(dst + 3, sum.w, tag);
                 }
                 if (threadIdx.x < grp) {
-                    float* dst = p.attn_part + ((int64_t)(g * grp + threadIdx.x) * kSegMaxSplits + sp) * (m.D + 4) + m.D;
+                    Tagged* dst = p.attn_part + ((int64_t)(g * grp + threadIdx.x) * kSegMaxSplits + sp) * (m.D + 4) + m.D;
                     st_tagged(dst, s.ml[2 * threadIdx.x], tag);
                     st_tagged(dst + 1, s.ml[2 * threadIdx.x + 1], tag);
                 }
@@ -1195,29 +1227,26 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
                     if (cols) *dst = make_float4(0.f, 0.f, 0.f, 0.f);
                     continue;
                 }
-                const float* base = p.attn_part + (int64_t)h * kSegMaxSplits * (m.D + 4);
-                const float* st = base + lane * (m.D + 4) + m.D;
-                const float* oc = base + lane * 4;
-                constexpr int kB = 12;
+                const Tagged* base = p.attn_part + (int64_t)h * kSegMaxSplits * (m.D + 4);
+                const Tagged* st = base + lane * (m.D + 4) + m.D;
+                const Tagged* oc = base + lane * 4;
+                constexpr int kB = 11;
                 float mk = -INFINITY, lk = 0.f;
                 float4 ob[kB];
                 Bound bd;
                 for (;;) {  // one round of loads, again until every lane has its values
                     uint32_t bad = 0;
                     if (lane < ns) {
-                        const uint32_t a = ld_strong(st), b = ld_strong(st + 1);
-                        bad |= ((a ^ tag) | (b ^ tag)) & 31u;
+                        unsigned long long a, b;
+                        ld_strong2(st, a, b);
+                        bad |= (tag_of(a) ^ tag) | (tag_of(b) ^ tag);
                         mk = untag(a);
                         lk = untag(b);
                     }
 #pragma unroll
                     for (int u = 0; u < kB; ++u) {
                         ob[u] = make_float4(0.f, 0.f, 0.f, 0.f);
-                        if (u < ns && cols) {
-                            const uint4 v = ld_strong4(oc + u * (m.D + 4));
-                            bad |= mismatch4(v, tag);
-                            ob[u] = untag4(v);
-                        }
+                        if (u < ns && cols) ob[u] = load4(oc + u * (m.D + 4), tag, bad);
                     }
                     if (!__any_sync(0xffffffffu, bad != 0)) break;
                     const bool more = pl.again(bd);
@@ -1235,11 +1264,7 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
 #pragma unroll
                             for (int u = 0; u < kB; ++u) {
                                 ob[u] = make_float4(0.f, 0.f, 0.f, 0.f);
-                                if (k0 + u < ns && cols) {
-                                    const uint4 v = ld_strong4(oc + (k0 + u) * (m.D + 4));
-                                    bad |= mismatch4(v, tag);
-                                    ob[u] = untag4(v);
-                                }
+                                if (k0 + u < ns && cols) ob[u] = load4(oc + (k0 + u) * (m.D + 4), tag, bad);
                             }
                             if (!__any_sync(0xffffffffu, bad != 0)) break;
                             const bool more = pl.again(bd2);
@@ -1300,8 +1325,7 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
             gather4<4>(s.xa, (idn.hi - idn.lo) * kColsPerChunk, pl, [&](int e, uint32_t& bad) {
                 const int i = idn.lo + e / kColsPerChunk, col = e % kColsPerChunk;
                 const int ch = i % idn.nc, f = ch * kColsPerChunk + col;
-                return f < m.F ? add_tagged(make_float4(0.f, 0.f, 0.f, 0.f), ld_strong4(p.a + f), tag, bad)
-                               : make_float4(0.f, 0.f, 0.f, 0.f);
+                return f < m.F ? load4(p.a + f, tag, bad) : make_float4(0.f, 0.f, 0.f, 0.f);
             });
             csync();
             float acc = 0.f;
@@ -1382,7 +1406,7 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_vocab_ring(VocabArgs v, int 
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     __syncthreads();
-    volatile int* err = v.ctl ? &v.ctl->err : &err_local;
+    const Waits wt{v.ctl ? &v.ctl->err : &err_local, kSegStallCycles, kSegCheckCycles};
     const int n_tiles = (v.V + kTileRows - 1) / kTileRows, nc = (v.d + kColsPerChunk - 1) / kColsPerChunk;
     int t0, t1;
     whole_tiles(n_tiles, gridDim.x, blockIdx.x, t0, t1);
@@ -1390,7 +1414,7 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_vocab_ring(VocabArgs v, int 
 
     if (threadIdx.x >= kCT) {  // producer
         if (threadIdx.x != kCT) return;
-        Producer pr(s, stages, stages, err);
+        Producer pr(s, stages, stages, wt);
         for (int t = t0; t < t1 && pr.ok; ++t)
             for (int c = 0; c < nc; ++c)
                 pr.push(U + (int64_t)t * kTileRows * v.d * 2 + (int64_t)c * kSegChunk, chunk_bytes(v.d, c), pr.pol_w);
@@ -1398,7 +1422,7 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_vocab_ring(VocabArgs v, int 
         return;
     }
 
-    Consumer cs(s, stages, err);
+    Consumer cs(s, stages, wt);
     vr_pdl_wait();
     vr_pdl_launch();
     // RMSNorm(x) * gain
@@ -1531,6 +1555,8 @@ bool seg_plan(const DevModel& m, int n_sm, SegPlan& p) {
     const size_t fixed = floats * 4 + (size_t)p.n_tiles[3] + 256;
     const size_t budget = 227 * 1024;
     if (fixed + 4 * (size_t)(kSegChunk + 16) > budget) return false;
+    // the attention unit's three bf16 parts of the group's queries fit in xs
+    if ((size_t)3 * grp * (m.D + 8) * 2 > (size_t)4 * ((std::max(m.d, m.A * m.D) + 3) & ~3)) return false;
     p.stages = (int)std::min<size_t>(16, (budget - fixed) / (kSegChunk + 16));
     p.smem = (size_t)p.stages * (kSegChunk + 16) + floats * 4 + (size_t)p.n_tiles[3];
     p.inflight = p.stages;

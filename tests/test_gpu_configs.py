@@ -1,0 +1,165 @@
+"""GPU parity on the large workloads at their stated lengths (needs a GB300).
+
+- 3B shape (36 layers, width 2048, 16/2 heads of 128, SwiGLU 11008, readout
+  at layer 18): 1024-token prompt, 32 gated steps at thresholds calibrated for
+  50% and 96% exits, on both layer paths.
+- 1.5B long-context shape (readouts at layers 7, 14 and 21): 8192-token
+  prompt, 16 gated steps at about 50% exits overall (first passing readout
+  exits), so attention runs over 8.2k positions.
+- 1.5B shape: 2048-token prompt and 64 gated steps, so the attended length
+  reaches 2112, and the whole cache (values and computed/filled marks) is
+  compared afterwards.
+
+The oracle runs free once per threshold (Section 4, step five); the GPU
+replays its inputs and exit decisions teacher-forced through the C ABI.
+Thresholds follow the exit-rate calibration: the quantile of the readouts'
+confidences over a full-depth oracle run of the same steps (tau > 1).  On
+steps outside the exclusion band token ids, gate verdicts and exit counts must
+match bit for bit, KV positions bit for bit, hidden states, logits and cache
+values within 1e-2 relative error.
+"""
+import math
+
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from helpers import (check_exit_counts, check_kv, check_records, gpu_replay, oracle_steps, p_errors, parity_log)
+
+pytestmark = pytest.mark.gpu
+
+
+def tau_for_rate(p, rate: float) -> float:
+    """Lowest tau with a fraction `rate` of p strictly above it (rate 0 ->
+    1.01, rate 1 -> 0)."""
+    if rate <= 0.0:
+        return 1.01
+    if rate >= 1.0:
+        return 0.0
+    s = np.sort(np.asarray(p, np.float32))
+    k = int(math.ceil((1.0 - rate) * len(s)))
+    return float(s[max(0, min(len(s) - 1, k - 1))])
+
+
+class OracleRuns:
+    """One oracle prefilled once; each threshold's run starts again from the
+    end of the prompt (truncate), and the last run's cache stays in place for
+    the KV comparison."""
+
+    def __init__(self, shape, model, prompt, n):
+        self.shape, self.n, self.P = shape, n, len(prompt)
+        self.orc = oracle.Oracle(shape, model, max_ctx=len(prompt) + n)
+        self.first = self.orc.prefill(prompt)
+        self.key = None
+        self.recs = None
+
+    def run(self, taus, capture=True):
+        key = (tuple(taus), capture)
+        if key != self.key:
+            self.orc.truncate(self.P)
+            self.recs = oracle_steps(self.orc, self.first, self.n, taus, capture=capture)
+            self.key = key
+        return self.recs
+
+    def calibrate(self):
+        """Every readout's confidence over the steps at full depth."""
+        R = len(self.shape.readout_layers)
+        recs = self.run([1.01] * R, capture=False)
+        return np.array([[r["o"]["confidence"][k] for k in range(R)] for r in recs])
+
+
+def replay(shape, model, runs: OracleRuns, prompt, taus, persistent: bool, capture: bool = True):
+    from paper_2609_14144_gb300 import OPT_DEBUG_LOGITS, OPT_PERSISTENT, Engine
+
+    recs = runs.run(taus, capture=capture)
+    eng = Engine(shape, model, max_ctx=len(prompt) + runs.n)
+    eng.set_option(OPT_PERSISTENT, 1 if persistent else 0)
+    eng.set_option(OPT_DEBUG_LOGITS, capture)
+    assert eng.prefill(prompt) == runs.first
+    return eng, gpu_replay(eng, recs, taus, capture=capture)
+
+
+# ------------------------------------------------------------------ 3B
+@pytest.fixture(scope="module")
+def three_b():
+    shape = synth.CONFIGS["3b"].replace(new_tokens=32)
+    model = synth.make_model(shape)
+    prompt = synth.prompt(shape)
+    runs = OracleRuns(shape, model, prompt, shape.new_tokens)
+    p = runs.calibrate()[:, 0]
+    taus = {r: tau_for_rate(p, r) for r in (0.5, 0.96)}
+    return shape, model, prompt, runs, taus
+
+
+@pytest.mark.parametrize("rate,persistent", [(0.5, True), (0.5, False), (0.96, True), (0.96, False)])
+def test_3b_teacher_forced(three_b, rate, persistent):
+    shape, model, prompt, runs, taus = three_b
+    tau = [taus[rate]]
+    eng, recs = replay(shape, model, runs, prompt, tau, persistent)
+    excluded = check_records(recs, tau)
+    check_exit_counts(recs, tau, 1)
+    pe = p_errors(recs)
+    exits = sum(r["o"]["exited"] for r in recs)
+    parity_log("3b", rate=rate, tau=tau[0], persistent=persistent, exits=int(exits), steps=len(recs),
+               excluded=excluded, p_err_max=float(pe.max()), p_err_mean=float(pe.mean()))
+    assert excluded <= len(recs) // 4
+    if rate > 0.9:
+        assert exits >= len(recs) // 2
+    # the cache: every layer at the decoded positions and the prompt's last 16
+    P = len(prompt)
+    check_kv(runs.orc, eng, shape, 0,
+             pairs=[(j, t) for j in range(shape.n_layers) for t in range(P - 16, P + runs.n)])
+    eng.close()
+
+
+# ------------------------------------------------------------------ 1.5B long context
+@pytest.fixture(scope="module")
+def long_ctx():
+    shape = synth.CONFIGS["1.5b-long"].replace(new_tokens=16)
+    model = synth.make_model(shape)
+    prompt = synth.prompt(shape)
+    runs = OracleRuns(shape, model, prompt, shape.new_tokens)
+    p = runs.calibrate()
+    # each readout at its 80th percentile: about half the steps exit at one
+    taus = [tau_for_rate(p[:, k], 0.2) for k in range(p.shape[1])]
+    return shape, model, prompt, runs, taus
+
+
+@pytest.mark.parametrize("persistent", [True, False])
+def test_1p5b_long_context_three_readouts(long_ctx, persistent):
+    shape, model, prompt, runs, taus = long_ctx
+    eng, recs = replay(shape, model, runs, prompt, taus, persistent)
+    excluded = check_records(recs, taus)
+    check_exit_counts(recs, taus, 3)
+    pe = p_errors(recs)
+    by = [sum(r["o"]["exit_readout"] == k for r in recs) for k in range(3)]
+    parity_log("1.5b-long", persistent=persistent, taus=taus, exits_by_readout=[int(x) for x in by],
+               steps=len(recs), excluded=excluded, p_err_max=float(pe.max()), p_err_mean=float(pe.mean()))
+    assert excluded <= len(recs) // 4
+    P = len(prompt)
+    rng = np.random.default_rng(5)
+    sample = [(int(j), int(t)) for j, t in zip(rng.integers(0, shape.n_layers, 400), rng.integers(0, P, 400))]
+    check_kv(runs.orc, eng, shape, 0,
+             pairs=sample + [(j, t) for j in range(shape.n_layers) for t in range(P - 4, P + runs.n)])
+    eng.close()
+
+
+# ------------------------------------------------------------------ 1.5B, 64 steps to 2112 positions
+def test_1p5b_64_steps_whole_cache():
+    shape = synth.CONFIGS["1.5b"].replace(prompt_len=2048, new_tokens=64)
+    model = synth.make_model(shape)
+    prompt = synth.prompt(shape)
+    runs = OracleRuns(shape, model, prompt, shape.new_tokens)
+    tau = [tau_for_rate(runs.calibrate()[:, 0], 0.5)]
+    eng, recs = replay(shape, model, runs, prompt, tau, True)
+    excluded = check_records(recs, tau)
+    check_exit_counts(recs, tau, 1)
+    pe = p_errors(recs)
+    exits = sum(r["o"]["exited"] for r in recs)
+    parity_log("1.5b-64", tau=tau[0], exits=int(exits), steps=len(recs), excluded=excluded,
+               p_err_max=float(pe.max()), p_err_mean=float(pe.mean()))
+    assert excluded <= len(recs) // 4
+    assert 0 < exits < len(recs)
+    check_kv(runs.orc, eng, shape, len(prompt) + runs.n)
+    eng.close()

@@ -5,7 +5,7 @@ and exit decisions through the C ABI.  On steps outside the exclusion band
 (|p - tau| or a top-2 gap below 1e-3) token ids and gate verdicts must match
 bit for bit; KV positions (which layer/position was computed or filled) must
 match bit for bit; hidden states, logits and KV values within 1e-2 relative
-error (max |diff| / max |ref|); confidences within 5e-3."""
+error (max |diff| / max |ref|); confidences within helpers.P_TOL."""
 import numpy as np
 import pytest
 

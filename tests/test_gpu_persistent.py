@@ -5,8 +5,9 @@ test_gpu_parity."""
 import numpy as np
 import pytest
 
+import oracle
 import synth
-from helpers import check_kv, check_records, teacher_forced
+from helpers import check_kv, check_records, gpu_replay, oracle_steps, teacher_forced
 
 pytestmark = pytest.mark.gpu
 
@@ -100,3 +101,30 @@ def test_1p5b_persistent_agrees_with_five_launch_path():
     first_diff = np.argmax(~agree) if not agree.all() else len(agree)
     assert first_diff == len(agree) or near[first_diff]
     assert np.max(np.abs(c0[:first_diff] - c1[:first_diff]), initial=0) < 1e-3
+
+
+def test_waits_that_run_out_report_a_stall_and_reset_recovers():
+    """Failure detection of the persistent layer kernel's bounded waits: with
+    the wait bound lowered to 400 SM cycles, ordinary waits (ring stages,
+    values from other CTAs) run out.  The launch ends by itself with the
+    device error word set, the call reports EE_EDEVICE, and after ee_reset
+    with the normal bound the engine decodes like the oracle again."""
+    from paper_2609_14144_gb300 import OPT_WAIT_LIMIT, EEError, Engine
+
+    tiny = synth.CONFIGS["tiny"]
+    model = synth.make_model(tiny)
+    prompt = synth.prompt(tiny)
+    eng = Engine(tiny, model)
+    assert eng.persistent
+    eng.set_option(OPT_WAIT_LIMIT, 400)
+    with pytest.raises(EEError) as e:
+        eng.prefill(prompt)
+    assert e.value.code == -5 and "timed out" in str(e.value)
+    eng.set_option(OPT_WAIT_LIMIT, 0)
+    eng.reset()
+    orc = oracle.Oracle(tiny, model)
+    first = orc.prefill(prompt)
+    assert eng.prefill(prompt) == first
+    recs = gpu_replay(eng, oracle_steps(orc, first, 12, [0.5]), [0.5], capture=False)
+    check_records(recs, [0.5], capture=False)
+    eng.close()

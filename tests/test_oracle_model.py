@@ -499,6 +499,35 @@ def test_prefill_matrix_product_form_matches_position_by_position(kw, lens):
     assert n_diff <= n_all // 1000
 
 
+def test_truncate_then_decode_equals_a_fresh_run():
+    """Forgetting the decoded positions and decoding again (another tau, so
+    other exits and fills) gives, bit for bit, what a fresh oracle gives."""
+    shape = micro()
+    model = synth.make_model(shape)
+    ids = synth.prompt(shape)
+    P, n = len(ids), shape.new_tokens
+    a = oracle.Oracle(shape, model)
+    first = a.prefill(ids)
+    tok = first
+    for _ in range(n):
+        tok = a.decode_step(tok, [0.0])["token"]
+    a.truncate(P)
+    assert a.pos == P and a.stats()["steps"] == 0
+    b = oracle.Oracle(shape, model)
+    assert b.prefill(ids) == first
+    ta = tb = first
+    for _ in range(n):
+        ra, rb = a.decode_step(ta, [0.4]), b.decode_step(tb, [0.4])
+        assert ra == rb
+        ta, tb = ra["token"], rb["token"]
+    assert a.stats() == b.stats()
+    for j in range(shape.n_layers):
+        for t in range(shape.max_ctx):
+            ka, va, sa = a.kv(j, t)
+            kb, vb, sb = b.kv(j, t)
+            assert sa == sb and np.array_equal(ka, kb) and np.array_equal(va, vb)
+
+
 def test_qkv_bias_and_tied_head_options():
     shape = micro(qkv_bias=True, tied_embedding=True)
     model = synth.make_model(shape)
