@@ -7,14 +7,16 @@ a 512-token prompt and 512 greedy tokens.  tau is calibrated as the quantile
 of the readout's top-1 probability over a seeded 2048-token calibration
 stream (teacher-forced at full depth) to hit the target exit rate.
 
-One benchmark step = one ee_decode_n call producing 64 tokens (a graph
-launch that runs 64 gated decode steps with on-device token feedback).
---warmup W steps, then --steps K timed steps, continuing the same sequence:
-the default 3 + 5 steps generate exactly the workload's 512 tokens.
+The timed region decodes exactly the workload's 512 greedy tokens after the
+prompt, in --steps ee_decode_n calls (one benchmark step = one call: a graph
+launch running its share of the gated decode steps with on-device token
+feedback).  --warmup calls run first on a sequence of their own; the prompt is
+then prefilled again outside the timed region.
 
 The JSON line reports tokens/s at the 50% exit target, the exit-rate sweep
 (calibrated tau and imposed exits), the unmodified model (no readout) as the
-speedup denominator, the achieved HBM bandwidth of the whole step from the
+speedup denominator, the 0.5B, 3B and long-context workloads at their own
+calibrated exit rates, the achieved HBM bandwidth of the whole step from the
 algorithmic byte count, the dominant kernel's roofline, an end-to-end number
 through the host-buffer API, SM clocks during the timed region, and the CPU
 oracle's speed on a bounded sample.  ``--impl reference`` times the CPU
@@ -277,8 +279,9 @@ def run_reference(args, rank: int, world: int):
     import oracle
 
     tokens_per_step = 2
-    orc = oracle.Oracle(shape, model, max_ctx=64 + tokens_per_step * (args.steps + args.warmup))
-    tok = orc.prefill(synth.prompt(shape, 16))
+    P = shape.prompt_len
+    orc = oracle.Oracle(shape, model, max_ctx=P + tokens_per_step * (args.steps + args.warmup))
+    tok = orc.prefill(synth.prompt(shape, P))
     sched = synth.exit_schedule(shape, 4096, HEADLINE_RATE, index=7)
     i = 0
 
@@ -297,7 +300,7 @@ def run_reference(args, rank: int, world: int):
     dt = time.perf_counter() - t0
     value = args.steps * tokens_per_step / dt
     cores = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
-    sample = (f"{shape.name}: 16-token prompt, {tokens_per_step} gated decode steps per benchmark step with exits "
+    sample = (f"{shape.name}: {P}-token prompt, {tokens_per_step} gated decode steps per benchmark step with exits "
               f"imposed at {HEADLINE_RATE:.0%} (Bernoulli schedule), {args.steps} timed steps")
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": dt / args.steps * 1e3, "higher_is_better": True,
@@ -316,34 +319,52 @@ def _workload_desc(shape) -> str:
 
 
 # --------------------------------------------------------------------- GPU arm
+def chunk_sizes(n_new: int, steps: int) -> list:
+    """`steps` chunk lengths that add up to n_new tokens (the first n_new mod
+    steps one longer)."""
+    base, extra = divmod(n_new, steps)
+    return [base + (1 if i < extra else 0) for i in range(steps)]
+
+
 class Runner:
-    def __init__(self, eng, shape, world, chunk):
+    """Timed decodes of one workload: the prompt is prefilled outside the
+    timed region, then the workload's new tokens are decoded in `steps`
+    ee_decode_n calls (benchmark steps) that together produce exactly the
+    configuration's number of greedy tokens.  Warm-up calls run on a sequence
+    of their own, before a reset and a fresh prefill."""
+
+    def __init__(self, eng, shape, world, n_new):
         import torch
         self.torch = torch
-        self.eng, self.shape, self.world, self.chunk = eng, shape, world, chunk
+        self.eng, self.shape, self.world, self.n_new = eng, shape, world, n_new
         self.dims = bm.Dims.of(shape)
 
+    def _prefill(self, prompt):
+        self.eng.reset()
+        self.eng.prefill(prompt)
+
     def run(self, taus, warmup, steps, schedule=None, prompt=None, clocks=None):
-        """reset + prefill (untimed), `warmup` chunks, then `steps` timed chunks."""
-        torch, eng, C = self.torch, self.eng, self.chunk
+        torch, eng = self.torch, self.eng
         from paper_2609_14144_gb300 import DEVICE
         prompt = synth.prompt(self.shape) if prompt is None else prompt
-        eng.reset()
-        eng.prefill(prompt)
-        P = len(prompt)
-        n = (warmup + steps) * C
+        P, n = len(prompt), self.n_new
+        sizes = chunk_sizes(n, steps)
         tok = torch.empty(n, dtype=torch.int32, device=eng.device)
         ex = torch.empty(n, dtype=torch.int32, device=eng.device)
         cf = torch.empty(n, dtype=torch.float32, device=eng.device)
-
-        def chunk(i):
-            sl = slice(i * C, (i + 1) * C)
-            sch = None if schedule is None else schedule[sl]
-            eng.decode_n(C, taus, schedule=sch, where=DEVICE, tokens=tok[sl], exit_readout=ex[sl], confidence=cf[sl])
-
-        for i in range(warmup):
-            chunk(i)
-        eng.sync()
+        if warmup:
+            self._prefill(prompt)
+            at = 0
+            for i in range(warmup):
+                c = min(sizes[0], n - at)
+                if c <= 0:
+                    break
+                sch = None if schedule is None else schedule[at:at + c]
+                eng.decode_n(c, taus, schedule=sch, where=DEVICE, tokens=tok[at:at + c], exit_readout=ex[at:at + c],
+                             confidence=cf[at:at + c])
+                at += c
+            eng.sync()
+        self._prefill(prompt)
         barrier(self.world)
         e0 = torch.cuda.Event(enable_timing=True)
         e1 = torch.cuda.Event(enable_timing=True)
@@ -351,8 +372,12 @@ class Runner:
         ctx = clocks if clocks is not None else _Null()
         with ctx:
             e0.record(eng.stream)
-            for i in range(warmup, warmup + steps):
-                chunk(i)
+            at = 0
+            for c in sizes:
+                sch = None if schedule is None else schedule[at:at + c]
+                eng.decode_n(c, taus, schedule=sch, where=DEVICE, tokens=tok[at:at + c], exit_readout=ex[at:at + c],
+                             confidence=cf[at:at + c])
+                at += c
             e1.record(eng.stream)
             e1.synchronize()
         torch.cuda.synchronize()
@@ -360,32 +385,38 @@ class Runner:
         ms = e0.elapsed_time(e1)
         ms_max = max_over_ranks(ms, self.world)
         exits = ex.cpu().numpy()
-        timed = exits[warmup * C:]
-        T0 = P + warmup * C
         ro = list(self.shape.readout_layers)
-        bytes_total = sum(bm.step_bytes(self.dims, T0 + i + 1, ro, None if e < 0 else int(e))
-                          for i, e in enumerate(timed))
-        launches = sum(step_launches(self.shape.n_layers, ro, int(e), self.eng.persistent) for e in timed) + steps
-        n_tok = steps * C
-        return {"ms": ms_max, "tokens": n_tok * self.world, "tok_s": n_tok * self.world / (ms_max / 1e3),
-                "exit_rate": float(np.mean(timed >= 0)) if len(ro) else 0.0,
-                "bytes_per_token": bytes_total / n_tok, "gbs": bytes_total * self.world / (ms_max / 1e3) / 1e9,
-                "launches": launches, "tokens_out": tok.cpu().numpy(), "exits": exits}
+        bytes_total = sum(bm.step_bytes(self.dims, P + i + 1, ro, None if e < 0 else int(e))
+                          for i, e in enumerate(exits))
+        launches = sum(step_launches(self.shape.n_layers, ro, int(e), self.eng.persistent) for e in exits) + steps
+        return {"ms": ms_max, "tokens": n * self.world, "tok_s": n * self.world / (ms_max / 1e3),
+                "exit_rate": float(np.mean(exits >= 0)) if len(ro) else 0.0,
+                "exits_by_readout": [int(np.sum(exits == k)) for k in range(len(ro))],
+                "bytes_per_token": bytes_total / n, "gbs": bytes_total * self.world / (ms_max / 1e3) / 1e9,
+                "launches": launches, "tokens_out": tok.cpu().numpy(), "exits": exits,
+                "attended": [P + 1, P + n]}
 
-    def run_host(self, taus, warmup, steps):
-        """The same through the host-buffer API: each call copies its results
-        back and synchronises (end to end)."""
-        eng, C = self.eng, self.chunk
-        eng.reset()
-        eng.prefill(synth.prompt(self.shape))
+    def run_host(self, taus, warmup, steps, prompt):
+        """The same decode through the host-buffer API: every call copies tau
+        in and its tokens, exits and confidences (and the control block) back
+        and synchronises (end to end)."""
+        eng, n = self.eng, self.n_new
+        sizes = chunk_sizes(n, steps)
+        self._prefill(prompt)
+        at = 0
         for _ in range(warmup):
-            eng.decode_n(C, taus)
+            c = min(sizes[0], n - at)
+            if c <= 0:
+                break
+            eng.decode_n(c, taus)
+            at += c
+        self._prefill(prompt)
         barrier(self.world)
         t0 = time.perf_counter()
-        for _ in range(steps):
-            eng.decode_n(C, taus)
+        for c in sizes:
+            eng.decode_n(c, taus)
         dt = max_over_ranks(time.perf_counter() - t0, self.world)
-        return steps * C * self.world / dt
+        return n * self.world / dt
 
 
 class _Null:
@@ -426,6 +457,85 @@ def calibrate(eng, shape, n: int = CALIB_TOKENS, p_nuc: float = 0.9, fidelity: f
     return p, summary
 
 
+def taus_for_overall_rate(p: np.ndarray, rate: float) -> list:
+    """Thresholds for several readouts (shallowest first, first passing one
+    exits): every readout at the same per-readout quantile level, chosen by
+    bisection so that the share of calibration positions at which some
+    readout passes is about `rate`."""
+    lo, hi = 0.0, rate
+    taus = None
+    for _ in range(40):
+        mid = 0.5 * (lo + hi)
+        taus = [tau_for_rate(p[:, k], mid) for k in range(p.shape[1])]
+        overall = float(np.mean(np.any(p > np.asarray(taus, np.float32)[None, :], axis=1)))
+        if overall < rate:
+            lo = mid
+        else:
+            hi = mid
+    return taus
+
+
+def kernel_roofline(eng, run, shape, prompt, taus, exit_rate, W_tokens, peak) -> dict:
+    """Per-kernel device time (direct launches, CUDA events on the engine's
+    stream) after a prefill and W_tokens decoded tokens, and the dominant
+    kernel's algorithmic GB/s against the measured copy bandwidth."""
+    eng.reset()
+    eng.prefill(prompt)
+    if W_tokens:
+        eng.decode_n(W_tokens, taus)
+    kms = eng.profile_kernels(iters=2 * shape.n_layers)
+    T_prof = eng.position + 1
+    kb = kernel_bytes(run.dims, T_prof, shape.readout_layers[0])
+    per_tok = kernel_launches_per_token(shape.n_layers, shape.readout_layers[0], exit_rate, eng.persistent)
+    share = {k: kms[k] * per_tok[k] for k in kms}
+    dom = max(share, key=share.get)
+    ach = kb[dom] / (kms[dom] / 1e3) / 1e9
+    return {"bound": "hbm", "kernel": dom, "achieved": ach, "peak": peak["hbm_gbs"], "unit": "GB/s",
+            "frac": ach / peak["hbm_gbs"], "peak_source": peak["source"],
+            "traffic": ncu_traffic(dom, shape.name, T_prof, run.dims), "bytes_per_launch": kb[dom],
+            "ms_per_launch": kms[dom], "attended_positions": T_prof,
+            "kernels": {k: {"ms": kms[k], "GBps": kb[k] / (kms[k] / 1e3) / 1e9 if kms[k] > 0 else None,
+                            "share": share[k] / sum(share.values())} for k in kms}}
+
+
+def extra_workload(name: str, args, world: int, local: int, peak: dict) -> dict:
+    """Decode throughput of another workload at its calibrated exit rates:
+    its own prompt and new-token count, the timed region covering exactly
+    those tokens (args.steps calls, one warm-up call), the step's algorithmic
+    GB/s and its fraction of the measured copy bandwidth, and the layer
+    kernel's roofline."""
+    from paper_2609_14144_gb300 import OPT_ROWS, Engine
+
+    shape = synth.CONFIGS[name]
+    t0 = time.perf_counter()
+    model = synth.make_model(shape)
+    prompt = synth.prompt(shape)
+    eng = Engine(shape, model, max_ctx=max(shape.prompt_len + shape.new_tokens, CALIB_TOKENS), device=local)
+    run = Runner(eng, shape, world, shape.new_tokens)
+    p_all, _ = calibrate(eng, shape)
+    # long prompts: the multi-position pass fills the cache (the prompt is not timed)
+    eng.set_option(OPT_ROWS, 1 if shape.prompt_len >= 4096 else 0)
+    if len(shape.readout_layers) > 1:
+        plan = [(r, taus_for_overall_rate(p_all, r)) for r in shape.exit_rates]
+    else:
+        plan = [(r, [tau_for_rate(p_all[:, 0], r)]) for r in shape.exit_rates]
+    sweep = []
+    for r, taus in plan:
+        res = run.run(taus, 1, args.steps, prompt=prompt)
+        sweep.append({"target_rate": r, "tau": taus if len(taus) > 1 else taus[0], "exit_rate": res["exit_rate"],
+                      "exits_by_readout": res["exits_by_readout"], "tok_s": res["tok_s"], "GBps": res["gbs"],
+                      "frac": res["gbs"] / peak["hbm_gbs"], "MB_per_token": res["bytes_per_token"] / 1e6})
+        _log(f"[bench] {name} r={r}: rate={res['exit_rate']:.3f} {res['tok_s']:.1f} tok/s {res['gbs']:.0f} GB/s")
+    mid = plan[len(plan) // 2]
+    roof = kernel_roofline(eng, run, shape, prompt, mid[1], sweep[len(plan) // 2]["exit_rate"],
+                           min(64, shape.new_tokens), peak)
+    eng.close()
+    del eng, model
+    return {"workload": _workload_desc(shape), "timed": f"{shape.new_tokens} tokens after the {shape.prompt_len}-"
+            f"token prompt in {args.steps} calls", "sweep": sweep, "roofline": roof,
+            "s": time.perf_counter() - t0}
+
+
 def run_ours(args, rank: int, world: int, local: int):
     import torch
 
@@ -433,15 +543,16 @@ def run_ours(args, rank: int, world: int, local: int):
 
     torch.cuda.set_device(local)
     shape = synth.CONFIGS[WORKLOAD]
-    C, W, K = args.chunk, args.warmup, args.steps
-    n_new = (W + K) * C
+    W, K = args.warmup, args.steps
+    n_new = shape.new_tokens
     t0 = time.perf_counter()
     model = synth.make_model(shape.replace(seed=shape.seed))
     prompt = synth.token_ids(shape.seed + 1000 * rank, synth.SID_PROMPT, shape.prompt_len, shape.vocab)
     _log(f"[bench] rank {rank}: model generated in {time.perf_counter() - t0:.1f} s")
     max_ctx = max(shape.prompt_len + n_new, CALIB_TOKENS)
     eng = Engine(shape, model, max_ctx=max_ctx, device=local)
-    run = Runner(eng, shape, world, C)
+    run = Runner(eng, shape, world, n_new)
+    peak = _peaks()
 
     t0 = time.perf_counter()
     p_all, cal = calibrate(eng, shape)
@@ -454,7 +565,7 @@ def run_ours(args, rank: int, world: int, local: int):
 
     # headline: calibrated tau at the 50% target
     tau_h = taus[HEADLINE_RATE]
-    run.run([tau_h], 1, 1, prompt=prompt)  # build graphs, warm the path
+    run.run([tau_h], 1, K, prompt=prompt)  # build graphs, warm the path
     clocks = ClockSampler(local)
     head = run.run([tau_h], W, K, prompt=prompt, clocks=clocks)
     clk = clocks.summary()
@@ -464,13 +575,15 @@ def run_ours(args, rank: int, world: int, local: int):
     sweep = []
     if not args.no_sweep:
         for r in sorted(taus):
-            res = run.run([taus[r]], W, K, prompt=prompt)
+            res = run.run([taus[r]], 1, K, prompt=prompt)
             sched = np.where(synth.exit_schedule(shape, n_new, r, index=1) == 1, FORCE_EXIT_AT(0),
                              FORCE_FULL).astype(np.int8)
-            imp = run.run([0.5], W, K, schedule=sched, prompt=prompt)
+            imp = run.run([0.5], 1, K, schedule=sched, prompt=prompt)
             sweep.append({"target_rate": r, "tau": taus[r], "exit_rate": res["exit_rate"],
-                          "tok_s": res["tok_s"], "GBps": res["gbs"], "MB_per_token": res["bytes_per_token"] / 1e6,
+                          "tok_s": res["tok_s"], "GBps": res["gbs"], "frac": res["gbs"] / peak["hbm_gbs"],
+                          "MB_per_token": res["bytes_per_token"] / 1e6,
                           "imposed": {"exit_rate": imp["exit_rate"], "tok_s": imp["tok_s"], "GBps": imp["gbs"],
+                                      "frac": imp["gbs"] / peak["hbm_gbs"],
                                       "MB_per_token": imp["bytes_per_token"] / 1e6}})
             _log(f"[bench] sweep r={r}: tau={taus[r]:.4f} rate={res['exit_rate']:.3f} {res['tok_s']:.1f} tok/s "
                  f"{res['gbs']:.0f} GB/s | imposed rate={imp['exit_rate']:.3f} {imp['tok_s']:.1f} tok/s")
@@ -479,10 +592,10 @@ def run_ours(args, rank: int, world: int, local: int):
     plain_line = None
     if not args.no_sweep:
         eng_plain = Engine(shape, model, max_ctx=max_ctx, device=local, readouts=False)
-        rp = Runner(eng_plain, shape.replace(readout_layers=()), world, C)
-        rp.run(None, 1, 1, prompt=prompt)
-        pl = rp.run(None, W, K, prompt=prompt)
-        plain_line = {"tok_s": pl["tok_s"], "GBps": pl["gbs"], "MB_per_token": pl["bytes_per_token"] / 1e6,
+        rp = Runner(eng_plain, shape.replace(readout_layers=()), world, n_new)
+        pl = rp.run(None, 1, K, prompt=prompt)
+        plain_line = {"tok_s": pl["tok_s"], "GBps": pl["gbs"], "frac": pl["gbs"] / peak["hbm_gbs"],
+                      "MB_per_token": pl["bytes_per_token"] / 1e6,
                       "speedup_at_headline": head["tok_s"] / pl["tok_s"]}
         _log(f"[bench] plain model: {pl['tok_s']:.1f} tok/s, {pl['gbs']:.0f} GB/s")
         eng_plain.close()
@@ -535,33 +648,25 @@ def run_ours(args, rank: int, world: int, local: int):
              f"one position at a time")
 
     # end to end through the host-buffer API
-    e2e = run.run_host([tau_h], W, K)
+    e2e = run.run_host([tau_h], W, K, prompt)
 
     # per-kernel device time (direct launches) and the dominant kernel's roofline
-    eng.reset()
-    eng.prefill(prompt)
-    eng.decode_n(W * C, [tau_h])
-    kms = eng.profile_kernels(iters=2 * shape.n_layers)
-    T_prof = eng.position + 1
-    kb = kernel_bytes(run.dims, T_prof, shape.readout_layers[0])
-    per_tok = kernel_launches_per_token(shape.n_layers, shape.readout_layers[0], head["exit_rate"], eng.persistent)
-    share = {k: kms[k] * per_tok[k] for k in kms}
-    dom = max(share, key=share.get)
-    peak = _peaks()
-    ach = kb[dom] / (kms[dom] / 1e3) / 1e9
-    roofline = {"bound": "hbm", "kernel": dom, "achieved": ach, "peak": peak["hbm_gbs"], "unit": "GB/s",
-                "frac": ach / peak["hbm_gbs"], "peak_source": peak["source"],
-                "traffic": ncu_traffic(dom, WORKLOAD, T_prof, run.dims), "bytes_per_launch": kb[dom],
-                "ms_per_launch": kms[dom],
-                "kernels": {k: {"ms": kms[k], "GBps": kb[k] / (kms[k] / 1e3) / 1e9 if kms[k] > 0 else None,
-                                "share": share[k] / sum(share.values())} for k in kms}}
+    roofline = kernel_roofline(eng, run, shape, prompt, [tau_h], head["exit_rate"], n_new // 2, peak)
     step_roof = {"achieved": head["gbs"], "peak": peak["hbm_gbs"], "unit": "GB/s",
                  "frac": head["gbs"] / peak["hbm_gbs"], "frac_of_nominal_7900": head["gbs"] / 7900.0,
                  "MB_per_token": head["bytes_per_token"] / 1e6}
+    eng.close()
+    del eng
+
+    # the other large workloads, each at its calibrated exit rates
+    workloads = {}
+    if not args.no_sweep and world == 1:
+        for name in ("0.5b", "3b", "1.5b-long"):
+            workloads[name] = extra_workload(name, args, world, local, peak)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
-        cpu = oracle_sample(shape, model, seconds=args.cpu_seconds)
+        cpu = oracle_sample(shape, model, seconds=args.cpu_seconds, prompt_len=shape.prompt_len)
         _log(f"[bench] cpu oracle: {cpu['value']:.2f} tok/s on {cpu['cores']} cores")
 
     ms_per_step = head["ms"] / K
@@ -569,14 +674,19 @@ def run_ours(args, rank: int, world: int, local: int):
         "metric": METRIC, "value": head["tok_s"], "unit": UNIT, "n_gpus": world, "steps": K, "warmup": W,
         "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": _workload_desc(shape), "tokens_per_step": C, "exit_rate_target": HEADLINE_RATE,
-                   "tau": tau_h, "exit_rate": head["exit_rate"], "parallelism": f"replicas x{world}",
+        "config": {"workload": _workload_desc(shape),
+                   "timed": f"the {n_new} greedy tokens after the {shape.prompt_len}-token prompt (attended "
+                            f"positions {head['attended'][0]}..{head['attended'][1]}), in {K} ee_decode_n calls of "
+                            f"{min(chunk_sizes(n_new, K))}-{max(chunk_sizes(n_new, K))} tokens; warm-up calls on a "
+                            f"sequence of their own",
+                   "exit_rate_target": HEADLINE_RATE, "tau": tau_h, "exit_rate": head["exit_rate"],
+                   "parallelism": f"replicas x{world}",
                    "l2": "inputs larger than L2: every token streams 1.8-3.6 GB of weights",
                    "numerics": "bf16 weights and KV cache, fp32 activations and accumulation (values exchanged "
-                               "between CTAs rounded to 19 significant bits; attention scores from bf16 high/low query "
-                               "parts on the tensor cores)"},
+                               "between CTAs whole fp32; attention scores from three bf16 parts of the query on "
+                               "the tensor cores, exact products)"},
         "e2e": {"value": e2e, "unit": UNIT, "h2d_bytes_per_step": 4 * 8,
-                "d2h_bytes_per_step": 12 * C + CTL_BYTES},
+                "d2h_bytes_per_step": 12 * max(chunk_sizes(n_new, K)) + CTL_BYTES},
         "gpu_launches": head["launches"],
         "roofline": roofline,
         "step_roofline": step_roof,
@@ -584,11 +694,11 @@ def run_ours(args, rank: int, world: int, local: int):
         "clocks": clk,
         "sweep": sweep,
         "plain_model": plain_line,
+        "workloads": workloads,
         "calibration": cal,
         "repass": repass,
         "prefill": prefill,
     }
-    eng.close()
     if rank == 0:
         print(json.dumps(line), flush=True)
 
@@ -661,7 +771,6 @@ def main():
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=5)
     ap.add_argument("--warmup", type=int, default=3)
-    ap.add_argument("--chunk", type=int, default=64, help="tokens per benchmark step")
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--no-sweep", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")

@@ -1230,7 +1230,7 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
                 const Tagged* base = p.attn_part + (int64_t)h * kSegMaxSplits * (m.D + 4);
                 const Tagged* st = base + lane * (m.D + 4) + m.D;
                 const Tagged* oc = base + lane * 4;
-                constexpr int kB = 11;
+                constexpr int kB = 8;
                 float mk = -INFINITY, lk = 0.f;
                 float4 ob[kB];
                 Bound bd;

@@ -74,3 +74,18 @@ def test_launch_and_byte_accounting_agree_with_the_cost_model():
     assert lp["qkv"] == 0 and lp["layers"] == 1 + 0.5 * (L - k) / k
     per_token_pers = kb["layers"] * L / k + kb["readout"] + 2 * kb["vocab"]
     assert per_token_pers == pytest.approx(model_full, rel=2e-3)
+
+
+def test_timed_calls_cover_exactly_the_workload_tokens():
+    for n, k in ((512, 20), (512, 5), (1024, 7), (256, 256), (256, 3)):
+        sizes = bench.chunk_sizes(n, k)
+        assert len(sizes) == k and sum(sizes) == n and max(sizes) - min(sizes) <= 1
+
+
+def test_thresholds_for_an_overall_exit_rate_over_three_readouts():
+    rng = np.random.default_rng(1)
+    p = rng.random((2047, 3)).astype(np.float32)
+    for r in (0.3, 0.5, 0.8):
+        taus = bench.taus_for_overall_rate(p, r)
+        overall = np.mean(np.any(p > np.asarray(taus, np.float32)[None, :], axis=1))
+        assert abs(overall - r) < 0.01
