@@ -531,7 +531,6 @@ struct Poll {
         if (!failed) {
             Bound bd;
             for (;;) {
-                __nanosleep(64);
                 const unsigned long long b = ld_strong(p);
                 if (tag_of(b) == tag) return untag(b);
                 if (bd.expired(wt)) break;
@@ -545,7 +544,6 @@ struct Poll {
     // the wait has run out (kErrStall set; the caller keeps what it has).
     __device__ __forceinline__ bool again(Bound& bd) {
         if (failed) return false;
-        __nanosleep(64);
         if (!bd.expired(wt)) return true;
         atomicOr((int*)wt.err, kErrStall);
         failed = true;
@@ -699,23 +697,21 @@ __device__ __forceinline__ void tile_gemv(Consumer& cs, int t0, int t1, int K, i
 }
 
 // Residual entering layer j at row i: the embedding (first layer of a step),
-// the model's h (first layer of a later segment), or the previous layer's O
-// slots (its mid residual) plus its down slots, tagged with that layer's tag.
+// the model's h (first layer of a later segment), or the sum of the previous
+// layer's down slots (slot 0 of each tile carries that layer's mid residual),
+// tagged with that layer's tag.
 struct ResidIn {
     const SegPlan* p;
     const uint16_t* emb;  // embedding row, or null
     const float* src;     // m.h, or null for the slot sums
-    const Tagged* opart;  // the previous layer's O slots
     const uint8_t* nsd;
     uint32_t tag;         // the previous layer's tag
     __device__ __forceinline__ float operator()(int i, Poll& pl) const {
         if (emb) return bf(emb[i]);
         if (src) return src[i];
-        const int t = i >> 5, l = i & 31, nco = p->n_chunks[1], ns = nsd[t];
-        const Tagged* qo = opart + (int64_t)t * nco * 32 + l;
+        const int t = i >> 5, l = i & 31, ns = nsd[t];
         const Tagged* qd = p->dpart + (int64_t)t * p->n_chunks[3] * 32 + l;
         float v = 0.f;
-        for (int k = 0; k < nco; ++k) v += pl.get(qo + k * 32, tag);
         for (int k = 0; k < ns; ++k) v += pl.get(qd + k * 32, tag);
         return v;
     }
@@ -723,13 +719,9 @@ struct ResidIn {
     __device__ __forceinline__ float4 four(int i, uint32_t& bad) const {
         if (emb) return bf4(emb + i);
         if (src) return ldg4(src + i);
-        const int t = i >> 5, l = i & 31, nco = p->n_chunks[1], ns = nsd[t];
-        const Tagged* qo = opart + (int64_t)t * nco * 32 + l;
+        const int t = i >> 5, l = i & 31, ns = nsd[t];
         const Tagged* qd = p->dpart + (int64_t)t * p->n_chunks[3] * 32 + l;
         float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-        for (int k = 0; k < kSegMaxSlots; ++k)
-            if (k < nco) v = add_tagged(v, qo + k * 32, tag, bad);
 #pragma unroll
         for (int k = 0; k < kSegMaxSlots; ++k)
             if (k < ns) v = add_tagged(v, qd + k * 32, tag, bad);
@@ -905,8 +897,19 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
         const uint32_t tag = seq_tag(seq);
         const uint16_t* lw = m.layers + (int64_t)j * m.layer_stride;
         Tagged* op_cur = opart_of(p, seq);
-        const ResidIn rin{&p,          (j == j0 && first) ? m.embed + (int64_t)tok * m.d : nullptr,
-                          j == j0 ? m.h : nullptr, opart_of(p, seq - 1), s.nsd, seq_tag(seq - 1)};
+        const ResidIn rin{&p, (j == j0 && first) ? m.embed + (int64_t)tok * m.d : nullptr, j == j0 ? m.h : nullptr,
+                          s.nsd, seq_tag(seq - 1)};
+        // The RMSNorm gains the next gathers read (this layer's MLP gain, the
+        // next layer's attention gain, or after the last layer the final gain
+        // the vocabulary pass reads): into L2 now, so that those gathers do
+        // not wait on HBM.  A few CTAs issue them, one 128-byte line per lane.
+        if (cta < 2 && w == 1) {
+            const uint16_t* gsrc = cta == 0 ? lw + m.off_gmlp
+                                            : (j + 1 < m.L ? m.layers + (int64_t)(j + 1) * m.layer_stride + m.off_gattn
+                                                           : m.g_final);
+            for (int b = lane * 64; b < m.d; b += 32 * 64)
+                asm volatile("prefetch.global.L2 [%0];" ::"l"(gsrc + b));
+        }
 
         // ---------------- Q/K/V tiles: RMSNorm, projection, bias, RoPE, KV append
         if (tq1 > tq0) {
@@ -1185,54 +1188,55 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
         // project, write the chunk's slot (chunk 0 adds the residual)
         if (io.hi > io.lo) {
             const int ns = ag.splits;
-            {   // the last split's maximum of the first item's first head
-                const int h0 = min(m.A - 1, (io.lo % io.nc) * (kColsPerChunk / m.D));
-                pl.probe(p.attn_part + ((int64_t)h0 * kSegMaxSplits + ns - 1) * (m.D + 4) + m.D, tag);
-            }
             const int nit = io.hi - io.lo, ncol = nit * kColsPerChunk;
             const int hpc = kColsPerChunk / m.D;  // heads per chunk
             float* rows = s.xa + ncol;
-            // One warp per (item, head): the head's split statistics (lane =
-            // split) and this lane's four columns of every split's partial o
-            // in one round of loads, then o = sum_s w_s o_s / sum_s w_s l_s with
-            // w_s = exp(m_s - max m).  One more warp per chunk-0 item gathers
-            // the residual rows its slot carries.
-            for (int wi = w; wi < nit * (hpc + 1); wi += kCW) {
-                if (wi >= nit * hpc) {
-                    const int it = wi - nit * hpc, i = io.lo + it, t = i / io.nc;
-                    if (lane < 8) {
-                        const int row = t * 32 + 4 * lane;
-                        float4 r = make_float4(0.f, 0.f, 0.f, 0.f);
-                        if (i - t * io.nc == 0 && row < m.d) {
-                            uint32_t bad = 0;
-                            r = rin.four(row, bad);
-                            if (bad) {
-                                Bound bd;
-                                while (pl.again(bd)) {
-                                    bad = 0;
-                                    r = rin.four(row, bad);
-                                    if (!bad) break;
-                                }
+            // The residual rows a chunk-0 item's slot carries: the previous
+            // layer's (or the segment's input), complete since this layer's
+            // Q/K/V phase read them, so gathered before the wait below.
+            for (int it = w; it < nit; it += kCW) {
+                const int i = io.lo + it, t = i / io.nc;
+                if (lane < 8) {
+                    const int row = t * 32 + 4 * lane;
+                    float4 r = make_float4(0.f, 0.f, 0.f, 0.f);
+                    if (i - t * io.nc == 0 && row < m.d) {
+                        uint32_t bad = 0;
+                        r = rin.four(row, bad);
+                        if (bad) {
+                            Bound bd;
+                            while (pl.again(bd)) {
+                                bad = 0;
+                                r = rin.four(row, bad);
+                                if (!bad) break;
                             }
                         }
-                        reinterpret_cast<float4*>(rows + it * 32)[lane] = r;
                     }
-                    continue;
+                    reinterpret_cast<float4*>(rows + it * 32)[lane] = r;
                 }
-                const int it = wi / hpc, hc = wi - it * hpc, ch = (io.lo + it) % io.nc;
-                const int h = ch * hpc + hc;
-                const bool cols = lane * 4 < m.D;
-                float4* dst = reinterpret_cast<float4*>(s.xa + it * kColsPerChunk + hc * m.D) + lane;
+            }
+            {   // the last split's maximum of the first item's first head
+                const int h0 = min(m.A - 1, (io.lo % io.nc) * hpc);
+                pl.probe(p.attn_part + ((int64_t)h0 * kSegMaxSplits + ns - 1) * (m.D + 4) + m.D, tag);
+            }
+            // D / 64 warps per (item, head), each over 64 columns: the head's
+            // split statistics (lane = split) and this lane's two columns of
+            // every split's partial o in one round of loads (up to kB splits),
+            // then o = sum_s w_s o_s / sum_s w_s l_s with w_s = exp(m_s - max m).
+            const int wph = m.D >> 6;
+            for (int wi = w; wi < nit * hpc * wph; wi += kCW) {
+                const int it = wi / (hpc * wph), r = wi - it * hpc * wph, hc = r / wph, c0 = (r - hc * wph) * 64;
+                const int h = ((io.lo + it) % io.nc) * hpc + hc;
+                float2* dst = reinterpret_cast<float2*>(s.xa + it * kColsPerChunk + hc * m.D + c0) + lane;
                 if (h >= m.A) {
-                    if (cols) *dst = make_float4(0.f, 0.f, 0.f, 0.f);
+                    *dst = make_float2(0.f, 0.f);
                     continue;
                 }
                 const Tagged* base = p.attn_part + (int64_t)h * kSegMaxSplits * (m.D + 4);
                 const Tagged* st = base + lane * (m.D + 4) + m.D;
-                const Tagged* oc = base + lane * 4;
-                constexpr int kB = 8;
+                const Tagged* oc = base + c0 + 2 * lane;
+                constexpr int kB = 12;
                 float mk = -INFINITY, lk = 0.f;
-                float4 ob[kB];
+                float2 ob[kB];
                 Bound bd;
                 for (;;) {  // one round of loads, again until every lane has its values
                     uint32_t bad = 0;
@@ -1245,8 +1249,13 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
                     }
 #pragma unroll
                     for (int u = 0; u < kB; ++u) {
-                        ob[u] = make_float4(0.f, 0.f, 0.f, 0.f);
-                        if (u < ns && cols) ob[u] = load4(oc + u * (m.D + 4), tag, bad);
+                        ob[u] = make_float2(0.f, 0.f);
+                        if (u < ns) {
+                            unsigned long long a, b;
+                            ld_strong2(oc + u * (m.D + 4), a, b);
+                            bad |= (tag_of(a) ^ tag) | (tag_of(b) ^ tag);
+                            ob[u] = make_float2(untag(a), untag(b));
+                        }
                     }
                     if (!__any_sync(0xffffffffu, bad != 0)) break;
                     const bool more = pl.again(bd);
@@ -1255,7 +1264,7 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
                 const float mx = warp_max(mk);
                 const float wk = lane < ns ? expf(mk - mx) : 0.f;
                 const float dn = warp_sum(wk * lk);
-                float4 num = make_float4(0.f, 0.f, 0.f, 0.f);
+                float2 num = make_float2(0.f, 0.f);
                 for (int k0 = 0; k0 < ns; k0 += kB) {
                     if (k0 > 0) {  // the next splits (their statistics are in hand)
                         Bound bd2;
@@ -1263,8 +1272,13 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
                             uint32_t bad = 0;
 #pragma unroll
                             for (int u = 0; u < kB; ++u) {
-                                ob[u] = make_float4(0.f, 0.f, 0.f, 0.f);
-                                if (k0 + u < ns && cols) ob[u] = load4(oc + (k0 + u) * (m.D + 4), tag, bad);
+                                ob[u] = make_float2(0.f, 0.f);
+                                if (k0 + u < ns) {
+                                    unsigned long long a, b;
+                                    ld_strong2(oc + (k0 + u) * (m.D + 4), a, b);
+                                    bad |= (tag_of(a) ^ tag) | (tag_of(b) ^ tag);
+                                    ob[u] = make_float2(untag(a), untag(b));
+                                }
                             }
                             if (!__any_sync(0xffffffffu, bad != 0)) break;
                             const bool more = pl.again(bd2);
@@ -1277,13 +1291,11 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
                         if (k0 + u < ns) {
                             num.x = fmaf(wu, ob[u].x, num.x);
                             num.y = fmaf(wu, ob[u].y, num.y);
-                            num.z = fmaf(wu, ob[u].z, num.z);
-                            num.w = fmaf(wu, ob[u].w, num.w);
                         }
                     }
                 }
                 const float inv = 1.0f / dn;
-                if (cols) *dst = make_float4(num.x * inv, num.y * inv, num.z * inv, num.w * inv);
+                *dst = make_float2(num.x * inv, num.y * inv);
             }
             csync();
             for (int i = io.lo; i < io.hi; ++i) {
@@ -1319,8 +1331,29 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
             });
         }
 
-        // ---------------- down items: partial slots of h_out - h_mid
+        // ---------------- down items: partial slots of h_out (slot 0 of a tile
+        // adds the tile's mid residual rows, so the slots sum to h_out)
         if (idn.hi > idn.lo) {
+            // the mid residual rows of the tiles whose first item is this
+            // CTA's (the O slots are complete: this CTA's gate/up gather read
+            // them), gathered before the wait for the SwiGLU products
+            float* hm = s.xa + (idn.hi - idn.lo) * kColsPerChunk;  // [items][32]
+            for (int it = w; it < idn.hi - idn.lo; it += kCW) {
+                const int i = idn.lo + it, t = i / idn.nc;
+                if (lane < 8 && i - t * idn.nc == 0) {
+                    uint32_t bad = 0;
+                    float4 r = resid_mid4(p, op_cur, t * 32 + 4 * lane, tag, bad);
+                    if (bad) {
+                        Bound bd;
+                        while (pl.again(bd)) {
+                            bad = 0;
+                            r = resid_mid4(p, op_cur, t * 32 + 4 * lane, tag, bad);
+                            if (!bad) break;
+                        }
+                    }
+                    reinterpret_cast<float4*>(hm + it * 32)[lane] = r;
+                }
+            }
             pl.probe(p.a + (idn.lo % idn.nc) * kColsPerChunk, tag);  // the first product this CTA reads
             gather4<4>(s.xa, (idn.hi - idn.lo) * kColsPerChunk, pl, [&](int e, uint32_t& bad) {
                 const int i = idn.lo + e / kColsPerChunk, col = e % kColsPerChunk;
@@ -1342,10 +1375,10 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
                     acc = 0.f;
                     csync();
                     if (w == 0) {
-                        float sum = 0.f;
+                        const int slot = cta - item_owner(idn, t * idn.nc);
+                        float sum = slot == 0 ? hm[(t * idn.nc - idn.lo) * 32 + lane] : 0.f;
 #pragma unroll
                         for (int k = 0; k < kCW; ++k) sum += r[k * 32 + lane];
-                        const int slot = cta - item_owner(idn, t * idn.nc);
                         st_tagged(p.dpart + ((int64_t)t * idn.nc + slot) * 32 + lane, sum, tag);
                     }
                     rb ^= 1;
@@ -1358,7 +1391,7 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
     {
         const unsigned last = seq0 + (unsigned)(j1 - j0 - 1);
         pl.probe(p.dpart + (last_dn_slot + s.nsd[p.n_tiles[3] - 1] - 1) * 32 + 31, seq_tag(last));
-        const ResidIn rout{&p, nullptr, nullptr, opart_of(p, last), s.nsd, seq_tag(last)};
+        const ResidIn rout{&p, nullptr, nullptr, s.nsd, seq_tag(last)};
         for (int i = slice0 + threadIdx.x; i < slice1; i += kCT) m.h[i] = rout(i, pl);  // slice: scalar
     }
     // the exit ticket: once every CTA has taken it, no CTA reads the launch
