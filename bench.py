@@ -51,7 +51,7 @@ HEADLINE_RATE = 0.5
 CALIB_TOKENS = 2048
 REPASS_W = 16  # positions in the measured full-depth re-pass
 ROWS_MAX = 64  # positions per batch of the multi-position layer pass (EE_OPT_ROWS)
-CTL_BYTES = 360  # device control block read back by a host-buffer ee_decode_n
+CTL_BYTES = 368  # device control block read back by a host-buffer ee_decode_n
 
 
 def _peaks() -> dict:
@@ -539,7 +539,7 @@ def extra_workload(name: str, args, world: int, local: int, peak: dict) -> dict:
 def run_ours(args, rank: int, world: int, local: int):
     import torch
 
-    from paper_2609_14144_gb300 import FORCE_EXIT_AT, FORCE_FULL, OPT_ROWS, Engine
+    from paper_2609_14144_gb300 import FORCE_EXIT_AT, FORCE_FULL, OPT_LAZY_FILL, OPT_ROWS, Engine
 
     torch.cuda.set_device(local)
     shape = synth.CONFIGS[WORKLOAD]
@@ -579,14 +579,21 @@ def run_ours(args, rank: int, world: int, local: int):
             sched = np.where(synth.exit_schedule(shape, n_new, r, index=1) == 1, FORCE_EXIT_AT(0),
                              FORCE_FULL).astype(np.int8)
             imp = run.run([0.5], 1, K, schedule=sched, prompt=prompt)
+            # the same decode with the deferred fill (the byte count above assumes eager fills)
+            eng.set_option(OPT_LAZY_FILL, 1)
+            lz = run.run([taus[r]], 1, K, prompt=prompt)
+            eng.set_option(OPT_LAZY_FILL, 0)
             sweep.append({"target_rate": r, "tau": taus[r], "exit_rate": res["exit_rate"],
                           "tok_s": res["tok_s"], "GBps": res["gbs"], "frac": res["gbs"] / peak["hbm_gbs"],
                           "MB_per_token": res["bytes_per_token"] / 1e6,
                           "imposed": {"exit_rate": imp["exit_rate"], "tok_s": imp["tok_s"], "GBps": imp["gbs"],
                                       "frac": imp["gbs"] / peak["hbm_gbs"],
-                                      "MB_per_token": imp["bytes_per_token"] / 1e6}})
+                                      "MB_per_token": imp["bytes_per_token"] / 1e6},
+                          "deferred_fill": {"exit_rate": lz["exit_rate"], "tok_s": lz["tok_s"],
+                                            "speedup": lz["tok_s"] / res["tok_s"]}})
             _log(f"[bench] sweep r={r}: tau={taus[r]:.4f} rate={res['exit_rate']:.3f} {res['tok_s']:.1f} tok/s "
-                 f"{res['gbs']:.0f} GB/s | imposed rate={imp['exit_rate']:.3f} {imp['tok_s']:.1f} tok/s")
+                 f"{res['gbs']:.0f} GB/s | imposed rate={imp['exit_rate']:.3f} {imp['tok_s']:.1f} tok/s | "
+                 f"deferred fill {lz['tok_s']:.1f} tok/s")
 
     # the unmodified model (no readout): the speedup denominator
     plain_line = None

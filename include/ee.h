@@ -232,6 +232,11 @@ int ee_calibrate(ee_ctx* ctx, const int32_t* ids, int n, float p_nuc, float* con
 int ee_repass(ee_ctx* ctx, int32_t t0, int32_t t1, int32_t* n_repassed);
 
 /* Wait for the context's stream and report the device error word. */
+/* Fill every key/value entry that EE_OPT_LAZY_FILL left pending: each
+ * skipped layer's entry of each exited position becomes the projection of
+ * the residual the position exited with (Section 4, step five), exactly as
+ * the eager fill computes it.  Synchronous; EE_OK with nothing to do. */
+int ee_flush_fills(ee_ctx* ctx);
 int ee_sync(ee_ctx* ctx);
 int ee_get_stats(ee_ctx* ctx, ee_stats* out);
 /* Position of the next step's input token. */
@@ -280,6 +285,16 @@ int ee_position(ee_ctx* ctx, int32_t* pos);
                                  returns EE_EDEVICE; ee_reset clears it.  A
                                  few thousand cycles make ordinary waits run
                                  out.                                        */
+#define EE_OPT_LAZY_FILL 11    /* 0 (default): an exit step fills the key/value
+                                 entries of the layers it skips (Section 4,
+                                 step five); 1: it only records the residual
+                                 it exited with, and the next step that runs
+                                 one of those layers first fills every such
+                                 pending entry of the layers it runs (one read
+                                 of their key/value weights for all pending
+                                 positions).  Tokens are the same either way;
+                                 ee_flush_fills fills what is still pending.
+                                 Turning it off flushes.                     */
 int ee_set_option(ee_ctx* ctx, int option, int value);
 
 #define EE_DBG_HIDDEN_READOUT 1 /* layer = readout r: residual h_k it read, d floats   */

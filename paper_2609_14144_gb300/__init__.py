@@ -13,7 +13,7 @@ import numpy as np
 from . import _lib
 from ._lib import (CONF_MARGIN, CONF_NEGENT, CONF_PMAX, DEVICE, FORCE_FULL, FREE, HOST, MAX_READOUTS,
                    OPT_CONFIDENCE, OPT_DEBUG_LOGITS, OPT_GRAPHS, OPT_NUCLEUS, OPT_PDL, OPT_PERSISTENT, OPT_REPASS,
-                   OPT_ROWS, OPT_WAIT_LIMIT,
+                   OPT_LAZY_FILL, OPT_ROWS, OPT_WAIT_LIMIT,
                    EEError, FORCE_EXIT_AT, check)
 
 __all__ = ["Engine", "EEError", "FREE", "FORCE_FULL", "FORCE_EXIT_AT", "HOST", "DEVICE", "attention_decode",
@@ -205,6 +205,10 @@ class Engine:
         n = ctypes.c_int32(0)
         check(self.lib.ee_repass(self.ctx, int(t0), int(t1), ctypes.byref(n)))
         return n.value
+
+    def flush_fills(self):
+        """Fill every key/value entry the deferred fill left pending."""
+        check(self.lib.ee_flush_fills(self.ctx))
 
     def sync(self):
         check(self.lib.ee_sync(self.ctx))

@@ -13,6 +13,7 @@ HOST, DEVICE = 0, 1
 OPT_GRAPHS, OPT_PDL, OPT_DEBUG_LOGITS, OPT_PERSISTENT, OPT_CONFIDENCE, OPT_NUCLEUS, OPT_REPASS = 1, 2, 3, 4, 5, 6, 7
 OPT_ROWS = 8
 OPT_WAIT_LIMIT = 9
+OPT_LAZY_FILL = 11
 CONF_PMAX, CONF_MARGIN, CONF_NEGENT = 0, 1, 2
 DBG_HIDDEN_READOUT, DBG_READOUT_Y, DBG_HIDDEN_FINAL, DBG_READOUT_LOGITS, DBG_FINAL_LOGITS, DBG_KV, DBG_KV_SRC = \
     1, 2, 3, 4, 5, 6, 7
@@ -22,7 +23,7 @@ SYMBOLS = ("ee_workspace_bytes", "ee_create", "ee_destroy", "ee_last_error", "ee
            "ee_set_page_table", "ee_reset", "ee_prefill", "ee_decode_step", "ee_decode_n", "ee_sync",
            "ee_get_stats", "ee_position", "ee_set_option", "ee_debug_read", "ee_attention_scratch_bytes",
            "ee_attention_decode", "ee_vocab_scratch_bytes", "ee_vocab_confidence", "ee_vocab_signals", "ee_profile_kernels",
-           "ee_attention_decode_static", "ee_calibrate", "ee_select_tau", "ee_repass")
+           "ee_attention_decode_static", "ee_calibrate", "ee_select_tau", "ee_repass", "ee_flush_fills")
 KERNELS = ("qkv", "attention", "oproj", "gateup", "down", "readout", "vocab", "kvfill", "layers")
 
 
@@ -103,6 +104,7 @@ def load(allow_build: bool = False):
     lib.ee_decode_step.argtypes = [_P, i32, _P, ctypes.c_int, ctypes.POINTER(StepResult)]
     lib.ee_decode_n.argtypes = [_P, ctypes.c_int, i32, _P, _P, _P, _P, _P, ctypes.c_int]
     lib.ee_sync.argtypes = [_P]
+    lib.ee_flush_fills.argtypes = [_P]
     lib.ee_get_stats.argtypes = [_P, ctypes.POINTER(Stats)]
     lib.ee_position.argtypes = [_P, ctypes.POINTER(i32)]
     lib.ee_set_option.argtypes = [_P, ctypes.c_int, ctypes.c_int]

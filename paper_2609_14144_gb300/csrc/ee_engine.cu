@@ -242,6 +242,7 @@ struct ee_ctx {
     bool vring_ok = false;  // ring-fed vocabulary pass supported (used with the persistent layers)
     VocabRing vring{};
     bool use_rows = false;  // EE_OPT_ROWS: prompt and re-pass in batches of positions
+    bool lazy_fill = false; // EE_OPT_LAZY_FILL: skipped layers' entries filled by the next step that runs them
     RowsBuf rows{};
     int dbg = 0;
     int conf_kind = EE_CONF_PMAX;  // signal the gates compare with tau
@@ -425,6 +426,7 @@ int capture_segment(ee_ctx* c, int depth, int j0, int r) {
     const int L = c->cfg.n_layers;
     const int j1 = r < c->n_readouts ? c->ro_layer[r] : L;
     bool pdl = false;
+    if (c->lazy_fill && j0 > 0) EE_CK(launch_fill_pending(c->dm, j0, j1, false, s));
     EE_TRY(enqueue_layers(c, s, j0, j1, pdl));
     if (r >= c->n_readouts) return enqueue_head(c, s, pdl);
     cudaGraph_t g;
@@ -439,7 +441,12 @@ int capture_segment(ee_ctx* c, int depth, int j0, int r) {
     EE_CK(cudaStreamBeginCaptureToGraph(s2, bodies[0], nullptr, nullptr, 0, cudaStreamCaptureModeRelaxed));
     int rc = EE_OK;
     if (j1 < L) {
-        rc = enqueue_fill(c, s2, j1, false);
+        if (c->lazy_fill) {
+            const cudaError_t e2 = launch_record_exit(c->dm, j1, false, s2);
+            if (e2 != cudaSuccess) rc = fail(EE_ECUDA, cudaGetErrorString(e2));
+        } else {
+            rc = enqueue_fill(c, s2, j1, false);
+        }
     }
     cudaGraph_t tmp;
     cudaError_t e = cudaStreamEndCapture(s2, &tmp);
@@ -660,6 +667,15 @@ int rows_prefill(ee_ctx* c, const int32_t* d_prompt, int n) {
     return EE_OK;
 }
 
+// Fill every entry the deferred fill left pending (all layers, positions
+// below the decode position); afterwards nothing below it is pending.
+int flush_pending(ee_ctx* c) {
+    const DevModel& m = c->dm;
+    EE_CK(launch_fill_pending(m, 1, m.L, false, c->stream));
+    EE_CK(cudaMemcpyAsync(&c->d_ctl->pend_lo, &c->d_ctl->pos, 4, cudaMemcpyDeviceToDevice, c->stream));
+    return EE_OK;
+}
+
 // Section 11's full-depth re-pass over positions [t0, t1) (t1 <= pos): each
 // position whose upper layers still hold filled entries runs them again from
 // the residual it exited with (h_exit), in position order, through the same
@@ -671,6 +687,7 @@ int repass_range(ee_ctx* c, int t0, int t1, int* n_done) {
     const int L = m.L, W = t1 - t0;
     if (n_done) *n_done = 0;
     if (W <= 0) return EE_OK;
+    if (c->lazy_fill) EE_TRY(flush_pending(c));  // the re-pass finds exited positions by their fills
     EE_CK(cudaStreamSynchronize(s));
     std::vector<int16_t> ex(W);
     std::vector<int8_t> src((size_t)L * W);
@@ -716,6 +733,7 @@ int eager_step(ee_ctx* c) {
     int j0 = 0;
     for (int r = 0; r <= c->n_readouts; ++r) {
         const int j1 = r < c->n_readouts ? c->ro_layer[r] : m.L;
+        if (c->lazy_fill && j0 > 0) EE_CK(launch_fill_pending(m, j0, j1, false, s));
         EE_TRY(enqueue_layers(c, s, j0, j1, pdl));
         if (r == c->n_readouts) {
             EE_TRY(enqueue_head(c, s, pdl));
@@ -725,7 +743,10 @@ int eager_step(ee_ctx* c) {
         EE_TRY(fetch_ctl(c));
         pdl = false;
         if (c->h_ctl->exit_readout == r) {
-            EE_TRY(enqueue_fill(c, s, j1, false));
+            if (j1 < m.L && c->lazy_fill)
+                EE_CK(launch_record_exit(m, j1, false, s));
+            else
+                EE_TRY(enqueue_fill(c, s, j1, false));
             break;
         }
         j0 = j1;
@@ -851,7 +872,8 @@ int ee_create(const ee_model_config* cfg, void* d_workspace, size_t workspace_by
     c->rows.ldx = l.rows_ldx;
 
     const int kmax = std::max({2 * m.d, m.A * m.D, m.F});
-    if (configure_kernels(kmax) != cudaSuccess) return bail(fail(EE_ECUDA, "kernel configuration failed"));
+    if (configure_kernels(kmax) != cudaSuccess || configure_fill_pending(m.d) != cudaSuccess)
+        return bail(fail(EE_ECUDA, "kernel configuration failed"));
     c->attn_cluster = attention_cluster_size(m.D, m.KH);
     if (seg_plan(m, c->n_sm, c->seg) && configure_layers(c->seg.smem) == cudaSuccess &&
         layers_blocks_per_sm(c->seg.smem) >= 1) {
@@ -1064,6 +1086,15 @@ int ee_set_option(ee_ctx* c, int option, int value) {
             return EE_OK;
         case EE_OPT_ROWS:
             c->use_rows = value != 0;
+            return EE_OK;
+        case EE_OPT_LAZY_FILL:
+            if (c->lazy_fill == (value != 0)) return EE_OK;
+            if (c->lazy_fill && c->prefilled) {  // off: fill what is pending first
+                EE_TRY(flush_pending(c));
+                EE_CK(cudaStreamSynchronize(c->stream));
+            }
+            drop_graphs(c);
+            c->lazy_fill = value != 0;
             return EE_OK;
         case EE_OPT_WAIT_LIMIT:
             if (value < 0) return fail(EE_EINVAL, "wait limit must be >= 0");
@@ -1295,6 +1326,14 @@ int ee_repass(ee_ctx* c, int32_t t0, int32_t t1, int32_t* n_repassed) {
     EE_TRY(repass_range(c, t0, t1, &n));
     if (n_repassed) *n_repassed = n;
     return EE_OK;
+}
+
+int ee_flush_fills(ee_ctx* c) {
+    if (!c) return fail(EE_EINVAL, "NULL context");
+    if (!c->prefilled) return EE_OK;
+    EE_TRY(flush_pending(c));
+    EE_TRY(fetch_ctl(c));
+    return device_error(c);
 }
 
 int ee_sync(ee_ctx* c) {

@@ -59,9 +59,11 @@ struct Ctl {
     int32_t* out_member;   // [n_steps] nucleus_member per step (may be null)
     float* out_mass;       // [n_steps] nucleus_mass per step (may be null)
     const int32_t* forced_in; // [n_steps] teacher-forced inputs (null: the emitted token is fed back)
+    int32_t pend_lo;          // positions below have no deferred (pending) KV entries
+    int32_t pad_;
 };
 
-static_assert(sizeof(Ctl) == 360, "control block size is part of the host read-back accounting");
+static_assert(sizeof(Ctl) == 368, "control block size is part of the host read-back accounting");
 
 // Device pointers and shape, passed by value to every kernel.
 struct DevModel {
@@ -170,6 +172,13 @@ cudaError_t launch_down(const DevModel& m, int layer, int grid, bool whole, bool
 cudaError_t launch_readout(const DevModel& m, int r, int grid, bool whole, bool pdl, cudaStream_t s);
 cudaError_t launch_vocab(const VocabArgs& v, int grid, bool pdl, cudaStream_t s);
 cudaError_t launch_kvfill(const DevModel& m, int exit_layer, int grid_x, bool whole, bool pdl, cudaStream_t s);
+// Deferred fill (EE_OPT_LAZY_FILL): an exit step only records its residual
+// and exit layer; before a later step runs layers [j0, j1) every pending
+// entry of those layers is filled (one read of their key/value weights).
+cudaError_t launch_record_exit(const DevModel& m, int exit_layer, bool pdl, cudaStream_t s);
+size_t fill_pending_smem(int d);
+cudaError_t configure_fill_pending(int d);
+cudaError_t launch_fill_pending(const DevModel& m, int j0, int j1, bool pdl, cudaStream_t s);
 cudaError_t launch_step_end(const DevModel& m, int has_cond, cudaGraphConditionalHandle cond, bool pdl,
                             cudaStream_t s);
 cudaError_t launch_prefill_advance(const DevModel& m, int has_cond, cudaGraphConditionalHandle cond, bool pdl,

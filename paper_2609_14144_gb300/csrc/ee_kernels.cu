@@ -669,6 +669,99 @@ __global__ void __launch_bounds__(kGemvThreads, 2) k_kvfill(DevModel m, int exit
     }
 }
 
+// An exit step under the deferred fill: record the residual the position
+// exited with and its exit layer (what a later fill or re-pass starts from);
+// its skipped layers' entries stay empty.
+__global__ void k_record_exit(DevModel m, int exit_layer) {
+    pdl_wait();
+    pdl_launch_dependents();
+    const int pos = m.ctl->pos;
+    if (pos < 0 || pos >= m.max_ctx) return;
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < m.d; i += gridDim.x * blockDim.x)
+        m.h_exit[(int64_t)pos * m.d + i] = m.h[i];
+    if (blockIdx.x == 0 && threadIdx.x == 0) m.exit_at[pos] = (int16_t)exit_layer;
+}
+
+// The deferred KV fill (Section 4, step five): a skipped entry of layer j at
+// position p is the residual p exited with, through layer j's input RMSNorm
+// and its key and value matrices (the key rotated at p); deferred to the
+// first later step that runs layer j, it changes no token, since only such
+// a step reads it.  CTA (x, y) takes key/value tile x of layer j0 + y, staged
+// once in shared memory, and fills every pending entry of that layer: each
+// position p in [ctl->pend_lo, ctl->pos) that exited at a layer <= j
+// (exit_at) and whose entry at layer j is still empty (kv_src 0).  The
+// weights are read once for all pending positions.
+constexpr int kFillThreads = 256;
+__global__ void __launch_bounds__(kFillThreads) k_fill_pending(DevModel m, int j0) {
+    extern __shared__ float4 smem_f4[];
+    const int d = m.d, j = j0 + blockIdx.y, tile = blockIdx.x;
+    float* xs = reinterpret_cast<float*>(smem_f4);                       // [d]
+    float* part = xs + ((d + 3) & ~3);                                    // [8][32]
+    int* list = reinterpret_cast<int*>(part + 8 * 32);                    // [kFillThreads] + count
+    uint4* tile_sm = reinterpret_cast<uint4*>(list + kFillThreads + 4);   // 32 rows x d bf16, tile-packed
+    __shared__ float red[32];
+    const uint16_t* lw = m.layers + (int64_t)j * m.layer_stride;
+    const int64_t nq = (int64_t)m.A * m.D / 2, nk = (int64_t)m.KH * m.D / 2;
+    const int Rc = d >> 3;  // 16-byte column chunks
+    const uint4* W = reinterpret_cast<const uint4*>(lw + m.off_wqkv + nq * 2 * d) + (int64_t)tile * Rc * 32;
+    for (int i = threadIdx.x; i < Rc * 32; i += kFillThreads) cp_async16(tile_sm + i, W + i);
+    cp_async_commit();
+    pdl_wait();
+    pdl_launch_dependents();
+    const Ctl* c = m.ctl;
+    const int pos = c->pos, lo = max(0, c->pend_lo);
+    const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    bool staged = false;
+    for (int base = lo; base < pos; base += kFillThreads) {
+        // this round's pending positions, in position order
+        if (threadIdx.x == 0) list[kFillThreads] = 0;
+        __syncthreads();
+        const int p = base + threadIdx.x;
+        const bool need = p < pos && m.exit_at[p] > 0 && m.exit_at[p] <= j &&
+                          m.kv_src[(int64_t)j * m.max_ctx + p] == 0;
+        const unsigned bal = __ballot_sync(0xffffffffu, need);
+        if (lane == 0) red[w] = __int_as_float(__popc(bal));
+        __syncthreads();
+        int before = 0;
+        for (int k = 0; k < w; ++k) before += __float_as_int(red[k]);
+        if (need) list[before + __popc(bal & ((1u << lane) - 1))] = p;
+        if (threadIdx.x == 0) {
+            int n = 0;
+            for (int k = 0; k < kFillThreads / 32; ++k) n += __float_as_int(red[k]);
+            list[kFillThreads] = n;
+        }
+        __syncthreads();
+        const int n = list[kFillThreads];
+        if (n > 0 && !staged) {
+            cp_async_wait_all();
+            __syncthreads();
+            staged = true;
+        }
+        for (int k = 0; k < n; ++k) {
+            const int q = list[k];
+            rmsnorm_to_smem(m.h_exit + (int64_t)q * d, lw + m.off_gattn, d, m.eps, xs, red);
+            // lane = row of the tile, warp w the 16-byte column chunks w, w + 8, ...
+            float acc = 0.f;
+            for (int cc = w; cc < Rc; cc += kFillThreads / 32) acc += dot8(tile_sm[cc * 32 + lane], xs + cc * 8);
+            part[w * 32 + lane] = acc;
+            __syncthreads();
+            if (w == 0) {
+                float sum = 0.f;
+#pragma unroll
+                for (int k2 = 0; k2 < kFillThreads / 32; ++k2) sum += part[k2 * 32 + lane];
+                const int64_t kvo = kv_slot_offset(m, j, q);
+                const EpiQKV epi{nullptr, m.kpool + kvo, m.vpool + kvo, (int64_t)m.page_size * m.D,
+                                 m.qkv_bias ? lw + m.off_bqkv : nullptr, m.rope + (int64_t)q * (m.D / 2), nq, m.D,
+                                 (int)nq, (int)nk};
+                epi(tile, sum);
+            }
+            if (tile == 0 && threadIdx.x == 0) m.kv_src[(int64_t)j * m.max_ctx + q] = 2;
+            __syncthreads();
+        }
+    }
+    if (!staged) cp_async_wait_all();
+}
+
 // Output projection with the residual add: h += W_o o.
 template <bool WHOLE>
 __global__ void __launch_bounds__(kGemvThreads, 2) k_oproj(DevModel m, int layer) {
@@ -1259,10 +1352,12 @@ __global__ void k_step_end(DevModel m, int has_cond, cudaGraphConditionalHandle 
     if (c->out_member) c->out_member[st] = c->nucleus_member;
     if (c->out_mass) c->out_mass[st] = c->nucleus_member >= 0 ? c->nucleus_mass : NAN;
     c->steps += 1;
-    if (r >= 0)
+    if (r >= 0) {
         c->exits[r] += 1;
-    else
+    } else {
         c->full_steps += 1;
+        c->pend_lo = c->pos + 1;  // a full step ran every layer after filling what was pending
+    }
     c->pos += 1;
     c->in_tok = (c->forced_in && st + 1 < c->n_steps) ? c->forced_in[st + 1] : tok;
     c->step = st + 1;
@@ -1292,6 +1387,7 @@ __global__ void k_prefill_end(DevModel m) {
     c->exit_readout = -1;
     c->n_evaluated = 0;
     c->nucleus_member = -1;
+    c->pend_lo = c->pos;  // prompt positions ran every layer
 }
 
 // Per-call inputs written into the control block ahead of a graph launch.
@@ -1461,6 +1557,20 @@ cudaError_t launch_kvfill(const DevModel& m, int exit_layer, int grid_x, bool wh
     const size_t sm = gemv_smem(m.d, 0, whole);
     if (whole) return launch_k(k_kvfill<true>, grid, dim3(kGemvThreads), sm, pdl, s, m, exit_layer);
     return launch_k(k_kvfill<false>, grid, dim3(kGemvThreads), sm, pdl, s, m, exit_layer);
+}
+cudaError_t launch_record_exit(const DevModel& m, int exit_layer, bool pdl, cudaStream_t s) {
+    return launch_k(k_record_exit, dim3((m.d + 255) / 256), dim3(256), 0, pdl, s, m, exit_layer);
+}
+size_t fill_pending_smem(int d) {
+    return 4 * (size_t)(((d + 3) & ~3) + 8 * 32 + kFillThreads + 4) + 2 * 32 * (size_t)d;
+}
+cudaError_t configure_fill_pending(int d) {
+    return cudaFuncSetAttribute(k_fill_pending, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)fill_pending_smem(d));
+}
+cudaError_t launch_fill_pending(const DevModel& m, int j0, int j1, bool pdl, cudaStream_t s) {
+    if (j1 <= j0) return cudaSuccess;
+    const dim3 grid((unsigned)((2LL * m.KH * m.D + 31) / 32), (unsigned)(j1 - j0));
+    return launch_k(k_fill_pending, grid, dim3(kFillThreads), fill_pending_smem(m.d), pdl, s, m, j0);
 }
 cudaError_t launch_oproj(const DevModel& m, int layer, int grid, bool whole, bool pdl, cudaStream_t s) {
     const size_t sm = gemv_smem(m.A * m.D, 0, whole);

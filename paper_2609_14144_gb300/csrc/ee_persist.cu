@@ -1125,7 +1125,7 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
                     const int nr = min(rpc, p1 - base);
                     if (pv && cs.ok) {
                         const float* pr0 = s.sc + (hg * hpg) * spc + (base - p0);
-#pragma unroll 2
+#pragma unroll 4
                         for (int r = pq; r < nr; r += npq) {
                             float v[4];
                             if (dpl == 4) {

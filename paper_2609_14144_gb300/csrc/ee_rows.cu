@@ -333,6 +333,7 @@ __global__ void k_rows_prefill_done(DevModel m, int n) {
     if (threadIdx.x != 0) return;
     Ctl* c = m.ctl;
     c->pos = n;
+    c->pend_lo = n;  // prompt positions ran every layer
     c->prefill_i = n;
     c->exit_readout = -1;
     c->n_evaluated = 0;
