@@ -269,11 +269,14 @@ int ee_position(ee_ctx* ctx, int32_t* pos);
                                  readout 0's token at share value/1000
                                  (Section 2 acceptance)                      */
 #define EE_OPT_ROWS 8         /* 1: ee_prefill and ee_repass run each layer
-                                 over batches of up to 64 positions (tensor-
-                                 core products, each weight read once per
-                                 batch, each activation carried as three bf16
-                                 parts: 24 significant bits); 0 (default):
-                                 one position at a time through the decode
+                                 over batches of up to 64 positions, each
+                                 weight read once per batch, each activation
+                                 carried as three bf16 parts (24 significant
+                                 bits), the projections on the tcgen05 tensor
+                                 cores with TMA-staged operands (EE_EINVAL
+                                 where unavailable); 2: the same batches with
+                                 warp-level mma products; 0 (default): one
+                                 position at a time through the decode
                                  step's layer kernels (fp32 activations)    */
 #define EE_OPT_WAIT_LIMIT 9    /* for testing the failure path: the bound, in SM
                                  clock cycles, on each wait of the persistent

@@ -16,7 +16,7 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libee.so")
-SOURCES = ["ee_kernels.cu", "ee_engine.cu", "ee_persist.cu", "ee_noalloc.cu", "ee_rows.cu"]
+SOURCES = ["ee_kernels.cu", "ee_engine.cu", "ee_persist.cu", "ee_noalloc.cu", "ee_rows.cu", "ee_umma.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

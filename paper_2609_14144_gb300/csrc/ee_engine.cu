@@ -59,7 +59,7 @@ struct Layout {
     size_t kpool, vpool, page_table, kv_src, h_exit, exit_at, repass_pos, h, q, o, a, y, hk, logits_ro, logits_final;
     size_t gemv_part, gemv_ticket, attn_part, attn_ticket, vocab_part, vocab_ticket;
     size_t seg_dpart, seg_opart, seg_q, seg_kvn, seg_a, seg_attn, seg_sync, seg_end;
-    size_t rows_H, rows_xhi, rows_xmid, rows_xlo, rows_Q, rows_part, rows_pos;
+    size_t rows_H, rows_x3, rows_Q, rows_part, rows_pos;
     size_t prompt, sched, out_tok, out_exit, out_conf, out_conf_all, out_member, out_mass, tau_scratch, total;
     int64_t layer_stride, off_wqkv, off_bqkv, off_gattn, off_wo, off_gmlp, off_wgu, off_wd;
     int64_t n_units_qkv, kv_layer_stride, gemv_ticket_stride, rows_part_floats;
@@ -165,12 +165,10 @@ Layout make_layout(const ee_model_config& c) {
     l.seg_sync = take(4 * 8);
     l.seg_end = b;
     // multi-position layer pass (prompt and re-pass batches)
-    l.rows_ldx = (int)((std::max({d, F, A * D}) + 7) / 8 * 8);
+    l.rows_ldx = (int)((std::max({d, F, A * D}) + 63) / 64 * 64);
     l.rows_part_floats = rows_part_floats((int)d, (int)A, (int)KH, (int)D, (int)F);
     l.rows_H = take(4 * (size_t)kRowsMax * d);
-    l.rows_xhi = take(2 * (size_t)kRowsMax * l.rows_ldx);
-    l.rows_xmid = take(2 * (size_t)kRowsMax * l.rows_ldx);
-    l.rows_xlo = take(2 * (size_t)kRowsMax * l.rows_ldx);
+    l.rows_x3 = take(2 * 3 * (size_t)kRowsMax * l.rows_ldx);
     l.rows_Q = take(4 * (size_t)kRowsMax * A * D);
     l.rows_part = take(4 * (size_t)l.rows_part_floats);
     l.rows_pos = take(4 * (size_t)kRowsMax);
@@ -862,14 +860,15 @@ int ee_create(const ee_model_config* cfg, void* d_workspace, size_t workspace_by
     m.ctl = (Ctl*)(w + l.ctl);
     c->d_ctl = m.ctl;
     c->rows.H = (float*)(w + l.rows_H);
-    c->rows.xhi = (uint16_t*)(w + l.rows_xhi);
-    c->rows.xmid = (uint16_t*)(w + l.rows_xmid);
-    c->rows.xlo = (uint16_t*)(w + l.rows_xlo);
+    c->rows.x3 = (uint16_t*)(w + l.rows_x3);
     c->rows.Q = (float*)(w + l.rows_Q);
     c->rows.part = (float*)(w + l.rows_part);
     c->rows.pos = (int32_t*)(w + l.rows_pos);
     c->rows.part_floats = l.rows_part_floats;
     c->rows.ldx = l.rows_ldx;
+    c->rows.n_sm = c->n_sm;
+    c->rows.err = &c->d_ctl->err;
+    c->rows.umma = 0;
 
     const int kmax = std::max({2 * m.d, m.A * m.D, m.F});
     if (configure_kernels(kmax) != cudaSuccess || configure_fill_pending(m.d) != cudaSuccess)
@@ -1085,7 +1084,11 @@ int ee_set_option(ee_ctx* c, int option, int value) {
             c->nucleus_permille = value;
             return EE_OK;
         case EE_OPT_ROWS:
+            if (value < 0 || value > 2) return fail(EE_EINVAL, "EE_OPT_ROWS takes 0, 1 or 2");
+            if (value == 1 && !umma_available())
+                return fail(EE_EINVAL, "the tcgen05 projections are not available on this device");
             c->use_rows = value != 0;
+            c->rows.umma = value == 1 ? 1 : 0;
             return EE_OK;
         case EE_OPT_LAZY_FILL:
             if (c->lazy_fill == (value != 0)) return EE_OK;

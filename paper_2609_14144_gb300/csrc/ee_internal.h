@@ -254,14 +254,16 @@ constexpr int kRowsMax = 64;             // positions per batch
 constexpr int kRowsTargetUnits = 2432;   // (tile, K split) units a projection aims for: 152 SMs x 16 warps
 struct RowsBuf {
     float* H;           // [kRowsMax][d] residual of each row
-    uint16_t* xhi;      // [kRowsMax][ldx] next product's input, bf16 high part
-    uint16_t* xmid;     // [kRowsMax][ldx] middle part: x - high, rounded
-    uint16_t* xlo;      // [kRowsMax][ldx] low part: x - high - middle, rounded
+    uint16_t* x3;       // next product's input as three bf16 parts (high, x - high, the rest),
+                        // chunk-major: [ldx / 8][3][kRowsMax][8]
     float* Q;           // [kRowsMax][A D] rotated queries
     float* part;        // split partials [S][M][n_rows padded to 32]
     int32_t* pos;       // [kRowsMax] positions of a prompt batch
     int64_t part_floats;
     int ldx;
+    int umma;           // 1: projections on the tcgen05 tensor cores (ee_umma.cu), 0: warp-level mma
+    int n_sm;
+    int* err;           // device error word
 };
 // Splits along K of an n_tiles x K projection for a batch of M rows.
 int rows_splits(int64_t n_tiles, int K, int M);
@@ -274,6 +276,14 @@ int64_t rows_part_floats(int d, int A, int KH, int D, int F);
 // the last layer stops after its cache entries.
 cudaError_t rows_pass(const DevModel& m, const RowsBuf& b, const int* start, int M, int32_t* d_pos,
                       const int32_t* ids, int pos_base, bool kv_only, cudaStream_t s);
+// tcgen05 projections of the multi-position pass (ee_umma.cu): available on
+// this device (tensor-map encoding and the kernel's shared memory), the K
+// splits for n_sm SMs, and one projection into part[S][M][Np] (the layout of
+// the warp-level path).
+bool umma_available();
+int umma_splits(int64_t n_tiles, int K, int n_sm);
+cudaError_t launch_mm_umma(const uint16_t* W, int64_t n_rows, int K, const uint16_t* x3, int M, int S, float* part,
+                           int Np, int* err, cudaStream_t s);
 // After a batched prompt: the control block as the per-position prefill
 // leaves it before its LM head (position n).
 cudaError_t launch_rows_prefill_done(const DevModel& m, int n, cudaStream_t s);

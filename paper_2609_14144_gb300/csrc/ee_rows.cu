@@ -52,22 +52,31 @@ __device__ __forceinline__ uint16_t r_f2bf(float f) { return __bfloat16_as_ushor
 __device__ __forceinline__ float r_lo(uint32_t u) { return __uint_as_float(u << 16); }
 __device__ __forceinline__ float r_hi(uint32_t u) { return __uint_as_float(u & 0xffff0000u); }
 
-// The three bf16 part arrays of a product's input (same layout each).
+// A product's input as three bf16 parts, stored chunk-major: for each
+// 16-byte column chunk (8 columns), the high parts of the kRowsMax rows, then
+// the middle parts, then the low parts, 16 bytes per row.  Eight chunks are
+// then one contiguous block in the tensor cores' canonical operand layout
+// (ee_umma.cu), and a warp-level product reads a row's chunk of one part as
+// 16 contiguous bytes.
 struct Parts {
-    uint16_t *hi, *mid, *lo;
+    uint16_t* p;
 };
+__device__ __forceinline__ int64_t x3_index(int part, int row, int col) {
+    return ((int64_t)((col >> 3) * 3 + part) * kRowsMax + row) * 8 + (col & 7);
+}
 
-// The three bf16 parts of x at element `at` of each part array: high =
-// bf16(x), middle = bf16(x - high), low = bf16(x - high - middle) (each
-// difference exact in fp32).
-__device__ __forceinline__ void split_store(float x, const Parts& p, int64_t at) {
+// The three bf16 parts of x at (row, col): high = bf16(x), middle = bf16(x -
+// high), low = bf16(x - high - middle) (each difference exact in fp32).
+__device__ __forceinline__ void split_store(float x, const Parts& p, int row, int col) {
     const uint16_t h = r_f2bf(x);
     const float r1 = x - r_bf2f(h);
     const uint16_t md = r_f2bf(r1);
-    p.hi[at] = h;
-    p.mid[at] = md;
-    p.lo[at] = r_f2bf(r1 - r_bf2f(md));
+    p.p[x3_index(0, row, col)] = h;
+    p.p[x3_index(1, row, col)] = md;
+    p.p[x3_index(2, row, col)] = r_f2bf(r1 - r_bf2f(md));
 }
+// Columns from n up to the next multiple of 64 (a tensor-core stage) read as 0.
+__host__ __device__ __forceinline__ int pad64(int n) { return (n + 63) & ~63; }
 
 // Weights are read once per batch: streamed past L1, first out of L2.
 __device__ __forceinline__ uint4 ld_weights(const uint4* p) {
@@ -110,7 +119,7 @@ __device__ __forceinline__ int64_t slot_offset(const DevModel& m, int j, int pos
 // ------------------------------------------------------------------ projection
 //
 // part[s][row][n] = sum over the k of split s of W[n][k] x[row][k], for the
-// M rows of x (three bf16 parts, row stride ldx) and every output n of
+// M rows of x (three bf16 parts, chunk-major) and every output n of
 // the tiled weights.  A unit is (tile, split, row group): NB blocks of 8 rows
 // starting at row group * 8 NB (rows past M read as zero and are not
 // stored); the row groups of one (tile, split) are neighbouring warps, so a
@@ -152,10 +161,10 @@ __global__ void __launch_bounds__(kRowsThreads) k_rows_mm(const uint4* __restric
                 for (int n = 0; n < NB; ++n) {
                     const int row = r0 + n * 8 + g;
                     const bool okx = ok && row < M;
-                    const int64_t at = (int64_t)row * ldx + ch * 8;
-                    bh[v][n] = okx ? ld_act(x3.hi + at) : make_uint4(0u, 0u, 0u, 0u);
-                    bm[v][n] = okx ? ld_act(x3.mid + at) : make_uint4(0u, 0u, 0u, 0u);
-                    bl[v][n] = okx ? ld_act(x3.lo + at) : make_uint4(0u, 0u, 0u, 0u);
+                    const uint16_t* at = x3.p + x3_index(0, okx ? row : 0, ch * 8);
+                    bh[v][n] = okx ? ld_act(at) : make_uint4(0u, 0u, 0u, 0u);
+                    bm[v][n] = okx ? ld_act(at + kRowsMax * 8) : make_uint4(0u, 0u, 0u, 0u);
+                    bl[v][n] = okx ? ld_act(at + 2 * kRowsMax * 8) : make_uint4(0u, 0u, 0u, 0u);
                 }
             }
 #pragma unroll
@@ -248,10 +257,8 @@ __global__ void __launch_bounds__(kNormThreads) k_rows_add_norm(float* __restric
     if (!gain) return;  // uniform over the block
     ss = r_block_sum<kNormThreads>(ss, red);
     const float inv = 1.0f / sqrtf(ss / (float)d + eps);
-    for (int n = threadIdx.x; n < d; n += kNormThreads) {
-        const float x = h[n] * inv * r_bf2f(gain[n]);
-        split_store(x, x3, (int64_t)i * ldx + n);
-    }
+    for (int n = threadIdx.x; n < pad64(d); n += kNormThreads)
+        split_store(n < d ? h[n] * inv * r_bf2f(gain[n]) : 0.f, x3, i, n);
 }
 
 // Q/K/V of layer j for row blockIdx.y: thread = one unit (the packed row pair
@@ -300,11 +307,15 @@ __global__ void __launch_bounds__(kRowsThreads) k_rows_swiglu(const float* __res
                                                               int F, const Parts x3, int ldx) {
     const int i = blockIdx.y;
     const int f = blockIdx.x * kRowsThreads + threadIdx.x;
-    if (f >= F) return;
+    if (f >= pad64(F)) return;
+    if (f >= F) {
+        split_store(0.f, x3, i, f);
+        return;
+    }
     const float* p = part + (int64_t)i * Np + 2 * f;
     const float gs = split_sum(p, (int64_t)M * Np, S), us = split_sum(p + 1, (int64_t)M * Np, S);
     const float a = gs / (1.0f + expf(-gs)) * us;
-    split_store(a, x3, (int64_t)i * ldx + f);
+    split_store(a, x3, i, f);
 }
 
 // Starting residual of row blockIdx.x: the embedding of ids[i] (a prompt;
@@ -492,14 +503,16 @@ __global__ void __launch_bounds__(kRowsThreads) k_rows_attn(DevModel m, int j, c
     }
     for (int idx = tid; idx < G * D; idx += kRowsThreads) {
         const int h = idx / D, e = idx - h * D;
-        const int64_t col = (int64_t)(g * G + h) * D + e;
-        split_store(acc[idx] / lrun[h], x3, (int64_t)i * ldx + col);
+        const int col = (g * G + h) * D + e;
+        split_store(acc[idx] / lrun[h], x3, i, col);
     }
+    if (g == 0)  // the columns past A D up to the tensor cores' stage
+        for (int col = m.A * D + tid; col < pad64(m.A * D); col += kRowsThreads) split_store(0.f, x3, i, col);
 }
 
 // ------------------------------------------------------------------ host side
 
-Parts parts(const RowsBuf& b) { return Parts{b.xhi, b.xmid, b.xlo}; }
+Parts parts(const RowsBuf& b) { return Parts{b.x3}; }
 
 // Row blocks of 8 a warp takes (1, 2 or 4) and the row groups of a batch.
 void row_groups(int M, int& NB, int& RG) {
@@ -514,6 +527,13 @@ void row_groups(int M, int& NB, int& RG) {
 cudaError_t launch_mm(const uint16_t* W, int64_t n_rows, int K, const RowsBuf& b, int M, int& S, int& Np,
                       cudaStream_t s) {
     const int64_t nt = tile_count(n_rows);
+    if (b.umma) {
+        Np = (int)(nt * kTileRows);
+        S = umma_splits(nt, K, b.n_sm);
+        S = (int)std::max<int64_t>(1, std::min<int64_t>(S, b.part_floats / ((int64_t)M * Np)));
+        const cudaError_t e = launch_mm_umma(W, n_rows, K, b.x3, M, S, b.part, Np, b.err, s);
+        if (e != cudaErrorNotSupported) return e;
+    }
     int NB, RG;
     row_groups(M, NB, RG);
     S = rows_splits(nt, K, M);
@@ -604,8 +624,8 @@ cudaError_t rows_pass(const DevModel& m, const RowsBuf& b, const int* start, int
                                                      b.ldx);
         RCK(cudaGetLastError());
         RCK(launch_mm(lw + m.off_wgu, 2LL * m.F, d, b, Mj, S, Np, s));
-        k_rows_swiglu<<<dim3((m.F + kRowsThreads - 1) / kRowsThreads, Mj), kRowsThreads, 0, s>>>(b.part, S, Mj, Np, m.F,
-                                                                                                 parts(b), b.ldx);
+        k_rows_swiglu<<<dim3((pad64(m.F) + kRowsThreads - 1) / kRowsThreads, Mj), kRowsThreads, 0, s>>>(
+            b.part, S, Mj, Np, m.F, parts(b), b.ldx);
         RCK(cudaGetLastError());
         RCK(launch_mm(lw + m.off_wd, d, m.F, b, Mj, S, Np, s));
         M_prev = Mj;

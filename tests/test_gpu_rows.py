@@ -1,7 +1,8 @@
 """The multi-position layer pass on the GPU (needs a GB300).
 
 With EE_OPT_ROWS = 1 the prompt and the re-pass run each layer over batches
-of up to 64 positions.  Checked against the oracle (first token exact outside
+of up to 64 positions, the projections on the tcgen05 tensor cores (2: the
+same batches with warp-level mma products).  Checked against the oracle (first token exact outside
 the 1e-3 top-2 band, final hidden state and logits and every cache entry
 within 1e-2 relative, which (layer, position) entries were computed bit for
 bit) and against the same engine one position at a time (EE_OPT_ROWS = 0,
@@ -45,14 +46,16 @@ def _engine(shape, model, max_ctx, rows=True, pages=None):
     return eng
 
 
+@pytest.mark.parametrize("mode", [1, 2])
 @pytest.mark.parametrize("n", [1, 7, 64, 65, 150])
-def test_tiny_prompt_batches_match_oracle(tiny_model, n):
+def test_tiny_prompt_batches_match_oracle(tiny_model, n, mode):
     """Prompts of one position, one partial batch, one full batch, a full
-    batch and one position, and two full batches and a ragged tail."""
+    batch and one position, and two full batches and a ragged tail, on the
+    tcgen05 and the warp-level products (F = 688: a ragged last K stage)."""
     prompt = synth.token_ids(TINY.seed, 901, n, TINY.vocab)
     orc = oracle.Oracle(TINY, tiny_model, max_ctx=n + 1)
     tok_o, cap = orc.prefill(prompt, capture=True)
-    eng = _engine(TINY, tiny_model, n + 1)
+    eng = _engine(TINY, tiny_model, n + 1, rows=mode)
     tok_g = eng.prefill(prompt)
     if _top2_gap(cap["final_logits"]) >= EXCLUDE_EPS:
         assert tok_g == tok_o
@@ -176,3 +179,25 @@ def test_1p5b_prompt_batches_sampled():
             kg, vg = eng.kv(j, t)
             assert eng.kv_src(j, t) == so == 1
             assert rel_err(kg, ko) <= REL_TOL and rel_err(vg, vo) <= REL_TOL, (j, t)
+
+
+@pytest.mark.parametrize("name", ["0.5b", "1.5b"])
+def test_tensor_core_paths_agree(name):
+    """The tcgen05 products (EE_OPT_ROWS = 1) against the warp-level ones
+    (2) on a 64-position batch and a 36-position one: same first token,
+    fp32 states within 1e-3, cache entries within 1e-2 (bf16 rounding)."""
+    shape = synth.CONFIGS[name].replace(prompt_len=100)
+    model = synth.make_model(shape)
+    prompt = synth.prompt(shape)
+    a = _engine(shape, model, 101, rows=1)
+    b = _engine(shape, model, 101, rows=2)
+    ta, tb = a.prefill(prompt), b.prefill(prompt)
+    if _top2_gap(b.final_logits()) >= EXCLUDE_EPS:
+        assert ta == tb
+    assert rel_err(a.hidden_final(), b.hidden_final()) <= PATH_TOL
+    assert rel_err(a.final_logits(), b.final_logits()) <= PATH_TOL
+    for j in (0, shape.n_layers // 2, shape.n_layers - 1):
+        for t in (0, 31, 63, 64, 99):
+            ka, va = a.kv(j, t)
+            kb, vb = b.kv(j, t)
+            assert rel_err(ka, kb) <= REL_TOL and rel_err(va, vb) <= REL_TOL, (j, t)
