@@ -275,9 +275,10 @@ int ee_position(ee_ctx* ctx, int32_t* pos);
                                  bits), the projections on the tcgen05 tensor
                                  cores with TMA-staged operands (EE_EINVAL
                                  where unavailable); 2: the same batches with
-                                 warp-level mma products; 0 (default): one
-                                 position at a time through the decode
-                                 step's layer kernels (fp32 activations)    */
+                                 warp-level mma products; 0: one position
+                                 at a time through the decode step's layer
+                                 kernels (fp32 activations).  Default: 1
+                                 where the tcgen05 path is available, else 0 */
 #define EE_OPT_WAIT_LIMIT 9    /* for testing the failure path: the bound, in SM
                                  clock cycles, on each wait of the persistent
                                  layer kernel (ring stages, values from other

@@ -868,10 +868,13 @@ int ee_create(const ee_model_config* cfg, void* d_workspace, size_t workspace_by
     c->rows.ldx = l.rows_ldx;
     c->rows.n_sm = c->n_sm;
     c->rows.err = &c->d_ctl->err;
-    c->rows.umma = 0;
+    // prompts and re-passes in batches on the tcgen05 tensor cores where available
+    c->rows.umma = umma_available() ? 1 : 0;
+    c->use_rows = c->rows.umma == 1;
 
     const int kmax = std::max({2 * m.d, m.A * m.D, m.F});
-    if (configure_kernels(kmax) != cudaSuccess || configure_fill_pending(m.d) != cudaSuccess)
+    if (configure_kernels(kmax) != cudaSuccess || configure_fill_pending(m.d) != cudaSuccess ||
+        configure_rows() != cudaSuccess)
         return bail(fail(EE_ECUDA, "kernel configuration failed"));
     c->attn_cluster = attention_cluster_size(m.D, m.KH);
     if (seg_plan(m, c->n_sm, c->seg) && configure_layers(c->seg.smem) == cudaSuccess &&

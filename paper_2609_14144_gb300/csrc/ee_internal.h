@@ -265,6 +265,8 @@ struct RowsBuf {
     int n_sm;
     int* err;           // device error word
 };
+// Shared-memory attributes of the multi-position pass's kernels.
+cudaError_t configure_rows();
 // Splits along K of an n_tiles x K projection for a batch of M rows.
 int rows_splits(int64_t n_tiles, int K, int M);
 // Floats of the partial buffer every batch size fits in.

@@ -110,6 +110,14 @@ __device__ __forceinline__ float r_warp_max(float v) {
     return v;
 }
 
+// Programmatic dependent launch: every kernel of the pass waits for its
+// predecessor's results first, then lets its successor launch, so that a
+// launch's setup overlaps the kernel before it.
+__device__ __forceinline__ void r_pdl() {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 __device__ __forceinline__ int64_t slot_offset(const DevModel& m, int j, int pos) {
     const int page = m.page_table[pos / m.page_size];
     const int slot = pos - (pos / m.page_size) * m.page_size;
@@ -130,6 +138,7 @@ template <int NB, int U>
 __global__ void __launch_bounds__(kRowsThreads) k_rows_mm(const uint4* __restrict__ W, int n_tiles, int K,
                                                           const Parts x3, int ldx, int M, int S,
                                                           int RG, float* __restrict__ part, int Np) {
+    r_pdl();
     const int lane = threadIdx.x & 31, g = lane >> 2, q = lane & 3;
     const int Rc = K >> 3;             // 16-byte chunks per weight row
     const int nsteps = (Rc + 3) >> 2;  // 32-column steps
@@ -242,6 +251,7 @@ __global__ void __launch_bounds__(kNormThreads) k_rows_add_norm(float* __restric
                                                                 const float* __restrict__ part, int S, int M_add,
                                                                 int Np, const uint16_t* __restrict__ gain, float eps,
                                                                 const Parts x3, int ldx) {
+    r_pdl();
     __shared__ float red[kNormThreads / 32];
     const int i = blockIdx.x;
     float* h = H + (int64_t)i * d;
@@ -267,6 +277,7 @@ __global__ void __launch_bounds__(kNormThreads) k_rows_add_norm(float* __restric
 __global__ void __launch_bounds__(kRowsThreads) k_rows_qkv(DevModel m, int j, const float* __restrict__ part,
                                                            int S, int M, int Np, const int32_t* __restrict__ pos,
                                                            float* __restrict__ Q) {
+    r_pdl();
     const int i = blockIdx.y;
     const int u = blockIdx.x * kRowsThreads + threadIdx.x;
     const int half = m.D >> 1;
@@ -305,6 +316,7 @@ __global__ void __launch_bounds__(kRowsThreads) k_rows_qkv(DevModel m, int j, co
 // packed (gate, up) row pair, as three bf16 parts.
 __global__ void __launch_bounds__(kRowsThreads) k_rows_swiglu(const float* __restrict__ part, int S, int M, int Np,
                                                               int F, const Parts x3, int ldx) {
+    r_pdl();
     const int i = blockIdx.y;
     const int f = blockIdx.x * kRowsThreads + threadIdx.x;
     if (f >= pad64(F)) return;
@@ -323,6 +335,7 @@ __global__ void __launch_bounds__(kRowsThreads) k_rows_swiglu(const float* __res
 // position exited with.
 __global__ void __launch_bounds__(kRowsThreads) k_rows_init(DevModel m, float* __restrict__ H, int32_t* pos,
                                                             const int32_t* __restrict__ ids, int pos_base) {
+    r_pdl();
     const int i = blockIdx.x;
     float* h = H + (int64_t)i * m.d;
     if (ids) {
@@ -341,6 +354,7 @@ __global__ void __launch_bounds__(kRowsThreads) k_rows_init(DevModel m, float* _
 }
 
 __global__ void k_rows_prefill_done(DevModel m, int n) {
+    r_pdl();
     if (threadIdx.x != 0) return;
     Ctl* c = m.ctl;
     c->pos = n;
@@ -364,8 +378,11 @@ template <int D>
 __global__ void __launch_bounds__(kRowsThreads) k_rows_attn(DevModel m, int j, const float* __restrict__ Q,
                                                             const int32_t* __restrict__ pos, const Parts x3,
                                                             int ldx) {
+    r_pdl();
     constexpr int kG = kSegMaxGroup;  // query heads per kv head (at most)
     constexpr int DL = D / 32;        // dimensions per lane in the value sums
+    constexpr int CPR = D / 8;        // 16-byte chunks of a key row
+    extern __shared__ uint4 ksm[];    // [kKeysPerChunk][CPR + 1]
     __shared__ float qs[kG * D];
     __shared__ float ps[kG * kKeysPerChunk];
     __shared__ int64_t offs[kKeysPerChunk];
@@ -393,14 +410,21 @@ __global__ void __launch_bounds__(kRowsThreads) k_rows_attn(DevModel m, int j, c
         const bool valid = t < T;
         const int64_t off = valid ? slot_offset(m, j, t) + head_off : 0;
         offs[tid] = off;
+        __syncthreads();
+        // the chunk's key rows into shared memory, consecutive threads along a
+        // row (coalesced), rows padded by 16 bytes (conflict-free row reads)
+        for (int e = tid; e < kKeysPerChunk * CPR; e += kRowsThreads) {
+            const int r = e / CPR, c = e - r * CPR;
+            if (c0 + r < T) ksm[r * (CPR + 1) + c] = *reinterpret_cast<const uint4*>(m.kpool + offs[r] + c * 8);
+        }
+        __syncthreads();
         float sc[kG];
 #pragma unroll
         for (int h = 0; h < kG; ++h) sc[h] = 0.f;
         if (valid) {
-            const uint4* kr = reinterpret_cast<const uint4*>(m.kpool + off);
             uint4 kv[D / 8];
 #pragma unroll
-            for (int c = 0; c < D / 8; ++c) kv[c] = kr[c];
+            for (int c = 0; c < D / 8; ++c) kv[c] = ksm[tid * (CPR + 1) + c];
 #pragma unroll
             for (int c = 0; c < D / 8; ++c) {
                 const float kf[8] = {r_lo(kv[c].x), r_hi(kv[c].x), r_lo(kv[c].y), r_hi(kv[c].y),
@@ -512,7 +536,24 @@ __global__ void __launch_bounds__(kRowsThreads) k_rows_attn(DevModel m, int j, c
 
 // ------------------------------------------------------------------ host side
 
+template <class... KArgs, class... Args>
+cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s, Args... args) {
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+}
+
 Parts parts(const RowsBuf& b) { return Parts{b.x3}; }
+
+size_t attn_smem(int D) { return (size_t)kKeysPerChunk * (D / 8 + 1) * 16; }
 
 // Row blocks of 8 a warp takes (1, 2 or 4) and the row groups of a batch.
 void row_groups(int M, int& NB, int& RG) {
@@ -531,8 +572,7 @@ cudaError_t launch_mm(const uint16_t* W, int64_t n_rows, int K, const RowsBuf& b
         Np = (int)(nt * kTileRows);
         S = umma_splits(nt, K, b.n_sm);
         S = (int)std::max<int64_t>(1, std::min<int64_t>(S, b.part_floats / ((int64_t)M * Np)));
-        const cudaError_t e = launch_mm_umma(W, n_rows, K, b.x3, M, S, b.part, Np, b.err, s);
-        if (e != cudaErrorNotSupported) return e;
+        return launch_mm_umma(W, n_rows, K, b.x3, M, S, b.part, Np, b.err, s);
     }
     int NB, RG;
     row_groups(M, NB, RG);
@@ -542,12 +582,14 @@ cudaError_t launch_mm(const uint16_t* W, int64_t n_rows, int K, const RowsBuf& b
     const int grid = (int)std::min<int64_t>((units + kRowsWarps - 1) / kRowsWarps, 65535);
     const uint4* w = reinterpret_cast<const uint4*>(W);
     if (NB == 1)
-        k_rows_mm<1, 2><<<grid, kRowsThreads, 0, s>>>(w, (int)nt, K, parts(b), b.ldx, M, S, RG, b.part, Np);
+        return launch_pdl(k_rows_mm<1, 2>, dim3(grid), dim3(kRowsThreads), 0, s, w, (int)nt, K, parts(b), b.ldx, M, S, RG,
+                          b.part, Np);
     else if (NB == 2)
-        k_rows_mm<2, 2><<<grid, kRowsThreads, 0, s>>>(w, (int)nt, K, parts(b), b.ldx, M, S, RG, b.part, Np);
+        return launch_pdl(k_rows_mm<2, 2>, dim3(grid), dim3(kRowsThreads), 0, s, w, (int)nt, K, parts(b), b.ldx, M, S, RG,
+                          b.part, Np);
     else
-        k_rows_mm<4, 1><<<grid, kRowsThreads, 0, s>>>(w, (int)nt, K, parts(b), b.ldx, M, S, RG, b.part, Np);
-    return cudaGetLastError();
+        return launch_pdl(k_rows_mm<4, 1>, dim3(grid), dim3(kRowsThreads), 0, s, w, (int)nt, K, parts(b), b.ldx, M, S, RG,
+                          b.part, Np);
 }
 
 }  // namespace
@@ -568,6 +610,14 @@ int rows_splits(int64_t n_tiles, int K, int M) {
     S = std::min(S, std::max(1, K / ((NB == 4 ? 2 : 4) * Mp)));
     S = std::min(S, nsteps);
     return std::max(S, 1);
+}
+
+cudaError_t configure_rows() {
+    cudaError_t e = cudaFuncSetAttribute(k_rows_attn<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)attn_smem(128));
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(k_rows_attn<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)attn_smem(64));
+    return e;
 }
 
 int64_t rows_part_floats(int d, int A, int KH, int D, int F) {
@@ -596,8 +646,7 @@ cudaError_t rows_pass(const DevModel& m, const RowsBuf& b, const int* start, int
         if (start[i] < start[i - 1]) return cudaErrorInvalidValue;
     const int L = m.L, d = m.d, AD = m.A * m.D;
     const int64_t nqkv = (int64_t)(m.A + 2 * m.KH) * m.D;
-    k_rows_init<<<M, kRowsThreads, 0, s>>>(m, b.H, d_pos, ids, pos_base);
-    RCK(cudaGetLastError());
+    RCK(launch_pdl(k_rows_init, dim3(M), dim3(kRowsThreads), 0, s, m, b.H, d_pos, ids, pos_base));
     int M_prev = 0, S_prev = 1, Np_prev = 0;
     for (int j = start[0]; j < L; ++j) {
         int Mj = M_prev;
@@ -605,42 +654,37 @@ cudaError_t rows_pass(const DevModel& m, const RowsBuf& b, const int* start, int
         const uint16_t* lw = m.layers + (int64_t)j * m.layer_stride;
         int S = 1, Np = 0;
         // the previous layer's down projection into the residual, this layer's input norm
-        k_rows_add_norm<<<Mj, kNormThreads, 0, s>>>(b.H, d, b.part, S_prev, M_prev, Np_prev, lw + m.off_gattn, m.eps,
-                                                     parts(b), b.ldx);
-        RCK(cudaGetLastError());
+        RCK(launch_pdl(k_rows_add_norm, dim3(Mj), dim3(kNormThreads), 0, s, b.H, d, (const float*)b.part, S_prev, M_prev,
+                       Np_prev, lw + m.off_gattn, m.eps, parts(b), b.ldx));
         RCK(launch_mm(lw + m.off_wqkv, nqkv, d, b, Mj, S, Np, s));
         const int nu = (int)(nqkv / 2);
-        k_rows_qkv<<<dim3((nu + kRowsThreads - 1) / kRowsThreads, Mj), kRowsThreads, 0, s>>>(m, j, b.part, S, Mj, Np,
-                                                                                             d_pos, b.Q);
-        RCK(cudaGetLastError());
+        RCK(launch_pdl(k_rows_qkv, dim3((nu + kRowsThreads - 1) / kRowsThreads, Mj), dim3(kRowsThreads), 0, s, m, j,
+                       (const float*)b.part, S, Mj, Np, (const int32_t*)d_pos, b.Q));
         if (kv_only && j == L - 1) return cudaSuccess;
         if (m.D == 128)
-            k_rows_attn<128><<<dim3(m.KH, Mj), kRowsThreads, 0, s>>>(m, j, b.Q, d_pos, parts(b), b.ldx);
+            RCK(launch_pdl(k_rows_attn<128>, dim3(m.KH, Mj), dim3(kRowsThreads), attn_smem(128), s, m, j,
+                           (const float*)b.Q, (const int32_t*)d_pos, parts(b), b.ldx));
         else
-            k_rows_attn<64><<<dim3(m.KH, Mj), kRowsThreads, 0, s>>>(m, j, b.Q, d_pos, parts(b), b.ldx);
-        RCK(cudaGetLastError());
+            RCK(launch_pdl(k_rows_attn<64>, dim3(m.KH, Mj), dim3(kRowsThreads), attn_smem(64), s, m, j,
+                           (const float*)b.Q, (const int32_t*)d_pos, parts(b), b.ldx));
         RCK(launch_mm(lw + m.off_wo, d, AD, b, Mj, S, Np, s));
-        k_rows_add_norm<<<Mj, kNormThreads, 0, s>>>(b.H, d, b.part, S, Mj, Np, lw + m.off_gmlp, m.eps, parts(b),
-                                                     b.ldx);
-        RCK(cudaGetLastError());
+        RCK(launch_pdl(k_rows_add_norm, dim3(Mj), dim3(kNormThreads), 0, s, b.H, d, (const float*)b.part, S, Mj, Np,
+                       lw + m.off_gmlp, m.eps, parts(b), b.ldx));
         RCK(launch_mm(lw + m.off_wgu, 2LL * m.F, d, b, Mj, S, Np, s));
-        k_rows_swiglu<<<dim3((pad64(m.F) + kRowsThreads - 1) / kRowsThreads, Mj), kRowsThreads, 0, s>>>(
-            b.part, S, Mj, Np, m.F, parts(b), b.ldx);
-        RCK(cudaGetLastError());
+        RCK(launch_pdl(k_rows_swiglu, dim3((pad64(m.F) + kRowsThreads - 1) / kRowsThreads, Mj), dim3(kRowsThreads), 0, s,
+                       (const float*)b.part, S, Mj, Np, m.F, parts(b), b.ldx));
         RCK(launch_mm(lw + m.off_wd, d, m.F, b, Mj, S, Np, s));
         M_prev = Mj;
         S_prev = S;
         Np_prev = Np;
     }
     // the last down projection into the residual (no norm)
-    k_rows_add_norm<<<M_prev, kNormThreads, 0, s>>>(b.H, d, b.part, S_prev, M_prev, Np_prev, nullptr, m.eps,
-                                                    parts(b), b.ldx);
-    return cudaGetLastError();
+    return launch_pdl(k_rows_add_norm, dim3(M_prev), dim3(kNormThreads), 0, s, b.H, d, (const float*)b.part, S_prev,
+                      M_prev, Np_prev, (const uint16_t*)nullptr, m.eps, parts(b), b.ldx);
 }
 
 cudaError_t launch_rows_prefill_done(const DevModel& m, int n, cudaStream_t s) {
-    k_rows_prefill_done<<<1, 32, 0, s>>>(m, n);
-    return cudaGetLastError();
+    return launch_pdl(k_rows_prefill_done, dim3(1), dim3(32), 0, s, m, n);
 }
 
 }  // namespace ee

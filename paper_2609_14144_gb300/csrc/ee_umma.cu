@@ -180,6 +180,9 @@ __global__ void __launch_bounds__(kUThreads, 1)
     __syncthreads();
     u_fence_after();
     const uint32_t tmem = *tmem_slot;
+    // the set-up above overlaps the previous kernel (programmatic launch)
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
     if (w == 0 && lane == 0) {
         // producer: stage i of this split, the ring reused once its MMAs are done
@@ -298,10 +301,12 @@ bool umma_available() {
     return ok == 1;
 }
 
+// K splits: as many as keep the grid within one wave (one CTA per SM: the
+// stages take most of the shared memory), at most one per stage.
 int umma_splits(int64_t n_tiles, int K, int n_sm) {
     const int64_t mt = (n_tiles + 3) / 4;
     const int nk = (K + kUKStage - 1) / kUKStage;
-    const int64_t want = (n_sm + mt - 1) / mt;
+    const int64_t want = n_sm / mt;
     return (int)std::max<int64_t>(1, std::min<int64_t>(want, nk));
 }
 
@@ -311,8 +316,17 @@ cudaError_t launch_mm_umma(const uint16_t* W, int64_t n_rows, int K, const uint1
     CUtensorMap map;
     if (!weight_map(&map, W, nt, K)) return cudaErrorNotSupported;
     const dim3 grid((unsigned)((nt + 3) / 4), (unsigned)S);
-    k_rows_umma<<<grid, kUThreads, umma_smem(), s>>>(map, x3, (int)nt, K, M, S, part, Np, err);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = grid;
+    cfg.blockDim = dim3(kUThreads);
+    cfg.dynamicSmemBytes = umma_smem();
+    cfg.stream = s;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, k_rows_umma, map, x3, (int)nt, K, M, S, part, Np, err);
 }
 
 }  // namespace ee

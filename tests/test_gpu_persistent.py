@@ -116,9 +116,10 @@ def test_waits_that_run_out_report_a_stall_and_reset_recovers():
     prompt = synth.prompt(tiny)
     eng = Engine(tiny, model)
     assert eng.persistent
+    eng.prefill(prompt)
     eng.set_option(OPT_WAIT_LIMIT, 400)
     with pytest.raises(EEError) as e:
-        eng.prefill(prompt)
+        eng.decode_step(int(prompt[-1]), [0.5])
     assert e.value.code == -5 and "timed out" in str(e.value)
     eng.set_option(OPT_WAIT_LIMIT, 0)
     eng.reset()
