@@ -382,7 +382,8 @@ __global__ void __launch_bounds__(kRowsThreads) k_rows_attn(DevModel m, int j, c
     constexpr int kG = kSegMaxGroup;  // query heads per kv head (at most)
     constexpr int DL = D / 32;        // dimensions per lane in the value sums
     constexpr int CPR = D / 8;        // 16-byte chunks of a key row
-    extern __shared__ uint4 ksm[];    // [kKeysPerChunk][CPR + 1]
+    extern __shared__ uint4 ksm[];    // [kKeysPerChunk][CPR + 1] keys, then [kKeysPerChunk][CPR] values
+    uint4* vsm = ksm + kKeysPerChunk * (CPR + 1);
     __shared__ float qs[kG * D];
     __shared__ float ps[kG * kKeysPerChunk];
     __shared__ int64_t offs[kKeysPerChunk];
@@ -411,11 +412,17 @@ __global__ void __launch_bounds__(kRowsThreads) k_rows_attn(DevModel m, int j, c
         const int64_t off = valid ? slot_offset(m, j, t) + head_off : 0;
         offs[tid] = off;
         __syncthreads();
-        // the chunk's key rows into shared memory, consecutive threads along a
-        // row (coalesced), rows padded by 16 bytes (conflict-free row reads)
+        // the chunk's key and value rows into shared memory, consecutive
+        // threads along a row (coalesced); key rows padded by 16 bytes
+        // (conflict-free row reads), value rows past T zero
         for (int e = tid; e < kKeysPerChunk * CPR; e += kRowsThreads) {
             const int r = e / CPR, c = e - r * CPR;
-            if (c0 + r < T) ksm[r * (CPR + 1) + c] = *reinterpret_cast<const uint4*>(m.kpool + offs[r] + c * 8);
+            if (c0 + r < T) {
+                ksm[r * (CPR + 1) + c] = *reinterpret_cast<const uint4*>(m.kpool + offs[r] + c * 8);
+                vsm[r * CPR + c] = *reinterpret_cast<const uint4*>(m.vpool + offs[r] + c * 8);
+            } else {
+                vsm[r * CPR + c] = make_uint4(0u, 0u, 0u, 0u);
+            }
         }
         __syncthreads();
         float sc[kG];
@@ -484,7 +491,7 @@ __global__ void __launch_bounds__(kRowsThreads) k_rows_attn(DevModel m, int j, c
 #pragma unroll 8
         for (int kk = 0; kk < 32; ++kk) {
             const int tt = k0 + kk;
-            const uint16_t* vr = m.vpool + offs[tt] + lane * DL;
+            const uint16_t* vr = reinterpret_cast<const uint16_t*>(vsm + tt * CPR) + lane * DL;
             float v[DL];
             if constexpr (DL == 4) {
                 const uint2 u = *reinterpret_cast<const uint2*>(vr);
@@ -553,7 +560,7 @@ cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t sme
 
 Parts parts(const RowsBuf& b) { return Parts{b.x3}; }
 
-size_t attn_smem(int D) { return (size_t)kKeysPerChunk * (D / 8 + 1) * 16; }
+size_t attn_smem(int D) { return (size_t)kKeysPerChunk * (2 * (D / 8) + 1) * 16; }
 
 // Row blocks of 8 a warp takes (1, 2 or 4) and the row groups of a batch.
 void row_groups(int M, int& NB, int& RG) {
