@@ -637,7 +637,8 @@ int rows_repass(ee_ctx* c, const std::vector<int32_t>& todo, const std::vector<i
     for (int b0 = 0; b0 < n; b0 += kRowsMax) {
         const int M = std::min(kRowsMax, n - b0);
         const bool last = b0 + M == n;
-        EE_CK(rows_pass(m, c->rows, start.data() + b0, M, d_pos + b0, nullptr, 0, !last, s));
+        const int t_max = *std::max_element(pos.begin() + b0, pos.begin() + b0 + M) + 1;
+        EE_CK(rows_pass(m, c->rows, start.data() + b0, M, d_pos + b0, nullptr, 0, t_max, !last, s));
     }
     EE_CK(cudaMemcpyAsync(m.h, c->rows.H + (int64_t)last_row * m.d, 4 * (size_t)m.d, cudaMemcpyDeviceToDevice, s));
     EE_TRY(fetch_ctl(c));
@@ -654,7 +655,7 @@ int rows_prefill(ee_ctx* c, const int32_t* d_prompt, int n) {
     int last_row = 0;
     for (int b0 = 0; b0 < n; b0 += kRowsMax) {
         const int M = std::min(kRowsMax, n - b0);
-        EE_CK(rows_pass(m, c->rows, start.data(), M, c->rows.pos, d_prompt + b0, b0, b0 + M < n, s));
+        EE_CK(rows_pass(m, c->rows, start.data(), M, c->rows.pos, d_prompt + b0, b0, b0 + M, b0 + M < n, s));
         last_row = M - 1;
     }
     EE_CK(cudaMemcpyAsync(m.h, c->rows.H + (int64_t)last_row * m.d, 4 * (size_t)m.d, cudaMemcpyDeviceToDevice, s));

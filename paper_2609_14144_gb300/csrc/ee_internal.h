@@ -274,10 +274,11 @@ int64_t rows_part_floats(int d, int A, int KH, int D, int F);
 // Run layers over M rows at the device positions d_pos (ascending layer
 // start): row i starts at layer start[i] (host, non-decreasing).  With ids,
 // rows take the embedding of ids[i] and positions pos_base + i (written to
-// d_pos); otherwise each row starts from h_exit at its position.  kv_only:
-// the last layer stops after its cache entries.
+// d_pos); otherwise each row starts from h_exit at its position.  t_max:
+// the largest position of the batch + 1.  kv_only: the last layer stops
+// after its cache entries.
 cudaError_t rows_pass(const DevModel& m, const RowsBuf& b, const int* start, int M, int32_t* d_pos,
-                      const int32_t* ids, int pos_base, bool kv_only, cudaStream_t s);
+                      const int32_t* ids, int pos_base, int t_max, bool kv_only, cudaStream_t s);
 // tcgen05 projections of the multi-position pass (ee_umma.cu): available on
 // this device (tensor-map encoding and the kernel's shared memory), the K
 // splits for n_sm SMs, and one projection into part[S][M][Np] (the layout of

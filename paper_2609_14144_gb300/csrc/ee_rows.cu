@@ -3,16 +3,18 @@
 // positions run each layer over a batch of up to kRowsMax positions, so a
 // weight byte is read once per batch instead of once per position.
 //
-// A layer is nine launches, each reading what the previous one wrote:
+// A layer is ten launches, each reading what the previous one wrote:
 //   k_rows_add_norm  residual add of the previous projection's split
 //                    partials (in a fixed order), then RMSNorm with the next
 //                    gain, written as three bf16 parts
 //   k_rows_mm        a projection: Y[row][n] = sum_k W[n][k] x[row][k]
 //   k_rows_qkv       split sum, bias, RoPE at each row's position; q kept in
 //                    fp32, k and v stored bf16 into the paged cache
-//   k_rows_attn      causal attention of every row over the cache up to its
-//                    position (rows of the batch at earlier positions were
-//                    written by k_rows_qkv of this layer)
+//   k_rows_fattn     causal attention of every row over the cache up to its
+//                    position on the tensor cores, keys split over CTAs
+//                    (rows of the batch at earlier positions were written by
+//                    k_rows_qkv of this layer); k_rows_amerge combines the
+//                    splits
 //   k_rows_mm (O), k_rows_add_norm (mid residual, MLP norm),
 //   k_rows_mm (gate/up), k_rows_swiglu, k_rows_mm (down)
 //
@@ -45,7 +47,6 @@ namespace {
 
 constexpr int kRowsThreads = 256;
 constexpr int kRowsWarps = kRowsThreads / 32;
-constexpr int kKeysPerChunk = kRowsThreads;  // attention: one key per thread per chunk
 
 __device__ __forceinline__ float r_bf2f(uint16_t b) { return __uint_as_float((uint32_t)b << 16); }
 __device__ __forceinline__ uint16_t r_f2bf(float f) { return __bfloat16_as_ushort(__float2bfloat16_rn(f)); }
@@ -366,179 +367,264 @@ __global__ void k_rows_prefill_done(DevModel m, int n) {
     c->nucleus_member = -1;
 }
 
-// Causal attention of row blockIdx.y and kv head blockIdx.x over cache
-// positions 0..pos[i] of layer j, for the head group's G query heads, in
-// chunks of one key per thread: scores q.k / sqrt(D) per thread, a running
-// maximum and sum per head, and the weighted values summed with each warp
-// taking its own 32 keys of the chunk (lane l owning dimensions
-// l*D/32 .. l*D/32 + D/32 - 1 of every head), rescaled whenever the maximum
-// grows; the warps' sums are added in warp order at the end (Section 2's
-// softmax attention).  Output o at column h*D + e as three bf16 parts.
+// ------------------------------------------------------------ flash attention
+//
+// Causal attention of the batch on the tensor cores, its keys split over
+// CTAs (flash-decoding over a prompt batch).  CTA (kv head g, key split s,
+// head z of the group) takes query head h = g G + z for all kRowsMax rows of
+// the batch (4 warps x 16 rows) against keys [s KC, (s + 1) KC) of the
+// layer's cache, in blocks of kFaKeys keys staged in shared memory:
+//   S = Q K^T as mma m16n8k16 with the query (scaled by 1/sqrt(D)) split into
+//     three bf16 parts (high + middle + low = q exactly), each multiplied
+//     with the bf16 keys into the same fp32 accumulators (exact products);
+//   keys past a row's position are masked (Section 2's causal softmax), and
+//     a running maximum and sum per row rescale the output as blocks pass;
+//   O += P V with the probabilities split into three bf16 parts the same
+//     way, the values read transposed from shared memory (ldmatrix.trans).
+// Each split writes its unnormalised output, maximum and sum per (row,
+// head); k_rows_amerge combines the splits of each row in split order and
+// writes the attention output as the O projection's three bf16 parts.
+constexpr int kFaWarps = 4;
+constexpr int kFaThreads = 32 * kFaWarps;
+constexpr int kFaKeys = 64;        // keys per shared-memory block
+constexpr int kFaMaxSplits = 32;   // key splits per batch (at most)
+
+__host__ __device__ constexpr int fa_ld(int D) { return D + 8; }  // padded row (bf16): conflict-free ldmatrix
+__host__ __device__ constexpr size_t fa_smem(int D) {
+    return (size_t)(kFaWarps * 3 * 16 + 2 * kFaKeys) * fa_ld(D) * 2;
+}
+
+__device__ __forceinline__ uint32_t fa_saddr(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+__device__ __forceinline__ void ldsm_x4(uint32_t a, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                 : "r"(a));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t a, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                 : "r"(a));
+}
+// Two floats as three packed bf16 parts (high, middle, low; the first float
+// in the low halves).
+__device__ __forceinline__ void fa_split2(float x0, float x1, uint32_t& hi, uint32_t& md, uint32_t& lo) {
+    const uint16_t h0 = r_f2bf(x0), h1 = r_f2bf(x1);
+    const float a0 = x0 - r_bf2f(h0), a1 = x1 - r_bf2f(h1);
+    const uint16_t m0 = r_f2bf(a0), m1 = r_f2bf(a1);
+    hi = (uint32_t)h0 | ((uint32_t)h1 << 16);
+    md = (uint32_t)m0 | ((uint32_t)m1 << 16);
+    lo = (uint32_t)r_f2bf(a0 - r_bf2f(m0)) | ((uint32_t)r_f2bf(a1 - r_bf2f(m1)) << 16);
+}
+
 template <int D>
-__global__ void __launch_bounds__(kRowsThreads) k_rows_attn(DevModel m, int j, const float* __restrict__ Q,
-                                                            const int32_t* __restrict__ pos, const Parts x3,
-                                                            int ldx) {
+__global__ void __launch_bounds__(kFaThreads) k_rows_fattn(DevModel m, int j, const float* __restrict__ Q,
+                                                           const int32_t* __restrict__ pos, int Mj, int KC,
+                                                           float* __restrict__ part) {
     r_pdl();
-    constexpr int kG = kSegMaxGroup;  // query heads per kv head (at most)
-    constexpr int DL = D / 32;        // dimensions per lane in the value sums
-    constexpr int CPR = D / 8;        // 16-byte chunks of a key row
-    extern __shared__ uint4 ksm[];    // [kKeysPerChunk][CPR + 1] keys, then [kKeysPerChunk][CPR] values
-    uint4* vsm = ksm + kKeysPerChunk * (CPR + 1);
-    __shared__ float qs[kG * D];
-    __shared__ float ps[kG * kKeysPerChunk];
-    __shared__ int64_t offs[kKeysPerChunk];
-    __shared__ float redm[kRowsWarps][kG], reds[kRowsWarps][kG];
-    __shared__ float mrun[kG], lrun[kG], resc[kG];
-    const int g = blockIdx.x, i = blockIdx.y, G = m.A / m.KH;
-    const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
-    const int T = pos[i] + 1;
+    constexpr int LD = fa_ld(D);
+    constexpr int NT = D / 8;   // n8 tiles of the output
+    constexpr int KS = D / 16;  // k16 steps of a score
+    extern __shared__ __align__(16) uint16_t fsm[];
+    uint16_t* qs = fsm;                                // [warp][part][16][LD]
+    uint16_t* ks = qs + kFaWarps * 3 * 16 * LD;        // [kFaKeys][LD]
+    uint16_t* vs = ks + kFaKeys * LD;                  // [kFaKeys][LD]
+    const int g = blockIdx.x, s = blockIdx.y, G = m.A / m.KH, h = g * G + blockIdx.z;
+    const int tid = threadIdx.x, w = tid >> 5, lane = tid & 31, g8 = lane >> 2, t4 = lane & 3;
+    const int k0 = s * KC;
+    // rows of this warp, their positions (-1: not in the batch)
+    const int r0 = 16 * w + g8, r1 = r0 + 8;
+    const int p0 = r0 < Mj ? pos[r0] : -1, p1 = r1 < Mj ? pos[r1] : -1;
+    int pw = max(p0, p1);
+#pragma unroll
+    for (int o = 4; o < 32; o <<= 1) pw = max(pw, __shfl_xor_sync(0xffffffffu, pw, o));
+    // the CTA's last key: the largest position of the batch, within the split
+    int pc = -1;
+    for (int i = 0; i < Mj; ++i) pc = max(pc, pos[i]);
+    const int kend = min(k0 + KC, pc + 1);
+    const bool act = pw >= k0;  // this warp has a row with a key in the split
+    // the warp's queries, scaled, as three bf16 parts
     const float scale = 1.0f / sqrtf((float)D);
-    const float* qrow = Q + (int64_t)i * m.A * D + (int64_t)g * G * D;
-    for (int x = tid; x < G * D; x += kRowsThreads) qs[x] = qrow[x] * scale;
-    if (tid < kG) {
-        mrun[tid] = -INFINITY;
-        lrun[tid] = 0.f;
+    uint16_t* qw = qs + w * 3 * 16 * LD;
+    for (int e = lane; e < 16 * (D / 2); e += 32) {
+        const int r = e / (D / 2), c = 2 * (e - r * (D / 2)), i = 16 * w + r;
+        float x0 = 0.f, x1 = 0.f;
+        if (i < Mj) {
+            const float2 q = *reinterpret_cast<const float2*>(Q + (int64_t)i * m.A * D + (int64_t)h * D + c);
+            x0 = q.x * scale;
+            x1 = q.y * scale;
+        }
+        uint32_t hi, md, lo;
+        fa_split2(x0, x1, hi, md, lo);
+        *reinterpret_cast<uint32_t*>(qw + (0 * 16 + r) * LD + c) = hi;
+        *reinterpret_cast<uint32_t*>(qw + (1 * 16 + r) * LD + c) = md;
+        *reinterpret_cast<uint32_t*>(qw + (2 * 16 + r) * LD + c) = lo;
     }
-    float o[kG][DL];
+    float o[NT][4];
 #pragma unroll
-    for (int h = 0; h < kG; ++h)
-#pragma unroll
-        for (int x = 0; x < DL; ++x) o[h][x] = 0.f;
+    for (int n = 0; n < NT; ++n) o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.f;
+    float mr0 = -INFINITY, mr1 = -INFINITY, l0 = 0.f, l1 = 0.f;
     const int64_t head_off = (int64_t)g * m.page_size * D;
-    __syncthreads();
-    for (int c0 = 0; c0 < T; c0 += kKeysPerChunk) {
-        const int t = c0 + tid;
-        const bool valid = t < T;
-        const int64_t off = valid ? slot_offset(m, j, t) + head_off : 0;
-        offs[tid] = off;
-        __syncthreads();
-        // the chunk's key and value rows into shared memory, consecutive
-        // threads along a row (coalesced); key rows padded by 16 bytes
-        // (conflict-free row reads), value rows past T zero
-        for (int e = tid; e < kKeysPerChunk * CPR; e += kRowsThreads) {
-            const int r = e / CPR, c = e - r * CPR;
-            if (c0 + r < T) {
-                ksm[r * (CPR + 1) + c] = *reinterpret_cast<const uint4*>(m.kpool + offs[r] + c * 8);
-                vsm[r * CPR + c] = *reinterpret_cast<const uint4*>(m.vpool + offs[r] + c * 8);
-            } else {
-                vsm[r * CPR + c] = make_uint4(0u, 0u, 0u, 0u);
+    // ldmatrix row addresses: matrix q = lane / 8, row lane % 8
+    const int lq = lane >> 3, lr = lane & 7;
+    const uint32_t qa = fa_saddr(qw) + ((lq & 1) * 8 + lr) * LD * 2 + (lq >> 1) * 16;       // A: rows +8, cols +8
+    const uint32_t kb_a = fa_saddr(ks) + ((lq >> 1) * 8 + lr) * LD * 2 + (lq & 1) * 16;     // B of K: keys +8, dims +8
+    const uint32_t vb_a = fa_saddr(vs) + ((lq & 1) * 8 + lr) * LD * 2 + (lq >> 1) * 16;     // B of V^T: keys +8, dims +8
+    for (int kb = k0; kb < kend; kb += kFaKeys) {
+        __syncthreads();  // the previous block's keys and values are consumed (and the queries stored)
+        // the block's key and value rows (keys past the last position read as zero)
+        for (int e = tid; e < kFaKeys * (D / 8); e += kFaThreads) {
+            const int r = e / (D / 8), c = e - r * (D / 8), t = kb + r;
+            uint4 kv = make_uint4(0u, 0u, 0u, 0u), vv = kv;
+            if (t < kend) {
+                const int64_t off = slot_offset(m, j, t) + head_off + c * 8;
+                kv = *reinterpret_cast<const uint4*>(m.kpool + off);
+                vv = *reinterpret_cast<const uint4*>(m.vpool + off);
             }
+            *reinterpret_cast<uint4*>(ks + r * LD + c * 8) = kv;
+            *reinterpret_cast<uint4*>(vs + r * LD + c * 8) = vv;
         }
         __syncthreads();
-        float sc[kG];
+        if (!act || kb > pw) continue;
+        // scores of the warp's 16 rows against the block's 64 keys
+        float sc[8][4];
 #pragma unroll
-        for (int h = 0; h < kG; ++h) sc[h] = 0.f;
-        if (valid) {
-            uint4 kv[D / 8];
+        for (int n = 0; n < 8; ++n) sc[n][0] = sc[n][1] = sc[n][2] = sc[n][3] = 0.f;
 #pragma unroll
-            for (int c = 0; c < D / 8; ++c) kv[c] = ksm[tid * (CPR + 1) + c];
+        for (int kk = 0; kk < KS; ++kk) {
+            uint32_t a[3][4];
 #pragma unroll
-            for (int c = 0; c < D / 8; ++c) {
-                const float kf[8] = {r_lo(kv[c].x), r_hi(kv[c].x), r_lo(kv[c].y), r_hi(kv[c].y),
-                                     r_lo(kv[c].z), r_hi(kv[c].z), r_lo(kv[c].w), r_hi(kv[c].w)};
+            for (int pt = 0; pt < 3; ++pt)
+                ldsm_x4(qa + pt * 16 * LD * 2 + kk * 32, a[pt][0], a[pt][1], a[pt][2], a[pt][3]);
 #pragma unroll
-                for (int h = 0; h < kG; ++h) {
-                    if (h < G) {
-                        const float* qh = qs + h * D + c * 8;
-                        float a = sc[h];
+            for (int np = 0; np < 4; ++np) {
+                uint32_t b0, b1, b2, b3;
+                ldsm_x4(kb_a + np * 16 * LD * 2 + kk * 32, b0, b1, b2, b3);
 #pragma unroll
-                        for (int e = 0; e < 8; ++e) a = fmaf(qh[e], kf[e], a);
-                        sc[h] = a;
-                    }
+                for (int pt = 0; pt < 3; ++pt) {
+                    mma_16816(sc[2 * np], a[pt][0], a[pt][1], a[pt][2], a[pt][3], b0, b1);
+                    mma_16816(sc[2 * np + 1], a[pt][0], a[pt][1], a[pt][2], a[pt][3], b2, b3);
                 }
             }
         }
+        // causal mask, block maxima, rescale
+        float bm0 = -INFINITY, bm1 = -INFINITY;
 #pragma unroll
-        for (int h = 0; h < kG; ++h) {
-            if (h < G) {
-                sc[h] = valid ? sc[h] : -INFINITY;
-                const float mx = r_warp_max(sc[h]);
-                if (lane == 0) redm[w][h] = mx;
-            }
+        for (int n = 0; n < 8; ++n) {
+            const int t = kb + n * 8 + 2 * t4;
+            sc[n][0] = t <= p0 ? sc[n][0] : -INFINITY;
+            sc[n][1] = t + 1 <= p0 ? sc[n][1] : -INFINITY;
+            sc[n][2] = t <= p1 ? sc[n][2] : -INFINITY;
+            sc[n][3] = t + 1 <= p1 ? sc[n][3] : -INFINITY;
+            bm0 = fmaxf(bm0, fmaxf(sc[n][0], sc[n][1]));
+            bm1 = fmaxf(bm1, fmaxf(sc[n][2], sc[n][3]));
         }
-        __syncthreads();
-        if (tid < G) {
-            float cm = redm[0][tid];
-            for (int ww = 1; ww < kRowsWarps; ++ww) cm = fmaxf(cm, redm[ww][tid]);
-            const float mo = mrun[tid], mn = fmaxf(mo, cm);
-            resc[tid] = mo == -INFINITY ? 0.f : expf(mo - mn);
-            mrun[tid] = mn;
+        bm0 = fmaxf(bm0, __shfl_xor_sync(0xffffffffu, bm0, 1));
+        bm0 = fmaxf(bm0, __shfl_xor_sync(0xffffffffu, bm0, 2));
+        bm1 = fmaxf(bm1, __shfl_xor_sync(0xffffffffu, bm1, 1));
+        bm1 = fmaxf(bm1, __shfl_xor_sync(0xffffffffu, bm1, 2));
+        const float mn0 = fmaxf(mr0, bm0), mn1 = fmaxf(mr1, bm1);
+        // a row with no key yet keeps maximum -inf, probabilities 0
+        const float c0 = mn0 == -INFINITY ? 1.f : expf(mr0 - mn0);
+        const float c1 = mn1 == -INFINITY ? 1.f : expf(mr1 - mn1);
+        float s0 = 0.f, s1 = 0.f;
+#pragma unroll
+        for (int n = 0; n < 8; ++n) {
+            sc[n][0] = mn0 == -INFINITY ? 0.f : expf(sc[n][0] - mn0);
+            sc[n][1] = mn0 == -INFINITY ? 0.f : expf(sc[n][1] - mn0);
+            sc[n][2] = mn1 == -INFINITY ? 0.f : expf(sc[n][2] - mn1);
+            sc[n][3] = mn1 == -INFINITY ? 0.f : expf(sc[n][3] - mn1);
+            s0 += sc[n][0] + sc[n][1];
+            s1 += sc[n][2] + sc[n][3];
         }
-        __syncthreads();
+        s0 += __shfl_xor_sync(0xffffffffu, s0, 1);
+        s0 += __shfl_xor_sync(0xffffffffu, s0, 2);
+        s1 += __shfl_xor_sync(0xffffffffu, s1, 1);
+        s1 += __shfl_xor_sync(0xffffffffu, s1, 2);
+        l0 = l0 * c0 + s0;
+        l1 = l1 * c1 + s1;
+        mr0 = mn0;
+        mr1 = mn1;
 #pragma unroll
-        for (int h = 0; h < kG; ++h) {
-            if (h < G) {
-                const float p = valid ? expf(sc[h] - mrun[h]) : 0.f;
-                ps[h * kKeysPerChunk + tid] = p;
-                const float sum = r_warp_sum(p);
-                if (lane == 0) reds[w][h] = sum;
-            }
+        for (int n = 0; n < NT; ++n) {
+            o[n][0] *= c0;
+            o[n][1] *= c0;
+            o[n][2] *= c1;
+            o[n][3] *= c1;
         }
-        __syncthreads();
-        if (tid < G) {
-            float sum = 0.f;
-            for (int ww = 0; ww < kRowsWarps; ++ww) sum += reds[ww][tid];
-            lrun[tid] = lrun[tid] * resc[tid] + sum;
-        }
+        // O += P V over the block's keys, 16 at a time
 #pragma unroll
-        for (int h = 0; h < kG; ++h) {
-            const float r = h < G ? resc[h] : 0.f;
+        for (int kk = 0; kk < kFaKeys / 16; ++kk) {
+            uint32_t a[3][4];
+            fa_split2(sc[2 * kk][0], sc[2 * kk][1], a[0][0], a[1][0], a[2][0]);
+            fa_split2(sc[2 * kk][2], sc[2 * kk][3], a[0][1], a[1][1], a[2][1]);
+            fa_split2(sc[2 * kk + 1][0], sc[2 * kk + 1][1], a[0][2], a[1][2], a[2][2]);
+            fa_split2(sc[2 * kk + 1][2], sc[2 * kk + 1][3], a[0][3], a[1][3], a[2][3]);
 #pragma unroll
-            for (int x = 0; x < DL; ++x) o[h][x] *= r;
-        }
-        // this warp's keys of the chunk (invalid keys have p = 0 and offset 0)
-        const int k0 = w * 32;
-#pragma unroll 8
-        for (int kk = 0; kk < 32; ++kk) {
-            const int tt = k0 + kk;
-            const uint16_t* vr = reinterpret_cast<const uint16_t*>(vsm + tt * CPR) + lane * DL;
-            float v[DL];
-            if constexpr (DL == 4) {
-                const uint2 u = *reinterpret_cast<const uint2*>(vr);
-                v[0] = r_lo(u.x);
-                v[1] = r_hi(u.x);
-                v[2] = r_lo(u.y);
-                v[3] = r_hi(u.y);
-            } else {
-                const uint32_t u = *reinterpret_cast<const uint32_t*>(vr);
-                v[0] = r_lo(u);
-                v[1] = r_hi(u);
-            }
+            for (int np = 0; np < NT / 2; ++np) {
+                uint32_t b0, b1, b2, b3;
+                ldsm_x4_t(vb_a + kk * 16 * LD * 2 + np * 32, b0, b1, b2, b3);
 #pragma unroll
-            for (int h = 0; h < kG; ++h) {
-                if (h < G) {
-                    const float p = ps[h * kKeysPerChunk + tt];
-#pragma unroll
-                    for (int x = 0; x < DL; ++x) o[h][x] = fmaf(p, v[x], o[h][x]);
+                for (int pt = 0; pt < 3; ++pt) {
+                    mma_16816(o[2 * np], a[pt][0], a[pt][1], a[pt][2], a[pt][3], b0, b1);
+                    mma_16816(o[2 * np + 1], a[pt][0], a[pt][1], a[pt][2], a[pt][3], b2, b3);
                 }
             }
         }
-        __syncthreads();
     }
-    // add the warps' sums in warp order through shared memory (ps is free)
-    float* acc = ps;  // kG * D <= kG * kKeysPerChunk floats
-    for (int ww = 0; ww < kRowsWarps; ++ww) {
-        if (w == ww) {
+    if (!act) return;
+    // the split's unnormalised output, maximum and sum of each row:
+    // part[((s kRowsMax + row) A + h)][D + 2]
+    const int ld = D + 2;
+    float* q0 = part + ((int64_t)(s * kRowsMax + r0) * m.A + h) * ld;
+    float* q1 = part + ((int64_t)(s * kRowsMax + r1) * m.A + h) * ld;
 #pragma unroll
-            for (int h = 0; h < kG; ++h) {
-                if (h < G) {
-#pragma unroll
-                    for (int x = 0; x < DL; ++x) {
-                        float* a = acc + h * D + lane * DL + x;
-                        *a = ww == 0 ? o[h][x] : *a + o[h][x];
-                    }
-                }
-            }
+    for (int n = 0; n < NT; ++n) {
+        const int c = n * 8 + 2 * t4;
+        if (p0 >= 0) {
+            q0[c] = o[n][0];
+            q0[c + 1] = o[n][1];
         }
-        __syncthreads();
+        if (p1 >= 0) {
+            q1[c] = o[n][2];
+            q1[c + 1] = o[n][3];
+        }
     }
-    for (int idx = tid; idx < G * D; idx += kRowsThreads) {
-        const int h = idx / D, e = idx - h * D;
-        const int col = (g * G + h) * D + e;
-        split_store(acc[idx] / lrun[h], x3, i, col);
+    if (t4 == 0) {
+        if (p0 >= 0) {
+            q0[D] = mr0;
+            q0[D + 1] = l0;
+        }
+        if (p1 >= 0) {
+            q1[D] = mr1;
+            q1[D + 1] = l1;
+        }
     }
-    if (g == 0)  // the columns past A D up to the tensor cores' stage
-        for (int col = m.A * D + tid; col < pad64(m.A * D); col += kRowsThreads) split_store(0.f, x3, i, col);
+}
+
+// The splits of row i, head h (blockIdx.x = h, blockIdx.y = i; D threads):
+// o = sum_s exp(m_s - M) o_s / sum_s exp(m_s - M) l_s over the splits that
+// hold a key at or before the row's position, in split order; written as the
+// O projection's three bf16 parts at column h D + e.
+template <int D>
+__global__ void __launch_bounds__(D) k_rows_amerge(DevModel m, const float* __restrict__ part,
+                                                   const int32_t* __restrict__ pos, int KC, const Parts x3) {
+    r_pdl();
+    const int h = blockIdx.x, i = blockIdx.y, e = threadIdx.x;
+    const int ns = pos[i] / KC + 1, ld = D + 2;
+    const float* q = part + ((int64_t)i * m.A + h) * ld;
+    const int64_t step = (int64_t)kRowsMax * m.A * ld;  // one split
+    float M = -INFINITY;
+    for (int s = 0; s < ns; ++s) M = fmaxf(M, q[s * step + D]);
+    float num = 0.f, den = 0.f;
+    for (int s = 0; s < ns; ++s) {
+        const float* qs = q + s * step;
+        const float wgt = expf(qs[D] - M);
+        num = fmaf(wgt, qs[e], num);
+        den = fmaf(wgt, qs[D + 1], den);
+    }
+    split_store(num / den, x3, i, h * D + e);
+    if (h == 0)  // the columns past A D up to the tensor cores' stage
+        for (int col = m.A * D + e; col < pad64(m.A * D); col += D) split_store(0.f, x3, i, col);
 }
 
 // ------------------------------------------------------------------ host side
@@ -560,13 +646,47 @@ cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t sme
 
 Parts parts(const RowsBuf& b) { return Parts{b.x3}; }
 
-size_t attn_smem(int D) { return (size_t)kKeysPerChunk * (2 * (D / 8) + 1) * 16; }
+#define RCKA(x)                                   \
+    do {                                          \
+        cudaError_t e_ = (x);                     \
+        if (e_ != cudaSuccess) return e_;         \
+    } while (0)
 
 // Row blocks of 8 a warp takes (1, 2 or 4) and the row groups of a batch.
 void row_groups(int M, int& NB, int& RG) {
     const int blocks = (M + 7) / 8;
     NB = blocks <= 1 ? 1 : blocks <= 2 ? 2 : 4;
     RG = (blocks + NB - 1) / NB;
+}
+
+// Keys per split of the flash attention: a multiple of kFaKeys, large enough
+// that the splits of a batch whose last position is t_max - 1 number about
+// two CTAs per SM over the (kv head, query head) pairs, and at most
+// kFaMaxSplits.
+int fa_keys_per_split(int t_max, int n_heads, int n_sm) {
+    const int target = std::max(1, std::min(kFaMaxSplits, 2 * n_sm / std::max(1, n_heads)));
+    int kc = (t_max + target - 1) / target;
+    kc = std::max(kFaKeys, (kc + kFaKeys - 1) / kFaKeys * kFaKeys);
+    while ((t_max + kc - 1) / kc > kFaMaxSplits) kc += kFaKeys;
+    return kc;
+}
+
+// The batch's attention at layer j: the split kernel, then the merge into
+// the O projection's input parts.
+cudaError_t launch_attn(const DevModel& m, const RowsBuf& b, int j, int Mj, const int32_t* d_pos, int t_max,
+                        cudaStream_t s) {
+    const int KC = fa_keys_per_split(t_max, m.A, b.n_sm);
+    const int S = (t_max + KC - 1) / KC;
+    const dim3 grid(m.KH, S, m.A / m.KH);
+    if (m.D == 128) {
+        RCKA(launch_pdl(k_rows_fattn<128>, grid, dim3(kFaThreads), fa_smem(128), s, m, j, (const float*)b.Q, d_pos, Mj,
+                        KC, b.part));
+        return launch_pdl(k_rows_amerge<128>, dim3(m.A, Mj), dim3(128), 0, s, m, (const float*)b.part, d_pos, KC,
+                          parts(b));
+    }
+    RCKA(launch_pdl(k_rows_fattn<64>, grid, dim3(kFaThreads), fa_smem(64), s, m, j, (const float*)b.Q, d_pos, Mj, KC,
+                    b.part));
+    return launch_pdl(k_rows_amerge<64>, dim3(m.A, Mj), dim3(64), 0, s, m, (const float*)b.part, d_pos, KC, parts(b));
 }
 
 // One projection of the batch: W (n_rows x K, tiled) times the M rows of
@@ -620,10 +740,10 @@ int rows_splits(int64_t n_tiles, int K, int M) {
 }
 
 cudaError_t configure_rows() {
-    cudaError_t e = cudaFuncSetAttribute(k_rows_attn<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)attn_smem(128));
+    cudaError_t e = cudaFuncSetAttribute(k_rows_fattn<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)fa_smem(128));
     if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(k_rows_attn<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)attn_smem(64));
+        e = cudaFuncSetAttribute(k_rows_fattn<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)fa_smem(64));
     return e;
 }
 
@@ -636,7 +756,8 @@ int64_t rows_part_floats(int d, int A, int KH, int D, int F) {
             const int64_t nt = tile_count(rows[p]);
             most = std::max(most, (int64_t)rows_splits(nt, K[p], M) * M * nt * kTileRows);
         }
-    return most;
+    // the flash attention's split outputs: [kFaMaxSplits][kRowsMax][A][D + 2]
+    return std::max(most, (int64_t)kFaMaxSplits * kRowsMax * A * (D + 2));
 }
 
 #define RCK(x)                                    \
@@ -646,8 +767,9 @@ int64_t rows_part_floats(int d, int A, int KH, int D, int F) {
     } while (0)
 
 cudaError_t rows_pass(const DevModel& m, const RowsBuf& b, const int* start, int M, int32_t* d_pos,
-                      const int32_t* ids, int pos_base, bool kv_only, cudaStream_t s) {
+                      const int32_t* ids, int pos_base, int t_max, bool kv_only, cudaStream_t s) {
     if (M <= 0) return cudaSuccess;
+    if (t_max <= 0 || t_max > m.max_ctx) return cudaErrorInvalidValue;
     if (M > kRowsMax || start[0] < 0 || start[M - 1] >= m.L) return cudaErrorInvalidValue;
     for (int i = 1; i < M; ++i)
         if (start[i] < start[i - 1]) return cudaErrorInvalidValue;
@@ -668,12 +790,7 @@ cudaError_t rows_pass(const DevModel& m, const RowsBuf& b, const int* start, int
         RCK(launch_pdl(k_rows_qkv, dim3((nu + kRowsThreads - 1) / kRowsThreads, Mj), dim3(kRowsThreads), 0, s, m, j,
                        (const float*)b.part, S, Mj, Np, (const int32_t*)d_pos, b.Q));
         if (kv_only && j == L - 1) return cudaSuccess;
-        if (m.D == 128)
-            RCK(launch_pdl(k_rows_attn<128>, dim3(m.KH, Mj), dim3(kRowsThreads), attn_smem(128), s, m, j,
-                           (const float*)b.Q, (const int32_t*)d_pos, parts(b), b.ldx));
-        else
-            RCK(launch_pdl(k_rows_attn<64>, dim3(m.KH, Mj), dim3(kRowsThreads), attn_smem(64), s, m, j,
-                           (const float*)b.Q, (const int32_t*)d_pos, parts(b), b.ldx));
+        RCK(launch_attn(m, b, j, Mj, d_pos, t_max, s));
         RCK(launch_mm(lw + m.off_wo, d, AD, b, Mj, S, Np, s));
         RCK(launch_pdl(k_rows_add_norm, dim3(Mj), dim3(kNormThreads), 0, s, b.H, d, (const float*)b.part, S, Mj, Np,
                        lw + m.off_gmlp, m.eps, parts(b), b.ldx));
