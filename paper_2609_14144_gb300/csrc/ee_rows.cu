@@ -419,7 +419,7 @@ __device__ __forceinline__ void fa_split2(float x0, float x1, uint32_t& hi, uint
 template <int D>
 __global__ void __launch_bounds__(kFaThreads) k_rows_fattn(DevModel m, int j, const float* __restrict__ Q,
                                                            const int32_t* __restrict__ pos, int Mj, int KC,
-                                                           float* __restrict__ part) {
+                                                           int t_max, float* __restrict__ part) {
     r_pdl();
     constexpr int LD = fa_ld(D);
     constexpr int NT = D / 8;   // n8 tiles of the output
@@ -437,10 +437,8 @@ __global__ void __launch_bounds__(kFaThreads) k_rows_fattn(DevModel m, int j, co
     int pw = max(p0, p1);
 #pragma unroll
     for (int o = 4; o < 32; o <<= 1) pw = max(pw, __shfl_xor_sync(0xffffffffu, pw, o));
-    // the CTA's last key: the largest position of the batch, within the split
-    int pc = -1;
-    for (int i = 0; i < Mj; ++i) pc = max(pc, pos[i]);
-    const int kend = min(k0 + KC, pc + 1);
+    // the CTA's keys end at the split's end or past the batch's last position
+    const int kend = min(k0 + KC, t_max);
     const bool act = pw >= k0;  // this warp has a row with a key in the split
     // the warp's queries, scaled, as three bf16 parts
     const float scale = 1.0f / sqrtf((float)D);
@@ -680,12 +678,12 @@ cudaError_t launch_attn(const DevModel& m, const RowsBuf& b, int j, int Mj, cons
     const dim3 grid(m.KH, S, m.A / m.KH);
     if (m.D == 128) {
         RCKA(launch_pdl(k_rows_fattn<128>, grid, dim3(kFaThreads), fa_smem(128), s, m, j, (const float*)b.Q, d_pos, Mj,
-                        KC, b.part));
+                        KC, t_max, b.part));
         return launch_pdl(k_rows_amerge<128>, dim3(m.A, Mj), dim3(128), 0, s, m, (const float*)b.part, d_pos, KC,
                           parts(b));
     }
     RCKA(launch_pdl(k_rows_fattn<64>, grid, dim3(kFaThreads), fa_smem(64), s, m, j, (const float*)b.Q, d_pos, Mj, KC,
-                    b.part));
+                    t_max, b.part));
     return launch_pdl(k_rows_amerge<64>, dim3(m.A, Mj), dim3(64), 0, s, m, (const float*)b.part, d_pos, KC, parts(b));
 }
 

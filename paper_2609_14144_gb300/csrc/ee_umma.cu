@@ -45,7 +45,7 @@ namespace ee {
 namespace {
 
 constexpr int kUThreads = 128;
-constexpr int kUStages = 4;
+constexpr int kUStages = 5;
 constexpr int kUMRows = 128;                       // weight rows per CTA (UMMA M)
 constexpr int kUN = 3 * kRowsMax;                  // operand rows of the activations (UMMA N)
 constexpr int kUKStage = 64;                       // K columns per stage
