@@ -7,7 +7,7 @@
 //   k_rows_add_norm  residual add of the previous projection's split
 //                    partials (in a fixed order), then RMSNorm with the next
 //                    gain, written as three bf16 parts
-//   k_rows_mm        a projection: Y[row][n] = sum_k W[n][k] x[row][k]
+//   k_rows_umma / k_rows_mm   a projection: Y[row][n] = sum_k W[n][k] x[row][k]
 //   k_rows_qkv       split sum, bias, RoPE at each row's position; q kept in
 //                    fp32, k and v stored bf16 into the paged cache
 //   k_rows_fattn     causal attention of every row over the cache up to its
@@ -15,11 +15,12 @@
 //                    (rows of the batch at earlier positions were written by
 //                    k_rows_qkv of this layer); k_rows_amerge combines the
 //                    splits
-//   k_rows_mm (O), k_rows_add_norm (mid residual, MLP norm),
-//   k_rows_mm (gate/up), k_rows_swiglu, k_rows_mm (down)
+//   the O projection, k_rows_add_norm (mid residual, MLP norm), the gate/up
+//   projection, k_rows_swiglu, the down projection
 //
-// Projections use the legacy warp-level tensor-core mma (m16n8k16, bf16
-// operands, fp32 accumulation).  A warp owns one (32-row weight tile, K
+// Projections run on the tcgen05 tensor cores by default (k_rows_umma,
+// ee_umma.cu).  The warp-level build here (EE_OPT_ROWS = 2) uses the legacy
+// mma (m16n8k16, bf16 operands, fp32 accumulation).  A warp owns one (32-row weight tile, K
 // range) unit: the tiled weight layout gives each lane the 16-byte chunk of
 // one row, and the order of k inside one mma is free as long as both
 // operands agree, so a lane's chunk feeds its A fragment as loaded (slots
@@ -390,11 +391,15 @@ constexpr int kFaKeys = 64;        // keys per shared-memory block
 constexpr int kFaMaxSplits = 32;   // key splits per batch (at most)
 
 __host__ __device__ constexpr int fa_ld(int D) { return D + 8; }  // padded row (bf16): conflict-free ldmatrix
-__host__ __device__ constexpr size_t fa_smem(int D) {
-    return (size_t)(kFaWarps * 3 * 16 + 2 * kFaKeys) * fa_ld(D) * 2;
+__host__ __device__ constexpr size_t fa_smem(int D) {  // queries, then two blocks of keys and values
+    return (size_t)(kFaWarps * 3 * 16 + 4 * kFaKeys) * fa_ld(D) * 2;
 }
 
 __device__ __forceinline__ uint32_t fa_saddr(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+// 16 bytes global -> shared, asynchronously; the bytes past src_bytes (0 or 16) are zero.
+__device__ __forceinline__ void fa_cp16(uint32_t dst, const void* src, int src_bytes) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
+}
 __device__ __forceinline__ void ldsm_x4(uint32_t a, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
     asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
                  : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
@@ -426,148 +431,168 @@ __global__ void __launch_bounds__(kFaThreads) k_rows_fattn(DevModel m, int j, co
     constexpr int KS = D / 16;  // k16 steps of a score
     extern __shared__ __align__(16) uint16_t fsm[];
     uint16_t* qs = fsm;                                // [warp][part][16][LD]
-    uint16_t* ks = qs + kFaWarps * 3 * 16 * LD;        // [kFaKeys][LD]
-    uint16_t* vs = ks + kFaKeys * LD;                  // [kFaKeys][LD]
+    uint16_t* ks = qs + kFaWarps * 3 * 16 * LD;        // [2][kFaKeys][LD]
+    uint16_t* vs = ks + 2 * kFaKeys * LD;              // [2][kFaKeys][LD]
     const int g = blockIdx.x, s = blockIdx.y, G = m.A / m.KH, h = g * G + blockIdx.z;
     const int tid = threadIdx.x, w = tid >> 5, lane = tid & 31, g8 = lane >> 2, t4 = lane & 3;
     const int k0 = s * KC;
+    // the CTA's keys end at the split's end or past the batch's last position
+    const int kend = min(k0 + KC, t_max);
+    const int64_t head_off = (int64_t)g * m.page_size * D;
+    // A block of keys and values into buffer `buf`: cp.async, all of a
+    // thread's copies issued together; keys past kend read as zero.
+    auto load_block = [&](int kb, int buf) {
+        const uint32_t kd = fa_saddr(ks + buf * kFaKeys * LD), vd = fa_saddr(vs + buf * kFaKeys * LD);
+#pragma unroll
+        for (int u = 0; u < kFaKeys * (D / 8) / kFaThreads; ++u) {
+            const int e = tid + u * kFaThreads, r = e / (D / 8), c = e - r * (D / 8), t = kb + r;
+            const bool ok = t < kend;
+            const int64_t off = ok ? slot_offset(m, j, t) + head_off + c * 8 : 0;
+            fa_cp16(kd + (r * LD + c * 8) * 2, m.kpool + off, ok ? 16 : 0);
+            fa_cp16(vd + (r * LD + c * 8) * 2, m.vpool + off, ok ? 16 : 0);
+        }
+        asm volatile("cp.async.commit_group;" ::: "memory");
+    };
+    if (k0 < kend) load_block(k0, 0);
     // rows of this warp, their positions (-1: not in the batch)
     const int r0 = 16 * w + g8, r1 = r0 + 8;
     const int p0 = r0 < Mj ? pos[r0] : -1, p1 = r1 < Mj ? pos[r1] : -1;
     int pw = max(p0, p1);
 #pragma unroll
     for (int o = 4; o < 32; o <<= 1) pw = max(pw, __shfl_xor_sync(0xffffffffu, pw, o));
-    // the CTA's keys end at the split's end or past the batch's last position
-    const int kend = min(k0 + KC, t_max);
     const bool act = pw >= k0;  // this warp has a row with a key in the split
-    // the warp's queries, scaled, as three bf16 parts
+    // the warp's queries, scaled, as three bf16 parts (all loads issued first)
     const float scale = 1.0f / sqrtf((float)D);
     uint16_t* qw = qs + w * 3 * 16 * LD;
-    for (int e = lane; e < 16 * (D / 2); e += 32) {
-        const int r = e / (D / 2), c = 2 * (e - r * (D / 2)), i = 16 * w + r;
-        float x0 = 0.f, x1 = 0.f;
-        if (i < Mj) {
-            const float2 q = *reinterpret_cast<const float2*>(Q + (int64_t)i * m.A * D + (int64_t)h * D + c);
-            x0 = q.x * scale;
-            x1 = q.y * scale;
+    {
+        constexpr int QV = 16 * D / 4 / 32;  // float4 per lane
+        float4 qv[QV];
+#pragma unroll
+        for (int u = 0; u < QV; ++u) {
+            const int e = lane + 32 * u, r = e / (D / 4), c = 4 * (e - r * (D / 4)), i = 16 * w + r;
+            qv[u] = i < Mj ? *reinterpret_cast<const float4*>(Q + (int64_t)i * m.A * D + (int64_t)h * D + c)
+                           : make_float4(0.f, 0.f, 0.f, 0.f);
         }
-        uint32_t hi, md, lo;
-        fa_split2(x0, x1, hi, md, lo);
-        *reinterpret_cast<uint32_t*>(qw + (0 * 16 + r) * LD + c) = hi;
-        *reinterpret_cast<uint32_t*>(qw + (1 * 16 + r) * LD + c) = md;
-        *reinterpret_cast<uint32_t*>(qw + (2 * 16 + r) * LD + c) = lo;
+#pragma unroll
+        for (int u = 0; u < QV; ++u) {
+            const int e = lane + 32 * u, r = e / (D / 4), c = 4 * (e - r * (D / 4));
+            uint32_t h0, m0, l0_, h1, m1, l1_;
+            fa_split2(qv[u].x * scale, qv[u].y * scale, h0, m0, l0_);
+            fa_split2(qv[u].z * scale, qv[u].w * scale, h1, m1, l1_);
+            *reinterpret_cast<uint2*>(qw + (0 * 16 + r) * LD + c) = make_uint2(h0, h1);
+            *reinterpret_cast<uint2*>(qw + (1 * 16 + r) * LD + c) = make_uint2(m0, m1);
+            *reinterpret_cast<uint2*>(qw + (2 * 16 + r) * LD + c) = make_uint2(l0_, l1_);
+        }
     }
     float o[NT][4];
 #pragma unroll
     for (int n = 0; n < NT; ++n) o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.f;
     float mr0 = -INFINITY, mr1 = -INFINITY, l0 = 0.f, l1 = 0.f;
-    const int64_t head_off = (int64_t)g * m.page_size * D;
     // ldmatrix row addresses: matrix q = lane / 8, row lane % 8
     const int lq = lane >> 3, lr = lane & 7;
     const uint32_t qa = fa_saddr(qw) + ((lq & 1) * 8 + lr) * LD * 2 + (lq >> 1) * 16;       // A: rows +8, cols +8
-    const uint32_t kb_a = fa_saddr(ks) + ((lq >> 1) * 8 + lr) * LD * 2 + (lq & 1) * 16;     // B of K: keys +8, dims +8
-    const uint32_t vb_a = fa_saddr(vs) + ((lq & 1) * 8 + lr) * LD * 2 + (lq >> 1) * 16;     // B of V^T: keys +8, dims +8
-    for (int kb = k0; kb < kend; kb += kFaKeys) {
-        __syncthreads();  // the previous block's keys and values are consumed (and the queries stored)
-        // the block's key and value rows (keys past the last position read as zero)
-        for (int e = tid; e < kFaKeys * (D / 8); e += kFaThreads) {
-            const int r = e / (D / 8), c = e - r * (D / 8), t = kb + r;
-            uint4 kv = make_uint4(0u, 0u, 0u, 0u), vv = kv;
-            if (t < kend) {
-                const int64_t off = slot_offset(m, j, t) + head_off + c * 8;
-                kv = *reinterpret_cast<const uint4*>(m.kpool + off);
-                vv = *reinterpret_cast<const uint4*>(m.vpool + off);
+    const uint32_t kb_a0 = fa_saddr(ks) + ((lq >> 1) * 8 + lr) * LD * 2 + (lq & 1) * 16;    // B of K: keys +8, dims +8
+    const uint32_t vb_a0 = fa_saddr(vs) + ((lq & 1) * 8 + lr) * LD * 2 + (lq >> 1) * 16;    // B of V^T: keys +8, dims +8
+    int buf = 0;
+    for (int kb = k0; kb < kend; kb += kFaKeys, buf ^= 1) {
+        // the next block into the other buffer (free: every warp passed the
+        // barrier at the end of the previous block), then wait for this one
+        const bool next = kb + kFaKeys < kend;
+        if (next) load_block(kb + kFaKeys, buf ^ 1);
+        if (next)
+            asm volatile("cp.async.wait_group 1;" ::: "memory");
+        else
+            asm volatile("cp.async.wait_group 0;" ::: "memory");
+        __syncthreads();  // the block (and the queries) visible to every warp
+        const uint32_t kb_a = kb_a0 + buf * kFaKeys * LD * 2, vb_a = vb_a0 + buf * kFaKeys * LD * 2;
+        if (act && kb <= pw) {
+            // scores of the warp's 16 rows against the block's 64 keys
+            float sc[8][4];
+#pragma unroll
+            for (int n = 0; n < 8; ++n) sc[n][0] = sc[n][1] = sc[n][2] = sc[n][3] = 0.f;
+#pragma unroll
+            for (int kk = 0; kk < KS; ++kk) {
+                uint32_t a[3][4];
+#pragma unroll
+                for (int pt = 0; pt < 3; ++pt)
+                    ldsm_x4(qa + pt * 16 * LD * 2 + kk * 32, a[pt][0], a[pt][1], a[pt][2], a[pt][3]);
+#pragma unroll
+                for (int np = 0; np < 4; ++np) {
+                    uint32_t b0, b1, b2, b3;
+                    ldsm_x4(kb_a + np * 16 * LD * 2 + kk * 32, b0, b1, b2, b3);
+#pragma unroll
+                    for (int pt = 0; pt < 3; ++pt) {
+                        mma_16816(sc[2 * np], a[pt][0], a[pt][1], a[pt][2], a[pt][3], b0, b1);
+                        mma_16816(sc[2 * np + 1], a[pt][0], a[pt][1], a[pt][2], a[pt][3], b2, b3);
+                    }
+                }
             }
-            *reinterpret_cast<uint4*>(ks + r * LD + c * 8) = kv;
-            *reinterpret_cast<uint4*>(vs + r * LD + c * 8) = vv;
-        }
-        __syncthreads();
-        if (!act || kb > pw) continue;
-        // scores of the warp's 16 rows against the block's 64 keys
-        float sc[8][4];
+            // causal mask, block maxima, rescale
+            float bm0 = -INFINITY, bm1 = -INFINITY;
 #pragma unroll
-        for (int n = 0; n < 8; ++n) sc[n][0] = sc[n][1] = sc[n][2] = sc[n][3] = 0.f;
+            for (int n = 0; n < 8; ++n) {
+                const int t = kb + n * 8 + 2 * t4;
+                sc[n][0] = t <= p0 ? sc[n][0] : -INFINITY;
+                sc[n][1] = t + 1 <= p0 ? sc[n][1] : -INFINITY;
+                sc[n][2] = t <= p1 ? sc[n][2] : -INFINITY;
+                sc[n][3] = t + 1 <= p1 ? sc[n][3] : -INFINITY;
+                bm0 = fmaxf(bm0, fmaxf(sc[n][0], sc[n][1]));
+                bm1 = fmaxf(bm1, fmaxf(sc[n][2], sc[n][3]));
+            }
+            bm0 = fmaxf(bm0, __shfl_xor_sync(0xffffffffu, bm0, 1));
+            bm0 = fmaxf(bm0, __shfl_xor_sync(0xffffffffu, bm0, 2));
+            bm1 = fmaxf(bm1, __shfl_xor_sync(0xffffffffu, bm1, 1));
+            bm1 = fmaxf(bm1, __shfl_xor_sync(0xffffffffu, bm1, 2));
+            const float mn0 = fmaxf(mr0, bm0), mn1 = fmaxf(mr1, bm1);
+            // a row with no key yet keeps maximum -inf, probabilities 0
+            const float c0 = mn0 == -INFINITY ? 1.f : expf(mr0 - mn0);
+            const float c1 = mn1 == -INFINITY ? 1.f : expf(mr1 - mn1);
+            float s0 = 0.f, s1 = 0.f;
 #pragma unroll
-        for (int kk = 0; kk < KS; ++kk) {
-            uint32_t a[3][4];
+            for (int n = 0; n < 8; ++n) {
+                sc[n][0] = mn0 == -INFINITY ? 0.f : expf(sc[n][0] - mn0);
+                sc[n][1] = mn0 == -INFINITY ? 0.f : expf(sc[n][1] - mn0);
+                sc[n][2] = mn1 == -INFINITY ? 0.f : expf(sc[n][2] - mn1);
+                sc[n][3] = mn1 == -INFINITY ? 0.f : expf(sc[n][3] - mn1);
+                s0 += sc[n][0] + sc[n][1];
+                s1 += sc[n][2] + sc[n][3];
+            }
+            s0 += __shfl_xor_sync(0xffffffffu, s0, 1);
+            s0 += __shfl_xor_sync(0xffffffffu, s0, 2);
+            s1 += __shfl_xor_sync(0xffffffffu, s1, 1);
+            s1 += __shfl_xor_sync(0xffffffffu, s1, 2);
+            l0 = l0 * c0 + s0;
+            l1 = l1 * c1 + s1;
+            mr0 = mn0;
+            mr1 = mn1;
 #pragma unroll
-            for (int pt = 0; pt < 3; ++pt)
-                ldsm_x4(qa + pt * 16 * LD * 2 + kk * 32, a[pt][0], a[pt][1], a[pt][2], a[pt][3]);
+            for (int n = 0; n < NT; ++n) {
+                o[n][0] *= c0;
+                o[n][1] *= c0;
+                o[n][2] *= c1;
+                o[n][3] *= c1;
+            }
+            // O += P V over the block's keys, 16 at a time
 #pragma unroll
-            for (int np = 0; np < 4; ++np) {
-                uint32_t b0, b1, b2, b3;
-                ldsm_x4(kb_a + np * 16 * LD * 2 + kk * 32, b0, b1, b2, b3);
+            for (int kk = 0; kk < kFaKeys / 16; ++kk) {
+                uint32_t a[3][4];
+                fa_split2(sc[2 * kk][0], sc[2 * kk][1], a[0][0], a[1][0], a[2][0]);
+                fa_split2(sc[2 * kk][2], sc[2 * kk][3], a[0][1], a[1][1], a[2][1]);
+                fa_split2(sc[2 * kk + 1][0], sc[2 * kk + 1][1], a[0][2], a[1][2], a[2][2]);
+                fa_split2(sc[2 * kk + 1][2], sc[2 * kk + 1][3], a[0][3], a[1][3], a[2][3]);
 #pragma unroll
-                for (int pt = 0; pt < 3; ++pt) {
-                    mma_16816(sc[2 * np], a[pt][0], a[pt][1], a[pt][2], a[pt][3], b0, b1);
-                    mma_16816(sc[2 * np + 1], a[pt][0], a[pt][1], a[pt][2], a[pt][3], b2, b3);
+                for (int np = 0; np < NT / 2; ++np) {
+                    uint32_t b0, b1, b2, b3;
+                    ldsm_x4_t(vb_a + kk * 16 * LD * 2 + np * 32, b0, b1, b2, b3);
+#pragma unroll
+                    for (int pt = 0; pt < 3; ++pt) {
+                        mma_16816(o[2 * np], a[pt][0], a[pt][1], a[pt][2], a[pt][3], b0, b1);
+                        mma_16816(o[2 * np + 1], a[pt][0], a[pt][1], a[pt][2], a[pt][3], b2, b3);
+                    }
                 }
             }
         }
-        // causal mask, block maxima, rescale
-        float bm0 = -INFINITY, bm1 = -INFINITY;
-#pragma unroll
-        for (int n = 0; n < 8; ++n) {
-            const int t = kb + n * 8 + 2 * t4;
-            sc[n][0] = t <= p0 ? sc[n][0] : -INFINITY;
-            sc[n][1] = t + 1 <= p0 ? sc[n][1] : -INFINITY;
-            sc[n][2] = t <= p1 ? sc[n][2] : -INFINITY;
-            sc[n][3] = t + 1 <= p1 ? sc[n][3] : -INFINITY;
-            bm0 = fmaxf(bm0, fmaxf(sc[n][0], sc[n][1]));
-            bm1 = fmaxf(bm1, fmaxf(sc[n][2], sc[n][3]));
-        }
-        bm0 = fmaxf(bm0, __shfl_xor_sync(0xffffffffu, bm0, 1));
-        bm0 = fmaxf(bm0, __shfl_xor_sync(0xffffffffu, bm0, 2));
-        bm1 = fmaxf(bm1, __shfl_xor_sync(0xffffffffu, bm1, 1));
-        bm1 = fmaxf(bm1, __shfl_xor_sync(0xffffffffu, bm1, 2));
-        const float mn0 = fmaxf(mr0, bm0), mn1 = fmaxf(mr1, bm1);
-        // a row with no key yet keeps maximum -inf, probabilities 0
-        const float c0 = mn0 == -INFINITY ? 1.f : expf(mr0 - mn0);
-        const float c1 = mn1 == -INFINITY ? 1.f : expf(mr1 - mn1);
-        float s0 = 0.f, s1 = 0.f;
-#pragma unroll
-        for (int n = 0; n < 8; ++n) {
-            sc[n][0] = mn0 == -INFINITY ? 0.f : expf(sc[n][0] - mn0);
-            sc[n][1] = mn0 == -INFINITY ? 0.f : expf(sc[n][1] - mn0);
-            sc[n][2] = mn1 == -INFINITY ? 0.f : expf(sc[n][2] - mn1);
-            sc[n][3] = mn1 == -INFINITY ? 0.f : expf(sc[n][3] - mn1);
-            s0 += sc[n][0] + sc[n][1];
-            s1 += sc[n][2] + sc[n][3];
-        }
-        s0 += __shfl_xor_sync(0xffffffffu, s0, 1);
-        s0 += __shfl_xor_sync(0xffffffffu, s0, 2);
-        s1 += __shfl_xor_sync(0xffffffffu, s1, 1);
-        s1 += __shfl_xor_sync(0xffffffffu, s1, 2);
-        l0 = l0 * c0 + s0;
-        l1 = l1 * c1 + s1;
-        mr0 = mn0;
-        mr1 = mn1;
-#pragma unroll
-        for (int n = 0; n < NT; ++n) {
-            o[n][0] *= c0;
-            o[n][1] *= c0;
-            o[n][2] *= c1;
-            o[n][3] *= c1;
-        }
-        // O += P V over the block's keys, 16 at a time
-#pragma unroll
-        for (int kk = 0; kk < kFaKeys / 16; ++kk) {
-            uint32_t a[3][4];
-            fa_split2(sc[2 * kk][0], sc[2 * kk][1], a[0][0], a[1][0], a[2][0]);
-            fa_split2(sc[2 * kk][2], sc[2 * kk][3], a[0][1], a[1][1], a[2][1]);
-            fa_split2(sc[2 * kk + 1][0], sc[2 * kk + 1][1], a[0][2], a[1][2], a[2][2]);
-            fa_split2(sc[2 * kk + 1][2], sc[2 * kk + 1][3], a[0][3], a[1][3], a[2][3]);
-#pragma unroll
-            for (int np = 0; np < NT / 2; ++np) {
-                uint32_t b0, b1, b2, b3;
-                ldsm_x4_t(vb_a + kk * 16 * LD * 2 + np * 32, b0, b1, b2, b3);
-#pragma unroll
-                for (int pt = 0; pt < 3; ++pt) {
-                    mma_16816(o[2 * np], a[pt][0], a[pt][1], a[pt][2], a[pt][3], b0, b1);
-                    mma_16816(o[2 * np + 1], a[pt][0], a[pt][1], a[pt][2], a[pt][3], b2, b3);
-                }
-            }
-        }
+        __syncthreads();  // every warp is done with this buffer before the next load into it
     }
     if (!act) return;
     // the split's unnormalised output, maximum and sum of each row:
