@@ -750,10 +750,10 @@ def profile_run(args, local: int):
 
 
 def rows_launches(L: int, M: int, kv_only: bool) -> int:
-    """Kernels of one multi-position batch: the start, nine per layer (the
+    """Kernels of one multi-position batch: the start, ten per layer (the
     last layer three when only its cache entries are needed), and the final
     residual add."""
-    return 1 + 9 * (L - 1) + (3 if kv_only else 10)
+    return 1 + 10 * (L - 1) + (3 if kv_only else 11)
 
 
 def profile_rows(shape, model, local: int):
