@@ -30,10 +30,21 @@ def model():
     torch.set_num_threads(4)
     yield synth.make_model(SHAPE)
     torch.set_num_threads(n)
+    _CACHE.clear()
+
+
+_CACHE = {}
 
 
 def _f(a, dt):
-    return torch.from_numpy((np.asarray(a).astype(np.uint32) << 16).view(np.float32)).to(dt)
+    """bf16 bits as a tensor of dtype dt (weights converted once per dtype)."""
+    a = np.asarray(a)
+    if a.ndim < 2:
+        return torch.from_numpy((a.astype(np.uint32) << 16).view(np.float32)).to(dt)
+    key = (id(a), dt)
+    if key not in _CACHE:
+        _CACHE[key] = torch.from_numpy((a.astype(np.uint32) << 16).view(np.float32)).to(dt)
+    return _CACHE[key]
 
 
 def _readout(model, ids, dt, bf16_cache):
