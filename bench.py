@@ -50,7 +50,7 @@ WORKLOAD = "1.5b"
 HEADLINE_RATE = 0.5
 CALIB_TOKENS = 2048
 REPASS_W = 16  # positions in the measured full-depth re-pass
-ROWS_MAX = 64  # positions per batch of the multi-position layer pass (EE_OPT_ROWS)
+ROWS_MAX = 128  # positions per batch of the multi-position layer pass (EE_OPT_ROWS)
 CTL_BYTES = 368  # device control block read back by a host-buffer ee_decode_n
 
 
@@ -758,12 +758,12 @@ def rows_launches(L: int, M: int, kv_only: bool) -> int:
 
 def profile_rows(shape, model, local: int):
     """--profile-run --rows: the multi-position layer pass for ncu captures.
-    A 128-position prompt in two batches, 16 exit steps (direct launches),
+    A 256-position prompt in two batches, 16 exit steps (direct launches),
     then one re-pass of those 16 positions in one batch.  Prints the launch
     counts of each part."""
     from paper_2609_14144_gb300 import DEVICE, FORCE_EXIT_AT, OPT_GRAPHS, OPT_ROWS, Engine
 
-    P, n = 128, REPASS_W
+    P, n = 2 * ROWS_MAX, REPASS_W
     eng = Engine(shape, model, max_ctx=P + n, device=local)
     eng.set_option(OPT_GRAPHS, 0)
     eng.set_option(OPT_ROWS, 1)

@@ -55,16 +55,19 @@ __device__ __forceinline__ float r_lo(uint32_t u) { return __uint_as_float(u << 
 __device__ __forceinline__ float r_hi(uint32_t u) { return __uint_as_float(u & 0xffff0000u); }
 
 // A product's input as three bf16 parts, stored chunk-major: for each
-// 16-byte column chunk (8 columns), the high parts of the kRowsMax rows, then
-// the middle parts, then the low parts, 16 bytes per row.  Eight chunks are
-// then one contiguous block in the tensor cores' canonical operand layout
-// (ee_umma.cu), and a warp-level product reads a row's chunk of one part as
-// 16 contiguous bytes.
+// 16-byte column chunk (8 columns) and each block of kRowsHalf rows, the high
+// parts of the block's rows, then the middle parts, then the low parts, 16
+// bytes per row.  One block's three parts of a chunk are then 192 operand
+// rows in the tensor cores' canonical layout (ee_umma.cu), eight chunks one
+// contiguous stage, and a warp-level product reads a row's chunk of one part
+// as 16 contiguous bytes.
 struct Parts {
     uint16_t* p;
 };
 __device__ __forceinline__ int64_t x3_index(int part, int row, int col) {
-    return ((int64_t)((col >> 3) * 3 + part) * kRowsMax + row) * 8 + (col & 7);
+    constexpr int kBlocks = kRowsMax / kRowsHalf;
+    return ((((int64_t)(col >> 3) * kBlocks + row / kRowsHalf) * 3 + part) * kRowsHalf + row % kRowsHalf) * 8 +
+           (col & 7);
 }
 
 // The three bf16 parts of x at (row, col): high = bf16(x), middle = bf16(x -
@@ -174,8 +177,8 @@ __global__ void __launch_bounds__(kRowsThreads) k_rows_mm(const uint4* __restric
                     const bool okx = ok && row < M;
                     const uint16_t* at = x3.p + x3_index(0, okx ? row : 0, ch * 8);
                     bh[v][n] = okx ? ld_act(at) : make_uint4(0u, 0u, 0u, 0u);
-                    bm[v][n] = okx ? ld_act(at + kRowsMax * 8) : make_uint4(0u, 0u, 0u, 0u);
-                    bl[v][n] = okx ? ld_act(at + 2 * kRowsMax * 8) : make_uint4(0u, 0u, 0u, 0u);
+                    bm[v][n] = okx ? ld_act(at + kRowsHalf * 8) : make_uint4(0u, 0u, 0u, 0u);
+                    bl[v][n] = okx ? ld_act(at + 2 * kRowsHalf * 8) : make_uint4(0u, 0u, 0u, 0u);
                 }
             }
 #pragma unroll
@@ -372,8 +375,8 @@ __global__ void k_rows_prefill_done(DevModel m, int n) {
 //
 // Causal attention of the batch on the tensor cores, its keys split over
 // CTAs (flash-decoding over a prompt batch).  CTA (kv head g, key split s,
-// head z of the group) takes query head h = g G + z for all kRowsMax rows of
-// the batch (4 warps x 16 rows) against keys [s KC, (s + 1) KC) of the
+// z = (row block b, head z' of the group)) takes query head h = g G + z' for
+// the 64 rows of block b of the batch (4 warps x 16 rows) against keys [s KC, (s + 1) KC) of the
 // layer's cache, in blocks of kFaKeys keys staged in shared memory:
 //   S = Q K^T as mma m16n8k16 with the query (scaled by 1/sqrt(D)) split into
 //     three bf16 parts (high + middle + low = q exactly), each multiplied
@@ -433,7 +436,9 @@ __global__ void __launch_bounds__(kFaThreads) k_rows_fattn(DevModel m, int j, co
     uint16_t* qs = fsm;                                // [warp][part][16][LD]
     uint16_t* ks = qs + kFaWarps * 3 * 16 * LD;        // [2][kFaKeys][LD]
     uint16_t* vs = ks + 2 * kFaKeys * LD;              // [2][kFaKeys][LD]
-    const int g = blockIdx.x, s = blockIdx.y, G = m.A / m.KH, h = g * G + blockIdx.z;
+    const int g = blockIdx.x, s = blockIdx.y, G = m.A / m.KH, h = g * G + (int)blockIdx.z % G;
+    const int row0 = ((int)blockIdx.z / G) * kFaWarps * 16;  // the CTA's first row of the batch
+    if (row0 >= Mj) return;                                  // a block with no row at this layer
     const int tid = threadIdx.x, w = tid >> 5, lane = tid & 31, g8 = lane >> 2, t4 = lane & 3;
     const int k0 = s * KC;
     // the CTA's keys end at the split's end or past the batch's last position
@@ -455,7 +460,7 @@ __global__ void __launch_bounds__(kFaThreads) k_rows_fattn(DevModel m, int j, co
     };
     if (k0 < kend) load_block(k0, 0);
     // rows of this warp, their positions (-1: not in the batch)
-    const int r0 = 16 * w + g8, r1 = r0 + 8;
+    const int r0 = row0 + 16 * w + g8, r1 = r0 + 8;
     const int p0 = r0 < Mj ? pos[r0] : -1, p1 = r1 < Mj ? pos[r1] : -1;
     int pw = max(p0, p1);
 #pragma unroll
@@ -469,7 +474,7 @@ __global__ void __launch_bounds__(kFaThreads) k_rows_fattn(DevModel m, int j, co
         float4 qv[QV];
 #pragma unroll
         for (int u = 0; u < QV; ++u) {
-            const int e = lane + 32 * u, r = e / (D / 4), c = 4 * (e - r * (D / 4)), i = 16 * w + r;
+            const int e = lane + 32 * u, r = e / (D / 4), c = 4 * (e - r * (D / 4)), i = row0 + 16 * w + r;
             qv[u] = i < Mj ? *reinterpret_cast<const float4*>(Q + (int64_t)i * m.A * D + (int64_t)h * D + c)
                            : make_float4(0.f, 0.f, 0.f, 0.f);
         }
@@ -700,7 +705,7 @@ cudaError_t launch_attn(const DevModel& m, const RowsBuf& b, int j, int Mj, cons
                         cudaStream_t s) {
     const int KC = fa_keys_per_split(t_max, m.A, b.n_sm);
     const int S = (t_max + KC - 1) / KC;
-    const dim3 grid(m.KH, S, m.A / m.KH);
+    const dim3 grid(m.KH, S, (m.A / m.KH) * (kRowsMax / (kFaWarps * 16)));
     if (m.D == 128) {
         RCKA(launch_pdl(k_rows_fattn<128>, grid, dim3(kFaThreads), fa_smem(128), s, m, j, (const float*)b.Q, d_pos, Mj,
                         KC, t_max, b.part));

@@ -3,12 +3,13 @@
 // with operands staged in shared memory by TMA and the fp32 accumulator in
 // tensor memory.
 //
-// One projection of a batch of M <= 64 positions: Y[row][n] = sum_k W[n][k]
+// One projection of a batch of M <= 128 positions: Y[row][n] = sum_k W[n][k]
 // x[row][k] for the n_rows x K tile-packed bf16 weights W.  Each activation
 // is carried as three bf16 parts (x = high + middle + low, ee_rows.cu), and
-// the three part arrays of a batch are stacked as 192 operand rows, so one
-// MMA of shape M = 128 (weight rows) x N = 192 (3 parts x 64 positions)
-// multiplies every part at once; bf16 products are exact in the fp32
+// the three part arrays of a block of 64 positions are stacked as 192
+// operand rows, so one MMA of shape M = 128 (weight rows) x N = 192 (3 parts
+// x 64 positions) multiplies every part of a block at once, into one of two
+// accumulators (one per block); bf16 products are exact in the fp32
 // accumulator and the epilogue adds the three columns of each position.
 //
 // CTA (x, s): weight rows [128 x, 128 x + 128) (four 32-row tiles) over the
@@ -17,13 +18,15 @@
 //     tensor copy (a four-dimensional view of the tile-packed layout whose
 //     box lands in shared memory in the UMMA canonical K-major layout with
 //     no swizzle: 8-row x 16-byte core matrices, 128 bytes apart along the
-//     rows, 2048 along K) and the 192 x 64 activation block with one bulk
-//     copy (the activation buffer is stored chunk-major, so a stage is one
-//     contiguous 24 KB range in the same canonical layout, 3072 bytes apart
-//     along K);
-//   - warp 1, lane 0 issues four K = 16 MMAs per stage into the tensor-memory
-//     accumulator and commits each stage back to its producer barrier;
-//   - after the last stage all four warps read the accumulator (warp w holds
+//     rows, 2048 along K) and the two 192 x 64 activation blocks with one
+//     bulk copy (the activation buffer is stored chunk-major, so a stage is
+//     one contiguous 48 KB range in the same canonical layout: a block's
+//     192 rows 3072 bytes long, the two blocks of a chunk side by side, 6144
+//     bytes apart along K);
+//   - warp 1, lane 0 issues four K = 16 MMAs per stage and row block (the
+//     second block only when the batch has rows there) into the tensor-memory
+//     accumulators and commits each stage back to its producer barrier;
+//   - after the last stage all four warps read the accumulators (warp w holds
 //     tensor-memory lanes 32 w .. 32 w + 31, the weight rows of tile w) and
 //     write the split's partial sums part[s][row][n], which the consumer adds
 //     in split order as with the warp-level path.
@@ -45,14 +48,17 @@ namespace ee {
 namespace {
 
 constexpr int kUThreads = 128;
-constexpr int kUStages = 5;
+constexpr int kUStages = 3;
 constexpr int kUMRows = 128;                       // weight rows per CTA (UMMA M)
-constexpr int kUN = 3 * kRowsMax;                  // operand rows of the activations (UMMA N)
+constexpr int kUBlocks = kRowsMax / kRowsHalf;     // row blocks of a batch, one accumulator each
+constexpr int kUN = 3 * kRowsHalf;                 // operand rows of one block's activations (UMMA N)
 constexpr int kUKStage = 64;                       // K columns per stage
 constexpr int kUABytes = kUMRows * kUKStage * 2;   // 16 KB
-constexpr int kUBBytes = kUN * kUKStage * 2;       // 24 KB
-constexpr int kUStageBytes = kUABytes + kUBBytes;  // 40 KB
-constexpr int kUTmemCols = 256;                    // power of two >= kUN
+constexpr int kUBBlock = kUN * 16;                 // one block's three parts of one 16-byte chunk: 3 KB
+constexpr int kUBBytes = kUBlocks * kUN * kUKStage * 2;  // 48 KB
+constexpr int kUStageBytes = kUABytes + kUBBytes;  // 64 KB
+constexpr int kUAccCols = 256;                     // tensor-memory columns per accumulator (>= kUN)
+constexpr int kUTmemCols = kUBlocks * kUAccCols;   // 512
 constexpr long long kUWaitCycles = 4000000000ll;   // about 2 s
 
 __device__ __forceinline__ uint32_t u_saddr(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
@@ -199,7 +205,7 @@ __global__ void __launch_bounds__(kUThreads, 1)
             const int kc = (k0 + i) * (kUKStage / 8);  // first 16-byte chunk of the stage
             u_expect_tx(&full[st], kUStageBytes);
             u_tma_w(a, &wmap, tile0, kc, &full[st]);
-            u_bulk(a + kUABytes, x3 + (int64_t)kc * kUN * 8, kUBBytes, &full[st]);
+            u_bulk(a + kUABytes, x3 + (int64_t)kc * kUBlocks * kUN * 8, kUBBytes, &full[st]);
             ++issued;
         }
         // every issued copy lands before the CTA may leave
@@ -217,8 +223,12 @@ __global__ void __launch_bounds__(kUThreads, 1)
             const uint32_t a = u_saddr(sm + st * kUStageBytes), b = a + kUABytes;
 #pragma unroll
             for (int kk = 0; kk < kUKStage / 16; ++kk)
-                u_mma(tmem, u_desc(a + kk * 2 * 2048, 2048, 128), u_desc(b + kk * 2 * 3072, 3072, 128),
-                      (i > 0 || kk > 0) ? 1u : 0u);
+#pragma unroll
+                for (int rb = 0; rb < kUBlocks; ++rb)
+                    if (rb * kRowsHalf < M)
+                        u_mma(tmem + rb * kUAccCols, u_desc(a + kk * 2 * 2048, 2048, 128),
+                              u_desc(b + rb * kUBBlock + kk * 2 * kUBlocks * kUBBlock, kUBlocks * kUBBlock, 128),
+                              (i > 0 || kk > 0) ? 1u : 0u);
             u_commit(&empty[st]);
         }
         u_commit(done);  // after every MMA this thread issued
@@ -234,10 +244,11 @@ __global__ void __launch_bounds__(kUThreads, 1)
         const uint32_t lane_addr = tmem + ((uint32_t)(32 * w) << 16);
         float* ps = part + (int64_t)s * M * Np;
         for (int c0 = 0; c0 < M; c0 += 16) {
+            const uint32_t acc = lane_addr + (c0 / kRowsHalf) * kUAccCols + c0 % kRowsHalf;  // row block's accumulator
             float hi[16], md[16], lo[16];
-            u_ld16(lane_addr + c0, hi);
-            u_ld16(lane_addr + kRowsMax + c0, md);
-            u_ld16(lane_addr + 2 * kRowsMax + c0, lo);
+            u_ld16(acc, hi);
+            u_ld16(acc + kRowsHalf, md);
+            u_ld16(acc + 2 * kRowsHalf, lo);
             if (tile0 + w < n_tiles)
 #pragma unroll
                 for (int i = 0; i < 16; ++i)
