@@ -638,7 +638,7 @@ def run_ours(args, rank: int, world: int, local: int):
         _log(f"[bench] re-pass of {b['repassed']} exited positions: {b['ms']:.2f} ms ({b['token_times']:.2f} "
              f"token-times); one position at a time {repass['one_position_at_a_time']['ms']:.2f} ms")
 
-    # the prompt: batches of up to 64 positions, and one position at a time
+    # the prompt: batches of up to ROWS_MAX positions, and one position at a time
     prefill = None
     if not args.no_sweep:
         P = len(prompt)
