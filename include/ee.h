@@ -30,7 +30,13 @@
  *     product, readout output, logits) fp32; products of bf16 weights and fp32
  *     activations accumulate in fp32; the KV cache is bf16 (round to nearest
  *     even).  The gate compares fp32 p > fp32 tau (strict).  Argmax ties go
- *     to the lowest token id.
+ *     to the lowest token id.  Where a tensor core multiplies an fp32 value
+ *     (the decode step's attention scores; every product of the batched
+ *     prompt and re-pass, EE_OPT_ROWS), the value enters as three bf16 parts
+ *     whose sum is the value (24 significant bits), each part's products with
+ *     bf16 operands exact in the fp32 accumulator.  Values handed between
+ *     CTAs inside the persistent layer kernel keep all 32 bits.  Results
+ *     therefore differ from a plain fp32 loop only in summation order.
  */
 #ifndef EE_H_
 #define EE_H_

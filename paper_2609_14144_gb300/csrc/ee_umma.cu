@@ -278,13 +278,13 @@ bool encode_fn() {
 }
 
 // The tile-packed weights as {8 elements, 32 rows, tiles, 16-byte chunks}
-// with byte strides {-, 16, 64 K, 512}; a box of {8, 32, 4, 8} lands as
+// with byte strides {-, 16, 64 K, 512}; a box of {8, 32, 4, kUKStage / 8} lands as
 // row * 16 + chunk * 2048 bytes (row = 32 tile + row within the tile).
 bool weight_map(CUtensorMap* map, const uint16_t* W, int64_t n_tiles, int K) {
     if (!encode_fn() || K % 8 || ((uintptr_t)W & 15)) return false;
     const cuuint64_t dim[4] = {8, 32, (cuuint64_t)n_tiles, (cuuint64_t)(K / 8)};
     const cuuint64_t stride[3] = {16, (cuuint64_t)K * 64, 512};
-    const cuuint32_t box[4] = {8, 32, 4, 8};
+    const cuuint32_t box[4] = {8, 32, 4, kUKStage / 8};
     const cuuint32_t estr[4] = {1, 1, 1, 1};
     return g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<uint16_t*>(W), dim, stride, box, estr,
                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
