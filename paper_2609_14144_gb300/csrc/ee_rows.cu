@@ -51,8 +51,6 @@ constexpr int kRowsWarps = kRowsThreads / 32;
 
 __device__ __forceinline__ float r_bf2f(uint16_t b) { return __uint_as_float((uint32_t)b << 16); }
 __device__ __forceinline__ uint16_t r_f2bf(float f) { return __bfloat16_as_ushort(__float2bfloat16_rn(f)); }
-__device__ __forceinline__ float r_lo(uint32_t u) { return __uint_as_float(u << 16); }
-__device__ __forceinline__ float r_hi(uint32_t u) { return __uint_as_float(u & 0xffff0000u); }
 
 // A product's input as three bf16 parts, stored chunk-major: for each
 // 16-byte column chunk (8 columns) and each block of kRowsHalf rows, the high
@@ -107,11 +105,6 @@ __device__ __forceinline__ void mma_16816(float (&c)[4], uint32_t a0, uint32_t a
 __device__ __forceinline__ float r_warp_sum(float v) {
 #pragma unroll
     for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-    return v;
-}
-__device__ __forceinline__ float r_warp_max(float v) {
-#pragma unroll
-    for (int o = 16; o; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
     return v;
 }
 

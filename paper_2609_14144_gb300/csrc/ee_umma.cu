@@ -186,6 +186,15 @@ __global__ void __launch_bounds__(kUThreads, 1)
     __syncthreads();
     u_fence_after();
     const uint32_t tmem = *tmem_slot;
+    // The weights do not depend on the previous kernel: the first stages'
+    // weight blocks are requested before the programmatic wait, so that
+    // their HBM latency overlaps the previous kernel's tail.
+    const int pre = ks < kUStages ? ks : kUStages;
+    if (w == 0 && lane == 0)
+        for (int i = 0; i < pre; ++i) {
+            u_expect_tx(&full[i], kUStageBytes);
+            u_tma_w(sm + i * kUStageBytes, &wmap, tile0, (k0 + i) * (kUKStage / 8), &full[i]);
+        }
     // the set-up above overlaps the previous kernel (programmatic launch)
     asm volatile("griddepcontrol.wait;" ::: "memory");
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
@@ -203,8 +212,10 @@ __global__ void __launch_bounds__(kUThreads, 1)
             }
             uint8_t* a = sm + st * kUStageBytes;
             const int kc = (k0 + i) * (kUKStage / 8);  // first 16-byte chunk of the stage
-            u_expect_tx(&full[st], kUStageBytes);
-            u_tma_w(a, &wmap, tile0, kc, &full[st]);
+            if (i >= pre) {  // (the first stages' weights are in flight already)
+                u_expect_tx(&full[st], kUStageBytes);
+                u_tma_w(a, &wmap, tile0, kc, &full[st]);
+            }
             u_bulk(a + kUABytes, x3 + (int64_t)kc * kUBlocks * kUN * 8, kUBBytes, &full[st]);
             ++issued;
         }
