@@ -195,7 +195,7 @@ cudaError_t launch_select_tau(const float* conf, int stride, const int32_t* memb
 constexpr int kSegConsumerWarps = 8;
 constexpr int kSegThreads = 32 * (kSegConsumerWarps + 1);
 constexpr int kSegChunk = 32768;   // bytes per ring stage: 32 rows x 512 bf16 columns
-constexpr int kSegMaxSplits = 32;  // attention splits per kv head (at most)
+constexpr int kSegMaxSplits = 64;  // attention splits per kv head (at most; the O merge's lanes hold two each)
 constexpr int kSegMaxGroup = 8;    // query heads per kv head (at most)
 constexpr int kSegMaxSlots = 8;    // CTAs sharing one down tile, chunks of one O tile (at most)
 // A value handed from one CTA to another inside a launch of the persistent
@@ -212,6 +212,7 @@ struct SegPlan {
     int stages;             // ring stages
     int inflight;           // ring chunks a producer keeps in flight (at most)
     int max_pps;            // attention pages per split (at most)
+    int max_splits;         // attention splits per kv head any step can use (at most)
     int rows_per_kv_chunk;  // cache positions per ring chunk
     int max_items;          // O / down-projection items per CTA (at most)
     int n_tiles[4], n_chunks[4], K[4];  // Q/K/V, O, gate/up, down

@@ -882,7 +882,7 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
     }
     {   // attention partials of the splits this launch does not use: 0 (no
         // tag), so a later launch that uses them again cannot take an old value
-        const int per_head = (kSegMaxSplits - ag.splits) * (m.D + 4);
+        const int per_head = max(0, p.max_splits - ag.splits) * (m.D + 4);
         const int64_t n = (int64_t)m.A * per_head;
         for (int64_t e = (int64_t)cta * kCT + threadIdx.x; e < n; e += (int64_t)G * kCT) {
             const int h = (int)(e / per_head), r = (int)(e - (int64_t)h * per_head);
@@ -1234,8 +1234,9 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
                 const Tagged* base = p.attn_part + (int64_t)h * kSegMaxSplits * (m.D + 4);
                 const Tagged* st = base + lane * (m.D + 4) + m.D;
                 const Tagged* oc = base + c0 + 2 * lane;
-                constexpr int kB = 12;
-                float mk = -INFINITY, lk = 0.f;
+                constexpr int kB = 8;
+                // lane l holds the statistics of splits l and l + 32
+                float mk = -INFINITY, lk = 0.f, mk2 = -INFINITY, lk2 = 0.f;
                 float2 ob[kB];
                 Bound bd;
                 for (;;) {  // one round of loads, again until every lane has its values
@@ -1246,6 +1247,13 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
                         bad |= (tag_of(a) ^ tag) | (tag_of(b) ^ tag);
                         mk = untag(a);
                         lk = untag(b);
+                    }
+                    if (lane + 32 < ns) {
+                        unsigned long long a, b;
+                        ld_strong2(st + 32 * (m.D + 4), a, b);
+                        bad |= (tag_of(a) ^ tag) | (tag_of(b) ^ tag);
+                        mk2 = untag(a);
+                        lk2 = untag(b);
                     }
 #pragma unroll
                     for (int u = 0; u < kB; ++u) {
@@ -1261,9 +1269,10 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
                     const bool more = pl.again(bd);
                     if (!__all_sync(0xffffffffu, more)) break;
                 }
-                const float mx = warp_max(mk);
+                const float mx = warp_max(fmaxf(mk, mk2));
                 const float wk = lane < ns ? expf(mk - mx) : 0.f;
-                const float dn = warp_sum(wk * lk);
+                const float wk2 = lane + 32 < ns ? expf(mk2 - mx) : 0.f;
+                const float dn = warp_sum(wk * lk + wk2 * lk2);
                 float2 num = make_float2(0.f, 0.f);
                 for (int k0 = 0; k0 < ns; k0 += kB) {
                     if (k0 > 0) {  // the next splits (their statistics are in hand)
@@ -1287,7 +1296,7 @@ __global__ void __launch_bounds__(kSegThreads, 1) k_layers(DevModel m, SegPlan p
                     }
 #pragma unroll
                     for (int u = 0; u < kB; ++u) {
-                        const float wu = __shfl_sync(0xffffffffu, wk, (k0 + u) & 31);
+                        const float wu = __shfl_sync(0xffffffffu, k0 + u < 32 ? wk : wk2, (k0 + u) & 31);
                         if (k0 + u < ns) {
                             num.x = fmaf(wu, ob[u].x, num.x);
                             num.y = fmaf(wu, ob[u].y, num.y);
@@ -1581,6 +1590,7 @@ bool seg_plan(const DevModel& m, int n_sm, SegPlan& p) {
     const int cap = std::max(1, std::min(kSegMaxSplits, p.G / m.KH));
     const int np_max = (m.max_ctx + m.page_size - 1) / m.page_size;
     p.max_pps = std::max(1, (np_max + cap - 1) / cap);
+    p.max_splits = std::min(cap, np_max);
     // xs, xa, rope, red (+ norm partials), qa, kv, sc, ml (the carve above)
     const size_t floats = (size_t)((std::max(m.d, m.A * m.D) + 3) & ~3) + (size_t)p.max_items * (kColsPerChunk + 32) +
                           (size_t)m.D + 2 * kCW * 32 + kCW + (size_t)grp * m.D + 2 * (size_t)m.D +
