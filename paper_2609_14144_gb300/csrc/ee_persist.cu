@@ -19,7 +19,7 @@
 //
 // Phases hand results to each other through global memory as tagged
 // values (see "tagged values" below): every float one CTA hands to another
-// carries its layer's tag in the low mantissa bits, and the reader loads
+// travels in a 64-bit word beside its layer's tag, and the reader loads
 // until the tags are the expected ones, so there are no phase counters and
 // no fences.  Q/K/V and gate/up are split by whole 32-row tiles, so each
 // tile's epilogue (bias, RoPE and the KV append; SiLU(gate) * up) runs in
@@ -27,8 +27,8 @@
 // they are split into (tile, 512-column chunk) items over all CTAs, each
 // writing the partial sums of its tiles into slots; the residual is rebuilt
 // by its readers from the slots in slot order (no dependence on timing).  The
-// attention of kv head g over the step's positions is split over CTAs by
-// pages (scores on the tensor cores); the O items merge the splits
+// attention of kv head g over the step's positions is split over up to 64
+// CTAs by pages (scores on the tensor cores); the O items merge the splits
 // (flash-decoding combine).
 //
 // Every wait is bounded: after kStallCycles the waiting thread sets kErrStall
