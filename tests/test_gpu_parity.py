@@ -188,6 +188,9 @@ def test_api_errors(tiny_model):
     with pytest.raises(EEError) as e:
         eng.prefill([0, TINY.vocab])
     assert e.value.code == -1
+    with pytest.raises(EEError) as e:
+        eng.prefill([])  # an empty prompt
+    assert e.value.code == -1
     eng.prefill(synth.prompt(TINY))
     with pytest.raises(EEError) as e:
         eng.decode_step(TINY.vocab, [0.5])
@@ -205,6 +208,28 @@ def test_api_errors(tiny_model):
     eng.reset()
     assert eng.position == 0
     eng.prefill(synth.prompt(TINY))
+
+
+def test_tiny_prompt_of_max_ctx_positions(tiny_model):
+    """The largest prompt a context holds (max_ctx positions, two batches of
+    the multi-position pass with a ragged tail): first token as the oracle's,
+    and the next step is refused (no room for its position)."""
+    from paper_2609_14144_gb300 import EEError, Engine
+
+    n = 150
+    prompt = synth.token_ids(TINY.seed, 907, n, TINY.vocab)
+    orc = oracle.Oracle(TINY, tiny_model, max_ctx=n)
+    tok_o, cap = orc.prefill(prompt, capture=True)
+    eng = Engine(TINY, tiny_model, max_ctx=n)
+    tok_g = eng.prefill(prompt)
+    z = np.sort(np.asarray(cap["final_logits"], np.float64))
+    p = np.exp(z - z[-1])
+    if (p[-1] - p[-2]) / p.sum() >= 1e-3:
+        assert tok_g == tok_o
+    with pytest.raises(EEError) as e:
+        eng.decode_step(tok_g, [0.5])
+    assert e.value.code == -4
+    eng.close()
 
 
 def test_half_b_teacher_forced():
