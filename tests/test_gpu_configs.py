@@ -1,5 +1,8 @@
 """GPU parity on the large workloads at their stated lengths (needs a GB300).
 
+- 0.5B shape (24 layers, width 896, 14/2 heads of 64, SwiGLU 4864, readout at
+  layer 12): 256-token prompt and its 256 gated steps at thresholds calibrated
+  for 50% and 100% exits, on both layer paths.
 - 3B shape (36 layers, width 2048, 16/2 heads of 128, SwiGLU 11008, readout
   at layer 18): 1024-token prompt, 32 gated steps at thresholds calibrated for
   50% and 96% exits, on both layer paths.
@@ -78,6 +81,36 @@ def replay(shape, model, runs: OracleRuns, prompt, taus, persistent: bool, captu
     eng.set_option(OPT_DEBUG_LOGITS, capture)
     assert eng.prefill(prompt) == runs.first
     return eng, gpu_replay(eng, recs, taus, capture=capture)
+
+
+# ------------------------------------------------------------------ 0.5B
+@pytest.fixture(scope="module")
+def half_b():
+    shape = synth.CONFIGS["0.5b"]
+    model = synth.make_model(shape)
+    prompt = synth.prompt(shape)
+    runs = OracleRuns(shape, model, prompt, shape.new_tokens)
+    p = runs.calibrate()[:, 0]
+    taus = {r: tau_for_rate(p, r) for r in (0.5, 1.0)}
+    return shape, model, prompt, runs, taus
+
+
+@pytest.mark.parametrize("rate,persistent", [(0.5, True), (0.5, False), (1.0, True)])
+def test_half_b_full_length(half_b, rate, persistent):
+    shape, model, prompt, runs, taus = half_b
+    tau = [taus[rate]]
+    eng, recs = replay(shape, model, runs, prompt, tau, persistent, capture=rate < 1.0)
+    excluded = check_records(recs, tau, capture=rate < 1.0)
+    check_exit_counts(recs, tau, 1)
+    pe = p_errors(recs)
+    exits = sum(r["o"]["exited"] for r in recs)
+    parity_log("0.5b", rate=rate, tau=tau[0], persistent=persistent, exits=int(exits), steps=len(recs),
+               excluded=excluded, p_err_max=float(pe.max()), p_err_mean=float(pe.mean()))
+    assert excluded <= len(recs) // 4
+    if rate >= 1.0:
+        assert exits == len(recs)
+    check_kv(runs.orc, eng, shape, len(prompt) + runs.n)
+    eng.close()
 
 
 # ------------------------------------------------------------------ 3B
