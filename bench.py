@@ -50,7 +50,7 @@ WORKLOAD = "1.5b"
 HEADLINE_RATE = 0.5
 CALIB_TOKENS = 2048
 REPASS_W = 16  # positions in the measured full-depth re-pass
-ROWS_MAX = 128  # positions per batch of the multi-position layer pass (EE_OPT_ROWS)
+ROWS_MAX = 256  # positions per batch of the multi-position layer pass (EE_OPT_ROWS)
 CTL_BYTES = 368  # device control block read back by a host-buffer ee_decode_n
 
 

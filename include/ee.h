@@ -275,7 +275,7 @@ int ee_position(ee_ctx* ctx, int32_t* pos);
                                  readout 0's token at share value/1000
                                  (Section 2 acceptance)                      */
 #define EE_OPT_ROWS 8         /* 1: ee_prefill and ee_repass run each layer
-                                 over batches of up to 128 positions, each
+                                 over batches of up to 256 positions, each
                                  weight read once per batch, each activation
                                  carried as three bf16 parts (24 significant
                                  bits), the projections on the tcgen05 tensor

@@ -53,19 +53,16 @@ __device__ __forceinline__ float r_bf2f(uint16_t b) { return __uint_as_float((ui
 __device__ __forceinline__ uint16_t r_f2bf(float f) { return __bfloat16_as_ushort(__float2bfloat16_rn(f)); }
 
 // A product's input as three bf16 parts, stored chunk-major: for each
-// 16-byte column chunk (8 columns) and each block of kRowsHalf rows, the high
-// parts of the block's rows, then the middle parts, then the low parts, 16
-// bytes per row.  One block's three parts of a chunk are then 192 operand
-// rows in the tensor cores' canonical layout (ee_umma.cu), eight chunks one
-// contiguous stage, and a warp-level product reads a row's chunk of one part
-// as 16 contiguous bytes.
+// 16-byte column chunk (8 columns), the high parts of the batch's kRowsMax
+// rows, then the middle parts, then the low parts, 16 bytes per row.  One
+// part of a chunk is then kRowsMax operand rows in the tensor cores'
+// canonical layout (ee_umma.cu), a few chunks one contiguous stage, and a
+// warp-level product reads a row's chunk of one part as 16 contiguous bytes.
 struct Parts {
     uint16_t* p;
 };
 __device__ __forceinline__ int64_t x3_index(int part, int row, int col) {
-    constexpr int kBlocks = kRowsMax / kRowsHalf;
-    return ((((int64_t)(col >> 3) * kBlocks + row / kRowsHalf) * 3 + part) * kRowsHalf + row % kRowsHalf) * 8 +
-           (col & 7);
+    return (((int64_t)(col >> 3) * 3 + part) * kRowsMax + row) * 8 + (col & 7);
 }
 
 // The three bf16 parts of x at (row, col): high = bf16(x), middle = bf16(x -
@@ -170,8 +167,8 @@ __global__ void __launch_bounds__(kRowsThreads) k_rows_mm(const uint4* __restric
                     const bool okx = ok && row < M;
                     const uint16_t* at = x3.p + x3_index(0, okx ? row : 0, ch * 8);
                     bh[v][n] = okx ? ld_act(at) : make_uint4(0u, 0u, 0u, 0u);
-                    bm[v][n] = okx ? ld_act(at + kRowsHalf * 8) : make_uint4(0u, 0u, 0u, 0u);
-                    bl[v][n] = okx ? ld_act(at + 2 * kRowsHalf * 8) : make_uint4(0u, 0u, 0u, 0u);
+                    bm[v][n] = okx ? ld_act(at + kRowsMax * 8) : make_uint4(0u, 0u, 0u, 0u);
+                    bl[v][n] = okx ? ld_act(at + 2 * kRowsMax * 8) : make_uint4(0u, 0u, 0u, 0u);
                 }
             }
 #pragma unroll

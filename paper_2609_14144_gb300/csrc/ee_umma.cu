@@ -3,28 +3,29 @@
 // with operands staged in shared memory by TMA and the fp32 accumulator in
 // tensor memory.
 //
-// One projection of a batch of M <= 128 positions: Y[row][n] = sum_k W[n][k]
+// One projection of a batch of M <= 256 positions: Y[row][n] = sum_k W[n][k]
 // x[row][k] for the n_rows x K tile-packed bf16 weights W.  Each activation
-// is carried as three bf16 parts (x = high + middle + low, ee_rows.cu), and
-// the three part arrays of a block of 64 positions are stacked as 192
-// operand rows, so one MMA of shape M = 128 (weight rows) x N = 192 (3 parts
-// x 64 positions) multiplies every part of a block at once, into one of two
-// accumulators (one per block); bf16 products are exact in the fp32
-// accumulator and the epilogue adds the three columns of each position.
+// is carried as three bf16 parts (x = high + middle + low, ee_rows.cu), each
+// part of the batch stored as 256 operand rows; every K = 16 step issues
+// three MMAs of shape M = 128 (weight rows) x N (the batch's rows rounded up
+// to 16), one per part, into two fp32 accumulators whose column is the batch
+// row: the high parts' products into the first, the middle and low parts'
+// (2^-8 of the size and less) into the second, so that their small terms are
+// not added into the large sum step by step; the epilogue adds the two.  The
+// bf16 products are exact.
 //
 // CTA (x, s): weight rows [128 x, 128 x + 128) (four 32-row tiles) over the
-// K range of split s, 64 columns per pipeline stage:
-//   - warp 0, lane 0 loads a stage: the 128 x 64 weight block with one TMA
-//     tensor copy (a four-dimensional view of the tile-packed layout whose
+// K range of split s, 32 columns per pipeline stage, four stages in flight:
+//   - warp 0, lane 0 loads a stage: the 128 x 32 weight block with one TMA
+//     tensor copy (a three-dimensional view of the tile-packed layout whose
 //     box lands in shared memory in the UMMA canonical K-major layout with
 //     no swizzle: 8-row x 16-byte core matrices, 128 bytes apart along the
-//     rows, 2048 along K) and the two 192 x 64 activation blocks with one
-//     bulk copy (the activation buffer is stored chunk-major, so a stage is
-//     one contiguous 48 KB range in the same canonical layout: a block's
-//     192 rows 3072 bytes long, the two blocks of a chunk side by side, 6144
-//     bytes apart along K);
-//   - warp 1, lane 0 issues four K = 16 MMAs per stage and row block (the
-//     second block only when the batch has rows there) into the tensor-memory
+//     rows, 2048 along K) and the batch's activations with bulk copies (the
+//     activation buffer is stored chunk-major, so a full batch's stage is one
+//     contiguous 48 KB range in the same canonical layout: a part's 256 rows
+//     4 KB long, the three parts of a chunk side by side, chunks 12 KB apart
+//     along K; a smaller batch copies the first N rows of each part);
+//   - warp 1, lane 0 issues six MMAs per stage into the tensor-memory
 //     accumulators and commits each stage back to its producer barrier;
 //   - after the last stage all four warps read the accumulators (warp w holds
 //     tensor-memory lanes 32 w .. 32 w + 31, the weight rows of tile w) and
@@ -48,17 +49,15 @@ namespace ee {
 namespace {
 
 constexpr int kUThreads = 128;
-constexpr int kUStages = 3;
-constexpr int kUMRows = 128;                       // weight rows per CTA (UMMA M)
-constexpr int kUBlocks = kRowsMax / kRowsHalf;     // row blocks of a batch, one accumulator each
-constexpr int kUN = 3 * kRowsHalf;                 // operand rows of one block's activations (UMMA N)
-constexpr int kUKStage = 64;                       // K columns per stage
-constexpr int kUABytes = kUMRows * kUKStage * 2;   // 16 KB
-constexpr int kUBBlock = kUN * 16;                 // one block's three parts of one 16-byte chunk: 3 KB
-constexpr int kUBBytes = kUBlocks * kUN * kUKStage * 2;  // 48 KB
-constexpr int kUStageBytes = kUABytes + kUBBytes;  // 64 KB
-constexpr int kUAccCols = 256;                     // tensor-memory columns per accumulator (>= kUN)
-constexpr int kUTmemCols = kUBlocks * kUAccCols;   // 512
+constexpr int kUStages = 4;
+constexpr int kUMRows = 128;                        // weight rows per CTA (UMMA M)
+constexpr int kUKStage = 32;                        // K columns per stage
+constexpr int kUABytes = kUMRows * kUKStage * 2;    // 8 KB
+constexpr int kUPartBytes = kRowsMax * 16;          // one part of one 16-byte chunk: 4 KB
+constexpr int kUChunkBytes = 3 * kUPartBytes;       // the three parts of a chunk: 12 KB
+constexpr int kUBBytes = kUKStage / 8 * kUChunkBytes;  // 48 KB
+constexpr int kUStageBytes = kUABytes + kUBBytes;   // 56 KB
+constexpr int kUTmemCols = 2 * kRowsMax;            // two accumulators of one fp32 column per position
 constexpr long long kUWaitCycles = 4000000000ll;   // about 2 s
 
 __device__ __forceinline__ uint32_t u_saddr(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
@@ -101,15 +100,16 @@ __device__ __forceinline__ uint64_t u_desc(uint32_t saddr, uint32_t lbo, uint32_
     return d;                // base offset 0, layout type 0 (no swizzle)
 }
 // Instruction descriptor of kind::f16: fp32 accumulator, bf16 A and B, both
-// K-major, N = kUN, M = kUMRows.
-constexpr uint32_t kUIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(kUN >> 3) << 17) |
-                             ((uint32_t)(kUMRows >> 4) << 24);
+// K-major, M = kUMRows, N = n (a multiple of 16, 16 <= n <= 256).
+__device__ __forceinline__ uint32_t u_idesc(int n) {
+    return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(kUMRows >> 4) << 24);
+}
 
-__device__ __forceinline__ void u_mma(uint32_t tmem_d, uint64_t a, uint64_t b, uint32_t accumulate) {
+__device__ __forceinline__ void u_mma(uint32_t tmem_d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t accumulate) {
     asm volatile(
         "{ .reg .pred p; setp.ne.u32 p, %4, 0; tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p; }" ::"r"(
             tmem_d),
-        "l"(a), "l"(b), "r"(kUIdesc), "r"(accumulate)
+        "l"(a), "l"(b), "r"(idesc), "r"(accumulate)
         : "memory");
 }
 __device__ __forceinline__ void u_commit(uint64_t* bar) {
@@ -138,12 +138,13 @@ __device__ __forceinline__ void u_expect_tx(uint64_t* bar, uint32_t bytes) {
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(u_saddr(bar)), "r"(bytes) : "memory");
 }
 // The 128 x 64 weight block at (tile t0, 16-byte column chunk c0) of the
-// four-dimensional view {8 elements, 32 rows, tiles, chunks}.
+// three-dimensional view {256 elements (one chunk of a 32-row tile), tiles,
+// chunks}.
 __device__ __forceinline__ void u_tma_w(void* dst, const CUtensorMap* map, int t0, int c0, uint64_t* bar) {
     asm volatile(
-        "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4, %5}], "
-        "[%6];" ::"r"(u_saddr(dst)),
-        "l"(map), "r"(0), "r"(0), "r"(t0), "r"(c0), "r"(u_saddr(bar))
+        "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], "
+        "[%5];" ::"r"(u_saddr(dst)),
+        "l"(map), "r"(0), "r"(t0), "r"(c0), "r"(u_saddr(bar))
         : "memory");
 }
 __device__ __forceinline__ void u_bulk(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
@@ -166,6 +167,10 @@ __global__ void __launch_bounds__(kUThreads, 1)
     const int tile0 = blockIdx.x * 4, s = blockIdx.y;
     const int nk = (K + kUKStage - 1) / kUKStage;
     const int k0 = (int)((int64_t)nk * s / S), k1 = (int)((int64_t)nk * (s + 1) / S), ks = k1 - k0;
+    // operand rows of the batch (UMMA N): M rounded up to 16; the rows past M
+    // give accumulator columns that are never read
+    const int N = (M + 15) & ~15;
+    const uint32_t stage_tx = (uint32_t)(kUABytes + kUKStage / 8 * 3 * N * 16);
     volatile int* everr = err;
 
     if (threadIdx.x == 0) {
@@ -192,7 +197,7 @@ __global__ void __launch_bounds__(kUThreads, 1)
     const int pre = ks < kUStages ? ks : kUStages;
     if (w == 0 && lane == 0)
         for (int i = 0; i < pre; ++i) {
-            u_expect_tx(&full[i], kUStageBytes);
+            u_expect_tx(&full[i], stage_tx);
             u_tma_w(sm + i * kUStageBytes, &wmap, tile0, (k0 + i) * (kUKStage / 8), &full[i]);
         }
     // the set-up above overlaps the previous kernel (programmatic launch)
@@ -213,10 +218,16 @@ __global__ void __launch_bounds__(kUThreads, 1)
             uint8_t* a = sm + st * kUStageBytes;
             const int kc = (k0 + i) * (kUKStage / 8);  // first 16-byte chunk of the stage
             if (i >= pre) {  // (the first stages' weights are in flight already)
-                u_expect_tx(&full[st], kUStageBytes);
+                u_expect_tx(&full[st], stage_tx);
                 u_tma_w(a, &wmap, tile0, kc, &full[st]);
             }
-            u_bulk(a + kUABytes, x3 + (int64_t)kc * kUBlocks * kUN * 8, kUBBytes, &full[st]);
+            if (N == kRowsMax) {  // the stage's activations are one contiguous range
+                u_bulk(a + kUABytes, x3 + (int64_t)kc * 3 * kRowsMax * 8, kUBBytes, &full[st]);
+            } else {  // the first N rows of each (chunk, part)
+                for (int cp = 0; cp < kUKStage / 8 * 3; ++cp)
+                    u_bulk(a + kUABytes + cp * kUPartBytes, x3 + ((int64_t)kc * 3 + cp) * kRowsMax * 8,
+                           (uint32_t)N * 16, &full[st]);
+            }
             ++issued;
         }
         // every issued copy lands before the CTA may leave
@@ -224,6 +235,7 @@ __global__ void __launch_bounds__(kUThreads, 1)
             u_mb_wait(&full[i % kUStages], (i / kUStages) & 1, nullptr);
     } else if (w == 1 && lane == 0) {
         // MMA issuer
+        const uint32_t idesc = u_idesc(N);
         for (int i = 0; i < ks; ++i) {
             const int st = i % kUStages;
             if (!u_mb_wait(&full[st], (i / kUStages) & 1, everr)) {
@@ -232,14 +244,16 @@ __global__ void __launch_bounds__(kUThreads, 1)
             }
             u_fence_after();
             const uint32_t a = u_saddr(sm + st * kUStageBytes), b = a + kUABytes;
+            // each K = 16 step: the weights times the high parts of the batch
+            // into the first accumulator, times the middle and the low parts
+            // into the second
 #pragma unroll
             for (int kk = 0; kk < kUKStage / 16; ++kk)
 #pragma unroll
-                for (int rb = 0; rb < kUBlocks; ++rb)
-                    if (rb * kRowsHalf < M)
-                        u_mma(tmem + rb * kUAccCols, u_desc(a + kk * 2 * 2048, 2048, 128),
-                              u_desc(b + rb * kUBBlock + kk * 2 * kUBlocks * kUBBlock, kUBlocks * kUBBlock, 128),
-                              (i > 0 || kk > 0) ? 1u : 0u);
+                for (int pp = 0; pp < 3; ++pp)
+                    u_mma(tmem + (pp ? kRowsMax : 0), u_desc(a + kk * 2 * 2048, 2048, 128),
+                          u_desc(b + (kk * 2 * 3 + pp) * kUPartBytes, kUChunkBytes, 128), idesc,
+                          (i > 0 || kk > 0 || pp == 2) ? 1u : 0u);
             u_commit(&empty[st]);
         }
         u_commit(done);  // after every MMA this thread issued
@@ -254,16 +268,14 @@ __global__ void __launch_bounds__(kUThreads, 1)
         const int n = (tile0 + w) * 32 + lane;  // output row of the projection
         const uint32_t lane_addr = tmem + ((uint32_t)(32 * w) << 16);
         float* ps = part + (int64_t)s * M * Np;
-        for (int c0 = 0; c0 < M; c0 += 16) {
-            const uint32_t acc = lane_addr + (c0 / kRowsHalf) * kUAccCols + c0 % kRowsHalf;  // row block's accumulator
-            float hi[16], md[16], lo[16];
-            u_ld16(acc, hi);
-            u_ld16(acc + kRowsHalf, md);
-            u_ld16(acc + 2 * kRowsHalf, lo);
+        for (int c0 = 0; c0 < M; c0 += 16) {  // accumulator column = batch row
+            float hi[16], ml[16];
+            u_ld16(lane_addr + c0, hi);
+            u_ld16(lane_addr + kRowsMax + c0, ml);
             if (tile0 + w < n_tiles)
 #pragma unroll
                 for (int i = 0; i < 16; ++i)
-                    if (c0 + i < M) ps[(int64_t)(c0 + i) * Np + n] = (hi[i] + md[i]) + lo[i];
+                    if (c0 + i < M) ps[(int64_t)(c0 + i) * Np + n] = hi[i] + ml[i];
         }
     }
     u_fence_before();
@@ -288,16 +300,18 @@ bool encode_fn() {
     return g_encode != nullptr;
 }
 
-// The tile-packed weights as {8 elements, 32 rows, tiles, 16-byte chunks}
-// with byte strides {-, 16, 64 K, 512}; a box of {8, 32, 4, kUKStage / 8} lands as
-// row * 16 + chunk * 2048 bytes (row = 32 tile + row within the tile).
+// The tile-packed weights as {256 elements, tiles, 16-byte chunks} with byte
+// strides {-, 64 K, 512}: the 32 rows of one tile's chunk are 512 contiguous
+// bytes.  A box of {256, 4, kUKStage / 8} lands as row * 16 + chunk * 2048
+// bytes (row = 32 tile + row within the tile), the canonical layout, in 512-byte
+// rows of the copy.
 bool weight_map(CUtensorMap* map, const uint16_t* W, int64_t n_tiles, int K) {
     if (!encode_fn() || K % 8 || ((uintptr_t)W & 15)) return false;
-    const cuuint64_t dim[4] = {8, 32, (cuuint64_t)n_tiles, (cuuint64_t)(K / 8)};
-    const cuuint64_t stride[3] = {16, (cuuint64_t)K * 64, 512};
-    const cuuint32_t box[4] = {8, 32, 4, kUKStage / 8};
-    const cuuint32_t estr[4] = {1, 1, 1, 1};
-    return g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<uint16_t*>(W), dim, stride, box, estr,
+    const cuuint64_t dim[3] = {256, (cuuint64_t)n_tiles, (cuuint64_t)(K / 8)};
+    const cuuint64_t stride[2] = {(cuuint64_t)K * 64, 512};
+    const cuuint32_t box[3] = {256, 4, kUKStage / 8};
+    const cuuint32_t estr[3] = {1, 1, 1};
+    return g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<uint16_t*>(W), dim, stride, box, estr,
                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }

@@ -1,7 +1,7 @@
 """The multi-position layer pass on the GPU (needs a GB300).
 
 With EE_OPT_ROWS = 1 the prompt and the re-pass run each layer over batches
-of up to 128 positions, the projections on the tcgen05 tensor cores (2: the
+of up to 256 positions, the projections on the tcgen05 tensor cores (2: the
 same batches with warp-level mma products).  Checked against the oracle (first token exact outside
 the 1e-3 top-2 band, final hidden state and logits and every cache entry
 within 1e-2 relative, which (layer, position) entries were computed bit for
@@ -47,12 +47,13 @@ def _engine(shape, model, max_ctx, rows=True, pages=None):
 
 
 @pytest.mark.parametrize("mode", [1, 2])
-@pytest.mark.parametrize("n", [1, 7, 64, 65, 128, 129, 300])
+@pytest.mark.parametrize("n", [1, 7, 16, 17, 255, 256, 257, 600])
 def test_tiny_prompt_batches_match_oracle(tiny_model, n, mode):
-    """Prompts of one position, a partial first row block, one full block, a
-    full block and one row of the second, one full batch, a full batch and one
-    position, and two full batches and a ragged tail, on the tcgen05 and the
-    warp-level products (F = 688: a ragged last K stage)."""
+    """Prompts of one position, a partial first group of 16 rows (the
+    tcgen05 products' N step), one full group, a full group and one row, one
+    short of a full batch, one full batch, a full batch and one position, and
+    two full batches and a ragged tail, on the tcgen05 and the warp-level
+    products (F = 688: a ragged last K stage)."""
     prompt = synth.token_ids(TINY.seed, 901, n, TINY.vocab)
     orc = oracle.Oracle(TINY, tiny_model, max_ctx=n + 1)
     tok_o, cap = orc.prefill(prompt, capture=True)
@@ -124,7 +125,8 @@ def _exit_decode(shape, model, n, force_of, rows=True):
 
 
 def test_tiny_repass_in_several_batches(tiny_model):
-    """450 decoded positions, two of three exited: three batches of rows."""
+    """450 decoded positions, two of three exited: 300 rows, a full batch and
+    a partial one."""
     n, P = 450, TINY.prompt_len
     force = lambda i: oracle.FORCE_FULL if i % 3 == 0 else oracle.FORCE_EXIT_AT(0)
     orc, eng = _exit_decode(TINY, tiny_model, n, force)
@@ -161,11 +163,11 @@ def test_tiny_repass_paths_agree(tiny_model):
 
 
 def test_1p5b_prompt_batches_sampled():
-    """The 1.5B shape with a 200-position prompt (a full batch and a partial
+    """The 1.5B shape with a 300-position prompt (a full batch and a partial
     one): first token, final state and sampled cache entries."""
-    shape = synth.CONFIGS["1.5b"].replace(prompt_len=200)
+    shape = synth.CONFIGS["1.5b"].replace(prompt_len=300)
     model = synth.make_model(shape)
-    n = 200
+    n = 300
     prompt = synth.prompt(shape)
     orc = oracle.Oracle(shape, model, max_ctx=n + 1)
     tok_o, cap = orc.prefill(prompt, capture=True)
@@ -175,7 +177,7 @@ def test_1p5b_prompt_batches_sampled():
         assert tok_g == tok_o
     assert rel_err(eng.hidden_final(), cap["h_final"]) <= REL_TOL
     for j in (0, 13, 27):
-        for t in (0, 63, 64, 127, 128, 199):
+        for t in (0, 127, 128, 255, 256, 299):
             ko, vo, so = orc.kv(j, t)
             kg, vg = eng.kv(j, t)
             assert eng.kv_src(j, t) == so == 1
@@ -185,20 +187,20 @@ def test_1p5b_prompt_batches_sampled():
 @pytest.mark.parametrize("name", ["0.5b", "1.5b"])
 def test_tensor_core_paths_agree(name):
     """The tcgen05 products (EE_OPT_ROWS = 1) against the warp-level ones
-    (2) on a 128-position batch and a 72-position one: same first token,
+    (2) on a 256-position batch and a 44-position one: same first token,
     fp32 states within 1e-3, cache entries within 1e-2 (bf16 rounding)."""
-    shape = synth.CONFIGS[name].replace(prompt_len=200)
+    shape = synth.CONFIGS[name].replace(prompt_len=300)
     model = synth.make_model(shape)
     prompt = synth.prompt(shape)
-    a = _engine(shape, model, 201, rows=1)
-    b = _engine(shape, model, 201, rows=2)
+    a = _engine(shape, model, 301, rows=1)
+    b = _engine(shape, model, 301, rows=2)
     ta, tb = a.prefill(prompt), b.prefill(prompt)
     if _top2_gap(b.final_logits()) >= EXCLUDE_EPS:
         assert ta == tb
     assert rel_err(a.hidden_final(), b.hidden_final()) <= PATH_TOL
     assert rel_err(a.final_logits(), b.final_logits()) <= PATH_TOL
     for j in (0, shape.n_layers // 2, shape.n_layers - 1):
-        for t in (0, 31, 63, 64, 127, 128, 199):
+        for t in (0, 31, 127, 255, 256, 299):
             ka, va = a.kv(j, t)
             kb, vb = b.kv(j, t)
             assert rel_err(ka, kb) <= REL_TOL and rel_err(va, vb) <= REL_TOL, (j, t)
