@@ -678,11 +678,13 @@ void row_groups(int M, int& NB, int& RG) {
 }
 
 // Keys per split of the flash attention: a multiple of kFaKeys, large enough
-// that the splits of a batch whose last position is t_max - 1 number about
-// two CTAs per SM over the (kv head, query head) pairs, and at most
-// kFaMaxSplits.
-int fa_keys_per_split(int t_max, int n_heads, int n_sm) {
-    const int target = std::max(1, std::min(kFaMaxSplits, 2 * n_sm / std::max(1, n_heads)));
+// that the splits of a batch whose last position is t_max - 1, times the
+// (query head, block of 64 rows) pairs, make about one wave of CTAs (one
+// resident per SM: its stages take over half the shared memory), and at most
+// kFaMaxSplits.  (Two or four waves of shorter splits were slower: every
+// split is a partial result written, merged and read again.)
+int fa_keys_per_split(int t_max, int units, int n_sm) {
+    const int target = std::max(1, std::min(kFaMaxSplits, n_sm / std::max(1, units)));
     int kc = (t_max + target - 1) / target;
     kc = std::max(kFaKeys, (kc + kFaKeys - 1) / kFaKeys * kFaKeys);
     while ((t_max + kc - 1) / kc > kFaMaxSplits) kc += kFaKeys;
@@ -693,9 +695,10 @@ int fa_keys_per_split(int t_max, int n_heads, int n_sm) {
 // the O projection's input parts.
 cudaError_t launch_attn(const DevModel& m, const RowsBuf& b, int j, int Mj, const int32_t* d_pos, int t_max,
                         cudaStream_t s) {
-    const int KC = fa_keys_per_split(t_max, m.A, b.n_sm);
+    const int row_blocks = (Mj + kFaWarps * 16 - 1) / (kFaWarps * 16);
+    const int KC = fa_keys_per_split(t_max, m.A * row_blocks, b.n_sm);
     const int S = (t_max + KC - 1) / KC;
-    const dim3 grid(m.KH, S, (m.A / m.KH) * (kRowsMax / (kFaWarps * 16)));
+    const dim3 grid(m.KH, S, (m.A / m.KH) * row_blocks);
     if (m.D == 128) {
         RCKA(launch_pdl(k_rows_fattn<128>, grid, dim3(kFaThreads), fa_smem(128), s, m, j, (const float*)b.Q, d_pos, Mj,
                         KC, t_max, b.part));
