@@ -252,11 +252,13 @@ cudaError_t launch_vocab_ring(const VocabArgs& v, const VocabRing& vr, bool pdl,
 // once per batch.  Products are tensor-core mma of the bf16 weights with the
 // fp32 activations split into three bf16 parts (high, middle, low).
 constexpr int kRowsMax = 256;            // positions per batch (the tcgen05 products' largest N)
+// Row stride of a batch's activation parts: M rounded up to 16.
+__host__ __device__ constexpr int x3_rows(int M) { return (M + 15) & ~15; }
 constexpr int kRowsTargetUnits = 2432;   // (tile, K split) units a projection aims for: 152 SMs x 16 warps
 struct RowsBuf {
     float* H;           // [kRowsMax][d] residual of each row
     uint16_t* x3;       // next product's input as three bf16 parts (high, x - high, the rest),
-                        // chunk-major: [ldx / 8][3][kRowsMax][8]
+                        // chunk-major: [ldx / 8][3][x3_rows(M)][8] for a batch of M rows
     float* Q;           // [kRowsMax][A D] rotated queries
     float* part;        // split partials [S][M][n_rows padded to 32]
     int32_t* pos;       // [kRowsMax] positions of a prompt batch

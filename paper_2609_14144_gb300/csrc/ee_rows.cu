@@ -53,16 +53,19 @@ __device__ __forceinline__ float r_bf2f(uint16_t b) { return __uint_as_float((ui
 __device__ __forceinline__ uint16_t r_f2bf(float f) { return __bfloat16_as_ushort(__float2bfloat16_rn(f)); }
 
 // A product's input as three bf16 parts, stored chunk-major: for each
-// 16-byte column chunk (8 columns), the high parts of the batch's kRowsMax
-// rows, then the middle parts, then the low parts, 16 bytes per row.  One
-// part of a chunk is then kRowsMax operand rows in the tensor cores'
-// canonical layout (ee_umma.cu), a few chunks one contiguous stage, and a
-// warp-level product reads a row's chunk of one part as 16 contiguous bytes.
+// 16-byte column chunk (8 columns), the high parts of the batch's rows, then
+// the middle parts, then the low parts, 16 bytes per row and `rows` rows a
+// part (the batch's row count rounded up to 16).  One part of a chunk is then
+// the tensor cores' operand of N = rows rows in their canonical layout
+// (ee_umma.cu), a few chunks one contiguous stage whatever the batch size,
+// and a warp-level product reads a row's chunk of one part as 16 contiguous
+// bytes.
 struct Parts {
     uint16_t* p;
+    int rows;
 };
-__device__ __forceinline__ int64_t x3_index(int part, int row, int col) {
-    return (((int64_t)(col >> 3) * 3 + part) * kRowsMax + row) * 8 + (col & 7);
+__device__ __forceinline__ int64_t x3_index(int part, int row, int col, int rows) {
+    return (((int64_t)(col >> 3) * 3 + part) * rows + row) * 8 + (col & 7);
 }
 
 // The three bf16 parts of x at (row, col): high = bf16(x), middle = bf16(x -
@@ -71,9 +74,9 @@ __device__ __forceinline__ void split_store(float x, const Parts& p, int row, in
     const uint16_t h = r_f2bf(x);
     const float r1 = x - r_bf2f(h);
     const uint16_t md = r_f2bf(r1);
-    p.p[x3_index(0, row, col)] = h;
-    p.p[x3_index(1, row, col)] = md;
-    p.p[x3_index(2, row, col)] = r_f2bf(r1 - r_bf2f(md));
+    p.p[x3_index(0, row, col, p.rows)] = h;
+    p.p[x3_index(1, row, col, p.rows)] = md;
+    p.p[x3_index(2, row, col, p.rows)] = r_f2bf(r1 - r_bf2f(md));
 }
 // Columns from n up to the next multiple of 64 (a tensor-core stage) read as 0.
 __host__ __device__ __forceinline__ int pad64(int n) { return (n + 63) & ~63; }
@@ -165,10 +168,10 @@ __global__ void __launch_bounds__(kRowsThreads) k_rows_mm(const uint4* __restric
                 for (int n = 0; n < NB; ++n) {
                     const int row = r0 + n * 8 + g;
                     const bool okx = ok && row < M;
-                    const uint16_t* at = x3.p + x3_index(0, okx ? row : 0, ch * 8);
+                    const uint16_t* at = x3.p + x3_index(0, okx ? row : 0, ch * 8, x3.rows);
                     bh[v][n] = okx ? ld_act(at) : make_uint4(0u, 0u, 0u, 0u);
-                    bm[v][n] = okx ? ld_act(at + kRowsMax * 8) : make_uint4(0u, 0u, 0u, 0u);
-                    bl[v][n] = okx ? ld_act(at + 2 * kRowsMax * 8) : make_uint4(0u, 0u, 0u, 0u);
+                    bm[v][n] = okx ? ld_act(at + x3.rows * 8) : make_uint4(0u, 0u, 0u, 0u);
+                    bl[v][n] = okx ? ld_act(at + 2 * x3.rows * 8) : make_uint4(0u, 0u, 0u, 0u);
                 }
             }
 #pragma unroll
@@ -662,7 +665,9 @@ cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t sme
     return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
 }
 
-Parts parts(const RowsBuf& b) { return Parts{b.x3}; }
+// The activation parts of a batch of M rows (row stride M rounded up to 16,
+// the operand rows of the tensor-core products).
+Parts parts(const RowsBuf& b, int M) { return Parts{b.x3, x3_rows(M)}; }
 
 #define RCKA(x)                                   \
     do {                                          \
@@ -703,11 +708,11 @@ cudaError_t launch_attn(const DevModel& m, const RowsBuf& b, int j, int Mj, cons
         RCKA(launch_pdl(k_rows_fattn<128>, grid, dim3(kFaThreads), fa_smem(128), s, m, j, (const float*)b.Q, d_pos, Mj,
                         KC, t_max, b.part));
         return launch_pdl(k_rows_amerge<128>, dim3(m.A, Mj), dim3(128), 0, s, m, (const float*)b.part, d_pos, KC,
-                          parts(b));
+                          parts(b, Mj));
     }
     RCKA(launch_pdl(k_rows_fattn<64>, grid, dim3(kFaThreads), fa_smem(64), s, m, j, (const float*)b.Q, d_pos, Mj, KC,
                     t_max, b.part));
-    return launch_pdl(k_rows_amerge<64>, dim3(m.A, Mj), dim3(64), 0, s, m, (const float*)b.part, d_pos, KC, parts(b));
+    return launch_pdl(k_rows_amerge<64>, dim3(m.A, Mj), dim3(64), 0, s, m, (const float*)b.part, d_pos, KC, parts(b, Mj));
 }
 
 // One projection of the batch: W (n_rows x K, tiled) times the M rows of
@@ -730,13 +735,13 @@ cudaError_t launch_mm(const uint16_t* W, int64_t n_rows, int K, const RowsBuf& b
     const int grid = (int)std::min<int64_t>((units + kRowsWarps - 1) / kRowsWarps, 65535);
     const uint4* w = reinterpret_cast<const uint4*>(W);
     if (NB == 1)
-        return launch_pdl(k_rows_mm<1, 2>, dim3(grid), dim3(kRowsThreads), 0, s, w, (int)nt, K, parts(b), b.ldx, M, S, RG,
+        return launch_pdl(k_rows_mm<1, 2>, dim3(grid), dim3(kRowsThreads), 0, s, w, (int)nt, K, parts(b, M), b.ldx, M, S, RG,
                           b.part, Np);
     else if (NB == 2)
-        return launch_pdl(k_rows_mm<2, 2>, dim3(grid), dim3(kRowsThreads), 0, s, w, (int)nt, K, parts(b), b.ldx, M, S, RG,
+        return launch_pdl(k_rows_mm<2, 2>, dim3(grid), dim3(kRowsThreads), 0, s, w, (int)nt, K, parts(b, M), b.ldx, M, S, RG,
                           b.part, Np);
     else
-        return launch_pdl(k_rows_mm<4, 1>, dim3(grid), dim3(kRowsThreads), 0, s, w, (int)nt, K, parts(b), b.ldx, M, S, RG,
+        return launch_pdl(k_rows_mm<4, 1>, dim3(grid), dim3(kRowsThreads), 0, s, w, (int)nt, K, parts(b, M), b.ldx, M, S, RG,
                           b.part, Np);
 }
 
@@ -805,7 +810,7 @@ cudaError_t rows_pass(const DevModel& m, const RowsBuf& b, const int* start, int
         int S = 1, Np = 0;
         // the previous layer's down projection into the residual, this layer's input norm
         RCK(launch_pdl(k_rows_add_norm, dim3(Mj), dim3(kNormThreads), 0, s, b.H, d, (const float*)b.part, S_prev, M_prev,
-                       Np_prev, lw + m.off_gattn, m.eps, parts(b), b.ldx));
+                       Np_prev, lw + m.off_gattn, m.eps, parts(b, Mj), b.ldx));
         RCK(launch_mm(lw + m.off_wqkv, nqkv, d, b, Mj, S, Np, s));
         const int nu = (int)(nqkv / 2);
         RCK(launch_pdl(k_rows_qkv, dim3((nu + kRowsThreads - 1) / kRowsThreads, Mj), dim3(kRowsThreads), 0, s, m, j,
@@ -814,10 +819,10 @@ cudaError_t rows_pass(const DevModel& m, const RowsBuf& b, const int* start, int
         RCK(launch_attn(m, b, j, Mj, d_pos, t_max, s));
         RCK(launch_mm(lw + m.off_wo, d, AD, b, Mj, S, Np, s));
         RCK(launch_pdl(k_rows_add_norm, dim3(Mj), dim3(kNormThreads), 0, s, b.H, d, (const float*)b.part, S, Mj, Np,
-                       lw + m.off_gmlp, m.eps, parts(b), b.ldx));
+                       lw + m.off_gmlp, m.eps, parts(b, Mj), b.ldx));
         RCK(launch_mm(lw + m.off_wgu, 2LL * m.F, d, b, Mj, S, Np, s));
         RCK(launch_pdl(k_rows_swiglu, dim3((pad64(m.F) + kRowsThreads - 1) / kRowsThreads, Mj), dim3(kRowsThreads), 0, s,
-                       (const float*)b.part, S, Mj, Np, m.F, parts(b), b.ldx));
+                       (const float*)b.part, S, Mj, Np, m.F, parts(b, Mj), b.ldx));
         RCK(launch_mm(lw + m.off_wd, d, m.F, b, Mj, S, Np, s));
         M_prev = Mj;
         S_prev = S;
@@ -825,7 +830,7 @@ cudaError_t rows_pass(const DevModel& m, const RowsBuf& b, const int* start, int
     }
     // the last down projection into the residual (no norm)
     return launch_pdl(k_rows_add_norm, dim3(M_prev), dim3(kNormThreads), 0, s, b.H, d, (const float*)b.part, S_prev,
-                      M_prev, Np_prev, (const uint16_t*)nullptr, m.eps, parts(b), b.ldx);
+                      M_prev, Np_prev, (const uint16_t*)nullptr, m.eps, parts(b, M_prev), b.ldx);
 }
 
 cudaError_t launch_rows_prefill_done(const DevModel& m, int n, cudaStream_t s) {

@@ -6,7 +6,7 @@
 // One projection of a batch of M <= 256 positions: Y[row][n] = sum_k W[n][k]
 // x[row][k] for the n_rows x K tile-packed bf16 weights W.  Each activation
 // is carried as three bf16 parts (x = high + middle + low, ee_rows.cu), each
-// part of the batch stored as 256 operand rows; every K = 16 step issues
+// part of the batch stored as N operand rows; every K = 16 step issues
 // three MMAs of shape M = 128 (weight rows) x N (the batch's rows rounded up
 // to 16), one per part, into two fp32 accumulators whose column is the batch
 // row: the high parts' products into the first, the middle and low parts'
@@ -21,10 +21,10 @@
 //     box lands in shared memory in the UMMA canonical K-major layout with
 //     no swizzle: 8-row x 16-byte core matrices, 128 bytes apart along the
 //     rows, 2048 along K) and the batch's activations with bulk copies (the
-//     activation buffer is stored chunk-major, so a full batch's stage is one
-//     contiguous 48 KB range in the same canonical layout: a part's 256 rows
-//     4 KB long, the three parts of a chunk side by side, chunks 12 KB apart
-//     along K; a smaller batch copies the first N rows of each part);
+//     activation buffer is stored chunk-major with a row stride of N, so a
+//     stage is one contiguous range in the same canonical layout: a part's N
+//     rows N x 16 bytes long, the three parts of a chunk side by side, chunks
+//     3 N x 16 bytes apart along K; 48 KB for a full batch);
 //   - warp 1, lane 0 issues six MMAs per stage into the tensor-memory
 //     accumulators and commits each stage back to its producer barrier;
 //   - after the last stage all four warps read the accumulators (warp w holds
@@ -53,9 +53,7 @@ constexpr int kUStages = 4;
 constexpr int kUMRows = 128;                        // weight rows per CTA (UMMA M)
 constexpr int kUKStage = 32;                        // K columns per stage
 constexpr int kUABytes = kUMRows * kUKStage * 2;    // 8 KB
-constexpr int kUPartBytes = kRowsMax * 16;          // one part of one 16-byte chunk: 4 KB
-constexpr int kUChunkBytes = 3 * kUPartBytes;       // the three parts of a chunk: 12 KB
-constexpr int kUBBytes = kUKStage / 8 * kUChunkBytes;  // 48 KB
+constexpr int kUBBytes = kUKStage / 8 * 3 * kRowsMax * 16;  // a full batch's activations: 48 KB
 constexpr int kUStageBytes = kUABytes + kUBBytes;   // 56 KB
 constexpr int kUTmemCols = 2 * kRowsMax;            // two accumulators of one fp32 column per position
 constexpr long long kUWaitCycles = 4000000000ll;   // about 2 s
@@ -169,8 +167,11 @@ __global__ void __launch_bounds__(kUThreads, 1)
     const int k0 = (int)((int64_t)nk * s / S), k1 = (int)((int64_t)nk * (s + 1) / S), ks = k1 - k0;
     // operand rows of the batch (UMMA N): M rounded up to 16; the rows past M
     // give accumulator columns that are never read
-    const int N = (M + 15) & ~15;
-    const uint32_t stage_tx = (uint32_t)(kUABytes + kUKStage / 8 * 3 * N * 16);
+    // (the activation parts are stored with this row stride, x3_rows(M))
+    const int N = x3_rows(M);
+    const int part_bytes = N * 16;  // one part of one 16-byte chunk
+    const uint32_t act_bytes = (uint32_t)(kUKStage / 8 * 3 * part_bytes);
+    const uint32_t stage_tx = (uint32_t)kUABytes + act_bytes;
     volatile int* everr = err;
 
     if (threadIdx.x == 0) {
@@ -221,13 +222,8 @@ __global__ void __launch_bounds__(kUThreads, 1)
                 u_expect_tx(&full[st], stage_tx);
                 u_tma_w(a, &wmap, tile0, kc, &full[st]);
             }
-            if (N == kRowsMax) {  // the stage's activations are one contiguous range
-                u_bulk(a + kUABytes, x3 + (int64_t)kc * 3 * kRowsMax * 8, kUBBytes, &full[st]);
-            } else {  // the first N rows of each (chunk, part)
-                for (int cp = 0; cp < kUKStage / 8 * 3; ++cp)
-                    u_bulk(a + kUABytes + cp * kUPartBytes, x3 + ((int64_t)kc * 3 + cp) * kRowsMax * 8,
-                           (uint32_t)N * 16, &full[st]);
-            }
+            // the stage's activations: one contiguous range
+            u_bulk(a + kUABytes, x3 + (int64_t)kc * 3 * N * 8, act_bytes, &full[st]);
             ++issued;
         }
         // every issued copy lands before the CTA may leave
@@ -252,7 +248,7 @@ __global__ void __launch_bounds__(kUThreads, 1)
 #pragma unroll
                 for (int pp = 0; pp < 3; ++pp)
                     u_mma(tmem + (pp ? kRowsMax : 0), u_desc(a + kk * 2 * 2048, 2048, 128),
-                          u_desc(b + (kk * 2 * 3 + pp) * kUPartBytes, kUChunkBytes, 128), idesc,
+                          u_desc(b + (kk * 2 * 3 + pp) * part_bytes, 3 * part_bytes, 128), idesc,
                           (i > 0 || kk > 0 || pp == 2) ? 1u : 0u);
             u_commit(&empty[st]);
         }
