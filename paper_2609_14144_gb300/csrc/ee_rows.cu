@@ -148,13 +148,16 @@ __global__ void __launch_bounds__(kRowsThreads) k_rows_mm(const uint4* __restric
         const int r0 = rg * 8 * NB;
         const int st0 = (int)((int64_t)nsteps * s / S), st1 = (int)((int64_t)nsteps * (s + 1) / S);
         const uint4* wt = W + (int64_t)tile * Rc * 32;
-        float acc[2][NB][4];
+        // the high parts' products and the middle and low parts' products in
+        // separate accumulators (small terms added into a large running sum
+        // lose their low bits), added at the end
+        float acc[2][NB][4], acm[2][NB][4];
 #pragma unroll
         for (int a = 0; a < 2; ++a)
 #pragma unroll
             for (int n = 0; n < NB; ++n)
 #pragma unroll
-                for (int e = 0; e < 4; ++e) acc[a][n][e] = 0.f;
+                for (int e = 0; e < 4; ++e) acc[a][n][e] = acm[a][n][e] = 0.f;
         for (int st = st0; st < st1; st += U) {
             uint4 w[U][4], bh[U][NB], bm[U][NB], bl[U][NB];
 #pragma unroll
@@ -183,11 +186,13 @@ __global__ void __launch_bounds__(kRowsThreads) k_rows_mm(const uint4* __restric
 #pragma unroll
                     for (int pp = 0; pp < 3; ++pp) {
                         const uint4 b = parts[pp];
+                        float(&c0)[4] = pp ? acm[0][n] : acc[0][n];
+                        float(&c1)[4] = pp ? acm[1][n] : acc[1][n];
                         // first mma of the step: chunk elements 0..3; second: 4..7
-                        mma_16816(acc[0][n], x[0].x, x[1].x, x[0].y, x[1].y, b.x, b.y);
-                        mma_16816(acc[0][n], x[0].z, x[1].z, x[0].w, x[1].w, b.z, b.w);
-                        mma_16816(acc[1][n], x[2].x, x[3].x, x[2].y, x[3].y, b.x, b.y);
-                        mma_16816(acc[1][n], x[2].z, x[3].z, x[2].w, x[3].w, b.z, b.w);
+                        mma_16816(c0, x[0].x, x[1].x, x[0].y, x[1].y, b.x, b.y);
+                        mma_16816(c0, x[0].z, x[1].z, x[0].w, x[1].w, b.z, b.w);
+                        mma_16816(c1, x[2].x, x[3].x, x[2].y, x[3].y, b.x, b.y);
+                        mma_16816(c1, x[2].z, x[3].z, x[2].w, x[3].w, b.z, b.w);
                     }
                 }
             }
@@ -203,7 +208,7 @@ __global__ void __launch_bounds__(kRowsThreads) k_rows_mm(const uint4* __restric
                 for (int e = 0; e < 4; ++e) {
                     const int row = r0 + n * 8 + 2 * q + (e & 1);
                     const int out = tile * 32 + a * 16 + g + (e >> 1) * 8;
-                    if (row < M) ps[(int64_t)row * Np + out] = acc[a][n][e];
+                    if (row < M) ps[(int64_t)row * Np + out] = acc[a][n][e] + acm[a][n][e];
                 }
     }
 }
